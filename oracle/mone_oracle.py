@@ -1,0 +1,343 @@
+"""fp64 CPU oracle of MoNe's test-time learning (TTL) and memory read.
+
+TEST INFRASTRUCTURE ONLY.  Only tests, the smoke entry point and the CPU
+baseline leg of the benchmark may import this module.  The product path (the
+CUDA library and its binding) never calls it, and it shares no code with it.
+
+Everything is plain NumPy in float64, written step by step in the order the
+paper states the method, with library matmuls as the only building blocks.
+Inputs may be float32 or bfloat16 values; they are upcast exactly.
+
+Paper map (MoNe, "Modular Neural Memory for Efficient Long Context
+Inference"):
+  Sec. 3.1            segments of T tokens, s = 1..S, state W_0 -> W_S
+  Eq. 3 (Sec. 3.2)    the memory network; the workloads use its two-matrix
+                      SiLU-MLP form (rows of W1, W2 = hidden units, as Eq. 3
+                      stores W_in / W_out); the three-matrix per-head SwiGLU of
+                      Eq. 3 itself is implemented too (``memory="swiglu"``)
+  Eq. 4               memory read h_j = M(phi(x_j); W_S)
+  Sec. 3.2 (after Eq. 4), App. A
+                      per-head RMSNorm of the read output, learned per-head gate
+  Sec. 3.3, App. A    key/query transform: affine rescale -> SiLU -> L2 norm
+  Eq. 7               loss l_{s,j} = -v^T M(k; W), segment mean L_s = (1/T) sum_j l
+  Eq. 8               W_s = W_{s-1} - mu_s
+  App. A              per-token learning rate (softplus), momentum decay
+                      (sigmoid, from the chunk's hidden states), channel-wise
+                      L2 renormalisation after each update
+  Eq. 9-11            sequential chain over segments; gradient local to layer
+
+Readings of passages the paper leaves open (each also listed in the design
+notes):
+  R1  M maps the hidden activations (width d_in) straight to [K || V]
+      (width d_out); the backbone projections W_q, W_k, W_v are folded away.
+  R2  Targets y_j = [k_j || v_j] are used as given (no SiLU/L2 on targets).
+  R3  eta_j = softplus(w_eta . x_j + b_eta) scales token j's gradient;
+      beta_s = sigmoid(w_beta . mean_j x_j + b_beta);
+      mu_s = beta_s mu_{s-1} + sum_j (eta_j / T') grad l_j.
+  R4  "Channel" = hidden unit = row of W1 and row of W2; each row is rescaled
+      to its norm in W_0 after every update.
+  R5  A last partial segment of T' < T tokens averages over T' tokens.
+  R6  Read normalisation: each output head (width head_dim; K heads then V
+      heads) is divided by sqrt(mean(o_h^2) + eps) and multiplied by a scalar
+      gate g_h; eps = 1e-6.
+  R7  Key/query transform u = z / sqrt(|z|^2 + 1e-12), z = SiLU(alpha*x + gamma).
+  R8  Plain mode: u = x, eta_j = lr, beta = 0, no renormalisation.
+
+Pinned by tests (tests/test_oracle_pins.py): the gradient (finite
+differences), the loss (closed-form one-hot case), the update (closed form of
+one step of a linear memory, Hebbian for Eq. 7 and the delta rule for a
+squared-error loss), the momentum recurrence (geometric-sum closed form), the
+renormalisation invariant, lr = 0 leaving W bit-identical, the read's
+RMS = |gate| invariant, the read of a linear memory against brute force, and
+the chain identities (context = loop of segments = split contexts).
+Parity unpinned: the exact numbers of the paper-mode readings R3, R6, R7
+(their forms are the build's reading; only the invariants above constrain
+them).
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Optional
+
+import numpy as np
+
+PLAIN = 0
+PAPER = 1
+
+RMS_EPS = 1e-6      # R6
+L2_EPS = 1e-12      # R7
+
+
+# --------------------------------------------------------------------------- scalar maps
+
+def sigmoid(z):
+    """Logistic function, written through tanh so it cannot overflow."""
+    z = np.asarray(z, dtype=np.float64)
+    return 0.5 * (1.0 + np.tanh(0.5 * z))
+
+
+def silu(z):
+    """SiLU(z) = z * sigmoid(z) (Eq. 3)."""
+    z = np.asarray(z, dtype=np.float64)
+    return z * sigmoid(z)
+
+
+def silu_prime(z):
+    """d SiLU / dz = sigmoid(z) * (1 + z * (1 - sigmoid(z)))."""
+    z = np.asarray(z, dtype=np.float64)
+    s = sigmoid(z)
+    return s * (1.0 + z * (1.0 - s))
+
+
+def softplus(z):
+    """softplus(z) = ln(1 + e^z) (App. A: per-token learning rate activation)."""
+    return np.logaddexp(0.0, np.asarray(z, dtype=np.float64))
+
+
+def f64(a):
+    """Exact upcast of a float32 / bfloat16 array (NumPy or torch) to float64."""
+    if hasattr(a, "detach"):
+        a = a.detach().to("cpu").double().numpy()
+    return np.array(a, dtype=np.float64)
+
+
+# --------------------------------------------------------------------------- hyper-parameters and state
+
+@dataclasses.dataclass
+class Hyper:
+    """How one chain learns.
+
+    memory:  "mlp"    O = SiLU(U W1^T) W2                     (workload form of Eq. 3)
+             "swiglu" per head: O_h = (SiLU(U_h Win^T) * (U_h Wg^T)) Wout   (Eq. 3)
+             "linear" O = U W^T                              (closed-form checks only)
+    loss:    "neg_inner" Eq. 7;  "mse" 0.5 |M(u) - y|^2 (delta-rule check only)
+    """
+    mode: int = PLAIN
+    lr: float = 1e-2
+    memory: str = "mlp"
+    loss: str = "neg_inner"
+    momentum: Optional[bool] = None     # default: on in PAPER mode
+    renorm: Optional[bool] = None       # default: on in PAPER mode
+    n_heads: int = 1                    # swiglu heads
+    rms_eps: float = RMS_EPS
+
+    @property
+    def use_momentum(self) -> bool:
+        return (self.mode == PAPER) if self.momentum is None else self.momentum
+
+    @property
+    def use_renorm(self) -> bool:
+        return (self.mode == PAPER) if self.renorm is None else self.renorm
+
+
+@dataclasses.dataclass
+class Meta:
+    """Per-chain meta-parameters (App. A); all float64."""
+    alpha: np.ndarray
+    gamma: np.ndarray
+    w_eta: np.ndarray
+    b_eta: float
+    w_beta: np.ndarray
+    b_beta: float
+    gate: np.ndarray
+
+    @staticmethod
+    def from_torch(m: dict, chain: int) -> "Meta":
+        return Meta(f64(m["alpha"][chain]), f64(m["gamma"][chain]), f64(m["w_eta"][chain]),
+                    float(m["b_eta"][chain]), f64(m["w_beta"][chain]), float(m["b_beta"][chain]),
+                    f64(m["gate"][chain]))
+
+
+@dataclasses.dataclass
+class State:
+    """Fast-weight state of one chain: weights, momentum, renorm targets (Sec. 3.3, App. A)."""
+    W: dict            # name -> float64 array (rows = hidden units for mlp/swiglu)
+    mu: dict
+    n0: dict           # name -> row norms of W_0
+
+    def copy(self) -> "State":
+        return State({k: v.copy() for k, v in self.W.items()},
+                     {k: v.copy() for k, v in self.mu.items()},
+                     {k: v.copy() for k, v in self.n0.items()})
+
+
+def row_norms(W):
+    return np.sqrt(np.sum(W * W, axis=-1))
+
+
+def init_state(**W0) -> State:
+    """W_0 given by the caller (learned in the paper, Sec. 3.3); mu_0 = 0."""
+    W = {k: f64(v) for k, v in W0.items()}
+    return State(W, {k: np.zeros_like(v) for k, v in W.items()}, {k: row_norms(v) for k, v in W.items()})
+
+
+# --------------------------------------------------------------------------- input transform (prepass)
+
+def transform_inputs(X, hp: Hyper, meta: Optional[Meta]):
+    """Memory input u_j (Sec. 3.3 / App. A; R7, R8)."""
+    X = f64(X)
+    if hp.mode == PLAIN:
+        return X
+    z = silu(meta.alpha * X + meta.gamma)
+    return z / np.sqrt(np.sum(z * z, axis=1, keepdims=True) + L2_EPS)
+
+
+def token_rates(X, hp: Hyper, meta: Optional[Meta], eta=None):
+    """Per-token learning rate eta_j (App. A; R3, R8); a caller's eta wins."""
+    X = f64(X)
+    if eta is not None:
+        return f64(eta)
+    if hp.mode == PLAIN:
+        return np.full(X.shape[0], hp.lr)
+    return softplus(X @ meta.w_eta + meta.b_eta)
+
+
+def momentum_decay(X, hp: Hyper, meta: Optional[Meta]) -> float:
+    """beta_s in (0,1) from the chunk's hidden states (App. A; R3); 0 without momentum."""
+    if not hp.use_momentum:
+        return 0.0
+    xbar = np.mean(f64(X), axis=0)
+    return float(sigmoid(xbar @ meta.w_beta + meta.b_beta))
+
+
+# --------------------------------------------------------------------------- memory network
+
+def memory_forward(U, W: dict, hp: Hyper):
+    """M(u; W) for every row of U, with the intermediates backprop needs."""
+    if hp.memory == "mlp":
+        Hh = U @ W["W1"].T
+        A = silu(Hh)
+        return A @ W["W2"], (Hh, A)
+    if hp.memory == "linear":
+        return U @ W["W"].T, None
+    if hp.memory == "swiglu":
+        n, d = U.shape
+        dh = d // hp.n_heads
+        O = np.empty((n, hp.n_heads * W["Wout"].shape[2]))
+        cache = []
+        for h in range(hp.n_heads):
+            Uh = U[:, h * dh:(h + 1) * dh]
+            P = Uh @ W["Win"][h].T          # W_in x
+            Gt = Uh @ W["Wg"][h].T          # W_gate x
+            Z = silu(P) * Gt
+            O[:, h * dh:(h + 1) * dh] = Z @ W["Wout"][h]
+            cache.append((Uh, P, Gt, Z))
+        return O, cache
+    raise ValueError(hp.memory)
+
+
+def memory_backward(U, W: dict, hp: Hyper, cache, dO):
+    """Gradient of sum_j dO_j . M(u_j; W) with respect to every fast weight (Eq. 10)."""
+    if hp.memory == "mlp":
+        Hh, A = cache
+        G2 = A.T @ dO
+        dA = dO @ W["W2"].T
+        dH = dA * silu_prime(Hh)
+        G1 = dH.T @ U
+        return {"W1": G1, "W2": G2}
+    if hp.memory == "linear":
+        return {"W": dO.T @ U}
+    if hp.memory == "swiglu":
+        dh = U.shape[1] // hp.n_heads
+        G = {k: np.zeros_like(v) for k, v in W.items()}
+        for h, (Uh, P, Gt, Z) in enumerate(cache):
+            dOh = dO[:, h * dh:(h + 1) * dh]
+            G["Wout"][h] = Z.T @ dOh
+            dZ = dOh @ W["Wout"][h].T
+            dP = dZ * Gt * silu_prime(P)
+            dG = dZ * silu(P)
+            G["Win"][h] = dP.T @ Uh
+            G["Wg"][h] = dG.T @ Uh
+        return G
+    raise ValueError(hp.memory)
+
+
+def segment_loss(U, Y, W: dict, hp: Hyper) -> float:
+    """L_s = (1/T') sum_j l_{s,j}; l = -y^T M(u) (Eq. 7) or 0.5|M(u) - y|^2 (mse check)."""
+    O, _ = memory_forward(U, W, hp)
+    if hp.loss == "neg_inner":
+        per_tok = -np.sum(Y * O, axis=1)
+    else:
+        per_tok = 0.5 * np.sum((O - Y) ** 2, axis=1)
+    return float(np.mean(per_tok))
+
+
+def segment_gradient(U, Y, W: dict, hp: Hyper, eta):
+    """sum_j (eta_j / T') grad_W l_{s,j}  (Eq. 10 with per-token rates, R3).
+
+    Returns (gradient dict, loss L_s at W)."""
+    n = U.shape[0]
+    O, cache = memory_forward(U, W, hp)
+    if hp.loss == "neg_inner":
+        dL_dO = -Y                        # d l_j / d M(u_j) for Eq. 7
+        per_tok = -np.sum(Y * O, axis=1)
+    else:
+        dL_dO = O - Y
+        per_tok = 0.5 * np.sum((O - Y) ** 2, axis=1)
+    dO = (eta / n)[:, None] * dL_dO
+    return memory_backward(U, W, hp, cache, dO), float(np.mean(per_tok))
+
+
+# --------------------------------------------------------------------------- one segment, one chain
+
+def ttl_segment(state: State, X, Y, hp: Hyper, meta: Optional[Meta] = None, eta=None):
+    """One TTL step W_{s-1} -> W_s on one segment (Eq. 7-8, App. A).  Returns (state, L_s)."""
+    X = f64(X)
+    Y = f64(Y)
+    U = transform_inputs(X, hp, meta)
+    rates = token_rates(X, hp, meta, eta)
+    beta = momentum_decay(X, hp, meta)
+    G, loss = segment_gradient(U, Y, state.W, hp, rates)
+    new = state.copy()
+    for k in new.W:
+        new.mu[k] = beta * new.mu[k] + G[k]          # App. A momentum
+        new.W[k] = new.W[k] - new.mu[k]              # Eq. 8
+        if hp.use_renorm:                            # App. A, R4
+            Wk = new.W[k]
+            if Wk.ndim == 2:
+                new.W[k] = Wk * (new.n0[k] / row_norms(Wk))[:, None]
+            else:
+                for h in range(Wk.shape[0]):
+                    Wk[h] = Wk[h] * (new.n0[k][h] / row_norms(Wk[h]))[:, None]
+    return new, loss
+
+
+def ttl_context(state: State, X, Y, T: int, hp: Hyper, meta: Optional[Meta] = None, eta=None,
+                return_all: bool = False):
+    """Chain W_0 -> W_1 -> ... -> W_S over consecutive segments of T tokens (Eq. 9).
+
+    A last partial segment is allowed (R5).  With ``return_all`` the state after
+    every segment is returned as well (for per-step parity)."""
+    X = f64(X)
+    Y = f64(Y)
+    n = X.shape[0]
+    trail, losses = [], []
+    for s0 in range(0, n, T):
+        s1 = min(n, s0 + T)
+        e = None if eta is None else f64(eta)[s0:s1]
+        state, loss = ttl_segment(state, X[s0:s1], Y[s0:s1], hp, meta, e)
+        losses.append(loss)
+        if return_all:
+            trail.append(state.copy())
+    return (state, losses, trail) if return_all else (state, losses)
+
+
+# --------------------------------------------------------------------------- memory read
+
+def generate_kv(state: State, Xq, hp: Hyper, meta: Optional[Meta], n_kv_heads: int, head_dim: int,
+                eps: Optional[float] = None):
+    """Memory tokens for a query (Eq. 4 and the normalisation after it; R6).
+
+    Returns K_mem, V_mem each [n_kv_heads, Q, head_dim]."""
+    eps = hp.rms_eps if eps is None else eps
+    Uq = transform_inputs(Xq, hp, meta)
+    O, _ = memory_forward(Uq, state.W, hp)
+    Q = O.shape[0]
+    n_heads = 2 * n_kv_heads
+    out = np.empty((n_heads, Q, head_dim))
+    gate = np.ones(n_heads) if meta is None else meta.gate
+    for h in range(n_heads):
+        o = O[:, h * head_dim:(h + 1) * head_dim]
+        rms = np.sqrt(np.mean(o * o, axis=1, keepdims=True) + eps)
+        out[h] = gate[h] * o / rms
+    return out[:n_kv_heads], out[n_kv_heads:]
