@@ -1,0 +1,397 @@
+#!/usr/bin/env python
+"""Benchmark of MoNe test-time learning on GB300 (one JSON line on stdout).
+
+One step = one pass of the whole hot path over one synthetic context: reset the
+fast weights to W_0, test-time learning of every layer's memory over all N/T
+segments (prepass, phase A, phase B per segment, final renormalisation), then
+the memory read (generate_kv) for a Q-token query.  Inputs are resident in HBM
+when the timed region starts; the e2e figure repeats the step through the same
+C-ABI calls with the inputs copied from pinned host memory and the generated
+K/V copied back inside the timed region.
+
+--impl reference times the fp64 CPU oracle (the baseline of this build) on the
+host cores over a bounded sample of the same workload.
+
+Multi-GPU (torchrun): every rank runs an independent replica of the workload
+(independent contexts; no collective on the data path); value = all ranks'
+tokens / max time over ranks, scaling "weak".
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import hashlib
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "test-time-learning context tokens/sec at 128K (1 GB300); tensor-pipe util %"
+UNIT = "tokens/s"
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default="l16_d2048_128k")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=15.0, help="target CPU time of the oracle sample")
+    return p.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return d["hbm_gbs"], d["bf16_tflops"], d["bf16_tflops_sustained"], "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ------------------------------------------------------------------ algorithmic work per launch
+
+def kernel_work(wl, kind):
+    """(flops, bytes) of one launch of a phase kernel: one segment of every chain."""
+    C, T = wl.chains, wl.seg_T
+    di, dh, do = wl.d_in, wl.d_hid, wl.d_out
+    params = dh * (di + do)
+    flops = 2 * T * dh * (di + do) * C
+    act = T * (di + do) * 2            # U and Y tiles, bf16, read once
+    grads = T * dh * 2 * 2             # dH^T and At^T, bf16
+    if kind == "phase_a":
+        byts = C * (act + grads + params * 2)          # + bf16 weight operand read
+    else:
+        state = params * (4 + 4 + 2)                   # W fp32 read + write, bf16 copy write
+        if wl.mode == 1:
+            state += params * 8                        # momentum fp32 read + write
+        byts = C * (act + grads + state)
+    return flops, byts
+
+
+def ncu_traffic(kind):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+    src = os.path.join(ROOT, "paper_2608_17616_gb300", "csrc", "ttl_tc.cu")
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        for line in open(path):
+            parts = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
+            if parts.get("kernel") == kind and parts.get("source_sha") == sha:
+                return float(parts["bytes_per_launch"]), parts.get("scaled_from", "")
+    except Exception:
+        pass
+    return None, ""
+
+
+# ------------------------------------------------------------------ clocks
+
+class Clocks:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.p = None
+        self.idx = gpu_index
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.Q}",
+                                       "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.f,
+                                      stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return None
+        time.sleep(0.3)
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except Exception:
+            self.p.kill()
+        self.f.flush()
+        rows = []
+        with open(self.f.name) as fh:
+            for r in csv.reader(fh):
+                if len(r) >= 9:
+                    rows.append([x.strip() for x in r])
+        os.unlink(self.f.name)
+        if not rows:
+            return None
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1])]
+        mx = [num(r[2]) for r in rows if num(r[2])]
+        pw = [num(r[3]) for r in rows if num(r[3])]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        loaded = [s for s, p in zip(sm, pw) if p is not None and p > 0.35 * max(pw)] if pw else sm
+        return {"sm_mhz": statistics.median(loaded or sm), "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+# ------------------------------------------------------------------ oracle timing (CPU baseline / reference arm)
+
+def oracle_sample(wl, seconds, chain=0):
+    """Time the fp64 oracle on chain `chain` for as many segments as fit in ~`seconds`.
+
+    Returns (tokens_per_s in whole-context tokens, sample description, cores)."""
+    import numpy as np
+
+    import oracle as O
+    import workloads as wk
+    n_seg_max = wl.S
+    T = wl.seg_T
+    ctx, layer = divmod(chain, wl.n_layers)
+
+    def inputs(n):
+        x, k, v = wk.chain_inputs(wl, chain, "cpu", n)
+        return O.f64(x), np.concatenate([O.f64(k), O.f64(v)], axis=1)
+    W1all, W2all = wk.initial_weights(wl, "cpu")
+    W1, W2 = W1all[chain], W2all[chain]
+    meta = O.Meta.from_torch(wk.meta_params(wl, "cpu"), chain) if wl.mode == wk.PAPER else None
+    hp = O.Hyper(mode=wl.mode, lr=wl.lr)
+    X1, Y1 = inputs(T)
+    st = O.init_state(W1=O.f64(W1), W2=O.f64(W2))
+    t0 = time.perf_counter()
+    O.ttl_context(st, X1, Y1, T, hp, meta)
+    one = time.perf_counter() - t0
+    n_seg = int(max(1, min(n_seg_max, seconds / max(one, 1e-6))))
+    X, Y = inputs(n_seg * T)
+    st = O.init_state(W1=O.f64(W1), W2=O.f64(W2))
+    t0 = time.perf_counter()
+    O.ttl_context(st, X, Y, T, hp, meta)
+    dt = time.perf_counter() - t0
+    chain_tokens_per_s = n_seg * T / dt
+    # a context token needs one chain-token of work in every layer
+    tok_s = chain_tokens_per_s / wl.n_layers
+    cores = int(os.environ.get("OPENBLAS_NUM_THREADS", "0") or 0) or os.cpu_count()
+    sample = (f"oracle (fp64 NumPy) on chain {chain} of {wl.name}: {n_seg} segment(s) x T={T} = {n_seg * T} tokens "
+              f"of one layer in {dt:.2f} s; scaled to whole-context tokens by 1/{wl.n_layers} layers")
+    return tok_s, sample, cores, dt
+
+
+# ------------------------------------------------------------------ arms
+
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_reference(args, wl):
+    ws, rank, _ = dist_setup()
+    if rank != 0:
+        return
+    rates = []
+    sample = ""
+    cores = os.cpu_count()
+    per_step = max(2.0, min(20.0, 150.0 / max(1, args.steps + args.warmup)))
+    t_all = []
+    for i in range(args.warmup + args.steps):
+        r, sample, cores, dt = oracle_sample(wl, per_step)
+        if i >= args.warmup:
+            rates.append(r)
+            t_all.append(dt)
+    val = statistics.median(rates)
+    line = {"metric": METRIC, "value": val, "unit": UNIT, "impl": "reference", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * statistics.median(t_all),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_of(wl),
+            "cpu_baseline": {"value": val, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def config_of(wl):
+    return {"workload": wl.name, "n_ctx": wl.n_ctx, "n_layers": wl.n_layers, "chains": wl.chains,
+            "N": wl.N, "seg_T": wl.seg_T, "d_in": wl.d_in, "d_hid": wl.d_hid, "d_out": wl.d_out, "Q": wl.Q,
+            "mode": "paper" if wl.mode == 1 else "plain", "masters": "fp32", "operands": wl.dtype,
+            "l2": "inputs larger than L2 (no flush needed)"}
+
+
+def run_ours(args, wl):
+    import torch
+
+    ws, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2608_17616_gb300 as mone
+    import workloads as wk
+
+    dev = f"cuda:{local}"
+    W1_0, W2_0 = wk.initial_weights(wl, dev)
+    meta = wk.meta_params(wl, dev) if wl.mode == wk.PAPER else None
+    X, K, V = wk.all_inputs(wl, dev)
+    Xq = wk.query_inputs(wl, dev)
+    mu0_1 = torch.zeros_like(W1_0) if wl.mode == wk.PAPER else None
+    mu0_2 = torch.zeros_like(W2_0) if wl.mode == wk.PAPER else None
+    Kout = torch.empty(wl.n_ctx, wl.n_layers, wl.n_kv_heads, wl.Q, wl.head_dim, dtype=X.dtype, device=dev)
+    Vout = torch.empty_like(Kout)
+    strides = mone.kv_strides(wl.n_layers, wl.n_kv_heads, wl.Q, wl.head_dim)
+    cfg = mone.make_config(wl.n_ctx, wl.n_layers, wl.d_in, wl.d_hid, wl.d_out, wl.n_kv_heads, wl.head_dim, wl.seg_T,
+                           mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr)
+    h = mone.mone_mem_init(cfg, W1_0, W2_0, meta)
+    stream = torch.cuda.current_stream()
+
+    def step(x=X, k=K, v=V, xq=Xq):
+        mone.mone_mem_write_state(h, W1_0, W2_0, mu0_1, mu0_2)
+        mone.mone_ttl_context(h, x, k, v, wl.N)
+        mone.mone_mem_generate_kv(h, xq, wl.Q, Kout, Vout, strides)
+
+    def barrier():
+        if ws > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        step()
+    mone.mone_mem_sync(h)
+
+    clocks = Clocks(local)
+    mone.mone_mem_set_timing(h, True)
+    n0 = mone.mone_mem_launch_count(h)
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = mone.mone_mem_launch_count(h) - n0
+    ms = e0.elapsed_time(e1) / args.steps
+    ktimes = {name: mone.mone_mem_kernel_time(h, i) for i, name in enumerate(mone.KERNEL_KINDS)}
+    mone.mone_mem_set_timing(h, False)
+    clk = clocks.stop()
+    mone.mone_mem_sync(h)
+    if ws > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    tokens_per_step = wl.n_ctx * wl.N
+    value = ws * tokens_per_step / (ms / 1000.0)
+
+    # ---- end to end through the public calls with host buffers
+    e2e = None
+    if not args.no_e2e:
+        hX = torch.empty(X.shape, dtype=X.dtype, pin_memory=True)
+        hK = torch.empty(K.shape, dtype=K.dtype, pin_memory=True)
+        hV = torch.empty(V.shape, dtype=V.dtype, pin_memory=True)
+        hXq = torch.empty(Xq.shape, dtype=Xq.dtype, pin_memory=True)
+        hKo = torch.empty(Kout.shape, dtype=Kout.dtype, pin_memory=True)
+        hVo = torch.empty(Vout.shape, dtype=Vout.dtype, pin_memory=True)
+        for hst, d in ((hX, X), (hK, K), (hV, V), (hXq, Xq)):
+            hst.copy_(d)
+        dX, dK, dV, dXq = (torch.empty_like(t) for t in (X, K, V, Xq))
+
+        def e2e_step():
+            dX.copy_(hX, non_blocking=True)
+            dK.copy_(hK, non_blocking=True)
+            dV.copy_(hV, non_blocking=True)
+            dXq.copy_(hXq, non_blocking=True)
+            step(dX, dK, dV, dXq)
+            hKo.copy_(Kout, non_blocking=True)
+            hVo.copy_(Vout, non_blocking=True)
+        e2e_step()
+        torch.cuda.synchronize()
+        barrier()
+        e0.record(stream)
+        n_e2e = max(1, min(args.steps, 5))
+        for _ in range(n_e2e):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        ms_e2e = e0.elapsed_time(e1) / n_e2e
+        if ws > 1:
+            import torch.distributed as dist
+            t = torch.tensor([ms_e2e], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms_e2e = float(t.item())
+        h2d = sum(t.numel() * t.element_size() for t in (hX, hK, hV, hXq))
+        d2h = sum(t.numel() * t.element_size() for t in (hKo, hVo))
+        e2e = {"value": ws * tokens_per_step / (ms_e2e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e}
+        del hX, hK, hV
+
+    # ---- roofline of the dominant kernel
+    hbm, tf_burst, tf_sus, peak_src = peaks()
+    kern = {}
+    for name in ("phase_a", "phase_b"):
+        tot, n = ktimes[name]
+        if n == 0:
+            continue
+        avg_ms = tot / n
+        flops, byts = kernel_work(wl, name)
+        kern[name] = {"share": tot / max(1e-9, sum(v[0] for v in ktimes.values())), "avg_us": 1000 * avg_ms,
+                      "launches": n, "tflops": flops / (avg_ms / 1000) / 1e12,
+                      "gbs": byts / (avg_ms / 1000) / 1e9}
+    dom = max(kern, key=lambda k: kern[k]["share"])
+    d = kern[dom]
+    traffic, traffic_note = ncu_traffic(dom)
+    if dom == "phase_b":
+        roof = {"kernel": dom, "bound": "hbm", "achieved": d["gbs"], "peak": hbm, "unit": "GB/s",
+                "frac": d["gbs"] / hbm, "traffic": traffic, "peak_source": f"{peak_src} hbm_gbs"}
+    else:
+        roof = {"kernel": dom, "bound": "tensor", "achieved": d["tflops"], "peak": tf_sus, "unit": "TFLOP/s",
+                "frac": d["tflops"] / tf_sus, "traffic": traffic, "peak_source": f"{peak_src} bf16_tflops_sustained"}
+    total_flops = 4 * (wl.d_in * wl.d_hid + wl.d_hid * wl.d_out) * wl.N * wl.chains
+    tensor_util = total_flops / (ms / 1000) / 1e12 / tf_burst
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        r, sample, cores, _ = oracle_sample(wl, args.cpu_seconds)
+        cpu = {"value": r, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
+                "config": config_of(wl), "e2e": e2e, "gpu_launches": launches, "roofline": roof,
+                "cpu_baseline": cpu, "clocks": clk,
+                "tensor_util_of_burst_peak": tensor_util,
+                "kernels": kern}
+        print(json.dumps(line), flush=True)
+    mone.mone_mem_free(h)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    import workloads as wk
+    wl = wk.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, wl)
+    else:
+        run_ours(args, wl)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,188 @@
+/*
+ * mone.h -- C ABI of the MoNe test-time-learning library (libmone.so).
+ *
+ * MoNe ("Modular Neural Memory") attaches a fast-weight memory network to every
+ * layer of a frozen Transformer.  A context of N tokens is consumed in segments
+ * of T tokens (Sec. 3.1); on each segment every layer's memory takes one
+ * gradient step on a layer-local loss (Eq. 7-8, Sec. 3.4), so the state chains
+ * W_0 -> W_1 -> ... -> W_S (Eq. 9) independently per layer (Eq. 11) and per
+ * context.  At inference the final state turns query hidden states into memory
+ * keys and values (Eq. 4-5).
+ *
+ * This library implements that hot path on one GPU.  The backbone is not part
+ * of it: the caller hands in per-layer activations X and target keys/values K, V
+ * (Eq. 6 outputs), already in the backbone's dtype.
+ *
+ * Memory network (the two-matrix form of Eq. 3):
+ *     M(u; W1, W2) = SiLU(u W1^T) W2,   W1: [d_hid x d_in], W2: [d_hid x d_out]
+ * rows of W1 and W2 are hidden units ("channels"); d_out = 2*n_kv_heads*head_dim
+ * and the output is [K || V] (K heads first, then V heads).
+ *
+ * Conventions
+ *   - A "chain" is one (context, layer) pair: chain = ctx * n_layers + layer.
+ *     Multi-chain arrays are laid out [n_ctx][n_layers][...] row-major.
+ *   - Every data pointer is a DEVICE pointer owned by the caller unless stated;
+ *     the library owns only the state it allocates in mone_mem_init.
+ *   - Calls are asynchronous and ordered on the CUDA stream passed in
+ *     (a cudaStream_t cast to void*; NULL = legacy default stream).
+ *   - Argument errors are returned synchronously and nothing is launched.
+ *     Errors found on the device (a bounded wait that gave up, a non-finite
+ *     weight) are latched in a device status word; mone_mem_sync returns them.
+ *   - There is no CPU fallback: without a usable sm_103a GPU, init fails with
+ *     MONE_ERR_CUDA.
+ */
+#ifndef MONE_H_
+#define MONE_H_
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define MONE_ABI_VERSION 1
+
+typedef struct mone_mem mone_mem; /* opaque; created by mone_mem_init */
+
+typedef enum {
+    MONE_OK = 0,
+    MONE_ERR_INVALID_ARG = 1,       /* null/misaligned pointer, bad index or count, freed handle */
+    MONE_ERR_UNSUPPORTED_SHAPE = 2, /* widths or segment size outside what the kernels tile */
+    MONE_ERR_OOM = 3,               /* device allocation failed */
+    MONE_ERR_CUDA = 4,              /* a CUDA call failed (no device, launch failure, ...) */
+    MONE_ERR_TIMEOUT = 5,           /* a bounded device-side wait gave up (latched) */
+    MONE_ERR_NONFINITE = 6,         /* an updated fast weight was NaN/Inf (latched) */
+    MONE_ERR_UNSUPPORTED = 7        /* valid request this build does not implement */
+} mone_status;
+
+enum { MONE_FP32 = 0, MONE_BF16 = 1 };  /* dtype of X, K, V, Xq and generated K/V */
+enum { MONE_PLAIN = 0, MONE_PAPER = 1 };
+
+/*
+ * Configuration, fixed for the life of a handle.
+ *
+ * mode MONE_PLAIN: u_j = x_j, constant learning rate lr (or per-token rates the
+ *     caller passes to mone_ttl_segment), no momentum, no renormalisation.
+ * mode MONE_PAPER (App. A): u_j = SiLU(alpha*x_j + gamma) / |.|  (affine
+ *     rescale, SiLU, per-token L2 norm); per-token rate
+ *     eta_j = softplus(w_eta . x_j + b_eta); momentum
+ *     mu_s = beta_s mu_{s-1} + g_s with beta_s = sigmoid(w_beta . mean_j x_j + b_beta);
+ *     W_s = W_{s-1} - mu_s (Eq. 8); then every row of W1 and of W2 is rescaled to
+ *     its L2 norm in W_0 ("channel-wise L2 renormalisation").
+ * The gradient step on a segment of T' tokens is g = sum_j (eta_j / T') grad l_j
+ * with l_j = -y_j . M(u_j) (Eq. 7, Eq. 10).
+ *
+ * Supported shapes: FP32: d_in, d_hid, d_out multiples of 64, seg_T multiple of 64.
+ *   BF16: d_in, d_hid, d_out/2, seg_T multiples of 128.  Both: head_dim in {64,128},
+ *   d_out == 2*n_kv_heads*head_dim, seg_T <= 4096.
+ */
+typedef struct {
+    int n_ctx, n_layers;
+    int d_in, d_hid, d_out;
+    int n_kv_heads, head_dim;
+    int seg_T;
+    int dtype;     /* MONE_FP32 | MONE_BF16; fast-weight masters are always fp32 */
+    int mode;      /* MONE_PLAIN | MONE_PAPER */
+    float lr;      /* plain-mode learning rate */
+    float rms_eps; /* epsilon of the read-side RMSNorm (Sec. 3.2 after Eq. 4); e.g. 1e-6 */
+} mone_config;
+
+/*
+ * Per-chain meta-parameters (Sec. 3.3: trained offline, frozen at test time).
+ * Device fp32 arrays: alpha, gamma, w_eta, w_beta are [chains][d_in]; b_eta,
+ * b_beta are [chains]; gate is [chains][2*n_kv_heads] (one scalar gate per
+ * output head, K heads then V heads).  Copied at init; the caller may free them
+ * afterwards.  In MONE_PLAIN mode only gate is read (NULL = all gates 1).
+ */
+typedef struct {
+    const float *alpha, *gamma, *w_eta, *b_eta, *w_beta, *b_beta, *gate;
+} mone_meta;
+
+/*
+ * Allocate the fast-weight state of every chain and set it to W_0.
+ * W1_0: [chains][d_hid][d_in] fp32, W2_0: [chains][d_hid][d_out] fp32 (device;
+ * copied).  Momentum starts at 0; renormalisation targets are the row norms of
+ * W_0.  meta may be NULL in MONE_PLAIN mode.  On success *out owns the state.
+ * Errors: INVALID_ARG, UNSUPPORTED_SHAPE, OOM, CUDA.
+ */
+mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float* W2_0,
+                          const mone_meta* meta, void* stream, mone_mem** out);
+
+/*
+ * One TTL step (Eq. 7-8) of ONE chain on one segment of n_tok <= seg_T tokens.
+ * X: [n_tok][d_in], K, V: [n_tok][d_out/2], dtype cfg->dtype, rows contiguous,
+ * 16-byte aligned.  eta: optional device fp32 [n_tok] per-token learning rates
+ * that replace lr / the softplus rates.  loss_out: optional device fp32 scalar
+ * that receives L_s = -(1/n_tok) sum_j y_j . M(u_j; W_{s-1}) (Eq. 7).
+ * Errors: INVALID_ARG (bad ctx/layer/n_tok/pointer), CUDA.
+ */
+mone_status mone_ttl_segment(mone_mem* m, int ctx, int layer, const void* X, const void* K,
+                             const void* V, int n_tok, const float* eta, float* loss_out,
+                             void* stream);
+
+/*
+ * Test-time learning of a whole context on every chain (Eq. 9): consecutive
+ * segments of seg_T tokens (the last may be shorter and is averaged over its own
+ * length), continuing from the current state, so two calls on N1 (a multiple of
+ * seg_T) and N2 tokens equal one call on N1+N2.
+ * X: [n_ctx][n_layers][N][d_in]; K, V: [n_ctx][n_layers][N][d_out/2]; dtype
+ * cfg->dtype, contiguous, 16-byte aligned.  N >= 1.
+ * Errors: INVALID_ARG, CUDA.
+ */
+mone_status mone_ttl_context(mone_mem* m, const void* X, const void* K, const void* V,
+                             long long N, void* stream);
+
+/*
+ * Memory read (Eq. 4 and the normalisation after it): for every chain and query
+ * token, o = M(phi(x_q); W_S) with phi the key/query transform of the mode, then
+ * every output head h (width head_dim) becomes gate_h * o_h / sqrt(mean(o_h^2) + eps).
+ * K heads are written to K_out, V heads to V_out, dtype cfg->dtype.
+ * Xq: [n_ctx][n_layers][Q][d_in] contiguous.  strides[4] are ELEMENT strides of the
+ * output for (ctx, layer, kv_head, q); head_dim is contiguous, so memory tokens can
+ * be written straight into an attention cache (e.g. after the query's own K/V,
+ * as in Eq. 5's concatenation).  1 <= Q <= 4096.
+ * Errors: INVALID_ARG, OOM (first call with a larger Q allocates scratch), CUDA.
+ */
+mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out, void* V_out,
+                                 const long long strides[4], void* stream);
+
+/* Release the state.  The handle is invalid afterwards; a second free returns
+ * MONE_ERR_INVALID_ARG.  Synchronises the device. */
+mone_status mone_mem_free(mone_mem* m);
+
+/*
+ * Copy the fp32 state out ([chains][d_hid][d_in] / [chains][d_hid][d_out]); any
+ * argument may be NULL to skip it.  Device pointers; stream-ordered.
+ */
+mone_status mone_mem_read_state(const mone_mem* m, float* W1, float* W2, float* mu1, float* mu2,
+                                void* stream);
+
+/* Overwrite the fp32 state (NULL = keep); the renormalisation targets stay those
+ * of W_0.  Device pointers; stream-ordered. */
+mone_status mone_mem_write_state(mone_mem* m, const float* W1, const float* W2, const float* mu1,
+                                 const float* mu2, void* stream);
+
+/* Synchronise the stream and return (and clear) any latched device error. */
+mone_status mone_mem_sync(mone_mem* m, void* stream);
+
+/* Number of device kernels the library has launched on this handle so far. */
+long long mone_mem_launch_count(const mone_mem* m);
+
+/*
+ * Per-kernel device timing for measurement.  While enabled, the library records
+ * a pair of CUDA events on the caller's stream around every kernel it launches
+ * (this adds host work per launch; leave it off outside measurement).
+ * mone_mem_kernel_time waits for the recorded events and returns, for one kernel
+ * kind, the summed device milliseconds and the launch count since timing was
+ * last enabled.  Kinds: 0 input prepass, 1 phase A (forward + fused backward
+ * epilogue), 2 phase B (gradient + fused update), 3 finalize (renorm apply /
+ * operand refresh), 4 memory read.  Errors: INVALID_ARG, CUDA.
+ */
+mone_status mone_mem_set_timing(mone_mem* m, int enable);
+mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches);
+
+const char* mone_status_string(mone_status s);
+int mone_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MONE_H_ */

@@ -1,0 +1,503 @@
+// C-ABI front end of libmone.so: argument validation, state allocation, the
+// segment loop of test-time learning (Eq. 9), and the memory read (Eq. 4).
+// All arithmetic runs in the kernels of ttl_prepass.cu, ttl_simt.cu and ttl_tc.cu.
+#include <algorithm>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <set>
+#include <vector>
+
+#include "mone.h"
+#include "mone_internal.h"
+
+using namespace mone;
+
+// Optional per-kernel device timing (mone_mem_set_timing).
+struct KernelTiming {
+    bool on = false;
+    struct Pending {
+        int kind;
+        cudaEvent_t a, b;
+    };
+    std::vector<cudaEvent_t> pool;
+    std::vector<Pending> pending;
+    double ms[5] = {0, 0, 0, 0, 0};
+    long long n[5] = {0, 0, 0, 0, 0};
+
+    cudaEvent_t get() {
+        if (!pool.empty()) {
+            cudaEvent_t e = pool.back();
+            pool.pop_back();
+            return e;
+        }
+        cudaEvent_t e = nullptr;
+        if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+        return e;
+    }
+    cudaError_t drain() {
+        cudaError_t rc = cudaSuccess;
+        for (auto& p : pending) {
+            cudaError_t e = cudaEventSynchronize(p.b);
+            float t = 0.f;
+            if (e == cudaSuccess) e = cudaEventElapsedTime(&t, p.a, p.b);
+            if (e == cudaSuccess) {
+                ms[p.kind] += t;
+                n[p.kind] += 1;
+            } else {
+                rc = e;
+            }
+            pool.push_back(p.a);
+            pool.push_back(p.b);
+        }
+        pending.clear();
+        return rc;
+    }
+    ~KernelTiming() {
+        drain();
+        for (cudaEvent_t e : pool) cudaEventDestroy(e);
+    }
+};
+
+struct mone_mem {
+    mone_config cfg;
+    DevState s;
+    TcMaps maps;
+    long long launches;
+    KernelTiming* timing;
+};
+
+namespace {
+
+std::mutex g_live_mu;
+std::set<const mone_mem*> g_live;
+
+bool is_live(const mone_mem* m) {
+    std::lock_guard<std::mutex> lk(g_live_mu);
+    return m && g_live.count(m);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+mone_status validate_config(const mone_config* c) {
+    if (!c) return MONE_ERR_INVALID_ARG;
+    if (c->n_ctx < 1 || c->n_layers < 1 || c->d_in < 1 || c->d_hid < 1 || c->d_out < 2 || c->n_kv_heads < 1 ||
+        c->head_dim < 1 || c->seg_T < 1)
+        return MONE_ERR_INVALID_ARG;
+    if (c->dtype != MONE_FP32 && c->dtype != MONE_BF16) return MONE_ERR_INVALID_ARG;
+    if (c->mode != MONE_PLAIN && c->mode != MONE_PAPER) return MONE_ERR_INVALID_ARG;
+    if (!std::isfinite(c->lr) || !(c->rms_eps >= 0.0f) || !std::isfinite(c->rms_eps)) return MONE_ERR_INVALID_ARG;
+    if (c->head_dim != 64 && c->head_dim != 128) return MONE_ERR_UNSUPPORTED_SHAPE;
+    if (c->d_out != 2 * c->n_kv_heads * c->head_dim) return MONE_ERR_UNSUPPORTED_SHAPE;
+    if (c->seg_T > 4096) return MONE_ERR_UNSUPPORTED_SHAPE;
+    if ((long long)c->n_ctx * c->n_layers > 65535) return MONE_ERR_UNSUPPORTED_SHAPE;
+    if (c->dtype == MONE_FP32) {
+        if (c->d_in % 64 || c->d_hid % 64 || c->d_out % 64 || c->seg_T % 64) return MONE_ERR_UNSUPPORTED_SHAPE;
+    } else {
+        if (c->d_in % 128 || c->d_hid % 128 || (c->d_out / 2) % 128 || c->seg_T % 128)
+            return MONE_ERR_UNSUPPORTED_SHAPE;
+    }
+    return MONE_OK;
+}
+
+mone_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return MONE_OK;
+    if (e == cudaErrorMemoryAllocation) return MONE_ERR_OOM;
+    return MONE_ERR_CUDA;
+}
+
+template <typename T>
+mone_status dalloc(T** p, size_t n) {
+    *p = nullptr;
+    if (n == 0) return MONE_OK;
+    const char* f = std::getenv("MONE_FAULT_ALLOC");
+    if (f && std::atoi(f) == 1) return MONE_ERR_OOM;  // host-side allocation-failure injection
+    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(p), n * sizeof(T));
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        *p = nullptr;
+        return e == cudaErrorMemoryAllocation ? MONE_ERR_OOM : MONE_ERR_CUDA;
+    }
+    return MONE_OK;
+}
+
+void free_state(DevState& s) {
+    void* ptrs[] = {s.W1, s.W2, s.mu1, s.mu2, s.W1b, s.W2b, s.n1, s.n2, s.sumsq, s.status, s.alpha, s.gamma,
+                    s.w_eta, s.b_eta, s.w_beta, s.b_beta, s.gate, s.U, s.eta, s.dbeta, s.dHt, s.Att, s.Uq, s.Aq,
+                    s.Oq};
+    for (void* p : ptrs)
+        if (p) cudaFree(p);
+    std::memset(&s, 0, sizeof(s));
+}
+
+size_t elsize(int dtype) { return dtype == MONE_FP32 ? 4 : 2; }
+
+#define MONE_TRY(x)                           \
+    do {                                      \
+        mone_status _st = (x);                \
+        if (_st != MONE_OK) return _st;       \
+    } while (0)
+#define MONE_CUDA(x)                              \
+    do {                                          \
+        cudaError_t _e = (x);                     \
+        if (_e != cudaSuccess) return cuda_status(_e); \
+    } while (0)
+
+mone_status build_state_maps(mone_mem* m) {
+    DevState& s = m->s;
+    if (s.dtype != MONE_BF16) return MONE_OK;
+    bool ok = encode_map_bf16_3d(&m->maps.W1b, s.W1b, s.d_in, s.d_hid, s.C, 64, 128) &&
+              encode_map_bf16_3d(&m->maps.W2b, s.W2b, s.d_out, s.d_hid, s.C, 64, 128) &&
+              encode_map_bf16_3d(&m->maps.dHt, s.dHt, s.T, s.d_hid, s.C, 64, 128) &&
+              encode_map_bf16_3d(&m->maps.Att, s.Att, s.T, s.d_hid, s.C, 64, 128);
+    if (ok && s.U)
+        ok = encode_map_bf16_3d(&m->maps.Ua, s.U, s.d_in, s.T, s.C, 64, 128) &&
+             encode_map_bf16_3d(&m->maps.Ub, s.U, s.d_in, s.T, s.C, 64, 64);
+    return ok ? MONE_OK : MONE_ERR_CUDA;
+}
+
+// Inputs of one call: tensor maps over the caller's X, K, V ([chains][rows][width]).
+mone_status build_input_maps(const DevState& s, TcInputMaps* in, const void* X, const void* K, const void* V,
+                             long long rows, int chains) {
+    const int dh = s.d_out / 2;
+    bool ok = encode_map_bf16_3d(&in->Ka, K, dh, rows, chains, 64, 128) &&
+              encode_map_bf16_3d(&in->Kb, K, dh, rows, chains, 64, 64) &&
+              encode_map_bf16_3d(&in->Va, V, dh, rows, chains, 64, 128) &&
+              encode_map_bf16_3d(&in->Vb, V, dh, rows, chains, 64, 64);
+    if (ok && s.mode == MONE_PLAIN)
+        ok = encode_map_bf16_3d(&in->Xa, X, s.d_in, rows, chains, 64, 128) &&
+             encode_map_bf16_3d(&in->Xb, X, s.d_in, rows, chains, 64, 64);
+    return ok ? MONE_OK : MONE_ERR_CUDA;
+}
+
+enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4 };
+
+// Launch through `fn` (which returns a cudaError_t), bracketed by timing events
+// when timing is on; `kernels` is the number of device kernels `fn` launches.
+template <class F>
+mone_status timed(mone_mem* m, int kind, cudaStream_t st, int kernels, F&& fn) {
+    KernelTiming* T = m->timing;
+    cudaEvent_t a = nullptr, b = nullptr;
+    if (T && T->on) {
+        a = T->get();
+        b = T->get();
+        if (!a || !b) return MONE_ERR_CUDA;
+        if (cudaEventRecord(a, st) != cudaSuccess) return MONE_ERR_CUDA;
+    }
+    const cudaError_t e = fn();
+    if (e != cudaSuccess) return cuda_status(e);
+    if (a) {
+        if (cudaEventRecord(b, st) != cudaSuccess) return MONE_ERR_CUDA;
+        T->pending.push_back({kind, a, b});
+    }
+    m->launches += kernels;
+    return MONE_OK;
+}
+
+// Run segments [0, S) of one call.  w carries chain range and input geometry.
+mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
+    DevState& s = m->s;
+    TcInputMaps in;
+    std::memset(&in, 0, sizeof(in));
+    if (s.dtype == MONE_BF16) MONE_TRY(build_input_maps(s, &in, w.X, w.K, w.V, w.n_rows, w.nc));
+    const long long S = (N + s.T - 1) / s.T;
+    for (long long i = 0; i < S; ++i) {
+        w.row0 = i * s.T;
+        w.Tp = (int)std::min<long long>(s.T, N - w.row0);
+        w.parity = (int)(i & 1);
+        w.renorm_pending = (s.renorm && i > 0) ? 1 : 0;
+        if (s.mode == MONE_PAPER) MONE_TRY(timed(m, K_PREPASS, st, 1, [&] { return launch_prepass(s, w, st); }));
+        if (s.dtype == MONE_BF16) {
+            MONE_TRY(timed(m, K_PHASE_A, st, 1, [&] { return launch_phase_a_tc(s, m->maps, in, w, st); }));
+            MONE_TRY(timed(m, K_PHASE_B, st, 1, [&] { return launch_phase_b_tc(s, m->maps, in, w, st); }));
+        } else {
+            MONE_TRY(timed(m, K_PHASE_A, st, 1, [&] { return launch_phase_a_f32(s, w, st); }));
+            MONE_TRY(timed(m, K_PHASE_B, st, 1, [&] { return launch_phase_b_f32(s, w, st); }));
+        }
+    }
+    if (s.renorm) {
+        const int par = (int)((S - 1) & 1);
+        MONE_TRY(timed(m, K_FINALIZE, st, 1, [&] { return launch_finalize(s, w.c0, w.nc, par, 1, st); }));
+    }
+    return MONE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int mone_abi_version(void) { return MONE_ABI_VERSION; }
+
+const char* mone_status_string(mone_status st) {
+    switch (st) {
+        case MONE_OK: return "ok";
+        case MONE_ERR_INVALID_ARG: return "invalid argument";
+        case MONE_ERR_UNSUPPORTED_SHAPE: return "unsupported shape";
+        case MONE_ERR_OOM: return "device out of memory";
+        case MONE_ERR_CUDA: return "CUDA error";
+        case MONE_ERR_TIMEOUT: return "device wait timed out";
+        case MONE_ERR_NONFINITE: return "non-finite fast weight";
+        case MONE_ERR_UNSUPPORTED: return "unsupported request";
+    }
+    return "unknown status";
+}
+
+mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float* W2_0, const mone_meta* meta,
+                          void* stream, mone_mem** out) {
+    if (!out) return MONE_ERR_INVALID_ARG;
+    *out = nullptr;
+    MONE_TRY(validate_config(cfg));
+    if (!W1_0 || !W2_0 || !aligned16(W1_0) || !aligned16(W2_0)) return MONE_ERR_INVALID_ARG;
+    if (cfg->mode == MONE_PAPER &&
+        (!meta || !meta->alpha || !meta->gamma || !meta->w_eta || !meta->b_eta || !meta->w_beta || !meta->b_beta))
+        return MONE_ERR_INVALID_ARG;
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev < 1) {
+        cudaGetLastError();
+        return MONE_ERR_CUDA;
+    }
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    mone_mem* m = new (std::nothrow) mone_mem;
+    if (!m) return MONE_ERR_OOM;
+    std::memset(m, 0, sizeof(*m));
+    m->cfg = *cfg;
+    DevState& s = m->s;
+    s.C = cfg->n_ctx * cfg->n_layers;
+    s.d_in = cfg->d_in; s.d_hid = cfg->d_hid; s.d_out = cfg->d_out;
+    s.n_kv = cfg->n_kv_heads; s.hd = cfg->head_dim; s.T = cfg->seg_T;
+    s.dtype = cfg->dtype; s.mode = cfg->mode;
+    s.momentum = cfg->mode == MONE_PAPER; s.renorm = cfg->mode == MONE_PAPER;
+    s.lr = cfg->lr; s.rms_eps = cfg->rms_eps;
+    const size_t C = s.C, n1 = C * s.d_hid * s.d_in, n2 = C * s.d_hid * s.d_out;
+    mone_status rc = MONE_OK;
+    auto step = [&](mone_status r) { if (rc == MONE_OK) rc = r; };
+    step(dalloc(&s.W1, n1));
+    step(dalloc(&s.W2, n2));
+    if (s.momentum) {
+        step(dalloc(&s.mu1, n1));
+        step(dalloc(&s.mu2, n2));
+    }
+    if (s.dtype == MONE_BF16) {
+        step(dalloc(&s.W1b, n1));
+        step(dalloc(&s.W2b, n2));
+    }
+    step(dalloc(&s.n1, C * s.d_hid));
+    step(dalloc(&s.n2, C * s.d_hid));
+    step(dalloc(&s.sumsq, 4 * C * s.d_hid));
+    step(dalloc(&s.status, 1));
+    if (s.mode == MONE_PAPER) {
+        step(dalloc(&s.alpha, C * s.d_in));
+        step(dalloc(&s.gamma, C * s.d_in));
+        step(dalloc(&s.w_eta, C * s.d_in));
+        step(dalloc(&s.w_beta, C * s.d_in));
+        step(dalloc(&s.b_eta, C));
+        step(dalloc(&s.b_beta, C));
+        step(dalloc(reinterpret_cast<uint8_t**>(&s.U), C * s.T * s.d_in * elsize(s.dtype)));
+        step(dalloc(&s.eta, C * s.T));
+        step(dalloc(&s.dbeta, C * s.T));
+    }
+    if (meta && meta->gate) step(dalloc(&s.gate, C * 2 * s.n_kv));
+    const size_t elt = s.dtype == MONE_BF16 ? 2 : 4;
+    step(dalloc(reinterpret_cast<uint8_t**>(&s.dHt), C * s.d_hid * s.T * elt));
+    step(dalloc(reinterpret_cast<uint8_t**>(&s.Att), C * s.d_hid * s.T * elt));
+    auto cp = [&](void* dst, const void* src, size_t bytes) {
+        if (rc == MONE_OK) rc = cuda_status(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, st));
+    };
+    cp(s.W1, W1_0, n1 * 4);
+    cp(s.W2, W2_0, n2 * 4);
+    if (s.mode == MONE_PAPER) {
+        cp(s.alpha, meta->alpha, C * s.d_in * 4);
+        cp(s.gamma, meta->gamma, C * s.d_in * 4);
+        cp(s.w_eta, meta->w_eta, C * s.d_in * 4);
+        cp(s.w_beta, meta->w_beta, C * s.d_in * 4);
+        cp(s.b_eta, meta->b_eta, C * 4);
+        cp(s.b_beta, meta->b_beta, C * 4);
+    }
+    if (s.gate) cp(s.gate, meta->gate, C * 2 * s.n_kv * 4);
+    if (rc == MONE_OK && s.momentum) {
+        step(cuda_status(cudaMemsetAsync(s.mu1, 0, n1 * 4, st)));
+        step(cuda_status(cudaMemsetAsync(s.mu2, 0, n2 * 4, st)));
+    }
+    if (rc == MONE_OK) step(cuda_status(cudaMemsetAsync(s.sumsq, 0, 4 * C * s.d_hid * 4, st)));
+    if (rc == MONE_OK) step(cuda_status(cudaMemsetAsync(s.status, 0, 4, st)));
+    if (rc == MONE_OK) step(cuda_status(launch_row_norms(s, st)));
+    if (rc == MONE_OK && s.dtype == MONE_BF16) step(cuda_status(launch_finalize(s, 0, s.C, 0, 0, st)));
+    if (rc == MONE_OK) step(build_state_maps(m));
+    if (rc == MONE_OK) step(cuda_status(cudaStreamSynchronize(st)));
+    if (rc != MONE_OK) {
+        cudaStreamSynchronize(st);
+        cudaGetLastError();
+        free_state(s);
+        delete m;
+        return rc;
+    }
+    m->launches = 1 + (s.dtype == MONE_BF16 ? 1 : 0);
+    {
+        std::lock_guard<std::mutex> lk(g_live_mu);
+        g_live.insert(m);
+    }
+    *out = m;
+    return MONE_OK;
+}
+
+mone_status mone_ttl_segment(mone_mem* m, int ctx, int layer, const void* X, const void* K, const void* V,
+                             int n_tok, const float* eta, float* loss_out, void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    const DevState& s = m->s;
+    if (ctx < 0 || ctx >= m->cfg.n_ctx || layer < 0 || layer >= m->cfg.n_layers) return MONE_ERR_INVALID_ARG;
+    if (n_tok < 1 || n_tok > s.T) return MONE_ERR_INVALID_ARG;
+    if (!X || !K || !V || !aligned16(X) || !aligned16(K) || !aligned16(V)) return MONE_ERR_INVALID_ARG;
+    if (eta && (reinterpret_cast<uintptr_t>(eta) & 3u)) return MONE_ERR_INVALID_ARG;
+    if (loss_out && (reinterpret_cast<uintptr_t>(loss_out) & 3u)) return MONE_ERR_INVALID_ARG;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    SegWork w{};
+    w.c0 = ctx * m->cfg.n_layers + layer;
+    w.nc = 1;
+    w.X = X; w.K = K; w.V = V;
+    w.x_cstride = 0; w.y_cstride = 0;
+    w.n_rows = n_tok;
+    w.eta_in = eta;
+    w.eta_cstride = 0;
+    w.loss = loss_out;
+    if (loss_out) MONE_CUDA(cudaMemsetAsync(loss_out, 0, sizeof(float), st));
+    return run_segments(m, w, n_tok, st);
+}
+
+mone_status mone_ttl_context(mone_mem* m, const void* X, const void* K, const void* V, long long N, void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    const DevState& s = m->s;
+    if (N < 1 || N > (1ll << 31) - 1) return MONE_ERR_INVALID_ARG;
+    if (!X || !K || !V || !aligned16(X) || !aligned16(K) || !aligned16(V)) return MONE_ERR_INVALID_ARG;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    SegWork w{};
+    w.c0 = 0;
+    w.nc = s.C;
+    w.X = X; w.K = K; w.V = V;
+    w.x_cstride = N * s.d_in;
+    w.y_cstride = N * (s.d_out / 2);
+    w.n_rows = N;
+    w.eta_in = nullptr;
+    w.loss = nullptr;
+    return run_segments(m, w, N, st);
+}
+
+mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out, void* V_out,
+                                 const long long strides[4], void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    if (Q < 1 || Q > 4096 || !Xq || !K_out || !V_out || !strides) return MONE_ERR_INVALID_ARG;
+    for (int i = 0; i < 4; ++i)
+        if (strides[i] < 0) return MONE_ERR_INVALID_ARG;
+    DevState& s = m->s;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (Q > s.q_cap) {
+        MONE_CUDA(cudaStreamSynchronize(st));
+        if (s.Uq) cudaFree(s.Uq);
+        if (s.Aq) cudaFree(s.Aq);
+        if (s.Oq) cudaFree(s.Oq);
+        s.Uq = s.Aq = s.Oq = nullptr;
+        s.q_cap = 0;
+        const size_t C = s.C;
+        MONE_TRY(dalloc(&s.Uq, C * Q * s.d_in));
+        MONE_TRY(dalloc(&s.Aq, C * Q * s.d_hid));
+        MONE_TRY(dalloc(&s.Oq, C * Q * s.d_out));
+        s.q_cap = Q;
+    }
+    const int L = m->cfg.n_layers;
+    return timed(m, K_READ, st, 4, [&] {
+        cudaError_t e = launch_query_transform(s, Xq, Q, st);
+        return e != cudaSuccess ? e : launch_read(s, Q, L, K_out, V_out, strides, st);
+    });
+}
+
+mone_status mone_mem_free(mone_mem* m) {
+    {
+        std::lock_guard<std::mutex> lk(g_live_mu);
+        if (!m || !g_live.count(m)) return MONE_ERR_INVALID_ARG;
+        g_live.erase(m);
+    }
+    cudaDeviceSynchronize();
+    delete m->timing;
+    free_state(m->s);
+    delete m;
+    return MONE_OK;
+}
+
+mone_status mone_mem_read_state(const mone_mem* m, float* W1, float* W2, float* mu1, float* mu2, void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    const DevState& s = m->s;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t n1 = (size_t)s.C * s.d_hid * s.d_in * 4, n2 = (size_t)s.C * s.d_hid * s.d_out * 4;
+    if (W1) MONE_CUDA(cudaMemcpyAsync(W1, s.W1, n1, cudaMemcpyDeviceToDevice, st));
+    if (W2) MONE_CUDA(cudaMemcpyAsync(W2, s.W2, n2, cudaMemcpyDeviceToDevice, st));
+    if (mu1) {
+        if (s.mu1) MONE_CUDA(cudaMemcpyAsync(mu1, s.mu1, n1, cudaMemcpyDeviceToDevice, st));
+        else MONE_CUDA(cudaMemsetAsync(mu1, 0, n1, st));
+    }
+    if (mu2) {
+        if (s.mu2) MONE_CUDA(cudaMemcpyAsync(mu2, s.mu2, n2, cudaMemcpyDeviceToDevice, st));
+        else MONE_CUDA(cudaMemsetAsync(mu2, 0, n2, st));
+    }
+    return MONE_OK;
+}
+
+mone_status mone_mem_write_state(mone_mem* m, const float* W1, const float* W2, const float* mu1, const float* mu2,
+                                 void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    DevState& s = m->s;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t n1 = (size_t)s.C * s.d_hid * s.d_in * 4, n2 = (size_t)s.C * s.d_hid * s.d_out * 4;
+    if ((mu1 || mu2) && !s.momentum) return MONE_ERR_INVALID_ARG;
+    if (W1) MONE_CUDA(cudaMemcpyAsync(s.W1, W1, n1, cudaMemcpyDeviceToDevice, st));
+    if (W2) MONE_CUDA(cudaMemcpyAsync(s.W2, W2, n2, cudaMemcpyDeviceToDevice, st));
+    if (mu1) MONE_CUDA(cudaMemcpyAsync(s.mu1, mu1, n1, cudaMemcpyDeviceToDevice, st));
+    if (mu2) MONE_CUDA(cudaMemcpyAsync(s.mu2, mu2, n2, cudaMemcpyDeviceToDevice, st));
+    if (s.dtype == MONE_BF16 && (W1 || W2))
+        return timed(m, K_FINALIZE, st, 1, [&] { return launch_finalize(s, 0, s.C, 0, 0, st); });
+    return MONE_OK;
+}
+
+mone_status mone_mem_sync(mone_mem* m, void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    MONE_CUDA(cudaStreamSynchronize(st));
+    int flag = 0;
+    MONE_CUDA(cudaMemcpy(&flag, m->s.status, sizeof(int), cudaMemcpyDeviceToHost));
+    if (flag) MONE_CUDA(cudaMemset(m->s.status, 0, sizeof(int)));
+    if (flag & DEV_TIMEOUT) return MONE_ERR_TIMEOUT;
+    if (flag & DEV_NONFINITE) return MONE_ERR_NONFINITE;
+    return MONE_OK;
+}
+
+long long mone_mem_launch_count(const mone_mem* m) { return is_live(m) ? m->launches : -1; }
+
+mone_status mone_mem_set_timing(mone_mem* m, int enable) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    if (!m->timing) {
+        m->timing = new (std::nothrow) KernelTiming;
+        if (!m->timing) return MONE_ERR_OOM;
+    }
+    KernelTiming* T = m->timing;
+    const cudaError_t e = T->drain();
+    T->on = enable != 0;
+    if (enable)
+        for (int k = 0; k < 5; ++k) {
+            T->ms[k] = 0;
+            T->n[k] = 0;
+        }
+    return cuda_status(e);
+}
+
+mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches) {
+    if (!is_live(m) || kind < 0 || kind > 4 || !ms || !launches) return MONE_ERR_INVALID_ARG;
+    *ms = 0;
+    *launches = 0;
+    if (!m->timing) return MONE_OK;
+    MONE_CUDA(m->timing->drain());
+    *ms = m->timing->ms[kind];
+    *launches = m->timing->n[kind];
+    return MONE_OK;
+}
+
+}  // extern "C"

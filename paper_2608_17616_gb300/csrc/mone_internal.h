@@ -1,0 +1,90 @@
+// Internal interface between the C-ABI front end (mone_api.cu) and the kernel
+// translation units.  Host-side launchers only; no torch types anywhere.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace mone {
+
+using bf16 = __nv_bfloat16;
+
+// Bits of the device status word (latched until mone_mem_sync reads it).
+enum : int { DEV_TIMEOUT = 1, DEV_NONFINITE = 2 };
+
+// Device-resident state of all chains (see mone_mem_init).
+struct DevState {
+    int C, d_in, d_hid, d_out, n_kv, hd, T, dtype, mode, momentum, renorm;
+    float lr, rms_eps;
+    float *W1, *W2, *mu1, *mu2;   // fp32 masters [C][d_hid][d_in|d_out]; mu only with momentum
+    bf16 *W1b, *W2b;              // bf16 operand copies (bf16 path)
+    float *n1, *n2;               // renormalisation targets [C][d_hid]
+    float* sumsq;                 // [2 parity][2 matrix][C][d_hid] row sums of squares
+    int* status;                  // device status word
+    // meta-parameters (owned copies)
+    float *alpha, *gamma, *w_eta, *b_eta, *w_beta, *b_beta, *gate;
+    // per-segment scratch
+    void* U;                      // [C][T][d_in] transformed inputs (paper mode), dtype of X
+    float* eta;                   // [C][T] per-token rates (paper mode)
+    float* dbeta;                 // [C][T] w_beta . x_t (paper mode)
+    void* dHt;                    // bf16: [C][d_hid][T] (c_t dH)^T ; fp32: [C][T][d_hid]
+    void* Att;                    // bf16: [C][d_hid][T] (c_t A)^T  ; fp32: [C][T][d_hid]
+    // read scratch (grown on demand)
+    int q_cap;
+    float *Uq, *Aq, *Oq;          // [C][q_cap][d_in|d_hid|d_out]
+};
+
+inline float* sumsq_ptr(const DevState& s, int parity, int which) {
+    return s.sumsq + ((size_t)(parity * 2 + which) * s.C) * s.d_hid;
+}
+
+// One segment of work for chains [c0, c0+nc).
+struct SegWork {
+    int c0, nc;
+    const void *X, *K, *V;       // inputs (caller's buffers)
+    long long x_cstride, y_cstride;  // element stride between chains in X and in K/V
+    long long n_rows;            // rows per chain in the caller's buffers
+    long long row0;              // first token row of this segment
+    int Tp;                      // tokens present in this segment (<= T)
+    const float* eta_in;         // caller per-token rates or null
+    long long eta_cstride;
+    int parity;                  // segment index parity within the call
+    int renorm_pending;          // previous segment's renorm scale still to apply
+    float* loss;                 // [C] loss accumulator or null
+};
+
+// ---- kernels in ttl_prepass.cu
+cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st);
+cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, cudaStream_t st);
+
+// ---- kernels in ttl_simt.cu (fp32 path, state upkeep, read path)
+cudaError_t launch_phase_a_f32(const DevState& s, const SegWork& w, cudaStream_t st);
+cudaError_t launch_phase_b_f32(const DevState& s, const SegWork& w, cudaStream_t st);
+cudaError_t launch_finalize(const DevState& s, int c0, int nc, int parity, int apply_scale, cudaStream_t st);
+cudaError_t launch_row_norms(const DevState& s, cudaStream_t st);
+cudaError_t launch_read(const DevState& s, int Q, int n_layers, void* K_out, void* V_out,
+                        const long long* strides, cudaStream_t st);
+cudaError_t launch_zero_f32(float* p, size_t n, cudaStream_t st);
+
+// ---- kernels in ttl_tc.cu (bf16 tcgen05 path)
+struct TcMaps {
+    CUtensorMap W1b, W2b;        // K-major boxes {64, 128}
+    CUtensorMap dHt, Att;        // K-major boxes {64, 128}
+    CUtensorMap Ua, Ub;          // scratch U: K-major {64,128} and MN {64,64}
+};
+struct TcInputMaps {
+    CUtensorMap Xa, Xb, Ka, Kb, Va, Vb;  // per call: K-major {64,128} (a) and MN {64,64} (b)
+};
+cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,
+                              cudaStream_t st);
+cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,
+                              cudaStream_t st);
+int tc_kernels_per_segment();
+
+// Tensor-map encoder (driver entry point, resolved at run time).
+bool encode_map_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t chains,
+                        uint32_t box_inner, uint32_t box_rows);
+
+}  // namespace mone

@@ -1,0 +1,102 @@
+"""Shared test plumbing: run a workload through the C ABI and through the oracle.
+
+Inputs come from ``workloads`` (seeded); the GPU path is driven only through the
+ctypes binding of libmone.so; the oracle is ``oracle`` (fp64 NumPy).  The two
+never exchange intermediate values: both start from the same generated inputs.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle as O
+import paper_2608_17616_gb300 as mone
+import workloads as wk
+
+
+def rel_fro(a, b) -> float:
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def config_of(wl: wk.Workload) -> "mone.mone_config":
+    return mone.make_config(wl.n_ctx, wl.n_layers, wl.d_in, wl.d_hid, wl.d_out, wl.n_kv_heads, wl.head_dim,
+                            wl.seg_T, mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr)
+
+
+class GpuRun:
+    """A live libmone handle for one workload plus its generated device inputs."""
+
+    def __init__(self, wl: wk.Workload, n_tokens=None, device="cuda"):
+        self.wl = wl
+        self.N = wl.N if n_tokens is None else n_tokens
+        self.dev = device
+        self.W1_0, self.W2_0 = wk.initial_weights(wl, device)
+        self.meta = wk.meta_params(wl, device) if wl.mode == wk.PAPER else None
+        self.X, self.K, self.V = wk.all_inputs(wl, device, self.N)
+        self.h = mone.mone_mem_init(config_of(wl), self.W1_0, self.W2_0, self.meta)
+
+    def close(self):
+        if self.h:
+            mone.mone_mem_free(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def state(self):
+        wl = self.wl
+        W1 = torch.empty(wl.chains, wl.d_hid, wl.d_in, device=self.dev)
+        W2 = torch.empty(wl.chains, wl.d_hid, wl.d_out, device=self.dev)
+        mu1 = torch.empty_like(W1)
+        mu2 = torch.empty_like(W2)
+        mone.mone_mem_read_state(self.h, W1, W2, mu1, mu2)
+        torch.cuda.synchronize()
+        return W1.cpu(), W2.cpu(), mu1.cpu(), mu2.cpu()
+
+    def ttl_context(self, X=None, K=None, V=None, N=None):
+        X = self.X if X is None else X
+        K = self.K if K is None else K
+        V = self.V if V is None else V
+        mone.mone_ttl_context(self.h, X, K, V, self.N if N is None else N)
+        mone.mone_mem_sync(self.h)
+
+    def generate_kv(self, Xq):
+        wl = self.wl
+        Q = Xq.shape[2]
+        Kout = torch.empty(wl.n_ctx, wl.n_layers, wl.n_kv_heads, Q, wl.head_dim, dtype=Xq.dtype, device=self.dev)
+        Vout = torch.empty_like(Kout)
+        mone.mone_mem_generate_kv(self.h, Xq, Q, Kout, Vout, mone.kv_strides(wl.n_layers, wl.n_kv_heads, Q,
+                                                                             wl.head_dim))
+        mone.mone_mem_sync(self.h)
+        return Kout.cpu(), Vout.cpu()
+
+
+def oracle_hyper(wl: wk.Workload) -> O.Hyper:
+    return O.Hyper(mode=wl.mode, lr=wl.lr)
+
+
+def oracle_meta(run: GpuRun, chain: int):
+    return O.Meta.from_torch(run.meta, chain) if run.meta is not None else None
+
+
+def oracle_chain(run: GpuRun, chain: int, n_tokens=None, return_all=False):
+    """Replay one chain in the oracle from the run's own generated inputs."""
+    wl = run.wl
+    n = run.N if n_tokens is None else n_tokens
+    ctx, layer = divmod(chain, wl.n_layers)
+    X = O.f64(run.X[ctx, layer, :n])
+    Y = np.concatenate([O.f64(run.K[ctx, layer, :n]), O.f64(run.V[ctx, layer, :n])], axis=1)
+    st = O.init_state(W1=O.f64(run.W1_0[chain]), W2=O.f64(run.W2_0[chain]))
+    return O.ttl_context(st, X, Y, wl.seg_T, oracle_hyper(wl), oracle_meta(run, chain), return_all=return_all)
+
+
+def oracle_read(run: GpuRun, state: O.State, chain: int, Xq):
+    wl = run.wl
+    ctx, layer = divmod(chain, wl.n_layers)
+    return O.generate_kv(state, O.f64(Xq[ctx, layer]), oracle_hyper(wl), oracle_meta(run, chain),
+                         wl.n_kv_heads, wl.head_dim)

@@ -1,0 +1,94 @@
+"""C-ABI checks that need no GPU: the library loads, exports every symbol the
+header declares, and rejects bad arguments before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2608_17616_gb300 as mone
+from paper_2608_17616_gb300 import build as mbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    mbuild.build()
+    return mone.lib()
+
+
+def header_functions():
+    text = open(os.path.join(ROOT, "include", "mone.h")).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?(?:\w+\**\s+)+\**(mone_\w+)\(", text, re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = header_functions()
+    for required in ("mone_mem_init", "mone_ttl_segment", "mone_ttl_context", "mone_mem_generate_kv",
+                     "mone_mem_free"):
+        assert required in names
+    assert set(names) == set(mone.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(L):
+    raw = ctypes.CDLL(mone.LIB_PATH)
+    for name in header_functions():
+        assert hasattr(raw, name), name
+    assert L.mone_abi_version() == 1
+
+
+def test_status_strings(L):
+    for code in range(8):
+        assert mone.mone_status_string(code)
+    assert mone.mone_status_string(0) == "ok"
+
+
+def cfg(**kw):
+    base = dict(n_ctx=1, n_layers=2, d_in=256, d_hid=256, d_out=256, n_kv_heads=2, head_dim=64, seg_T=128,
+                dtype=mone.MONE_BF16, mode=mone.MONE_PLAIN, lr=1e-2)
+    base.update(kw)
+    return mone.make_config(**base)
+
+
+def init_rc(L, c, w1=16, w2=16, meta=None):
+    h = ctypes.c_void_p()
+    return L.mone_mem_init(ctypes.byref(c) if c is not None else None, w1, w2, meta, None, ctypes.byref(h))
+
+
+def test_init_rejects_bad_arguments_without_a_device(L):
+    assert init_rc(L, None) == 1
+    assert init_rc(L, cfg(), w1=None) == 1
+    assert init_rc(L, cfg(), w1=8) == 1                     # misaligned
+    assert init_rc(L, cfg(dtype=7)) == 1
+    assert init_rc(L, cfg(mode=3)) == 1
+    assert init_rc(L, cfg(n_layers=0)) == 1
+    assert init_rc(L, cfg(lr=float("nan"))) == 1
+    assert init_rc(L, cfg(mode=mone.MONE_PAPER)) == 1         # paper mode needs meta-parameters
+
+
+def test_init_rejects_unsupported_shapes(L):
+    assert init_rc(L, cfg(head_dim=96, d_out=384, n_kv_heads=2)) == 2
+    assert init_rc(L, cfg(d_out=512)) == 2                    # d_out != 2 * n_kv * hd
+    assert init_rc(L, cfg(d_in=192)) == 2                     # bf16 tiles are 128 wide
+    assert init_rc(L, cfg(seg_T=192)) == 2
+    assert init_rc(L, cfg(seg_T=8192)) == 2
+    assert init_rc(L, cfg(dtype=mone.MONE_FP32, d_in=96)) == 2
+
+
+def test_calls_on_invalid_handles(L):
+    bogus = 0x1000
+    assert L.mone_mem_free(None) == 1
+    assert L.mone_mem_free(bogus) == 1
+    assert L.mone_ttl_context(bogus, 16, 16, 16, 128, None) == 1
+    assert L.mone_ttl_segment(bogus, 0, 0, 16, 16, 16, 1, None, None, None) == 1
+    arr = (ctypes.c_longlong * 4)(0, 0, 0, 0)
+    assert L.mone_mem_generate_kv(bogus, 16, 1, 16, 16, arr, None) == 1
+    assert L.mone_mem_sync(bogus, None) == 1
+    assert L.mone_mem_launch_count(bogus) == -1
+
+
+@pytest.mark.skipif(os.path.exists("/dev/nvidia0"), reason="checks the behaviour on a machine without a GPU")
+def test_init_without_gpu_fails_loudly(L):
+    # valid arguments, no device: the library reports a CUDA error, it never falls back to the CPU
+    assert init_rc(L, cfg()) == 4

@@ -1,0 +1,223 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle.
+
+Tolerances: fp32 path, per-step relative Frobenius error of W1 and W2 <= 1e-4;
+bf16 path, <= 2e-2 after the full context (and the same bound on the weight
+*change* W_S - W_0, which is the part the kernels compute); generated K/V
+<= 2e-2 (fp32 path: 1e-4).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import paper_2608_17616_gb300 as mone
+import workloads as wk
+from harness import GpuRun, oracle_chain, oracle_read, rel_fro
+
+pytestmark = pytest.mark.gpu
+
+F32_TOL = 1e-4
+BF16_TOL = 2e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2608_17616_gb300 import build
+    build.build()
+    assert torch.cuda.is_available()
+    mone.lib()
+
+
+def small(mode, dtype="bf16", n_ctx=2, n_layers=2, d_in=256, d_hid=256, d_out=256, T=256, N=4 * 256 + 37, lr=0.3,
+          hd=64, Q=40):
+    return wk.Workload(f"small_{dtype}_{mode}", 10 + mode, n_ctx, n_layers, d_in, d_hid, d_out, d_out // (2 * hd), hd,
+                       T, N, Q, dtype, mode, lr)
+
+
+def check_chain(run, chain, W1, W2, tol, n_tokens=None):
+    st, _ = oracle_chain(run, chain, n_tokens)
+    e1 = rel_fro(W1[chain], st.W["W1"])
+    e2 = rel_fro(W2[chain], st.W["W2"])
+    d1 = rel_fro(W1[chain].double() - run.W1_0[chain].cpu().double(), st.W["W1"] - O.f64(run.W1_0[chain]))
+    d2 = rel_fro(W2[chain].double() - run.W2_0[chain].cpu().double(), st.W["W2"] - O.f64(run.W2_0[chain]))
+    assert e1 <= tol and e2 <= tol, (chain, e1, e2)
+    assert d1 <= max(tol, 5e-2) and d2 <= max(tol, 5e-2), (chain, d1, d2)
+    return st
+
+
+# ----------------------------------------------------------------- fp32 path (tiny workload)
+
+def test_tiny_f32_per_step_parity_and_loss():
+    wl = wk.WORKLOADS["tiny_f32"]
+    run = GpuRun(wl)
+    _, losses, trail = oracle_chain(run, 0, return_all=True)
+    loss_dev = torch.zeros(1, device="cuda")
+    T = wl.seg_T
+    for s in range(wl.S):
+        sl = slice(s * T, (s + 1) * T)
+        mone.mone_ttl_segment(run.h, 0, 0, run.X[0, 0, sl], run.K[0, 0, sl], run.V[0, 0, sl], T, None, loss_dev)
+        mone.mone_mem_sync(run.h)
+        W1, W2, _, _ = run.state()
+        assert rel_fro(W1[0], trail[s].W["W1"]) <= F32_TOL, s
+        assert rel_fro(W2[0], trail[s].W["W2"]) <= F32_TOL, s
+        assert abs(loss_dev.item() - losses[s]) <= F32_TOL * max(1.0, abs(losses[s])), s
+    run.close()
+
+
+def test_tiny_f32_context_equals_segment_loop_and_read():
+    wl = wk.WORKLOADS["tiny_f32"]
+    a = GpuRun(wl)
+    a.ttl_context()
+    W1a, W2a, _, _ = a.state()
+    b = GpuRun(wl)
+    T = wl.seg_T
+    for s in range(wl.S):
+        sl = slice(s * T, (s + 1) * T)
+        mone.mone_ttl_segment(b.h, 0, 0, b.X[0, 0, sl], b.K[0, 0, sl], b.V[0, 0, sl], T)
+    mone.mone_mem_sync(b.h)
+    W1b, W2b, _, _ = b.state()
+    assert torch.equal(W1a, W1b) and torch.equal(W2a, W2b)
+    st = check_chain(a, 0, W1a, W2a, F32_TOL)
+    Xq = wk.query_inputs(wl, "cuda")
+    Kg, Vg = a.generate_kv(Xq)
+    Ko, Vo = oracle_read(a, st, 0, Xq)
+    assert rel_fro(Kg[0, 0], Ko) <= F32_TOL and rel_fro(Vg[0, 0], Vo) <= F32_TOL
+    a.close()
+    b.close()
+
+
+def test_f32_paper_mode_ragged():
+    wl = small(wk.PAPER, "f32", T=128, N=3 * 128 + 50, d_in=128, d_hid=192, d_out=256, lr=0.5)
+    run = GpuRun(wl)
+    run.ttl_context()
+    W1, W2, mu1, mu2 = run.state()
+    for c in range(wl.chains):
+        st = check_chain(run, c, W1, W2, F32_TOL)
+        assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+    Xq = wk.query_inputs(wl, "cuda")
+    Kg, Vg = run.generate_kv(Xq)
+    for c in range(wl.chains):
+        st, _ = oracle_chain(run, c)
+        Ko, Vo = oracle_read(run, st, c, Xq)
+        assert rel_fro(Kg[c // 2, c % 2], Ko) <= F32_TOL and rel_fro(Vg[c // 2, c % 2], Vo) <= F32_TOL
+    run.close()
+
+
+# ----------------------------------------------------------------- bf16 tensor-core path (small shapes)
+
+@pytest.mark.parametrize("mode", [wk.PLAIN, wk.PAPER])
+def test_bf16_small_context_parity(mode):
+    wl = small(mode)
+    run = GpuRun(wl)
+    run.ttl_context()
+    W1, W2, mu1, mu2 = run.state()
+    Xq = wk.query_inputs(wl, "cuda")
+    Kg, Vg = run.generate_kv(Xq)
+    for c in range(wl.chains):
+        st = check_chain(run, c, W1, W2, BF16_TOL)
+        Ko, Vo = oracle_read(run, st, c, Xq)
+        assert rel_fro(Kg[c // 2, c % 2].float(), Ko) <= BF16_TOL
+        assert rel_fro(Vg[c // 2, c % 2].float(), Vo) <= BF16_TOL
+    run.close()
+
+
+def test_bf16_segment_with_caller_rates_and_loss():
+    wl = small(wk.PLAIN, n_ctx=1, n_layers=3, N=256)
+    run = GpuRun(wl)
+    eta = wk.token_lr(wl, 1, 200, "cuda")
+    loss = torch.zeros(1, device="cuda")
+    mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, :200], run.K[0, 1, :200], run.V[0, 1, :200], 200, eta, loss)
+    mone.mone_mem_sync(run.h)
+    W1, W2, _, _ = run.state()
+    X = O.f64(run.X[0, 1, :200])
+    Y = np.concatenate([O.f64(run.K[0, 1, :200]), O.f64(run.V[0, 1, :200])], axis=1)
+    st = O.init_state(W1=O.f64(run.W1_0[1]), W2=O.f64(run.W2_0[1]))
+    st, L = O.ttl_segment(st, X, Y, O.Hyper(mode=wk.PLAIN, lr=wl.lr), None, eta=O.f64(eta))
+    assert rel_fro(W1[1], st.W["W1"]) <= BF16_TOL and rel_fro(W2[1], st.W["W2"]) <= BF16_TOL
+    assert rel_fro(W1[1].double() - run.W1_0[1].cpu().double(), st.W["W1"] - O.f64(run.W1_0[1])) <= 5e-2
+    assert abs(loss.item() - L) <= BF16_TOL * max(1.0, abs(L))
+    # untouched chains keep W_0 exactly
+    for c in (0, 2):
+        assert torch.equal(W1[c], run.W1_0[c].cpu()) and torch.equal(W2[c], run.W2_0[c].cpu())
+    run.close()
+
+
+def test_bf16_context_split_equals_whole():
+    wl = small(wk.PAPER, N=6 * 256)
+    a = GpuRun(wl)
+    a.ttl_context()
+    b = GpuRun(wl)
+    n1 = 2 * 256
+    X1, K1, V1 = (t[:, :, :n1].contiguous() for t in (b.X, b.K, b.V))
+    X2, K2, V2 = (t[:, :, n1:].contiguous() for t in (b.X, b.K, b.V))
+    b.ttl_context(X1, K1, V1, n1)
+    b.ttl_context(X2, K2, V2, wl.N - n1)
+    for ta, tb in zip(a.state(), b.state()):
+        assert rel_fro(tb, ta) <= 1e-5
+    a.close()
+    b.close()
+
+
+def test_bf16_layer_permutation_permutes_results():
+    wl = small(wk.PAPER, n_ctx=1, n_layers=4, N=512)
+    a = GpuRun(wl)
+    a.ttl_context()
+    W1a, W2a, _, _ = a.state()
+    perm = [2, 0, 3, 1]
+    b = GpuRun(wl)
+    mone.mone_mem_free(b.h)
+    meta = {k: v[perm].contiguous() for k, v in a.meta.items()}
+    from harness import config_of
+    b.h = mone.mone_mem_init(config_of(wl), a.W1_0[perm].contiguous(), a.W2_0[perm].contiguous(), meta)
+    b.ttl_context(a.X[:, perm].contiguous(), a.K[:, perm].contiguous(), a.V[:, perm].contiguous())
+    W1b, W2b, _, _ = b.state()
+    for i, p in enumerate(perm):
+        assert rel_fro(W1b[i], W1a[p]) <= 1e-5 and rel_fro(W2b[i], W2a[p]) <= 1e-5
+    a.close()
+    b.close()
+
+
+def test_generate_kv_into_strided_cache_and_reuse():
+    wl = small(wk.PAPER, N=512)
+    run = GpuRun(wl)
+    run.ttl_context()
+    Q, off, S_tot = wl.Q, 7, wl.Q + 19
+    Xq = wk.query_inputs(wl, "cuda")
+    cache_k = torch.full((wl.n_ctx, wl.n_layers, wl.n_kv_heads, S_tot, wl.head_dim), 7.0, dtype=torch.bfloat16,
+                         device="cuda")
+    cache_v = cache_k.clone()
+    strides = cache_k.stride()[:4]
+    mone.mone_mem_generate_kv(run.h, Xq, Q, cache_k[:, :, :, off:], cache_v[:, :, :, off:], strides)
+    mone.mone_mem_sync(run.h)
+    Kd, Vd = run.generate_kv(Xq)
+    assert torch.equal(cache_k[:, :, :, off:off + Q].cpu(), Kd) and torch.equal(cache_v[:, :, :, off:off + Q].cpu(), Vd)
+    assert bool((cache_k[:, :, :, :off] == 7).all()) and bool((cache_k[:, :, :, off + Q:] == 7).all())
+    K2, V2 = run.generate_kv(Xq)          # multi-query reuse: reading does not change the state
+    assert torch.equal(K2, Kd) and torch.equal(V2, Vd)
+    run.close()
+
+
+# ----------------------------------------------------------------- full-size workloads, sampled chains
+
+@pytest.mark.parametrize("name,chains,n_tokens", [
+    ("l16_d2048_128k", (0, 15), None),
+    ("l16_d2048_32k", (7,), None),
+    ("l28_d3072_128k", (27,), 16 * 1024),
+    ("ctx8_l16_T256", (77,), 8192),
+    ("ctx8_l16_T2048", (5,), 8192),
+])
+def test_full_size_sampled_chains(name, chains, n_tokens):
+    wl = wk.WORKLOADS[name]
+    run = GpuRun(wl, n_tokens=n_tokens)
+    run.ttl_context()
+    W1, W2, _, _ = run.state()
+    Xq = wk.query_inputs(wl, "cuda")
+    Kg, Vg = run.generate_kv(Xq)
+    for c in chains:
+        st = check_chain(run, c, W1, W2, BF16_TOL)
+        Ko, Vo = oracle_read(run, st, c, Xq)
+        ctx, layer = divmod(c, wl.n_layers)
+        assert rel_fro(Kg[ctx, layer].float(), Ko) <= BF16_TOL
+        assert rel_fro(Vg[ctx, layer].float(), Vo) <= BF16_TOL
+    run.close()
+    torch.cuda.empty_cache()
