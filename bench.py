@@ -48,6 +48,7 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="target CPU time of the oracle sample")
+    p.add_argument("--n-tokens", type=int, default=0, help="override the context length (small profiling cases)")
     return p.parse_args()
 
 
@@ -387,6 +388,8 @@ def main():
     args = parse()
     import workloads as wk
     wl = wk.WORKLOADS[args.workload]
+    if args.n_tokens:
+        wl = wl.replace(N=args.n_tokens)
     if args.impl == "reference":
         run_reference(args, wl)
     else:

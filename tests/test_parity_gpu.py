@@ -152,8 +152,10 @@ def test_bf16_context_split_equals_whole():
     X2, K2, V2 = (t[:, :, n1:].contiguous() for t in (b.X, b.K, b.V))
     b.ttl_context(X1, K1, V1, n1)
     b.ttl_context(X2, K2, V2, wl.N - n1)
+    # equal up to bf16 operand rounding: the split run rounds the renormalised
+    # weights at rest, the whole run rounds the raw weights and rescales in fp32
     for ta, tb in zip(a.state(), b.state()):
-        assert rel_fro(tb, ta) <= 1e-5
+        assert rel_fro(tb, ta) <= 1e-3
     a.close()
     b.close()
 
