@@ -71,7 +71,7 @@ enum { MONE_PLAIN = 0, MONE_PAPER = 1 };
  * with l_j = -y_j . M(u_j) (Eq. 7, Eq. 10).
  *
  * Supported shapes: FP32: d_in, d_hid, d_out multiples of 64, seg_T multiple of 64.
- *   BF16: d_in, d_hid, d_out/2, seg_T multiples of 128.  Both: head_dim in {64,128},
+ *   BF16: d_in, d_out/2, seg_T multiples of 128; d_hid a multiple of 256.  Both: head_dim in {64,128},
  *   d_out == 2*n_kv_heads*head_dim, seg_T <= 4096.
  */
 typedef struct {

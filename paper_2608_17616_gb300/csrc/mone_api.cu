@@ -96,7 +96,7 @@ mone_status validate_config(const mone_config* c) {
     if (c->dtype == MONE_FP32) {
         if (c->d_in % 64 || c->d_hid % 64 || c->d_out % 64 || c->seg_T % 64) return MONE_ERR_UNSUPPORTED_SHAPE;
     } else {
-        if (c->d_in % 128 || c->d_hid % 128 || (c->d_out / 2) % 128 || c->seg_T % 128)
+        if (c->d_in % 128 || c->d_hid % 256 || (c->d_out / 2) % 128 || c->seg_T % 128)
             return MONE_ERR_UNSUPPORTED_SHAPE;
     }
     return MONE_OK;
@@ -150,8 +150,8 @@ mone_status build_state_maps(mone_mem* m) {
     if (s.dtype != MONE_BF16) return MONE_OK;
     bool ok = encode_map_bf16_3d(&m->maps.W1b, s.W1b, s.d_in, s.d_hid, s.C, 64, 128) &&
               encode_map_bf16_3d(&m->maps.W2b, s.W2b, s.d_out, s.d_hid, s.C, 64, 128) &&
-              encode_map_bf16_3d(&m->maps.dHt, s.dHt, s.T, s.d_hid, s.C, 64, 128) &&
-              encode_map_bf16_3d(&m->maps.Att, s.Att, s.T, s.d_hid, s.C, 64, 128);
+              encode_map_bf16_3d(&m->maps.dH, s.dHt, s.d_hid, s.T, s.C, 64, 64) &&
+              encode_map_bf16_3d(&m->maps.At, s.Att, s.d_hid, s.T, s.C, 64, 64);
     if (ok && s.U)
         ok = encode_map_bf16_3d(&m->maps.Ua, s.U, s.d_in, s.T, s.C, 64, 128) &&
              encode_map_bf16_3d(&m->maps.Ub, s.U, s.d_in, s.T, s.C, 64, 64);

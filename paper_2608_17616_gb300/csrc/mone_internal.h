@@ -29,8 +29,8 @@ struct DevState {
     void* U;                      // [C][T][d_in] transformed inputs (paper mode), dtype of X
     float* eta;                   // [C][T] per-token rates (paper mode)
     float* dbeta;                 // [C][T] w_beta . x_t (paper mode)
-    void* dHt;                    // bf16: [C][d_hid][T] (c_t dH)^T ; fp32: [C][T][d_hid]
-    void* Att;                    // bf16: [C][d_hid][T] (c_t A)^T  ; fp32: [C][T][d_hid]
+    void* dHt;                    // [C][T][d_hid] c_t dH (bf16 or fp32 by path)
+    void* Att;                    // [C][T][d_hid] c_t A
     // read scratch (grown on demand)
     int q_cap;
     float *Uq, *Aq, *Oq;          // [C][q_cap][d_in|d_hid|d_out]
@@ -71,7 +71,7 @@ cudaError_t launch_zero_f32(float* p, size_t n, cudaStream_t st);
 // ---- kernels in ttl_tc.cu (bf16 tcgen05 path)
 struct TcMaps {
     CUtensorMap W1b, W2b;        // K-major boxes {64, 128}
-    CUtensorMap dHt, Att;        // K-major boxes {64, 128}
+    CUtensorMap dH, At;          // MN-major boxes {64, 64} over [C][T][d_hid]
     CUtensorMap Ua, Ub;          // scratch U: K-major {64,128} and MN {64,64}
 };
 struct TcInputMaps {

@@ -6,9 +6,8 @@
 // rate eta_j = softplus(w_eta . x_j + b_eta) and the per-token term
 // w_beta . x_j of the momentum decay beta_s = sigmoid(mean_j(w_beta . x_j) + b_beta).
 //
-// One warp per token row; the row is read twice (statistics, then output) and
-// the second read hits L1/L2.  Streaming, HBM-bound: reads d_in elements and
-// writes d_in elements per token.
+// One warp per token row, 16-byte vector loads, the row held in registers.
+// Streaming, HBM-bound: reads d_in elements and writes d_in elements per token.
 #include "mone_common.cuh"
 
 namespace mone {
@@ -34,8 +33,58 @@ struct PrepassArgs {
     float* dbeta;         // [C][rows]
 };
 
+// 16-byte vector of inputs: 8 bf16 or 4 fp32 values, kept packed in registers.
+template <typename T> struct Vec;
+template <> struct Vec<bf16> {
+    static constexpr int N = 8;
+    __device__ static void unpack(const uint4& r, float (&v)[8]) {
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&r);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(h[i]);
+            v[2 * i] = f.x;
+            v[2 * i + 1] = f.y;
+        }
+    }
+};
+template <> struct Vec<float> {
+    static constexpr int N = 4;
+    __device__ static void unpack(const uint4& r, float (&v)[4]) {
+        v[0] = __uint_as_float(r.x); v[1] = __uint_as_float(r.y);
+        v[2] = __uint_as_float(r.z); v[3] = __uint_as_float(r.w);
+    }
+};
+
+template <typename T, int N> __device__ __forceinline__ void store_vec(T* p, const float (&v)[N]);
+template <> __device__ __forceinline__ void store_vec<bf16, 8>(bf16* p, const float (&v)[8]) {
+    uint4 r;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&r);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+    *reinterpret_cast<uint4*>(p) = r;
+}
+template <> __device__ __forceinline__ void store_vec<float, 4>(float* p, const float (&v)[4]) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+}
+template <> __device__ __forceinline__ void store_vec<float, 8>(float* p, const float (&v)[8]) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
+}
+
+template <int N>
+__device__ __forceinline__ void load_f32(const float* p, float (&v)[N]) {
+#pragma unroll
+    for (int i = 0; i < N; i += 4) {
+        const float4 r = *reinterpret_cast<const float4*>(p + i);
+        v[i] = r.x; v[i + 1] = r.y; v[i + 2] = r.z; v[i + 3] = r.w;
+    }
+}
+
+// One warp per token row, 16-byte vector loads.  Statistics first; the output
+// pass re-reads the row (an L1/L2 hit: the row was read just before).
 template <typename Tin, typename Tout>
 __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
+    constexpr int V = Vec<Tin>::N;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int t = blockIdx.x * 8 + warp;
     const int cz = blockIdx.y;
@@ -45,7 +94,10 @@ __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
     Tout* u = reinterpret_cast<Tout*>(a.U) + ((size_t)cs * a.rows + t) * d;
     const bool present = t < a.Tp && (a.row0 + t) < a.n_rows;
     if (!present) {
-        for (int i = lane; i < d; i += 32) u[i] = from_f<Tout>(0.0f);
+        float z[V];
+#pragma unroll
+        for (int e = 0; e < V; ++e) z[e] = 0.f;
+        for (int i0 = lane * V; i0 < d; i0 += 32 * V) store_vec<Tout, V>(u + i0, z);
         if (!a.query && lane == 0) {
             a.eta[(size_t)cs * a.rows + t] = 0.0f;
             a.dbeta[(size_t)cs * a.rows + t] = 0.0f;
@@ -54,19 +106,30 @@ __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
     }
     const Tin* x = reinterpret_cast<const Tin*>(a.X) + cz * a.x_cstride + (a.row0 + t) * d;
     float ss = 0.f, de = 0.f, db = 0.f;
+    const float* al = a.paper ? a.alpha + (size_t)cs * d : nullptr;
+    const float* ga = a.paper ? a.gamma + (size_t)cs * d : nullptr;
     if (a.paper) {
-        const float* al = a.alpha + (size_t)cs * d;
-        const float* ga = a.gamma + (size_t)cs * d;
-        const float* we = a.w_eta + (size_t)cs * d;
-        const float* wb = a.w_beta + (size_t)cs * d;
-        for (int i = lane; i < d; i += 32) {
-            const float xv = to_f<Tin>(x[i]);
-            const float zp = al[i] * xv + ga[i];
-            const float z = zp * sigmoidf_(zp);
-            ss += z * z;
+#pragma unroll 4
+        for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
+            float xv[V], av[V], gv[V];
+            Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x + i0), xv);
+            load_f32<V>(al + i0, av);
+            load_f32<V>(ga + i0, gv);
             if (!a.query) {
-                de += we[i] * xv;
-                db += wb[i] * xv;
+                float we[V], wb[V];
+                load_f32<V>(a.w_eta + (size_t)cs * d + i0, we);
+                load_f32<V>(a.w_beta + (size_t)cs * d + i0, wb);
+#pragma unroll
+                for (int e = 0; e < V; ++e) {
+                    de = fmaf(we[e], xv[e], de);
+                    db = fmaf(wb[e], xv[e], db);
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < V; ++e) {
+                const float zp = fmaf(av[e], xv[e], gv[e]);
+                const float z = zp * sigmoidf_(zp);
+                ss = fmaf(z, z, ss);
             }
         }
         ss = warp_sum(ss);
@@ -74,14 +137,23 @@ __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
             de = warp_sum(de);
             db = warp_sum(db);
         }
-        const float inv = 1.0f / sqrtf(ss + 1e-12f);
-        for (int i = lane; i < d; i += 32) {
-            const float xv = to_f<Tin>(x[i]);
-            const float zp = al[i] * xv + ga[i];
-            u[i] = from_f<Tout>(zp * sigmoidf_(zp) * inv);
+    }
+    const float inv = a.paper ? 1.0f / sqrtf(ss + 1e-12f) : 1.0f;
+#pragma unroll 4
+    for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
+        float xv[V];
+        Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x + i0), xv);
+        if (a.paper) {
+            float av[V], gv[V];
+            load_f32<V>(al + i0, av);
+            load_f32<V>(ga + i0, gv);
+#pragma unroll
+            for (int e = 0; e < V; ++e) {
+                const float zp = fmaf(av[e], xv[e], gv[e]);
+                xv[e] = zp * sigmoidf_(zp) * inv;
+            }
         }
-    } else {
-        for (int i = lane; i < d; i += 32) u[i] = from_f<Tout>(to_f<Tin>(x[i]));
+        store_vec<Tout, V>(u + i0, xv);
     }
     if (!a.query && lane == 0) {
         float e;

@@ -1,28 +1,33 @@
 // bf16 tensor-core path of one TTL segment step (tcgen05 + TMEM + TMA, sm_103a).
 //
 // A segment step of the SiLU-MLP memory M(u) = SiLU(u W1^T) W2 (Eq. 3 form) on
-// T tokens is four dense contractions (Eq. 10):
-//   phase A (per token tile x hidden tile, two TMEM accumulators)
-//       H = U W1^T            K = d_in      (memory forward)
-//       R = Y W2^T            K = d_out     (Y = [K || V] the targets of Eq. 7)
-//     fused epilogue: A = SiLU(H), dH = c_t R * SiLU'(H), At = c_t A with
-//     c_t = -eta_t / T' (Eq. 7's loss is linear in M, so dL/dO = -eta Y / T'
-//     does not depend on W and the target tile can be multiplied directly);
-//     writes dH^T and At^T (bf16, [hidden][token]) and the loss partial
-//     sum_t sum_h A_th R_th = sum_t y_t . M(u_t).
-//   phase B (per hidden tile x column tile of [W1 | W2])
-//       G1 = dH^T U           K = T'        (gradient of W1)
-//       G2 = At^T Y           K = T'        (gradient of W2)
-//     fused epilogue (Eq. 8, App. A): mu = beta mu + G; W = s W_raw - mu with s
-//     the previous segment's pending row renormalisation; stores W (fp32), mu,
-//     the bf16 operand copy of W and the new row sums of squares.
+// T tokens is four dense contractions (Eq. 10), done in two persistent kernels:
 //
-// Each CTA: 4 warps.  Warp 0 lane 0 drives TMA into a 3-stage shared-memory ring
-// (128-byte swizzle), warp 1 lane 0 issues tcgen05.mma (M = 128, N = 128,
-// K = 16 per instruction) into TMEM, then all 4 warps drain TMEM (one TMEM lane
-// quarter per warp).  ~98 KB of shared memory per CTA, so two CTAs share an SM
-// and one CTA's memory-bound epilogue overlaps the other's MMA main loop.
-// Every wait is bounded (kWaitLimitNs); a timeout latches DEV_TIMEOUT.
+//   phase A, tile = (chain, 128 tokens, 128 hidden units), two TMEM accumulators
+//       H = U W1^T            K = d_in      (memory forward)
+//       R = Y W2^T            K = d_out     (Y = [K || V], the targets of Eq. 7)
+//     fused epilogue: A = SiLU(H), dH = c_t R * SiLU'(H), At = c_t A with
+//     c_t = -eta_t / T'.  Eq. 7's loss is linear in M, so dL/dO = -eta Y / T'
+//     does not depend on W and the raw target tile is the right operand.
+//     Writes dH and At row-major (bf16 [token][hidden]) and the loss partial
+//     sum_t sum_h A_th R_th = sum_t y_t . M(u_t).
+//
+//   phase B, tile = (chain, 128 columns of [W1 | W2], 256 hidden units)
+//       G1^T = U^T dH         K = T'        (gradient of W1, transposed)
+//       G2^T = Y^T At         K = T'        (gradient of W2, transposed)
+//     Both operands are read MN-major straight from the row-major buffers.
+//     The accumulator is transposed (TMEM lane = weight column) so the fused
+//     update epilogue (Eq. 8, App. A) walks the fp32 state row by row with
+//     128-byte coalesced loads and stores: mu = beta mu + G; W = s W_raw - mu
+//     (s = the previous segment's pending row renormalisation); it writes W,
+//     mu, the bf16 operand copy and the new row sums of squares.
+//
+// Both kernels: one CTA per SM, persistent over a static tile schedule, 10 warps.
+// Warp 0 lane 0 streams operand tiles with TMA into a shared-memory ring
+// (128-byte swizzle), warp 1 lane 0 issues tcgen05.mma into one of two TMEM
+// accumulator buffers, warps 2..9 drain the other buffer, so the epilogue of
+// tile i overlaps the main loop of tile i+1.  Every mbarrier wait is bounded
+// (kWaitLimitNs); a timeout latches DEV_TIMEOUT and the kernel winds down.
 #include <mutex>
 
 #include "mone_common.cuh"
@@ -31,21 +36,37 @@ namespace mone {
 
 namespace {
 
-constexpr int BM = 128;                 // MMA M (TMEM lanes)
-constexpr int BN = 128;                 // MMA N
-constexpr int BK = 64;                  // 64 bf16 = one 128-byte swizzle row
-constexpr int STAGES = 3;
-constexpr int A_TILE = BM * BK * 2;     // 16 KB
-constexpr int B_TILE = BN * BK * 2;     // 16 KB
-constexpr int STAGE_BYTES = A_TILE + B_TILE;
-constexpr int RING_BYTES = STAGES * STAGE_BYTES;
-constexpr int SMEM_BYTES = RING_BYTES + 1024 /*align slack*/ + 2048 /*barriers, scales*/;
+constexpr int BK = 64;                    // 64 bf16 = one 128-byte swizzle row
+constexpr int EPI_WARPS = 8;
+constexpr int THREADS = 64 + EPI_WARPS * 32;
+constexpr int EPI_THREADS = EPI_WARPS * 32;
+constexpr uint32_t EPI_BAR = 1;           // named barrier among the epilogue warps
 
-static_assert(2 * BN * BM * 2 <= RING_BYTES, "phase A staging must fit in the ring");
-static_assert(BM * BN * 4 <= RING_BYTES, "phase B staging must fit in the ring");
+// phase A
+constexpr int A_BM = 128, A_BN = 128, A_STAGES = 6;
+constexpr int A_STAGE = (A_BM + A_BN) * BK * 2;           // 32 KB
+// phase B
+constexpr int B_BM = 128, B_BN = 256, B_STAGES = 4;
+constexpr int B_STAGE = (B_BM + B_BN) * BK * 2;           // 48 KB
+constexpr int BOX = 64 * BK * 2;                          // one 64 x 64 MN-major box, 8 KB
+
+template <int STAGES, int STAGE, int TABLE>
+struct Layout {
+    static constexpr int RING = STAGES * STAGE;
+    static constexpr int BARS = RING;                     // full[S], empty[S], tfull[2], tempty[2]
+    static constexpr int SLOT = BARS + (2 * STAGES + 4) * 8;
+    static constexpr int FLAG = SLOT + 16;
+    static constexpr int TAB = FLAG + 16;
+    static constexpr int END = TAB + TABLE * 4;
+    static constexpr int DYN = END + 1024;                // + alignment slack
+};
+// phase A table: [2 parity][2 matrix][A_BN] scales; phase B: [2][B_BN] scales + [2][8] beta partials
+using LA = Layout<A_STAGES, A_STAGE, 4 * A_BN>;
+using LB = Layout<B_STAGES, B_STAGE, 2 * B_BN + 16>;
+static_assert(LA::DYN <= 227 * 1024 && LB::DYN <= 227 * 1024, "shared memory budget");
 
 struct TcArgs {
-    int d_in, d_out, d_hid, T, Tp, c0, C, paper, momentum, renorm_pending, parity;
+    int d_in, d_out, d_hid, T, Tp, c0, nc, C, paper, momentum, renorm_pending, parity;
     int u_row0, u_chain0, y_row0;
     float lr;
     const float* eta_in;        // plain-mode caller rates, offset to the segment start, or null
@@ -57,7 +78,7 @@ struct TcArgs {
     bf16 *W1b, *W2b;
     const float *n1, *n2;
     float* sumsq;               // [2 parity][2 matrix][C][d_hid]
-    bf16 *dHt, *Att;            // [C][d_hid][T]
+    bf16 *dH, *At;              // [C][T][d_hid]
     float* loss;                // [nc] or null
     int* status;
 };
@@ -66,232 +87,90 @@ __device__ __forceinline__ float* ss_row(const TcArgs& a, int parity, int which,
     return a.sumsq + ((size_t)(parity * 2 + which) * a.C + cs) * a.d_hid;
 }
 
-struct Smem {
-    uint8_t* ring;
-    uint32_t full0, empty0, accb;
-    uint32_t* tmem_slot;
-    float* scratch;             // 2*BN + 8 floats
+struct Ctl {
+    uint8_t* base;
+    uint32_t bars;
+    __device__ uint32_t full(int s) const { return bars + 8 * s; }
+    __device__ uint32_t empty(int s, int S) const { return bars + 8 * (S + s); }
+    __device__ uint32_t tfull(int b, int S) const { return bars + 8 * (2 * S + b); }
+    __device__ uint32_t tempty(int b, int S) const { return bars + 8 * (2 * S + 2 + b); }
 };
 
-__device__ __forceinline__ Smem carve(uint8_t* raw) {
-    Smem s;
-    s.ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
-    uint64_t* bars = reinterpret_cast<uint64_t*>(s.ring + RING_BYTES);
-    s.full0 = smem_u32(bars);
-    s.empty0 = s.full0 + 8 * STAGES;
-    s.accb = s.full0 + 16 * STAGES;
-    s.tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 1);
-    s.scratch = reinterpret_cast<float*>(s.tmem_slot + 4);
-    return s;
+template <class L, int STAGES>
+__device__ __forceinline__ Ctl setup(uint8_t* raw) {
+    Ctl c;
+    c.base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
+    c.bars = smem_u32(c.base + L::BARS);
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < STAGES; ++i) {
+            mbar_init(c.full(i), 1);
+            mbar_init(c.empty(i, STAGES), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(c.tfull(b, STAGES), 1);
+            mbar_init(c.tempty(b, STAGES), EPI_WARPS);
+        }
+        fence_mbar_init();
+    }
+    if (threadIdx.x / 32 == 0) {
+        tmem_alloc(smem_u32(c.base + L::SLOT), 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    return c;
 }
 
-__device__ __forceinline__ void init_barriers(const Smem& s) {
-    for (int i = 0; i < STAGES; ++i) {
-        mbar_init(s.full0 + 8 * i, 1);
-        mbar_init(s.empty0 + 8 * i, 1);
-    }
-    mbar_init(s.accb, 1);
-    fence_mbar_init();
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
 }
 
 // ------------------------------------------------------------------ phase A
 
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(THREADS, 1)
 tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmW1,
                   const __grid_constant__ CUtensorMap tmW2, const TcArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    const Smem sm = carve(smem_raw);
-    float* s_sc1 = sm.scratch;
-    float* s_sc2 = sm.scratch + BN;
-    float* s_red = sm.scratch + 2 * BN;
-
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int ttile = blockIdx.x, h0 = blockIdx.y * BN, cz = blockIdx.z, cs = a.c0 + cz;
-
-    if (tid == 0) {
-        init_barriers(sm);
-        tma_prefetch_map(&tmU);
-        tma_prefetch_map(&tmK);
-        tma_prefetch_map(&tmV);
-        tma_prefetch_map(&tmW1);
-        tma_prefetch_map(&tmW2);
-    }
-    if (warp == 0) {
-        tmem_alloc(smem_u32(sm.tmem_slot), 2 * BN);
-        tmem_relinquish();
-    }
-    {   // renorm scales of this hidden tile; zero this segment's row sums
-        const int h = h0 + tid;
-        float s1 = 1.f, s2 = 1.f;
-        if (a.renorm_pending) {
-            s1 = renorm_scale(a.n1[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 0, cs)[h]);
-            s2 = renorm_scale(a.n2[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 1, cs)[h]);
-        }
-        s_sc1[tid] = s1;
-        s_sc2[tid] = s2;
-        if (ttile == 0) {
-            ss_row(a, a.parity, 0, cs)[h] = 0.f;
-            ss_row(a, a.parity, 1, cs)[h] = 0.f;
-        }
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *sm.tmem_slot;
-
-    const int KB1 = a.d_in / BK, KB2 = a.d_out / BK, KB = KB1 + KB2, half = (a.d_out / 2) / BK;
-    const int trow = ttile * BM;
+    const Ctl c = setup<LA, A_STAGES>(smem_raw);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + LA::SLOT);
+    const int n_tt = a.T / A_BM, n_ht = a.d_hid / A_BN;
+    const int ntiles = a.nc * n_ht * n_tt;
+    const int KB1 = a.d_in / BK, KB = KB1 + a.d_out / BK, half = (a.d_out / 2) / BK;
 
     if (warp == 0) {
         if (lane == 0) {
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % STAGES;
-                const uint32_t it = kb / STAGES;
-                if (kb >= STAGES && !mbar_wait(sm.empty0 + 8 * s, (it - 1) & 1, a.status)) break;
-                const uint32_t sa = smem_u32(sm.ring + s * STAGE_BYTES), sb = sa + A_TILE, fb = sm.full0 + 8 * s;
-                mbar_expect_tx(fb, STAGE_BYTES);
-                if (kb < KB1) {
-                    tma_load_3d(sa, &tmU, fb, kb * BK, a.u_row0 + trow, a.u_chain0 + cz);
-                    tma_load_3d(sb, &tmW1, fb, kb * BK, h0, cs);
-                } else {
-                    const int k2 = kb - KB1;
-                    if (k2 < half)
-                        tma_load_3d(sa, &tmK, fb, k2 * BK, a.y_row0 + trow, cz);
-                    else
-                        tma_load_3d(sa, &tmV, fb, (k2 - half) * BK, a.y_row0 + trow, cz);
-                    tma_load_3d(sb, &tmW2, fb, k2 * BK, h0, cs);
-                }
-            }
-        }
-        __syncwarp();
-    } else if (warp == 1) {
-        if (lane == 0) {
-            const uint32_t idesc = idesc_bf16_f32(BM, BN, false, false);
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % STAGES;
-                if (!mbar_wait(sm.full0 + 8 * s, (kb / STAGES) & 1, a.status)) break;
-                tc_fence_after();
-                const uint32_t sa = smem_u32(sm.ring + s * STAGE_BYTES), sb = sa + A_TILE;
-                const uint32_t d = tmem + (kb < KB1 ? 0u : (uint32_t)BN);
-                const bool first = (kb == 0 || kb == KB1);
-#pragma unroll
-                for (int k = 0; k < BK / 16; ++k)
-                    umma_bf16(d, sdesc_sw128(sa + k * 32, 16), sdesc_sw128(sb + k * 32, 16), idesc,
-                              (first && k == 0) ? 0u : 1u);
-                umma_commit(sm.empty0 + 8 * s);
-            }
-            umma_commit(sm.accb);
-        }
-        __syncwarp();
-    }
-
-    // ---- epilogue: thread = token row of the tile
-    mbar_wait(sm.accb, 0, a.status);
-    tc_fence_after();
-    const int row = warp * 32 + lane;
-    const int t = trow + row;
-    float ct = 0.f;
-    if (t < a.Tp) {
-        const float e = a.paper ? a.eta[(size_t)cs * a.T + t]
-                                : (a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr);
-        ct = -e / (float)a.Tp;
-    }
-    bf16* sdH = reinterpret_cast<bf16*>(sm.ring);      // [BN][BM]
-    bf16* sA = sdH + BN * BM;                          // [BN][BM]
-    float lsum = 0.f;
-    const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
-#pragma unroll 1
-    for (int j0 = 0; j0 < BN; j0 += 32) {
-        float hv[32], rv[32];
-        tmem_ld32(lane_base + j0, hv);
-        tmem_ld32(lane_base + BN + j0, rv);
-#pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-            const int h = j0 + jj;
-            const float x = hv[jj] * s_sc1[h];
-            const float r = rv[jj] * s_sc2[h];
-            const float sg = sigmoidf_(x);
-            const float av = x * sg;
-            const float ds = sg * (1.f + x * (1.f - sg));
-            lsum = fmaf(av, r, lsum);
-            sdH[h * BM + row] = __float2bfloat16_rn(ct * r * ds);
-            sA[h * BM + row] = __float2bfloat16_rn(ct * av);
-        }
-    }
-    tc_fence_before();
-    __syncthreads();
-    {
-        constexpr int VPR = BM / 8;  // 16-byte vectors per hidden row
-        const size_t base = ((size_t)cs * a.d_hid + h0) * a.T + trow;
-        for (int v = tid; v < BN * VPR; v += 128) {
-            const int h = v / VPR, q = v % VPR;
-            const size_t off = base + (size_t)h * a.T + q * 8;
-            *reinterpret_cast<uint4*>(a.dHt + off) = *reinterpret_cast<const uint4*>(sdH + h * BM + q * 8);
-            *reinterpret_cast<uint4*>(a.Att + off) = *reinterpret_cast<const uint4*>(sA + h * BM + q * 8);
-        }
-    }
-    if (a.loss) {
-        lsum = warp_sum(lsum);
-        if (lane == 0) s_red[warp] = lsum;
-        __syncthreads();
-        if (tid == 0) atomicAdd(&a.loss[cz], -(s_red[0] + s_red[1] + s_red[2] + s_red[3]) / (float)a.Tp);
-    }
-    __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, 2 * BN);
-}
-
-// ------------------------------------------------------------------ phase B
-
-__global__ void __launch_bounds__(128, 1)
-tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmDH, const __grid_constant__ CUtensorMap tmAT,
-                  const __grid_constant__ CUtensorMap tmUb, const __grid_constant__ CUtensorMap tmKb,
-                  const __grid_constant__ CUtensorMap tmVb, const TcArgs a) {
-    extern __shared__ uint8_t smem_raw[];
-    const Smem sm = carve(smem_raw);
-    float* s_red = sm.scratch;
-
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int col0 = blockIdx.x * BN, h0 = blockIdx.y * BM, cz = blockIdx.z, cs = a.c0 + cz;
-    const bool isW1 = col0 < a.d_in;
-    const int dh = a.d_out / 2;
-
-    if (tid == 0) {
-        init_barriers(sm);
-        tma_prefetch_map(isW1 ? &tmDH : &tmAT);
-        tma_prefetch_map(isW1 ? &tmUb : &tmKb);
-        if (!isW1) tma_prefetch_map(&tmVb);
-    }
-    if (warp == 0) {
-        tmem_alloc(smem_u32(sm.tmem_slot), BN);
-        tmem_relinquish();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *sm.tmem_slot;
-
-    const int KB = (a.Tp + BK - 1) / BK;  // tokens beyond T' carry zero dH / At
-    if (warp == 0) {
-        if (lane == 0) {
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % STAGES;
-                const uint32_t it = kb / STAGES;
-                if (kb >= STAGES && !mbar_wait(sm.empty0 + 8 * s, (it - 1) & 1, a.status)) break;
-                const uint32_t sa = smem_u32(sm.ring + s * STAGE_BYTES), sb = sa + A_TILE, fb = sm.full0 + 8 * s;
-                mbar_expect_tx(fb, STAGE_BYTES);
-                tma_load_3d(sa, isW1 ? &tmDH : &tmAT, fb, kb * BK, h0, cs);
-#pragma unroll
-                for (int b = 0; b < BN / 64; ++b) {
-                    const uint32_t dst = sb + b * (64 * BK * 2);
-                    if (isW1) {
-                        tma_load_3d(dst, &tmUb, fb, col0 + b * 64, a.u_row0 + kb * BK, a.u_chain0 + cz);
+            tma_prefetch_map(&tmU);
+            tma_prefetch_map(&tmK);
+            tma_prefetch_map(&tmV);
+            tma_prefetch_map(&tmW1);
+            tma_prefetch_map(&tmW2);
+            uint32_t kc = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+                const int cz = tile / (n_ht * n_tt), ht = (tile / n_tt) % n_ht, tt = tile % n_tt;
+                const int cs = a.c0 + cz, h0 = ht * A_BN, trow = tt * A_BM;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % A_STAGES;
+                    if (kc >= A_STAGES && !mbar_wait(c.empty(s, A_STAGES), ((kc / A_STAGES) - 1) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sa = smem_u32(c.base + s * A_STAGE), sb = sa + A_BM * BK * 2, fb = c.full(s);
+                    mbar_expect_tx(fb, A_STAGE);
+                    if (kb < KB1) {
+                        tma_load_3d(sa, &tmU, fb, kb * BK, a.u_row0 + trow, a.u_chain0 + cz);
+                        tma_load_3d(sb, &tmW1, fb, kb * BK, h0, cs);
                     } else {
-                        const int o = col0 - a.d_in + b * 64;
-                        if (o < dh)
-                            tma_load_3d(dst, &tmKb, fb, o, a.y_row0 + kb * BK, cz);
+                        const int k2 = kb - KB1;
+                        if (k2 < half)
+                            tma_load_3d(sa, &tmK, fb, k2 * BK, a.y_row0 + trow, cz);
                         else
-                            tma_load_3d(dst, &tmVb, fb, o - dh, a.y_row0 + kb * BK, cz);
+                            tma_load_3d(sa, &tmV, fb, (k2 - half) * BK, a.y_row0 + trow, cz);
+                        tma_load_3d(sb, &tmW2, fb, k2 * BK, h0, cs);
                     }
                 }
             }
@@ -299,115 +178,307 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmDH, const __grid_constan
         __syncwarp();
     } else if (warp == 1) {
         if (lane == 0) {
-            const uint32_t idesc = idesc_bf16_f32(BM, BN, false, true);
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % STAGES;
-                if (!mbar_wait(sm.full0 + 8 * s, (kb / STAGES) & 1, a.status)) break;
+            const uint32_t idesc = idesc_bf16_f32(A_BM, A_BN, false, false);
+            uint32_t kc = 0;
+            int local = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++local) {
+                const int b = local & 1;
+                if (local >= 2 && !mbar_wait(c.tempty(b, A_STAGES), ((local >> 1) - 1) & 1, a.status)) break;
                 tc_fence_after();
-                const uint32_t sa = smem_u32(sm.ring + s * STAGE_BYTES), sb = sa + A_TILE;
+                const uint32_t dH = tmem + b * 256, dR = dH + A_BN;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % A_STAGES;
+                    if (!mbar_wait(c.full(s), (kc / A_STAGES) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(c.base + s * A_STAGE), sb = sa + A_BM * BK * 2;
+                    const bool first = (kb == 0 || kb == KB1);
 #pragma unroll
-                for (int k = 0; k < BK / 16; ++k)
-                    umma_bf16(tmem, sdesc_sw128(sa + k * 32, 16), sdesc_sw128(sb + k * 16 * 128, 64 * BK * 2),
-                              idesc, (kb == 0 && k == 0) ? 0u : 1u);
-                umma_commit(sm.empty0 + 8 * s);
+                    for (int k = 0; k < BK / 16; ++k)
+                        umma_bf16(kb < KB1 ? dH : dR, sdesc_sw128(sa + k * 32, 16), sdesc_sw128(sb + k * 32, 16),
+                                  idesc, (first && k == 0) ? 0u : 1u);
+                    umma_commit(c.empty(s, A_STAGES));
+                }
+                umma_commit(c.tfull(b, A_STAGES));
             }
-            umma_commit(sm.accb);
         }
         __syncwarp();
-    }
-
-    // momentum decay beta_s = sigmoid(mean_t w_beta . x_t + b_beta) while the MMAs run
-    float beta = 0.f;
-    if (a.momentum) {
-        float v = 0.f;
-        for (int t = tid; t < a.Tp; t += 128) v += a.dbeta[(size_t)cs * a.T + t];
-        v = warp_sum(v);
-        if (lane == 0) s_red[warp] = v;
-        __syncthreads();
-        beta = sigmoidf_((s_red[0] + s_red[1] + s_red[2] + s_red[3]) / (float)a.Tp + a.b_beta[cs]);
-    }
-
-    // ---- epilogue part 1: TMEM -> shared staging (thread = hidden row)
-    mbar_wait(sm.accb, 0, a.status);
-    tc_fence_after();
-    float4* stg = reinterpret_cast<float4*>(sm.ring);  // [BM rows][BN/4 float4], XOR-swizzled
-    {
-        const int r = warp * 32 + lane;
-        const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+    } else {
+        // ---- epilogue warps: TMEM lane quarter q, hidden-column half ch
+        const int e = warp - 2, q = warp & 3, ch = e >> 2, et = threadIdx.x - 64;
+        float* table = reinterpret_cast<float*>(c.base + LA::TAB);
+        int* flag = reinterpret_cast<int*>(c.base + LA::FLAG);
+        int local = 0;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local) {
+            const int cz = tile / (n_ht * n_tt), ht = (tile / n_tt) % n_ht, tt = tile % n_tt;
+            const int cs = a.c0 + cz, h0 = ht * A_BN, trow = tt * A_BM;
+            const int b = local & 1;
+            float* tab = table + b * 2 * A_BN;
+            if (et < A_BN) {
+                const int h = h0 + et;
+                float s1 = 1.f, s2 = 1.f;
+                if (a.renorm_pending) {
+                    s1 = renorm_scale(a.n1[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 0, cs)[h]);
+                    s2 = renorm_scale(a.n2[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 1, cs)[h]);
+                }
+                tab[et] = s1;
+                tab[A_BN + et] = s2;
+                if (tt == 0) {
+                    ss_row(a, a.parity, 0, cs)[h] = 0.f;
+                    ss_row(a, a.parity, 1, cs)[h] = 0.f;
+                }
+            }
+            if (et == 0) flag[b] = mbar_wait(c.tfull(b, A_STAGES), (local >> 1) & 1, a.status) ? 1 : 0;
+            __syncwarp();
+            named_bar_sync(EPI_BAR, EPI_THREADS);
+            if (!flag[b]) break;
+            tc_fence_after();
+            const int row = q * 32 + lane;
+            const int t = trow + row;
+            float ct = 0.f;
+            if (t < a.Tp) {
+                const float ev = a.paper ? a.eta[(size_t)cs * a.T + t]
+                                         : (a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr);
+                ct = -ev / (float)a.Tp;
+            }
+            const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
+            bf16* dHrow = a.dH + ((size_t)cs * a.T + t) * a.d_hid + h0;
+            bf16* Arow = a.At + ((size_t)cs * a.T + t) * a.d_hid + h0;
+            float lsum = 0.f;
 #pragma unroll 1
-        for (int q = 0; q < BN / 32; ++q) {
-            float g[32];
-            tmem_ld32(lane_base + q * 32, g);
+            for (int cc = 0; cc < 2; ++cc) {
+                const int c0 = ch * 64 + cc * 32;
+                float hv[32], rv[32];
+                tmem_ld32(lane_base + c0, hv);
+                tmem_ld32(lane_base + A_BN + c0, rv);
+                if (cc == 1) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(c.tempty(b, A_STAGES));
+                }
+                uint32_t pd[16], pa[16];
 #pragma unroll
-            for (int v = 0; v < 8; ++v) {
-                const int f = q * 8 + v;
-                stg[r * (BN / 4) + (f ^ (r & 31))] = make_float4(g[4 * v], g[4 * v + 1], g[4 * v + 2], g[4 * v + 3]);
+                for (int j = 0; j < 32; j += 2) {
+                    float dv[2], av2[2];
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        const float x = hv[j + u] * tab[c0 + j + u];
+                        const float r = rv[j + u] * tab[A_BN + c0 + j + u];
+                        const float sg = sigmoid_fast(x);
+                        const float av = x * sg;
+                        lsum = fmaf(av, r, lsum);
+                        dv[u] = ct * r * (sg * (1.f + x * (1.f - sg)));
+                        av2[u] = ct * av;
+                    }
+                    pd[j / 2] = pack_bf16(dv[0], dv[1]);
+                    pa[j / 2] = pack_bf16(av2[0], av2[1]);
+                }
+#pragma unroll
+                for (int v = 0; v < 4; ++v) {
+                    *reinterpret_cast<uint4*>(dHrow + c0 + v * 8) =
+                        make_uint4(pd[4 * v], pd[4 * v + 1], pd[4 * v + 2], pd[4 * v + 3]);
+                    *reinterpret_cast<uint4*>(Arow + c0 + v * 8) =
+                        make_uint4(pa[4 * v], pa[4 * v + 1], pa[4 * v + 2], pa[4 * v + 3]);
+                }
+            }
+            if (a.loss) {
+                lsum = warp_sum(lsum);
+                if (lane == 0) atomicAdd(&a.loss[cz], -lsum / (float)a.Tp);
             }
         }
     }
-    tc_fence_before();
     __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, 512);
+}
 
-    // ---- epilogue part 2: row-wise fused update, coalesced along columns
-    const int which = isW1 ? 0 : 1;
-    const int width = isW1 ? a.d_in : a.d_out;
-    const int cl = isW1 ? col0 : col0 - a.d_in;
-    float* W = (isW1 ? a.W1 : a.W2) + (size_t)cs * a.d_hid * width;
-    float* M = a.momentum ? (isW1 ? a.mu1 : a.mu2) + (size_t)cs * a.d_hid * width : nullptr;
-    bf16* Wb = (isW1 ? a.W1b : a.W2b) + (size_t)cs * a.d_hid * width;
-    const float* n0 = (isW1 ? a.n1 : a.n2) + (size_t)cs * a.d_hid;
-    const float* prev = ss_row(a, a.parity ^ 1, which, cs);
-    float* cur = ss_row(a, a.parity, which, cs);
-    bool finite = true;
-    constexpr int RB = 8;  // rows in flight per warp
+// ------------------------------------------------------------------ phase B
+
+__global__ void __maxnreg__(200)
+tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant__ CUtensorMap tmKb,
+                  const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmDH,
+                  const __grid_constant__ CUtensorMap tmAT, const TcArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    const Ctl c = setup<LB, B_STAGES>(smem_raw);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + LB::SLOT);
+    const int n_ct = (a.d_in + a.d_out) / B_BM, n_ht = a.d_hid / B_BN;
+    const int ntiles = a.nc * n_ht * n_ct;
+    const int KB = (a.Tp + BK - 1) / BK;  // tokens beyond T' carry zero dH / At
+    const int dhalf = a.d_out / 2;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            tma_prefetch_map(&tmUb);
+            tma_prefetch_map(&tmKb);
+            tma_prefetch_map(&tmVb);
+            tma_prefetch_map(&tmDH);
+            tma_prefetch_map(&tmAT);
+            uint32_t kc = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+                const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
+                const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
+                const bool isW1 = col0 < a.d_in;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % B_STAGES;
+                    if (kc >= B_STAGES && !mbar_wait(c.empty(s, B_STAGES), ((kc / B_STAGES) - 1) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sa = smem_u32(c.base + s * B_STAGE), sb = sa + B_BM * BK * 2, fb = c.full(s);
+                    mbar_expect_tx(fb, B_STAGE);
+#pragma unroll
+                    for (int bx = 0; bx < B_BM / 64; ++bx) {
+                        const uint32_t dst = sa + bx * BOX;
+                        if (isW1) {
+                            tma_load_3d(dst, &tmUb, fb, col0 + bx * 64, a.u_row0 + kb * BK, a.u_chain0 + cz);
+                        } else {
+                            const int o = col0 - a.d_in + bx * 64;
+                            if (o < dhalf)
+                                tma_load_3d(dst, &tmKb, fb, o, a.y_row0 + kb * BK, cz);
+                            else
+                                tma_load_3d(dst, &tmVb, fb, o - dhalf, a.y_row0 + kb * BK, cz);
+                        }
+                    }
+#pragma unroll
+                    for (int bx = 0; bx < B_BN / 64; ++bx)
+                        tma_load_3d(sb + bx * BOX, isW1 ? &tmDH : &tmAT, fb, h0 + bx * 64, kb * BK, cs);
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(B_BM, B_BN, true, true);
+            uint32_t kc = 0;
+            int local = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++local) {
+                const int b = local & 1;
+                if (local >= 2 && !mbar_wait(c.tempty(b, B_STAGES), ((local >> 1) - 1) & 1, a.status)) break;
+                tc_fence_after();
+                const uint32_t d = tmem + b * 256;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % B_STAGES;
+                    if (!mbar_wait(c.full(s), (kc / B_STAGES) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(c.base + s * B_STAGE), sb = sa + B_BM * BK * 2;
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k)
+                        umma_bf16(d, sdesc_sw128(sa + k * 16 * 128, BOX), sdesc_sw128(sb + k * 16 * 128, BOX), idesc,
+                                  (kb == 0 && k == 0) ? 0u : 1u);
+                    umma_commit(c.empty(s, B_STAGES));
+                }
+                umma_commit(c.tfull(b, B_STAGES));
+            }
+        }
+        __syncwarp();
+    } else {
+        // ---- epilogue warps: TMEM lane quarter q (= 32 weight columns), hidden half hh
+        const int e = warp - 2, q = warp & 3, hh = e >> 2, et = threadIdx.x - 64;
+        float* table = reinterpret_cast<float*>(c.base + LB::TAB);
+        float* bred = table + 2 * B_BN;  // [2][8]
+        int* flag = reinterpret_cast<int*>(c.base + LB::FLAG);
+        bool finite = true;
+        int local = 0;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local) {
+            const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
+            const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
+            const bool isW1 = col0 < a.d_in;
+            const int which = isW1 ? 0 : 1;
+            const int b = local & 1;
+            float* tab = table + b * B_BN;
+            {   // renorm scales of this tile's 256 rows, momentum decay partials
+                const int h = h0 + et;
+                tab[et] = a.renorm_pending
+                              ? renorm_scale((isW1 ? a.n1 : a.n2)[(size_t)cs * a.d_hid + h],
+                                             ss_row(a, a.parity ^ 1, which, cs)[h])
+                              : 1.f;
+                if (a.momentum) {
+                    float v = 0.f;
+                    for (int t = et; t < a.Tp; t += EPI_THREADS) v += a.dbeta[(size_t)cs * a.T + t];
+                    v = warp_sum(v);
+                    if (lane == 0) bred[b * 8 + e] = v;
+                }
+            }
+            if (et == 0) flag[b] = mbar_wait(c.tfull(b, B_STAGES), (local >> 1) & 1, a.status) ? 1 : 0;
+            __syncwarp();
+            named_bar_sync(EPI_BAR, EPI_THREADS);
+            if (!flag[b]) break;
+            tc_fence_after();
+            float beta = 0.f;
+            if (a.momentum) {
+                float tot = 0.f;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) tot += bred[b * 8 + i];
+                beta = sigmoidf_(tot / (float)a.Tp + a.b_beta[cs]);
+            }
+            const int width = isW1 ? a.d_in : a.d_out;
+            const int col = (isW1 ? col0 : col0 - a.d_in) + q * 32 + lane;
+            float* W = (isW1 ? a.W1 : a.W2) + (size_t)cs * a.d_hid * width + col;
+            float* M = a.momentum ? (isW1 ? a.mu1 : a.mu2) + (size_t)cs * a.d_hid * width + col : nullptr;
+            bf16* Wb = (isW1 ? a.W1b : a.W2b) + (size_t)cs * a.d_hid * width + col;
+            float* cur = ss_row(a, a.parity, which, cs);
+            const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
 #pragma unroll 1
-    for (int rb = 0; rb < 32; rb += RB) {
-        float4 gv[RB], wv[RB], mv[RB];
+            for (int g = 0; g < 4; ++g) {
+                const int hb = hh * 128 + g * 32;  // first hidden unit of this group, within the tile
+                float gv[32];
+                tmem_ld32(lane_base + hb, gv);
+                if (g == 3) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(c.tempty(b, B_STAGES));
+                }
+                float wv[32], mv[32];
+                float* wp = W + (size_t)(h0 + hb) * width;
+                float* mp = M ? M + (size_t)(h0 + hb) * width : nullptr;
+                bf16* bp = Wb + (size_t)(h0 + hb) * width;
 #pragma unroll
-        for (int u = 0; u < RB; ++u) {
-            const int r = warp * 32 + rb + u;
-            const size_t off = (size_t)(h0 + r) * width + cl + lane * 4;
-            gv[u] = stg[r * (BN / 4) + (lane ^ (r & 31))];
-            wv[u] = *reinterpret_cast<const float4*>(W + off);
-            mv[u] = M ? *reinterpret_cast<const float4*>(M + off) : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
+                for (int j = 0; j < 32; ++j) {
+                    wv[j] = wp[j * width];
+                    mv[j] = mp ? mp[j * width] : 0.f;
+                }
 #pragma unroll
-        for (int u = 0; u < RB; ++u) {
-            const int r = warp * 32 + rb + u;
-            const int h = h0 + r;
-            const size_t off = (size_t)h * width + cl + lane * 4;
-            const float s = a.renorm_pending ? renorm_scale(n0[h], prev[h]) : 1.f;
-            float4 mn, wn;
-            mn.x = fmaf(beta, mv[u].x, gv[u].x);
-            mn.y = fmaf(beta, mv[u].y, gv[u].y);
-            mn.z = fmaf(beta, mv[u].z, gv[u].z);
-            mn.w = fmaf(beta, mv[u].w, gv[u].w);
-            wn.x = s * wv[u].x - mn.x;
-            wn.y = s * wv[u].y - mn.y;
-            wn.z = s * wv[u].z - mn.z;
-            wn.w = s * wv[u].w - mn.w;
-            *reinterpret_cast<float4*>(W + off) = wn;
-            if (M) *reinterpret_cast<float4*>(M + off) = mn;
-            __nv_bfloat162 b01 = __floats2bfloat162_rn(wn.x, wn.y);
-            __nv_bfloat162 b23 = __floats2bfloat162_rn(wn.z, wn.w);
-            uint2 packed;
-            packed.x = *reinterpret_cast<uint32_t*>(&b01);
-            packed.y = *reinterpret_cast<uint32_t*>(&b23);
-            *reinterpret_cast<uint2*>(Wb + off) = packed;
-            float ss = wn.x * wn.x + wn.y * wn.y + wn.z * wn.z + wn.w * wn.w;
-            finite = finite && isfinite(ss);
-            ss = warp_sum(ss);
-            if (lane == 0) atomicAdd(&cur[h], ss);
+                for (int j = 0; j < 32; ++j) {
+                    const float mn = fmaf(beta, mv[j], gv[j]);
+                    const float wn = fmaf(tab[hb + j], wv[j], -mn);
+                    wp[j * width] = wn;
+                    if (mp) mp[j * width] = mn;
+                    bp[j * width] = __float2bfloat16_rn(wn);
+                    finite = finite && isfinite(wn);
+                    wv[j] = wn * wn;
+                }
+                // transpose-reduce: afterwards lane j holds the 32-column partial of row hb + j
+#pragma unroll
+                for (int sft = 16; sft >= 1; sft >>= 1) {
+                    const bool upper = (lane & sft) != 0;
+#pragma unroll
+                    for (int k = 0; k < sft; ++k) {
+                        const float send = upper ? wv[k] : wv[k + sft];
+                        const float keep = upper ? wv[k + sft] : wv[k];
+                        wv[k] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+                    }
+                }
+                atomicAdd(&cur[h0 + hb + lane], wv[0]);
+            }
         }
+        if (!finite) atomicOr(a.status, DEV_NONFINITE);
     }
-    if (!finite) atomicOr(a.status, DEV_NONFINITE);
     __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, BN);
+    if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
 TcArgs make_args(const DevState& s, const SegWork& w) {
     TcArgs a{};
-    a.d_in = s.d_in; a.d_out = s.d_out; a.d_hid = s.d_hid; a.T = s.T; a.Tp = w.Tp; a.c0 = w.c0; a.C = s.C;
+    a.d_in = s.d_in; a.d_out = s.d_out; a.d_hid = s.d_hid; a.T = s.T; a.Tp = w.Tp; a.c0 = w.c0; a.nc = w.nc;
+    a.C = s.C;
     a.paper = s.mode == 1; a.momentum = s.momentum; a.renorm_pending = w.renorm_pending; a.parity = w.parity;
     a.u_row0 = a.paper ? 0 : (int)w.row0;
     a.u_chain0 = a.paper ? w.c0 : 0;
@@ -418,20 +489,25 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
     a.eta = s.eta; a.dbeta = s.dbeta; a.b_beta = s.b_beta;
     a.W1 = s.W1; a.W2 = s.W2; a.mu1 = s.mu1; a.mu2 = s.mu2; a.W1b = s.W1b; a.W2b = s.W2b;
     a.n1 = s.n1; a.n2 = s.n2; a.sumsq = s.sumsq;
-    a.dHt = reinterpret_cast<bf16*>(s.dHt); a.Att = reinterpret_cast<bf16*>(s.Att);
+    a.dH = reinterpret_cast<bf16*>(s.dHt); a.At = reinterpret_cast<bf16*>(s.Att);
     a.loss = w.loss; a.status = s.status;
     return a;
 }
 
 std::once_flag g_attr_once;
 cudaError_t g_attr_err = cudaSuccess;
+int g_sms = 0;
 
 cudaError_t ensure_attrs() {
     std::call_once(g_attr_once, [] {
-        g_attr_err = cudaFuncSetAttribute(tc_phase_a_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+        int dev = 0;
+        g_attr_err = cudaGetDevice(&dev);
         if (g_attr_err == cudaSuccess)
-            g_attr_err =
-                cudaFuncSetAttribute(tc_phase_b_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+            g_attr_err = cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err = cudaFuncSetAttribute(tc_phase_a_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LA::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LB::DYN);
     });
     return g_attr_err;
 }
@@ -443,8 +519,9 @@ cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputM
     cudaError_t e = ensure_attrs();
     if (e != cudaSuccess) return e;
     const TcArgs a = make_args(s, w);
-    dim3 grid(s.T / BM, s.d_hid / BN, w.nc);
-    tc_phase_a_kernel<<<grid, 128, SMEM_BYTES, st>>>(s.mode == 1 ? m.Ua : in.Xa, in.Ka, in.Va, m.W1b, m.W2b, a);
+    const int ntiles = w.nc * (s.T / A_BM) * (s.d_hid / A_BN);
+    const int grid = ntiles < g_sms ? ntiles : g_sms;
+    tc_phase_a_kernel<<<grid, THREADS, LA::DYN, st>>>(s.mode == 1 ? m.Ua : in.Xa, in.Ka, in.Va, m.W1b, m.W2b, a);
     return cudaGetLastError();
 }
 
@@ -453,8 +530,9 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
     cudaError_t e = ensure_attrs();
     if (e != cudaSuccess) return e;
     const TcArgs a = make_args(s, w);
-    dim3 grid((s.d_in + s.d_out) / BN, s.d_hid / BM, w.nc);
-    tc_phase_b_kernel<<<grid, 128, SMEM_BYTES, st>>>(m.dHt, m.Att, s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, a);
+    const int ntiles = w.nc * ((s.d_in + s.d_out) / B_BM) * (s.d_hid / B_BN);
+    const int grid = ntiles < g_sms ? ntiles : g_sms;
+    tc_phase_b_kernel<<<grid, THREADS, LB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.dH, m.At, a);
     return cudaGetLastError();
 }
 

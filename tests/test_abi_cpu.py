@@ -71,6 +71,7 @@ def test_init_rejects_unsupported_shapes(L):
     assert init_rc(L, cfg(head_dim=96, d_out=384, n_kv_heads=2)) == 2
     assert init_rc(L, cfg(d_out=512)) == 2                    # d_out != 2 * n_kv * hd
     assert init_rc(L, cfg(d_in=192)) == 2                     # bf16 tiles are 128 wide
+    assert init_rc(L, cfg(d_hid=384)) == 2                    # bf16 hidden tiles are 256 wide
     assert init_rc(L, cfg(seg_T=192)) == 2
     assert init_rc(L, cfg(seg_T=8192)) == 2
     assert init_rc(L, cfg(dtype=mone.MONE_FP32, d_in=96)) == 2
