@@ -180,6 +180,10 @@ mone_status mone_mem_set_timing(mone_mem* m, int enable);
 mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches);
 
 const char* mone_status_string(mone_status s);
+
+/* Text of the last CUDA error this thread saw inside the library ("" if none);
+ * valid until the thread's next library call. */
+const char* mone_last_error(void);
 int mone_abi_version(void);
 
 #ifdef __cplusplus

@@ -25,15 +25,16 @@ STATUS = {0: "MONE_OK", 1: "MONE_ERR_INVALID_ARG", 2: "MONE_ERR_UNSUPPORTED_SHAP
 # Every symbol include/mone.h declares.
 EXPORTS = ("mone_mem_init", "mone_ttl_segment", "mone_ttl_context", "mone_mem_generate_kv", "mone_mem_free",
            "mone_mem_read_state", "mone_mem_write_state", "mone_mem_sync", "mone_mem_launch_count",
-           "mone_status_string", "mone_abi_version", "mone_mem_set_timing", "mone_mem_kernel_time")
+           "mone_status_string", "mone_abi_version", "mone_mem_set_timing", "mone_mem_kernel_time",
+           "mone_last_error")
 
 KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read")
 
 
 class MoneError(RuntimeError):
-    def __init__(self, fn: str, code: int):
+    def __init__(self, fn: str, code: int, detail: str = ""):
         self.code = code
-        super().__init__(f"{fn} failed: {STATUS.get(code, code)}")
+        super().__init__(f"{fn} failed: {STATUS.get(code, code)}" + (f" ({detail})" if detail else ""))
 
 
 class mone_config(ctypes.Structure):
@@ -73,6 +74,7 @@ def lib(path: Optional[str] = None) -> ctypes.CDLL:
         "mone_mem_launch_count": ([vp], ll),
         "mone_status_string": ([i], ctypes.c_char_p),
         "mone_abi_version": ([], i),
+        "mone_last_error": ([], ctypes.c_char_p),
         "mone_mem_set_timing": ([vp, i], i),
         "mone_mem_kernel_time": ([vp, i, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ll)], i),
     }
@@ -104,7 +106,8 @@ def _stream(stream) -> Optional[int]:
 
 def _check(fn: str, rc: int):
     if rc != 0:
-        raise MoneError(fn, rc)
+        detail = lib().mone_last_error().decode() if rc in (3, 4) else ""
+        raise MoneError(fn, rc, detail)
 
 
 def make_config(n_ctx, n_layers, d_in, d_hid, d_out, n_kv_heads, head_dim, seg_T, dtype, mode, lr,
@@ -171,6 +174,10 @@ def mone_status_string(code: int) -> str:
 
 def mone_abi_version() -> int:
     return lib().mone_abi_version()
+
+
+def mone_last_error() -> str:
+    return lib().mone_last_error().decode()
 
 
 def mone_mem_set_timing(h: int, enable: bool):

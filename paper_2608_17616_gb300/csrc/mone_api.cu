@@ -3,6 +3,7 @@
 // All arithmetic runs in the kernels of ttl_prepass.cu, ttl_simt.cu and ttl_tc.cu.
 #include <algorithm>
 #include <cmath>
+#include <cstdio>
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
@@ -102,8 +103,11 @@ mone_status validate_config(const mone_config* c) {
     return MONE_OK;
 }
 
+thread_local char g_last_error[256] = "";
+
 mone_status cuda_status(cudaError_t e) {
     if (e == cudaSuccess) return MONE_OK;
+    std::snprintf(g_last_error, sizeof(g_last_error), "%s: %s", cudaGetErrorName(e), cudaGetErrorString(e));
     if (e == cudaErrorMemoryAllocation) return MONE_ERR_OOM;
     return MONE_ERR_CUDA;
 }
@@ -229,6 +233,8 @@ mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
 extern "C" {
 
 int mone_abi_version(void) { return MONE_ABI_VERSION; }
+
+const char* mone_last_error(void) { return g_last_error; }
 
 const char* mone_status_string(mone_status st) {
     switch (st) {

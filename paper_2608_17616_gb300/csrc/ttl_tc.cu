@@ -296,7 +296,7 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
 
 // ------------------------------------------------------------------ phase B
 
-__global__ void __maxnreg__(200)
+__global__ void __launch_bounds__(THREADS, 1)
 tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant__ CUtensorMap tmKb,
                   const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmDH,
                   const __grid_constant__ CUtensorMap tmAT, const TcArgs a) {
