@@ -73,6 +73,8 @@ struct TcMaps {
     CUtensorMap W1b, W2b;        // K-major boxes {64, 128}
     CUtensorMap dH, At;          // MN-major boxes {64, 64} over [C][T][d_hid]
     CUtensorMap Ua, Ub;          // scratch U: K-major {64,128} and MN {64,64}
+    CUtensorMap W1s, W2s, M1s, M2s;  // fp32 state chunks {128 cols, 32 rows}, no swizzle
+    CUtensorMap W1o, W2o;            // bf16 operand-copy chunks {128 cols, 32 rows}, no swizzle
 };
 struct TcInputMaps {
     CUtensorMap Xa, Xb, Ka, Kb, Va, Vb;  // per call: K-major {64,128} (a) and MN {64,64} (b)
@@ -83,8 +85,11 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
                               cudaStream_t st);
 int tc_kernels_per_segment();
 
-// Tensor-map encoder (driver entry point, resolved at run time).
+// Tensor-map encoders (driver entry point, resolved at run time).  3-D maps over
+// [chains][rows][inner]; bf16 maps use 128-byte swizzle, the *_plain ones none.
 bool encode_map_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t chains,
                         uint32_t box_inner, uint32_t box_rows);
+bool encode_map_plain_3d(CUtensorMap* map, const void* base, bool f32, uint64_t inner, uint64_t rows,
+                         uint64_t chains, uint32_t box_inner, uint32_t box_rows);
 
 }  // namespace mone

@@ -46,7 +46,7 @@ constexpr uint32_t EPI_BAR = 1;           // named barrier among the epilogue wa
 constexpr int A_BM = 128, A_BN = 128, A_STAGES = 6;
 constexpr int A_STAGE = (A_BM + A_BN) * BK * 2;           // 32 KB
 // phase B
-constexpr int B_BM = 128, B_BN = 256, B_STAGES = 4;
+constexpr int B_BM = 128, B_BN = 256;
 constexpr int B_STAGE = (B_BM + B_BN) * BK * 2;           // 48 KB
 constexpr int BOX = 64 * BK * 2;                          // one 64 x 64 MN-major box, 8 KB
 
@@ -62,8 +62,7 @@ struct Layout {
 };
 // phase A table: [2 parity][2 matrix][A_BN] scales; phase B: [2][B_BN] scales + [2][8] beta partials
 using LA = Layout<A_STAGES, A_STAGE, 4 * A_BN>;
-using LB = Layout<B_STAGES, B_STAGE, 2 * B_BN + 16>;
-static_assert(LA::DYN <= 227 * 1024 && LB::DYN <= 227 * 1024, "shared memory budget");
+static_assert(LA::DYN <= 227 * 1024, "shared memory budget");
 
 struct TcArgs {
     int d_in, d_out, d_hid, T, Tp, c0, nc, C, paper, momentum, renorm_pending, parity;
@@ -295,19 +294,81 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
 }
 
 // ------------------------------------------------------------------ phase B
+//
+// Warps: 0 operand producer (TMA), 1 MMA issuer, 2..5 epilogue (one per TMEM lane
+// quarter; thread = one weight column), 6 state producer.  The fp32 state of a
+// tile (256 rows x 128 columns of W and mu) moves in chunks of 32 rows through a
+// 3-slot shared-memory ring: the state producer TMA-loads a chunk ahead of time,
+// the epilogue updates it in place and TMA-stores it (with the bf16 copy) back.
 
-__global__ void __launch_bounds__(THREADS, 1)
+constexpr int S_ROWS = 32;                                 // hidden rows per state chunk
+constexpr int S_SLOTS = 3;
+constexpr int S_F32 = S_ROWS * B_BM * 4;                   // 16 KB
+constexpr int S_SLOT = 2 * S_F32 + S_ROWS * B_BM * 2;      // W, mu, bf16 copy: 40 KB
+constexpr int B_STAGES_V3 = 2;
+constexpr int B_THREADS = 7 * 32;
+constexpr int B_EPI_THREADS = 4 * 32;
+
+struct LayoutB {
+    static constexpr int RING = B_STAGES_V3 * B_STAGE;
+    static constexpr int STATE = RING;
+    static constexpr int BARS = STATE + S_SLOTS * S_SLOT;  // full[S] empty[S] tfull[2] tempty[2] sfull[N] sempty[N]
+    static constexpr int NBARS = 2 * B_STAGES_V3 + 4 + 2 * S_SLOTS;
+    static constexpr int SLOT = BARS + NBARS * 8;
+    static constexpr int FLAG = SLOT + 16;
+    static constexpr int TAB = FLAG + 16;                  // [2][B_BN] scales + [2][4] beta partials
+    static constexpr int END = TAB + (2 * B_BN + 8) * 4;
+    static constexpr int DYN = END + 1024;
+};
+static_assert(LayoutB::DYN <= 227 * 1024, "phase B shared memory budget");
+
+__global__ void __launch_bounds__(B_THREADS, 1)
 tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant__ CUtensorMap tmKb,
                   const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmDH,
-                  const __grid_constant__ CUtensorMap tmAT, const TcArgs a) {
+                  const __grid_constant__ CUtensorMap tmAT, const __grid_constant__ CUtensorMap tmW1s,
+                  const __grid_constant__ CUtensorMap tmW2s, const __grid_constant__ CUtensorMap tmM1s,
+                  const __grid_constant__ CUtensorMap tmM2s, const __grid_constant__ CUtensorMap tmW1o,
+                  const __grid_constant__ CUtensorMap tmW2o, const TcArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    const Ctl c = setup<LB, B_STAGES>(smem_raw);
+    using L = LayoutB;
+    uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const uint32_t bars = smem_u32(base + L::BARS);
+    auto full = [&](int s) { return bars + 8 * s; };
+    auto empty = [&](int s) { return bars + 8 * (B_STAGES_V3 + s); };
+    auto tfull = [&](int b) { return bars + 8 * (2 * B_STAGES_V3 + b); };
+    auto tempty = [&](int b) { return bars + 8 * (2 * B_STAGES_V3 + 2 + b); };
+    auto sfull = [&](int k) { return bars + 8 * (2 * B_STAGES_V3 + 4 + k); };
+    auto sempty = [&](int k) { return bars + 8 * (2 * B_STAGES_V3 + 4 + S_SLOTS + k); };
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + LB::SLOT);
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < B_STAGES_V3; ++i) {
+            mbar_init(full(i), 1);
+            mbar_init(empty(i), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(tfull(b), 1);
+            mbar_init(tempty(b), 4);
+        }
+        for (int k = 0; k < S_SLOTS; ++k) {
+            mbar_init(sfull(k), 1);
+            mbar_init(sempty(k), 1);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(base + L::SLOT), 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<uint32_t*>(base + L::SLOT);
+
     const int n_ct = (a.d_in + a.d_out) / B_BM, n_ht = a.d_hid / B_BN;
     const int ntiles = a.nc * n_ht * n_ct;
     const int KB = (a.Tp + BK - 1) / BK;  // tokens beyond T' carry zero dH / At
     const int dhalf = a.d_out / 2;
+    const int chunk_bytes = a.momentum ? 2 * S_F32 : S_F32;
 
     if (warp == 0) {
         if (lane == 0) {
@@ -323,12 +384,12 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
                 const bool isW1 = col0 < a.d_in;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
-                    const int s = kc % B_STAGES;
-                    if (kc >= B_STAGES && !mbar_wait(c.empty(s, B_STAGES), ((kc / B_STAGES) - 1) & 1, a.status)) {
+                    const int s = kc % B_STAGES_V3;
+                    if (kc >= B_STAGES_V3 && !mbar_wait(empty(s), ((kc / B_STAGES_V3) - 1) & 1, a.status)) {
                         ok = false;
                         break;
                     }
-                    const uint32_t sa = smem_u32(c.base + s * B_STAGE), sb = sa + B_BM * BK * 2, fb = c.full(s);
+                    const uint32_t sa = smem_u32(base + s * B_STAGE), sb = sa + B_BM * BK * 2, fb = full(s);
                     mbar_expect_tx(fb, B_STAGE);
 #pragma unroll
                     for (int bx = 0; bx < B_BM / 64; ++bx) {
@@ -358,117 +419,162 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             bool ok = true;
             for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++local) {
                 const int b = local & 1;
-                if (local >= 2 && !mbar_wait(c.tempty(b, B_STAGES), ((local >> 1) - 1) & 1, a.status)) break;
+                if (local >= 2 && !mbar_wait(tempty(b), ((local >> 1) - 1) & 1, a.status)) break;
                 tc_fence_after();
                 const uint32_t d = tmem + b * 256;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
-                    const int s = kc % B_STAGES;
-                    if (!mbar_wait(c.full(s), (kc / B_STAGES) & 1, a.status)) {
+                    const int s = kc % B_STAGES_V3;
+                    if (!mbar_wait(full(s), (kc / B_STAGES_V3) & 1, a.status)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t sa = smem_u32(c.base + s * B_STAGE), sb = sa + B_BM * BK * 2;
+                    const uint32_t sa = smem_u32(base + s * B_STAGE), sb = sa + B_BM * BK * 2;
 #pragma unroll
                     for (int k = 0; k < BK / 16; ++k)
                         umma_bf16(d, sdesc_sw128(sa + k * 16 * 128, BOX), sdesc_sw128(sb + k * 16 * 128, BOX), idesc,
                                   (kb == 0 && k == 0) ? 0u : 1u);
-                    umma_commit(c.empty(s, B_STAGES));
+                    umma_commit(empty(s));
                 }
-                umma_commit(c.tfull(b, B_STAGES));
+                umma_commit(tfull(b));
+            }
+        }
+        __syncwarp();
+    } else if (warp == 6) {
+        // ---- state producer: W (and mu) chunks of every tile, in epilogue order
+        if (lane == 0) {
+            tma_prefetch_map(&tmW1s);
+            tma_prefetch_map(&tmW2s);
+            if (a.momentum) {
+                tma_prefetch_map(&tmM1s);
+                tma_prefetch_map(&tmM2s);
+            }
+            uint32_t seq = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+                const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
+                const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
+                const bool isW1 = col0 < a.d_in;
+                const int cl = isW1 ? col0 : col0 - a.d_in;
+                for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
+                    const int k = seq % S_SLOTS;
+                    if (seq >= S_SLOTS && !mbar_wait(sempty(k), ((seq / S_SLOTS) - 1) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t dst = smem_u32(base + L::STATE + k * S_SLOT);
+                    mbar_expect_tx(sfull(k), chunk_bytes);
+                    tma_load_3d(dst, isW1 ? &tmW1s : &tmW2s, sfull(k), cl, h0 + g * S_ROWS, cs);
+                    if (a.momentum) tma_load_3d(dst + S_F32, isW1 ? &tmM1s : &tmM2s, sfull(k), cl, h0 + g * S_ROWS, cs);
+                }
             }
         }
         __syncwarp();
     } else {
-        // ---- epilogue warps: TMEM lane quarter q (= 32 weight columns), hidden half hh
-        const int e = warp - 2, q = warp & 3, hh = e >> 2, et = threadIdx.x - 64;
-        float* table = reinterpret_cast<float*>(c.base + LB::TAB);
-        float* bred = table + 2 * B_BN;  // [2][8]
-        int* flag = reinterpret_cast<int*>(c.base + LB::FLAG);
+        // ---- epilogue warps 2..5: TMEM lane quarter q = 32 weight columns
+        const int q = warp & 3, et = threadIdx.x - 64;
+        float* table = reinterpret_cast<float*>(base + L::TAB);
+        float* bred = table + 2 * B_BN;  // [2][4]
+        int* flag = reinterpret_cast<int*>(base + L::FLAG);
         bool finite = true;
+        uint32_t seq = 0;
         int local = 0;
         for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local) {
             const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
             const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
             const bool isW1 = col0 < a.d_in;
             const int which = isW1 ? 0 : 1;
+            const int cl = isW1 ? col0 : col0 - a.d_in;
             const int b = local & 1;
             float* tab = table + b * B_BN;
-            {   // renorm scales of this tile's 256 rows, momentum decay partials
-                const int h = h0 + et;
-                tab[et] = a.renorm_pending
-                              ? renorm_scale((isW1 ? a.n1 : a.n2)[(size_t)cs * a.d_hid + h],
-                                             ss_row(a, a.parity ^ 1, which, cs)[h])
-                              : 1.f;
-                if (a.momentum) {
-                    float v = 0.f;
-                    for (int t = et; t < a.Tp; t += EPI_THREADS) v += a.dbeta[(size_t)cs * a.T + t];
-                    v = warp_sum(v);
-                    if (lane == 0) bred[b * 8 + e] = v;
-                }
+            for (int r = et; r < B_BN; r += B_EPI_THREADS) {
+                const int h = h0 + r;
+                tab[r] = a.renorm_pending ? renorm_scale((isW1 ? a.n1 : a.n2)[(size_t)cs * a.d_hid + h],
+                                                         ss_row(a, a.parity ^ 1, which, cs)[h])
+                                          : 1.f;
             }
-            if (et == 0) flag[b] = mbar_wait(c.tfull(b, B_STAGES), (local >> 1) & 1, a.status) ? 1 : 0;
+            if (a.momentum) {
+                float v = 0.f;
+                for (int t = et; t < a.Tp; t += B_EPI_THREADS) v += a.dbeta[(size_t)cs * a.T + t];
+                v = warp_sum(v);
+                if (lane == 0) bred[b * 4 + (warp - 2)] = v;
+            }
+            if (et == 0) flag[0] = mbar_wait(tfull(b), (local >> 1) & 1, a.status) ? 1 : 0;
             __syncwarp();
-            named_bar_sync(EPI_BAR, EPI_THREADS);
-            if (!flag[b]) break;
+            named_bar_sync(EPI_BAR, B_EPI_THREADS);
+            if (!flag[0]) break;
             tc_fence_after();
             float beta = 0.f;
-            if (a.momentum) {
-                float tot = 0.f;
-#pragma unroll
-                for (int i = 0; i < 8; ++i) tot += bred[b * 8 + i];
-                beta = sigmoidf_(tot / (float)a.Tp + a.b_beta[cs]);
-            }
-            const int width = isW1 ? a.d_in : a.d_out;
-            const int col = (isW1 ? col0 : col0 - a.d_in) + q * 32 + lane;
-            float* W = (isW1 ? a.W1 : a.W2) + (size_t)cs * a.d_hid * width + col;
-            float* M = a.momentum ? (isW1 ? a.mu1 : a.mu2) + (size_t)cs * a.d_hid * width + col : nullptr;
-            bf16* Wb = (isW1 ? a.W1b : a.W2b) + (size_t)cs * a.d_hid * width + col;
+            if (a.momentum)
+                beta = sigmoidf_((bred[b * 4] + bred[b * 4 + 1] + bred[b * 4 + 2] + bred[b * 4 + 3]) / (float)a.Tp +
+                                 a.b_beta[cs]);
             float* cur = ss_row(a, a.parity, which, cs);
+            const int col = q * 32 + lane;  // column within the tile (= TMEM lane)
             const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
+            bool ok = true;
 #pragma unroll 1
-            for (int g = 0; g < 4; ++g) {
-                const int hb = hh * 128 + g * 32;  // first hidden unit of this group, within the tile
+            for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
+                const int k = seq % S_SLOTS;
                 float gv[32];
-                tmem_ld32(lane_base + hb, gv);
-                if (g == 3) {
+                tmem_ld32(lane_base + g * S_ROWS, gv);
+                if (g == B_BN / S_ROWS - 1) {
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(c.tempty(b, B_STAGES));
+                    if (lane == 0) mbar_arrive(tempty(b));
                 }
-                float wv[32], mv[32];
-                float* wp = W + (size_t)(h0 + hb) * width;
-                float* mp = M ? M + (size_t)(h0 + hb) * width : nullptr;
-                bf16* bp = Wb + (size_t)(h0 + hb) * width;
+                if (et == 0) flag[1] = mbar_wait(sfull(k), (seq / S_SLOTS) & 1, a.status) ? 1 : 0;
+                __syncwarp();
+                named_bar_sync(EPI_BAR, B_EPI_THREADS);
+                if (!flag[1]) {
+                    ok = false;
+                    break;
+                }
+                uint8_t* slot = base + L::STATE + k * S_SLOT;
+                float* Ws = reinterpret_cast<float*>(slot);
+                float* Ms = reinterpret_cast<float*>(slot + S_F32);
+                bf16* Bs = reinterpret_cast<bf16*>(slot + 2 * S_F32);
+                float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
-                    wv[j] = wp[j * width];
-                    mv[j] = mp ? mp[j * width] : 0.f;
-                }
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const float mn = fmaf(beta, mv[j], gv[j]);
-                    const float wn = fmaf(tab[hb + j], wv[j], -mn);
-                    wp[j * width] = wn;
-                    if (mp) mp[j * width] = mn;
-                    bp[j * width] = __float2bfloat16_rn(wn);
+                    const float m = a.momentum ? Ms[j * B_BM + col] : 0.f;
+                    const float mn = fmaf(beta, m, gv[j]);
+                    const float wn = fmaf(tab[g * S_ROWS + j], Ws[j * B_BM + col], -mn);
+                    Ws[j * B_BM + col] = wn;
+                    if (a.momentum) Ms[j * B_BM + col] = mn;
+                    Bs[j * B_BM + col] = __float2bfloat16_rn(wn);
                     finite = finite && isfinite(wn);
-                    wv[j] = wn * wn;
+                    v[j] = wn * wn;
                 }
-                // transpose-reduce: afterwards lane j holds the 32-column partial of row hb + j
+                // transpose-reduce: afterwards lane j holds this warp's 32-column partial of row j
 #pragma unroll
                 for (int sft = 16; sft >= 1; sft >>= 1) {
                     const bool upper = (lane & sft) != 0;
 #pragma unroll
-                    for (int k = 0; k < sft; ++k) {
-                        const float send = upper ? wv[k] : wv[k + sft];
-                        const float keep = upper ? wv[k + sft] : wv[k];
-                        wv[k] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+                    for (int i = 0; i < sft; ++i) {
+                        const float send = upper ? v[i] : v[i + sft];
+                        const float keep = upper ? v[i + sft] : v[i];
+                        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
                     }
                 }
-                atomicAdd(&cur[h0 + hb + lane], wv[0]);
+                atomicAdd(&cur[h0 + g * S_ROWS + lane], v[0]);
+                fence_proxy_async_smem();
+                __syncwarp();
+                named_bar_sync(EPI_BAR, B_EPI_THREADS);
+                if (et == 0) {
+                    const int row = h0 + g * S_ROWS;
+                    const uint32_t src = smem_u32(slot);
+                    tma_store_3d(isW1 ? &tmW1s : &tmW2s, src, cl, row, cs);
+                    if (a.momentum) tma_store_3d(isW1 ? &tmM1s : &tmM2s, src + S_F32, cl, row, cs);
+                    tma_store_3d(isW1 ? &tmW1o : &tmW2o, src + 2 * S_F32, cl, row, cs);
+                    bulk_commit();
+                    bulk_wait_read_all();
+                    mbar_arrive(sempty(k));
+                }
+                __syncwarp();
             }
+            if (!ok) break;
         }
+        if (et == 0) bulk_wait_all();
         if (!finite) atomicOr(a.status, DEV_NONFINITE);
     }
     __syncthreads();
@@ -507,7 +613,8 @@ cudaError_t ensure_attrs() {
         if (g_attr_err == cudaSuccess)
             g_attr_err = cudaFuncSetAttribute(tc_phase_a_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LA::DYN);
         if (g_attr_err == cudaSuccess)
-            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LB::DYN);
+            g_attr_err =
+                cudaFuncSetAttribute(tc_phase_b_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LayoutB::DYN);
     });
     return g_attr_err;
 }
@@ -532,7 +639,8 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
     const TcArgs a = make_args(s, w);
     const int ntiles = w.nc * ((s.d_in + s.d_out) / B_BM) * (s.d_hid / B_BN);
     const int grid = ntiles < g_sms ? ntiles : g_sms;
-    tc_phase_b_kernel<<<grid, THREADS, LB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.dH, m.At, a);
+    tc_phase_b_kernel<<<grid, B_THREADS, LayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.dH, m.At,
+                                                              m.W1s, m.W2s, m.M1s, m.M2s, m.W1o, m.W2o, a);
     return cudaGetLastError();
 }
 
@@ -546,10 +654,8 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 EncodeTiledFn g_encode = nullptr;
 std::once_flag g_encode_once;
-}  // namespace
 
-bool encode_map_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t chains,
-                        uint32_t box_inner, uint32_t box_rows) {
+EncodeTiledFn encoder() {
     std::call_once(g_encode_once, [] {
         void* fn = nullptr;
         cudaDriverEntryPointQueryResult q;
@@ -558,13 +664,33 @@ bool encode_map_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint
             q == cudaDriverEntryPointSuccess)
             g_encode = reinterpret_cast<EncodeTiledFn>(fn);
     });
-    if (!g_encode) return false;
+    return g_encode;
+}
+}  // namespace
+
+bool encode_map_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t chains,
+                        uint32_t box_inner, uint32_t box_rows) {
+    if (!encoder() || !map) return false;
     const cuuint64_t dims[3] = {inner, rows, chains};
     const cuuint64_t strides[2] = {inner * 2, inner * rows * 2};
     const cuuint32_t box[3] = {box_inner, box_rows, 1};
     const cuuint32_t estr[3] = {1, 1, 1};
     return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_map_plain_3d(CUtensorMap* map, const void* base, bool f32, uint64_t inner, uint64_t rows,
+                         uint64_t chains, uint32_t box_inner, uint32_t box_rows) {
+    if (!encoder() || !map) return false;
+    const uint64_t es = f32 ? 4 : 2;
+    const cuuint64_t dims[3] = {inner, rows, chains};
+    const cuuint64_t strides[2] = {inner * es, inner * rows * es};
+    const cuuint32_t box[3] = {box_inner, box_rows, 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return g_encode(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                    const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
