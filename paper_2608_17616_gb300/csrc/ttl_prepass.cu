@@ -6,7 +6,6 @@
 // rate eta_j = softplus(w_eta . x_j + b_eta) and the per-token term
 // w_beta . x_j of the momentum decay beta_s = sigmoid(mean_j(w_beta . x_j) + b_beta).
 //
-// One warp per token row, 16-byte vector loads, the row held in registers.
 // Streaming, HBM-bound: reads d_in elements and writes d_in elements per token.
 #include "mone_common.cuh"
 
@@ -80,90 +79,135 @@ __device__ __forceinline__ void load_f32(const float* p, float (&v)[N]) {
     }
 }
 
-// One warp per token row, 16-byte vector loads.  Statistics first; the output
-// pass re-reads the row (an L1/L2 hit: the row was read just before).
+template <int N>
+__device__ __forceinline__ void load_smem(const float* p, float (&v)[N]) {
+#pragma unroll
+    for (int i = 0; i < N; i += 4) {
+        const float4 r = *reinterpret_cast<const float4*>(p + i);
+        v[i] = r.x; v[i + 1] = r.y; v[i + 2] = r.z; v[i + 3] = r.w;
+    }
+}
+
+// Logistic function: fast form for bf16 data (error far below bf16 rounding), the
+// accurate one for the fp32 path.
+template <typename T> __device__ __forceinline__ float sig(float z);
+template <> __device__ __forceinline__ float sig<bf16>(float z) { return sigmoid_fast(z); }
+template <> __device__ __forceinline__ float sig<float>(float z) { return sigmoidf_(z); }
+
+constexpr int PRE_ROWS = 32;  // token rows per CTA (4 per warp)
+
+// One warp per token row, 16-byte vector loads.  The chain's meta-parameters are
+// staged once per CTA in shared memory ([4][d_in]: alpha, gamma, w_eta, w_beta).
+// Statistics first; the output pass re-reads the row (an L1/L2 hit).
 template <typename Tin, typename Tout>
 __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
+    extern __shared__ float4 meta4[];
+    float* meta = reinterpret_cast<float*>(meta4);
     constexpr int V = Vec<Tin>::N;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int t = blockIdx.x * 8 + warp;
     const int cz = blockIdx.y;
     const int cs = a.c0 + cz;
-    if (t >= a.rows) return;
     const int d = a.d_in;
-    Tout* u = reinterpret_cast<Tout*>(a.U) + ((size_t)cs * a.rows + t) * d;
-    const bool present = t < a.Tp && (a.row0 + t) < a.n_rows;
-    if (!present) {
-        float z[V];
-#pragma unroll
-        for (int e = 0; e < V; ++e) z[e] = 0.f;
-        for (int i0 = lane * V; i0 < d; i0 += 32 * V) store_vec<Tout, V>(u + i0, z);
-        if (!a.query && lane == 0) {
-            a.eta[(size_t)cs * a.rows + t] = 0.0f;
-            a.dbeta[(size_t)cs * a.rows + t] = 0.0f;
-        }
-        return;
+    const int nmeta = a.paper ? (a.query ? 2 : 4) : 0;
+    for (int m = 0; m < nmeta; ++m) {
+        const float* src = (m == 0 ? a.alpha : m == 1 ? a.gamma : m == 2 ? a.w_eta : a.w_beta) + (size_t)cs * d;
+        for (int i = threadIdx.x * 4; i < d; i += 256 * 4)
+            *reinterpret_cast<float4*>(meta + m * d + i) = *reinterpret_cast<const float4*>(src + i);
     }
-    const Tin* x = reinterpret_cast<const Tin*>(a.X) + cz * a.x_cstride + (a.row0 + t) * d;
-    float ss = 0.f, de = 0.f, db = 0.f;
-    const float* al = a.paper ? a.alpha + (size_t)cs * d : nullptr;
-    const float* ga = a.paper ? a.gamma + (size_t)cs * d : nullptr;
-    if (a.paper) {
+    __syncthreads();
+    const float* al = meta;
+    const float* ga = meta + d;
+    const float* we = meta + 2 * d;
+    const float* wb = meta + 3 * d;
+    const int t_end = min(a.rows, (int)(blockIdx.x + 1) * PRE_ROWS);
+    for (int t = blockIdx.x * PRE_ROWS + warp; t < t_end; t += 8) {
+        Tout* u = reinterpret_cast<Tout*>(a.U) + ((size_t)cs * a.rows + t) * d;
+        const bool present = t < a.Tp && (a.row0 + t) < a.n_rows;
+        if (!present) {
+            float z[V];
+#pragma unroll
+            for (int e = 0; e < V; ++e) z[e] = 0.f;
+            for (int i0 = lane * V; i0 < d; i0 += 32 * V) store_vec<Tout, V>(u + i0, z);
+            if (!a.query && lane == 0) {
+                a.eta[(size_t)cs * a.rows + t] = 0.0f;
+                a.dbeta[(size_t)cs * a.rows + t] = 0.0f;
+            }
+            continue;
+        }
+        const Tin* x = reinterpret_cast<const Tin*>(a.X) + cz * a.x_cstride + (a.row0 + t) * d;
+        float ss = 0.f, de = 0.f, db = 0.f;
+        if (a.paper) {
 #pragma unroll 4
-        for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
-            float xv[V], av[V], gv[V];
-            Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x + i0), xv);
-            load_f32<V>(al + i0, av);
-            load_f32<V>(ga + i0, gv);
-            if (!a.query) {
-                float we[V], wb[V];
-                load_f32<V>(a.w_eta + (size_t)cs * d + i0, we);
-                load_f32<V>(a.w_beta + (size_t)cs * d + i0, wb);
+            for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
+                float xv[V], av[V], gv[V];
+                Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x + i0), xv);
+                load_smem<V>(al + i0, av);
+                load_smem<V>(ga + i0, gv);
+                if (!a.query) {
+                    float wev[V], wbv[V];
+                    load_smem<V>(we + i0, wev);
+                    load_smem<V>(wb + i0, wbv);
+#pragma unroll
+                    for (int e = 0; e < V; ++e) {
+                        de = fmaf(wev[e], xv[e], de);
+                        db = fmaf(wbv[e], xv[e], db);
+                    }
+                }
 #pragma unroll
                 for (int e = 0; e < V; ++e) {
-                    de = fmaf(we[e], xv[e], de);
-                    db = fmaf(wb[e], xv[e], db);
+                    const float zp = fmaf(av[e], xv[e], gv[e]);
+                    const float z = zp * sig<Tin>(zp);
+                    ss = fmaf(z, z, ss);
                 }
             }
-#pragma unroll
-            for (int e = 0; e < V; ++e) {
-                const float zp = fmaf(av[e], xv[e], gv[e]);
-                const float z = zp * sigmoidf_(zp);
-                ss = fmaf(z, z, ss);
+            ss = warp_sum(ss);
+            if (!a.query) {
+                de = warp_sum(de);
+                db = warp_sum(db);
             }
         }
-        ss = warp_sum(ss);
-        if (!a.query) {
-            de = warp_sum(de);
-            db = warp_sum(db);
-        }
-    }
-    const float inv = a.paper ? 1.0f / sqrtf(ss + 1e-12f) : 1.0f;
+        const float inv = a.paper ? 1.0f / sqrtf(ss + 1e-12f) : 1.0f;
 #pragma unroll 4
-    for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
-        float xv[V];
-        Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x + i0), xv);
-        if (a.paper) {
-            float av[V], gv[V];
-            load_f32<V>(al + i0, av);
-            load_f32<V>(ga + i0, gv);
+        for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
+            float xv[V];
+            Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x + i0), xv);
+            if (a.paper) {
+                float av[V], gv[V];
+                load_smem<V>(al + i0, av);
+                load_smem<V>(ga + i0, gv);
 #pragma unroll
-            for (int e = 0; e < V; ++e) {
-                const float zp = fmaf(av[e], xv[e], gv[e]);
-                xv[e] = zp * sigmoidf_(zp) * inv;
+                for (int e = 0; e < V; ++e) {
+                    const float zp = fmaf(av[e], xv[e], gv[e]);
+                    xv[e] = zp * sig<Tin>(zp) * inv;
+                }
             }
+            store_vec<Tout, V>(u + i0, xv);
         }
-        store_vec<Tout, V>(u + i0, xv);
+        if (!a.query && lane == 0) {
+            float e;
+            if (a.eta_in)
+                e = a.eta_in[cz * a.eta_cstride + a.row0 + t];
+            else
+                e = softplusf_(de + a.b_eta[cs]);
+            a.eta[(size_t)cs * a.rows + t] = e;
+            a.dbeta[(size_t)cs * a.rows + t] = db;
+        }
     }
-    if (!a.query && lane == 0) {
-        float e;
-        if (a.eta_in)
-            e = a.eta_in[cz * a.eta_cstride + a.row0 + t];
-        else
-            e = softplusf_(de + a.b_eta[cs]);
-        a.eta[(size_t)cs * a.rows + t] = e;
-        a.dbeta[(size_t)cs * a.rows + t] = db;
+}
+
+template <typename Tin, typename Tout>
+cudaError_t launch_one(const PrepassArgs& a, int nchains, cudaStream_t st) {
+    const size_t smem = (size_t)(a.paper ? (a.query ? 2 : 4) : 0) * a.d_in * sizeof(float);
+    static bool attr_set = false;  // set once per process: the largest supported d_in needs 64 KB
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(prepass_kernel<Tin, Tout>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             4 * 4096 * (int)sizeof(float));
+        if (e != cudaSuccess) return e;
+        attr_set = true;
     }
+    dim3 grid((a.rows + PRE_ROWS - 1) / PRE_ROWS, nchains);
+    prepass_kernel<Tin, Tout><<<grid, 256, smem, st>>>(a);
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -190,12 +234,7 @@ cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st)
     a.U = s.U;
     a.eta = s.eta;
     a.dbeta = s.dbeta;
-    dim3 grid((s.T + 7) / 8, w.nc);
-    if (s.dtype == 0)
-        prepass_kernel<float, float><<<grid, 256, 0, st>>>(a);
-    else
-        prepass_kernel<bf16, bf16><<<grid, 256, 0, st>>>(a);
-    return cudaGetLastError();
+    return s.dtype == 0 ? launch_one<float, float>(a, w.nc, st) : launch_one<bf16, bf16>(a, w.nc, st);
 }
 
 cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, cudaStream_t st) {
@@ -213,12 +252,7 @@ cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, cud
     a.alpha = s.alpha;
     a.gamma = s.gamma;
     a.U = s.Uq;
-    dim3 grid((Q + 7) / 8, s.C);
-    if (s.dtype == 0)
-        prepass_kernel<float, float><<<grid, 256, 0, st>>>(a);
-    else
-        prepass_kernel<bf16, float><<<grid, 256, 0, st>>>(a);
-    return cudaGetLastError();
+    return s.dtype == 0 ? launch_one<float, float>(a, s.C, st) : launch_one<bf16, float>(a, s.C, st);
 }
 
 }  // namespace mone

@@ -298,13 +298,15 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
 // Warps: 0 operand producer (TMA), 1 MMA issuer, 2..5 epilogue (one per TMEM lane
 // quarter; thread = one weight column), 6 state producer.  The fp32 state of a
 // tile (256 rows x 128 columns of W and mu) moves in chunks of 32 rows through a
-// 3-slot shared-memory ring: the state producer TMA-loads a chunk ahead of time,
-// the epilogue updates it in place and TMA-stores it (with the bf16 copy) back.
+// 4-slot shared-memory ring: the state producer TMA-loads chunks ahead of time,
+// the epilogue updates a chunk in place and TMA-stores it back (the bf16 copy
+// goes out with coalesced 64-byte warp stores); a slot is handed back to the
+// producer once its store has read it, one chunk later.
 
 constexpr int S_ROWS = 32;                                 // hidden rows per state chunk
-constexpr int S_SLOTS = 3;
+constexpr int S_SLOTS = 4;
 constexpr int S_F32 = S_ROWS * B_BM * 4;                   // 16 KB
-constexpr int S_SLOT = 2 * S_F32 + S_ROWS * B_BM * 2;      // W, mu, bf16 copy: 40 KB
+constexpr int S_SLOT = 2 * S_F32;                          // W and mu: 32 KB
 constexpr int B_STAGES_V3 = 2;
 constexpr int B_THREADS = 7 * 32;
 constexpr int B_EPI_THREADS = 4 * 32;
@@ -316,8 +318,8 @@ struct LayoutB {
     static constexpr int NBARS = 2 * B_STAGES_V3 + 4 + 2 * S_SLOTS;
     static constexpr int SLOT = BARS + NBARS * 8;
     static constexpr int FLAG = SLOT + 16;
-    static constexpr int TAB = FLAG + 16;                  // [2][B_BN] scales + [2][4] beta partials
-    static constexpr int END = TAB + (2 * B_BN + 8) * 4;
+    static constexpr int TAB = FLAG + 16;                  // [2][4] momentum-decay partials
+    static constexpr int END = TAB + 8 * 4;
     static constexpr int DYN = END + 1024;
 };
 static_assert(LayoutB::DYN <= 227 * 1024, "phase B shared memory budget");
@@ -473,11 +475,11 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
     } else {
         // ---- epilogue warps 2..5: TMEM lane quarter q = 32 weight columns
         const int q = warp & 3, et = threadIdx.x - 64;
-        float* table = reinterpret_cast<float*>(base + L::TAB);
-        float* bred = table + 2 * B_BN;  // [2][4]
+        float* bred = reinterpret_cast<float*>(base + L::TAB);  // [2][4]
         int* flag = reinterpret_cast<int*>(base + L::FLAG);
         bool finite = true;
         uint32_t seq = 0;
+        int prev_slot = -1;
         int local = 0;
         for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local) {
             const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
@@ -485,14 +487,8 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             const bool isW1 = col0 < a.d_in;
             const int which = isW1 ? 0 : 1;
             const int cl = isW1 ? col0 : col0 - a.d_in;
+            const int width = isW1 ? a.d_in : a.d_out;
             const int b = local & 1;
-            float* tab = table + b * B_BN;
-            for (int r = et; r < B_BN; r += B_EPI_THREADS) {
-                const int h = h0 + r;
-                tab[r] = a.renorm_pending ? renorm_scale((isW1 ? a.n1 : a.n2)[(size_t)cs * a.d_hid + h],
-                                                         ss_row(a, a.parity ^ 1, which, cs)[h])
-                                          : 1.f;
-            }
             if (a.momentum) {
                 float v = 0.f;
                 for (int t = et; t < a.Tp; t += B_EPI_THREADS) v += a.dbeta[(size_t)cs * a.T + t];
@@ -509,12 +505,16 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 beta = sigmoidf_((bred[b * 4] + bred[b * 4 + 1] + bred[b * 4 + 2] + bred[b * 4 + 3]) / (float)a.Tp +
                                  a.b_beta[cs]);
             float* cur = ss_row(a, a.parity, which, cs);
+            const float* prevss = ss_row(a, a.parity ^ 1, which, cs);
+            const float* n0 = (isW1 ? a.n1 : a.n2) + (size_t)cs * a.d_hid;
             const int col = q * 32 + lane;  // column within the tile (= TMEM lane)
+            bf16* Wb = (isW1 ? a.W1b : a.W2b) + (size_t)cs * a.d_hid * width + cl + col;
             const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
             bool ok = true;
 #pragma unroll 1
             for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
                 const int k = seq % S_SLOTS;
+                const int r0 = h0 + g * S_ROWS;
                 float gv[32];
                 tmem_ld32(lane_base + g * S_ROWS, gv);
                 if (g == B_BN / S_ROWS - 1) {
@@ -522,6 +522,8 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                     __syncwarp();
                     if (lane == 0) mbar_arrive(tempty(b));
                 }
+                // pending renormalisation scale of this chunk's rows: lane j computes row r0 + j
+                const float sc_l = a.renorm_pending ? renorm_scale(n0[r0 + lane], prevss[r0 + lane]) : 1.f;
                 if (et == 0) flag[1] = mbar_wait(sfull(k), (seq / S_SLOTS) & 1, a.status) ? 1 : 0;
                 __syncwarp();
                 named_bar_sync(EPI_BAR, B_EPI_THREADS);
@@ -532,16 +534,17 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 uint8_t* slot = base + L::STATE + k * S_SLOT;
                 float* Ws = reinterpret_cast<float*>(slot);
                 float* Ms = reinterpret_cast<float*>(slot + S_F32);
-                bf16* Bs = reinterpret_cast<bf16*>(slot + 2 * S_F32);
+                bf16* bp = Wb + (size_t)r0 * width;
                 float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
+                    const float sc = __shfl_sync(0xffffffffu, sc_l, j);
                     const float m = a.momentum ? Ms[j * B_BM + col] : 0.f;
                     const float mn = fmaf(beta, m, gv[j]);
-                    const float wn = fmaf(tab[g * S_ROWS + j], Ws[j * B_BM + col], -mn);
+                    const float wn = fmaf(sc, Ws[j * B_BM + col], -mn);
                     Ws[j * B_BM + col] = wn;
                     if (a.momentum) Ms[j * B_BM + col] = mn;
-                    Bs[j * B_BM + col] = __float2bfloat16_rn(wn);
+                    bp[j * width] = __float2bfloat16_rn(wn);
                     finite = finite && isfinite(wn);
                     v[j] = wn * wn;
                 }
@@ -556,25 +559,28 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                         v[i] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
                     }
                 }
-                atomicAdd(&cur[h0 + g * S_ROWS + lane], v[0]);
+                atomicAdd(&cur[r0 + lane], v[0]);
                 fence_proxy_async_smem();
                 __syncwarp();
                 named_bar_sync(EPI_BAR, B_EPI_THREADS);
                 if (et == 0) {
-                    const int row = h0 + g * S_ROWS;
                     const uint32_t src = smem_u32(slot);
-                    tma_store_3d(isW1 ? &tmW1s : &tmW2s, src, cl, row, cs);
-                    if (a.momentum) tma_store_3d(isW1 ? &tmM1s : &tmM2s, src + S_F32, cl, row, cs);
-                    tma_store_3d(isW1 ? &tmW1o : &tmW2o, src + 2 * S_F32, cl, row, cs);
+                    tma_store_3d(isW1 ? &tmW1s : &tmW2s, src, cl, r0, cs);
+                    if (a.momentum) tma_store_3d(isW1 ? &tmM1s : &tmM2s, src + S_F32, cl, r0, cs);
                     bulk_commit();
-                    bulk_wait_read_all();
-                    mbar_arrive(sempty(k));
+                    // the previous chunk's stores have read their slot: hand it back
+                    bulk_wait_read_1();
+                    if (prev_slot >= 0) mbar_arrive(sempty(prev_slot));
                 }
+                prev_slot = k;
                 __syncwarp();
             }
             if (!ok) break;
         }
-        if (et == 0) bulk_wait_all();
+        if (et == 0) {
+            bulk_wait_all();
+            if (prev_slot >= 0) mbar_arrive(sempty(prev_slot));
+        }
         if (!finite) atomicOr(a.status, DEV_NONFINITE);
     }
     __syncthreads();
