@@ -79,134 +79,130 @@ __device__ __forceinline__ void load_f32(const float* p, float (&v)[N]) {
     }
 }
 
-template <int N>
-__device__ __forceinline__ void load_smem(const float* p, float (&v)[N]) {
-#pragma unroll
-    for (int i = 0; i < N; i += 4) {
-        const float4 r = *reinterpret_cast<const float4*>(p + i);
-        v[i] = r.x; v[i + 1] = r.y; v[i + 2] = r.z; v[i + 3] = r.w;
-    }
-}
-
 // Logistic function: fast form for bf16 data (error far below bf16 rounding), the
 // accurate one for the fp32 path.
 template <typename T> __device__ __forceinline__ float sig(float z);
 template <> __device__ __forceinline__ float sig<bf16>(float z) { return sigmoid_fast(z); }
 template <> __device__ __forceinline__ float sig<float>(float z) { return sigmoidf_(z); }
 
-constexpr int PRE_ROWS = 32;  // token rows per CTA (4 per warp)
+constexpr int RPW = 4;                 // token rows per warp, processed together
+constexpr int PRE_ROWS = 8 * RPW;      // token rows per CTA
 
-// One warp per token row, 16-byte vector loads.  The chain's meta-parameters are
-// staged once per CTA in shared memory ([4][d_in]: alpha, gamma, w_eta, w_beta).
-// Statistics first; the output pass re-reads the row (an L1/L2 hit).
+// Each warp transforms RPW token rows at once with 16-byte vector loads, so every
+// load of the chain's meta-parameters (alpha, gamma, w_eta, w_beta) serves RPW
+// rows.  Statistics first; the output pass re-reads the rows (L1/L2 hits).
 template <typename Tin, typename Tout>
 __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
-    extern __shared__ float4 meta4[];
-    float* meta = reinterpret_cast<float*>(meta4);
     constexpr int V = Vec<Tin>::N;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int cz = blockIdx.y;
     const int cs = a.c0 + cz;
     const int d = a.d_in;
-    const int nmeta = a.paper ? (a.query ? 2 : 4) : 0;
-    for (int m = 0; m < nmeta; ++m) {
-        const float* src = (m == 0 ? a.alpha : m == 1 ? a.gamma : m == 2 ? a.w_eta : a.w_beta) + (size_t)cs * d;
-        for (int i = threadIdx.x * 4; i < d; i += 256 * 4)
-            *reinterpret_cast<float4*>(meta + m * d + i) = *reinterpret_cast<const float4*>(src + i);
+    const int t0 = blockIdx.x * PRE_ROWS + warp * RPW;
+    const float* al = a.paper ? a.alpha + (size_t)cs * d : nullptr;
+    const float* ga = a.paper ? a.gamma + (size_t)cs * d : nullptr;
+    const float* we = (a.paper && !a.query) ? a.w_eta + (size_t)cs * d : nullptr;
+    const float* wb = (a.paper && !a.query) ? a.w_beta + (size_t)cs * d : nullptr;
+    bool live[RPW];
+    const Tin* x[RPW];
+    Tout* u[RPW];
+#pragma unroll
+    for (int r = 0; r < RPW; ++r) {
+        const int t = t0 + r;
+        live[r] = t < a.rows && t < a.Tp && (a.row0 + t) < a.n_rows;
+        x[r] = reinterpret_cast<const Tin*>(a.X) + cz * a.x_cstride + (a.row0 + (live[r] ? t : 0)) * d;
+        u[r] = reinterpret_cast<Tout*>(a.U) + ((size_t)cs * a.rows + (t < a.rows ? t : 0)) * d;
     }
-    __syncthreads();
-    const float* al = meta;
-    const float* ga = meta + d;
-    const float* we = meta + 2 * d;
-    const float* wb = meta + 3 * d;
-    const int t_end = min(a.rows, (int)(blockIdx.x + 1) * PRE_ROWS);
-    for (int t = blockIdx.x * PRE_ROWS + warp; t < t_end; t += 8) {
-        Tout* u = reinterpret_cast<Tout*>(a.U) + ((size_t)cs * a.rows + t) * d;
-        const bool present = t < a.Tp && (a.row0 + t) < a.n_rows;
-        if (!present) {
-            float z[V];
+    float ss[RPW], de[RPW], db[RPW];
 #pragma unroll
-            for (int e = 0; e < V; ++e) z[e] = 0.f;
-            for (int i0 = lane * V; i0 < d; i0 += 32 * V) store_vec<Tout, V>(u + i0, z);
-            if (!a.query && lane == 0) {
-                a.eta[(size_t)cs * a.rows + t] = 0.0f;
-                a.dbeta[(size_t)cs * a.rows + t] = 0.0f;
+    for (int r = 0; r < RPW; ++r) ss[r] = de[r] = db[r] = 0.f;
+    if (a.paper) {
+#pragma unroll 2
+        for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
+            float av[V], gv[V];
+            load_f32<V>(al + i0, av);
+            load_f32<V>(ga + i0, gv);
+            float wev[V], wbv[V];
+            if (!a.query) {
+                load_f32<V>(we + i0, wev);
+                load_f32<V>(wb + i0, wbv);
             }
-            continue;
-        }
-        const Tin* x = reinterpret_cast<const Tin*>(a.X) + cz * a.x_cstride + (a.row0 + t) * d;
-        float ss = 0.f, de = 0.f, db = 0.f;
-        if (a.paper) {
-#pragma unroll 4
-            for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
-                float xv[V], av[V], gv[V];
-                Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x + i0), xv);
-                load_smem<V>(al + i0, av);
-                load_smem<V>(ga + i0, gv);
-                if (!a.query) {
-                    float wev[V], wbv[V];
-                    load_smem<V>(we + i0, wev);
-                    load_smem<V>(wb + i0, wbv);
 #pragma unroll
-                    for (int e = 0; e < V; ++e) {
-                        de = fmaf(wev[e], xv[e], de);
-                        db = fmaf(wbv[e], xv[e], db);
-                    }
-                }
+            for (int r = 0; r < RPW; ++r) {
+                if (!live[r]) continue;
+                float xv[V];
+                Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x[r] + i0), xv);
 #pragma unroll
                 for (int e = 0; e < V; ++e) {
+                    if (!a.query) {
+                        de[r] = fmaf(wev[e], xv[e], de[r]);
+                        db[r] = fmaf(wbv[e], xv[e], db[r]);
+                    }
                     const float zp = fmaf(av[e], xv[e], gv[e]);
                     const float z = zp * sig<Tin>(zp);
-                    ss = fmaf(z, z, ss);
+                    ss[r] = fmaf(z, z, ss[r]);
                 }
             }
-            ss = warp_sum(ss);
-            if (!a.query) {
-                de = warp_sum(de);
-                db = warp_sum(db);
-            }
         }
-        const float inv = a.paper ? 1.0f / sqrtf(ss + 1e-12f) : 1.0f;
-#pragma unroll 4
-        for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
-            float xv[V];
-            Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x + i0), xv);
-            if (a.paper) {
-                float av[V], gv[V];
-                load_smem<V>(al + i0, av);
-                load_smem<V>(ga + i0, gv);
 #pragma unroll
-                for (int e = 0; e < V; ++e) {
-                    const float zp = fmaf(av[e], xv[e], gv[e]);
-                    xv[e] = zp * sig<Tin>(zp) * inv;
-                }
+        for (int r = 0; r < RPW; ++r) {
+            ss[r] = warp_sum(ss[r]);
+            if (!a.query) {
+                de[r] = warp_sum(de[r]);
+                db[r] = warp_sum(db[r]);
             }
-            store_vec<Tout, V>(u + i0, xv);
         }
-        if (!a.query && lane == 0) {
-            float e;
-            if (a.eta_in)
-                e = a.eta_in[cz * a.eta_cstride + a.row0 + t];
-            else
-                e = softplusf_(de + a.b_eta[cs]);
+    }
+    float inv[RPW];
+#pragma unroll
+    for (int r = 0; r < RPW; ++r) inv[r] = a.paper ? 1.0f / sqrtf(ss[r] + 1e-12f) : 1.0f;
+#pragma unroll 2
+    for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
+        float av[V], gv[V];
+        if (a.paper) {
+            load_f32<V>(al + i0, av);
+            load_f32<V>(ga + i0, gv);
+        }
+#pragma unroll
+        for (int r = 0; r < RPW; ++r) {
+            if (t0 + r >= a.rows) continue;
+            float xv[V];
+            if (live[r]) {
+                Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x[r] + i0), xv);
+                if (a.paper) {
+#pragma unroll
+                    for (int e = 0; e < V; ++e) {
+                        const float zp = fmaf(av[e], xv[e], gv[e]);
+                        xv[e] = zp * sig<Tin>(zp) * inv[r];
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int e = 0; e < V; ++e) xv[e] = 0.f;
+            }
+            store_vec<Tout, V>(u[r] + i0, xv);
+        }
+    }
+    if (!a.query && lane == 0) {
+#pragma unroll
+        for (int r = 0; r < RPW; ++r) {
+            const int t = t0 + r;
+            if (t >= a.rows) continue;
+            float e = 0.f, dbv = 0.f;
+            if (live[r]) {
+                e = a.eta_in ? a.eta_in[cz * a.eta_cstride + a.row0 + t] : softplusf_(de[r] + a.b_eta[cs]);
+                dbv = db[r];
+            }
             a.eta[(size_t)cs * a.rows + t] = e;
-            a.dbeta[(size_t)cs * a.rows + t] = db;
+            a.dbeta[(size_t)cs * a.rows + t] = dbv;
         }
     }
 }
 
 template <typename Tin, typename Tout>
 cudaError_t launch_one(const PrepassArgs& a, int nchains, cudaStream_t st) {
-    const size_t smem = (size_t)(a.paper ? (a.query ? 2 : 4) : 0) * a.d_in * sizeof(float);
-    static bool attr_set = false;  // set once per process: the largest supported d_in needs 64 KB
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(prepass_kernel<Tin, Tout>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             4 * 4096 * (int)sizeof(float));
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
     dim3 grid((a.rows + PRE_ROWS - 1) / PRE_ROWS, nchains);
-    prepass_kernel<Tin, Tout><<<grid, 256, smem, st>>>(a);
+    prepass_kernel<Tin, Tout><<<grid, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 

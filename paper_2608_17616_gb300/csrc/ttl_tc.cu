@@ -318,8 +318,8 @@ struct LayoutB {
     static constexpr int NBARS = 2 * B_STAGES_V3 + 4 + 2 * S_SLOTS;
     static constexpr int SLOT = BARS + NBARS * 8;
     static constexpr int FLAG = SLOT + 16;
-    static constexpr int TAB = FLAG + 16;                  // [2][4] momentum-decay partials
-    static constexpr int END = TAB + 8 * 4;
+    static constexpr int TAB = FLAG + 16;                  // [B_BN] renorm scales + [4] momentum-decay partials
+    static constexpr int END = TAB + (B_BN + 4) * 4;
     static constexpr int DYN = END + 1024;
 };
 static_assert(LayoutB::DYN <= 227 * 1024, "phase B shared memory budget");
@@ -475,7 +475,10 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
     } else {
         // ---- epilogue warps 2..5: TMEM lane quarter q = 32 weight columns
         const int q = warp & 3, et = threadIdx.x - 64;
-        float* bred = reinterpret_cast<float*>(base + L::TAB);  // [2][4]
+        // Single-buffered per-tile tables: a warp writes tile i+1's entries only after
+        // every epilogue warp has passed the last chunk barrier of tile i.
+        float* tab = reinterpret_cast<float*>(base + L::TAB);   // [B_BN]
+        float* bred = tab + B_BN;                                // [4]
         int* flag = reinterpret_cast<int*>(base + L::FLAG);
         bool finite = true;
         uint32_t seq = 0;
@@ -489,11 +492,15 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             const int cl = isW1 ? col0 : col0 - a.d_in;
             const int width = isW1 ? a.d_in : a.d_out;
             const int b = local & 1;
+            const float* n0 = (isW1 ? a.n1 : a.n2) + (size_t)cs * a.d_hid;
+            const float* prevss = ss_row(a, a.parity ^ 1, which, cs);
+            for (int r = et; r < B_BN; r += B_EPI_THREADS)
+                tab[r] = a.renorm_pending ? renorm_scale(n0[h0 + r], prevss[h0 + r]) : 1.f;
             if (a.momentum) {
                 float v = 0.f;
                 for (int t = et; t < a.Tp; t += B_EPI_THREADS) v += a.dbeta[(size_t)cs * a.T + t];
                 v = warp_sum(v);
-                if (lane == 0) bred[b * 4 + (warp - 2)] = v;
+                if (lane == 0) bred[warp - 2] = v;
             }
             if (et == 0) flag[0] = mbar_wait(tfull(b), (local >> 1) & 1, a.status) ? 1 : 0;
             __syncwarp();
@@ -502,11 +509,8 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             tc_fence_after();
             float beta = 0.f;
             if (a.momentum)
-                beta = sigmoidf_((bred[b * 4] + bred[b * 4 + 1] + bred[b * 4 + 2] + bred[b * 4 + 3]) / (float)a.Tp +
-                                 a.b_beta[cs]);
+                beta = sigmoidf_((bred[0] + bred[1] + bred[2] + bred[3]) / (float)a.Tp + a.b_beta[cs]);
             float* cur = ss_row(a, a.parity, which, cs);
-            const float* prevss = ss_row(a, a.parity ^ 1, which, cs);
-            const float* n0 = (isW1 ? a.n1 : a.n2) + (size_t)cs * a.d_hid;
             const int col = q * 32 + lane;  // column within the tile (= TMEM lane)
             bf16* Wb = (isW1 ? a.W1b : a.W2b) + (size_t)cs * a.d_hid * width + cl + col;
             const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
@@ -522,8 +526,6 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                     __syncwarp();
                     if (lane == 0) mbar_arrive(tempty(b));
                 }
-                // pending renormalisation scale of this chunk's rows: lane j computes row r0 + j
-                const float sc_l = a.renorm_pending ? renorm_scale(n0[r0 + lane], prevss[r0 + lane]) : 1.f;
                 if (et == 0) flag[1] = mbar_wait(sfull(k), (seq / S_SLOTS) & 1, a.status) ? 1 : 0;
                 __syncwarp();
                 named_bar_sync(EPI_BAR, B_EPI_THREADS);
@@ -538,7 +540,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
-                    const float sc = __shfl_sync(0xffffffffu, sc_l, j);
+                    const float sc = tab[g * S_ROWS + j];
                     const float m = a.momentum ? Ms[j * B_BM + col] : 0.f;
                     const float mn = fmaf(beta, m, gv[j]);
                     const float wn = fmaf(sc, Ws[j * B_BM + col], -mn);
