@@ -129,7 +129,7 @@ mone_status dalloc(T** p, size_t n) {
 
 void free_state(DevState& s) {
     void* ptrs[] = {s.W1, s.W2, s.mu1, s.mu2, s.W1b, s.W2b, s.n1, s.n2, s.sumsq, s.status, s.alpha, s.gamma,
-                    s.w_eta, s.b_eta, s.w_beta, s.b_beta, s.gate, s.U, s.eta, s.dbeta, s.dHt, s.Att, s.Uq, s.Aq,
+                    s.w_eta, s.b_eta, s.w_beta, s.b_beta, s.gate, s.U, s.eta, s.dbeta, s.zinv, s.dHt, s.Att, s.Uq, s.Aq,
                     s.Oq};
     for (void* p : ptrs)
         if (p) cudaFree(p);
@@ -311,6 +311,7 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
         step(dalloc(reinterpret_cast<uint8_t**>(&s.U), C * s.T * s.d_in * elsize(s.dtype)));
         step(dalloc(&s.eta, C * s.T));
         step(dalloc(&s.dbeta, C * s.T));
+        step(dalloc(&s.zinv, C * s.T));
     }
     if (meta && meta->gate) step(dalloc(&s.gate, C * 2 * s.n_kv));
     const size_t elt = s.dtype == MONE_BF16 ? 2 : 4;

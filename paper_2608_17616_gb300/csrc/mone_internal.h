@@ -29,6 +29,7 @@ struct DevState {
     void* U;                      // [C][T][d_in] transformed inputs (paper mode), dtype of X
     float* eta;                   // [C][T] per-token rates (paper mode)
     float* dbeta;                 // [C][T] w_beta . x_t (paper mode)
+    float* zinv;                  // [C][T] 1 / |z_t| (paper mode, bf16 path: U holds unnormalised z)
     void* dHt;                    // [C][T][d_hid] c_t dH (bf16 or fp32 by path)
     void* Att;                    // [C][T][d_hid] c_t A
     // read scratch (grown on demand)

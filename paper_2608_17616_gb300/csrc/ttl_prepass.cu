@@ -1,4 +1,7 @@
 // Input prepass of a segment (paper mode) and the query transform of the read.
+// On the bf16 path the segment prepass writes the unnormalised z and 1/|z| per
+// token in one pass; phase A applies the scale (H = diag(1/|z|) Z W1^T, and
+// dH^T U = (diag(1/|z|) dH)^T Z), which is exact algebra, not an approximation.
 //
 // Paper mode (App. A): keys and queries go through an affine rescale, SiLU and a
 // per-token L2 normalisation: u_j = z_j / sqrt(|z_j|^2 + 1e-12),
@@ -30,6 +33,7 @@ struct PrepassArgs {
     void* U;              // [C][rows][d_in], type Tout
     float* eta;           // [C][rows]
     float* dbeta;         // [C][rows]
+    float* zinv;          // [C][rows] 1/|z_t|; when set, U receives the unnormalised z (one pass)
 };
 
 // 16-byte vector of inputs: 8 bf16 or 4 fp32 values, kept packed in registers.
@@ -116,6 +120,46 @@ __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
     float ss[RPW], de[RPW], db[RPW];
 #pragma unroll
     for (int r = 0; r < RPW; ++r) ss[r] = de[r] = db[r] = 0.f;
+    if (a.paper && a.zinv) {
+        // one pass: write z = SiLU(alpha x + gamma) unnormalised; the row scale 1/|z|
+        // is applied by the consumer (it commutes with the contraction over d_in)
+#pragma unroll 2
+        for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
+            float av[V], gv[V], wev[V], wbv[V];
+            load_f32<V>(al + i0, av);
+            load_f32<V>(ga + i0, gv);
+            load_f32<V>(we + i0, wev);
+            load_f32<V>(wb + i0, wbv);
+#pragma unroll
+            for (int r = 0; r < RPW; ++r) {
+                if (t0 + r >= a.rows) continue;
+                float xv[V];
+                if (live[r]) {
+                    Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x[r] + i0), xv);
+#pragma unroll
+                    for (int e = 0; e < V; ++e) {
+                        de[r] = fmaf(wev[e], xv[e], de[r]);
+                        db[r] = fmaf(wbv[e], xv[e], db[r]);
+                        const float zp = fmaf(av[e], xv[e], gv[e]);
+                        xv[e] = zp * sig<Tin>(zp);
+                        ss[r] = fmaf(xv[e], xv[e], ss[r]);
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < V; ++e) xv[e] = 0.f;
+                }
+                store_vec<Tout, V>(u[r] + i0, xv);
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < RPW; ++r) {
+            ss[r] = warp_sum(ss[r]);
+            de[r] = warp_sum(de[r]);
+            db[r] = warp_sum(db[r]);
+            const int t = t0 + r;
+            if (lane == 0 && t < a.rows) a.zinv[(size_t)cs * a.rows + t] = live[r] ? 1.0f / sqrtf(ss[r] + 1e-12f) : 0.f;
+        }
+    } else {
     if (a.paper) {
 #pragma unroll 2
         for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
@@ -183,6 +227,7 @@ __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
             store_vec<Tout, V>(u[r] + i0, xv);
         }
     }
+    }
     if (!a.query && lane == 0) {
 #pragma unroll
         for (int r = 0; r < RPW; ++r) {
@@ -230,6 +275,7 @@ cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st)
     a.U = s.U;
     a.eta = s.eta;
     a.dbeta = s.dbeta;
+    a.zinv = s.dtype == 1 ? s.zinv : nullptr;  // bf16 path: unnormalised z + row scale
     return s.dtype == 0 ? launch_one<float, float>(a, w.nc, st) : launch_one<bf16, bf16>(a, w.nc, st);
 }
 

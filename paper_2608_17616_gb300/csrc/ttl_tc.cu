@@ -72,6 +72,7 @@ struct TcArgs {
     long long eta_cstride;
     const float* eta;           // paper-mode rates [C][T]
     const float* dbeta;         // [C][T]
+    const float* zinv;          // [C][T] 1/|z_t| (paper mode), or null
     const float* b_beta;        // [C]
     float *W1, *W2, *mu1, *mu2;
     bf16 *W1b, *W2b;
@@ -237,11 +238,12 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             tc_fence_after();
             const int row = q * 32 + lane;
             const int t = trow + row;
-            float ct = 0.f;
+            float ct = 0.f, zi = 1.f;
             if (t < a.Tp) {
                 const float ev = a.paper ? a.eta[(size_t)cs * a.T + t]
                                          : (a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr);
                 ct = -ev / (float)a.Tp;
+                if (a.zinv) zi = a.zinv[(size_t)cs * a.T + t];
             }
             const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
             bf16* dHrow = a.dH + ((size_t)cs * a.T + t) * a.d_hid + h0;
@@ -264,12 +266,12 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                     float dv[2], av2[2];
 #pragma unroll
                     for (int u = 0; u < 2; ++u) {
-                        const float x = hv[j + u] * tab[c0 + j + u];
+                        const float x = hv[j + u] * tab[c0 + j + u] * zi;
                         const float r = rv[j + u] * tab[A_BN + c0 + j + u];
                         const float sg = sigmoid_fast(x);
                         const float av = x * sg;
                         lsum = fmaf(av, r, lsum);
-                        dv[u] = ct * r * (sg * (1.f + x * (1.f - sg)));
+                        dv[u] = ct * zi * r * (sg * (1.f + x * (1.f - sg)));
                         av2[u] = ct * av;
                     }
                     pd[j / 2] = pack_bf16(dv[0], dv[1]);
@@ -601,6 +603,7 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
     a.eta_in = w.eta_in ? w.eta_in + w.row0 : nullptr;
     a.eta_cstride = w.eta_cstride;
     a.eta = s.eta; a.dbeta = s.dbeta; a.b_beta = s.b_beta;
+    a.zinv = a.paper ? s.zinv : nullptr;
     a.W1 = s.W1; a.W2 = s.W2; a.mu1 = s.mu1; a.mu2 = s.mu2; a.W1b = s.W1b; a.W2b = s.W2b;
     a.n1 = s.n1; a.n2 = s.n2; a.sumsq = s.sumsq;
     a.dH = reinterpret_cast<bf16*>(s.dHt); a.At = reinterpret_cast<bf16*>(s.Att);
