@@ -89,7 +89,7 @@ template <typename T> __device__ __forceinline__ float sig(float z);
 template <> __device__ __forceinline__ float sig<bf16>(float z) { return sigmoid_fast(z); }
 template <> __device__ __forceinline__ float sig<float>(float z) { return sigmoidf_(z); }
 
-constexpr int RPW = 4;                 // token rows per warp, processed together
+constexpr int RPW = 2;                 // token rows per warp, processed together
 constexpr int PRE_ROWS = 8 * RPW;      // token rows per CTA
 
 // Each warp transforms RPW token rows at once with 16-byte vector loads, so every

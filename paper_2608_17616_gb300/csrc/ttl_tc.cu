@@ -297,21 +297,22 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
 
 // ------------------------------------------------------------------ phase B
 //
-// Warps: 0 operand producer (TMA), 1 MMA issuer, 2..5 epilogue (one per TMEM lane
-// quarter; thread = one weight column), 6 state producer.  The fp32 state of a
-// tile (256 rows x 128 columns of W and mu) moves in chunks of 32 rows through a
-// 4-slot shared-memory ring: the state producer TMA-loads chunks ahead of time,
-// the epilogue updates a chunk in place and TMA-stores it back (the bf16 copy
-// goes out with coalesced 64-byte warp stores); a slot is handed back to the
-// producer once its store has read it, one chunk later.
+// Warps: 0 operand producer (TMA), 1 MMA issuer, 2..9 epilogue in two groups of
+// four (one warp per TMEM lane quarter; thread = one weight column), 10 state
+// producer.  The fp32 state of a tile (256 rows x 128 columns of W and mu) moves
+// in chunks of 32 rows through a 4-slot shared-memory ring: the state producer
+// TMA-loads chunks ahead of time; the two epilogue groups take alternate chunks,
+// update a chunk in place and TMA-store it back (the bf16 copy goes out with
+// coalesced 64-byte warp stores), and hand the slot back once the store has read it.
 
 constexpr int S_ROWS = 32;                                 // hidden rows per state chunk
 constexpr int S_SLOTS = 4;
 constexpr int S_F32 = S_ROWS * B_BM * 4;                   // 16 KB
 constexpr int S_SLOT = 2 * S_F32;                          // W and mu: 32 KB
 constexpr int B_STAGES_V3 = 2;
-constexpr int B_THREADS = 7 * 32;
-constexpr int B_EPI_THREADS = 4 * 32;
+constexpr int B_THREADS = 11 * 32;
+constexpr int B_EPI_THREADS = 4 * 32;     // per epilogue group
+constexpr int B_STATE_WARP = 10;
 
 struct LayoutB {
     static constexpr int RING = B_STAGES_V3 * B_STAGE;
@@ -320,8 +321,8 @@ struct LayoutB {
     static constexpr int NBARS = 2 * B_STAGES_V3 + 4 + 2 * S_SLOTS;
     static constexpr int SLOT = BARS + NBARS * 8;
     static constexpr int FLAG = SLOT + 16;
-    static constexpr int TAB = FLAG + 16;                  // [B_BN] renorm scales + [4] momentum-decay partials
-    static constexpr int END = TAB + (B_BN + 4) * 4;
+    static constexpr int TAB = FLAG + 16;                  // per group: [B_BN/2] renorm scales + [4] decay partials
+    static constexpr int END = TAB + 2 * (B_BN / 2 + 4) * 4;
     static constexpr int DYN = END + 1024;
 };
 static_assert(LayoutB::DYN <= 227 * 1024, "phase B shared memory budget");
@@ -351,7 +352,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull(b), 1);
-            mbar_init(tempty(b), 4);
+            mbar_init(tempty(b), 8);
         }
         for (int k = 0; k < S_SLOTS; ++k) {
             mbar_init(sfull(k), 1);
@@ -444,7 +445,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             }
         }
         __syncwarp();
-    } else if (warp == 6) {
+    } else if (warp == B_STATE_WARP) {
         // ---- state producer: W (and mu) chunks of every tile, in epilogue order
         if (lane == 0) {
             tma_prefetch_map(&tmW1s);
@@ -475,18 +476,19 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
         }
         __syncwarp();
     } else {
-        // ---- epilogue warps 2..5: TMEM lane quarter q = 32 weight columns
-        const int q = warp & 3, et = threadIdx.x - 64;
+        // ---- epilogue warps 2..9: group grp takes the tile's chunks grp, grp+2, grp+4, grp+6;
+        //      within a group, TMEM lane quarter q = 32 weight columns
+        const int grp = (warp - 2) >> 2, q = warp & 3, et = threadIdx.x - 64 - grp * B_EPI_THREADS;
+        const uint32_t bar_id = 1 + grp;
         // Single-buffered per-tile tables: a warp writes tile i+1's entries only after
-        // every epilogue warp has passed the last chunk barrier of tile i.
-        float* tab = reinterpret_cast<float*>(base + L::TAB);   // [B_BN]
-        float* bred = tab + B_BN;                                // [4]
-        int* flag = reinterpret_cast<int*>(base + L::FLAG);
+        // every warp of its group has passed the last chunk barrier of tile i.
+        float* tab = reinterpret_cast<float*>(base + L::TAB) + grp * (B_BN / 2 + 4);  // [B_BN/2]
+        float* bred = tab + B_BN / 2;                                                  // [4]
+        int* flag = reinterpret_cast<int*>(base + L::FLAG) + grp * 2;
         bool finite = true;
-        uint32_t seq = 0;
-        int prev_slot = -1;
+        uint32_t tile_seq0 = 0;  // chunk sequence number of the current tile's first chunk
         int local = 0;
-        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local) {
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local, tile_seq0 += B_BN / S_ROWS) {
             const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
             const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
             const bool isW1 = col0 < a.d_in;
@@ -496,41 +498,45 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             const int b = local & 1;
             const float* n0 = (isW1 ? a.n1 : a.n2) + (size_t)cs * a.d_hid;
             const float* prevss = ss_row(a, a.parity ^ 1, which, cs);
-            for (int r = et; r < B_BN; r += B_EPI_THREADS)
-                tab[r] = a.renorm_pending ? renorm_scale(n0[h0 + r], prevss[h0 + r]) : 1.f;
+            {   // scales of this group's 4 chunks x 32 rows
+                const int i = et >> 5, j = et & 31;
+                const int row = h0 + (2 * i + grp) * S_ROWS + j;
+                tab[et] = a.renorm_pending ? renorm_scale(n0[row], prevss[row]) : 1.f;
+            }
             if (a.momentum) {
                 float v = 0.f;
                 for (int t = et; t < a.Tp; t += B_EPI_THREADS) v += a.dbeta[(size_t)cs * a.T + t];
                 v = warp_sum(v);
-                if (lane == 0) bred[warp - 2] = v;
+                if (lane == 0) bred[q] = v;
             }
             if (et == 0) flag[0] = mbar_wait(tfull(b), (local >> 1) & 1, a.status) ? 1 : 0;
             __syncwarp();
-            named_bar_sync(EPI_BAR, B_EPI_THREADS);
+            named_bar_sync(bar_id, B_EPI_THREADS);
             if (!flag[0]) break;
             tc_fence_after();
             float beta = 0.f;
-            if (a.momentum)
-                beta = sigmoidf_((bred[0] + bred[1] + bred[2] + bred[3]) / (float)a.Tp + a.b_beta[cs]);
+            if (a.momentum) beta = sigmoidf_((bred[0] + bred[1] + bred[2] + bred[3]) / (float)a.Tp + a.b_beta[cs]);
             float* cur = ss_row(a, a.parity, which, cs);
             const int col = q * 32 + lane;  // column within the tile (= TMEM lane)
             bf16* Wb = (isW1 ? a.W1b : a.W2b) + (size_t)cs * a.d_hid * width + cl + col;
             const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
             bool ok = true;
 #pragma unroll 1
-            for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
+            for (int i = 0; i < B_BN / S_ROWS / 2; ++i) {
+                const int c = 2 * i + grp;
+                const uint32_t seq = tile_seq0 + c;
                 const int k = seq % S_SLOTS;
-                const int r0 = h0 + g * S_ROWS;
+                const int r0 = h0 + c * S_ROWS;
                 float gv[32];
-                tmem_ld32(lane_base + g * S_ROWS, gv);
-                if (g == B_BN / S_ROWS - 1) {
+                tmem_ld32(lane_base + c * S_ROWS, gv);
+                if (i == B_BN / S_ROWS / 2 - 1) {
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(tempty(b));
                 }
                 if (et == 0) flag[1] = mbar_wait(sfull(k), (seq / S_SLOTS) & 1, a.status) ? 1 : 0;
                 __syncwarp();
-                named_bar_sync(EPI_BAR, B_EPI_THREADS);
+                named_bar_sync(bar_id, B_EPI_THREADS);
                 if (!flag[1]) {
                     ok = false;
                     break;
@@ -542,7 +548,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
-                    const float sc = tab[g * S_ROWS + j];
+                    const float sc = tab[i * S_ROWS + j];
                     const float m = a.momentum ? Ms[j * B_BM + col] : 0.f;
                     const float mn = fmaf(beta, m, gv[j]);
                     const float wn = fmaf(sc, Ws[j * B_BM + col], -mn);
@@ -557,34 +563,29 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 for (int sft = 16; sft >= 1; sft >>= 1) {
                     const bool upper = (lane & sft) != 0;
 #pragma unroll
-                    for (int i = 0; i < sft; ++i) {
-                        const float send = upper ? v[i] : v[i + sft];
-                        const float keep = upper ? v[i + sft] : v[i];
-                        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+                    for (int u = 0; u < sft; ++u) {
+                        const float send = upper ? v[u] : v[u + sft];
+                        const float keep = upper ? v[u + sft] : v[u];
+                        v[u] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
                     }
                 }
                 atomicAdd(&cur[r0 + lane], v[0]);
                 fence_proxy_async_smem();
                 __syncwarp();
-                named_bar_sync(EPI_BAR, B_EPI_THREADS);
+                named_bar_sync(bar_id, B_EPI_THREADS);
                 if (et == 0) {
                     const uint32_t src = smem_u32(slot);
                     tma_store_3d(isW1 ? &tmW1s : &tmW2s, src, cl, r0, cs);
                     if (a.momentum) tma_store_3d(isW1 ? &tmM1s : &tmM2s, src + S_F32, cl, r0, cs);
                     bulk_commit();
-                    // the previous chunk's stores have read their slot: hand it back
-                    bulk_wait_read_1();
-                    if (prev_slot >= 0) mbar_arrive(sempty(prev_slot));
+                    bulk_wait_read_all();  // the store has read the slot: hand it back
+                    mbar_arrive(sempty(k));
                 }
-                prev_slot = k;
                 __syncwarp();
             }
             if (!ok) break;
         }
-        if (et == 0) {
-            bulk_wait_all();
-            if (prev_slot >= 0) mbar_arrive(sempty(prev_slot));
-        }
+        if (et == 0) bulk_wait_all();
         if (!finite) atomicOr(a.status, DEV_NONFINITE);
     }
     __syncthreads();
