@@ -157,8 +157,8 @@ mone_status build_state_maps(mone_mem* m) {
               encode_map_bf16_3d(&m->maps.dH, s.dHt, s.d_hid, s.T, s.C, 64, 64) &&
               encode_map_bf16_3d(&m->maps.At, s.Att, s.d_hid, s.T, s.C, 64, 64);
     if (ok && s.U)
-        ok = encode_map_bf16_3d(&m->maps.Ua, s.U, s.d_in, s.T, s.C, 64, 128) &&
-             encode_map_bf16_3d(&m->maps.Ub, s.U, s.d_in, s.T, s.C, 64, 64);
+        ok = encode_map_bf16_3d(&m->maps.Ua, s.U, s.d_in, s.win_rows, s.C, 64, 128) &&
+             encode_map_bf16_3d(&m->maps.Ub, s.U, s.d_in, s.win_rows, s.C, 64, 64);
     if (ok)
         ok = encode_map_plain_3d(&m->maps.W1s, s.W1, true, s.d_in, s.d_hid, s.C, 128, 32) &&
              encode_map_plain_3d(&m->maps.W2s, s.W2, true, s.d_out, s.d_hid, s.C, 128, 32) &&
@@ -215,12 +215,24 @@ mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
     std::memset(&in, 0, sizeof(in));
     if (s.dtype == MONE_BF16) MONE_TRY(build_input_maps(s, &in, w.X, w.K, w.V, w.n_rows, w.nc));
     const long long S = (N + s.T - 1) / s.T;
+    long long win0 = -1;  // first token of the current paper-mode input window
     for (long long i = 0; i < S; ++i) {
         w.row0 = i * s.T;
         w.Tp = (int)std::min<long long>(s.T, N - w.row0);
         w.parity = (int)(i & 1);
         w.renorm_pending = (s.renorm && i > 0) ? 1 : 0;
-        if (s.mode == MONE_PAPER) MONE_TRY(timed(m, K_PREPASS, st, 1, [&] { return launch_prepass(s, w, st); }));
+        if (s.mode == MONE_PAPER) {
+            if (win0 < 0 || w.row0 >= win0 + s.win_rows) {
+                // input transform of the next window of segments: depends on the inputs only
+                win0 = w.row0;
+                SegWork pw = w;
+                pw.Tp = (int)std::min<long long>(s.win_rows, N - win0);
+                MONE_TRY(timed(m, K_PREPASS, st, 1, [&] { return launch_prepass(s, pw, st); }));
+            }
+            w.u_off = w.row0 - win0;
+        } else {
+            w.u_off = 0;
+        }
         if (s.dtype == MONE_BF16) {
             MONE_TRY(timed(m, K_PHASE_A, st, 1, [&] { return launch_phase_a_tc(s, m->maps, in, w, st); }));
             MONE_TRY(timed(m, K_PHASE_B, st, 1, [&] { return launch_phase_b_tc(s, m->maps, in, w, st); }));
@@ -284,6 +296,13 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
     s.dtype = cfg->dtype; s.mode = cfg->mode;
     s.momentum = cfg->mode == MONE_PAPER; s.renorm = cfg->mode == MONE_PAPER;
     s.lr = cfg->lr; s.rms_eps = cfg->rms_eps;
+    if (s.mode == MONE_PAPER) {
+        // the input transform covers a window of whole segments whose scratch stays within ~2 GiB
+        const size_t row_bytes = (size_t)s.C * s.d_in * elsize(s.dtype);
+        long long segs = (long long)((size_t(2) << 30) / (row_bytes * (size_t)s.T));
+        segs = std::max(1ll, std::min(64ll, segs));
+        s.win_rows = (int)(segs * s.T);
+    }
     const size_t C = s.C, n1 = C * s.d_hid * s.d_in, n2 = C * s.d_hid * s.d_out;
     mone_status rc = MONE_OK;
     auto step = [&](mone_status r) { if (rc == MONE_OK) rc = r; };
@@ -308,10 +327,10 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
         step(dalloc(&s.w_beta, C * s.d_in));
         step(dalloc(&s.b_eta, C));
         step(dalloc(&s.b_beta, C));
-        step(dalloc(reinterpret_cast<uint8_t**>(&s.U), C * s.T * s.d_in * elsize(s.dtype)));
-        step(dalloc(&s.eta, C * s.T));
-        step(dalloc(&s.dbeta, C * s.T));
-        step(dalloc(&s.zinv, C * s.T));
+        step(dalloc(reinterpret_cast<uint8_t**>(&s.U), C * s.win_rows * s.d_in * elsize(s.dtype)));
+        step(dalloc(&s.eta, C * s.win_rows));
+        step(dalloc(&s.dbeta, C * s.win_rows));
+        step(dalloc(&s.zinv, C * s.win_rows));
     }
     if (meta && meta->gate) step(dalloc(&s.gate, C * 2 * s.n_kv));
     const size_t elt = s.dtype == MONE_BF16 ? 2 : 4;

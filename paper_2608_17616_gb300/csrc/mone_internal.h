@@ -25,11 +25,12 @@ struct DevState {
     int* status;                  // device status word
     // meta-parameters (owned copies)
     float *alpha, *gamma, *w_eta, *b_eta, *w_beta, *b_beta, *gate;
-    // per-segment scratch
-    void* U;                      // [C][T][d_in] transformed inputs (paper mode), dtype of X
-    float* eta;                   // [C][T] per-token rates (paper mode)
-    float* dbeta;                 // [C][T] w_beta . x_t (paper mode)
-    float* zinv;                  // [C][T] 1 / |z_t| (paper mode, bf16 path: U holds unnormalised z)
+    // paper-mode input scratch for a window of win_rows tokens (a multiple of T)
+    int win_rows;
+    void* U;                      // [C][win_rows][d_in] transformed inputs, dtype of X
+    float* eta;                   // [C][win_rows] per-token rates
+    float* dbeta;                 // [C][win_rows] w_beta . x_t
+    float* zinv;                  // [C][win_rows] 1 / |z_t| (bf16 path: U holds unnormalised z)
     void* dHt;                    // [C][T][d_hid] c_t dH (bf16 or fp32 by path)
     void* Att;                    // [C][T][d_hid] c_t A
     // read scratch (grown on demand)
@@ -48,6 +49,7 @@ struct SegWork {
     long long x_cstride, y_cstride;  // element stride between chains in X and in K/V
     long long n_rows;            // rows per chain in the caller's buffers
     long long row0;              // first token row of this segment
+    long long u_off;             // row of the segment in the paper-mode input scratch window
     int Tp;                      // tokens present in this segment (<= T)
     const float* eta_in;         // caller per-token rates or null
     long long eta_cstride;

@@ -10,6 +10,8 @@
 // w_beta . x_j of the momentum decay beta_s = sigmoid(mean_j(w_beta . x_j) + b_beta).
 //
 // Streaming, HBM-bound: reads d_in elements and writes d_in elements per token.
+#include <algorithm>
+
 #include "mone_common.cuh"
 
 namespace mone {
@@ -22,7 +24,8 @@ struct PrepassArgs {
     long long row0;       // first row of the segment in X
     long long n_rows;     // rows per chain in X (beyond: out of range)
     int Tp;               // tokens present
-    int rows;             // rows to produce (segment size T, or Q for queries)
+    int rows;             // rows to produce (a window of tokens, or Q for queries)
+    int row_stride;       // rows per chain in the output buffers
     int c0;               // state chain offset
     int d_in;
     int paper;            // transform on/off
@@ -115,7 +118,7 @@ __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
         const int t = t0 + r;
         live[r] = t < a.rows && t < a.Tp && (a.row0 + t) < a.n_rows;
         x[r] = reinterpret_cast<const Tin*>(a.X) + cz * a.x_cstride + (a.row0 + (live[r] ? t : 0)) * d;
-        u[r] = reinterpret_cast<Tout*>(a.U) + ((size_t)cs * a.rows + (t < a.rows ? t : 0)) * d;
+        u[r] = reinterpret_cast<Tout*>(a.U) + ((size_t)cs * a.row_stride + (t < a.rows ? t : 0)) * d;
     }
     float ss[RPW], de[RPW], db[RPW];
 #pragma unroll
@@ -157,7 +160,8 @@ __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
             de[r] = warp_sum(de[r]);
             db[r] = warp_sum(db[r]);
             const int t = t0 + r;
-            if (lane == 0 && t < a.rows) a.zinv[(size_t)cs * a.rows + t] = live[r] ? 1.0f / sqrtf(ss[r] + 1e-12f) : 0.f;
+            if (lane == 0 && t < a.rows)
+                a.zinv[(size_t)cs * a.row_stride + t] = live[r] ? 1.0f / sqrtf(ss[r] + 1e-12f) : 0.f;
         }
     } else {
     if (a.paper) {
@@ -238,8 +242,8 @@ __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
                 e = a.eta_in ? a.eta_in[cz * a.eta_cstride + a.row0 + t] : softplusf_(de[r] + a.b_eta[cs]);
                 dbv = db[r];
             }
-            a.eta[(size_t)cs * a.rows + t] = e;
-            a.dbeta[(size_t)cs * a.rows + t] = dbv;
+            a.eta[(size_t)cs * a.row_stride + t] = e;
+            a.dbeta[(size_t)cs * a.row_stride + t] = dbv;
         }
     }
 }
@@ -259,8 +263,10 @@ cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st)
     a.x_cstride = w.x_cstride;
     a.row0 = w.row0;
     a.n_rows = w.n_rows;
-    a.Tp = w.Tp;
-    a.rows = s.T;
+    a.Tp = w.Tp;  // tokens present in the window
+    // write whole segments: rows past the context end are zero, never stale scratch
+    a.rows = (int)std::min<long long>(s.win_rows, ((long long)w.Tp + s.T - 1) / s.T * s.T);
+    a.row_stride = s.win_rows;
     a.c0 = w.c0;
     a.d_in = s.d_in;
     a.paper = 1;
@@ -287,6 +293,7 @@ cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, cud
     a.n_rows = Q;
     a.Tp = Q;
     a.rows = Q;
+    a.row_stride = Q;
     a.c0 = 0;
     a.d_in = s.d_in;
     a.paper = s.mode == 1;

@@ -55,6 +55,8 @@ __device__ __forceinline__ void simt_tile(float (&acc)[4][4], const float* A, lo
 
 struct F32SegArgs {
     int d_in, d_hid, d_out, T, Tp, c0, paper, momentum, renorm_pending, parity, C;
+    long long tok0;           // per-token tables: entry of token t of chain cs is [cs * win + tok0 + t]
+    int win;
     float lr;
     const float *U;           // base of the memory input rows of this segment for chain cz (see below)
     long long u_cstride;      // element stride between chains of U
@@ -119,7 +121,7 @@ __global__ void __launch_bounds__(256) phase_a_f32_kernel(const F32SegArgs a) {
         if (t < a.Tp && t - t0 < m_valid) {
             float e;
             if (a.paper)
-                e = a.eta[(size_t)cs * a.T + t];
+                e = a.eta[(size_t)cs * a.win + a.tok0 + t];
             else
                 e = a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr;
             ct = -e / (float)a.Tp;
@@ -171,7 +173,7 @@ __global__ void __launch_bounds__(256) phase_b_f32_kernel(const F32SegArgs a) {
     // momentum decay beta_s = sigmoid(mean_t w_beta . x_t + b_beta)
     if (a.momentum) {
         float v = 0.f;
-        for (int t = tid; t < a.Tp; t += 256) v += a.dbeta[(size_t)cs * a.T + t];
+        for (int t = tid; t < a.Tp; t += 256) v += a.dbeta[(size_t)cs * a.win + a.tok0 + t];
         v = warp_sum(v);
         if ((tid & 31) == 0) red[tid >> 5] = v;
         __syncthreads();
@@ -222,11 +224,12 @@ F32SegArgs make_f32_args(const DevState& s, const SegWork& w) {
     F32SegArgs a{};
     a.d_in = s.d_in; a.d_hid = s.d_hid; a.d_out = s.d_out; a.T = s.T; a.Tp = w.Tp; a.c0 = w.c0;
     a.paper = s.mode == 1; a.momentum = s.momentum; a.renorm_pending = w.renorm_pending;
+    a.tok0 = w.u_off; a.win = s.win_rows;
     a.parity = w.parity; a.C = s.C; a.lr = s.lr;
     const int dh = s.d_out / 2;
     if (a.paper) {
-        a.U = reinterpret_cast<const float*>(s.U) + (size_t)w.c0 * s.T * s.d_in;
-        a.u_cstride = (long long)s.T * s.d_in;
+        a.U = reinterpret_cast<const float*>(s.U) + ((size_t)w.c0 * s.win_rows + w.u_off) * s.d_in;
+        a.u_cstride = (long long)s.win_rows * s.d_in;
     } else {
         a.U = reinterpret_cast<const float*>(w.X) + w.row0 * s.d_in;
         a.u_cstride = w.x_cstride;

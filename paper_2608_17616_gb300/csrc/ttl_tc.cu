@@ -67,6 +67,8 @@ static_assert(LA::DYN <= 227 * 1024, "shared memory budget");
 struct TcArgs {
     int d_in, d_out, d_hid, T, Tp, c0, nc, C, paper, momentum, renorm_pending, parity;
     int u_row0, u_chain0, y_row0;
+    long long tok0;             // per-token tables: entry of token t of chain cs is [cs * win + tok0 + t]
+    int win;
     float lr;
     const float* eta_in;        // plain-mode caller rates, offset to the segment start, or null
     long long eta_cstride;
@@ -240,10 +242,10 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             const int t = trow + row;
             float ct = 0.f, zi = 1.f;
             if (t < a.Tp) {
-                const float ev = a.paper ? a.eta[(size_t)cs * a.T + t]
+                const float ev = a.paper ? a.eta[(size_t)cs * a.win + a.tok0 + t]
                                          : (a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr);
                 ct = -ev / (float)a.Tp;
-                if (a.zinv) zi = a.zinv[(size_t)cs * a.T + t];
+                if (a.zinv) zi = a.zinv[(size_t)cs * a.win + a.tok0 + t];
             }
             const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
             bf16* dHrow = a.dH + ((size_t)cs * a.T + t) * a.d_hid + h0;
@@ -505,7 +507,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             }
             if (a.momentum) {
                 float v = 0.f;
-                for (int t = et; t < a.Tp; t += B_EPI_THREADS) v += a.dbeta[(size_t)cs * a.T + t];
+                for (int t = et; t < a.Tp; t += B_EPI_THREADS) v += a.dbeta[(size_t)cs * a.win + a.tok0 + t];
                 v = warp_sum(v);
                 if (lane == 0) bred[q] = v;
             }
@@ -597,7 +599,9 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
     a.d_in = s.d_in; a.d_out = s.d_out; a.d_hid = s.d_hid; a.T = s.T; a.Tp = w.Tp; a.c0 = w.c0; a.nc = w.nc;
     a.C = s.C;
     a.paper = s.mode == 1; a.momentum = s.momentum; a.renorm_pending = w.renorm_pending; a.parity = w.parity;
-    a.u_row0 = a.paper ? 0 : (int)w.row0;
+    a.u_row0 = a.paper ? (int)w.u_off : (int)w.row0;
+    a.tok0 = w.u_off;
+    a.win = s.win_rows;
     a.u_chain0 = a.paper ? w.c0 : 0;
     a.y_row0 = (int)w.row0;
     a.lr = s.lr;
