@@ -154,10 +154,6 @@ mone_status build_state_maps(mone_mem* m) {
     if (s.dtype != MONE_BF16) return MONE_OK;
     bool ok = encode_map_bf16_3d(&m->maps.W1b, s.W1b, s.d_in, s.d_hid, s.C, 64, 128) &&
               encode_map_bf16_3d(&m->maps.W2b, s.W2b, s.d_out, s.d_hid, s.C, 64, 128) &&
-              encode_map_bf16_3d(&m->maps.W1m2, s.W1b, s.d_in, s.d_hid, s.C, 64, 64) &&
-              encode_map_bf16_3d(&m->maps.W2m2, s.W2b, s.d_out, s.d_hid, s.C, 64, 64) &&
-              encode_map_bf16_3d(&m->maps.W1m4, s.W1b, s.d_in, s.d_hid, s.C, 64, 32) &&
-              encode_map_bf16_3d(&m->maps.W2m4, s.W2b, s.d_out, s.d_hid, s.C, 64, 32) &&
               encode_map_bf16_3d(&m->maps.dH, s.dHt, s.d_hid, s.T, s.C, 64, 64) &&
               encode_map_bf16_3d(&m->maps.At, s.Att, s.d_hid, s.T, s.C, 64, 64);
     if (ok && s.U)

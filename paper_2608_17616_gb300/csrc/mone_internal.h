@@ -74,8 +74,6 @@ cudaError_t launch_zero_f32(float* p, size_t n, cudaStream_t st);
 // ---- kernels in ttl_tc.cu (bf16 tcgen05 path)
 struct TcMaps {
     CUtensorMap W1b, W2b;        // K-major boxes {64, 128}
-    CUtensorMap W1m2, W2m2;      // K-major slices {64, 64} (phase A clusters of 2)
-    CUtensorMap W1m4, W2m4;      // K-major slices {64, 32} (phase A clusters of 4)
     CUtensorMap dH, At;          // MN-major boxes {64, 64} over [C][T][d_hid]
     CUtensorMap Ua, Ub;          // scratch U: K-major {64,128} and MN {64,64}
     CUtensorMap W1s, W2s, M1s, M2s;  // fp32 state chunks {128 cols, 32 rows}, no swizzle

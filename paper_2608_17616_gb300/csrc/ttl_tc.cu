@@ -67,7 +67,6 @@ static_assert(LA::DYN <= 227 * 1024, "shared memory budget");
 struct TcArgs {
     int d_in, d_out, d_hid, T, Tp, c0, nc, C, paper, momentum, renorm_pending, parity;
     int u_row0, u_chain0, y_row0;
-    int cl;                     // phase A cluster size (token tiles sharing one multicast W tile)
     long long tok0;             // per-token tables: entry of token t of chain cs is [cs * win + tok0 + t]
     int win;
     float lr;
@@ -100,14 +99,14 @@ struct Ctl {
 };
 
 template <class L, int STAGES>
-__device__ __forceinline__ Ctl setup(uint8_t* raw, uint32_t empty_count = 1) {
+__device__ __forceinline__ Ctl setup(uint8_t* raw) {
     Ctl c;
     c.base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
     c.bars = smem_u32(c.base + L::BARS);
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
             mbar_init(c.full(i), 1);
-            mbar_init(c.empty(i, STAGES), empty_count);
+            mbar_init(c.empty(i, STAGES), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(c.tfull(b, STAGES), 1);
@@ -137,20 +136,12 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmW1,
                   const __grid_constant__ CUtensorMap tmW2, const TcArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    // A cluster of a.cl CTAs takes a.cl consecutive token tiles of one (chain, hidden tile):
-    // they share the W tile, which each CTA loads one 128/cl-row slice of and multicasts.
-    const int CL = a.cl;
-    const Ctl c = setup<LA, A_STAGES>(smem_raw, (uint32_t)CL);
-    if (CL > 1) cluster_sync();  // peers' barriers are initialised before any multicast
+    const Ctl c = setup<LA, A_STAGES>(smem_raw);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + LA::SLOT);
-    const int rank = CL > 1 ? (int)cluster_ctarank() : 0;
-    const int cluster = blockIdx.x / CL, nclusters = gridDim.x / CL;
-    const uint16_t mask = (uint16_t)((1u << CL) - 1u);
-    const int n_tt = a.T / A_BM, n_ht = a.d_hid / A_BN, n_tg = n_tt / CL;
-    const int nct = a.nc * n_ht * n_tg;  // cluster tiles
+    const int n_tt = a.T / A_BM, n_ht = a.d_hid / A_BN;
+    const int ntiles = a.nc * n_ht * n_tt;
     const int KB1 = a.d_in / BK, KB = KB1 + a.d_out / BK, half = (a.d_out / 2) / BK;
-    const int wrows = A_BN / CL;         // rows of the W slice this CTA fetches
 
     if (warp == 0) {
         if (lane == 0) {
@@ -161,8 +152,8 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             tma_prefetch_map(&tmW2);
             uint32_t kc = 0;
             bool ok = true;
-            for (int ct = cluster; ct < nct && ok; ct += nclusters) {
-                const int cz = ct / (n_ht * n_tg), ht = (ct / n_tg) % n_ht, tt = (ct % n_tg) * CL + rank;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+                const int cz = tile / (n_ht * n_tt), ht = (tile / n_tt) % n_ht, tt = tile % n_tt;
                 const int cs = a.c0 + cz, h0 = ht * A_BN, trow = tt * A_BM;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
                     const int s = kc % A_STAGES;
@@ -172,30 +163,19 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                     }
                     const uint32_t sa = smem_u32(c.base + s * A_STAGE), sb = sa + A_BM * BK * 2, fb = c.full(s);
                     mbar_expect_tx(fb, A_STAGE);
-                    const CUtensorMap* wm = kb < KB1 ? &tmW1 : &tmW2;
-                    const int wk = kb < KB1 ? kb * BK : (kb - KB1) * BK;
                     if (kb < KB1) {
                         tma_load_3d(sa, &tmU, fb, kb * BK, a.u_row0 + trow, a.u_chain0 + cz);
+                        tma_load_3d(sb, &tmW1, fb, kb * BK, h0, cs);
                     } else {
                         const int k2 = kb - KB1;
                         if (k2 < half)
                             tma_load_3d(sa, &tmK, fb, k2 * BK, a.y_row0 + trow, cz);
                         else
                             tma_load_3d(sa, &tmV, fb, (k2 - half) * BK, a.y_row0 + trow, cz);
+                        tma_load_3d(sb, &tmW2, fb, k2 * BK, h0, cs);
                     }
-                    if (CL > 1)
-                        tma_load_3d_mc(sb + rank * wrows * BK * 2, wm, fb, wk, h0 + rank * wrows, cs, mask);
-                    else
-                        tma_load_3d(sb, wm, fb, wk, h0, cs);
                 }
             }
-            // every stage's last release (from all CTAs of the cluster) has landed here, so
-            // no multicast arrive is still in flight towards this CTA when it exits
-            for (int s = 0; s < A_STAGES && ok; ++s)
-                if (kc > (uint32_t)s) {
-                    const uint32_t uses = (kc - 1 - s) / A_STAGES + 1;
-                    ok = mbar_wait(c.empty(s, A_STAGES), (uses - 1) & 1, a.status);
-                }
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -204,7 +184,7 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             uint32_t kc = 0;
             int local = 0;
             bool ok = true;
-            for (int ct = cluster; ct < nct && ok; ct += nclusters, ++local) {
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++local) {
                 const int b = local & 1;
                 if (local >= 2 && !mbar_wait(c.tempty(b, A_STAGES), ((local >> 1) - 1) & 1, a.status)) break;
                 tc_fence_after();
@@ -222,10 +202,7 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                     for (int k = 0; k < BK / 16; ++k)
                         umma_bf16(kb < KB1 ? dH : dR, sdesc_sw128(sa + k * 32, 16), sdesc_sw128(sb + k * 32, 16),
                                   idesc, (first && k == 0) ? 0u : 1u);
-                    if (CL > 1)
-                        umma_commit_mc(c.empty(s, A_STAGES), mask);  // frees stage s in every CTA
-                    else
-                        umma_commit(c.empty(s, A_STAGES));
+                    umma_commit(c.empty(s, A_STAGES));
                 }
                 umma_commit(c.tfull(b, A_STAGES));
             }
@@ -237,8 +214,8 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
         float* table = reinterpret_cast<float*>(c.base + LA::TAB);
         int* flag = reinterpret_cast<int*>(c.base + LA::FLAG);
         int local = 0;
-        for (int cti = cluster; cti < nct; cti += nclusters, ++local) {
-            const int cz = cti / (n_ht * n_tg), ht = (cti / n_tg) % n_ht, tt = (cti % n_tg) * CL + rank;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local) {
+            const int cz = tile / (n_ht * n_tt), ht = (tile / n_tt) % n_ht, tt = tile % n_tt;
             const int cs = a.c0 + cz, h0 = ht * A_BN, trow = tt * A_BM;
             const int b = local & 1;
             float* tab = table + b * 2 * A_BN;
@@ -317,7 +294,6 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
         }
     }
     __syncthreads();
-    if (CL > 1) cluster_sync();  // no CTA leaves while a peer may still multicast into it
     if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
@@ -661,44 +637,15 @@ cudaError_t ensure_attrs() {
 
 }  // namespace
 
-int phase_a_cluster(int T) {
-    const int n_tt = T / A_BM;
-    return n_tt % 4 == 0 ? 4 : (n_tt % 2 == 0 ? 2 : 1);
-}
-
 cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,
                               cudaStream_t st) {
     cudaError_t e = ensure_attrs();
     if (e != cudaSuccess) return e;
-    TcArgs a = make_args(s, w);
-    const int CL = phase_a_cluster(s.T);
-    a.cl = CL;
-    const int nct = w.nc * (s.T / A_BM / CL) * (s.d_hid / A_BN);
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CL;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.blockDim = dim3(THREADS);
-    cfg.dynamicSmemBytes = LA::DYN;
-    cfg.stream = st;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    // persistent grid: as many whole clusters as can be resident at once
-    static int max_clusters[5] = {0, 0, 0, 0, 0};
-    if (max_clusters[CL] == 0) {
-        cfg.gridDim = dim3(g_sms / CL * CL);
-        int n = 0;
-        e = cudaOccupancyMaxActiveClusters(&n, tc_phase_a_kernel, &cfg);
-        if (e != cudaSuccess) return e;
-        max_clusters[CL] = n > 0 ? n : 1;
-    }
-    const int clusters = nct < max_clusters[CL] ? nct : max_clusters[CL];
-    cfg.gridDim = dim3(clusters * CL);
-    const CUtensorMap& W1 = CL == 4 ? m.W1m4 : (CL == 2 ? m.W1m2 : m.W1b);
-    const CUtensorMap& W2 = CL == 4 ? m.W2m4 : (CL == 2 ? m.W2m2 : m.W2b);
-    return cudaLaunchKernelEx(&cfg, tc_phase_a_kernel, s.mode == 1 ? m.Ua : in.Xa, in.Ka, in.Va, W1, W2, a);
+    const TcArgs a = make_args(s, w);
+    const int ntiles = w.nc * (s.T / A_BM) * (s.d_hid / A_BN);
+    const int grid = ntiles < g_sms ? ntiles : g_sms;
+    tc_phase_a_kernel<<<grid, THREADS, LA::DYN, st>>>(s.mode == 1 ? m.Ua : in.Xa, in.Ka, in.Va, m.W1b, m.W2b, a);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,
