@@ -144,6 +144,29 @@ mone_status mone_ttl_context(mone_mem* m, const void* X, const void* K, const vo
 mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out, void* V_out,
                                  const long long strides[4], void* stream);
 
+/*
+ * Memory read that allocates nothing.  The paper has no counterpart: this is a
+ * service entry point for callers that must not allocate device memory while
+ * serving, e.g. a framework whose caching allocator already owns the GPU's free
+ * memory, or a latency-bound serving loop that cannot afford cudaMalloc (which
+ * can synchronise the device and take a process-wide allocator lock).
+ * mone_mem_generate_kv may allocate read scratch on its first call or when Q
+ * grows; this variant instead uses one fixed 16 MiB device array compiled into
+ * the library (every GPU that loads the library holds it until the process
+ * exits).  Same arguments, outputs and error behaviour as mone_mem_generate_kv,
+ * plus MONE_ERR_UNSUPPORTED_SHAPE when chains * Q * (d_in + d_hid + d_out) exceeds
+ * 4,194,304 floats (the size is checked before any work; mone_last_error says why).
+ * It calls no cudaMalloc, cudaFree or allocating library routine.
+ * The first call on a device resolves the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call before
+ * any stream capture.  All calls on a device share the array and every call
+ * overwrites it completely before reading it, so nothing carries over between
+ * calls, but calls whose GPU work overlaps (e.g. on two streams) race on it:
+ * order them on one stream or with events.
+ */
+mone_status mone_mem_generate_kv_noalloc(mone_mem* m, const void* Xq, int Q, void* K_out, void* V_out,
+                                         const long long strides[4], void* stream);
+
 /* Release the state.  The handle is invalid afterwards; a second free returns
  * MONE_ERR_INVALID_ARG.  Synchronises the device. */
 mone_status mone_mem_free(mone_mem* m);

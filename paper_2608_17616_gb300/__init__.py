@@ -26,7 +26,7 @@ STATUS = {0: "MONE_OK", 1: "MONE_ERR_INVALID_ARG", 2: "MONE_ERR_UNSUPPORTED_SHAP
 EXPORTS = ("mone_mem_init", "mone_ttl_segment", "mone_ttl_context", "mone_mem_generate_kv", "mone_mem_free",
            "mone_mem_read_state", "mone_mem_write_state", "mone_mem_sync", "mone_mem_launch_count",
            "mone_status_string", "mone_abi_version", "mone_mem_set_timing", "mone_mem_kernel_time",
-           "mone_last_error")
+           "mone_last_error", "mone_mem_generate_kv_noalloc")
 
 KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read")
 
@@ -67,6 +67,7 @@ def lib(path: Optional[str] = None) -> ctypes.CDLL:
         "mone_ttl_segment": ([vp, i, i, vp, vp, vp, i, vp, vp, vp], i),
         "mone_ttl_context": ([vp, vp, vp, vp, ll, vp], i),
         "mone_mem_generate_kv": ([vp, vp, i, vp, vp, ctypes.POINTER(ll), vp], i),
+        "mone_mem_generate_kv_noalloc": ([vp, vp, i, vp, vp, ctypes.POINTER(ll), vp], i),
         "mone_mem_free": ([vp], i),
         "mone_mem_read_state": ([vp, vp, vp, vp, vp, vp], i),
         "mone_mem_write_state": ([vp, vp, vp, vp, vp, vp], i),
@@ -144,6 +145,13 @@ def mone_mem_generate_kv(h: int, Xq, Q: int, K_out, V_out, strides: Sequence[int
     arr = (ctypes.c_longlong * 4)(*[int(s) for s in strides])
     _check("mone_mem_generate_kv", lib().mone_mem_generate_kv(h, _ptr(Xq), Q, _ptr(K_out), _ptr(V_out), arr,
                                                               _stream(stream)))
+
+
+def mone_mem_generate_kv_noalloc(h: int, Xq, Q: int, K_out, V_out, strides: Sequence[int], stream=None):
+    """The memory read without any device allocation (fixed 16 MiB library scratch)."""
+    arr = (ctypes.c_longlong * 4)(*[int(s) for s in strides])
+    _check("mone_mem_generate_kv_noalloc", lib().mone_mem_generate_kv_noalloc(h, _ptr(Xq), Q, _ptr(K_out),
+                                                                              _ptr(V_out), arr, _stream(stream)))
 
 
 def mone_mem_free(h: int):

@@ -445,6 +445,26 @@ mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out
     });
 }
 
+mone_status mone_mem_generate_kv_noalloc(mone_mem* m, const void* Xq, int Q, void* K_out, void* V_out,
+                                         const long long strides[4], void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    if (Q < 1 || Q > 4096 || !Xq || !K_out || !V_out || !strides) return MONE_ERR_INVALID_ARG;
+    for (int i = 0; i < 4; ++i)
+        if (strides[i] < 0) return MONE_ERR_INVALID_ARG;
+    const DevState& s = m->s;
+    const size_t need = (size_t)s.C * Q * ((size_t)s.d_in + s.d_hid + s.d_out);
+    if (need > kNoAllocScratchFloats) {
+        std::snprintf(g_last_error, sizeof(g_last_error),
+                      "mone_mem_generate_kv_noalloc: chains*Q*(d_in+d_hid+d_out) = %zu floats exceeds the fixed "
+                      "scratch of %zu floats (16 MiB)",
+                      need, kNoAllocScratchFloats);
+        return MONE_ERR_UNSUPPORTED_SHAPE;
+    }
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const int L = m->cfg.n_layers;
+    return timed(m, K_READ, st, 4, [&] { return launch_read_noalloc(s, Xq, Q, L, K_out, V_out, strides, st); });
+}
+
 mone_status mone_mem_free(mone_mem* m) {
     {
         std::lock_guard<std::mutex> lk(g_live_mu);

@@ -71,6 +71,12 @@ cudaError_t launch_read(const DevState& s, int Q, int n_layers, void* K_out, voi
                         const long long* strides, cudaStream_t st);
 cudaError_t launch_zero_f32(float* p, size_t n, cudaStream_t st);
 
+// Allocation-free read (mone_mem_generate_kv_noalloc): fixed device scratch of
+// kNoAllocScratchFloats floats, shared by every call on a device.
+constexpr size_t kNoAllocScratchFloats = (size_t(16) << 20) / sizeof(float);  // 16 MiB
+cudaError_t launch_read_noalloc(const DevState& s, const void* Xq, int Q, int n_layers, void* K_out, void* V_out,
+                                const long long* strides, cudaStream_t st);
+
 // ---- kernels in ttl_tc.cu (bf16 tcgen05 path)
 struct TcMaps {
     CUtensorMap W1b, W2b;        // K-major boxes {64, 128}

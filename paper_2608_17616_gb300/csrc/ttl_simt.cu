@@ -11,6 +11,8 @@
 // (App. A), applied lazily so that no extra pass over the weights is needed.
 // The loss L_s = -(1/T') sum_t sum_h A_th R_th equals Eq. 7's segment mean
 // because sum_h A_th R_th = y_t . (A_t W2) = y_t . M(u_t).
+#include <mutex>
+
 #include "mone_common.cuh"
 
 namespace mone {
@@ -391,6 +393,53 @@ cudaError_t launch_read(const DevState& s, int Q, int n_layers, void* K_out, voi
         read_norm_kernel<bf16><<<grid, 256, 0, st>>>(s, Q, (bf16*)K_out, (bf16*)V_out, strides[0], strides[1],
                                                      strides[2], strides[3], n_layers);
     return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ allocation-free memory read
+//
+// Scratch of mone_mem_generate_kv_noalloc: a fixed file-scope device array that
+// every GPU loading the library holds until the process exits.  Host code cannot
+// use the array's name as a device address (it is a host-side stand-in), so the
+// address is resolved with cudaGetSymbolAddress, once per device, with that
+// device current.
+
+static __device__ __align__(256) float g_noalloc_scratch[kNoAllocScratchFloats];
+
+namespace {
+std::mutex g_noalloc_mu;
+float* g_noalloc_ptr[64] = {};  // per device ordinal
+}  // namespace
+
+cudaError_t noalloc_scratch(float** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) return e;
+        g_noalloc_ptr[dev] = static_cast<float*>(p);
+    }
+    *out = g_noalloc_ptr[dev];
+    return cudaSuccess;
+}
+
+cudaError_t launch_read_noalloc(const DevState& s, const void* Xq, int Q, int n_layers, void* K_out, void* V_out,
+                                const long long* strides, cudaStream_t st) {
+    float* base = nullptr;
+    cudaError_t e = noalloc_scratch(&base);
+    if (e != cudaSuccess) return e;
+    // the same kernels as the allocating read, pointed at the fixed scratch; every
+    // element of the three regions is written before it is read, so nothing needs
+    // clearing between calls
+    DevState t = s;
+    t.Uq = base;
+    t.Aq = t.Uq + (size_t)s.C * Q * s.d_in;
+    t.Oq = t.Aq + (size_t)s.C * Q * s.d_hid;
+    e = launch_query_transform(t, Xq, Q, st);
+    return e != cudaSuccess ? e : launch_read(t, Q, n_layers, K_out, V_out, strides, st);
 }
 
 cudaError_t launch_zero_f32(float* p, size_t n, cudaStream_t st) {
