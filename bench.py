@@ -88,6 +88,8 @@ def ncu_traffic(kind):
     try:
         sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
         for line in open(path):
+            if line.lstrip().startswith("#"):
+                continue
             parts = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
             if parts.get("kernel") == kind and parts.get("source_sha") == sha:
                 return float(parts["bytes_per_launch"]), parts.get("scaled_from", "")
