@@ -68,12 +68,6 @@ struct mone_mem {
     TcMaps maps;
     long long launches;
     KernelTiming* timing;
-    // Two internal streams for the bf16 path: chains are split into two groups that
-    // run half a step apart, so one group's tensor-bound phase A overlaps the other
-    // group's HBM-bound phase B.  Forked from and joined back to the caller's stream.
-    int sms;
-    cudaStream_t aux[2];
-    cudaEvent_t ev_fork, ev_stagger, ev_join[2];
 };
 
 namespace {
@@ -143,18 +137,6 @@ void free_state(DevState& s) {
 }
 
 size_t elsize(int dtype) { return dtype == MONE_FP32 ? 4 : 2; }
-
-void free_streams(mone_mem* m) {
-    for (int k = 0; k < 2; ++k) {
-        if (m->aux[k]) cudaStreamDestroy(m->aux[k]);
-        if (m->ev_join[k]) cudaEventDestroy(m->ev_join[k]);
-        m->aux[k] = nullptr;
-        m->ev_join[k] = nullptr;
-    }
-    if (m->ev_fork) cudaEventDestroy(m->ev_fork);
-    if (m->ev_stagger) cudaEventDestroy(m->ev_stagger);
-    m->ev_fork = m->ev_stagger = nullptr;
-}
 
 #define MONE_TRY(x)                           \
     do {                                      \
@@ -226,79 +208,42 @@ mone_status timed(mone_mem* m, int kind, cudaStream_t st, int kernels, F&& fn) {
     return MONE_OK;
 }
 
-// Launch segment i of one chain group (prepass of a new window, phase A, phase B).
-mone_status segment_step(mone_mem* m, const TcInputMaps& in, SegWork& w, long long i, long long N, long long& win0,
-                         cudaStream_t st, cudaEvent_t after_phase_a = nullptr) {
-    DevState& s = m->s;
-    w.row0 = i * s.T;
-    w.Tp = (int)std::min<long long>(s.T, N - w.row0);
-    w.parity = (int)(i & 1);
-    w.renorm_pending = (s.renorm && i > 0) ? 1 : 0;
-    if (s.mode == MONE_PAPER) {
-        if (win0 < 0 || w.row0 >= win0 + s.win_rows) {
-            // input transform of the next window of segments: depends on the inputs only
-            win0 = w.row0;
-            SegWork pw = w;
-            pw.Tp = (int)std::min<long long>(s.win_rows, N - win0);
-            MONE_TRY(timed(m, K_PREPASS, st, 1, [&] { return launch_prepass(s, pw, st); }));
-        }
-        w.u_off = w.row0 - win0;
-    } else {
-        w.u_off = 0;
-    }
-    if (s.dtype == MONE_BF16) {
-        MONE_TRY(timed(m, K_PHASE_A, st, 1, [&] { return launch_phase_a_tc(s, m->maps, in, w, st); }));
-        if (after_phase_a) MONE_CUDA(cudaEventRecord(after_phase_a, st));
-        MONE_TRY(timed(m, K_PHASE_B, st, 1, [&] { return launch_phase_b_tc(s, m->maps, in, w, st); }));
-    } else {
-        MONE_TRY(timed(m, K_PHASE_A, st, 1, [&] { return launch_phase_a_f32(s, w, st); }));
-        MONE_TRY(timed(m, K_PHASE_B, st, 1, [&] { return launch_phase_b_f32(s, w, st); }));
-    }
-    return MONE_OK;
-}
-
-mone_status finish(mone_mem* m, const SegWork& w, long long S, cudaStream_t st) {
-    DevState& s = m->s;
-    if (s.renorm) {
-        const int par = (int)((S - 1) & 1);
-        MONE_TRY(timed(m, K_FINALIZE, st, 1, [&] { return launch_finalize(s, w.c0, w.nc, par, 1, st); }));
-    }
-    return MONE_OK;
-}
-
 // Run segments [0, S) of one call.  w carries chain range and input geometry.
 mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
     DevState& s = m->s;
     TcInputMaps in;
     std::memset(&in, 0, sizeof(in));
-    if (s.dtype == MONE_BF16) MONE_TRY(build_input_maps(s, &in, w.X, w.K, w.V, w.n_rows, w.in_c0 + w.nc));
+    if (s.dtype == MONE_BF16) MONE_TRY(build_input_maps(s, &in, w.X, w.K, w.V, w.n_rows, w.nc));
     const long long S = (N + s.T - 1) / s.T;
-    if (s.dtype != MONE_BF16 || w.nc < 2) {
-        long long win0 = -1;
-        for (long long i = 0; i < S; ++i) MONE_TRY(segment_step(m, in, w, i, N, win0, st));
-        return finish(m, w, S, st);
-    }
-    // two chain groups on the internal streams, each on half of the SMs
-    SegWork g[2] = {w, w};
-    const int half = w.nc / 2;
-    g[0].nc = half;
-    g[1].c0 = w.c0 + half;
-    g[1].in_c0 = w.in_c0 + half;
-    g[1].nc = w.nc - half;
-    g[0].sm_budget = g[1].sm_budget = m->sms / 2;
-    MONE_CUDA(cudaEventRecord(m->ev_fork, st));
-    for (int k = 0; k < 2; ++k) MONE_CUDA(cudaStreamWaitEvent(m->aux[k], m->ev_fork, 0));
-    long long win[2] = {-1, -1};
+    long long win0 = -1;  // first token of the current paper-mode input window
     for (long long i = 0; i < S; ++i) {
-        // the second group starts once the first has finished its first phase A
-        MONE_TRY(segment_step(m, in, g[0], i, N, win[0], m->aux[0], i == 0 ? m->ev_stagger : nullptr));
-        if (i == 0) MONE_CUDA(cudaStreamWaitEvent(m->aux[1], m->ev_stagger, 0));
-        MONE_TRY(segment_step(m, in, g[1], i, N, win[1], m->aux[1]));
+        w.row0 = i * s.T;
+        w.Tp = (int)std::min<long long>(s.T, N - w.row0);
+        w.parity = (int)(i & 1);
+        w.renorm_pending = (s.renorm && i > 0) ? 1 : 0;
+        if (s.mode == MONE_PAPER) {
+            if (win0 < 0 || w.row0 >= win0 + s.win_rows) {
+                // input transform of the next window of segments: depends on the inputs only
+                win0 = w.row0;
+                SegWork pw = w;
+                pw.Tp = (int)std::min<long long>(s.win_rows, N - win0);
+                MONE_TRY(timed(m, K_PREPASS, st, 1, [&] { return launch_prepass(s, pw, st); }));
+            }
+            w.u_off = w.row0 - win0;
+        } else {
+            w.u_off = 0;
+        }
+        if (s.dtype == MONE_BF16) {
+            MONE_TRY(timed(m, K_PHASE_A, st, 1, [&] { return launch_phase_a_tc(s, m->maps, in, w, st); }));
+            MONE_TRY(timed(m, K_PHASE_B, st, 1, [&] { return launch_phase_b_tc(s, m->maps, in, w, st); }));
+        } else {
+            MONE_TRY(timed(m, K_PHASE_A, st, 1, [&] { return launch_phase_a_f32(s, w, st); }));
+            MONE_TRY(timed(m, K_PHASE_B, st, 1, [&] { return launch_phase_b_f32(s, w, st); }));
+        }
     }
-    for (int k = 0; k < 2; ++k) {
-        MONE_TRY(finish(m, g[k], S, m->aux[k]));
-        MONE_CUDA(cudaEventRecord(m->ev_join[k], m->aux[k]));
-        MONE_CUDA(cudaStreamWaitEvent(st, m->ev_join[k], 0));
+    if (s.renorm) {
+        const int par = (int)((S - 1) & 1);
+        MONE_TRY(timed(m, K_FINALIZE, st, 1, [&] { return launch_finalize(s, w.c0, w.nc, par, 1, st); }));
     }
     return MONE_OK;
 }
@@ -414,22 +359,10 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
     if (rc == MONE_OK) step(cuda_status(launch_row_norms(s, st)));
     if (rc == MONE_OK && s.dtype == MONE_BF16) step(cuda_status(launch_finalize(s, 0, s.C, 0, 0, st)));
     if (rc == MONE_OK) step(build_state_maps(m));
-    if (rc == MONE_OK) {
-        int dev = 0;
-        step(cuda_status(cudaGetDevice(&dev)));
-        if (rc == MONE_OK) step(cuda_status(cudaDeviceGetAttribute(&m->sms, cudaDevAttrMultiProcessorCount, dev)));
-        for (int k = 0; k < 2 && rc == MONE_OK; ++k)
-            step(cuda_status(cudaStreamCreateWithFlags(&m->aux[k], cudaStreamNonBlocking)));
-        if (rc == MONE_OK) step(cuda_status(cudaEventCreateWithFlags(&m->ev_fork, cudaEventDisableTiming)));
-        if (rc == MONE_OK) step(cuda_status(cudaEventCreateWithFlags(&m->ev_stagger, cudaEventDisableTiming)));
-        for (int k = 0; k < 2 && rc == MONE_OK; ++k)
-            step(cuda_status(cudaEventCreateWithFlags(&m->ev_join[k], cudaEventDisableTiming)));
-    }
     if (rc == MONE_OK) step(cuda_status(cudaStreamSynchronize(st)));
     if (rc != MONE_OK) {
         cudaStreamSynchronize(st);
         cudaGetLastError();
-        free_streams(m);
         free_state(s);
         delete m;
         return rc;
@@ -540,7 +473,6 @@ mone_status mone_mem_free(mone_mem* m) {
     }
     cudaDeviceSynchronize();
     delete m->timing;
-    free_streams(m);
     free_state(m->s);
     delete m;
     return MONE_OK;

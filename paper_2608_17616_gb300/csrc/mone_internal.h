@@ -44,9 +44,7 @@ inline float* sumsq_ptr(const DevState& s, int parity, int which) {
 
 // One segment of work for chains [c0, c0+nc).
 struct SegWork {
-    int c0, nc;                  // state chains [c0, c0+nc)
-    int in_c0;                   // chain index of state chain c0 within the caller's input buffers
-    int sm_budget;               // persistent kernels use at most this many SMs (0 = all)
+    int c0, nc;
     const void *X, *K, *V;       // inputs (caller's buffers)
     long long x_cstride, y_cstride;  // element stride between chains in X and in K/V
     long long n_rows;            // rows per chain in the caller's buffers

@@ -259,7 +259,7 @@ cudaError_t launch_one(const PrepassArgs& a, int nchains, cudaStream_t st) {
 
 cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st) {
     PrepassArgs a{};
-    a.X = static_cast<const uint8_t*>(w.X) + (size_t)w.in_c0 * w.x_cstride * (s.dtype == 0 ? 4 : 2);
+    a.X = w.X;
     a.x_cstride = w.x_cstride;
     a.row0 = w.row0;
     a.n_rows = w.n_rows;
@@ -276,7 +276,7 @@ cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st)
     a.w_eta = s.w_eta;
     a.b_eta = s.b_eta;
     a.w_beta = s.w_beta;
-    a.eta_in = w.eta_in ? w.eta_in + (size_t)w.in_c0 * w.eta_cstride : nullptr;
+    a.eta_in = w.eta_in;
     a.eta_cstride = w.eta_cstride;
     a.U = s.U;
     a.eta = s.eta;

@@ -233,21 +233,21 @@ F32SegArgs make_f32_args(const DevState& s, const SegWork& w) {
         a.U = reinterpret_cast<const float*>(s.U) + ((size_t)w.c0 * s.win_rows + w.u_off) * s.d_in;
         a.u_cstride = (long long)s.win_rows * s.d_in;
     } else {
-        a.U = reinterpret_cast<const float*>(w.X) + w.in_c0 * w.x_cstride + w.row0 * s.d_in;
+        a.U = reinterpret_cast<const float*>(w.X) + w.row0 * s.d_in;
         a.u_cstride = w.x_cstride;
     }
-    a.K = reinterpret_cast<const float*>(w.K) + w.in_c0 * w.y_cstride + w.row0 * dh;
-    a.V = reinterpret_cast<const float*>(w.V) + w.in_c0 * w.y_cstride + w.row0 * dh;
+    a.K = reinterpret_cast<const float*>(w.K) + w.row0 * dh;
+    a.V = reinterpret_cast<const float*>(w.V) + w.row0 * dh;
     a.y_cstride = w.y_cstride;
     a.row_avail = w.n_rows - w.row0;
-    a.eta_in = w.eta_in ? w.eta_in + w.in_c0 * w.eta_cstride + w.row0 : nullptr;
+    a.eta_in = w.eta_in ? w.eta_in + w.row0 : nullptr;
     a.eta_cstride = w.eta_cstride;
     a.eta = s.eta; a.dbeta = s.dbeta; a.b_beta = s.b_beta;
     a.W1 = s.W1; a.W2 = s.W2; a.mu1 = s.mu1; a.mu2 = s.mu2; a.n1 = s.n1; a.n2 = s.n2;
     a.sumsq = s.sumsq;
     a.dH = reinterpret_cast<float*>(s.dHt);
     a.At = reinterpret_cast<float*>(s.Att);
-    a.loss = w.loss ? w.loss + w.in_c0 : nullptr;
+    a.loss = w.loss;
     a.status = s.status;
     return a;
 }

@@ -67,7 +67,6 @@ static_assert(LA::DYN <= 227 * 1024, "shared memory budget");
 struct TcArgs {
     int d_in, d_out, d_hid, T, Tp, c0, nc, C, paper, momentum, renorm_pending, parity;
     int u_row0, u_chain0, y_row0;
-    int in_c0;                  // chain coordinate of this launch's first chain in the caller's K/V maps
     long long tok0;             // per-token tables: entry of token t of chain cs is [cs * win + tok0 + t]
     int win;
     float lr;
@@ -170,9 +169,9 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                     } else {
                         const int k2 = kb - KB1;
                         if (k2 < half)
-                            tma_load_3d(sa, &tmK, fb, k2 * BK, a.y_row0 + trow, a.in_c0 + cz);
+                            tma_load_3d(sa, &tmK, fb, k2 * BK, a.y_row0 + trow, cz);
                         else
-                            tma_load_3d(sa, &tmV, fb, (k2 - half) * BK, a.y_row0 + trow, a.in_c0 + cz);
+                            tma_load_3d(sa, &tmV, fb, (k2 - half) * BK, a.y_row0 + trow, cz);
                         tma_load_3d(sb, &tmW2, fb, k2 * BK, h0, cs);
                     }
                 }
@@ -407,9 +406,9 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                         } else {
                             const int o = col0 - a.d_in + bx * 64;
                             if (o < dhalf)
-                                tma_load_3d(dst, &tmKb, fb, o, a.y_row0 + kb * BK, a.in_c0 + cz);
+                                tma_load_3d(dst, &tmKb, fb, o, a.y_row0 + kb * BK, cz);
                             else
-                                tma_load_3d(dst, &tmVb, fb, o - dhalf, a.y_row0 + kb * BK, a.in_c0 + cz);
+                                tma_load_3d(dst, &tmVb, fb, o - dhalf, a.y_row0 + kb * BK, cz);
                         }
                     }
 #pragma unroll
@@ -603,18 +602,17 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
     a.u_row0 = a.paper ? (int)w.u_off : (int)w.row0;
     a.tok0 = w.u_off;
     a.win = s.win_rows;
-    a.u_chain0 = a.paper ? w.c0 : w.in_c0;
-    a.in_c0 = w.in_c0;
+    a.u_chain0 = a.paper ? w.c0 : 0;
     a.y_row0 = (int)w.row0;
     a.lr = s.lr;
-    a.eta_in = w.eta_in ? w.eta_in + w.in_c0 * w.eta_cstride + w.row0 : nullptr;
+    a.eta_in = w.eta_in ? w.eta_in + w.row0 : nullptr;
     a.eta_cstride = w.eta_cstride;
     a.eta = s.eta; a.dbeta = s.dbeta; a.b_beta = s.b_beta;
     a.zinv = a.paper ? s.zinv : nullptr;
     a.W1 = s.W1; a.W2 = s.W2; a.mu1 = s.mu1; a.mu2 = s.mu2; a.W1b = s.W1b; a.W2b = s.W2b;
     a.n1 = s.n1; a.n2 = s.n2; a.sumsq = s.sumsq;
     a.dH = reinterpret_cast<bf16*>(s.dHt); a.At = reinterpret_cast<bf16*>(s.Att);
-    a.loss = w.loss ? w.loss + w.in_c0 : nullptr; a.status = s.status;
+    a.loss = w.loss; a.status = s.status;
     return a;
 }
 
@@ -645,8 +643,7 @@ cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputM
     if (e != cudaSuccess) return e;
     const TcArgs a = make_args(s, w);
     const int ntiles = w.nc * (s.T / A_BM) * (s.d_hid / A_BN);
-    const int budget = w.sm_budget > 0 && w.sm_budget < g_sms ? w.sm_budget : g_sms;
-    const int grid = ntiles < budget ? ntiles : budget;
+    const int grid = ntiles < g_sms ? ntiles : g_sms;
     tc_phase_a_kernel<<<grid, THREADS, LA::DYN, st>>>(s.mode == 1 ? m.Ua : in.Xa, in.Ka, in.Va, m.W1b, m.W2b, a);
     return cudaGetLastError();
 }
@@ -657,8 +654,7 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
     if (e != cudaSuccess) return e;
     const TcArgs a = make_args(s, w);
     const int ntiles = w.nc * ((s.d_in + s.d_out) / B_BM) * (s.d_hid / B_BN);
-    const int budget = w.sm_budget > 0 && w.sm_budget < g_sms ? w.sm_budget : g_sms;
-    const int grid = ntiles < budget ? ntiles : budget;
+    const int grid = ntiles < g_sms ? ntiles : g_sms;
     tc_phase_b_kernel<<<grid, B_THREADS, LayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.dH, m.At,
                                                               m.W1s, m.W2s, m.M1s, m.M2s, m.W1o, m.W2o, a);
     return cudaGetLastError();
