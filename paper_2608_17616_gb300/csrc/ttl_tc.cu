@@ -312,15 +312,16 @@ constexpr int S_SLOTS = 4;
 constexpr int S_F32 = S_ROWS * B_BM * 4;                   // 16 KB
 constexpr int S_SLOT = 2 * S_F32;                          // W and mu: 32 KB
 constexpr int B_STAGES_V3 = 2;
-constexpr int B_THREADS = 11 * 32;
+constexpr int B_THREADS = 12 * 32;
 constexpr int B_EPI_THREADS = 4 * 32;     // per epilogue group
-constexpr int B_STATE_WARP = 10;
+constexpr int B_STATE_WARP = 10;          // TMA loads of state chunks
+constexpr int B_STORE_WARP = 11;          // TMA stores of updated chunks, slot release
 
 struct LayoutB {
     static constexpr int RING = B_STAGES_V3 * B_STAGE;
     static constexpr int STATE = RING;
-    static constexpr int BARS = STATE + S_SLOTS * S_SLOT;  // full[S] empty[S] tfull[2] tempty[2] sfull[N] sempty[N]
-    static constexpr int NBARS = 2 * B_STAGES_V3 + 4 + 2 * S_SLOTS;
+    static constexpr int BARS = STATE + S_SLOTS * S_SLOT;  // full[S] empty[S] tfull[2] tempty[2] sfull/sdone/sempty[N]
+    static constexpr int NBARS = 2 * B_STAGES_V3 + 4 + 3 * S_SLOTS;
     static constexpr int SLOT = BARS + NBARS * 8;
     static constexpr int FLAG = SLOT + 16;
     static constexpr int TAB = FLAG + 16;                  // per group: [B_BN/2] renorm scales + [4] decay partials
@@ -346,6 +347,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
     auto tempty = [&](int b) { return bars + 8 * (2 * B_STAGES_V3 + 2 + b); };
     auto sfull = [&](int k) { return bars + 8 * (2 * B_STAGES_V3 + 4 + k); };
     auto sempty = [&](int k) { return bars + 8 * (2 * B_STAGES_V3 + 4 + S_SLOTS + k); };
+    auto sdone = [&](int k) { return bars + 8 * (2 * B_STAGES_V3 + 4 + 2 * S_SLOTS + k); };
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
         for (int i = 0; i < B_STAGES_V3; ++i) {
@@ -359,6 +361,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
         for (int k = 0; k < S_SLOTS; ++k) {
             mbar_init(sfull(k), 1);
             mbar_init(sempty(k), 1);
+            mbar_init(sdone(k), 4);  // the four warps of the epilogue group that updated the chunk
         }
         fence_mbar_init();
     }
@@ -477,6 +480,33 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             }
         }
         __syncwarp();
+    } else if (warp == B_STORE_WARP) {
+        // ---- store warp: write every updated chunk back with TMA, then free its slot
+        if (lane == 0) {
+            uint32_t seq = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+                const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
+                const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
+                const bool isW1 = col0 < a.d_in;
+                const int cl = isW1 ? col0 : col0 - a.d_in;
+                for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
+                    const int k = seq % S_SLOTS;
+                    if (!mbar_wait(sdone(k), (seq / S_SLOTS) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t src = smem_u32(base + L::STATE + k * S_SLOT);
+                    tma_store_3d(isW1 ? &tmW1s : &tmW2s, src, cl, h0 + g * S_ROWS, cs);
+                    if (a.momentum) tma_store_3d(isW1 ? &tmM1s : &tmM2s, src + S_F32, cl, h0 + g * S_ROWS, cs);
+                    bulk_commit();
+                    bulk_wait_read_all();  // the store has read the slot: hand it back
+                    mbar_arrive(sempty(k));
+                }
+            }
+            bulk_wait_all();
+        }
+        __syncwarp();
     } else {
         // ---- epilogue warps 2..9: group grp takes the tile's chunks grp, grp+2, grp+4, grp+6;
         //      within a group, TMEM lane quarter q = 32 weight columns
@@ -557,8 +587,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                     Ws[j * B_BM + col] = wn;
                     if (a.momentum) Ms[j * B_BM + col] = mn;
                     bp[j * width] = __float2bfloat16_rn(wn);
-                    finite = finite && isfinite(wn);
-                    v[j] = wn * wn;
+                    v[j] = wn * wn;  // a NaN or Inf weight makes its row's sum non-finite
                 }
                 // transpose-reduce: afterwards lane j holds this warp's 32-column partial of row j
 #pragma unroll
@@ -571,23 +600,15 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                         v[u] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
                     }
                 }
+                finite = finite && isfinite(v[0]);
                 atomicAdd(&cur[r0 + lane], v[0]);
+                // make this warp's shared-memory writes visible to the TMA store, then tell the store warp
                 fence_proxy_async_smem();
                 __syncwarp();
-                named_bar_sync(bar_id, B_EPI_THREADS);
-                if (et == 0) {
-                    const uint32_t src = smem_u32(slot);
-                    tma_store_3d(isW1 ? &tmW1s : &tmW2s, src, cl, r0, cs);
-                    if (a.momentum) tma_store_3d(isW1 ? &tmM1s : &tmM2s, src + S_F32, cl, r0, cs);
-                    bulk_commit();
-                    bulk_wait_read_all();  // the store has read the slot: hand it back
-                    mbar_arrive(sempty(k));
-                }
-                __syncwarp();
+                if (lane == 0) mbar_arrive(sdone(k));
             }
             if (!ok) break;
         }
-        if (et == 0) bulk_wait_all();
         if (!finite) atomicOr(a.status, DEV_NONFINITE);
     }
     __syncthreads();
