@@ -44,7 +44,6 @@ constexpr uint32_t EPI_BAR = 1;           // named barrier among the epilogue wa
 
 // phase A
 constexpr int A_BM = 128, A_BN = 128, A_STAGES = 6;
-constexpr uint32_t A_PF = 12;    // k-blocks whose tiles are prefetched into L2 ahead of their load
 constexpr int A_STAGE = (A_BM + A_BN) * BK * 2;           // 32 KB
 // phase B
 constexpr int B_BM = 128, B_BN = 256;
@@ -151,42 +150,31 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             tma_prefetch_map(&tmV);
             tma_prefetch_map(&tmW1);
             tma_prefetch_map(&tmW2);
-            // k-block number kc of this CTA (over all its tiles): the two tiles it needs.
-            // With prefetch, only warm L2 (the real load follows A_PF k-blocks later).
-            auto issue = [&](uint32_t kc, bool prefetch, uint32_t sa, uint32_t sb, uint32_t fb) {
-                const int tile = blockIdx.x + (int)(kc / KB) * gridDim.x;
-                if (tile >= ntiles) return;
-                const int kb = kc % KB;
+            uint32_t kc = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
                 const int cz = tile / (n_ht * n_tt), ht = (tile / n_tt) % n_ht, tt = tile % n_tt;
                 const int cs = a.c0 + cz, h0 = ht * A_BN, trow = tt * A_BM;
-                const CUtensorMap* am;
-                int ax, ay, az;
-                if (kb < KB1) {
-                    am = &tmU; ax = kb * BK; ay = a.u_row0 + trow; az = a.u_chain0 + cz;
-                } else {
-                    const int k2 = kb - KB1;
-                    am = k2 < half ? &tmK : &tmV;
-                    ax = (k2 < half ? k2 : k2 - half) * BK; ay = a.y_row0 + trow; az = cz;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % A_STAGES;
+                    if (kc >= A_STAGES && !mbar_wait(c.empty(s, A_STAGES), ((kc / A_STAGES) - 1) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sa = smem_u32(c.base + s * A_STAGE), sb = sa + A_BM * BK * 2, fb = c.full(s);
+                    mbar_expect_tx(fb, A_STAGE);
+                    if (kb < KB1) {
+                        tma_load_3d(sa, &tmU, fb, kb * BK, a.u_row0 + trow, a.u_chain0 + cz);
+                        tma_load_3d(sb, &tmW1, fb, kb * BK, h0, cs);
+                    } else {
+                        const int k2 = kb - KB1;
+                        if (k2 < half)
+                            tma_load_3d(sa, &tmK, fb, k2 * BK, a.y_row0 + trow, cz);
+                        else
+                            tma_load_3d(sa, &tmV, fb, (k2 - half) * BK, a.y_row0 + trow, cz);
+                        tma_load_3d(sb, &tmW2, fb, k2 * BK, h0, cs);
+                    }
                 }
-                const CUtensorMap* bm = kb < KB1 ? &tmW1 : &tmW2;
-                const int bx = (kb < KB1 ? kb : kb - KB1) * BK;
-                if (prefetch) {
-                    tma_prefetch_l2_3d(am, ax, ay, az);
-                    tma_prefetch_l2_3d(bm, bx, h0, cs);
-                } else {
-                    tma_load_3d(sa, am, fb, ax, ay, az);
-                    tma_load_3d(sb, bm, fb, bx, h0, cs);
-                }
-            };
-            const uint32_t total = (uint32_t)(((ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x) * KB);
-            for (uint32_t kc = 0; kc < A_PF && kc < total; ++kc) issue(kc, true, 0, 0, 0);
-            for (uint32_t kc = 0; kc < total; ++kc) {
-                const int s = kc % A_STAGES;
-                if (kc >= A_STAGES && !mbar_wait(c.empty(s, A_STAGES), ((kc / A_STAGES) - 1) & 1, a.status)) break;
-                if (kc + A_PF < total) issue(kc + A_PF, true, 0, 0, 0);
-                const uint32_t sa = smem_u32(c.base + s * A_STAGE), sb = sa + A_BM * BK * 2, fb = c.full(s);
-                mbar_expect_tx(fb, A_STAGE);
-                issue(kc, false, sa, sb, fb);
             }
         }
         __syncwarp();
@@ -324,8 +312,6 @@ constexpr int S_SLOTS = 4;
 constexpr int S_F32 = S_ROWS * B_BM * 4;                   // 16 KB
 constexpr int S_SLOT = 2 * S_F32;                          // W and mu: 32 KB
 constexpr int B_STAGES_V3 = 2;
-constexpr uint32_t B_PF = 6;      // operand k-blocks prefetched into L2 ahead of their load
-constexpr uint32_t S_PF = 8;      // state chunks prefetched into L2 ahead of their load
 constexpr int B_THREADS = 12 * 32;
 constexpr int B_EPI_THREADS = 4 * 32;     // per epilogue group
 constexpr int B_STATE_WARP = 10;          // TMA loads of state chunks
@@ -401,47 +387,37 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             tma_prefetch_map(&tmVb);
             tma_prefetch_map(&tmDH);
             tma_prefetch_map(&tmAT);
-            // k-block number kc of this CTA over all its tiles; prefetch only warms L2
-            auto issue = [&](uint32_t kc, bool prefetch, uint32_t sa, uint32_t sb, uint32_t fb) {
-                const int tile = blockIdx.x + (int)(kc / KB) * gridDim.x;
-                if (tile >= ntiles) return;
-                const int kb = kc % KB;
+            uint32_t kc = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
                 const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
                 const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
                 const bool isW1 = col0 < a.d_in;
-#pragma unroll
-                for (int bx = 0; bx < B_BM / 64; ++bx) {
-                    const CUtensorMap* m;
-                    int x, z;
-                    if (isW1) {
-                        m = &tmUb; x = col0 + bx * 64; z = a.u_chain0 + cz;
-                    } else {
-                        const int o = col0 - a.d_in + bx * 64;
-                        m = o < dhalf ? &tmKb : &tmVb; x = o < dhalf ? o : o - dhalf; z = cz;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % B_STAGES_V3;
+                    if (kc >= B_STAGES_V3 && !mbar_wait(empty(s), ((kc / B_STAGES_V3) - 1) & 1, a.status)) {
+                        ok = false;
+                        break;
                     }
-                    const int y = (isW1 ? a.u_row0 : a.y_row0) + kb * BK;
-                    if (prefetch)
-                        tma_prefetch_l2_3d(m, x, y, z);
-                    else
-                        tma_load_3d(sa + bx * BOX, m, fb, x, y, z);
-                }
+                    const uint32_t sa = smem_u32(base + s * B_STAGE), sb = sa + B_BM * BK * 2, fb = full(s);
+                    mbar_expect_tx(fb, B_STAGE);
 #pragma unroll
-                for (int bx = 0; bx < B_BN / 64; ++bx) {
-                    if (prefetch)
-                        tma_prefetch_l2_3d(isW1 ? &tmDH : &tmAT, h0 + bx * 64, kb * BK, cs);
-                    else
+                    for (int bx = 0; bx < B_BM / 64; ++bx) {
+                        const uint32_t dst = sa + bx * BOX;
+                        if (isW1) {
+                            tma_load_3d(dst, &tmUb, fb, col0 + bx * 64, a.u_row0 + kb * BK, a.u_chain0 + cz);
+                        } else {
+                            const int o = col0 - a.d_in + bx * 64;
+                            if (o < dhalf)
+                                tma_load_3d(dst, &tmKb, fb, o, a.y_row0 + kb * BK, cz);
+                            else
+                                tma_load_3d(dst, &tmVb, fb, o - dhalf, a.y_row0 + kb * BK, cz);
+                        }
+                    }
+#pragma unroll
+                    for (int bx = 0; bx < B_BN / 64; ++bx)
                         tma_load_3d(sb + bx * BOX, isW1 ? &tmDH : &tmAT, fb, h0 + bx * 64, kb * BK, cs);
                 }
-            };
-            const uint32_t total = (uint32_t)(((ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x) * KB);
-            for (uint32_t kc = 0; kc < B_PF && kc < total; ++kc) issue(kc, true, 0, 0, 0);
-            for (uint32_t kc = 0; kc < total; ++kc) {
-                const int s = kc % B_STAGES_V3;
-                if (kc >= B_STAGES_V3 && !mbar_wait(empty(s), ((kc / B_STAGES_V3) - 1) & 1, a.status)) break;
-                if (kc + B_PF < total) issue(kc + B_PF, true, 0, 0, 0);
-                const uint32_t sa = smem_u32(base + s * B_STAGE), sb = sa + B_BM * BK * 2, fb = full(s);
-                mbar_expect_tx(fb, B_STAGE);
-                issue(kc, false, sa, sb, fb);
             }
         }
         __syncwarp();
@@ -483,32 +459,24 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 tma_prefetch_map(&tmM1s);
                 tma_prefetch_map(&tmM2s);
             }
-            // chunk number seq of this CTA over all its tiles; prefetch only warms L2
-            constexpr int CPT = B_BN / S_ROWS;  // chunks per tile
-            auto issue = [&](uint32_t seq, bool prefetch, uint32_t dst, uint32_t bar) {
-                const int tile = blockIdx.x + (int)(seq / CPT) * gridDim.x;
-                if (tile >= ntiles) return;
-                const int g = seq % CPT;
+            uint32_t seq = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
                 const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
-                const int cs = a.c0 + cz, row = ht * B_BN + g * S_ROWS, col0 = ct * B_BM;
+                const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
                 const bool isW1 = col0 < a.d_in;
                 const int cl = isW1 ? col0 : col0 - a.d_in;
-                if (prefetch) {
-                    tma_prefetch_l2_3d(isW1 ? &tmW1s : &tmW2s, cl, row, cs);
-                    if (a.momentum) tma_prefetch_l2_3d(isW1 ? &tmM1s : &tmM2s, cl, row, cs);
-                } else {
-                    tma_load_3d(dst, isW1 ? &tmW1s : &tmW2s, bar, cl, row, cs);
-                    if (a.momentum) tma_load_3d(dst + S_F32, isW1 ? &tmM1s : &tmM2s, bar, cl, row, cs);
+                for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
+                    const int k = seq % S_SLOTS;
+                    if (seq >= S_SLOTS && !mbar_wait(sempty(k), ((seq / S_SLOTS) - 1) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t dst = smem_u32(base + L::STATE + k * S_SLOT);
+                    mbar_expect_tx(sfull(k), chunk_bytes);
+                    tma_load_3d(dst, isW1 ? &tmW1s : &tmW2s, sfull(k), cl, h0 + g * S_ROWS, cs);
+                    if (a.momentum) tma_load_3d(dst + S_F32, isW1 ? &tmM1s : &tmM2s, sfull(k), cl, h0 + g * S_ROWS, cs);
                 }
-            };
-            const uint32_t total = (uint32_t)(((ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x) * CPT);
-            for (uint32_t q = 0; q < S_PF && q < total; ++q) issue(q, true, 0, 0);
-            for (uint32_t seq = 0; seq < total; ++seq) {
-                const int k = seq % S_SLOTS;
-                if (seq >= S_SLOTS && !mbar_wait(sempty(k), ((seq / S_SLOTS) - 1) & 1, a.status)) break;
-                if (seq + S_PF < total) issue(seq + S_PF, true, 0, 0);
-                mbar_expect_tx(sfull(k), chunk_bytes);
-                issue(seq, false, smem_u32(base + L::STATE + k * S_SLOT), sfull(k));
             }
         }
         __syncwarp();
