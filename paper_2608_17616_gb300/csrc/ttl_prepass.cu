@@ -125,33 +125,47 @@ __global__ void __launch_bounds__(256) prepass_kernel(const PrepassArgs a) {
     for (int r = 0; r < RPW; ++r) ss[r] = de[r] = db[r] = 0.f;
     if (a.paper && a.zinv) {
         // one pass: write z = SiLU(alpha x + gamma) unnormalised; the row scale 1/|z|
-        // is applied by the consumer (it commutes with the contraction over d_in)
-#pragma unroll 2
-        for (int i0 = lane * V; i0 < d; i0 += 32 * V) {
-            float av[V], gv[V], wev[V], wbv[V];
-            load_f32<V>(al + i0, av);
-            load_f32<V>(ga + i0, gv);
-            load_f32<V>(we + i0, wev);
-            load_f32<V>(wb + i0, wbv);
+        // is applied by the consumer (it commutes with the contraction over d_in).
+        // Loads of a 4-vector super-chunk are all issued before any arithmetic.
+        constexpr int SC = 4;
+        for (int base = lane * V; base < d; base += SC * 32 * V) {
+            uint4 xr[RPW][SC];
 #pragma unroll
-            for (int r = 0; r < RPW; ++r) {
-                if (t0 + r >= a.rows) continue;
-                float xv[V];
-                if (live[r]) {
-                    Vec<Tin>::unpack(*reinterpret_cast<const uint4*>(x[r] + i0), xv);
+            for (int r = 0; r < RPW; ++r)
 #pragma unroll
-                    for (int e = 0; e < V; ++e) {
-                        de[r] = fmaf(wev[e], xv[e], de[r]);
-                        db[r] = fmaf(wbv[e], xv[e], db[r]);
-                        const float zp = fmaf(av[e], xv[e], gv[e]);
-                        xv[e] = zp * sig<Tin>(zp);
-                        ss[r] = fmaf(xv[e], xv[e], ss[r]);
-                    }
-                } else {
-#pragma unroll
-                    for (int e = 0; e < V; ++e) xv[e] = 0.f;
+                for (int q = 0; q < SC; ++q) {
+                    const int i0 = base + q * 32 * V;
+                    if (live[r] && i0 < d) xr[r][q] = __ldg(reinterpret_cast<const uint4*>(x[r] + i0));
                 }
-                store_vec<Tout, V>(u[r] + i0, xv);
+#pragma unroll
+            for (int q = 0; q < SC; ++q) {
+                const int i0 = base + q * 32 * V;
+                if (i0 >= d) break;
+                float av[V], gv[V], wev[V], wbv[V];
+                load_f32<V>(al + i0, av);
+                load_f32<V>(ga + i0, gv);
+                load_f32<V>(we + i0, wev);
+                load_f32<V>(wb + i0, wbv);
+#pragma unroll
+                for (int r = 0; r < RPW; ++r) {
+                    if (t0 + r >= a.rows) continue;
+                    float xv[V];
+                    if (live[r]) {
+                        Vec<Tin>::unpack(xr[r][q], xv);
+#pragma unroll
+                        for (int e = 0; e < V; ++e) {
+                            de[r] = fmaf(wev[e], xv[e], de[r]);
+                            db[r] = fmaf(wbv[e], xv[e], db[r]);
+                            const float zp = fmaf(av[e], xv[e], gv[e]);
+                            xv[e] = zp * sig<Tin>(zp);
+                            ss[r] = fmaf(xv[e], xv[e], ss[r]);
+                        }
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < V; ++e) xv[e] = 0.f;
+                    }
+                    store_vec<Tout, V>(u[r] + i0, xv);
+                }
             }
         }
 #pragma unroll
