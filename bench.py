@@ -193,6 +193,23 @@ def oracle_sample(wl, seconds, chain=0):
 
 # ------------------------------------------------------------------ arms
 
+def max_over_ranks(x: float, device="cpu") -> float:
+    """The largest value of x over all ranks (x itself without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(ms_local: float, tokens_per_rank: int, world: int, device="cpu"):
+    """(ms per step, whole-job tokens/s): every rank's tokens over the slowest rank's time."""
+    ms = max_over_ranks(ms_local, device)
+    return ms, world * tokens_per_rank / (ms / 1000.0)
+
+
 def dist_setup():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -291,13 +308,8 @@ def run_ours(args, wl):
     mone.mone_mem_set_timing(h, False)
     clk = clocks.stop()
     mone.mone_mem_sync(h)
-    if ws > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
     tokens_per_step = wl.n_ctx * wl.N
-    value = ws * tokens_per_step / (ms / 1000.0)
+    ms, value = job_rate(ms, tokens_per_step, ws, dev)
 
     # ---- end to end through the public calls with host buffers: the context arrives from
     # pinned host memory in chunks of whole segments; chunk k+1 is copied (copy stream) while
@@ -358,12 +370,7 @@ def run_ours(args, wl):
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
-        ms_e2e = e0.elapsed_time(e1) / n_e2e
-        if ws > 1:
-            import torch.distributed as dist
-            t = torch.tensor([ms_e2e], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms_e2e = float(t.item())
+        ms_e2e, _ = job_rate(e0.elapsed_time(e1) / n_e2e, tokens_per_step, ws, dev)
         h2d = sum(t.numel() * t.element_size() for t in (*hX, *hK, *hV, hXq))
         d2h = sum(t.numel() * t.element_size() for t in (hKo, hVo))
         e2e = {"value": ws * tokens_per_step / (ms_e2e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
