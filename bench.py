@@ -63,9 +63,10 @@ def peaks():
 
 # ------------------------------------------------------------------ algorithmic work per launch
 
-def kernel_work(wl, kind):
-    """(flops, bytes) of one launch of a phase kernel: one segment of every chain."""
-    C, T = wl.chains, wl.seg_T
+def kernel_work(wl, kind, chains=None):
+    """(flops, bytes) of one launch of a phase kernel: one segment of `chains` chains
+    (all of them by default; the library runs the chains of a call in two groups)."""
+    C, T = (wl.chains if chains is None else chains), wl.seg_T
     di, dh, do = wl.d_in, wl.d_hid, wl.d_out
     params = dh * (di + do)
     flops = 2 * T * dh * (di + do) * C
@@ -304,6 +305,7 @@ def run_ours(args, wl):
     barrier()
     launches = mone.mone_mem_launch_count(h) - n0
     ms = e0.elapsed_time(e1) / args.steps
+    timed_segments = args.steps * ((wl.N + wl.seg_T - 1) // wl.seg_T)
     ktimes = {name: mone.mone_mem_kernel_time(h, i) for i, name in enumerate(mone.KERNEL_KINDS)}
     mone.mone_mem_set_timing(h, False)
     clk = clocks.stop()
@@ -384,7 +386,9 @@ def run_ours(args, wl):
         if n == 0:
             continue
         avg_ms = tot / n
-        flops, byts = kernel_work(wl, name)
+        # chains per launch, from the launches the library made for the timed steps
+        chains = wl.chains * timed_segments / n
+        flops, byts = kernel_work(wl, name, chains)
         kern[name] = {"share": tot / max(1e-9, sum(v[0] for v in ktimes.values())), "avg_us": 1000 * avg_ms,
                       "launches": n, "tflops": flops / (avg_ms / 1000) / 1e12,
                       "gbs": byts / (avg_ms / 1000) / 1e9}

@@ -68,6 +68,8 @@ struct mone_mem {
     TcMaps maps;
     long long launches;
     KernelTiming* timing;
+    cudaStream_t side;               // second chain group's stream (bf16 path, >= 2 chains), or null
+    cudaEvent_t ev_fork, ev_join;    // caller stream -> side stream, side stream -> caller stream
 };
 
 namespace {
@@ -137,6 +139,14 @@ void free_state(DevState& s) {
 }
 
 size_t elsize(int dtype) { return dtype == MONE_FP32 ? 4 : 2; }
+
+void destroy_streams(mone_mem* m) {
+    if (m->ev_fork) cudaEventDestroy(m->ev_fork);
+    if (m->ev_join) cudaEventDestroy(m->ev_join);
+    if (m->side) cudaStreamDestroy(m->side);
+    m->ev_fork = m->ev_join = nullptr;
+    m->side = nullptr;
+}
 
 #define MONE_TRY(x)                           \
     do {                                      \
@@ -209,43 +219,104 @@ mone_status timed(mone_mem* m, int kind, cudaStream_t st, int kernels, F&& fn) {
 }
 
 // Run segments [0, S) of one call.  w carries chain range and input geometry.
-mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
+//
+// The chains of a call are independent (Eq. 11).  On the tensor-core path they
+// run as two groups, one on the caller's stream and one on the handle's side
+// stream, each group stepping through its segments in order.  Phase A (tensor
+// and L2 bound) and phase B (HBM bound) of one group overlap the other group's
+// kernels, which fills the SMs a single kernel leaves idle in its last wave and
+// between launches.  The side stream forks from the caller's stream before the
+// first phase launch and joins it before every input-transform window and at
+// the end, so the call stays ordered on the caller's stream.
+mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, int G, const SegWork& w, long long N,
+                             cudaStream_t st, bool& forked) {
     DevState& s = m->s;
-    TcInputMaps in;
-    std::memset(&in, 0, sizeof(in));
-    if (s.dtype == MONE_BF16) MONE_TRY(build_input_maps(s, &in, w.X, w.K, w.V, w.n_rows, w.nc));
+    const cudaStream_t gs[2] = {st, m->side};
+    auto join = [&]() -> mone_status {
+        if (forked) {
+            forked = false;
+            MONE_CUDA(cudaEventRecord(m->ev_join, m->side));
+            MONE_CUDA(cudaStreamWaitEvent(st, m->ev_join, 0));
+        }
+        return MONE_OK;
+    };
     const long long S = (N + s.T - 1) / s.T;
     long long win0 = -1;  // first token of the current paper-mode input window
     for (long long i = 0; i < S; ++i) {
-        w.row0 = i * s.T;
-        w.Tp = (int)std::min<long long>(s.T, N - w.row0);
-        w.parity = (int)(i & 1);
-        w.renorm_pending = (s.renorm && i > 0) ? 1 : 0;
+        const long long row0 = i * s.T;
+        long long u_off = 0;
         if (s.mode == MONE_PAPER) {
-            if (win0 < 0 || w.row0 >= win0 + s.win_rows) {
-                // input transform of the next window of segments: depends on the inputs only
-                win0 = w.row0;
+            if (win0 < 0 || row0 >= win0 + s.win_rows) {
+                // input transform of the next window of segments: depends on the inputs only,
+                // and overwrites the previous window, so both groups must be done with it
+                MONE_TRY(join());
+                win0 = row0;
                 SegWork pw = w;
+                pw.row0 = row0;
                 pw.Tp = (int)std::min<long long>(s.win_rows, N - win0);
                 MONE_TRY(timed(m, K_PREPASS, st, 1, [&] { return launch_prepass(s, pw, st); }));
             }
-            w.u_off = w.row0 - win0;
-        } else {
-            w.u_off = 0;
+            u_off = row0 - win0;
         }
-        if (s.dtype == MONE_BF16) {
-            MONE_TRY(timed(m, K_PHASE_A, st, 1, [&] { return launch_phase_a_tc(s, m->maps, in, w, st); }));
-            MONE_TRY(timed(m, K_PHASE_B, st, 1, [&] { return launch_phase_b_tc(s, m->maps, in, w, st); }));
-        } else {
-            MONE_TRY(timed(m, K_PHASE_A, st, 1, [&] { return launch_phase_a_f32(s, w, st); }));
-            MONE_TRY(timed(m, K_PHASE_B, st, 1, [&] { return launch_phase_b_f32(s, w, st); }));
+        if (G > 1 && !forked) {
+            MONE_CUDA(cudaEventRecord(m->ev_fork, st));
+            MONE_CUDA(cudaStreamWaitEvent(m->side, m->ev_fork, 0));
+            forked = true;
+        }
+        for (int g = 0; g < G; ++g) {
+            SegWork& x = gw[g];
+            const cudaStream_t sg = gs[g];
+            x.row0 = row0;
+            x.Tp = (int)std::min<long long>(s.T, N - row0);
+            x.parity = (int)(i & 1);
+            x.renorm_pending = (s.renorm && i > 0) ? 1 : 0;
+            x.u_off = u_off;
+            if (s.dtype == MONE_BF16) {
+                MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_phase_a_tc(s, m->maps, gin[g], x, sg); }));
+                MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_phase_b_tc(s, m->maps, gin[g], x, sg); }));
+            } else {
+                MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_phase_a_f32(s, x, sg); }));
+                MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_phase_b_f32(s, x, sg); }));
+            }
         }
     }
+    MONE_TRY(join());
     if (s.renorm) {
         const int par = (int)((S - 1) & 1);
         MONE_TRY(timed(m, K_FINALIZE, st, 1, [&] { return launch_finalize(s, w.c0, w.nc, par, 1, st); }));
     }
     return MONE_OK;
+}
+
+mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
+    DevState& s = m->s;
+    const int G = (m->side && w.nc >= 2) ? 2 : 1;
+    SegWork gw[2];
+    TcInputMaps gin[2];
+    const size_t el = elsize(s.dtype);
+    for (int g = 0, off = 0; g < G; ++g) {
+        const int n = w.nc / G + (g < w.nc % G ? 1 : 0);
+        gw[g] = w;
+        gw[g].c0 = w.c0 + off;
+        gw[g].nc = n;
+        gw[g].X = static_cast<const uint8_t*>(w.X) + (size_t)off * w.x_cstride * el;
+        gw[g].K = static_cast<const uint8_t*>(w.K) + (size_t)off * w.y_cstride * el;
+        gw[g].V = static_cast<const uint8_t*>(w.V) + (size_t)off * w.y_cstride * el;
+        if (w.eta_in) gw[g].eta_in = w.eta_in + (size_t)off * w.eta_cstride;
+        if (w.loss) gw[g].loss = w.loss + off;
+        std::memset(&gin[g], 0, sizeof(TcInputMaps));
+        if (s.dtype == MONE_BF16)
+            MONE_TRY(build_input_maps(s, &gin[g], gw[g].X, gw[g].K, gw[g].V, w.n_rows, n));
+        off += n;
+    }
+    bool forked = false;
+    const mone_status rc = run_segment_loop(m, gw, gin, G, w, N, st, forked);
+    if (forked) {
+        // error after the fork: still order the side stream's work before the caller's stream
+        cudaEventRecord(m->ev_join, m->side);
+        cudaStreamWaitEvent(st, m->ev_join, 0);
+    }
+    return rc;
 }
 
 }  // namespace
@@ -367,6 +438,19 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
         delete m;
         return rc;
     }
+    if (s.dtype == MONE_BF16 && s.C >= 2) {
+        // second chain group's stream and the fork/join events (see run_segments)
+        cudaError_t e = cudaStreamCreateWithFlags(&m->side, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&m->ev_fork, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&m->ev_join, cudaEventDisableTiming);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            destroy_streams(m);
+            free_state(s);
+            delete m;
+            return cuda_status(e);
+        }
+    }
     m->launches = 1 + (s.dtype == MONE_BF16 ? 1 : 0);
     {
         std::lock_guard<std::mutex> lk(g_live_mu);
@@ -473,6 +557,7 @@ mone_status mone_mem_free(mone_mem* m) {
     }
     cudaDeviceSynchronize();
     delete m->timing;
+    destroy_streams(m);
     free_state(m->s);
     delete m;
     return MONE_OK;
