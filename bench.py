@@ -82,8 +82,9 @@ def kernel_work(wl, kind, chains=None):
     return flops, byts
 
 
-def ncu_traffic(kind):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged."""
+def ncu_traffic(kind, chains):
+    """DRAM bytes per launch of `chains` chains from the committed ncu summary (scaled from the
+    captured launch's chain count), if the kernel source is unchanged."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
     src = os.path.join(ROOT, "paper_2608_17616_gb300", "csrc", "ttl_tc.cu")
     try:
@@ -93,7 +94,11 @@ def ncu_traffic(kind):
                 continue
             parts = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
             if parts.get("kernel") == kind and parts.get("source_sha") == sha:
-                return float(parts["bytes_per_launch"]), parts.get("scaled_from", "")
+                cap = float(parts.get("chains", chains))
+                note = parts.get("scaled_from", "")
+                if abs(cap - chains) > 1e-9:
+                    note = f"{note}; scaled from a {cap:g}-chain launch to {chains:g} chains"
+                return float(parts["bytes_per_launch"]) * chains / cap, note
     except Exception:
         pass
     return None, ""
@@ -389,18 +394,31 @@ def run_ours(args, wl):
         # chains per launch, from the launches the library made for the timed steps
         chains = wl.chains * timed_segments / n
         flops, byts = kernel_work(wl, name, chains)
-        kern[name] = {"share": tot / max(1e-9, sum(v[0] for v in ktimes.values())), "avg_us": 1000 * avg_ms,
+        kern[name] = {"chains_per_launch": chains,
+                      "share": tot / max(1e-9, sum(v[0] for v in ktimes.values())), "avg_us": 1000 * avg_ms,
                       "launches": n, "tflops": flops / (avg_ms / 1000) / 1e12,
                       "gbs": byts / (avg_ms / 1000) / 1e9}
     dom = max(kern, key=lambda k: kern[k]["share"])
     d = kern[dom]
-    traffic, traffic_note = ncu_traffic(dom)
+    traffic, traffic_note = ncu_traffic(dom, d["chains_per_launch"])
     if dom == "phase_b":
         roof = {"kernel": dom, "bound": "hbm", "achieved": d["gbs"], "peak": hbm, "unit": "GB/s",
                 "frac": d["gbs"] / hbm, "traffic": traffic, "peak_source": f"{peak_src} hbm_gbs"}
     else:
         roof = {"kernel": dom, "bound": "tensor", "achieved": d["tflops"], "peak": tf_sus, "unit": "TFLOP/s",
                 "frac": d["tflops"] / tf_sus, "traffic": traffic, "peak_source": f"{peak_src} bf16_tflops_sustained"}
+    if traffic_note.strip("; "):
+        roof["traffic_note"] = traffic_note.strip("; ")
+    if d["chains_per_launch"] < wl.chains:
+        roof["note"] = ("launches of the two chain groups run concurrently on two streams; a launch's "
+                        "duration includes the SMs and HBM bandwidth the other group's kernels take")
+    # the whole step against HBM: algorithmic bytes of every kernel of the step / step time
+    S = (wl.N + wl.seg_T - 1) // wl.seg_T
+    step_bytes = S * (kernel_work(wl, "phase_a")[1] + kernel_work(wl, "phase_b")[1])
+    if wl.mode == 1:
+        step_bytes += wl.chains * wl.N * wl.d_in * 2 * 2      # input transform: read X, write z (bf16)
+    step_roof = {"bytes_per_step": step_bytes, "achieved": step_bytes / (ms / 1000) / 1e9, "peak": hbm,
+                 "unit": "GB/s", "frac": step_bytes / (ms / 1000) / 1e9 / hbm}
     total_flops = 4 * (wl.d_in * wl.d_hid + wl.d_hid * wl.d_out) * wl.N * wl.chains
     tensor_util = total_flops / (ms / 1000) / 1e12 / tf_burst
 
@@ -415,7 +433,7 @@ def run_ours(args, wl):
                 "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
                 "config": config_of(wl), "e2e": e2e, "gpu_launches": launches, "roofline": roof,
                 "cpu_baseline": cpu, "clocks": clk,
-                "tensor_util_of_burst_peak": tensor_util,
+                "tensor_util_of_burst_peak": tensor_util, "step_roofline": step_roof,
                 "kernels": kern}
         print(json.dumps(line), flush=True)
     mone.mone_mem_free(h)
