@@ -18,6 +18,14 @@ __device__ __forceinline__ float softplusf_(float z) { return z > 20.0f ? z : lo
 // Fast logistic for bf16-output epilogues (relative error far below bf16 rounding).
 __device__ __forceinline__ float sigmoid_fast(float z) { return __fdividef(1.0f, 1.0f + __expf(-z)); }
 
+// Logistic through the identity sigma(z) = 1/2 + tanh(z/2)/2 and the hardware tanh
+// approximation (one MUFU op; relative error ~2^-11, far below bf16 output rounding).
+__device__ __forceinline__ float sigmoid_tanh(float z) {
+    float t;
+    asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(0.5f * z));
+    return fmaf(0.5f, t, 0.5f);
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

@@ -131,6 +131,132 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 
 // ------------------------------------------------------------------ phase A
 
+// Epilogue of one phase A tile (chain cs, token rows trow.., hidden columns h0..h0+BN)
+// held in TMEM at `tmem` (H in columns [0, BN), R in [BN, 2 BN), one token per lane), run
+// by the EPI_WARPS epilogue warps (warp = TMEM lane quarter x column half).  Builds the
+// tile's renormalisation scales, zeroes the segment's row sums of squares when `zero_ss`,
+// waits for the accumulators, then writes dH and At and adds the loss partial.
+// `release` is called by every epilogue warp once its last TMEM read of the tile is
+// done.  Returns false if the accumulator wait timed out.
+// Store a warp's 32 rows x 32 bf16 columns (lane = row, `pk` = its row packed in pairs)
+// to rows row0 .. row0 + 31 of a row-major matrix with `ld` elements per row.  The
+// chunk is transposed through the warp's 2 KB staging buffer (16-byte pieces XOR-
+// swizzled per row pair, conflict-free both ways) so that each global store
+// instruction writes 8 rows x 64 contiguous bytes instead of 32 scattered 16-byte pieces.
+__device__ __forceinline__ void store_rows_coalesced(uint8_t* stg, const uint32_t (&pk)[16], bf16* row0, int ld,
+                                                     int lane) {
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+        *reinterpret_cast<uint4*>(stg + lane * 64 + ((p ^ ((lane >> 1) & 3)) * 16)) =
+            make_uint4(pk[4 * p], pk[4 * p + 1], pk[4 * p + 2], pk[4 * p + 3]);
+    __syncwarp();
+    const int i = lane & 3;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int r = 8 * k + (lane >> 2);
+        const uint4 v = *reinterpret_cast<const uint4*>(stg + r * 64 + ((i ^ ((r >> 1) & 3)) * 16));
+        *reinterpret_cast<uint4*>(row0 + (size_t)r * ld + i * 8) = v;
+    }
+    __syncwarp();
+}
+
+template <int BN, class Release>
+__device__ __forceinline__ bool phase_a_epilogue(const TcArgs& a, uint32_t tmem, uint32_t tfull_bar, int parity_bit,
+                                                 float* tab, int* flag, int cz, int cs, int h0, int trow,
+                                                 bool zero_ss, uint8_t* stg, Release&& release) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int e = warp - 2, q = warp & 3, ch = e >> 2, et = threadIdx.x - 64;
+    static_assert(BN <= EPI_THREADS && BN % 64 == 0, "one scale per epilogue thread, 32-column chunks");
+    if (et < BN) {
+        const int h = h0 + et;
+        float s1 = 1.f, s2 = 1.f;
+        if (a.renorm_pending) {
+            s1 = renorm_scale(a.n1[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 0, cs)[h]);
+            s2 = renorm_scale(a.n2[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 1, cs)[h]);
+        }
+        tab[et] = s1;
+        tab[BN + et] = s2;
+        if (zero_ss) {
+            ss_row(a, a.parity, 0, cs)[h] = 0.f;
+            ss_row(a, a.parity, 1, cs)[h] = 0.f;
+        }
+    }
+    if (et == 0) *flag = mbar_wait(tfull_bar, parity_bit, a.status) ? 1 : 0;
+    __syncwarp();
+    named_bar_sync(EPI_BAR, EPI_THREADS);
+    if (!*flag) return false;
+    tc_fence_after();
+    const int row = q * 32 + lane;
+    const int t = trow + row;
+    float ct = 0.f, zi = 1.f;
+    if (t < a.Tp) {
+        const float ev = a.paper ? a.eta[(size_t)cs * a.win + a.tok0 + t]
+                                 : (a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr);
+        ct = -ev / (float)a.Tp;
+        if (a.zinv) zi = a.zinv[(size_t)cs * a.win + a.tok0 + t];
+    }
+    const float czi = ct * zi;
+    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+    bf16* dHrow = a.dH + ((size_t)cs * a.T + t) * a.d_hid + h0;
+    bf16* Arow = a.At + ((size_t)cs * a.T + t) * a.d_hid + h0;
+    float lsum = 0.f;
+    constexpr int CHUNKS = BN / 64;  // 32-column chunks per warp (each warp holds BN / 2 columns)
+#pragma unroll 1
+    for (int cc = 0; cc < CHUNKS; ++cc) {
+        const int c0 = ch * (BN / 2) + cc * 32;
+        float hv[32], rv[32];
+        tmem_ld32(lane_base + c0, hv);
+        tmem_ld32(lane_base + BN + c0, rv);
+        if (cc == CHUNKS - 1) {
+            tc_fence_before();
+            __syncwarp();
+            release();
+        }
+        uint32_t pd[16], pa[16];
+#pragma unroll
+        for (int j = 0; j < 32; j += 4) {
+            const float4 s1v = *reinterpret_cast<const float4*>(tab + c0 + j);
+            const float4 s2v = *reinterpret_cast<const float4*>(tab + BN + c0 + j);
+            const float s1a[4] = {s1v.x, s1v.y, s1v.z, s1v.w};
+            const float s2a[4] = {s2v.x, s2v.y, s2v.z, s2v.w};
+            float dv[4], av4[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float x = hv[j + u] * s1a[u] * zi;
+                const float r = rv[j + u] * s2a[u];
+                const float sg = sigmoid_tanh(x);
+                const float av = x * sg;
+                lsum = fmaf(av, r, lsum);
+                dv[u] = czi * r * (sg * fmaf(x, 1.f - sg, 1.f));  // c_t (dL/dA) SiLU'(x), scaled by 1/|z_t|
+                av4[u] = ct * av;
+            }
+            pd[j / 2] = pack_bf16(dv[0], dv[1]);
+            pd[j / 2 + 1] = pack_bf16(dv[2], dv[3]);
+            pa[j / 2] = pack_bf16(av4[0], av4[1]);
+            pa[j / 2 + 1] = pack_bf16(av4[2], av4[3]);
+        }
+        if (stg) {
+            // rows trow + q*32 .. +31 of this warp, columns h0 + c0 .. +31
+            const size_t r0 = ((size_t)cs * a.T + trow + q * 32) * a.d_hid + h0 + c0;
+            store_rows_coalesced(stg, pd, a.dH + r0, a.d_hid, lane);
+            store_rows_coalesced(stg, pa, a.At + r0, a.d_hid, lane);
+        } else {
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+                *reinterpret_cast<uint4*>(dHrow + c0 + v * 8) =
+                    make_uint4(pd[4 * v], pd[4 * v + 1], pd[4 * v + 2], pd[4 * v + 3]);
+                *reinterpret_cast<uint4*>(Arow + c0 + v * 8) =
+                    make_uint4(pa[4 * v], pa[4 * v + 1], pa[4 * v + 2], pa[4 * v + 3]);
+            }
+        }
+    }
+    if (a.loss) {
+        lsum = warp_sum(lsum);
+        if (lane == 0) atomicAdd(&a.loss[cz], -lsum / (float)a.Tp);
+    }
+    return true;
+}
+
 __global__ void __launch_bounds__(THREADS, 1)
 tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmW1,
@@ -209,92 +335,191 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
         }
         __syncwarp();
     } else {
-        // ---- epilogue warps: TMEM lane quarter q, hidden-column half ch
-        const int e = warp - 2, q = warp & 3, ch = e >> 2, et = threadIdx.x - 64;
         float* table = reinterpret_cast<float*>(c.base + LA::TAB);
         int* flag = reinterpret_cast<int*>(c.base + LA::FLAG);
         int local = 0;
         for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local) {
             const int cz = tile / (n_ht * n_tt), ht = (tile / n_tt) % n_ht, tt = tile % n_tt;
-            const int cs = a.c0 + cz, h0 = ht * A_BN, trow = tt * A_BM;
             const int b = local & 1;
-            float* tab = table + b * 2 * A_BN;
-            if (et < A_BN) {
-                const int h = h0 + et;
-                float s1 = 1.f, s2 = 1.f;
-                if (a.renorm_pending) {
-                    s1 = renorm_scale(a.n1[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 0, cs)[h]);
-                    s2 = renorm_scale(a.n2[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 1, cs)[h]);
-                }
-                tab[et] = s1;
-                tab[A_BN + et] = s2;
-                if (tt == 0) {
-                    ss_row(a, a.parity, 0, cs)[h] = 0.f;
-                    ss_row(a, a.parity, 1, cs)[h] = 0.f;
-                }
-            }
-            if (et == 0) flag[b] = mbar_wait(c.tfull(b, A_STAGES), (local >> 1) & 1, a.status) ? 1 : 0;
-            __syncwarp();
-            named_bar_sync(EPI_BAR, EPI_THREADS);
-            if (!flag[b]) break;
-            tc_fence_after();
-            const int row = q * 32 + lane;
-            const int t = trow + row;
-            float ct = 0.f, zi = 1.f;
-            if (t < a.Tp) {
-                const float ev = a.paper ? a.eta[(size_t)cs * a.win + a.tok0 + t]
-                                         : (a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr);
-                ct = -ev / (float)a.Tp;
-                if (a.zinv) zi = a.zinv[(size_t)cs * a.win + a.tok0 + t];
-            }
-            const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
-            bf16* dHrow = a.dH + ((size_t)cs * a.T + t) * a.d_hid + h0;
-            bf16* Arow = a.At + ((size_t)cs * a.T + t) * a.d_hid + h0;
-            float lsum = 0.f;
-#pragma unroll 1
-            for (int cc = 0; cc < 2; ++cc) {
-                const int c0 = ch * 64 + cc * 32;
-                float hv[32], rv[32];
-                tmem_ld32(lane_base + c0, hv);
-                tmem_ld32(lane_base + A_BN + c0, rv);
-                if (cc == 1) {
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(c.tempty(b, A_STAGES));
-                }
-                uint32_t pd[16], pa[16];
-#pragma unroll
-                for (int j = 0; j < 32; j += 2) {
-                    float dv[2], av2[2];
-#pragma unroll
-                    for (int u = 0; u < 2; ++u) {
-                        const float x = hv[j + u] * tab[c0 + j + u] * zi;
-                        const float r = rv[j + u] * tab[A_BN + c0 + j + u];
-                        const float sg = sigmoid_fast(x);
-                        const float av = x * sg;
-                        lsum = fmaf(av, r, lsum);
-                        dv[u] = ct * zi * r * (sg * (1.f + x * (1.f - sg)));
-                        av2[u] = ct * av;
-                    }
-                    pd[j / 2] = pack_bf16(dv[0], dv[1]);
-                    pa[j / 2] = pack_bf16(av2[0], av2[1]);
-                }
-#pragma unroll
-                for (int v = 0; v < 4; ++v) {
-                    *reinterpret_cast<uint4*>(dHrow + c0 + v * 8) =
-                        make_uint4(pd[4 * v], pd[4 * v + 1], pd[4 * v + 2], pd[4 * v + 3]);
-                    *reinterpret_cast<uint4*>(Arow + c0 + v * 8) =
-                        make_uint4(pa[4 * v], pa[4 * v + 1], pa[4 * v + 2], pa[4 * v + 3]);
-                }
-            }
-            if (a.loss) {
-                lsum = warp_sum(lsum);
-                if (lane == 0) atomicAdd(&a.loss[cz], -lsum / (float)a.Tp);
-            }
+            const uint32_t tempty = c.tempty(b, A_STAGES);
+            if (!phase_a_epilogue<A_BN>(a, tmem + b * 256, c.tfull(b, A_STAGES), (local >> 1) & 1, table + b * 2 * A_BN,
+                                  flag + b, cz, a.c0 + cz, ht * A_BN, tt * A_BM, tt == 0, nullptr, [&] {
+                                      if (lane == 0) mbar_arrive(tempty);
+                                  }))
+                break;
         }
     }
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, 512);
+}
+
+// ------------------------------------------------------------------ phase A on CTA pairs
+//
+// The same tile step on a cluster of two CTAs that share each tcgen05.mma
+// (cta_group::2): M = 256 tokens, 128 in each CTA, x N = 256 hidden units, whose W
+// rows are split between the pair (128 rows staged in each CTA).  Each CTA's TMEM
+// holds the H and R rows of its own tokens (256 + 256 columns: one accumulator
+// buffer).  A TMA tensor load costs the SM about the same whether its box has 64 or
+// 128 rows, and phase A is bounded by those loads: here an SM issues two 128-row
+// boxes per 64-deep k-block for a 128 x 256 accumulator, twice the work per load of
+// the one-CTA kernel's 128 x 128 tile.  Rank 0 of the pair issues the MMAs: both
+// CTAs' loads complete on rank 0's full barrier (a relay, with each CTA's loads on
+// its own barrier and one remote arrive per stage, measured 1.7x slower), each MMA
+// commit arrives on the empty and accumulator-full barriers of both CTAs, and all 16
+// epilogue warps of the pair release the accumulator on rank 0's tempty barrier.  The
+// epilogue stores dH and At through per-warp transpose buffers (coalesced rows).
+constexpr int P_BN = 256;
+constexpr int P_STAGES = 6;
+constexpr int P_A = A_BM * BK * 2;                  // 16 KB: this CTA's 128 token rows
+constexpr int P_STAGE = P_A + (P_BN / 2) * BK * 2;  // + 16 KB: this CTA's 128 W rows
+struct LP {
+    static constexpr int RING = P_STAGES * P_STAGE;
+    static constexpr int BARS = RING;  // full[S] empty[S] tfull[2] tempty[2]
+    static constexpr int NBARS = 2 * P_STAGES + 4;
+    static constexpr int SLOT = BARS + NBARS * 8;
+    static constexpr int FLAG = SLOT + 16;
+    static constexpr int TAB = FLAG + 16;               // scale tables of two consecutive tiles
+    static constexpr int STG = TAB + 4 * P_BN * 4;      // per epilogue warp: 32 x 64 B transpose buffer
+    static constexpr int END = STG + EPI_WARPS * 2048;
+    static constexpr int DYN = END + 1024;
+};
+static_assert(LP::DYN <= 227 * 1024, "shared memory budget");
+static_assert(LP::STG % 16 == 0, "staging buffers hold 16-byte pieces");
+
+// Spin for about `ns` nanoseconds (abort path: lets copies already issued land first).
+__device__ __forceinline__ void pause_ns(uint64_t ns) {
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < ns) __nanosleep(1000);
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmK,
+                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmW1,
+                       const __grid_constant__ CUtensorMap tmW2, const TcArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    Ctl c;
+    c.base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    c.bars = smem_u32(c.base + LP::BARS);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < P_STAGES; ++i) {
+            mbar_init(c.full(i), 1);
+            mbar_init(c.empty(i, P_STAGES), 1);
+        }
+        mbar_init(c.tfull(0, P_STAGES), 1);
+        mbar_init(c.tempty(0, P_STAGES), 2 * EPI_WARPS);
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc_pair(smem_u32(c.base + LP::SLOT), 512);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    cluster_sync();  // barriers of both CTAs initialised, TMEM of the pair allocated
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + LP::SLOT);
+    const int n_tp = a.T / (2 * A_BM), n_ht = a.d_hid / P_BN;
+    const int npairs = a.nc * n_ht * n_tp;
+    const int cluster = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
+    const int KB1 = a.d_in / BK, KB = KB1 + a.d_out / BK, half = (a.d_out / 2) / BK;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            tma_prefetch_map(&tmU);
+            tma_prefetch_map(&tmK);
+            tma_prefetch_map(&tmV);
+            tma_prefetch_map(&tmW1);
+            tma_prefetch_map(&tmW2);
+            uint32_t kc = 0;
+            bool ok = true;
+            for (int pt = cluster; pt < npairs && ok; pt += nclusters) {
+                const int cz = pt / (n_ht * n_tp), ht = (pt / n_tp) % n_ht, tp = pt % n_tp;
+                const int cs = a.c0 + cz, hrow = ht * P_BN + (int)rank * (P_BN / 2);
+                const int trow = tp * 2 * A_BM + (int)rank * A_BM;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % P_STAGES;
+                    if (kc >= P_STAGES && !mbar_wait(c.empty(s, P_STAGES), ((kc / P_STAGES) - 1) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    // both CTAs' loads complete on rank 0's full barrier
+                    const uint32_t sa = smem_u32(c.base + s * P_STAGE), sb = sa + P_A;
+                    const uint32_t fb = map_to_cta(c.full(s), 0);
+                    if (rank == 0) mbar_expect_tx(c.full(s), 2 * P_STAGE);
+                    if (kb < KB1) {
+                        tma_load_3d_pair(sa, &tmU, fb, kb * BK, a.u_row0 + trow, a.u_chain0 + cz);
+                        tma_load_3d_pair(sb, &tmW1, fb, kb * BK, hrow, cs);
+                    } else {
+                        const int k2 = kb - KB1;
+                        if (k2 < half)
+                            tma_load_3d_pair(sa, &tmK, fb, k2 * BK, a.y_row0 + trow, cz);
+                        else
+                            tma_load_3d_pair(sa, &tmV, fb, (k2 - half) * BK, a.y_row0 + trow, cz);
+                        tma_load_3d_pair(sb, &tmW2, fb, k2 * BK, hrow, cs);
+                    }
+                }
+            }
+            if (!ok) pause_ns(200000);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0 && rank == 0) {
+            const uint32_t idesc = idesc_bf16_f32(2 * A_BM, P_BN, false, false);
+            uint32_t kc = 0;
+            int local = 0;
+            bool ok = true;
+            for (int pt = cluster; pt < npairs && ok; pt += nclusters, ++local) {
+                // one accumulator buffer: wait until both CTAs' epilogues have read the last tile
+                if (local >= 1 && !mbar_wait(c.tempty(0, P_STAGES), (local - 1) & 1, a.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t dH = tmem, dR = tmem + P_BN;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % P_STAGES;
+                    if (!mbar_wait(c.full(s), (kc / P_STAGES) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(c.base + s * P_STAGE), sb = sa + P_A;
+                    const bool first = (kb == 0 || kb == KB1);
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k)
+                        umma_bf16_pair(kb < KB1 ? dH : dR, sdesc_sw128(sa + k * 32, 16),
+                                       sdesc_sw128(sb + k * 32, 16), idesc, (first && k == 0) ? 0u : 1u);
+                    umma_commit_pair(c.empty(s, P_STAGES), 0x3);
+                }
+                if (!ok) break;
+                umma_commit_pair(c.tfull(0, P_STAGES), 0x3);
+            }
+            if (!ok) pause_ns(200000);
+        }
+        __syncwarp();
+    } else {
+        float* table = reinterpret_cast<float*>(c.base + LP::TAB);
+        int* flag = reinterpret_cast<int*>(c.base + LP::FLAG);
+        const uint32_t tempty0 = map_to_cta(c.tempty(0, P_STAGES), 0);
+        int local = 0;
+        for (int pt = cluster; pt < npairs; pt += nclusters, ++local) {
+            const int cz = pt / (n_ht * n_tp), ht = (pt / n_tp) % n_ht, tp = pt % n_tp;
+            const int tt = tp * 2 + (int)rank;
+            // the scale table and flag alternate between tiles: a warp may start the next
+            // tile while another still reads this one's table
+            if (!phase_a_epilogue<P_BN>(a, tmem, c.tfull(0, P_STAGES), local & 1, table + (local & 1) * 2 * P_BN,
+                                        flag + (local & 1), cz, a.c0 + cz, ht * P_BN, tt * A_BM, tt == 0,
+                                        c.base + LP::STG + (warp - 2) * 2048, [&] {
+                                            if (lane == 0) mbar_arrive_remote(tempty0);
+                                        }))
+                break;
+        }
+    }
+    tc_fence_before();
+    cluster_sync();  // every MMA of the pair has completed and every TMEM read is done
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc_pair(tmem, 512);
 }
 
 // ------------------------------------------------------------------ phase B
@@ -640,6 +865,7 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
 std::once_flag g_attr_once;
 cudaError_t g_attr_err = cudaSuccess;
 int g_sms = 0;
+int g_pair_clusters = 0;  // co-resident CTA pairs of the pair kernel (0: use the one-CTA kernel)
 
 cudaError_t ensure_attrs() {
     std::call_once(g_attr_once, [] {
@@ -652,6 +878,26 @@ cudaError_t ensure_attrs() {
         if (g_attr_err == cudaSuccess)
             g_attr_err =
                 cudaFuncSetAttribute(tc_phase_b_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LayoutB::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err =
+                cudaFuncSetAttribute(tc_phase_a_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LP::DYN);
+        if (g_attr_err == cudaSuccess) {
+            cudaLaunchConfig_t cfg = {};
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = 2;
+            at[0].val.clusterDim.y = 1;
+            at[0].val.clusterDim.z = 1;
+            cfg.gridDim = dim3(2 * (g_sms / 2));
+            cfg.blockDim = dim3(THREADS);
+            cfg.dynamicSmemBytes = LP::DYN;
+            cfg.attrs = at;
+            cfg.numAttrs = 1;
+            if (cudaOccupancyMaxActiveClusters(&g_pair_clusters, tc_phase_a_pair_kernel, &cfg) != cudaSuccess) {
+                cudaGetLastError();
+                g_pair_clusters = 0;
+            }
+        }
     });
     return g_attr_err;
 }
@@ -663,9 +909,28 @@ cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputM
     cudaError_t e = ensure_attrs();
     if (e != cudaSuccess) return e;
     const TcArgs a = make_args(s, w);
+    const CUtensorMap& U = s.mode == 1 ? m.Ua : in.Xa;
+    if ((s.T / A_BM) % 2 == 0 && s.d_hid % P_BN == 0 && g_pair_clusters > 0) {
+        // CTA pairs over 256-token x 256-hidden tiles
+        const int npairs = w.nc * (s.T / (2 * A_BM)) * (s.d_hid / P_BN);
+        const int clusters = npairs < g_pair_clusters ? npairs : g_pair_clusters;
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 2;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(2 * clusters);
+        cfg.blockDim = dim3(THREADS);
+        cfg.dynamicSmemBytes = LP::DYN;
+        cfg.stream = st;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, tc_phase_a_pair_kernel, U, in.Ka, in.Va, m.W1b, m.W2b, a);
+    }
     const int ntiles = w.nc * (s.T / A_BM) * (s.d_hid / A_BN);
     const int grid = ntiles < g_sms ? ntiles : g_sms;
-    tc_phase_a_kernel<<<grid, THREADS, LA::DYN, st>>>(s.mode == 1 ? m.Ua : in.Xa, in.Ka, in.Va, m.W1b, m.W2b, a);
+    tc_phase_a_kernel<<<grid, THREADS, LA::DYN, st>>>(U, in.Ka, in.Va, m.W1b, m.W2b, a);
     return cudaGetLastError();
 }
 
