@@ -82,13 +82,23 @@ def kernel_work(wl, kind, chains=None):
     return flops, byts
 
 
+def kernel_source_sha(text, kind):
+    """sha256[:16] of one kernel's section of ttl_tc.cu (phase B: from its section banner to
+    make_args), so that the recorded counters stay valid while that kernel's source is unchanged."""
+    if kind != "phase_b":
+        return None
+    i = text.index("// ------------------------------------------------------------------ phase B")
+    j = text.index("TcArgs make_args(")
+    return hashlib.sha256(text[i:j].encode()).hexdigest()[:16]
+
+
 def ncu_traffic(kind, chains):
     """DRAM bytes per launch of `chains` chains from the committed ncu summary (scaled from the
     captured launch's chain count), if the kernel source is unchanged."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
     src = os.path.join(ROOT, "paper_2608_17616_gb300", "csrc", "ttl_tc.cu")
     try:
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        sha = kernel_source_sha(open(src).read(), kind)
         for line in open(path):
             if line.lstrip().startswith("#"):
                 continue
