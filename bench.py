@@ -419,6 +419,16 @@ def run_ours(args, wl):
                 "frac": d["tflops"] / tf_sus, "traffic": traffic, "peak_source": f"{peak_src} bf16_tflops_sustained"}
     if traffic_note.strip("; "):
         roof["traffic_note"] = traffic_note.strip("; ")
+    # the memory read: latency of one generate_kv call and its weight-streaming rate
+    gkv = None
+    t_read, n_read = ktimes["read"]
+    if n_read:
+        us = 1000 * t_read / n_read
+        el = 2 if wl.dtype == "bf16" else 4
+        byts = wl.chains * (wl.d_hid * (wl.d_in + wl.d_out) * 4            # fp32 W1, W2 streamed once
+                            + wl.Q * (wl.d_in + wl.d_out) * el)            # Xq in, K/V out
+        gkv = {"us": us, "bytes": byts, "gbs": byts / (us * 1e-6) / 1e9, "frac_of_hbm": byts / (us * 1e-6) / 1e9 / hbm,
+               "Q": wl.Q}
     if d["chains_per_launch"] < wl.chains:
         roof["note"] = ("launches of the two chain groups run concurrently on two streams; a launch's "
                         "duration includes the SMs and HBM bandwidth the other group's kernels take")
@@ -443,7 +453,7 @@ def run_ours(args, wl):
                 "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
                 "config": config_of(wl), "e2e": e2e, "gpu_launches": launches, "roofline": roof,
                 "cpu_baseline": cpu, "clocks": clk,
-                "tensor_util_of_burst_peak": tensor_util, "step_roofline": step_roof,
+                "tensor_util_of_burst_peak": tensor_util, "step_roofline": step_roof, "generate_kv": gkv,
                 "kernels": kern}
         print(json.dumps(line), flush=True)
     mone.mone_mem_free(h)
