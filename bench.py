@@ -425,8 +425,8 @@ def run_ours(args, wl):
     if n_read:
         us = 1000 * t_read / n_read
         el = 2 if wl.dtype == "bf16" else 4
-        byts = wl.chains * (wl.d_hid * (wl.d_in + wl.d_out) * 4            # fp32 W1, W2 streamed once
-                            + wl.Q * (wl.d_in + wl.d_out) * el)            # Xq in, K/V out
+        # weights streamed once: the bf16 operand copy on the bf16 path, the fp32 masters on the fp32 path
+        byts = wl.chains * (wl.d_hid * (wl.d_in + wl.d_out) * el + wl.Q * (wl.d_in + wl.d_out) * el)
         gkv = {"us": us, "bytes": byts, "gbs": byts / (us * 1e-6) / 1e9, "frac_of_hbm": byts / (us * 1e-6) / 1e9 / hbm,
                "Q": wl.Q}
     if d["chains_per_launch"] < wl.chains:

@@ -164,6 +164,7 @@ mone_status build_state_maps(mone_mem* m) {
     if (s.dtype != MONE_BF16) return MONE_OK;
     bool ok = encode_map_bf16_3d(&m->maps.W1b, s.W1b, s.d_in, s.d_hid, s.C, 64, 128) &&
               encode_map_bf16_3d(&m->maps.W2b, s.W2b, s.d_out, s.d_hid, s.C, 64, 128) &&
+              encode_map_bf16_3d(&m->maps.W2m, s.W2b, s.d_out, s.d_hid, s.C, 64, 64) &&
               encode_map_bf16_3d(&m->maps.dH, s.dHt, s.d_hid, s.T, s.C, 64, 64) &&
               encode_map_bf16_3d(&m->maps.At, s.Att, s.d_hid, s.T, s.C, 64, 64);
     if (ok && s.U)
@@ -523,8 +524,14 @@ mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out
         s.q_cap = Q;
     }
     const int L = m->cfg.n_layers;
+    if (s.dtype == MONE_BF16)
+        // tensor-core read: bf16 queries and hidden activations in the fp32 scratch buffers
+        return timed(m, K_READ, st, 3, [&] {
+            cudaError_t e = launch_query_transform(s, Xq, Q, s.Uq, true, st);
+            return e != cudaSuccess ? e : launch_read_tc(s, m->maps, s.Uq, s.Aq, Q, L, K_out, V_out, strides, st);
+        });
     return timed(m, K_READ, st, 4, [&] {
-        cudaError_t e = launch_query_transform(s, Xq, Q, st);
+        cudaError_t e = launch_query_transform(s, Xq, Q, s.Uq, false, st);
         return e != cudaSuccess ? e : launch_read(s, Q, L, K_out, V_out, strides, st);
     });
 }
@@ -546,7 +553,9 @@ mone_status mone_mem_generate_kv_noalloc(mone_mem* m, const void* Xq, int Q, voi
     }
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const int L = m->cfg.n_layers;
-    return timed(m, K_READ, st, 4, [&] { return launch_read_noalloc(s, Xq, Q, L, K_out, V_out, strides, st); });
+    const TcMaps* tc = s.dtype == MONE_BF16 ? &m->maps : nullptr;
+    return timed(m, K_READ, st, tc ? 3 : 4,
+                 [&] { return launch_read_noalloc(s, tc, Xq, Q, L, K_out, V_out, strides, st); });
 }
 
 mone_status mone_mem_free(mone_mem* m) {

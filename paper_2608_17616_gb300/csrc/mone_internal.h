@@ -60,7 +60,8 @@ struct SegWork {
 
 // ---- kernels in ttl_prepass.cu
 cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st);
-cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, cudaStream_t st);
+// Query transform of the read into U ([C][Q][d_in]: fp32, or bf16 when bf16_out).
+cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, void* U, bool bf16_out, cudaStream_t st);
 
 // ---- kernels in ttl_simt.cu (fp32 path, state upkeep, read path)
 cudaError_t launch_phase_a_f32(const DevState& s, const SegWork& w, cudaStream_t st);
@@ -74,8 +75,10 @@ cudaError_t launch_zero_f32(float* p, size_t n, cudaStream_t st);
 // Allocation-free read (mone_mem_generate_kv_noalloc): fixed device scratch of
 // kNoAllocScratchFloats floats, shared by every call on a device.
 constexpr size_t kNoAllocScratchFloats = (size_t(16) << 20) / sizeof(float);  // 16 MiB
-cudaError_t launch_read_noalloc(const DevState& s, const void* Xq, int Q, int n_layers, void* K_out, void* V_out,
-                                const long long* strides, cudaStream_t st);
+struct TcMaps;
+// tc: the handle's tensor maps on the bf16 path (tensor-core read), null on the fp32 path.
+cudaError_t launch_read_noalloc(const DevState& s, const TcMaps* tc, const void* Xq, int Q, int n_layers,
+                                void* K_out, void* V_out, const long long* strides, cudaStream_t st);
 
 // ---- kernels in ttl_tc.cu (bf16 tcgen05 path)
 struct TcMaps {
@@ -84,6 +87,7 @@ struct TcMaps {
     CUtensorMap Ua, Ub;          // scratch U: K-major {64,128} and MN {64,64}
     CUtensorMap W1s, W2s, M1s, M2s;  // fp32 state chunks {128 cols, 32 rows}, no swizzle
     CUtensorMap W1o, W2o;            // bf16 operand-copy chunks {128 cols, 32 rows}, no swizzle
+    CUtensorMap W2m;                 // bf16 W2 copy, MN-major boxes {64 outputs, 64 hidden} (memory read)
 };
 struct TcInputMaps {
     CUtensorMap Xa, Xb, Ka, Kb, Va, Vb;  // per call: K-major {64,128} (a) and MN {64,64} (b)
@@ -93,6 +97,10 @@ cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputM
 cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,
                               cudaStream_t st);
 int tc_kernels_per_segment();
+// Memory read on the tensor cores (bf16 path): Uq = transformed queries (bf16 [C][Q][d_in]),
+// Aq = bf16 scratch [C][Q][d_hid]; writes K/V (bf16) with the caller's strides.
+cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, void* Aq, int Q, int n_layers,
+                           void* K_out, void* V_out, const long long* strides, cudaStream_t st);
 
 // Tensor-map encoders (driver entry point, resolved at run time).  3-D maps over
 // [chains][rows][inner]; bf16 maps use 128-byte swizzle, the *_plain ones none.

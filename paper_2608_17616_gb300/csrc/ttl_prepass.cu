@@ -299,7 +299,7 @@ cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st)
     return s.dtype == 0 ? launch_one<float, float>(a, w.nc, st) : launch_one<bf16, bf16>(a, w.nc, st);
 }
 
-cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, cudaStream_t st) {
+cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, void* U, bool bf16_out, cudaStream_t st) {
     PrepassArgs a{};
     a.X = Xq;
     a.x_cstride = (long long)Q * s.d_in;
@@ -314,8 +314,9 @@ cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, cud
     a.query = 1;
     a.alpha = s.alpha;
     a.gamma = s.gamma;
-    a.U = s.Uq;
-    return s.dtype == 0 ? launch_one<float, float>(a, s.C, st) : launch_one<bf16, float>(a, s.C, st);
+    a.U = U;
+    if (s.dtype == 0) return launch_one<float, float>(a, s.C, st);
+    return bf16_out ? launch_one<bf16, bf16>(a, s.C, st) : launch_one<bf16, float>(a, s.C, st);
 }
 
 }  // namespace mone

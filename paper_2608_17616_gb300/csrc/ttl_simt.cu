@@ -426,19 +426,23 @@ cudaError_t noalloc_scratch(float** out) {
     return cudaSuccess;
 }
 
-cudaError_t launch_read_noalloc(const DevState& s, const void* Xq, int Q, int n_layers, void* K_out, void* V_out,
-                                const long long* strides, cudaStream_t st) {
+cudaError_t launch_read_noalloc(const DevState& s, const TcMaps* tc, const void* Xq, int Q, int n_layers,
+                                void* K_out, void* V_out, const long long* strides, cudaStream_t st) {
     float* base = nullptr;
     cudaError_t e = noalloc_scratch(&base);
     if (e != cudaSuccess) return e;
     // the same kernels as the allocating read, pointed at the fixed scratch; every
-    // element of the three regions is written before it is read, so nothing needs
-    // clearing between calls
+    // element of the regions is written before it is read, so nothing needs clearing
+    // between calls
     DevState t = s;
     t.Uq = base;
     t.Aq = t.Uq + (size_t)s.C * Q * s.d_in;
     t.Oq = t.Aq + (size_t)s.C * Q * s.d_hid;
-    e = launch_query_transform(t, Xq, Q, st);
+    if (tc) {
+        e = launch_query_transform(t, Xq, Q, t.Uq, true, st);
+        return e != cudaSuccess ? e : launch_read_tc(t, *tc, t.Uq, t.Aq, Q, n_layers, K_out, V_out, strides, st);
+    }
+    e = launch_query_transform(t, Xq, Q, t.Uq, false, st);
     return e != cudaSuccess ? e : launch_read(t, Q, n_layers, K_out, V_out, strides, st);
 }
 

@@ -139,12 +139,12 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 // `release` is called by every epilogue warp once its last TMEM read of the tile is
 // done.  Returns false if the accumulator wait timed out.
 // Store a warp's 32 rows x 32 bf16 columns (lane = row, `pk` = its row packed in pairs)
-// to rows row0 .. row0 + 31 of a row-major matrix with `ld` elements per row.  The
+// to rows row0 .. row0 + min(32, nrows) - 1 of a row-major matrix with `ld` elements per row.  The
 // chunk is transposed through the warp's 2 KB staging buffer (16-byte pieces XOR-
 // swizzled per row pair, conflict-free both ways) so that each global store
 // instruction writes 8 rows x 64 contiguous bytes instead of 32 scattered 16-byte pieces.
 __device__ __forceinline__ void store_rows_coalesced(uint8_t* stg, const uint32_t (&pk)[16], bf16* row0, int ld,
-                                                     int lane) {
+                                                     int lane, int nrows = 32) {
 #pragma unroll
     for (int p = 0; p < 4; ++p)
         *reinterpret_cast<uint4*>(stg + lane * 64 + ((p ^ ((lane >> 1) & 3)) * 16)) =
@@ -155,7 +155,7 @@ __device__ __forceinline__ void store_rows_coalesced(uint8_t* stg, const uint32_
     for (int k = 0; k < 4; ++k) {
         const int r = 8 * k + (lane >> 2);
         const uint4 v = *reinterpret_cast<const uint4*>(stg + r * 64 + ((i ^ ((r >> 1) & 3)) * 16));
-        *reinterpret_cast<uint4*>(row0 + (size_t)r * ld + i * 8) = v;
+        if (r < nrows) *reinterpret_cast<uint4*>(row0 + (size_t)r * ld + i * 8) = v;
     }
     __syncwarp();
 }
@@ -862,6 +862,178 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
     return a;
 }
 
+// ------------------------------------------------------------------ memory read (Eq. 4)
+//
+// The read of generate_kv on the bf16 path, on the tensor cores, in two kernels:
+//   hidden:  A_q = SiLU(U_q W1^T)    tile = (128 queries, 128 hidden units, chain), K = d_in
+//   out:     O = A_q W2, then per output head h of width hd: g_h o_h / sqrt(mean(o_h^2) + eps)
+//            written into the caller's K / V layout   tile = (128 queries, 128 outputs, chain), K = d_hid
+// One tile per CTA: warp 0 streams the query rows and the bf16 weight copy with TMA,
+// warp 1 issues tcgen05.mma into a 128-column TMEM accumulator, warps 2..5 (one per TMEM
+// lane quarter, lane = query) run the epilogue.  Each weight tile is read by ceil(Q/128)
+// CTAs; query rows >= Q arrive as TMA zero fill and are never stored.  W2 is [hidden][out],
+// so in the out kernel the weight operand is MN-major (64-column boxes, as in phase B).
+constexpr int R_STAGES = 4;
+constexpr int R_STAGE = 2 * 128 * BK * 2;  // 32 KB: 128 query rows + 128 weight rows / columns
+constexpr int R_THREADS = 6 * 32;
+constexpr uint32_t R_EPI_BAR = 1;
+struct LR {
+    static constexpr int RING = R_STAGES * R_STAGE;
+    static constexpr int BARS = RING;  // full[S] empty[S] tfull
+    static constexpr int NBARS = 2 * R_STAGES + 1;
+    static constexpr int SLOT = BARS + (NBARS * 8 + 15) / 16 * 16;
+    static constexpr int FLAG = SLOT + 16;
+    static constexpr int STG = FLAG + 16;  // 4 epilogue warps x 2 KB transpose buffers
+    static constexpr int END = STG + 4 * 2048;
+    static constexpr int DYN = END + 1024;
+};
+static_assert(LR::STG % 16 == 0, "staging buffers hold 16-byte pieces");
+
+struct ReadArgs {
+    int Q, d_in, d_hid, d_out, n_kv, L;
+    float eps;
+    const float* gate;     // [C][2 n_kv] per-head gates, or null (gate 1)
+    bf16* Aq;              // [C][Q][d_hid]
+    bf16 *Kout, *Vout;     // caller's K / V, element strides s0 (context), s1 (layer), s2 (head), s3 (query)
+    long long s0, s1, s2, s3;
+    int* status;
+};
+
+// MODE 0: hidden kernel.  MODE 64 / 128: out kernel with heads of that width.
+template <int MODE>
+__global__ void __launch_bounds__(R_THREADS, 1)
+tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const ReadArgs a) {
+    constexpr bool OUT = MODE != 0;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const uint32_t bars = smem_u32(base + LR::BARS);
+    auto full = [&](int s) { return bars + 8 * s; };
+    auto empty = [&](int s) { return bars + 8 * (R_STAGES + s); };
+    const uint32_t tfull = bars + 8 * (2 * R_STAGES);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < R_STAGES; ++s) {
+            mbar_init(full(s), 1);
+            mbar_init(empty(s), 1);
+        }
+        mbar_init(tfull, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(base + LR::SLOT), 128);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<uint32_t*>(base + LR::SLOT);
+    const int q0 = blockIdx.x * 128, n0 = blockIdx.y * 128, c = blockIdx.z;
+    const int KB = (OUT ? a.d_hid : a.d_in) / BK;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            tma_prefetch_map(&tmA);
+            tma_prefetch_map(&tmB);
+            for (int kb = 0; kb < KB; ++kb) {
+                const int s = kb % R_STAGES;
+                if (kb >= R_STAGES && !mbar_wait(empty(s), ((kb / R_STAGES) - 1) & 1, a.status)) break;
+                const uint32_t sa = smem_u32(base + s * R_STAGE), sb = sa + 128 * BK * 2, fb = full(s);
+                mbar_expect_tx(fb, R_STAGE);
+                tma_load_3d(sa, &tmA, fb, kb * BK, q0, c);
+                if (OUT) {
+                    tma_load_3d(sb, &tmB, fb, n0, kb * BK, c);
+                    tma_load_3d(sb + BOX, &tmB, fb, n0 + 64, kb * BK, c);
+                } else {
+                    tma_load_3d(sb, &tmB, fb, kb * BK, n0, c);
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, 128, false, OUT);
+            bool ok = true;
+            for (int kb = 0; kb < KB; ++kb) {
+                const int s = kb % R_STAGES;
+                if (!mbar_wait(full(s), (kb / R_STAGES) & 1, a.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sa = smem_u32(base + s * R_STAGE), sb = sa + 128 * BK * 2;
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k)
+                    umma_bf16(tmem, sdesc_sw128(sa + k * 32, 16),
+                              OUT ? sdesc_sw128(sb + k * 16 * 128, BOX) : sdesc_sw128(sb + k * 32, 16), idesc,
+                              (kb == 0 && k == 0) ? 0u : 1u);
+                umma_commit(empty(s));
+            }
+            if (ok) umma_commit(tfull);
+        }
+        __syncwarp();
+    } else {
+        const int q = warp & 3;  // TMEM lane quarter of this warp
+        int* flag = reinterpret_cast<int*>(base + LR::FLAG);
+        if (threadIdx.x == 64) *flag = mbar_wait(tfull, 0, a.status) ? 1 : 0;
+        __syncwarp();
+        named_bar_sync(R_EPI_BAR, 128);
+        if (*flag) {
+            tc_fence_after();
+            const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+            const int qw = q0 + q * 32;  // first query row of this warp
+            if constexpr (!OUT) {
+                uint8_t* stg = base + LR::STG + (warp - 2) * 2048;
+                bf16* row0 = a.Aq + ((size_t)c * a.Q + qw) * a.d_hid + n0;
+#pragma unroll 1
+                for (int cc = 0; cc < 4; ++cc) {
+                    float hv[32];
+                    tmem_ld32(lane_base + cc * 32, hv);
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                        pk[j] = pack_bf16(hv[2 * j] * sigmoidf_(hv[2 * j]), hv[2 * j + 1] * sigmoidf_(hv[2 * j + 1]));
+                    store_rows_coalesced(stg, pk, row0 + cc * 32, a.d_hid, lane, a.Q - qw);
+                }
+            } else {
+                constexpr int HD = MODE;
+                const int qi = qw + lane;
+                const int nh = 2 * a.n_kv;
+#pragma unroll 1
+                for (int hh = 0; hh < 128 / HD; ++hh) {
+                    float v[HD];
+#pragma unroll
+                    for (int cc = 0; cc < HD / 32; ++cc)
+                        tmem_ld32(lane_base + hh * HD + cc * 32, *reinterpret_cast<float(*)[32]>(v + cc * 32));
+                    float ss = 0.f;
+#pragma unroll
+                    for (int i = 0; i < HD; ++i) ss = fmaf(v[i], v[i], ss);
+                    const int head = n0 / HD + hh;
+                    const float g = a.gate ? a.gate[(size_t)c * nh + head] : 1.f;
+                    const float sc = g / sqrtf(ss / (float)HD + a.eps);
+                    if (qi < a.Q) {
+                        const int kvh = head < a.n_kv ? head : head - a.n_kv;
+                        bf16* out = (head < a.n_kv ? a.Kout : a.Vout) + (long long)(c / a.L) * a.s0 +
+                                    (long long)(c % a.L) * a.s1 + (long long)kvh * a.s2 + (long long)qi * a.s3;
+                        if ((reinterpret_cast<uintptr_t>(out) & 15u) == 0) {
+#pragma unroll
+                            for (int i = 0; i < HD; i += 8)
+                                *reinterpret_cast<uint4*>(out + i) =
+                                    make_uint4(pack_bf16(v[i] * sc, v[i + 1] * sc), pack_bf16(v[i + 2] * sc, v[i + 3] * sc),
+                                               pack_bf16(v[i + 4] * sc, v[i + 5] * sc), pack_bf16(v[i + 6] * sc, v[i + 7] * sc));
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < HD; ++i) out[i] = __float2bfloat16_rn(v[i] * sc);
+                        }
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, 128);
+}
+
 std::once_flag g_attr_once;
 cudaError_t g_attr_err = cudaSuccess;
 int g_sms = 0;
@@ -881,6 +1053,12 @@ cudaError_t ensure_attrs() {
         if (g_attr_err == cudaSuccess)
             g_attr_err =
                 cudaFuncSetAttribute(tc_phase_a_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LP::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err = cudaFuncSetAttribute(tc_read_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err = cudaFuncSetAttribute(tc_read_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err = cudaFuncSetAttribute(tc_read_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
         if (g_attr_err == cudaSuccess) {
             cudaLaunchConfig_t cfg = {};
             cudaLaunchAttribute at[1];
@@ -947,6 +1125,33 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
 }
 
 int tc_kernels_per_segment() { return 2; }
+
+cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, void* Aq, int Q, int n_layers,
+                           void* K_out, void* V_out, const long long* strides, cudaStream_t st) {
+    cudaError_t e = ensure_attrs();
+    if (e != cudaSuccess) return e;
+    if (s.hd != 64 && s.hd != 128) return cudaErrorInvalidValue;
+    CUtensorMap mu, ma;
+    if (!encode_map_bf16_3d(&mu, Uq, s.d_in, Q, s.C, 64, 128) || !encode_map_bf16_3d(&ma, Aq, s.d_hid, Q, s.C, 64, 128))
+        return cudaErrorInvalidValue;
+    ReadArgs a{};
+    a.Q = Q; a.d_in = s.d_in; a.d_hid = s.d_hid; a.d_out = s.d_out; a.n_kv = s.n_kv; a.L = n_layers;
+    a.eps = s.rms_eps;
+    a.gate = s.gate;
+    a.Aq = static_cast<bf16*>(Aq);
+    a.Kout = static_cast<bf16*>(K_out);
+    a.Vout = static_cast<bf16*>(V_out);
+    a.s0 = strides[0]; a.s1 = strides[1]; a.s2 = strides[2]; a.s3 = strides[3];
+    a.status = s.status;
+    const int nq = (Q + 127) / 128;
+    tc_read_kernel<0><<<dim3(nq, s.d_hid / 128, s.C), R_THREADS, LR::DYN, st>>>(mu, m.W1b, a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (s.hd == 64)
+        tc_read_kernel<64><<<dim3(nq, s.d_out / 128, s.C), R_THREADS, LR::DYN, st>>>(ma, m.W2m, a);
+    else
+        tc_read_kernel<128><<<dim3(nq, s.d_out / 128, s.C), R_THREADS, LR::DYN, st>>>(ma, m.W2m, a);
+    return cudaGetLastError();
+}
 
 // ------------------------------------------------------------------ tensor maps
 
