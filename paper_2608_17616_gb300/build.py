@@ -7,6 +7,7 @@ C-ABI symbol checks run there) and needs nothing but the driver on a GPU machine.
 from __future__ import annotations
 
 import concurrent.futures as cf
+import hashlib
 import os
 import shutil
 import subprocess
@@ -33,11 +34,31 @@ def _flags(extra=()):
                    "-I", CSRC, *extra]
 
 
-def _newer(target: str, deps) -> bool:
-    if not os.path.exists(target):
+def _digest(paths, extra=()) -> str:
+    """sha256 over file contents and strings: build outputs are reused only when this matches
+    the stamp written beside them (content, not modification times, which need not be
+    comparable between the machine that edited the sources and the one that builds)."""
+    h = hashlib.sha256()
+    for p in sorted(paths):
+        h.update(p.encode())
+        with open(p, "rb") as f:
+            h.update(f.read())
+    for e in extra:
+        h.update(str(e).encode())
+    return h.hexdigest()
+
+
+def _fresh(target: str, digest: str) -> bool:
+    try:
+        with open(target + ".sha") as f:
+            return os.path.exists(target) and f.read().strip() == digest
+    except OSError:
         return False
-    t = os.path.getmtime(target)
-    return all(os.path.getmtime(d) <= t for d in deps)
+
+
+def _stamp(target: str, digest: str) -> None:
+    with open(target + ".sha", "w") as f:
+        f.write(digest)
 
 
 def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False) -> str:
@@ -47,31 +68,36 @@ def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False) 
     cc = nvcc()
     extra = ["-Xptxas", "-v"] if ptxas_info else []
 
+    machine = os.uname().machine
+
     def compile_one(src):
         s = os.path.join(CSRC, src)
         o = os.path.join(BUILD, src.replace(".cu", ".o"))
-        if not force and not ptxas_info and _newer(o, [s, *headers]):
-            return o, ""
         cmd = [cc, *_flags(extra), "-c", s, "-o", o]
+        digest = _digest([s, *headers], [machine, *cmd])
+        if not force and not ptxas_info and _fresh(o, digest):
+            return o, "", digest
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
-        return o, r.stderr
+        _stamp(o, digest)
+        return o, r.stderr, digest
 
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         results = list(ex.map(compile_one, SOURCES))
-    objs = [o for o, _ in results]
+    objs = [o for o, _, _ in results]
     if verbose or ptxas_info:
-        for _, log in results:
+        for _, log, _ in results:
             if log:
                 sys.stderr.write(log)
-    if force or ptxas_info or not _newer(LIB, objs):
-        tmp = LIB + ".tmp"
-        cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs, "-cudart", "static", "-Xcompiler", "-fPIC"]
+    cmd = [cc, *ARCH, "-shared", "-o", LIB + ".tmp", *objs, "-cudart", "static", "-Xcompiler", "-fPIC"]
+    digest = _digest([], [machine, *cmd, *[d for _, _, d in results]])
+    if force or ptxas_info or not _fresh(LIB, digest):
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-        os.replace(tmp, LIB)
+        os.replace(LIB + ".tmp", LIB)
+        _stamp(LIB, digest)
     return LIB
 
 

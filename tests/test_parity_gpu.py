@@ -212,6 +212,24 @@ def test_bf16_chain_groups_match_one_chain_handles(mode):
     run.close()
 
 
+@pytest.mark.parametrize("Q,hd", [(200, 64), (131, 128)])
+def test_bf16_generate_kv_several_query_tiles(Q, hd):
+    """The tensor-core read takes queries 128 at a time: Q > 128 spans several tiles and a
+    ragged last one (rows beyond Q are never written); hd = 128 puts one head per tile."""
+    wl = small(wk.PAPER, n_ctx=1, n_layers=2, d_out=512, N=300, hd=hd, Q=Q)
+    run = GpuRun(wl)
+    run.ttl_context()
+    W1, W2, _, _ = run.state()
+    Xq = wk.query_inputs(wl, "cuda")
+    assert Xq.shape[2] == Q
+    Kg, Vg = run.generate_kv(Xq)
+    for c in range(wl.chains):
+        st, _ = oracle_chain(run, c)
+        Ko, Vo = oracle_read(run, st, c, Xq)
+        assert rel_fro(Kg[0, c].float(), Ko) <= BF16_TOL and rel_fro(Vg[0, c].float(), Vo) <= BF16_TOL
+    run.close()
+
+
 def test_generate_kv_into_strided_cache_and_reuse():
     wl = small(wk.PAPER, N=512)
     run = GpuRun(wl)
