@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define MONE_ABI_VERSION 1
+#define MONE_ABI_VERSION 2
 
 typedef struct mone_mem mone_mem; /* opaque; created by mone_mem_init */
 
@@ -55,6 +55,7 @@ typedef enum {
 
 enum { MONE_FP32 = 0, MONE_BF16 = 1 };  /* dtype of X, K, V, Xq and generated K/V */
 enum { MONE_PLAIN = 0, MONE_PAPER = 1 };
+enum { MONE_LOSS_DOT = 0, MONE_LOSS_MSE = 1 };  /* per-token loss of a segment step */
 
 /*
  * Configuration, fixed for the life of a handle.
@@ -68,7 +69,11 @@ enum { MONE_PLAIN = 0, MONE_PAPER = 1 };
  *     W_s = W_{s-1} - mu_s (Eq. 8); then every row of W1 and of W2 is rescaled to
  *     its L2 norm in W_0 ("channel-wise L2 renormalisation").
  * The gradient step on a segment of T' tokens is g = sum_j (eta_j / T') grad l_j
- * with l_j = -y_j . M(u_j) (Eq. 7, Eq. 10).
+ * with l_j = -y_j . M(u_j) (loss MONE_LOSS_DOT: Eq. 7, Eq. 10).  loss MONE_LOSS_MSE
+ * replaces l_j by 1/2 |M(u_j) - y_j|^2 (the squared-error, delta-rule form of the
+ * same step; its gradient needs M(u_j) at the segment's starting weights, computed
+ * by two more kernels per segment).  MONE_LOSS_MSE is supported on the BF16 path;
+ * on FP32 mone_mem_init returns MONE_ERR_UNSUPPORTED.
  *
  * Supported shapes: FP32: d_in, d_hid, d_out multiples of 64, seg_T multiple of 64.
  *   BF16: d_in, d_out/2, seg_T multiples of 128; d_hid a multiple of 256.  Both: head_dim in {64,128},
@@ -83,6 +88,7 @@ typedef struct {
     int mode;      /* MONE_PLAIN | MONE_PAPER */
     float lr;      /* plain-mode learning rate */
     float rms_eps; /* epsilon of the read-side RMSNorm (Sec. 3.2 after Eq. 4); e.g. 1e-6 */
+    int loss;      /* MONE_LOSS_DOT (Eq. 7) | MONE_LOSS_MSE */
 } mone_config;
 
 /*
@@ -197,7 +203,8 @@ long long mone_mem_launch_count(const mone_mem* m);
  * kind, the summed device milliseconds and the launch count since timing was
  * last enabled.  Kinds: 0 input prepass, 1 phase A (forward + fused backward
  * epilogue), 2 phase B (gradient + fused update), 3 finalize (renorm apply /
- * operand refresh), 4 memory read.  Errors: INVALID_ARG, CUDA.
+ * operand refresh), 4 memory read, 5 squared-error pre-pass (M(u) and the residual
+ * target, MONE_LOSS_MSE only).  Errors: INVALID_ARG, CUDA.
  */
 mone_status mone_mem_set_timing(mone_mem* m, int enable);
 mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches);

@@ -18,6 +18,7 @@ LIB_PATH = os.path.join(_PKG, "libmone.so")
 
 MONE_FP32, MONE_BF16 = 0, 1
 MONE_PLAIN, MONE_PAPER = 0, 1
+MONE_LOSS_DOT, MONE_LOSS_MSE = 0, 1
 
 STATUS = {0: "MONE_OK", 1: "MONE_ERR_INVALID_ARG", 2: "MONE_ERR_UNSUPPORTED_SHAPE", 3: "MONE_ERR_OOM",
           4: "MONE_ERR_CUDA", 5: "MONE_ERR_TIMEOUT", 6: "MONE_ERR_NONFINITE", 7: "MONE_ERR_UNSUPPORTED"}
@@ -28,7 +29,7 @@ EXPORTS = ("mone_mem_init", "mone_ttl_segment", "mone_ttl_context", "mone_mem_ge
            "mone_status_string", "mone_abi_version", "mone_mem_set_timing", "mone_mem_kernel_time",
            "mone_last_error", "mone_mem_generate_kv_noalloc")
 
-KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read")
+KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read", "mse")
 
 
 class MoneError(RuntimeError):
@@ -41,7 +42,7 @@ class mone_config(ctypes.Structure):
     _fields_ = [("n_ctx", ctypes.c_int), ("n_layers", ctypes.c_int), ("d_in", ctypes.c_int),
                 ("d_hid", ctypes.c_int), ("d_out", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("seg_T", ctypes.c_int), ("dtype", ctypes.c_int),
-                ("mode", ctypes.c_int), ("lr", ctypes.c_float), ("rms_eps", ctypes.c_float)]
+                ("mode", ctypes.c_int), ("lr", ctypes.c_float), ("rms_eps", ctypes.c_float), ("loss", ctypes.c_int)]
 
 
 class mone_meta(ctypes.Structure):
@@ -112,8 +113,9 @@ def _check(fn: str, rc: int):
 
 
 def make_config(n_ctx, n_layers, d_in, d_hid, d_out, n_kv_heads, head_dim, seg_T, dtype, mode, lr,
-                rms_eps=1e-6) -> mone_config:
-    return mone_config(n_ctx, n_layers, d_in, d_hid, d_out, n_kv_heads, head_dim, seg_T, dtype, mode, lr, rms_eps)
+                rms_eps=1e-6, loss=0) -> mone_config:
+    return mone_config(n_ctx, n_layers, d_in, d_hid, d_out, n_kv_heads, head_dim, seg_T, dtype, mode, lr, rms_eps,
+                       loss)
 
 
 def make_meta(meta: Optional[dict]) -> Optional[mone_meta]:

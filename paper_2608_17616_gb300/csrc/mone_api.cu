@@ -25,8 +25,8 @@ struct KernelTiming {
     };
     std::vector<cudaEvent_t> pool;
     std::vector<Pending> pending;
-    double ms[5] = {0, 0, 0, 0, 0};
-    long long n[5] = {0, 0, 0, 0, 0};
+    double ms[6] = {0, 0, 0, 0, 0, 0};
+    long long n[6] = {0, 0, 0, 0, 0, 0};
 
     cudaEvent_t get() {
         if (!pool.empty()) {
@@ -91,6 +91,8 @@ mone_status validate_config(const mone_config* c) {
         return MONE_ERR_INVALID_ARG;
     if (c->dtype != MONE_FP32 && c->dtype != MONE_BF16) return MONE_ERR_INVALID_ARG;
     if (c->mode != MONE_PLAIN && c->mode != MONE_PAPER) return MONE_ERR_INVALID_ARG;
+    if (c->loss != MONE_LOSS_DOT && c->loss != MONE_LOSS_MSE) return MONE_ERR_INVALID_ARG;
+    if (c->loss == MONE_LOSS_MSE && c->dtype != MONE_BF16) return MONE_ERR_UNSUPPORTED;
     if (!std::isfinite(c->lr) || !(c->rms_eps >= 0.0f) || !std::isfinite(c->rms_eps)) return MONE_ERR_INVALID_ARG;
     if (c->head_dim != 64 && c->head_dim != 128) return MONE_ERR_UNSUPPORTED_SHAPE;
     if (c->d_out != 2 * c->n_kv_heads * c->head_dim) return MONE_ERR_UNSUPPORTED_SHAPE;
@@ -132,7 +134,7 @@ mone_status dalloc(T** p, size_t n) {
 void free_state(DevState& s) {
     void* ptrs[] = {s.W1, s.W2, s.mu1, s.mu2, s.W1b, s.W2b, s.n1, s.n2, s.sumsq, s.status, s.alpha, s.gamma,
                     s.w_eta, s.b_eta, s.w_beta, s.b_beta, s.gate, s.U, s.eta, s.dbeta, s.zinv, s.dHt, s.Att, s.Uq, s.Aq,
-                    s.Oq};
+                    s.Oq, s.Amse, s.Kres, s.Vres};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     std::memset(&s, 0, sizeof(s));
@@ -167,6 +169,7 @@ mone_status build_state_maps(mone_mem* m) {
               encode_map_bf16_3d(&m->maps.W2m, s.W2b, s.d_out, s.d_hid, s.C, 64, 64) &&
               encode_map_bf16_3d(&m->maps.dH, s.dHt, s.d_hid, s.T, s.C, 64, 64) &&
               encode_map_bf16_3d(&m->maps.At, s.Att, s.d_hid, s.T, s.C, 64, 64);
+    if (ok && s.Amse) ok = encode_map_bf16_3d(&m->maps.Amse, s.Amse, s.d_hid, s.T, s.C, 64, 128);
     if (ok && s.U)
         ok = encode_map_bf16_3d(&m->maps.Ua, s.U, s.d_in, s.win_rows, s.C, 64, 128) &&
              encode_map_bf16_3d(&m->maps.Ub, s.U, s.d_in, s.win_rows, s.C, 64, 64);
@@ -195,7 +198,7 @@ mone_status build_input_maps(const DevState& s, TcInputMaps* in, const void* X, 
     return ok ? MONE_OK : MONE_ERR_CUDA;
 }
 
-enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4 };
+enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4, K_MSE = 5 };
 
 // Launch through `fn` (which returns a cudaError_t), bracketed by timing events
 // when timing is on; `kernels` is the number of device kernels `fn` launches.
@@ -229,8 +232,8 @@ mone_status timed(mone_mem* m, int kind, cudaStream_t st, int kernels, F&& fn) {
 // between launches.  The side stream forks from the caller's stream before the
 // first phase launch and joins it before every input-transform window and at
 // the end, so the call stays ordered on the caller's stream.
-mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, int G, const SegWork& w, long long N,
-                             cudaStream_t st, bool& forked) {
+mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInputMaps* rin, int G, const SegWork& w,
+                             long long N, cudaStream_t st, bool& forked) {
     DevState& s = m->s;
     const cudaStream_t gs[2] = {st, m->side};
     auto join = [&]() -> mone_status {
@@ -272,7 +275,16 @@ mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, int G, 
             x.parity = (int)(i & 1);
             x.renorm_pending = (s.renorm && i > 0) ? 1 : 0;
             x.u_off = u_off;
-            if (s.dtype == MONE_BF16) {
+            if (s.dtype == MONE_BF16 && s.loss == MONE_LOSS_MSE) {
+                // squared error: residual targets y - M(u) at the starting weights, then the
+                // same two phases with them in place of y (dL/dO = eta (M(u) - y) / T')
+                MONE_TRY(timed(m, K_MSE, sg, 2, [&] { return launch_mse_tc(s, m->maps, gin[g], x, sg); }));
+                SegWork xr = x;
+                xr.y_scratch = 1;
+                xr.loss = nullptr;  // the pre-pass accumulated the squared-error loss
+                MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_phase_a_tc(s, m->maps, rin[g], xr, sg); }));
+                MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_phase_b_tc(s, m->maps, rin[g], xr, sg); }));
+            } else if (s.dtype == MONE_BF16) {
                 MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_phase_a_tc(s, m->maps, gin[g], x, sg); }));
                 MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_phase_b_tc(s, m->maps, gin[g], x, sg); }));
             } else {
@@ -293,7 +305,7 @@ mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
     DevState& s = m->s;
     const int G = (m->side && w.nc >= 2) ? 2 : 1;
     SegWork gw[2];
-    TcInputMaps gin[2];
+    TcInputMaps gin[2], rin[2];
     const size_t el = elsize(s.dtype);
     for (int g = 0, off = 0; g < G; ++g) {
         const int n = w.nc / G + (g < w.nc % G ? 1 : 0);
@@ -306,12 +318,22 @@ mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
         if (w.eta_in) gw[g].eta_in = w.eta_in + (size_t)off * w.eta_cstride;
         if (w.loss) gw[g].loss = w.loss + off;
         std::memset(&gin[g], 0, sizeof(TcInputMaps));
+        std::memset(&rin[g], 0, sizeof(TcInputMaps));
         if (s.dtype == MONE_BF16)
             MONE_TRY(build_input_maps(s, &gin[g], gw[g].X, gw[g].K, gw[g].V, w.n_rows, n));
+        if (s.dtype == MONE_BF16 && s.loss == MONE_LOSS_MSE) {
+            // residual targets of this group's chains: [C][T][d_out/2] scratch, rows from 0
+            const size_t o = (size_t)gw[g].c0 * s.T * (s.d_out / 2);
+            MONE_TRY(build_input_maps(s, &rin[g], gw[g].X, s.Kres + o, s.Vres + o, s.T, n));
+            if (s.mode == MONE_PLAIN) {  // U stays the caller's X
+                rin[g].Xa = gin[g].Xa;
+                rin[g].Xb = gin[g].Xb;
+            }
+        }
         off += n;
     }
     bool forked = false;
-    const mone_status rc = run_segment_loop(m, gw, gin, G, w, N, st, forked);
+    const mone_status rc = run_segment_loop(m, gw, gin, rin, G, w, N, st, forked);
     if (forked) {
         // error after the fork: still order the side stream's work before the caller's stream
         cudaEventRecord(m->ev_join, m->side);
@@ -368,6 +390,7 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
     s.dtype = cfg->dtype; s.mode = cfg->mode;
     s.momentum = cfg->mode == MONE_PAPER; s.renorm = cfg->mode == MONE_PAPER;
     s.lr = cfg->lr; s.rms_eps = cfg->rms_eps;
+    s.loss = cfg->loss;
     if (s.mode == MONE_PAPER) {
         // the input transform covers a window of whole segments whose scratch stays within ~2 GiB
         const size_t row_bytes = (size_t)s.C * s.d_in * elsize(s.dtype);
@@ -387,6 +410,11 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
     if (s.dtype == MONE_BF16) {
         step(dalloc(&s.W1b, n1));
         step(dalloc(&s.W2b, n2));
+        if (s.loss == MONE_LOSS_MSE) {
+            step(dalloc(&s.Amse, C * s.T * s.d_hid));
+            step(dalloc(&s.Kres, C * s.T * (s.d_out / 2)));
+            step(dalloc(&s.Vres, C * s.T * (s.d_out / 2)));
+        }
     }
     step(dalloc(&s.n1, C * s.d_hid));
     step(dalloc(&s.n2, C * s.d_hid));
@@ -638,7 +666,7 @@ mone_status mone_mem_set_timing(mone_mem* m, int enable) {
 }
 
 mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches) {
-    if (!is_live(m) || kind < 0 || kind > 4 || !ms || !launches) return MONE_ERR_INVALID_ARG;
+    if (!is_live(m) || kind < 0 || kind > 5 || !ms || !launches) return MONE_ERR_INVALID_ARG;
     *ms = 0;
     *launches = 0;
     if (!m->timing) return MONE_OK;

@@ -16,7 +16,7 @@ enum : int { DEV_TIMEOUT = 1, DEV_NONFINITE = 2 };
 
 // Device-resident state of all chains (see mone_mem_init).
 struct DevState {
-    int C, d_in, d_hid, d_out, n_kv, hd, T, dtype, mode, momentum, renorm;
+    int C, d_in, d_hid, d_out, n_kv, hd, T, dtype, mode, momentum, renorm, loss;
     float lr, rms_eps;
     float *W1, *W2, *mu1, *mu2;   // fp32 masters [C][d_hid][d_in|d_out]; mu only with momentum
     bf16 *W1b, *W2b;              // bf16 operand copies (bf16 path)
@@ -33,6 +33,10 @@ struct DevState {
     float* zinv;                  // [C][win_rows] 1 / |z_t| (bf16 path: U holds unnormalised z)
     void* dHt;                    // [C][T][d_hid] c_t dH (bf16 or fp32 by path)
     void* Att;                    // [C][T][d_hid] c_t A
+    // squared-error loss (bf16 path): the segment's activations with the W2 row scales folded
+    // in, and the residual targets y - M(u) that phase A and phase B read in place of K, V
+    bf16* Amse;                   // [C][T][d_hid]
+    bf16 *Kres, *Vres;            // [C][T][d_out/2]
     // read scratch (grown on demand)
     int q_cap;
     float *Uq, *Aq, *Oq;          // [C][q_cap][d_in|d_hid|d_out]
@@ -56,6 +60,7 @@ struct SegWork {
     int parity;                  // segment index parity within the call
     int renorm_pending;          // previous segment's renorm scale still to apply
     float* loss;                 // [C] loss accumulator or null
+    int y_scratch;               // targets are the residual scratch (rows from 0), not the caller's K, V
 };
 
 // ---- kernels in ttl_prepass.cu
@@ -88,6 +93,7 @@ struct TcMaps {
     CUtensorMap W1s, W2s, M1s, M2s;  // fp32 state chunks {128 cols, 32 rows}, no swizzle
     CUtensorMap W1o, W2o;            // bf16 operand-copy chunks {128 cols, 32 rows}, no swizzle
     CUtensorMap W2m;                 // bf16 W2 copy, MN-major boxes {64 outputs, 64 hidden} (memory read)
+    CUtensorMap Amse;                // squared-error activations, K-major {64, 128}
 };
 struct TcInputMaps {
     CUtensorMap Xa, Xb, Ka, Kb, Va, Vb;  // per call: K-major {64,128} (a) and MN {64,64} (b)
@@ -101,6 +107,10 @@ int tc_kernels_per_segment();
 // Aq = bf16 scratch [C][Q][d_hid]; writes K/V (bf16) with the caller's strides.
 cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, void* Aq, int Q, int n_layers,
                            void* K_out, void* V_out, const long long* strides, cudaStream_t st);
+// Squared-error pre-pass of one segment (two kernels): M(u) at the segment's starting
+// weights and the residual targets y - M(u) into s.Kres / s.Vres (plus the loss into w.loss).
+cudaError_t launch_mse_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,
+                          cudaStream_t st);
 
 // Tensor-map encoders (driver entry point, resolved at run time).  3-D maps over
 // [chains][rows][inner]; bf16 maps use 128-byte swizzle, the *_plain ones none.

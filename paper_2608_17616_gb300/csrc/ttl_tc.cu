@@ -849,7 +849,7 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
     a.tok0 = w.u_off;
     a.win = s.win_rows;
     a.u_chain0 = a.paper ? w.c0 : 0;
-    a.y_row0 = (int)w.row0;
+    a.y_row0 = w.y_scratch ? 0 : (int)w.row0;
     a.lr = s.lr;
     a.eta_in = w.eta_in ? w.eta_in + w.row0 : nullptr;
     a.eta_cstride = w.eta_cstride;
@@ -883,7 +883,8 @@ struct LR {
     static constexpr int NBARS = 2 * R_STAGES + 1;
     static constexpr int SLOT = BARS + (NBARS * 8 + 15) / 16 * 16;
     static constexpr int FLAG = SLOT + 16;
-    static constexpr int STG = FLAG + 16;  // 4 epilogue warps x 2 KB transpose buffers
+    static constexpr int TAB = FLAG + 16;  // MSE_HIDDEN: renorm scales s1, s2 of the tile's rows
+    static constexpr int STG = TAB + 256 * 4;  // 4 epilogue warps x 2 KB transpose buffers
     static constexpr int END = STG + 4 * 2048;
     static constexpr int DYN = END + 1024;
 };
@@ -897,13 +898,28 @@ struct ReadArgs {
     bf16 *Kout, *Vout;     // caller's K / V, element strides s0 (context), s1 (layer), s2 (head), s3 (query)
     long long s0, s1, s2, s3;
     int* status;
+    // operand coordinates: A rows start at a_row0 + 128 * blockIdx.x of chain a_chain0 + blockIdx.z,
+    // weights of chain b_chain0 + blockIdx.z
+    int a_row0, a_chain0, b_chain0;
+    // squared-error loss pre-pass (MSE_* modes): one segment of chains b_chain0 + blockIdx.z
+    int C, T, Tp, win, parity, renorm_pending;
+    long long tok0, row0, n_rows, y_cstride;
+    const float *zinv, *n1, *n2, *sumsq;  // as in TcArgs
+    const bf16 *K, *V;     // caller's targets of the group (chain z at z * y_cstride)
+    bf16 *Kres, *Vres;     // [C][T][d_out/2] residual targets y - M(u)
+    float* loss;           // [nc] or null
 };
 
-// MODE 0: hidden kernel.  MODE 64 / 128: out kernel with heads of that width.
+enum { READ_HIDDEN = 0, MSE_HIDDEN = 1, MSE_OUT = 2 };  // other MODEs: read out with heads of width MODE
+
+// MODE READ_HIDDEN: A_q = SiLU(U_q W1^T).  MODE 64 / 128: the read's out kernel with heads
+// of that width.  MODE MSE_HIDDEN: A' = SiLU(s1 (1/|z_t|) H) s2, the segment's activations
+// with the pending renorm scales (s2 folded in, so A' W2raw = A W2).  MODE MSE_OUT: the
+// residual target y_t - M(u_t) = y_t - A'_t W2raw (and the segment's squared-error loss).
 template <int MODE>
 __global__ void __launch_bounds__(R_THREADS, 1)
 tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const ReadArgs a) {
-    constexpr bool OUT = MODE != 0;
+    constexpr bool OUT = MODE != READ_HIDDEN && MODE != MSE_HIDDEN;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const uint32_t bars = smem_u32(base + LR::BARS);
@@ -929,6 +945,7 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const uint32_t tmem = *reinterpret_cast<uint32_t*>(base + LR::SLOT);
     const int q0 = blockIdx.x * 128, n0 = blockIdx.y * 128, c = blockIdx.z;
     const int KB = (OUT ? a.d_hid : a.d_in) / BK;
+    float* table = reinterpret_cast<float*>(base + LR::TAB);
 
     if (warp == 0) {
         if (lane == 0) {
@@ -939,12 +956,12 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                 if (kb >= R_STAGES && !mbar_wait(empty(s), ((kb / R_STAGES) - 1) & 1, a.status)) break;
                 const uint32_t sa = smem_u32(base + s * R_STAGE), sb = sa + 128 * BK * 2, fb = full(s);
                 mbar_expect_tx(fb, R_STAGE);
-                tma_load_3d(sa, &tmA, fb, kb * BK, q0, c);
+                tma_load_3d(sa, &tmA, fb, kb * BK, a.a_row0 + q0, a.a_chain0 + c);
                 if (OUT) {
-                    tma_load_3d(sb, &tmB, fb, n0, kb * BK, c);
-                    tma_load_3d(sb + BOX, &tmB, fb, n0 + 64, kb * BK, c);
+                    tma_load_3d(sb, &tmB, fb, n0, kb * BK, a.b_chain0 + c);
+                    tma_load_3d(sb + BOX, &tmB, fb, n0 + 64, kb * BK, a.b_chain0 + c);
                 } else {
-                    tma_load_3d(sb, &tmB, fb, kb * BK, n0, c);
+                    tma_load_3d(sb, &tmB, fb, kb * BK, n0, a.b_chain0 + c);
                 }
             }
         }
@@ -974,6 +991,20 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     } else {
         const int q = warp & 3;  // TMEM lane quarter of this warp
         int* flag = reinterpret_cast<int*>(base + LR::FLAG);
+        if constexpr (MODE == MSE_HIDDEN) {
+            // renorm scales of this tile's 128 hidden rows (one per epilogue thread)
+            const int h = n0 + (int)threadIdx.x - 64, cs = a.b_chain0 + c;
+            float s1 = 1.f, s2 = 1.f;
+            if (a.renorm_pending) {
+                // row sums of squares of the last update: [2 parity][2 matrix][C][d_hid]
+                const float* ss1 = a.sumsq + ((size_t)((a.parity ^ 1) * 2 + 0) * a.C + cs) * a.d_hid;
+                const float* ss2 = a.sumsq + ((size_t)((a.parity ^ 1) * 2 + 1) * a.C + cs) * a.d_hid;
+                s1 = renorm_scale(a.n1[(size_t)cs * a.d_hid + h], ss1[h]);
+                s2 = renorm_scale(a.n2[(size_t)cs * a.d_hid + h], ss2[h]);
+            }
+            table[threadIdx.x - 64] = s1;
+            table[128 + threadIdx.x - 64] = s2;
+        }
         if (threadIdx.x == 64) *flag = mbar_wait(tfull, 0, a.status) ? 1 : 0;
         __syncwarp();
         named_bar_sync(R_EPI_BAR, 128);
@@ -981,7 +1012,59 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             tc_fence_after();
             const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
             const int qw = q0 + q * 32;  // first query row of this warp
-            if constexpr (!OUT) {
+            if constexpr (MODE == MSE_HIDDEN) {
+                const int cs = a.b_chain0 + c, t = qw + lane;
+                const float zi = (t < a.Tp) ? (a.zinv ? a.zinv[(size_t)cs * a.win + a.tok0 + t] : 1.f) : 0.f;
+                uint8_t* stg = base + LR::STG + (warp - 2) * 2048;
+                bf16* row0 = a.Aq + ((size_t)cs * a.T + qw) * a.d_hid + n0;
+#pragma unroll 1
+                for (int cc = 0; cc < 4; ++cc) {
+                    float hv[32];
+                    tmem_ld32(lane_base + cc * 32, hv);
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const int k0 = cc * 32 + 2 * j;
+                        const float x0 = hv[2 * j] * table[k0] * zi, x1 = hv[2 * j + 1] * table[k0 + 1] * zi;
+                        pk[j] = pack_bf16(x0 * sigmoidf_(x0) * table[128 + k0], x1 * sigmoidf_(x1) * table[128 + k0 + 1]);
+                    }
+                    store_rows_coalesced(stg, pk, row0 + cc * 32, a.d_hid, lane);
+                }
+            } else if constexpr (MODE == MSE_OUT) {
+                const int cs = a.b_chain0 + c, t = qw + lane, dh = a.d_out / 2;
+                const bool kpart = n0 < dh;
+                const int col0 = kpart ? n0 : n0 - dh;
+                const bool live = t < a.Tp && a.row0 + t < a.n_rows;
+                const bf16* yrow = (kpart ? a.K : a.V) + (size_t)c * a.y_cstride + (size_t)(a.row0 + t) * dh + col0;
+                uint8_t* stg = base + LR::STG + (warp - 2) * 2048;
+                bf16* row0 = (kpart ? a.Kres : a.Vres) + ((size_t)cs * a.T + qw) * dh + col0;
+                float lsum = 0.f;
+#pragma unroll 1
+                for (int cc = 0; cc < 4; ++cc) {
+                    float ov[32];
+                    tmem_ld32(lane_base + cc * 32, ov);
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) {
+                        uint4 y = make_uint4(0, 0, 0, 0);
+                        if (live) y = *reinterpret_cast<const uint4*>(yrow + cc * 32 + v * 8);
+                        const __nv_bfloat162* yb = reinterpret_cast<const __nv_bfloat162*>(&y);
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            const float2 yf = __bfloat1622float2(yb[u]);
+                            const int j = v * 8 + 2 * u;
+                            const float r0 = live ? yf.x - ov[j] : 0.f, r1 = live ? yf.y - ov[j + 1] : 0.f;
+                            lsum = fmaf(r0, r0, fmaf(r1, r1, lsum));
+                            pk[v * 4 + u] = pack_bf16(r0, r1);
+                        }
+                    }
+                    store_rows_coalesced(stg, pk, row0 + cc * 32, dh, lane);
+                }
+                if (a.loss) {
+                    lsum = warp_sum(lsum);
+                    if (lane == 0) atomicAdd(&a.loss[c], 0.5f * lsum / (float)a.Tp);
+                }
+            } else if constexpr (!OUT) {
                 uint8_t* stg = base + LR::STG + (warp - 2) * 2048;
                 bf16* row0 = a.Aq + ((size_t)c * a.Q + qw) * a.d_hid + n0;
 #pragma unroll 1
@@ -1059,6 +1142,12 @@ cudaError_t ensure_attrs() {
             g_attr_err = cudaFuncSetAttribute(tc_read_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
         if (g_attr_err == cudaSuccess)
             g_attr_err = cudaFuncSetAttribute(tc_read_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err = cudaFuncSetAttribute(tc_read_kernel<MSE_HIDDEN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              LR::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err =
+                cudaFuncSetAttribute(tc_read_kernel<MSE_OUT>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
         if (g_attr_err == cudaSuccess) {
             cudaLaunchConfig_t cfg = {};
             cudaLaunchAttribute at[1];
@@ -1125,6 +1214,37 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
 }
 
 int tc_kernels_per_segment() { return 2; }
+
+cudaError_t launch_mse_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,
+                          cudaStream_t st) {
+    cudaError_t e = ensure_attrs();
+    if (e != cudaSuccess) return e;
+    const bool paper = s.mode == 1;
+    ReadArgs a{};
+    a.d_in = s.d_in; a.d_hid = s.d_hid; a.d_out = s.d_out; a.n_kv = s.n_kv;
+    a.status = s.status;
+    a.C = s.C; a.T = s.T; a.Tp = w.Tp; a.win = s.win_rows; a.parity = w.parity; a.renorm_pending = w.renorm_pending;
+    a.tok0 = w.u_off; a.row0 = w.row0; a.n_rows = w.n_rows; a.y_cstride = w.y_cstride;
+    a.zinv = paper ? s.zinv : nullptr;
+    a.n1 = s.n1; a.n2 = s.n2; a.sumsq = s.sumsq;
+    a.K = static_cast<const bf16*>(w.K); a.V = static_cast<const bf16*>(w.V);
+    a.Kres = s.Kres; a.Vres = s.Vres;
+    a.loss = w.loss;
+    a.Aq = s.Amse;
+    // hidden: U rows of the segment (paper: the transformed window, absolute chain; plain: the
+    // caller's X of the group), W1 of chain c0 + z
+    a.a_row0 = paper ? (int)w.u_off : (int)w.row0;
+    a.a_chain0 = paper ? w.c0 : 0;
+    a.b_chain0 = w.c0;
+    tc_read_kernel<MSE_HIDDEN><<<dim3(s.T / 128, s.d_hid / 128, w.nc), R_THREADS, LR::DYN, st>>>(
+        paper ? m.Ua : in.Xa, m.W1b, a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    // out: the activations of the same chains (absolute), W2 MN-major
+    a.a_row0 = 0;
+    a.a_chain0 = w.c0;
+    tc_read_kernel<MSE_OUT><<<dim3(s.T / 128, s.d_out / 128, w.nc), R_THREADS, LR::DYN, st>>>(m.Amse, m.W2m, a);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, void* Aq, int Q, int n_layers,
                            void* K_out, void* V_out, const long long* strides, cudaStream_t st) {

@@ -22,7 +22,8 @@ def rel_fro(a, b) -> float:
 
 def config_of(wl: wk.Workload) -> "mone.mone_config":
     return mone.make_config(wl.n_ctx, wl.n_layers, wl.d_in, wl.d_hid, wl.d_out, wl.n_kv_heads, wl.head_dim,
-                            wl.seg_T, mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr)
+                            wl.seg_T, mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr,
+                            loss=mone.MONE_LOSS_MSE if wl.loss == "mse" else mone.MONE_LOSS_DOT)
 
 
 class GpuRun:
@@ -77,7 +78,7 @@ class GpuRun:
 
 
 def oracle_hyper(wl: wk.Workload) -> O.Hyper:
-    return O.Hyper(mode=wl.mode, lr=wl.lr)
+    return O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss)
 
 
 def oracle_meta(run: GpuRun, chain: int):

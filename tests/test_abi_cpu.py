@@ -35,7 +35,7 @@ def test_library_exports_every_declared_symbol(L):
     raw = ctypes.CDLL(mone.LIB_PATH)
     for name in header_functions():
         assert hasattr(raw, name), name
-    assert L.mone_abi_version() == 1
+    assert L.mone_abi_version() == 2
 
 
 def test_status_strings(L):
@@ -65,6 +65,12 @@ def test_init_rejects_bad_arguments_without_a_device(L):
     assert init_rc(L, cfg(n_layers=0)) == 1
     assert init_rc(L, cfg(lr=float("nan"))) == 1
     assert init_rc(L, cfg(mode=mone.MONE_PAPER)) == 1         # paper mode needs meta-parameters
+    assert init_rc(L, cfg(loss=2)) == 1                         # no such loss
+
+
+def test_squared_error_loss_is_bf16_only(L):
+    # the squared-error variant runs on the tensor-core path only: the fp32 path reports it unsupported
+    assert init_rc(L, cfg(dtype=mone.MONE_FP32, loss=mone.MONE_LOSS_MSE)) == 7
 
 
 def test_init_rejects_unsupported_shapes(L):

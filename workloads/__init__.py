@@ -49,6 +49,7 @@ class Workload:
     dtype: str               # "f32" or "bf16": activations and targets
     mode: int                # PLAIN or PAPER
     lr: float = 1e-2
+    loss: str = "neg_inner"  # "neg_inner" (Eq. 7) or "mse" (squared-error variant)
 
     @property
     def chains(self) -> int:
