@@ -49,6 +49,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="target CPU time of the oracle sample")
     p.add_argument("--n-tokens", type=int, default=0, help="override the context length (small profiling cases)")
+    p.add_argument("--loss", default="neg_inner", choices=["neg_inner", "mse"],
+                   help="per-token loss: Eq. 7 (the measured workload) or the squared-error variant")
     return p.parse_args()
 
 
@@ -186,7 +188,7 @@ def oracle_sample(wl, seconds, chain=0):
     W1all, W2all = wk.initial_weights(wl, "cpu")
     W1, W2 = W1all[chain], W2all[chain]
     meta = O.Meta.from_torch(wk.meta_params(wl, "cpu"), chain) if wl.mode == wk.PAPER else None
-    hp = O.Hyper(mode=wl.mode, lr=wl.lr)
+    hp = O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss)
     X1, Y1 = inputs(T)
     st = O.init_state(W1=O.f64(W1), W2=O.f64(W2))
     t0 = time.perf_counter()
@@ -260,7 +262,7 @@ def run_reference(args, wl):
 def config_of(wl):
     return {"workload": wl.name, "n_ctx": wl.n_ctx, "n_layers": wl.n_layers, "chains": wl.chains,
             "N": wl.N, "seg_T": wl.seg_T, "d_in": wl.d_in, "d_hid": wl.d_hid, "d_out": wl.d_out, "Q": wl.Q,
-            "mode": "paper" if wl.mode == 1 else "plain", "masters": "fp32", "operands": wl.dtype,
+            "mode": "paper" if wl.mode == 1 else "plain", "loss": wl.loss, "masters": "fp32", "operands": wl.dtype,
             "l2": "inputs larger than L2 (no flush needed)"}
 
 
@@ -288,7 +290,8 @@ def run_ours(args, wl):
     Vout = torch.empty_like(Kout)
     strides = mone.kv_strides(wl.n_layers, wl.n_kv_heads, wl.Q, wl.head_dim)
     cfg = mone.make_config(wl.n_ctx, wl.n_layers, wl.d_in, wl.d_hid, wl.d_out, wl.n_kv_heads, wl.head_dim, wl.seg_T,
-                           mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr)
+                           mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr,
+                           loss=mone.MONE_LOSS_MSE if wl.loss == "mse" else mone.MONE_LOSS_DOT)
     h = mone.mone_mem_init(cfg, W1_0, W2_0, meta)
     stream = torch.cuda.current_stream()
 
@@ -468,6 +471,8 @@ def main():
     wl = wk.WORKLOADS[args.workload]
     if args.n_tokens:
         wl = wl.replace(N=args.n_tokens)
+    if args.loss != "neg_inner":
+        wl = wl.replace(loss=args.loss)
     if args.impl == "reference":
         run_reference(args, wl)
     else:
