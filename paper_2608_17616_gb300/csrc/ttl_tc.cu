@@ -276,6 +276,7 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             tma_prefetch_map(&tmV);
             tma_prefetch_map(&tmW1);
             tma_prefetch_map(&tmW2);
+            const uint64_t wpol = l2_evict_last_policy();  // the bf16 W copy phase B wrote
             uint32_t kc = 0;
             bool ok = true;
             for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
@@ -291,14 +292,14 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                     mbar_expect_tx(fb, A_STAGE);
                     if (kb < KB1) {
                         tma_load_3d(sa, &tmU, fb, kb * BK, a.u_row0 + trow, a.u_chain0 + cz);
-                        tma_load_3d(sb, &tmW1, fb, kb * BK, h0, cs);
+                        tma_load_3d_hint(sb, &tmW1, fb, kb * BK, h0, cs, wpol);
                     } else {
                         const int k2 = kb - KB1;
                         if (k2 < half)
                             tma_load_3d(sa, &tmK, fb, k2 * BK, a.y_row0 + trow, cz);
                         else
                             tma_load_3d(sa, &tmV, fb, (k2 - half) * BK, a.y_row0 + trow, cz);
-                        tma_load_3d(sb, &tmW2, fb, k2 * BK, h0, cs);
+                        tma_load_3d_hint(sb, &tmW2, fb, k2 * BK, h0, cs, wpol);
                     }
                 }
             }
@@ -431,6 +432,7 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
             tma_prefetch_map(&tmV);
             tma_prefetch_map(&tmW1);
             tma_prefetch_map(&tmW2);
+            const uint64_t wpol = l2_evict_last_policy();  // the bf16 W copy phase B wrote
             uint32_t kc = 0;
             bool ok = true;
             for (int pt = cluster; pt < npairs && ok; pt += nclusters) {
@@ -449,14 +451,14 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
                     if (rank == 0) mbar_expect_tx(c.full(s), 2 * P_STAGE);
                     if (kb < KB1) {
                         tma_load_3d_pair(sa, &tmU, fb, kb * BK, a.u_row0 + trow, a.u_chain0 + cz);
-                        tma_load_3d_pair(sb, &tmW1, fb, kb * BK, hrow, cs);
+                        tma_load_3d_pair_hint(sb, &tmW1, fb, kb * BK, hrow, cs, wpol);
                     } else {
                         const int k2 = kb - KB1;
                         if (k2 < half)
                             tma_load_3d_pair(sa, &tmK, fb, k2 * BK, a.y_row0 + trow, cz);
                         else
                             tma_load_3d_pair(sa, &tmV, fb, (k2 - half) * BK, a.y_row0 + trow, cz);
-                        tma_load_3d_pair(sb, &tmW2, fb, k2 * BK, hrow, cs);
+                        tma_load_3d_pair_hint(sb, &tmW2, fb, k2 * BK, hrow, cs, wpol);
                     }
                 }
             }
@@ -776,6 +778,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             float* cur = ss_row(a, a.parity, which, cs);
             const int col = q * 32 + lane;  // column within the tile (= TMEM lane)
             bf16* Wb = (isW1 ? a.W1b : a.W2b) + (size_t)cs * a.d_hid * width + cl + col;
+            const uint64_t wpol = l2_evict_last_policy();  // phase A of the next segment reads the copy
             const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 256;
             bool ok = true;
 #pragma unroll 1
@@ -811,7 +814,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                     const float wn = fmaf(sc, Ws[j * B_BM + col], -mn);
                     Ws[j * B_BM + col] = wn;
                     if (a.momentum) Ms[j * B_BM + col] = mn;
-                    bp[j * width] = __float2bfloat16_rn(wn);
+                    st_bf16_hint(bp + j * width, __float2bfloat16_rn(wn), wpol);
                     v[j] = wn * wn;  // a NaN or Inf weight makes its row's sum non-finite
                 }
                 // transpose-reduce: afterwards lane j holds this warp's 32-column partial of row j
