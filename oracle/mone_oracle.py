@@ -25,6 +25,8 @@ Inference"):
                       (sigmoid, from the chunk's hidden states), channel-wise
                       L2 renormalisation after each update
   Eq. 9-11            sequential chain over segments; gradient local to layer
+  Eq. 2, Eq. 5        the consumer attention: softmax(q k^T / sqrt(d_h)) v over
+                      [memory tokens || the query tokens' own keys]
 
 Readings of passages the paper leaves open (each also listed in the design
 notes):
@@ -42,6 +44,9 @@ notes):
       gate g_h; eps = 1e-6.
   R7  Key/query transform u = z / sqrt(|z|^2 + 1e-12), z = SiLU(alpha*x + gamma).
   R8  Plain mode: u = x, eta_j = lr, beta = 0, no renormalisation.
+  R14 Consumer attention (Eq. 5): the memory tokens are a prefix every query
+      token sees; the query tokens are causal among themselves; query head h
+      reads key/value head h // (n_q / n_kv) (grouped heads).
 
 Pinned by tests (tests/test_oracle_pins.py): the gradient (finite
 differences), the loss (closed-form one-hot case), the update (closed form of
@@ -49,7 +54,9 @@ one step of a linear memory, Hebbian for Eq. 7 and the delta rule for a
 squared-error loss), the momentum recurrence (geometric-sum closed form), the
 renormalisation invariant, lr = 0 leaving W bit-identical, the read's
 RMS = |gate| invariant, the read of a linear memory against brute force, and
-the chain identities (context = loop of segments = split contexts).
+the chain identities (context = loop of segments = split contexts), and the
+consumer attention against its special cases (one visible key returns its
+value, equal keys average the visible values, causality, grouped heads).
 Parity unpinned: the exact numbers of the paper-mode readings R3, R6, R7
 (their forms are the build's reading; only the invariants above constrain
 them).
@@ -341,3 +348,26 @@ def generate_kv(state: State, Xq, hp: Hyper, meta: Optional[Meta], n_kv_heads: i
         rms = np.sqrt(np.mean(o * o, axis=1, keepdims=True) + eps)
         out[h] = gate[h] * o / rms
     return out[:n_kv_heads], out[n_kv_heads:]
+
+
+# --------------------------------------------------------------------------- consumer attention
+
+def attention(Q, K, V, n_mem: int):
+    """Eq. 5 with Eq. 2 per head (R14): out[h, i] = softmax_j(q_{h,i} . k_j / sqrt(d_h)) v_j over the
+    keys j visible to query token i: the n_mem memory tokens and query tokens 0..i.
+
+    Q [n_q, Lq, d_h]; K, V [n_kv, n_mem + Lq, d_h] (memory tokens first); n_q a multiple of n_kv,
+    query head h reading key/value head h // (n_q // n_kv).  Returns [n_q, Lq, d_h]."""
+    Q, K, V = f64(Q), f64(K), f64(V)
+    n_q, Lq, dh = Q.shape
+    group = n_q // K.shape[0]
+    out = np.empty((n_q, Lq, dh))
+    for h in range(n_q):
+        Kh, Vh = K[h // group], V[h // group]
+        for i in range(Lq):
+            vis = n_mem + i + 1                       # memory tokens, then query tokens up to i
+            z = Kh[:vis] @ Q[h, i] / np.sqrt(dh)
+            p = np.exp(z - z.max())
+            out[h, i] = (p / p.sum()) @ Vh[:vis]
+    return out
+

@@ -388,3 +388,52 @@ def test_swiglu_paper_mode_renorm_invariant():
         for h in range(H):
             np.testing.assert_allclose(np.linalg.norm(st.W[k][h], axis=1), np.linalg.norm(w0[h], axis=1),
                                        rtol=1e-13)
+
+
+# ----------------------------------------------------------------- consumer attention (Eq. 5, R14)
+
+def _attn_inputs(n_q=4, n_kv=2, Lq=5, n_mem=3, dh=8, seed=0):
+    r = np.random.default_rng(seed)
+    return (r.standard_normal((n_q, Lq, dh)), r.standard_normal((n_kv, n_mem + Lq, dh)),
+            r.standard_normal((n_kv, n_mem + Lq, dh)))
+
+
+def test_attention_one_visible_key_returns_its_value():
+    # no memory tokens: query token 0 sees only its own key, so its output is its own value
+    Q, K, V = _attn_inputs(n_mem=0)
+    out = O.attention(Q, K, V, 0)
+    for h in range(Q.shape[0]):
+        assert np.allclose(out[h, 0], V[h // 2, 0], rtol=0, atol=1e-14)
+
+
+def test_attention_equal_keys_average_the_visible_values():
+    Q, K, V = _attn_inputs()
+    K[:] = K[:, :1]                      # every key identical -> uniform weights
+    out = O.attention(Q, K, V, 3)
+    for h in range(4):
+        for i in range(5):
+            assert np.allclose(out[h, i], V[h // 2, :3 + i + 1].mean(axis=0), atol=1e-12)
+
+
+def test_attention_is_causal_over_query_tokens_and_sees_all_memory():
+    Q, K, V = _attn_inputs()
+    base = O.attention(Q, K, V, 3)
+    K2, V2 = K.copy(), V.copy()
+    K2[:, 3 + 4] += 5.0                  # the last query token's key and value
+    V2[:, 3 + 4] -= 3.0
+    out = O.attention(Q, K2, V2, 3)
+    assert np.array_equal(out[:, :4], base[:, :4])          # earlier tokens do not see it
+    assert not np.allclose(out[:, 4], base[:, 4])
+    K3 = K.copy()
+    K3[:, 0] += 5.0                      # a memory token changes every output
+    out3 = O.attention(Q, K3, V, 3)
+    assert all(not np.allclose(out3[:, i], base[:, i]) for i in range(5))
+
+
+def test_attention_grouped_heads_and_softmax_by_hand():
+    Q, K, V = _attn_inputs(n_q=6, n_kv=3, Lq=2, n_mem=2, dh=4, seed=3)
+    out = O.attention(Q, K, V, 2)
+    h, i = 3, 1                          # head 3 reads kv head 3 // 2 = 1 (not 3 % 3); token 1 sees 2 + 2 keys
+    w = [np.exp(np.dot(Q[h, i], K[1, j]) / 2.0) for j in range(4)]
+    want = sum(wj * V[1, j] for j, wj in enumerate(w)) / sum(w)
+    assert np.allclose(out[h, i], want, atol=1e-13)
