@@ -396,6 +396,44 @@ def run_ours(args, wl):
         e2e = {"value": ws * tokens_per_step / (ms_e2e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e, "chunks": n_chunks}
 
+    # ---- consumer attention of the read (Eq. 5): the query's tokens over [memory tokens || their own
+    # keys], timed on its own (it is not part of the test-time-learning step).  The memory tokens are
+    # this step's read (Q of them); the query tokens' own Q, K, V are synthetic; 2 query heads per
+    # key/value head.
+    attn = None
+    if ws == 1 or rank == 0:
+        n_q, Lq, n_mem = 2 * wl.n_kv_heads, wl.Q, wl.Q
+        ga = torch.Generator(device=dev).manual_seed(1234)
+        cache = (wl.n_ctx, wl.n_layers, wl.n_kv_heads, n_mem + Lq, wl.head_dim)
+        Kc = torch.randn(*cache, generator=ga, device=dev).to(X.dtype)
+        Vc = torch.randn(*cache, generator=ga, device=dev).to(X.dtype)
+        mone.mone_mem_generate_kv(h, Xq, wl.Q, Kc, Vc, Kc.stride()[:4])
+        Qa = torch.randn(wl.n_ctx, wl.n_layers, n_q, Lq, wl.head_dim, generator=ga, device=dev).to(X.dtype)
+        Oa = torch.empty_like(Qa)
+        for _ in range(3):
+            mone.mone_attention(h, Qa, n_q, Lq, Kc, Vc, Kc.stride()[:4], n_mem, Oa)
+        torch.cuda.synchronize()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = 20
+        a0.record(stream)
+        for _ in range(reps):
+            mone.mone_attention(h, Qa, n_q, Lq, Kc, Vc, Kc.stride()[:4], n_mem, Oa)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        mone.mone_mem_sync(h)
+        us = 1000 * a0.elapsed_time(a1) / reps
+        mone.mone_mem_set_timing(h, True)
+        mone.mone_attention(h, Qa, n_q, Lq, Kc, Vc, Kc.stride()[:4], n_mem, Oa)
+        t_k, n_k = mone.mone_mem_kernel_time(h, mone.KERNEL_KINDS.index("attention"))
+        mone.mone_mem_set_timing(h, False)
+        kernel_us = 1000 * t_k / max(1, n_k)
+        el = Qa.element_size()
+        byts = (Kc.numel() + Vc.numel() + Qa.numel() + Oa.numel()) * el
+        # causal over the query tokens: token i sees n_mem + i + 1 keys
+        flops = 4 * wl.chains * n_q * wl.head_dim * (Lq * n_mem + Lq * (Lq + 1) // 2)
+        attn = {"us": us, "kernel_us": kernel_us, "n_q_heads": n_q, "Lq": Lq, "n_mem": n_mem, "bytes": byts,
+                "gbs": byts / (us * 1e-6) / 1e9, "tflops": flops / (us * 1e-6) / 1e12}
+
     # ---- roofline of the dominant kernel
     hbm, tf_burst, tf_sus, peak_src = peaks()
     kern = {}
@@ -457,6 +495,7 @@ def run_ours(args, wl):
                 "config": config_of(wl), "e2e": e2e, "gpu_launches": launches, "roofline": roof,
                 "cpu_baseline": cpu, "clocks": clk,
                 "tensor_util_of_burst_peak": tensor_util, "step_roofline": step_roof, "generate_kv": gkv,
+                "consumer_attention": attn,
                 "kernels": kern}
         print(json.dumps(line), flush=True)
     mone.mone_mem_free(h)

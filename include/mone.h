@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define MONE_ABI_VERSION 2
+#define MONE_ABI_VERSION 3
 
 typedef struct mone_mem mone_mem; /* opaque; created by mone_mem_init */
 
@@ -196,6 +196,26 @@ mone_status mone_mem_sync(mone_mem* m, void* stream);
 long long mone_mem_launch_count(const mone_mem* m);
 
 /*
+ * Consumer attention of the read (Eq. 5, with the attention of Eq. 2 per head).  For every
+ * chain (context, layer), query head h and query token i:
+ *     out[h][i] = sum_j softmax_j(q[h][i] . k[g][j] / sqrt(head_dim)) v[g][j],
+ *     g = h / (n_q_heads / n_kv_heads)   (grouped heads),
+ * over the keys j that token i sees: the n_mem memory tokens at cache positions
+ * 0 .. n_mem-1 (for example written there by mone_mem_generate_kv) and the query
+ * tokens' own keys at positions n_mem .. n_mem+i (causal among the query tokens).
+ *   Q      [n_ctx][n_layers][n_q_heads][Lq][head_dim], dense, the handle's dtype
+ *   K, V   caches of the handle's dtype with element strides kv_strides[4] =
+ *          (context, layer, KV head, position), head_dim contiguous, holding at least
+ *          n_mem + Lq positions
+ *   out    [n_ctx][n_layers][n_q_heads][Lq][head_dim], dense, the handle's dtype
+ * Reads the caches only; the memory state is not touched.  Constraints: n_q_heads a
+ * multiple of n_kv_heads with n_q_heads / n_kv_heads <= 64; 1 <= Lq; 0 <= n_mem;
+ * n_mem + Lq <= 2^20.  Errors: INVALID_ARG.  Asynchronous on stream.
+ */
+mone_status mone_attention(mone_mem* m, const void* Q, int n_q_heads, int Lq, const void* K, const void* V,
+                           const long long kv_strides[4], int n_mem, void* out, void* stream);
+
+/*
  * Per-kernel device timing for measurement.  While enabled, the library records
  * a pair of CUDA events on the caller's stream around every kernel it launches
  * (this adds host work per launch; leave it off outside measurement).
@@ -204,7 +224,7 @@ long long mone_mem_launch_count(const mone_mem* m);
  * last enabled.  Kinds: 0 input prepass, 1 phase A (forward + fused backward
  * epilogue), 2 phase B (gradient + fused update), 3 finalize (renorm apply /
  * operand refresh), 4 memory read, 5 squared-error pre-pass (M(u) and the residual
- * target, MONE_LOSS_MSE only).  Errors: INVALID_ARG, CUDA.
+ * target, MONE_LOSS_MSE only), 6 consumer attention.  Errors: INVALID_ARG, CUDA.
  */
 mone_status mone_mem_set_timing(mone_mem* m, int enable);
 mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches);

@@ -27,9 +27,9 @@ STATUS = {0: "MONE_OK", 1: "MONE_ERR_INVALID_ARG", 2: "MONE_ERR_UNSUPPORTED_SHAP
 EXPORTS = ("mone_mem_init", "mone_ttl_segment", "mone_ttl_context", "mone_mem_generate_kv", "mone_mem_free",
            "mone_mem_read_state", "mone_mem_write_state", "mone_mem_sync", "mone_mem_launch_count",
            "mone_status_string", "mone_abi_version", "mone_mem_set_timing", "mone_mem_kernel_time",
-           "mone_last_error", "mone_mem_generate_kv_noalloc")
+           "mone_last_error", "mone_mem_generate_kv_noalloc", "mone_attention")
 
-KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read", "mse")
+KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read", "mse", "attention")
 
 
 class MoneError(RuntimeError):
@@ -69,6 +69,7 @@ def lib(path: Optional[str] = None) -> ctypes.CDLL:
         "mone_ttl_context": ([vp, vp, vp, vp, ll, vp], i),
         "mone_mem_generate_kv": ([vp, vp, i, vp, vp, ctypes.POINTER(ll), vp], i),
         "mone_mem_generate_kv_noalloc": ([vp, vp, i, vp, vp, ctypes.POINTER(ll), vp], i),
+        "mone_attention": ([vp, vp, i, i, vp, vp, ctypes.POINTER(ll), i, vp, vp], i),
         "mone_mem_free": ([vp], i),
         "mone_mem_read_state": ([vp, vp, vp, vp, vp, vp], i),
         "mone_mem_write_state": ([vp, vp, vp, vp, vp, vp], i),
@@ -154,6 +155,14 @@ def mone_mem_generate_kv_noalloc(h: int, Xq, Q: int, K_out, V_out, strides: Sequ
     arr = (ctypes.c_longlong * 4)(*[int(s) for s in strides])
     _check("mone_mem_generate_kv_noalloc", lib().mone_mem_generate_kv_noalloc(h, _ptr(Xq), Q, _ptr(K_out),
                                                                               _ptr(V_out), arr, _stream(stream)))
+
+
+def mone_attention(h: int, Q, n_q_heads: int, Lq: int, K, V, kv_strides: Sequence[int], n_mem: int, out,
+                   stream=None):
+    """Consumer attention of the read (Eq. 5): query tokens over [memory tokens || their own keys]."""
+    arr = (ctypes.c_longlong * 4)(*[int(s) for s in kv_strides])
+    _check("mone_attention", lib().mone_attention(h, _ptr(Q), n_q_heads, Lq, _ptr(K), _ptr(V), arr, n_mem, _ptr(out),
+                                                  _stream(stream)))
 
 
 def mone_mem_free(h: int):

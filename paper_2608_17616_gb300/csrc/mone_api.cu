@@ -25,8 +25,8 @@ struct KernelTiming {
     };
     std::vector<cudaEvent_t> pool;
     std::vector<Pending> pending;
-    double ms[6] = {0, 0, 0, 0, 0, 0};
-    long long n[6] = {0, 0, 0, 0, 0, 0};
+    double ms[7] = {0, 0, 0, 0, 0, 0, 0};
+    long long n[7] = {0, 0, 0, 0, 0, 0, 0};
 
     cudaEvent_t get() {
         if (!pool.empty()) {
@@ -198,7 +198,7 @@ mone_status build_input_maps(const DevState& s, TcInputMaps* in, const void* X, 
     return ok ? MONE_OK : MONE_ERR_CUDA;
 }
 
-enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4, K_MSE = 5 };
+enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4, K_MSE = 5, K_ATTN = 6 };
 
 // Launch through `fn` (which returns a cudaError_t), bracketed by timing events
 // when timing is on; `kernels` is the number of device kernels `fn` launches.
@@ -586,6 +586,23 @@ mone_status mone_mem_generate_kv_noalloc(mone_mem* m, const void* Xq, int Q, voi
                  [&] { return launch_read_noalloc(s, tc, Xq, Q, L, K_out, V_out, strides, st); });
 }
 
+mone_status mone_attention(mone_mem* m, const void* Q, int n_q_heads, int Lq, const void* K, const void* V,
+                           const long long kv_strides[4], int n_mem, void* out, void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    const DevState& s = m->s;
+    if (!Q || !K || !V || !out || !kv_strides) return MONE_ERR_INVALID_ARG;
+    if (n_q_heads < s.n_kv || n_q_heads % s.n_kv || n_q_heads / s.n_kv > 64) return MONE_ERR_INVALID_ARG;
+    if (Lq < 1 || n_mem < 0 || (long long)n_mem + Lq > (1ll << 20)) return MONE_ERR_INVALID_ARG;
+    for (int i = 0; i < 4; ++i)
+        if (kv_strides[i] < 0) return MONE_ERR_INVALID_ARG;
+    if (kv_strides[3] < s.hd) return MONE_ERR_INVALID_ARG;  // positions hold head_dim contiguous elements
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const int L = m->cfg.n_layers;
+    return timed(m, K_ATTN, st, 1, [&] {
+        return launch_attention(s, L, Q, n_q_heads, Lq, K, V, kv_strides, n_mem, out, st);
+    });
+}
+
 mone_status mone_mem_free(mone_mem* m) {
     {
         std::lock_guard<std::mutex> lk(g_live_mu);
@@ -666,7 +683,7 @@ mone_status mone_mem_set_timing(mone_mem* m, int enable) {
 }
 
 mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches) {
-    if (!is_live(m) || kind < 0 || kind > 5 || !ms || !launches) return MONE_ERR_INVALID_ARG;
+    if (!is_live(m) || kind < 0 || kind > 6 || !ms || !launches) return MONE_ERR_INVALID_ARG;
     *ms = 0;
     *launches = 0;
     if (!m->timing) return MONE_OK;

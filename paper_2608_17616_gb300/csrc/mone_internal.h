@@ -85,6 +85,10 @@ struct TcMaps;
 cudaError_t launch_read_noalloc(const DevState& s, const TcMaps* tc, const void* Xq, int Q, int n_layers,
                                 void* K_out, void* V_out, const long long* strides, cudaStream_t st);
 
+// ---- kernels in attention.cu
+cudaError_t launch_attention(const DevState& s, int n_layers, const void* Q, int n_q, int Lq, const void* K,
+                             const void* V, const long long* strides, int n_mem, void* out, cudaStream_t st);
+
 // ---- kernels in ttl_tc.cu (bf16 tcgen05 path)
 struct TcMaps {
     CUtensorMap W1b, W2b;        // K-major boxes {64, 128}

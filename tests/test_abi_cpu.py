@@ -35,7 +35,7 @@ def test_library_exports_every_declared_symbol(L):
     raw = ctypes.CDLL(mone.LIB_PATH)
     for name in header_functions():
         assert hasattr(raw, name), name
-    assert L.mone_abi_version() == 2
+    assert L.mone_abi_version() == 3
 
 
 def test_status_strings(L):
