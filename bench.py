@@ -65,15 +65,29 @@ def peaks():
 
 # ------------------------------------------------------------------ algorithmic work per launch
 
+def fast_params(wl):
+    """Fast weights per chain: d_hid (d_in + d_out) for the MLP, 3 d_hid d_in for the SwiGLU heads."""
+    return 3 * wl.d_hid * wl.d_in if wl.memory == "swiglu" else wl.d_hid * (wl.d_in + wl.d_out)
+
+
+def flops_per_token(wl):
+    """Algorithmic work of one token on one chain (forward + backward of the memory): the MLP's
+    4 (d_in d_hid + d_hid d_out); the SwiGLU heads' 4 x 3 d_hid dh per head (two forward
+    contractions, the backward one R, three gradients)."""
+    if wl.memory == "swiglu":
+        return 12 * wl.d_hid * wl.d_in
+    return 4 * (wl.d_in * wl.d_hid + wl.d_hid * wl.d_out)
+
+
 def kernel_work(wl, kind, chains=None):
     """(flops, bytes) of one launch of a phase kernel: one segment of `chains` chains
     (all of them by default; the library runs the chains of a call in two groups)."""
     C, T = (wl.chains if chains is None else chains), wl.seg_T
     di, dh, do = wl.d_in, wl.d_hid, wl.d_out
-    params = dh * (di + do)
-    flops = 2 * T * dh * (di + do) * C
+    params = fast_params(wl)
+    flops = T * flops_per_token(wl) * C // 2
     act = T * (di + do) * 2            # U and Y tiles, bf16, read once
-    grads = T * dh * 2 * 2             # dH^T and At^T, bf16
+    grads = T * dh * 2 * (2 if wl.memory == "mlp" else 3 * wl.heads)  # phase A outputs, bf16
     if kind == "phase_a":
         byts = C * (act + grads + params * 2)          # + bf16 weight operand read
     else:
@@ -188,15 +202,20 @@ def oracle_sample(wl, seconds, chain=0):
     W1all, W2all = wk.initial_weights(wl, "cpu")
     W1, W2 = W1all[chain], W2all[chain]
     meta = O.Meta.from_torch(wk.meta_params(wl, "cpu"), chain) if wl.mode == wk.PAPER else None
-    hp = O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss)
+    hp = O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss, memory=wl.memory, n_heads=wl.heads)
+
+    def init():
+        if wl.memory == "swiglu":
+            return O.init_state(Win=O.f64(W1[:, :wl.d_hid]), Wg=O.f64(W1[:, wl.d_hid:]), Wout=O.f64(W2))
+        return O.init_state(W1=O.f64(W1), W2=O.f64(W2))
     X1, Y1 = inputs(T)
-    st = O.init_state(W1=O.f64(W1), W2=O.f64(W2))
+    st = init()
     t0 = time.perf_counter()
     O.ttl_context(st, X1, Y1, T, hp, meta)
     one = time.perf_counter() - t0
     n_seg = int(max(1, min(n_seg_max, seconds / max(one, 1e-6))))
     X, Y = inputs(n_seg * T)
-    st = O.init_state(W1=O.f64(W1), W2=O.f64(W2))
+    st = init()
     t0 = time.perf_counter()
     O.ttl_context(st, X, Y, T, hp, meta)
     dt = time.perf_counter() - t0
@@ -262,7 +281,8 @@ def run_reference(args, wl):
 def config_of(wl):
     return {"workload": wl.name, "n_ctx": wl.n_ctx, "n_layers": wl.n_layers, "chains": wl.chains,
             "N": wl.N, "seg_T": wl.seg_T, "d_in": wl.d_in, "d_hid": wl.d_hid, "d_out": wl.d_out, "Q": wl.Q,
-            "mode": "paper" if wl.mode == 1 else "plain", "loss": wl.loss, "masters": "fp32", "operands": wl.dtype,
+            "mode": "paper" if wl.mode == 1 else "plain", "loss": wl.loss, "memory": wl.memory, "heads": wl.heads,
+            "masters": "fp32", "operands": wl.dtype,
             "l2": "inputs larger than L2 (no flush needed)"}
 
 
@@ -291,7 +311,9 @@ def run_ours(args, wl):
     strides = mone.kv_strides(wl.n_layers, wl.n_kv_heads, wl.Q, wl.head_dim)
     cfg = mone.make_config(wl.n_ctx, wl.n_layers, wl.d_in, wl.d_hid, wl.d_out, wl.n_kv_heads, wl.head_dim, wl.seg_T,
                            mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr,
-                           loss=mone.MONE_LOSS_MSE if wl.loss == "mse" else mone.MONE_LOSS_DOT)
+                           loss=mone.MONE_LOSS_MSE if wl.loss == "mse" else mone.MONE_LOSS_DOT,
+                           memory=mone.MONE_MEM_SWIGLU if wl.memory == "swiglu" else mone.MONE_MEM_MLP,
+                           mem_heads=wl.heads)
     h = mone.mone_mem_init(cfg, W1_0, W2_0, meta)
     stream = torch.cuda.current_stream()
 
@@ -467,7 +489,7 @@ def run_ours(args, wl):
         us = 1000 * t_read / n_read
         el = 2 if wl.dtype == "bf16" else 4
         # weights streamed once: the bf16 operand copy on the bf16 path, the fp32 masters on the fp32 path
-        byts = wl.chains * (wl.d_hid * (wl.d_in + wl.d_out) * el + wl.Q * (wl.d_in + wl.d_out) * el)
+        byts = wl.chains * (fast_params(wl) * el + wl.Q * (wl.d_in + wl.d_out) * el)
         gkv = {"us": us, "bytes": byts, "gbs": byts / (us * 1e-6) / 1e9, "frac_of_hbm": byts / (us * 1e-6) / 1e9 / hbm,
                "Q": wl.Q}
     if d["chains_per_launch"] < wl.chains:
@@ -480,7 +502,7 @@ def run_ours(args, wl):
         step_bytes += wl.chains * wl.N * wl.d_in * 2 * 2      # input transform: read X, write z (bf16)
     step_roof = {"bytes_per_step": step_bytes, "achieved": step_bytes / (ms / 1000) / 1e9, "peak": hbm,
                  "unit": "GB/s", "frac": step_bytes / (ms / 1000) / 1e9 / hbm}
-    total_flops = 4 * (wl.d_in * wl.d_hid + wl.d_hid * wl.d_out) * wl.N * wl.chains
+    total_flops = flops_per_token(wl) * wl.N * wl.chains
     tensor_util = total_flops / (ms / 1000) / 1e12 / tf_burst
 
     cpu = None

@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define MONE_ABI_VERSION 3
+#define MONE_ABI_VERSION 4
 
 typedef struct mone_mem mone_mem; /* opaque; created by mone_mem_init */
 
@@ -56,6 +56,7 @@ typedef enum {
 enum { MONE_FP32 = 0, MONE_BF16 = 1 };  /* dtype of X, K, V, Xq and generated K/V */
 enum { MONE_PLAIN = 0, MONE_PAPER = 1 };
 enum { MONE_LOSS_DOT = 0, MONE_LOSS_MSE = 1 };  /* per-token loss of a segment step */
+enum { MONE_MEM_MLP = 0, MONE_MEM_SWIGLU = 1 };  /* form of the memory network M */
 
 /*
  * Configuration, fixed for the life of a handle.
@@ -75,8 +76,15 @@ enum { MONE_LOSS_DOT = 0, MONE_LOSS_MSE = 1 };  /* per-token loss of a segment s
  * by two more kernels per segment).  MONE_LOSS_MSE is supported on the BF16 path;
  * on FP32 mone_mem_init returns MONE_ERR_UNSUPPORTED.
  *
+ * memory MONE_MEM_MLP: M(u) = SiLU(u W1^T) W2, W1 [d_hid][d_in], W2 [d_hid][d_out] per chain.
+ * memory MONE_MEM_SWIGLU (Eq. 3 itself): u splits into mem_heads heads of width dh = d_in / mem_heads;
+ *     head h: O_h = (SiLU(u_h Win^T) * (u_h Wg^T)) Wout with Win, Wg, Wout [d_hid][dh] (d_hid = hidden
+ *     units per head), O = [O_0 || ... ]; d_out == d_in.  Per chain W1 = [Win; Wg] for each head
+ *     ([mem_heads][2 d_hid][dh]) and W2 = Wout ([mem_heads][d_hid][dh]).  BF16 only, loss DOT only;
+ *     dh and d_hid multiples of 32 and <= 256, (d_out / 2) a multiple of dh, seg_T a multiple of 128.
+ *
  * Supported shapes: FP32: d_in, d_hid, d_out multiples of 64, seg_T multiple of 64.
- *   BF16: d_in, d_out/2, seg_T multiples of 128; d_hid a multiple of 256.  Both: head_dim in {64,128},
+ *   BF16 (MLP): d_in, d_out/2, seg_T multiples of 128; d_hid a multiple of 256.  Both: head_dim in {64,128},
  *   d_out == 2*n_kv_heads*head_dim, seg_T <= 4096.
  */
 typedef struct {
@@ -89,6 +97,8 @@ typedef struct {
     float lr;      /* plain-mode learning rate */
     float rms_eps; /* epsilon of the read-side RMSNorm (Sec. 3.2 after Eq. 4); e.g. 1e-6 */
     int loss;      /* MONE_LOSS_DOT (Eq. 7) | MONE_LOSS_MSE */
+    int memory;    /* MONE_MEM_MLP | MONE_MEM_SWIGLU */
+    int mem_heads; /* SwiGLU heads (ignored for the MLP; 0 reads as 1) */
 } mone_config;
 
 /*
@@ -105,7 +115,9 @@ typedef struct {
 /*
  * Allocate the fast-weight state of every chain and set it to W_0.
  * W1_0: [chains][d_hid][d_in] fp32, W2_0: [chains][d_hid][d_out] fp32 (device;
- * copied).  Momentum starts at 0; renormalisation targets are the row norms of
+ * copied); for MONE_MEM_SWIGLU W1_0 is [chains][mem_heads][2 d_hid][dh] ([Win; Wg]
+ * per head) and W2_0 [chains][mem_heads][d_hid][dh] (Wout); mone_mem_read_state /
+ * mone_mem_write_state use the same layouts.  Momentum starts at 0; renormalisation targets are the row norms of
  * W_0.  meta may be NULL in MONE_PLAIN mode.  On success *out owns the state.
  * Errors: INVALID_ARG, UNSUPPORTED_SHAPE, OOM, CUDA.
  */

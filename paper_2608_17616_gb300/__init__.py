@@ -19,6 +19,7 @@ LIB_PATH = os.path.join(_PKG, "libmone.so")
 MONE_FP32, MONE_BF16 = 0, 1
 MONE_PLAIN, MONE_PAPER = 0, 1
 MONE_LOSS_DOT, MONE_LOSS_MSE = 0, 1
+MONE_MEM_MLP, MONE_MEM_SWIGLU = 0, 1
 
 STATUS = {0: "MONE_OK", 1: "MONE_ERR_INVALID_ARG", 2: "MONE_ERR_UNSUPPORTED_SHAPE", 3: "MONE_ERR_OOM",
           4: "MONE_ERR_CUDA", 5: "MONE_ERR_TIMEOUT", 6: "MONE_ERR_NONFINITE", 7: "MONE_ERR_UNSUPPORTED"}
@@ -42,7 +43,8 @@ class mone_config(ctypes.Structure):
     _fields_ = [("n_ctx", ctypes.c_int), ("n_layers", ctypes.c_int), ("d_in", ctypes.c_int),
                 ("d_hid", ctypes.c_int), ("d_out", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("seg_T", ctypes.c_int), ("dtype", ctypes.c_int),
-                ("mode", ctypes.c_int), ("lr", ctypes.c_float), ("rms_eps", ctypes.c_float), ("loss", ctypes.c_int)]
+                ("mode", ctypes.c_int), ("lr", ctypes.c_float), ("rms_eps", ctypes.c_float), ("loss", ctypes.c_int),
+                ("memory", ctypes.c_int), ("mem_heads", ctypes.c_int)]
 
 
 class mone_meta(ctypes.Structure):
@@ -114,9 +116,9 @@ def _check(fn: str, rc: int):
 
 
 def make_config(n_ctx, n_layers, d_in, d_hid, d_out, n_kv_heads, head_dim, seg_T, dtype, mode, lr,
-                rms_eps=1e-6, loss=0) -> mone_config:
+                rms_eps=1e-6, loss=0, memory=0, mem_heads=1) -> mone_config:
     return mone_config(n_ctx, n_layers, d_in, d_hid, d_out, n_kv_heads, head_dim, seg_T, dtype, mode, lr, rms_eps,
-                       loss)
+                       loss, memory, mem_heads)
 
 
 def make_meta(meta: Optional[dict]) -> Optional[mone_meta]:

@@ -66,6 +66,7 @@ struct mone_mem {
     mone_config cfg;
     DevState s;
     TcMaps maps;
+    SwMaps swmaps;   // SwiGLU memory
     long long launches;
     KernelTiming* timing;
     cudaStream_t side;               // second chain group's stream (bf16 path, >= 2 chains), or null
@@ -93,6 +94,18 @@ mone_status validate_config(const mone_config* c) {
     if (c->mode != MONE_PLAIN && c->mode != MONE_PAPER) return MONE_ERR_INVALID_ARG;
     if (c->loss != MONE_LOSS_DOT && c->loss != MONE_LOSS_MSE) return MONE_ERR_INVALID_ARG;
     if (c->loss == MONE_LOSS_MSE && c->dtype != MONE_BF16) return MONE_ERR_UNSUPPORTED;
+    if (c->memory != MONE_MEM_MLP && c->memory != MONE_MEM_SWIGLU) return MONE_ERR_INVALID_ARG;
+    if (c->memory == MONE_MEM_SWIGLU) {
+        if (c->dtype != MONE_BF16 || c->loss != MONE_LOSS_DOT) return MONE_ERR_UNSUPPORTED;
+        if (c->mem_heads < 1 || c->d_in % c->mem_heads) return MONE_ERR_INVALID_ARG;
+        if (c->head_dim != 64 && c->head_dim != 128) return MONE_ERR_UNSUPPORTED_SHAPE;
+        if (c->d_out != 2 * c->n_kv_heads * c->head_dim) return MONE_ERR_UNSUPPORTED_SHAPE;
+        const int dh = c->d_in / c->mem_heads;
+        if (c->d_out != c->d_in || dh % 32 || dh > 256 || (c->d_out / 2) % dh || c->d_hid % 32 || c->d_hid > 256 ||
+            c->seg_T % 128 || c->seg_T > 4096 || (long long)c->n_ctx * c->n_layers * c->mem_heads > 65535)
+            return MONE_ERR_UNSUPPORTED_SHAPE;
+        return MONE_OK;
+    }
     if (!std::isfinite(c->lr) || !(c->rms_eps >= 0.0f) || !std::isfinite(c->rms_eps)) return MONE_ERR_INVALID_ARG;
     if (c->head_dim != 64 && c->head_dim != 128) return MONE_ERR_UNSUPPORTED_SHAPE;
     if (c->d_out != 2 * c->n_kv_heads * c->head_dim) return MONE_ERR_UNSUPPORTED_SHAPE;
@@ -161,9 +174,54 @@ void destroy_streams(mone_mem* m) {
         if (_e != cudaSuccess) return cuda_status(_e); \
     } while (0)
 
+mone_status build_swiglu_maps(mone_mem* m) {
+    DevState& s = m->s;
+    SwMaps& w = m->swmaps;
+    const uint64_t H = s.heads, dh = s.d_in / s.heads, F = s.d_hid, CH = (uint64_t)s.C * H, T = s.T;
+    bool ok = true;
+    {  // W1 = [Win; Wg] per head: (dh, F, 2, C*H)
+        const uint64_t d[4] = {dh, F, 2, CH}, st[3] = {dh * 2, F * dh * 2, 2 * F * dh * 2};
+        const uint32_t b[4] = {64, 128, 1, 1};
+        ok = ok && encode_map_bf16_4d(&w.W1a, s.W1b, d, st, b);
+    }
+    ok = ok && encode_map_bf16_3d(&w.W2a, s.W2b, dh, F, CH, 64, 128) &&
+         encode_map_bf16_3d(&w.W2m, s.W2b, dh, F, CH, 64, 64);
+    {  // phase A outputs, MN-major: (1/|z|) c [dP | dG] as (F, 2, T, C*H) and c Z as (F, T, C*H)
+        const uint64_t d[4] = {F, 2, T, CH}, st[3] = {F * 2, 2 * F * 2, T * 2 * F * 2};
+        const uint32_t b[4] = {64, 1, 64, 1};
+        ok = ok && encode_map_bf16_4d(&w.PG, s.dHt, d, st, b);
+    }
+    ok = ok && encode_map_bf16_3d(&w.Z, s.Att, F, T, CH, 64, 64);
+    if (ok && s.U) {  // input-transform window as (dh, H, rows, C)
+        const uint64_t d[4] = {dh, H, (uint64_t)s.win_rows, (uint64_t)s.C};
+        const uint64_t st[3] = {dh * 2, H * dh * 2, (uint64_t)s.win_rows * H * dh * 2};
+        const uint32_t ba[4] = {64, 1, 128, 1}, bb[4] = {64, 1, 64, 1};
+        ok = encode_map_bf16_4d(&w.Ua, s.U, d, st, ba) && encode_map_bf16_4d(&w.Ub, s.U, d, st, bb);
+    }
+    return ok ? MONE_OK : MONE_ERR_CUDA;
+}
+
+// Inputs of one call for the SwiGLU memory: head slices of X (plain mode), K and V of `chains` chains.
+mone_status build_swiglu_input_maps(const DevState& s, SwInputMaps* in, const void* X, const void* K, const void* V,
+                                    long long rows, int chains) {
+    const uint64_t H = s.heads, dh = s.d_in / s.heads, Hk = (s.d_out / 2) / dh;
+    const uint32_t ba[4] = {64, 1, 128, 1}, bb[4] = {64, 1, 64, 1};
+    const uint64_t dk[4] = {dh, Hk, (uint64_t)rows, (uint64_t)chains};
+    const uint64_t sk[3] = {dh * 2, Hk * dh * 2, (uint64_t)rows * Hk * dh * 2};
+    bool ok = encode_map_bf16_4d(&in->Ka, K, dk, sk, ba) && encode_map_bf16_4d(&in->Kb, K, dk, sk, bb) &&
+              encode_map_bf16_4d(&in->Va, V, dk, sk, ba) && encode_map_bf16_4d(&in->Vb, V, dk, sk, bb);
+    if (ok && s.mode == MONE_PLAIN) {
+        const uint64_t dx[4] = {dh, H, (uint64_t)rows, (uint64_t)chains};
+        const uint64_t sx[3] = {dh * 2, H * dh * 2, (uint64_t)rows * H * dh * 2};
+        ok = encode_map_bf16_4d(&in->Xa, X, dx, sx, ba) && encode_map_bf16_4d(&in->Xb, X, dx, sx, bb);
+    }
+    return ok ? MONE_OK : MONE_ERR_CUDA;
+}
+
 mone_status build_state_maps(mone_mem* m) {
     DevState& s = m->s;
     if (s.dtype != MONE_BF16) return MONE_OK;
+    if (s.memory == MONE_MEM_SWIGLU) return build_swiglu_maps(m);
     bool ok = encode_map_bf16_3d(&m->maps.W1b, s.W1b, s.d_in, s.d_hid, s.C, 64, 128) &&
               encode_map_bf16_3d(&m->maps.W2b, s.W2b, s.d_out, s.d_hid, s.C, 64, 128) &&
               encode_map_bf16_3d(&m->maps.W2m, s.W2b, s.d_out, s.d_hid, s.C, 64, 64) &&
@@ -232,8 +290,8 @@ mone_status timed(mone_mem* m, int kind, cudaStream_t st, int kernels, F&& fn) {
 // between launches.  The side stream forks from the caller's stream before the
 // first phase launch and joins it before every input-transform window and at
 // the end, so the call stays ordered on the caller's stream.
-mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInputMaps* rin, int G, const SegWork& w,
-                             long long N, cudaStream_t st, bool& forked) {
+mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInputMaps* rin, SwInputMaps* sin, int G,
+                             const SegWork& w, long long N, cudaStream_t st, bool& forked) {
     DevState& s = m->s;
     const cudaStream_t gs[2] = {st, m->side};
     auto join = [&]() -> mone_status {
@@ -275,7 +333,10 @@ mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInput
             x.parity = (int)(i & 1);
             x.renorm_pending = (s.renorm && i > 0) ? 1 : 0;
             x.u_off = u_off;
-            if (s.dtype == MONE_BF16 && s.loss == MONE_LOSS_MSE) {
+            if (s.memory == MONE_MEM_SWIGLU) {
+                MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_swiglu_phase_a(s, m->swmaps, sin[g], x, sg); }));
+                MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_swiglu_phase_b(s, m->swmaps, sin[g], x, sg); }));
+            } else if (s.dtype == MONE_BF16 && s.loss == MONE_LOSS_MSE) {
                 // squared error: residual targets y - M(u) at the starting weights, then the
                 // same two phases with them in place of y (dL/dO = eta (M(u) - y) / T')
                 MONE_TRY(timed(m, K_MSE, sg, 2, [&] { return launch_mse_tc(s, m->maps, gin[g], x, sg); }));
@@ -296,7 +357,10 @@ mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInput
     MONE_TRY(join());
     if (s.renorm) {
         const int par = (int)((S - 1) & 1);
-        MONE_TRY(timed(m, K_FINALIZE, st, 1, [&] { return launch_finalize(s, w.c0, w.nc, par, 1, st); }));
+        if (s.memory == MONE_MEM_SWIGLU)
+            MONE_TRY(timed(m, K_FINALIZE, st, 1, [&] { return launch_swiglu_rows(s, 1, par, w.c0, w.nc, st); }));
+        else
+            MONE_TRY(timed(m, K_FINALIZE, st, 1, [&] { return launch_finalize(s, w.c0, w.nc, par, 1, st); }));
     }
     return MONE_OK;
 }
@@ -306,6 +370,7 @@ mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
     const int G = (m->side && w.nc >= 2) ? 2 : 1;
     SegWork gw[2];
     TcInputMaps gin[2], rin[2];
+    SwInputMaps sin[2];
     const size_t el = elsize(s.dtype);
     for (int g = 0, off = 0; g < G; ++g) {
         const int n = w.nc / G + (g < w.nc % G ? 1 : 0);
@@ -319,7 +384,10 @@ mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
         if (w.loss) gw[g].loss = w.loss + off;
         std::memset(&gin[g], 0, sizeof(TcInputMaps));
         std::memset(&rin[g], 0, sizeof(TcInputMaps));
-        if (s.dtype == MONE_BF16)
+        std::memset(&sin[g], 0, sizeof(SwInputMaps));
+        if (s.memory == MONE_MEM_SWIGLU)
+            MONE_TRY(build_swiglu_input_maps(s, &sin[g], gw[g].X, gw[g].K, gw[g].V, w.n_rows, n));
+        else if (s.dtype == MONE_BF16)
             MONE_TRY(build_input_maps(s, &gin[g], gw[g].X, gw[g].K, gw[g].V, w.n_rows, n));
         if (s.dtype == MONE_BF16 && s.loss == MONE_LOSS_MSE) {
             // residual targets of this group's chains: [C][T][d_out/2] scratch, rows from 0
@@ -333,7 +401,7 @@ mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
         off += n;
     }
     bool forked = false;
-    const mone_status rc = run_segment_loop(m, gw, gin, rin, G, w, N, st, forked);
+    const mone_status rc = run_segment_loop(m, gw, gin, rin, sin, G, w, N, st, forked);
     if (forked) {
         // error after the fork: still order the side stream's work before the caller's stream
         cudaEventRecord(m->ev_join, m->side);
@@ -391,6 +459,8 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
     s.momentum = cfg->mode == MONE_PAPER; s.renorm = cfg->mode == MONE_PAPER;
     s.lr = cfg->lr; s.rms_eps = cfg->rms_eps;
     s.loss = cfg->loss;
+    s.memory = cfg->memory;
+    s.heads = cfg->memory == MONE_MEM_SWIGLU ? cfg->mem_heads : 1;
     if (s.mode == MONE_PAPER) {
         // the input transform covers a window of whole segments whose scratch stays within ~2 GiB
         const size_t row_bytes = (size_t)s.C * s.d_in * elsize(s.dtype);
@@ -398,7 +468,8 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
         segs = std::max(1ll, std::min(64ll, segs));
         s.win_rows = (int)(segs * s.T);
     }
-    const size_t C = s.C, n1 = C * s.d_hid * s.d_in, n2 = C * s.d_hid * s.d_out;
+    const size_t C = s.C, n1 = w1_elems(s), n2 = w2_elems(s);
+    const size_t r1 = w1_rows(s);  // rows of W1 over all chains (and heads): sizes the row tables
     mone_status rc = MONE_OK;
     auto step = [&](mone_status r) { if (rc == MONE_OK) rc = r; };
     step(dalloc(&s.W1, n1));
@@ -416,9 +487,9 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
             step(dalloc(&s.Vres, C * s.T * (s.d_out / 2)));
         }
     }
-    step(dalloc(&s.n1, C * s.d_hid));
-    step(dalloc(&s.n2, C * s.d_hid));
-    step(dalloc(&s.sumsq, 4 * C * s.d_hid));
+    step(dalloc(&s.n1, r1));
+    step(dalloc(&s.n2, w2_rows(s)));
+    step(dalloc(&s.sumsq, 4 * r1));
     step(dalloc(&s.status, 1));
     if (s.mode == MONE_PAPER) {
         step(dalloc(&s.alpha, C * s.d_in));
@@ -434,8 +505,9 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
     }
     if (meta && meta->gate) step(dalloc(&s.gate, C * 2 * s.n_kv));
     const size_t elt = s.dtype == MONE_BF16 ? 2 : 4;
-    step(dalloc(reinterpret_cast<uint8_t**>(&s.dHt), C * s.d_hid * s.T * elt));
-    step(dalloc(reinterpret_cast<uint8_t**>(&s.Att), C * s.d_hid * s.T * elt));
+    // phase A outputs: c dH and c A ([C][T][d_hid]); SwiGLU: c [dP | dG] ([C*H][T][2 d_hid]) and c Z
+    step(dalloc(reinterpret_cast<uint8_t**>(&s.dHt), r1 * s.T * elt));
+    step(dalloc(reinterpret_cast<uint8_t**>(&s.Att), w2_rows(s) * s.T * elt));
     auto cp = [&](void* dst, const void* src, size_t bytes) {
         if (rc == MONE_OK) rc = cuda_status(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, st));
     };
@@ -454,10 +526,14 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
         step(cuda_status(cudaMemsetAsync(s.mu1, 0, n1 * 4, st)));
         step(cuda_status(cudaMemsetAsync(s.mu2, 0, n2 * 4, st)));
     }
-    if (rc == MONE_OK) step(cuda_status(cudaMemsetAsync(s.sumsq, 0, 4 * C * s.d_hid * 4, st)));
+    if (rc == MONE_OK) step(cuda_status(cudaMemsetAsync(s.sumsq, 0, 4 * r1 * 4, st)));
     if (rc == MONE_OK) step(cuda_status(cudaMemsetAsync(s.status, 0, 4, st)));
-    if (rc == MONE_OK) step(cuda_status(launch_row_norms(s, st)));
-    if (rc == MONE_OK && s.dtype == MONE_BF16) step(cuda_status(launch_finalize(s, 0, s.C, 0, 0, st)));
+    if (s.memory == MONE_MEM_SWIGLU) {
+        if (rc == MONE_OK) step(cuda_status(launch_swiglu_rows(s, 0, 0, 0, s.C, st)));  // targets + bf16 copies
+    } else {
+        if (rc == MONE_OK) step(cuda_status(launch_row_norms(s, st)));
+        if (rc == MONE_OK && s.dtype == MONE_BF16) step(cuda_status(launch_finalize(s, 0, s.C, 0, 0, st)));
+    }
     if (rc == MONE_OK) step(build_state_maps(m));
     if (rc == MONE_OK) step(cuda_status(cudaStreamSynchronize(st)));
     if (rc != MONE_OK) {
@@ -547,11 +623,17 @@ mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out
         s.q_cap = 0;
         const size_t C = s.C;
         MONE_TRY(dalloc(&s.Uq, C * Q * s.d_in));
-        MONE_TRY(dalloc(&s.Aq, C * Q * s.d_hid));
+        MONE_TRY(dalloc(&s.Aq, C * Q * s.d_hid * s.heads));  // SwiGLU: bf16 Z_q of every head
         MONE_TRY(dalloc(&s.Oq, C * Q * s.d_out));
         s.q_cap = Q;
     }
     const int L = m->cfg.n_layers;
+    if (s.memory == MONE_MEM_SWIGLU)
+        return timed(m, K_READ, st, 4, [&] {
+            cudaError_t e = launch_query_transform(s, Xq, Q, s.Uq, true, st);
+            if (e == cudaSuccess) e = launch_swiglu_read(s, m->swmaps, s.Uq, s.Aq, Q, st);
+            return e != cudaSuccess ? e : launch_read_norm(s, Q, L, K_out, V_out, strides, st);
+        });
     if (s.dtype == MONE_BF16)
         // tensor-core read: bf16 queries and hidden activations in the fp32 scratch buffers
         return timed(m, K_READ, st, 3, [&] {
@@ -571,6 +653,11 @@ mone_status mone_mem_generate_kv_noalloc(mone_mem* m, const void* Xq, int Q, voi
     for (int i = 0; i < 4; ++i)
         if (strides[i] < 0) return MONE_ERR_INVALID_ARG;
     const DevState& s = m->s;
+    if (s.memory == MONE_MEM_SWIGLU) {
+        std::snprintf(g_last_error, sizeof(g_last_error),
+                      "mone_mem_generate_kv_noalloc: not available for the SwiGLU memory");
+        return MONE_ERR_UNSUPPORTED;
+    }
     const size_t need = (size_t)s.C * Q * ((size_t)s.d_in + s.d_hid + s.d_out);
     if (need > kNoAllocScratchFloats) {
         std::snprintf(g_last_error, sizeof(g_last_error),
@@ -621,7 +708,7 @@ mone_status mone_mem_read_state(const mone_mem* m, float* W1, float* W2, float* 
     if (!is_live(m)) return MONE_ERR_INVALID_ARG;
     const DevState& s = m->s;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    const size_t n1 = (size_t)s.C * s.d_hid * s.d_in * 4, n2 = (size_t)s.C * s.d_hid * s.d_out * 4;
+    const size_t n1 = w1_elems(s) * 4, n2 = w2_elems(s) * 4;
     if (W1) MONE_CUDA(cudaMemcpyAsync(W1, s.W1, n1, cudaMemcpyDeviceToDevice, st));
     if (W2) MONE_CUDA(cudaMemcpyAsync(W2, s.W2, n2, cudaMemcpyDeviceToDevice, st));
     if (mu1) {
@@ -640,12 +727,14 @@ mone_status mone_mem_write_state(mone_mem* m, const float* W1, const float* W2, 
     if (!is_live(m)) return MONE_ERR_INVALID_ARG;
     DevState& s = m->s;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    const size_t n1 = (size_t)s.C * s.d_hid * s.d_in * 4, n2 = (size_t)s.C * s.d_hid * s.d_out * 4;
+    const size_t n1 = w1_elems(s) * 4, n2 = w2_elems(s) * 4;
     if ((mu1 || mu2) && !s.momentum) return MONE_ERR_INVALID_ARG;
     if (W1) MONE_CUDA(cudaMemcpyAsync(s.W1, W1, n1, cudaMemcpyDeviceToDevice, st));
     if (W2) MONE_CUDA(cudaMemcpyAsync(s.W2, W2, n2, cudaMemcpyDeviceToDevice, st));
     if (mu1) MONE_CUDA(cudaMemcpyAsync(s.mu1, mu1, n1, cudaMemcpyDeviceToDevice, st));
     if (mu2) MONE_CUDA(cudaMemcpyAsync(s.mu2, mu2, n2, cudaMemcpyDeviceToDevice, st));
+    if (s.memory == MONE_MEM_SWIGLU && (W1 || W2))
+        return timed(m, K_FINALIZE, st, 1, [&] { return launch_swiglu_rows(s, 2, 0, 0, s.C, st); });
     if (s.dtype == MONE_BF16 && (W1 || W2))
         return timed(m, K_FINALIZE, st, 1, [&] { return launch_finalize(s, 0, s.C, 0, 0, st); });
     return MONE_OK;

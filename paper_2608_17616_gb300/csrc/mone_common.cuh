@@ -302,4 +302,41 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Store a warp's 32 rows x 32 bf16 columns (lane = row, `pk` = its row packed in pairs)
+// to rows row0 .. row0 + min(32, nrows) - 1 of a row-major matrix with `ld` elements per row.  The
+// chunk is transposed through the warp's 2 KB staging buffer (16-byte pieces XOR-
+// swizzled per row pair, conflict-free both ways) so that each global store
+// instruction writes 8 rows x 64 contiguous bytes instead of 32 scattered 16-byte pieces.
+__device__ __forceinline__ void store_rows_coalesced(uint8_t* stg, const uint32_t (&pk)[16], bf16* row0, int ld,
+                                                     int lane, int nrows = 32) {
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+        *reinterpret_cast<uint4*>(stg + lane * 64 + ((p ^ ((lane >> 1) & 3)) * 16)) =
+            make_uint4(pk[4 * p], pk[4 * p + 1], pk[4 * p + 2], pk[4 * p + 3]);
+    __syncwarp();
+    const int i = lane & 3;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int r = 8 * k + (lane >> 2);
+        const uint4 v = *reinterpret_cast<const uint4*>(stg + r * 64 + ((i ^ ((r >> 1) & 3)) * 16));
+        if (r < nrows) *reinterpret_cast<uint4*>(row0 + (size_t)r * ld + i * 8) = v;
+    }
+    __syncwarp();
+}
+
+// 4-D tiled bulk copy global -> shared (head slices of [..][H * dh] rows), completion on `bar`.
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* m, uint32_t bar, int x, int y, int z,
+                                            int w) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(x), "r"(y), "r"(z), "r"(w)
+        : "memory");
+}
+
 }  // namespace mone

@@ -17,6 +17,7 @@ enum : int { DEV_TIMEOUT = 1, DEV_NONFINITE = 2 };
 // Device-resident state of all chains (see mone_mem_init).
 struct DevState {
     int C, d_in, d_hid, d_out, n_kv, hd, T, dtype, mode, momentum, renorm, loss;
+    int memory, heads;            // MLP (heads 1) or per-head SwiGLU (d_hid = hidden units per head)
     float lr, rms_eps;
     float *W1, *W2, *mu1, *mu2;   // fp32 masters [C][d_hid][d_in|d_out]; mu only with momentum
     bf16 *W1b, *W2b;              // bf16 operand copies (bf16 path)
@@ -41,6 +42,17 @@ struct DevState {
     int q_cap;
     float *Uq, *Aq, *Oq;          // [C][q_cap][d_in|d_hid|d_out]
 };
+
+// Elements of the state matrices and rows per chain.  MLP: W1 [d_hid][d_in], W2 [d_hid][d_out].
+// SwiGLU: W1 [heads][2 d_hid][dh] (Win; Wg), W2 [heads][d_hid][dh] (Wout), dh = d_in / heads.
+inline size_t w1_elems(const DevState& s) {
+    return s.memory ? (size_t)s.C * s.heads * 2 * s.d_hid * (s.d_in / s.heads) : (size_t)s.C * s.d_hid * s.d_in;
+}
+inline size_t w2_elems(const DevState& s) {
+    return s.memory ? (size_t)s.C * s.heads * s.d_hid * (s.d_in / s.heads) : (size_t)s.C * s.d_hid * s.d_out;
+}
+inline size_t w1_rows(const DevState& s) { return s.memory ? (size_t)s.C * s.heads * 2 * s.d_hid : (size_t)s.C * s.d_hid; }
+inline size_t w2_rows(const DevState& s) { return s.memory ? (size_t)s.C * s.heads * s.d_hid : (size_t)s.C * s.d_hid; }
 
 inline float* sumsq_ptr(const DevState& s, int parity, int which) {
     return s.sumsq + ((size_t)(parity * 2 + which) * s.C) * s.d_hid;
@@ -85,6 +97,30 @@ struct TcMaps;
 cudaError_t launch_read_noalloc(const DevState& s, const TcMaps* tc, const void* Xq, int Q, int n_layers,
                                 void* K_out, void* V_out, const long long* strides, cudaStream_t st);
 
+// ---- kernels in swiglu_tc.cu (per-head SwiGLU memory, bf16 tcgen05 path)
+struct SwMaps {
+    CUtensorMap Ua, Ub;        // U window as (dh, heads, rows, chains): K-major {64,1,128,1}, MN {64,1,64,1}
+    CUtensorMap W1a;           // bf16 W1 as (dh, F, 2, chains*heads), K-major {64,128,1,1}
+    CUtensorMap W2a, W2m;      // bf16 W2 (dh, F, chains*heads): K-major {64,128}, MN {64 outputs, 64 hidden}
+    CUtensorMap PG, Z;         // phase A outputs, MN-major: (F, 2, T, chains*heads) {64,1,64,1}, (F, T, ..) {64,64}
+};
+struct SwInputMaps {
+    CUtensorMap Xa, Xb;        // caller's X of a group (dh, heads, rows, chains): K-major and MN boxes
+    CUtensorMap Ka, Kb, Va, Vb;  // caller's K, V (dh, heads per half, rows, chains)
+};
+cudaError_t launch_swiglu_phase_a(const DevState& s, const SwMaps& m, const SwInputMaps& in, const SegWork& w,
+                                  cudaStream_t st);
+cudaError_t launch_swiglu_phase_b(const DevState& s, const SwMaps& m, const SwInputMaps& in, const SegWork& w,
+                                  cudaStream_t st);
+// Rows of chains [c0, c0 + nc): mode 0: renormalisation targets from W (init); 1: apply the
+// pending row scales of `parity`; 2: none.  Every mode rewrites the bf16 operand copies.
+cudaError_t launch_swiglu_rows(const DevState& s, int mode, int parity, int c0, int nc, cudaStream_t st);
+// The read up to O (fp32, s.Oq): Uq bf16 [C][Q][d_in], Zq bf16 scratch [C*heads][Q][d_hid].
+cudaError_t launch_swiglu_read(const DevState& s, const SwMaps& m, const void* Uq, void* Zq, int Q, cudaStream_t st);
+// The read's per-head RMS norm and gate from s.Oq into the caller's K / V (ttl_simt.cu).
+cudaError_t launch_read_norm(const DevState& s, int Q, int n_layers, void* K_out, void* V_out,
+                             const long long* strides, cudaStream_t st);
+
 // ---- kernels in attention.cu
 cudaError_t launch_attention(const DevState& s, int n_layers, const void* Q, int n_q, int Lq, const void* K,
                              const void* V, const long long* strides, int n_mem, void* out, cudaStream_t st);
@@ -122,5 +158,8 @@ bool encode_map_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint
                         uint32_t box_inner, uint32_t box_rows);
 bool encode_map_plain_3d(CUtensorMap* map, const void* base, bool f32, uint64_t inner, uint64_t rows,
                          uint64_t chains, uint32_t box_inner, uint32_t box_rows);
+// 4-D bf16 map, 128-byte swizzle: dims[0] innermost, byte strides of dims 1..3.
+bool encode_map_bf16_4d(CUtensorMap* map, const void* base, const uint64_t dims[4], const uint64_t strides[3],
+                        const uint32_t box[4]);
 
 }  // namespace mone

@@ -377,6 +377,19 @@ cudaError_t launch_row_norms(const DevState& s, cudaStream_t st) {
     return cudaGetLastError();
 }
 
+cudaError_t launch_read_norm(const DevState& s, int Q, int n_layers, void* K_out, void* V_out,
+                             const long long* strides, cudaStream_t st) {
+    const long long jobs = (long long)s.C * Q * 2 * s.n_kv;
+    dim3 grid((unsigned)((jobs + 7) / 8));
+    if (s.dtype == 0)
+        read_norm_kernel<float><<<grid, 256, 0, st>>>(s, Q, (float*)K_out, (float*)V_out, strides[0], strides[1],
+                                                      strides[2], strides[3], n_layers);
+    else
+        read_norm_kernel<bf16><<<grid, 256, 0, st>>>(s, Q, (bf16*)K_out, (bf16*)V_out, strides[0], strides[1],
+                                                     strides[2], strides[3], n_layers);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_read(const DevState& s, int Q, int n_layers, void* K_out, void* V_out,
                         const long long* strides, cudaStream_t st) {
     read_hidden_kernel<<<dim3((Q + TM - 1) / TM, s.d_hid / TN, s.C), 256, 0, st>>>(s, Q);

@@ -124,10 +124,6 @@ __device__ __forceinline__ Ctl setup(uint8_t* raw) {
     return c;
 }
 
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<uint32_t*>(&v);
-}
 
 // ------------------------------------------------------------------ phase A
 
@@ -138,28 +134,6 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 // waits for the accumulators, then writes dH and At and adds the loss partial.
 // `release` is called by every epilogue warp once its last TMEM read of the tile is
 // done.  Returns false if the accumulator wait timed out.
-// Store a warp's 32 rows x 32 bf16 columns (lane = row, `pk` = its row packed in pairs)
-// to rows row0 .. row0 + min(32, nrows) - 1 of a row-major matrix with `ld` elements per row.  The
-// chunk is transposed through the warp's 2 KB staging buffer (16-byte pieces XOR-
-// swizzled per row pair, conflict-free both ways) so that each global store
-// instruction writes 8 rows x 64 contiguous bytes instead of 32 scattered 16-byte pieces.
-__device__ __forceinline__ void store_rows_coalesced(uint8_t* stg, const uint32_t (&pk)[16], bf16* row0, int ld,
-                                                     int lane, int nrows = 32) {
-#pragma unroll
-    for (int p = 0; p < 4; ++p)
-        *reinterpret_cast<uint4*>(stg + lane * 64 + ((p ^ ((lane >> 1) & 3)) * 16)) =
-            make_uint4(pk[4 * p], pk[4 * p + 1], pk[4 * p + 2], pk[4 * p + 3]);
-    __syncwarp();
-    const int i = lane & 3;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int r = 8 * k + (lane >> 2);
-        const uint4 v = *reinterpret_cast<const uint4*>(stg + r * 64 + ((i ^ ((r >> 1) & 3)) * 16));
-        if (r < nrows) *reinterpret_cast<uint4*>(row0 + (size_t)r * ld + i * 8) = v;
-    }
-    __syncwarp();
-}
-
 template <int BN, class Release>
 __device__ __forceinline__ bool phase_a_epilogue(const TcArgs& a, uint32_t tmem, uint32_t tfull_bar, int parity_bit,
                                                  float* tab, int* flag, int cz, int cs, int h0, int trow,
@@ -1306,6 +1280,18 @@ bool encode_map_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint
     const cuuint32_t box[3] = {box_inner, box_rows, 1};
     const cuuint32_t estr[3] = {1, 1, 1};
     return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_map_bf16_4d(CUtensorMap* map, const void* base, const uint64_t dims[4], const uint64_t strides[3],
+                        const uint32_t box[4]) {
+    if (!encoder() || !map) return false;
+    const cuuint64_t d[4] = {dims[0], dims[1], dims[2], dims[3]};
+    const cuuint64_t st[3] = {strides[0], strides[1], strides[2]};
+    const cuuint32_t b[4] = {box[0], box[1], box[2], box[3]};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), d, st, b, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }

@@ -23,7 +23,9 @@ def rel_fro(a, b) -> float:
 def config_of(wl: wk.Workload) -> "mone.mone_config":
     return mone.make_config(wl.n_ctx, wl.n_layers, wl.d_in, wl.d_hid, wl.d_out, wl.n_kv_heads, wl.head_dim,
                             wl.seg_T, mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr,
-                            loss=mone.MONE_LOSS_MSE if wl.loss == "mse" else mone.MONE_LOSS_DOT)
+                            loss=mone.MONE_LOSS_MSE if wl.loss == "mse" else mone.MONE_LOSS_DOT,
+                            memory=mone.MONE_MEM_SWIGLU if wl.memory == "swiglu" else mone.MONE_MEM_MLP,
+                            mem_heads=wl.heads)
 
 
 class GpuRun:
@@ -50,9 +52,8 @@ class GpuRun:
             pass
 
     def state(self):
-        wl = self.wl
-        W1 = torch.empty(wl.chains, wl.d_hid, wl.d_in, device=self.dev)
-        W2 = torch.empty(wl.chains, wl.d_hid, wl.d_out, device=self.dev)
+        W1 = torch.empty_like(self.W1_0)
+        W2 = torch.empty_like(self.W2_0)
         mu1 = torch.empty_like(W1)
         mu2 = torch.empty_like(W2)
         mone.mone_mem_read_state(self.h, W1, W2, mu1, mu2)
@@ -78,7 +79,22 @@ class GpuRun:
 
 
 def oracle_hyper(wl: wk.Workload) -> O.Hyper:
-    return O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss)
+    return O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss, memory=wl.memory, n_heads=wl.heads)
+
+
+def oracle_init(wl: wk.Workload, W1_0, W2_0) -> O.State:
+    """Oracle state from one chain's W_0 in the library's layout."""
+    if wl.memory == "swiglu":
+        W1 = O.f64(W1_0)
+        return O.init_state(Win=W1[:, :wl.d_hid], Wg=W1[:, wl.d_hid:], Wout=O.f64(W2_0))
+    return O.init_state(W1=O.f64(W1_0), W2=O.f64(W2_0))
+
+
+def gpu_layout(wl: wk.Workload, W: dict):
+    """(W1, W2) of an oracle weight dict in the library's layout."""
+    if wl.memory == "swiglu":
+        return np.concatenate([W["Win"], W["Wg"]], axis=1), W["Wout"]
+    return W["W1"], W["W2"]
 
 
 def oracle_meta(run: GpuRun, chain: int):
@@ -92,7 +108,7 @@ def oracle_chain(run: GpuRun, chain: int, n_tokens=None, return_all=False):
     ctx, layer = divmod(chain, wl.n_layers)
     X = O.f64(run.X[ctx, layer, :n])
     Y = np.concatenate([O.f64(run.K[ctx, layer, :n]), O.f64(run.V[ctx, layer, :n])], axis=1)
-    st = O.init_state(W1=O.f64(run.W1_0[chain]), W2=O.f64(run.W2_0[chain]))
+    st = oracle_init(wl, run.W1_0[chain], run.W2_0[chain])
     return O.ttl_context(st, X, Y, wl.seg_T, oracle_hyper(wl), oracle_meta(run, chain), return_all=return_all)
 
 

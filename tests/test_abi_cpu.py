@@ -35,7 +35,7 @@ def test_library_exports_every_declared_symbol(L):
     raw = ctypes.CDLL(mone.LIB_PATH)
     for name in header_functions():
         assert hasattr(raw, name), name
-    assert L.mone_abi_version() == 3
+    assert L.mone_abi_version() == 4
 
 
 def test_status_strings(L):
@@ -66,6 +66,18 @@ def test_init_rejects_bad_arguments_without_a_device(L):
     assert init_rc(L, cfg(lr=float("nan"))) == 1
     assert init_rc(L, cfg(mode=mone.MONE_PAPER)) == 1         # paper mode needs meta-parameters
     assert init_rc(L, cfg(loss=2)) == 1                         # no such loss
+
+
+def test_swiglu_memory_validation(L):
+    sw = dict(d_in=896, d_hid=224, d_out=896, n_kv_heads=7, head_dim=64, seg_T=128, memory=mone.MONE_MEM_SWIGLU,
+              mem_heads=4)
+    assert init_rc(L, cfg(memory=2)) == 1                                  # no such memory form
+    assert init_rc(L, cfg(**{**sw, "mem_heads": 3})) == 1                 # d_in not split evenly into heads
+    assert init_rc(L, cfg(**{**sw, "dtype": mone.MONE_FP32})) == 7        # tensor-core path only
+    assert init_rc(L, cfg(**{**sw, "loss": mone.MONE_LOSS_MSE})) == 7     # Eq. 7 loss only
+    assert init_rc(L, cfg(**{**sw, "d_hid": 300})) == 2                   # hidden units per head <= 256
+    assert init_rc(L, cfg(**{**sw, "mem_heads": 2})) == 2                 # dh = 448 > 256
+    assert init_rc(L, cfg(**{**sw, "d_out": 768, "n_kv_heads": 6})) == 2  # output width must equal d_in
 
 
 def test_squared_error_loss_is_bf16_only(L):

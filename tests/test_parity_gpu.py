@@ -12,7 +12,7 @@ import torch
 import oracle as O
 import paper_2608_17616_gb300 as mone
 import workloads as wk
-from harness import GpuRun, oracle_chain, oracle_read, rel_fro
+from harness import GpuRun, gpu_layout, oracle_chain, oracle_read, rel_fro
 
 pytestmark = pytest.mark.gpu
 
@@ -36,10 +36,11 @@ def small(mode, dtype="bf16", n_ctx=2, n_layers=2, d_in=256, d_hid=256, d_out=25
 
 def check_chain(run, chain, W1, W2, tol, n_tokens=None):
     st, _ = oracle_chain(run, chain, n_tokens)
-    e1 = rel_fro(W1[chain], st.W["W1"])
-    e2 = rel_fro(W2[chain], st.W["W2"])
-    d1 = rel_fro(W1[chain].double() - run.W1_0[chain].cpu().double(), st.W["W1"] - O.f64(run.W1_0[chain]))
-    d2 = rel_fro(W2[chain].double() - run.W2_0[chain].cpu().double(), st.W["W2"] - O.f64(run.W2_0[chain]))
+    o1, o2 = gpu_layout(run.wl, st.W)
+    e1 = rel_fro(W1[chain], o1)
+    e2 = rel_fro(W2[chain], o2)
+    d1 = rel_fro(W1[chain].double() - run.W1_0[chain].cpu().double(), o1 - O.f64(run.W1_0[chain]))
+    d2 = rel_fro(W2[chain].double() - run.W2_0[chain].cpu().double(), o2 - O.f64(run.W2_0[chain]))
     assert e1 <= tol and e2 <= tol, (chain, e1, e2)
     assert d1 <= max(tol, 5e-2) and d2 <= max(tol, 5e-2), (chain, d1, d2)
     return st

@@ -50,6 +50,8 @@ class Workload:
     mode: int                # PLAIN or PAPER
     lr: float = 1e-2
     loss: str = "neg_inner"  # "neg_inner" (Eq. 7) or "mse" (squared-error variant)
+    memory: str = "mlp"      # "mlp" (two-matrix SiLU MLP) or "swiglu" (per-head SwiGLU of Eq. 3)
+    heads: int = 1           # swiglu heads: each sees d_in / heads input dimensions, d_hid hidden units
 
     @property
     def chains(self) -> int:
@@ -76,6 +78,10 @@ WORKLOADS = {
     "l16_d2048_128k": Workload("l16_d2048_128k", 2, 1, 16, 2048, 1024, 1024, 8, 64, 512, 131072, 64, "bf16", PAPER),
     "l28_d3072_128k": Workload("l28_d3072_128k", 3, 1, 28, 3072, 2048, 2048, 8, 128, 1024, 131072, 64, "bf16", PAPER),
 }
+# The paper's own memory (Eq. 3): per-head SwiGLU, d = 896 split into 4 heads of 224 with 224
+# hidden units each, 24 layers; output [K || V] = 896 = 2 x 7 heads x 64.
+WORKLOADS["swiglu_l24_d896_32k"] = Workload("swiglu_l24_d896_32k", 5, 1, 24, 896, 224, 896, 7, 64, 512, 32768, 64,
+                                            "bf16", PAPER, memory="swiglu", heads=4)
 for _T in (256, 512, 1024, 2048):
     WORKLOADS[f"ctx8_l16_T{_T}"] = Workload(f"ctx8_l16_T{_T}", 4, 8, 16, 2048, 1024, 1024, 8, 64, _T, 32768, 64,
                                             "bf16", PAPER)
@@ -134,7 +140,18 @@ def all_inputs(wl: Workload, device="cpu", n_tokens: Optional[int] = None):
 
 
 def initial_weights(wl: Workload, device="cpu"):
-    """W1_0 [chains, d_hid, d_in] ~ N(0, 1/d_in); W2_0 [chains, d_hid, d_out] ~ N(0, 1/d_hid); fp32."""
+    """W1_0 [chains, d_hid, d_in] ~ N(0, 1/d_in); W2_0 [chains, d_hid, d_out] ~ N(0, 1/d_hid); fp32.
+
+    SwiGLU memory: W1_0 [chains, heads, 2 d_hid, dh] = [Win; Wg] per head ~ N(0, 1/dh) and
+    W2_0 [chains, heads, d_hid, dh] = Wout ~ N(0, 1/d_hid), dh = d_in / heads."""
+    if wl.memory == "swiglu":
+        H, dh, F = wl.heads, wl.d_in // wl.heads, wl.d_hid
+        W1 = torch.empty(wl.chains, H, 2 * F, dh, device=device)
+        W2 = torch.empty(wl.chains, H, F, dh, device=device)
+        for c in range(wl.chains):
+            W1[c] = torch.randn(H, 2 * F, dh, generator=_gen(wl, "w1", c, device), device=device) / math.sqrt(dh)
+            W2[c] = torch.randn(H, F, dh, generator=_gen(wl, "w2", c, device), device=device) / math.sqrt(F)
+        return W1, W2
     W1 = torch.empty(wl.chains, wl.d_hid, wl.d_in, device=device)
     W2 = torch.empty(wl.chains, wl.d_hid, wl.d_out, device=device)
     for c in range(wl.chains):
