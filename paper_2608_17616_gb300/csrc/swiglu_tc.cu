@@ -354,21 +354,27 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
             bool finite = true;
 #pragma unroll 1
             for (int cc = 0; cc < 4 && f0 + cc * 32 < a.F; ++cc) {
-                float gv[32], v[32];
+                float gv[32], v[32], mo[32];
+                // issue all 32 rows' loads before any store (the stores could alias them as far as
+                // the compiler knows, which would serialise one memory round trip per row)
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    const size_t idx = base + (size_t)(cc * 32 + j) * a.dh;
+                    v[j] = live ? W[idx] : 0.f;
+                    mo[j] = (live && a.momentum) ? M[idx] : 0.f;
+                }
                 tmem_ld32(lane_base + cc * 32, gv);
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
                     const size_t idx = base + (size_t)(cc * 32 + j) * a.dh;
-                    float wn = 0.f;
+                    const float mn = fmaf(beta, mo[j], gv[j]);
+                    const float wn = fmaf(tab[cc * 32 + j], v[j], -mn);
                     if (live) {
-                        const float mo = a.momentum ? M[idx] : 0.f;
-                        const float mn = fmaf(beta, mo, gv[j]);
-                        wn = fmaf(tab[cc * 32 + j], W[idx], -mn);
                         W[idx] = wn;
                         if (a.momentum) M[idx] = mn;
                         st_bf16_hint(Wb + idx, __float2bfloat16_rn(wn), wpol);
                     }
-                    v[j] = wn * wn;
+                    v[j] = live ? wn * wn : 0.f;
                 }
                 // transpose-reduce: afterwards lane j holds this warp's 32-column partial of row j
 #pragma unroll
@@ -525,34 +531,27 @@ swiglu_ro_kernel(const __grid_constant__ CUtensorMap tmZ, const __grid_constant_
 
 // ------------------------------------------------------------------ row upkeep (CUDA cores)
 
-// One block per state row (rows of W1 = [Win; Wg], then of W2 = Wout, per head).
+// One warp per state row (rows of W1 = [Win; Wg], then of W2 = Wout, per head), 8 rows a block.
 // mode 0: renormalisation target n = |row| (init); 1: apply the pending row scale; 2: none.
 // Every mode rewrites the row's bf16 operand copy.
 __global__ void __launch_bounds__(256) swiglu_rows_kernel(SwArgs a, int mode, int parity) {
-    const int CH = a.C * a.H;
-    const int r = blockIdx.x, ch = a.c0 * a.H + blockIdx.y, which = blockIdx.z;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int r = blockIdx.x * 8 + warp, ch = a.c0 * a.H + blockIdx.y, which = blockIdx.z;
     const int rows = which ? a.F : 2 * a.F;
-    if (r >= rows || ch >= CH) return;
+    if (r >= rows) return;
     float* W = (which ? a.W2 : a.W1) + ((size_t)ch * rows + r) * a.dh;
     bf16* Wb = (which ? a.W2b : a.W1b) + ((size_t)ch * rows + r) * a.dh;
     float* n = which ? a.n2 + (size_t)ch * a.F + r : a.n1 + (size_t)ch * 2 * a.F + r;
-    __shared__ float red[8];
-    __shared__ float sc;
+    float sc = 1.f;
     if (mode == 0) {
         float v = 0.f;
-        for (int i = threadIdx.x; i < a.dh; i += blockDim.x) v = fmaf(W[i], W[i], v);
+        for (int i = lane; i < a.dh; i += 32) v = fmaf(W[i], W[i], v);
         v = warp_sum(v);
-        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            float t = 0.f;
-            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
-            *n = sqrtf(t);
-        }
+        if (lane == 0) *n = sqrtf(v);
+    } else if (mode == 1) {
+        sc = renorm_scale(*n, sw_ss(a, parity, which, ch)[r]);
     }
-    if (threadIdx.x == 0) sc = mode == 1 ? renorm_scale(*n, sw_ss(a, parity, which, ch)[r]) : 1.f;
-    __syncthreads();
-    for (int i = threadIdx.x; i < a.dh; i += blockDim.x) {
+    for (int i = lane; i < a.dh; i += 32) {
         const float w = W[i] * sc;
         if (mode == 1) W[i] = w;
         Wb[i] = __float2bfloat16_rn(w);
@@ -621,7 +620,7 @@ cudaError_t launch_swiglu_rows(const DevState& s, int mode, int parity, int c0, 
     w.c0 = c0;
     w.nc = nc;
     SwArgs a = sw_args(s, w);
-    swiglu_rows_kernel<<<dim3(2 * a.F, nc * a.H, 2), 256, 0, st>>>(a, mode, parity);
+    swiglu_rows_kernel<<<dim3((2 * a.F + 7) / 8, nc * a.H, 2), 256, 0, st>>>(a, mode, parity);
     return cudaGetLastError();
 }
 
