@@ -32,23 +32,33 @@ namespace mone {
 
 namespace {
 
-constexpr int SW_STAGES = 4;
-constexpr int SW_STAGE = 48 * 1024;      // A tile 16 KB + up to 32 KB of B
 constexpr int SW_THREADS = 6 * 32;
 constexpr int SW_BOX = 64 * 64 * 2;      // one 64 x 64 MN-major box
 constexpr uint32_t SW_EPI_BAR = 1;
 
-struct SwLayout {
-    static constexpr int RING = SW_STAGES * SW_STAGE;
-    static constexpr int BARS = RING;    // full[S] empty[S] tfull
-    static constexpr int SLOT = BARS + 16 * 8;
+// Shared memory of one CTA: a ring of STAGES operand stages, then barriers (full[S] empty[S]
+// tfull), the TMEM slot, a flag, scale tables and (with STG) 4 epilogue warps x 2 KB
+// transpose buffers.
+template <int STAGES, int STAGE_BYTES, bool STG_BUFS>
+struct SwLayoutT {
+    static constexpr int NSTAGES = STAGES;
+    static constexpr int RING = STAGES * STAGE_BYTES;
+    static constexpr int BARS = RING;
+    static constexpr int SLOT = BARS + ((2 * STAGES + 1) * 8 + 15) / 16 * 16;
     static constexpr int FLAG = SLOT + 16;
     static constexpr int TAB = FLAG + 16;          // up to 3 x 128 scales (+ reduction scratch)
-    static constexpr int STG = TAB + 512 * 4;      // 4 epilogue warps x 2 KB transpose buffers
-    static constexpr int END = STG + 4 * 2048;
+    static constexpr int STG = TAB + 512 * 4;
+    static constexpr int END = STG + (STG_BUFS ? 4 * 2048 : 0);
     static constexpr int DYN = END + 1024;
 };
+// phase A and the read kernels: 4 stages of up to 48 KB (A tile 16 KB + up to 32 KB of B)
+using SwLayout = SwLayoutT<4, 48 * 1024, true>;
+// phase B: 2 stages of 32 KB and no transpose buffers, so that three CTAs share an SM and
+// one CTA's state update overlaps the others' operand loads and MMAs
+constexpr int SWB_CTAS_PER_SM = 3;
+using SwLayoutB = SwLayoutT<2, 4 * SW_BOX, false>;
 static_assert(SwLayout::DYN <= 227 * 1024, "shared memory budget");
+static_assert(SWB_CTAS_PER_SM * (SwLayoutB::DYN + 1024) <= 228 * 1024, "phase B CTAs per SM");
 
 struct SwArgs {
     int H, Hk, dh, F, T, Tp, C, c0, paper, momentum, renorm_pending, parity, win;
@@ -74,20 +84,22 @@ __device__ __forceinline__ float* sw_ss(const SwArgs& a, int parity, int which, 
     return a.sumsq + ((size_t)(parity * 2 + which) * a.C * a.H + ch) * (2 * a.F);
 }
 
+template <class L>
 struct SwCtl {
     uint8_t* base;
     uint32_t bars;
     __device__ uint32_t full(int s) const { return bars + 8 * s; }
-    __device__ uint32_t empty(int s) const { return bars + 8 * (SW_STAGES + s); }
-    __device__ uint32_t tfull() const { return bars + 8 * (2 * SW_STAGES); }
+    __device__ uint32_t empty(int s) const { return bars + 8 * (L::NSTAGES + s); }
+    __device__ uint32_t tfull() const { return bars + 8 * (2 * L::NSTAGES); }
 };
 
-__device__ __forceinline__ SwCtl sw_setup(uint8_t* raw, uint32_t tmem_cols) {
-    SwCtl c;
+template <class L = SwLayout>
+__device__ __forceinline__ SwCtl<L> sw_setup(uint8_t* raw, uint32_t tmem_cols) {
+    SwCtl<L> c;
     c.base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
-    c.bars = smem_u32(c.base + SwLayout::BARS);
+    c.bars = smem_u32(c.base + L::BARS);
     if (threadIdx.x == 0) {
-        for (int s = 0; s < SW_STAGES; ++s) {
+        for (int s = 0; s < L::NSTAGES; ++s) {
             mbar_init(c.full(s), 1);
             mbar_init(c.empty(s), 1);
         }
@@ -95,7 +107,7 @@ __device__ __forceinline__ SwCtl sw_setup(uint8_t* raw, uint32_t tmem_cols) {
         fence_mbar_init();
     }
     if (threadIdx.x / 32 == 0) {
-        tmem_alloc(smem_u32(c.base + SwLayout::SLOT), tmem_cols);
+        tmem_alloc(smem_u32(c.base + L::SLOT), tmem_cols);
         tmem_relinquish();
     }
     tc_fence_before();
@@ -111,8 +123,9 @@ __device__ __forceinline__ void sw_teardown(uint32_t tmem, uint32_t cols) {
 }
 
 // Epilogue entry: thread 64 waits for the accumulator, every epilogue warp learns the outcome.
-__device__ __forceinline__ bool sw_wait_acc(const SwCtl& c, int* status) {
-    int* flag = reinterpret_cast<int*>(c.base + SwLayout::FLAG);
+template <class L>
+__device__ __forceinline__ bool sw_wait_acc(const SwCtl<L>& c, int* status) {
+    int* flag = reinterpret_cast<int*>(c.base + L::FLAG);
     if (threadIdx.x == 64) *flag = mbar_wait(c.tfull(), 0, status) ? 1 : 0;
     __syncwarp();
     named_bar_sync(SW_EPI_BAR, 128);
@@ -128,7 +141,7 @@ swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmW1,
                 const __grid_constant__ CUtensorMap tmW2, const SwArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    const SwCtl c = sw_setup(smem_raw, 512);
+    const auto c = sw_setup(smem_raw, 512);
     const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + SwLayout::SLOT);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int t0 = blockIdx.x * 128, f0 = blockIdx.y * 128;
@@ -139,9 +152,9 @@ swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__
     if (warp == 0) {
         if (lane == 0) {
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SW_STAGES;
-                if (kb >= SW_STAGES && !mbar_wait(c.empty(s), ((kb / SW_STAGES) - 1) & 1, a.status)) break;
-                const uint32_t sa = smem_u32(c.base + s * SW_STAGE), sb = sa + 128 * 128, fb = c.full(s);
+                const int s = kb % SwLayout::NSTAGES;
+                if (kb >= SwLayout::NSTAGES && !mbar_wait(c.empty(s), ((kb / SwLayout::NSTAGES) - 1) & 1, a.status)) break;
+                const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128, fb = c.full(s);
                 if (kb < KU) {
                     mbar_expect_tx(fb, 3 * 128 * 128);
                     tma_load_4d(sa, &tmU, fb, kb * 64, h, a.u_row0 + t0, a.u_chain0 + cz);
@@ -164,13 +177,13 @@ swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__
             const uint32_t id_pg = idesc_bf16_f32(128, 256, false, false), id_r = idesc_bf16_f32(128, 128, false, false);
             bool ok = true;
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SW_STAGES;
-                if (!mbar_wait(c.full(s), (kb / SW_STAGES) & 1, a.status)) {
+                const int s = kb % SwLayout::NSTAGES;
+                if (!mbar_wait(c.full(s), (kb / SwLayout::NSTAGES) & 1, a.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t sa = smem_u32(c.base + s * SW_STAGE), sb = sa + 128 * 128;
+                const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128;
                 const bool u_part = kb < KU;
 #pragma unroll
                 for (int k = 0; k < 4; ++k)
@@ -260,13 +273,19 @@ swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__
 
 // ------------------------------------------------------------------ phase B (gradient + update)
 
-__global__ void __launch_bounds__(SW_THREADS, 1)
+// One tile (matrix m, 128 weight columns, 128 hidden rows, head) per CTA; three CTAs per SM
+// (two 32 KB operand stages each, 128 TMEM columns).  The update walks the tile's rows in
+// chunks of 16: every chunk's W and mu loads are issued before its stores.
+constexpr int SWB_ROWS = 16;
+
+__global__ void __launch_bounds__(SW_THREADS, SWB_CTAS_PER_SM)
 swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant__ CUtensorMap tmKb,
                 const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmPG,
                 const __grid_constant__ CUtensorMap tmZ, const SwArgs a) {
+    using L = SwLayoutB;
     extern __shared__ uint8_t smem_raw[];
-    const SwCtl c = sw_setup(smem_raw, 128);
-    const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + SwLayout::SLOT);
+    const auto c = sw_setup<L>(smem_raw, 128);
+    const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + L::SLOT);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int NC = (a.dh + 127) / 128;
     const int m = blockIdx.x / NC, col0 = (blockIdx.x % NC) * 128, f0 = blockIdx.y * 128;
@@ -277,9 +296,9 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
     if (warp == 0) {
         if (lane == 0) {
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SW_STAGES;
-                if (kb >= SW_STAGES && !mbar_wait(c.empty(s), ((kb / SW_STAGES) - 1) & 1, a.status)) break;
-                const uint32_t sa = smem_u32(c.base + s * SW_STAGE), sb = sa + 2 * SW_BOX, fb = c.full(s);
+                const int s = kb % L::NSTAGES;
+                if (kb >= L::NSTAGES && !mbar_wait(c.empty(s), ((kb / L::NSTAGES) - 1) & 1, a.status)) break;
+                const uint32_t sa = smem_u32(c.base + s * (4 * SW_BOX)), sb = sa + 2 * SW_BOX, fb = c.full(s);
                 mbar_expect_tx(fb, 4 * SW_BOX);
 #pragma unroll
                 for (int bx = 0; bx < 2; ++bx) {
@@ -303,13 +322,13 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
             const uint32_t idesc = idesc_bf16_f32(128, 128, true, true);
             bool ok = true;
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SW_STAGES;
-                if (!mbar_wait(c.full(s), (kb / SW_STAGES) & 1, a.status)) {
+                const int s = kb % L::NSTAGES;
+                if (!mbar_wait(c.full(s), (kb / L::NSTAGES) & 1, a.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t sa = smem_u32(c.base + s * SW_STAGE), sb = sa + 2 * SW_BOX;
+                const uint32_t sa = smem_u32(c.base + s * (4 * SW_BOX)), sb = sa + 2 * SW_BOX;
 #pragma unroll
                 for (int k = 0; k < 4; ++k)
                     umma_bf16(tmem, sdesc_sw128(sa + k * 16 * 128, SW_BOX), sdesc_sw128(sb + k * 16 * 128, SW_BOX),
@@ -321,7 +340,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
         __syncwarp();
     } else {
         const int q = warp & 3, et = threadIdx.x - 64;
-        float* tab = reinterpret_cast<float*>(c.base + SwLayout::TAB);  // row scales [128], beta partials [4]
+        float* tab = reinterpret_cast<float*>(c.base + L::TAB);  // row scales [128], beta partials [4]
         const int which = m < 2 ? 0 : 1;
         const int rowbase = (m < 2 ? m * a.F : 0) + f0;  // first state row of the tile (within the head)
         {
@@ -352,23 +371,24 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
             const uint64_t wpol = l2_evict_last_policy();  // phase A of the next segment reads the copy
             float* cur = sw_ss(a, a.parity, which, ch);
             bool finite = true;
+            // F is a multiple of 32, so a chunk of 16 rows is either wholly live or past F
 #pragma unroll 1
-            for (int cc = 0; cc < 4 && f0 + cc * 32 < a.F; ++cc) {
-                float gv[32], v[32], mo[32];
-                // issue all 32 rows' loads before any store (the stores could alias them as far as
-                // the compiler knows, which would serialise one memory round trip per row)
+            for (int cc = 0; cc < 128 / SWB_ROWS && f0 + cc * SWB_ROWS < a.F; ++cc) {
+                float gv[SWB_ROWS], v[SWB_ROWS], mo[SWB_ROWS];
+                // issue all the chunk's loads before any store (the stores could alias them as far
+                // as the compiler knows, which would serialise one memory round trip per row)
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const size_t idx = base + (size_t)(cc * 32 + j) * a.dh;
+                for (int j = 0; j < SWB_ROWS; ++j) {
+                    const size_t idx = base + (size_t)(cc * SWB_ROWS + j) * a.dh;
                     v[j] = live ? W[idx] : 0.f;
                     mo[j] = (live && a.momentum) ? M[idx] : 0.f;
                 }
-                tmem_ld32(lane_base + cc * 32, gv);
+                tmem_ld16(lane_base + cc * SWB_ROWS, gv);
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const size_t idx = base + (size_t)(cc * 32 + j) * a.dh;
+                for (int j = 0; j < SWB_ROWS; ++j) {
+                    const size_t idx = base + (size_t)(cc * SWB_ROWS + j) * a.dh;
                     const float mn = fmaf(beta, mo[j], gv[j]);
-                    const float wn = fmaf(tab[cc * 32 + j], v[j], -mn);
+                    const float wn = fmaf(tab[cc * SWB_ROWS + j], v[j], -mn);
                     if (live) {
                         W[idx] = wn;
                         if (a.momentum) M[idx] = mn;
@@ -376,9 +396,10 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
                     }
                     v[j] = live ? wn * wn : 0.f;
                 }
-                // transpose-reduce: afterwards lane j holds this warp's 32-column partial of row j
+                // transpose-reduce over the 16 rows: afterwards lane l holds the partial of row
+                // l & 15 over the 16 lanes that share bit 4 of l; the xor-16 exchange adds the rest
 #pragma unroll
-                for (int sft = 16; sft >= 1; sft >>= 1) {
+                for (int sft = SWB_ROWS / 2; sft >= 1; sft >>= 1) {
                     const bool upper = (lane & sft) != 0;
 #pragma unroll
                     for (int u = 0; u < sft; ++u) {
@@ -387,8 +408,9 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
                         v[u] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
                     }
                 }
+                v[0] += __shfl_xor_sync(0xffffffffu, v[0], 16);
                 finite = finite && isfinite(v[0]);
-                atomicAdd(&cur[rowbase + cc * 32 + lane], v[0]);
+                if (lane < SWB_ROWS) atomicAdd(&cur[rowbase + cc * SWB_ROWS + lane], v[0]);
             }
             if (!finite) atomicOr(a.status, DEV_NONFINITE);
         }
@@ -402,7 +424,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
 __global__ void __launch_bounds__(SW_THREADS, 1)
 swiglu_rh_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmW1, const SwArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    const SwCtl c = sw_setup(smem_raw, 256);
+    const auto c = sw_setup(smem_raw, 256);
     const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + SwLayout::SLOT);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q0 = blockIdx.x * 128, f0 = blockIdx.y * 128;
@@ -411,9 +433,9 @@ swiglu_rh_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant_
     if (warp == 0) {
         if (lane == 0) {
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SW_STAGES;
-                if (kb >= SW_STAGES && !mbar_wait(c.empty(s), ((kb / SW_STAGES) - 1) & 1, a.status)) break;
-                const uint32_t sa = smem_u32(c.base + s * SW_STAGE), sb = sa + 128 * 128, fb = c.full(s);
+                const int s = kb % SwLayout::NSTAGES;
+                if (kb >= SwLayout::NSTAGES && !mbar_wait(c.empty(s), ((kb / SwLayout::NSTAGES) - 1) & 1, a.status)) break;
+                const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128, fb = c.full(s);
                 mbar_expect_tx(fb, 3 * 128 * 128);
                 tma_load_4d(sa, &tmU, fb, kb * 64, h, q0, cl);
                 tma_load_4d(sb, &tmW1, fb, kb * 64, f0, 0, ch);
@@ -426,13 +448,13 @@ swiglu_rh_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant_
             const uint32_t idesc = idesc_bf16_f32(128, 256, false, false);
             bool ok = true;
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SW_STAGES;
-                if (!mbar_wait(c.full(s), (kb / SW_STAGES) & 1, a.status)) {
+                const int s = kb % SwLayout::NSTAGES;
+                if (!mbar_wait(c.full(s), (kb / SwLayout::NSTAGES) & 1, a.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t sa = smem_u32(c.base + s * SW_STAGE), sb = sa + 128 * 128;
+                const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128;
 #pragma unroll
                 for (int k = 0; k < 4; ++k)
                     umma_bf16(tmem, sdesc_sw128(sa + k * 32, 16), sdesc_sw128(sb + k * 32, 16), idesc,
@@ -469,7 +491,7 @@ swiglu_rh_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant_
 __global__ void __launch_bounds__(SW_THREADS, 1)
 swiglu_ro_kernel(const __grid_constant__ CUtensorMap tmZ, const __grid_constant__ CUtensorMap tmW2m, const SwArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    const SwCtl c = sw_setup(smem_raw, 128);
+    const auto c = sw_setup(smem_raw, 128);
     const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + SwLayout::SLOT);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q0 = blockIdx.x * 128, o0 = blockIdx.y * 128;
@@ -478,9 +500,9 @@ swiglu_ro_kernel(const __grid_constant__ CUtensorMap tmZ, const __grid_constant_
     if (warp == 0) {
         if (lane == 0) {
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SW_STAGES;
-                if (kb >= SW_STAGES && !mbar_wait(c.empty(s), ((kb / SW_STAGES) - 1) & 1, a.status)) break;
-                const uint32_t sa = smem_u32(c.base + s * SW_STAGE), sb = sa + 128 * 128, fb = c.full(s);
+                const int s = kb % SwLayout::NSTAGES;
+                if (kb >= SwLayout::NSTAGES && !mbar_wait(c.empty(s), ((kb / SwLayout::NSTAGES) - 1) & 1, a.status)) break;
+                const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128, fb = c.full(s);
                 mbar_expect_tx(fb, 128 * 128 + 2 * SW_BOX);
                 tma_load_3d(sa, &tmZ, fb, kb * 64, q0, ch);
                 tma_load_3d(sb, &tmW2m, fb, o0, kb * 64, ch);
@@ -493,13 +515,13 @@ swiglu_ro_kernel(const __grid_constant__ CUtensorMap tmZ, const __grid_constant_
             const uint32_t idesc = idesc_bf16_f32(128, 128, false, true);
             bool ok = true;
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SW_STAGES;
-                if (!mbar_wait(c.full(s), (kb / SW_STAGES) & 1, a.status)) {
+                const int s = kb % SwLayout::NSTAGES;
+                if (!mbar_wait(c.full(s), (kb / SwLayout::NSTAGES) & 1, a.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t sa = smem_u32(c.base + s * SW_STAGE), sb = sa + 128 * 128;
+                const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128;
 #pragma unroll
                 for (int k = 0; k < 4; ++k)
                     umma_bf16(tmem, sdesc_sw128(sa + k * 32, 16), sdesc_sw128(sb + k * 16 * 128, SW_BOX), idesc,
@@ -567,7 +589,9 @@ cudaError_t sw_attrs() {
                             reinterpret_cast<const void*>(swiglu_rh_kernel), reinterpret_cast<const void*>(swiglu_ro_kernel)};
         for (const void* k : ks)
             if (g_sw_err == cudaSuccess)
-                g_sw_err = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, SwLayout::DYN);
+                g_sw_err = cudaFuncSetAttribute(
+                    k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                    k == reinterpret_cast<const void*>(swiglu_b_kernel) ? SwLayoutB::DYN : SwLayout::DYN);
     });
     return g_sw_err;
 }
@@ -611,7 +635,7 @@ cudaError_t launch_swiglu_phase_b(const DevState& s, const SwMaps& m, const SwIn
     if (e != cudaSuccess) return e;
     const SwArgs a = sw_args(s, w);
     dim3 grid(3 * ((a.dh + 127) / 128), (a.F + 127) / 128, w.nc * a.H);
-    swiglu_b_kernel<<<grid, SW_THREADS, SwLayout::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.PG, m.Z, a);
+    swiglu_b_kernel<<<grid, SW_THREADS, SwLayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.PG, m.Z, a);
     return cudaGetLastError();
 }
 
