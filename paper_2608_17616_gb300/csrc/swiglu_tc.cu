@@ -53,10 +53,10 @@ struct SwLayoutT {
 };
 // phase A and the read kernels: 4 stages of up to 48 KB (A tile 16 KB + up to 32 KB of B)
 using SwLayout = SwLayoutT<4, 48 * 1024, true>;
-// phase B: 2 stages of 32 KB and no transpose buffers, so that three CTAs share an SM and
+// phase B: 3 stages of 32 KB and no transpose buffers, so that two CTAs share an SM and
 // one CTA's state update overlaps the others' operand loads and MMAs
-constexpr int SWB_CTAS_PER_SM = 3;
-using SwLayoutB = SwLayoutT<2, 4 * SW_BOX, false>;
+constexpr int SWB_CTAS_PER_SM = 2;
+using SwLayoutB = SwLayoutT<3, 4 * SW_BOX, false>;
 static_assert(SwLayout::DYN <= 227 * 1024, "shared memory budget");
 static_assert(SWB_CTAS_PER_SM * (SwLayoutB::DYN + 1024) <= 228 * 1024, "phase B CTAs per SM");
 
@@ -273,8 +273,8 @@ swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__
 
 // ------------------------------------------------------------------ phase B (gradient + update)
 
-// One tile (matrix m, 128 weight columns, 128 hidden rows, head) per CTA; three CTAs per SM
-// (two 32 KB operand stages each, 128 TMEM columns).  The update walks the tile's rows in
+// One tile (matrix m, 128 weight columns, 128 hidden rows, head) per CTA; two CTAs per SM
+// (three 32 KB operand stages each, 128 TMEM columns).  The update walks the tile's rows in
 // chunks of 16: every chunk's W and mu loads are issued before its stores.
 constexpr int SWB_ROWS = 16;
 
@@ -371,17 +371,28 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
             const uint64_t wpol = l2_evict_last_policy();  // phase A of the next segment reads the copy
             float* cur = sw_ss(a, a.parity, which, ch);
             bool finite = true;
-            // F is a multiple of 32, so a chunk of 16 rows is either wholly live or past F
+            // F is a multiple of 32, so a chunk of 16 rows is either wholly live or past F.  The loads
+            // of chunk cc + 1 are issued before chunk cc is updated and stored, so two chunks' loads
+            // are in flight per thread (the stores could alias them as far as the compiler knows,
+            // so it would not hoist them itself)
+            int nchunks = 0;
+            while (nchunks < 128 / SWB_ROWS && f0 + nchunks * SWB_ROWS < a.F) ++nchunks;
+            float v[SWB_ROWS], mo[SWB_ROWS];
+#pragma unroll
+            for (int j = 0; j < SWB_ROWS; ++j) {
+                const size_t idx = base + (size_t)j * a.dh;
+                v[j] = (live && nchunks > 0) ? W[idx] : 0.f;
+                mo[j] = (live && a.momentum && nchunks > 0) ? M[idx] : 0.f;
+            }
 #pragma unroll 1
-            for (int cc = 0; cc < 128 / SWB_ROWS && f0 + cc * SWB_ROWS < a.F; ++cc) {
-                float gv[SWB_ROWS], v[SWB_ROWS], mo[SWB_ROWS];
-                // issue all the chunk's loads before any store (the stores could alias them as far
-                // as the compiler knows, which would serialise one memory round trip per row)
+            for (int cc = 0; cc < nchunks; ++cc) {
+                float nv[SWB_ROWS], nmo[SWB_ROWS], gv[SWB_ROWS];
+                const bool more = cc + 1 < nchunks;
 #pragma unroll
                 for (int j = 0; j < SWB_ROWS; ++j) {
-                    const size_t idx = base + (size_t)(cc * SWB_ROWS + j) * a.dh;
-                    v[j] = live ? W[idx] : 0.f;
-                    mo[j] = (live && a.momentum) ? M[idx] : 0.f;
+                    const size_t idx = base + (size_t)((cc + 1) * SWB_ROWS + j) * a.dh;
+                    nv[j] = (live && more) ? W[idx] : 0.f;
+                    nmo[j] = (live && more && a.momentum) ? M[idx] : 0.f;
                 }
                 tmem_ld16(lane_base + cc * SWB_ROWS, gv);
 #pragma unroll
@@ -394,7 +405,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
                         if (a.momentum) M[idx] = mn;
                         st_bf16_hint(Wb + idx, __float2bfloat16_rn(wn), wpol);
                     }
-                    v[j] = live ? wn * wn : 0.f;
+                    gv[j] = live ? wn * wn : 0.f;
                 }
                 // transpose-reduce over the 16 rows: afterwards lane l holds the partial of row
                 // l & 15 over the 16 lanes that share bit 4 of l; the xor-16 exchange adds the rest
@@ -403,14 +414,19 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
                     const bool upper = (lane & sft) != 0;
 #pragma unroll
                     for (int u = 0; u < sft; ++u) {
-                        const float send = upper ? v[u] : v[u + sft];
-                        const float keep = upper ? v[u + sft] : v[u];
-                        v[u] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+                        const float send = upper ? gv[u] : gv[u + sft];
+                        const float keep = upper ? gv[u + sft] : gv[u];
+                        gv[u] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
                     }
                 }
-                v[0] += __shfl_xor_sync(0xffffffffu, v[0], 16);
-                finite = finite && isfinite(v[0]);
-                if (lane < SWB_ROWS) atomicAdd(&cur[rowbase + cc * SWB_ROWS + lane], v[0]);
+                gv[0] += __shfl_xor_sync(0xffffffffu, gv[0], 16);
+                finite = finite && isfinite(gv[0]);
+                if (lane < SWB_ROWS) atomicAdd(&cur[rowbase + cc * SWB_ROWS + lane], gv[0]);
+#pragma unroll
+                for (int j = 0; j < SWB_ROWS; ++j) {
+                    v[j] = nv[j];
+                    mo[j] = nmo[j];
+                }
             }
             if (!finite) atomicOr(a.status, DEV_NONFINITE);
         }
