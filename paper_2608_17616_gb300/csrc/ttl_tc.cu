@@ -231,6 +231,107 @@ __device__ __forceinline__ bool phase_a_epilogue(const TcArgs& a, uint32_t tmem,
     return true;
 }
 
+// The same epilogue split in two for a tile whose H accumulator (over d_in) completes before
+// its R accumulator (over d_out), the order phase A issues them in.  At = c SiLU(x) needs only
+// H, so once `hfull_bar` fires (H done, R still accumulating) the epilogue writes At and leaves
+// s' = c (1/|z|) SiLU'(x) in H's TMEM columns; once `tfull_bar` fires it forms dH = R s2 s'.
+// Only the second part runs after the main loop.  No loss partial (the caller uses
+// phase_a_epilogue when a loss is requested).
+template <int BN, class Release>
+__device__ __forceinline__ bool phase_a_epilogue_split(const TcArgs& a, uint32_t tmem, uint32_t hfull_bar,
+                                                       uint32_t tfull_bar, int parity_bit, float* tab, int* flag,
+                                                       int cz, int cs, int h0, int trow, bool zero_ss, uint8_t* stg,
+                                                       Release&& release) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int e = warp - 2, q = warp & 3, ch = e >> 2, et = threadIdx.x - 64;
+    static_assert(BN <= EPI_THREADS && BN % 64 == 0, "one scale per epilogue thread, 32-column chunks");
+    if (et < BN) {
+        const int h = h0 + et;
+        float s1 = 1.f, s2 = 1.f;
+        if (a.renorm_pending) {
+            s1 = renorm_scale(a.n1[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 0, cs)[h]);
+            s2 = renorm_scale(a.n2[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 1, cs)[h]);
+        }
+        tab[et] = s1;
+        tab[BN + et] = s2;
+        if (zero_ss) {
+            ss_row(a, a.parity, 0, cs)[h] = 0.f;
+            ss_row(a, a.parity, 1, cs)[h] = 0.f;
+        }
+    }
+    if (et == 0) *flag = mbar_wait(hfull_bar, parity_bit, a.status) ? 1 : 0;
+    __syncwarp();
+    named_bar_sync(EPI_BAR, EPI_THREADS);
+    if (!*flag) return false;
+    tc_fence_after();
+    const int row = q * 32 + lane;
+    const int t = trow + row;
+    float ct = 0.f, zi = 1.f;
+    if (t < a.Tp) {
+        const float ev = a.paper ? a.eta[(size_t)cs * a.win + a.tok0 + t]
+                                 : (a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr);
+        ct = -ev / (float)a.Tp;
+        if (a.zinv) zi = a.zinv[(size_t)cs * a.win + a.tok0 + t];
+    }
+    const float czi = ct * zi;
+    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+    const size_t r0 = ((size_t)cs * a.T + trow + q * 32) * a.d_hid + h0;  // this warp's first row
+    constexpr int CHUNKS = BN / 64;  // 32-column chunks per warp (each warp holds BN / 2 columns)
+    // ---- part 1, overlapping the R main loop: At, and s' into H's columns
+#pragma unroll 1
+    for (int cc = 0; cc < CHUNKS; ++cc) {
+        const int c0 = ch * (BN / 2) + cc * 32;
+        float hv[32];
+        tmem_ld32(lane_base + c0, hv);
+        uint32_t pa[16];
+#pragma unroll
+        for (int j = 0; j < 32; j += 4) {
+            const float4 s1v = *reinterpret_cast<const float4*>(tab + c0 + j);
+            const float s1a[4] = {s1v.x, s1v.y, s1v.z, s1v.w};
+            float av4[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float x = hv[j + u] * s1a[u] * zi;
+                const float sg = sigmoid_tanh(x);
+                av4[u] = ct * (x * sg);
+                hv[j + u] = czi * (sg * fmaf(x, 1.f - sg, 1.f));  // c_t SiLU'(x), scaled by 1/|z_t|
+            }
+            pa[j / 2] = pack_bf16(av4[0], av4[1]);
+            pa[j / 2 + 1] = pack_bf16(av4[2], av4[3]);
+        }
+        tmem_st32(lane_base + c0, hv);
+        store_rows_coalesced(stg, pa, a.At + r0 + c0, a.d_hid, lane);
+    }
+    tmem_wait_st();
+    // ---- part 2, after the main loop: dH = R s2 s'
+    if (et == 0) flag[2] = mbar_wait(tfull_bar, parity_bit, a.status) ? 1 : 0;
+    __syncwarp();
+    named_bar_sync(EPI_BAR, EPI_THREADS);
+    if (!flag[2]) return false;
+    tc_fence_after();
+#pragma unroll 1
+    for (int cc = 0; cc < CHUNKS; ++cc) {
+        const int c0 = ch * (BN / 2) + cc * 32;
+        float sp[32], rv[32];
+        tmem_ld32(lane_base + c0, sp);
+        tmem_ld32(lane_base + BN + c0, rv);
+        if (cc == CHUNKS - 1) {
+            tc_fence_before();
+            __syncwarp();
+            release();
+        }
+        uint32_t pd[16];
+#pragma unroll
+        for (int j = 0; j < 32; j += 4) {
+            const float4 s2v = *reinterpret_cast<const float4*>(tab + BN + c0 + j);
+            pd[j / 2] = pack_bf16(rv[j] * s2v.x * sp[j], rv[j + 1] * s2v.y * sp[j + 1]);
+            pd[j / 2 + 1] = pack_bf16(rv[j + 2] * s2v.z * sp[j + 2], rv[j + 3] * s2v.w * sp[j + 3]);
+        }
+        store_rows_coalesced(stg, pd, a.dH + r0 + c0, a.d_hid, lane);
+    }
+    return true;
+}
+
 __global__ void __launch_bounds__(THREADS, 1)
 tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmW1,
@@ -352,8 +453,8 @@ struct LP {
     static constexpr int BARS = RING;  // full[S] empty[S] tfull[2] tempty[2]
     static constexpr int NBARS = 2 * P_STAGES + 4;
     static constexpr int SLOT = BARS + NBARS * 8;
-    static constexpr int FLAG = SLOT + 16;
-    static constexpr int TAB = FLAG + 16;               // scale tables of two consecutive tiles
+    static constexpr int FLAG = SLOT + 16;              // 2 tiles x 4 flags
+    static constexpr int TAB = FLAG + 32;               // scale tables of two consecutive tiles
     static constexpr int STG = TAB + 4 * P_BN * 4;      // per epilogue warp: 32 x 64 B transpose buffer
     static constexpr int END = STG + EPI_WARPS * 2048;
     static constexpr int DYN = END + 1024;
@@ -383,6 +484,7 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
             mbar_init(c.empty(i, P_STAGES), 1);
         }
         mbar_init(c.tfull(0, P_STAGES), 1);
+        mbar_init(c.tfull(1, P_STAGES), 1);  // H accumulator complete (R still accumulating)
         mbar_init(c.tempty(0, P_STAGES), 2 * EPI_WARPS);
         fence_mbar_init();
     }
@@ -467,6 +569,7 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
                         umma_bf16_pair(kb < KB1 ? dH : dR, sdesc_sw128(sa + k * 32, 16),
                                        sdesc_sw128(sb + k * 32, 16), idesc, (first && k == 0) ? 0u : 1u);
                     umma_commit_pair(c.empty(s, P_STAGES), 0x3);
+                    if (kb == KB1 - 1) umma_commit_pair(c.tfull(1, P_STAGES), 0x3);  // H complete
                 }
                 if (!ok) break;
                 umma_commit_pair(c.tfull(0, P_STAGES), 0x3);
@@ -484,12 +587,18 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
             const int tt = tp * 2 + (int)rank;
             // the scale table and flag alternate between tiles: a warp may start the next
             // tile while another still reads this one's table
-            if (!phase_a_epilogue<P_BN>(a, tmem, c.tfull(0, P_STAGES), local & 1, table + (local & 1) * 2 * P_BN,
-                                        flag + (local & 1), cz, a.c0 + cz, ht * P_BN, tt * A_BM, tt == 0,
-                                        c.base + LP::STG + (warp - 2) * 2048, [&] {
-                                            if (lane == 0) mbar_arrive_remote(tempty0);
-                                        }))
-                break;
+            auto release = [&] {
+                if (lane == 0) mbar_arrive_remote(tempty0);
+            };
+            float* tab = table + (local & 1) * 2 * P_BN;
+            int* fl = flag + (local & 1) * 4;
+            uint8_t* stg = c.base + LP::STG + (warp - 2) * 2048;
+            const bool ok = a.loss ? phase_a_epilogue<P_BN>(a, tmem, c.tfull(0, P_STAGES), local & 1, tab, fl, cz,
+                                                             a.c0 + cz, ht * P_BN, tt * A_BM, tt == 0, stg, release)
+                                   : phase_a_epilogue_split<P_BN>(a, tmem, c.tfull(1, P_STAGES), c.tfull(0, P_STAGES),
+                                                                  local & 1, tab, fl, cz, a.c0 + cz, ht * P_BN,
+                                                                  tt * A_BM, tt == 0, stg, release);
+            if (!ok) break;
         }
     }
     tc_fence_before();
