@@ -959,7 +959,10 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
 // lane quarter, lane = query) run the epilogue.  Each weight tile is read by ceil(Q/128)
 // CTAs; query rows >= Q arrive as TMA zero fill and are never stored.  W2 is [hidden][out],
 // so in the out kernel the weight operand is MN-major (64-column boxes, as in phase B).
-constexpr int R_STAGES = 4;
+// Two CTAs share an SM (three 32 KB stages each), so one CTA's epilogue overlaps the other's
+// loads when a read has more tiles than SMs.
+constexpr int R_STAGES = 3;
+constexpr int R_CTAS_PER_SM = 2;
 constexpr int R_STAGE = 2 * 128 * BK * 2;  // 32 KB: 128 query rows + 128 weight rows / columns
 constexpr int R_THREADS = 6 * 32;
 constexpr uint32_t R_EPI_BAR = 1;
@@ -974,6 +977,7 @@ struct LR {
     static constexpr int END = STG + 4 * 2048;
     static constexpr int DYN = END + 1024;
 };
+static_assert(R_CTAS_PER_SM * (LR::DYN + 1024) <= 228 * 1024, "read kernel CTAs per SM");
 static_assert(LR::STG % 16 == 0, "staging buffers hold 16-byte pieces");
 
 struct ReadArgs {
@@ -1003,7 +1007,7 @@ enum { READ_HIDDEN = 0, MSE_HIDDEN = 1, MSE_OUT = 2 };  // other MODEs: read out
 // with the pending renorm scales (s2 folded in, so A' W2raw = A W2).  MODE MSE_OUT: the
 // residual target y_t - M(u_t) = y_t - A'_t W2raw (and the segment's squared-error loss).
 template <int MODE>
-__global__ void __launch_bounds__(R_THREADS, 1)
+__global__ void __launch_bounds__(R_THREADS, R_CTAS_PER_SM)
 tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const ReadArgs a) {
     constexpr bool OUT = MODE != READ_HIDDEN && MODE != MSE_HIDDEN;
     extern __shared__ uint8_t smem_raw[];
