@@ -317,13 +317,18 @@ def test_bf16_mse_chain_groups_match_one_chain_handles():
 
 # ----------------------------------------------------------------- full-size workloads, sampled chains
 
+# Every workload at its full context length (n_tokens None) in the launch configuration the
+# bench times (all chains of the workload in one handle, two chain groups), the oracle
+# replaying the sampled chains; the squared-error variant on a 16-segment prefix.
 @pytest.mark.parametrize("name,chains,n_tokens,loss", [
     ("l16_d2048_128k", (0, 15), None, "neg_inner"),
     ("l16_d2048_128k", (9,), 8192, "mse"),
     ("l16_d2048_32k", (7,), None, "neg_inner"),
-    ("l28_d3072_128k", (27,), 16 * 1024, "neg_inner"),
-    ("ctx8_l16_T256", (77,), 8192, "neg_inner"),
-    ("ctx8_l16_T2048", (5,), 8192, "neg_inner"),
+    ("l28_d3072_128k", (27,), None, "neg_inner"),
+    ("ctx8_l16_T256", (77,), None, "neg_inner"),
+    ("ctx8_l16_T512", (0, 127), None, "neg_inner"),
+    ("ctx8_l16_T1024", (64,), None, "neg_inner"),
+    ("ctx8_l16_T2048", (5,), None, "neg_inner"),
 ])
 def test_full_size_sampled_chains(name, chains, n_tokens, loss):
     wl = wk.WORKLOADS[name].replace(loss=loss)
