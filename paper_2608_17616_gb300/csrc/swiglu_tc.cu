@@ -37,14 +37,14 @@ constexpr int SW_BOX = 64 * 64 * 2;      // one 64 x 64 MN-major box
 constexpr uint32_t SW_EPI_BAR = 1;
 
 // Shared memory of one CTA: a ring of STAGES operand stages, then barriers (full[S] empty[S]
-// tfull), the TMEM slot, a flag, scale tables and (with STG) 4 epilogue warps x 2 KB
+// tfull tempty), the TMEM slot, a flag, scale tables and (with STG) 4 epilogue warps x 2 KB
 // transpose buffers.
 template <int STAGES, int STAGE_BYTES, bool STG_BUFS>
 struct SwLayoutT {
     static constexpr int NSTAGES = STAGES;
     static constexpr int RING = STAGES * STAGE_BYTES;
     static constexpr int BARS = RING;
-    static constexpr int SLOT = BARS + ((2 * STAGES + 1) * 8 + 15) / 16 * 16;
+    static constexpr int SLOT = BARS + ((2 * STAGES + 2) * 8 + 15) / 16 * 16;
     static constexpr int FLAG = SLOT + 16;
     static constexpr int TAB = FLAG + 16;          // up to 3 x 128 scales (+ reduction scratch)
     static constexpr int STG = TAB + 512 * 4;
@@ -76,6 +76,7 @@ struct SwArgs {
     int* status;
     // memory read
     int Q, d_out;
+    int nc_launch;           // chains of this launch (persistent phase A)
     bf16* Zq;                // [C*H][Q][F]
     float* Oq;               // [C][Q][d_out]
 };
@@ -91,6 +92,7 @@ struct SwCtl {
     __device__ uint32_t full(int s) const { return bars + 8 * s; }
     __device__ uint32_t empty(int s) const { return bars + 8 * (L::NSTAGES + s); }
     __device__ uint32_t tfull() const { return bars + 8 * (2 * L::NSTAGES); }
+    __device__ uint32_t tempty() const { return bars + 8 * (2 * L::NSTAGES + 1); }
 };
 
 template <class L = SwLayout>
@@ -104,6 +106,7 @@ __device__ __forceinline__ SwCtl<L> sw_setup(uint8_t* raw, uint32_t tmem_cols) {
             mbar_init(c.empty(s), 1);
         }
         mbar_init(c.tfull(), 1);
+        mbar_init(c.tempty(), 4);  // the four epilogue warps (persistent phase A)
         fence_mbar_init();
     }
     if (threadIdx.x / 32 == 0) {
@@ -136,6 +139,12 @@ __device__ __forceinline__ bool sw_wait_acc(const SwCtl<L>& c, int* status) {
 
 // ------------------------------------------------------------------ phase A (forward + backward epilogue)
 
+// Persistent: at most one CTA per SM walks the tiles (128 tokens, 128 hidden units, head) of
+// the launch.  The producer runs ahead into the next tile's operands while the epilogue
+// drains the current one; the MMA warp waits for the epilogue to hand the accumulator back
+// (tempty) before it starts the next tile.  (Two accumulator buffers would need 768 TMEM
+// columns; 64-unit tiles that fit two buffers reload U and Y twice as often and measured
+// slower.)
 __global__ void __launch_bounds__(SW_THREADS, 1)
 swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmW1,
@@ -144,30 +153,48 @@ swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__
     const auto c = sw_setup(smem_raw, 512);
     const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + SwLayout::SLOT);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int t0 = blockIdx.x * 128, f0 = blockIdx.y * 128;
-    const int cz = blockIdx.z / a.H, h = blockIdx.z % a.H;
-    const int cs = a.c0 + cz, ch = cs * a.H + h;
     const int KU = (a.dh + 63) / 64, KB = 2 * KU;
+    const int n_tt = a.T / 128, n_ft = (a.F + 127) / 128;
+    const int ntiles = n_tt * n_ft * a.nc_launch * a.H;
+    // tile -> (token tile, hidden tile, chain-head of the launch)
+    auto decode = [&](int tile, int& t0, int& f0, int& cz, int& h) {
+        const int zh = tile / (n_tt * n_ft), r = tile % (n_tt * n_ft);
+        f0 = (r / n_tt) * 128;
+        t0 = (r % n_tt) * 128;
+        cz = zh / a.H;
+        h = zh % a.H;
+    };
 
     if (warp == 0) {
         if (lane == 0) {
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SwLayout::NSTAGES;
-                if (kb >= SwLayout::NSTAGES && !mbar_wait(c.empty(s), ((kb / SwLayout::NSTAGES) - 1) & 1, a.status)) break;
-                const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128, fb = c.full(s);
-                if (kb < KU) {
-                    mbar_expect_tx(fb, 3 * 128 * 128);
-                    tma_load_4d(sa, &tmU, fb, kb * 64, h, a.u_row0 + t0, a.u_chain0 + cz);
-                    tma_load_4d(sb, &tmW1, fb, kb * 64, f0, 0, ch);             // Win rows
-                    tma_load_4d(sb + 128 * 128, &tmW1, fb, kb * 64, f0, 1, ch);  // Wg rows
-                } else {
-                    const int k2 = kb - KU;
-                    mbar_expect_tx(fb, 2 * 128 * 128);
-                    if (h < a.Hk)
-                        tma_load_4d(sa, &tmK, fb, k2 * 64, h, a.y_row0 + t0, cz);
-                    else
-                        tma_load_4d(sa, &tmV, fb, k2 * 64, h - a.Hk, a.y_row0 + t0, cz);
-                    tma_load_3d(sb, &tmW2, fb, k2 * 64, f0, ch);                 // Wout rows
+            uint32_t kc = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+                int t0, f0, cz, h;
+                decode(tile, t0, f0, cz, h);
+                const int ch = (a.c0 + cz) * a.H + h;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % SwLayout::NSTAGES;
+                    if (kc >= SwLayout::NSTAGES &&
+                        !mbar_wait(c.empty(s), ((kc / SwLayout::NSTAGES) - 1) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128, fb = c.full(s);
+                    if (kb < KU) {
+                        mbar_expect_tx(fb, 3 * 128 * 128);
+                        tma_load_4d(sa, &tmU, fb, kb * 64, h, a.u_row0 + t0, a.u_chain0 + cz);
+                        tma_load_4d(sb, &tmW1, fb, kb * 64, f0, 0, ch);             // Win rows
+                        tma_load_4d(sb + 128 * 128, &tmW1, fb, kb * 64, f0, 1, ch);  // Wg rows
+                    } else {
+                        const int k2 = kb - KU;
+                        mbar_expect_tx(fb, 2 * 128 * 128);
+                        if (h < a.Hk)
+                            tma_load_4d(sa, &tmK, fb, k2 * 64, h, a.y_row0 + t0, cz);
+                        else
+                            tma_load_4d(sa, &tmV, fb, k2 * 64, h - a.Hk, a.y_row0 + t0, cz);
+                        tma_load_3d(sb, &tmW2, fb, k2 * 64, f0, ch);                 // Wout rows
+                    }
                 }
             }
         }
@@ -175,97 +202,121 @@ swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__
     } else if (warp == 1) {
         if (lane == 0) {
             const uint32_t id_pg = idesc_bf16_f32(128, 256, false, false), id_r = idesc_bf16_f32(128, 128, false, false);
+            uint32_t kc = 0;
+            int local = 0;
             bool ok = true;
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % SwLayout::NSTAGES;
-                if (!mbar_wait(c.full(s), (kb / SwLayout::NSTAGES) & 1, a.status)) {
-                    ok = false;
-                    break;
-                }
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++local) {
+                if (local >= 1 && !mbar_wait(c.tempty(), (local - 1) & 1, a.status)) break;
                 tc_fence_after();
-                const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128;
-                const bool u_part = kb < KU;
-#pragma unroll
-                for (int k = 0; k < 4; ++k)
-                    umma_bf16(u_part ? tmem : tmem + 256, sdesc_sw128(sa + k * 32, 16), sdesc_sw128(sb + k * 32, 16),
-                              u_part ? id_pg : id_r, ((kb == 0 || kb == KU) && k == 0) ? 0u : 1u);
-                umma_commit(c.empty(s));
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % SwLayout::NSTAGES;
+                    if (!mbar_wait(c.full(s), (kc / SwLayout::NSTAGES) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(c.base + s * (48 * 1024)), sb = sa + 128 * 128;
+                    const bool u_part = kb < KU;
+    #pragma unroll
+                    for (int k = 0; k < 4; ++k)
+                        umma_bf16(u_part ? tmem : tmem + 256, sdesc_sw128(sa + k * 32, 16), sdesc_sw128(sb + k * 32, 16),
+                                  u_part ? id_pg : id_r, ((kb == 0 || kb == KU) && k == 0) ? 0u : 1u);
+                    umma_commit(c.empty(s));
+                }
+                if (ok) umma_commit(c.tfull());
             }
-            if (ok) umma_commit(c.tfull());
         }
         __syncwarp();
     } else {
         const int q = warp & 3, et = threadIdx.x - 64;
         float* tab = reinterpret_cast<float*>(c.base + SwLayout::TAB);  // s_in[128] s_g[128] s_out[128]
-        {
-            const int f = f0 + et;
-            float si = 1.f, sg = 1.f, so = 1.f;
-            if (f < a.F) {
-                if (a.renorm_pending) {
-                    si = renorm_scale(a.n1[(size_t)ch * 2 * a.F + f], sw_ss(a, a.parity ^ 1, 0, ch)[f]);
-                    sg = renorm_scale(a.n1[(size_t)ch * 2 * a.F + a.F + f], sw_ss(a, a.parity ^ 1, 0, ch)[a.F + f]);
-                    so = renorm_scale(a.n2[(size_t)ch * a.F + f], sw_ss(a, a.parity ^ 1, 1, ch)[f]);
-                }
-                if (t0 == 0) {  // this segment's row sums of squares start from zero
-                    sw_ss(a, a.parity, 0, ch)[f] = 0.f;
-                    sw_ss(a, a.parity, 0, ch)[a.F + f] = 0.f;
-                    sw_ss(a, a.parity, 1, ch)[f] = 0.f;
-                }
-            }
-            tab[et] = si;
-            tab[128 + et] = sg;
-            tab[256 + et] = so;
-        }
-        if (sw_wait_acc(c, a.status)) {
-            const int t = t0 + q * 32 + lane;
-            float ct = 0.f, zi = 1.f;
-            if (t < a.Tp) {
-                const float ev = a.paper ? a.eta[(size_t)cs * a.win + a.tok0 + t]
-                                         : (a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr);
-                ct = -ev / (float)a.Tp;
-                if (a.zinv) zi = a.zinv[(size_t)cs * a.win + a.tok0 + t];
-            }
-            const float czi = ct * zi;
-            const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
-            uint8_t* stg = c.base + SwLayout::STG + (warp - 2) * 2048;
-            const size_t rowoff = (size_t)ch * a.T + t0 + q * 32;  // first token row of this warp
-            float lsum = 0.f;
-#pragma unroll 1
-            for (int cc = 0; cc < 4 && f0 + cc * 32 < a.F; ++cc) {
-                const int fb = cc * 32;
-                float pv[32], gv[32], rv[32];
-                tmem_ld32(lane_base + fb, pv);
-                tmem_ld32(lane_base + 128 + fb, gv);
-                tmem_ld32(lane_base + 256 + fb, rv);
-                uint32_t pd[16], pg[16], pz[16];
-#pragma unroll
-                for (int j = 0; j < 32; j += 2) {
-                    float d0[2], d1[2], d2[2];
-#pragma unroll
-                    for (int u = 0; u < 2; ++u) {
-                        const int k = fb + j + u;
-                        const float x = pv[j + u] * tab[k] * zi;
-                        const float g = gv[j + u] * tab[128 + k] * zi;
-                        const float r = rv[j + u] * tab[256 + k];
-                        const float sgm = sigmoid_tanh(x);
-                        const float sl = x * sgm;
-                        lsum = fmaf(sl * g, r, lsum);
-                        d0[u] = czi * r * g * (sgm * fmaf(x, 1.f - sgm, 1.f));  // (1/|z|) c dP
-                        d1[u] = czi * r * sl;                                   // (1/|z|) c dG
-                        d2[u] = ct * sl * g;                                    // c Z
+        int* flag = reinterpret_cast<int*>(c.base + SwLayout::FLAG);
+        int local = 0;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local) {
+            int t0, f0, cz, h;
+            decode(tile, t0, f0, cz, h);
+            const int cs = a.c0 + cz, ch = cs * a.H + h;
+            {
+                const int f = f0 + et;
+                float si = 1.f, sg = 1.f, so = 1.f;
+                if (f < a.F) {
+                    if (a.renorm_pending) {
+                        si = renorm_scale(a.n1[(size_t)ch * 2 * a.F + f], sw_ss(a, a.parity ^ 1, 0, ch)[f]);
+                        sg = renorm_scale(a.n1[(size_t)ch * 2 * a.F + a.F + f], sw_ss(a, a.parity ^ 1, 0, ch)[a.F + f]);
+                        so = renorm_scale(a.n2[(size_t)ch * a.F + f], sw_ss(a, a.parity ^ 1, 1, ch)[f]);
                     }
-                    pd[j / 2] = pack_bf16(d0[0], d0[1]);
-                    pg[j / 2] = pack_bf16(d1[0], d1[1]);
-                    pz[j / 2] = pack_bf16(d2[0], d2[1]);
+                    if (t0 == 0) {  // this segment's row sums of squares start from zero
+                        sw_ss(a, a.parity, 0, ch)[f] = 0.f;
+                        sw_ss(a, a.parity, 0, ch)[a.F + f] = 0.f;
+                        sw_ss(a, a.parity, 1, ch)[f] = 0.f;
+                    }
                 }
-                store_rows_coalesced(stg, pd, a.dPG + rowoff * 2 * a.F + f0 + fb, 2 * a.F, lane);
-                store_rows_coalesced(stg, pg, a.dPG + rowoff * 2 * a.F + a.F + f0 + fb, 2 * a.F, lane);
-                store_rows_coalesced(stg, pz, a.Zt + rowoff * a.F + f0 + fb, a.F, lane);
+                tab[et] = si;
+                tab[128 + et] = sg;
+                tab[256 + et] = so;
             }
-            if (a.loss) {
-                lsum = warp_sum(lsum);
-                if (lane == 0) atomicAdd(&a.loss[cz], -lsum / (float)a.Tp);
+            if (et == 0) *flag = mbar_wait(c.tfull(), local & 1, a.status) ? 1 : 0;
+            __syncwarp();
+            named_bar_sync(SW_EPI_BAR, 128);
+            if (!*flag) break;
+            tc_fence_after();
+            {
+                const int t = t0 + q * 32 + lane;
+                float ct = 0.f, zi = 1.f;
+                if (t < a.Tp) {
+                    const float ev = a.paper ? a.eta[(size_t)cs * a.win + a.tok0 + t]
+                                             : (a.eta_in ? a.eta_in[cz * a.eta_cstride + t] : a.lr);
+                    ct = -ev / (float)a.Tp;
+                    if (a.zinv) zi = a.zinv[(size_t)cs * a.win + a.tok0 + t];
+                }
+                const float czi = ct * zi;
+                const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+                uint8_t* stg = c.base + SwLayout::STG + (warp - 2) * 2048;
+                const size_t rowoff = (size_t)ch * a.T + t0 + q * 32;  // first token row of this warp
+                float lsum = 0.f;
+    #pragma unroll 1
+                for (int cc = 0; cc < 4 && f0 + cc * 32 < a.F; ++cc) {
+                    const int fb = cc * 32;
+                    float pv[32], gv[32], rv[32];
+                    tmem_ld32(lane_base + fb, pv);
+                    tmem_ld32(lane_base + 128 + fb, gv);
+                    tmem_ld32(lane_base + 256 + fb, rv);
+                    uint32_t pd[16], pg[16], pz[16];
+    #pragma unroll
+                    for (int j = 0; j < 32; j += 2) {
+                        float d0[2], d1[2], d2[2];
+    #pragma unroll
+                        for (int u = 0; u < 2; ++u) {
+                            const int k = fb + j + u;
+                            const float x = pv[j + u] * tab[k] * zi;
+                            const float g = gv[j + u] * tab[128 + k] * zi;
+                            const float r = rv[j + u] * tab[256 + k];
+                            const float sgm = sigmoid_tanh(x);
+                            const float sl = x * sgm;
+                            lsum = fmaf(sl * g, r, lsum);
+                            d0[u] = czi * r * g * (sgm * fmaf(x, 1.f - sgm, 1.f));  // (1/|z|) c dP
+                            d1[u] = czi * r * sl;                                   // (1/|z|) c dG
+                            d2[u] = ct * sl * g;                                    // c Z
+                        }
+                        pd[j / 2] = pack_bf16(d0[0], d0[1]);
+                        pg[j / 2] = pack_bf16(d1[0], d1[1]);
+                        pz[j / 2] = pack_bf16(d2[0], d2[1]);
+                    }
+                    store_rows_coalesced(stg, pd, a.dPG + rowoff * 2 * a.F + f0 + fb, 2 * a.F, lane);
+                    store_rows_coalesced(stg, pg, a.dPG + rowoff * 2 * a.F + a.F + f0 + fb, 2 * a.F, lane);
+                    store_rows_coalesced(stg, pz, a.Zt + rowoff * a.F + f0 + fb, a.F, lane);
+                }
+                // every TMEM read of this tile is done: hand the accumulator back to the MMA warp
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(c.tempty());
+                if (a.loss) {
+                    lsum = warp_sum(lsum);
+                    if (lane == 0) atomicAdd(&a.loss[cz], -lsum / (float)a.Tp);
+                }
             }
+            // the scale table and flag are rewritten for the next tile only after every warp is done
+            named_bar_sync(SW_EPI_BAR, 128);
         }
     }
     sw_teardown(tmem, 512);
@@ -596,6 +647,19 @@ __global__ void __launch_bounds__(256) swiglu_rows_kernel(SwArgs a, int mode, in
     }
 }
 
+// SM count of the current device (grid of the persistent phase A).
+int sw_sms() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0, v = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) !=
+                                                      cudaSuccess || v <= 0)
+            return 1;
+        n = v;
+    }
+    return n;
+}
+
 std::once_flag g_sw_once;
 cudaError_t g_sw_err = cudaSuccess;
 
@@ -639,8 +703,10 @@ cudaError_t launch_swiglu_phase_a(const DevState& s, const SwMaps& m, const SwIn
                                   cudaStream_t st) {
     cudaError_t e = sw_attrs();
     if (e != cudaSuccess) return e;
-    const SwArgs a = sw_args(s, w);
-    dim3 grid(s.T / 128, (a.F + 127) / 128, w.nc * a.H);
+    SwArgs a = sw_args(s, w);
+    a.nc_launch = w.nc;
+    const int ntiles = (s.T / 128) * ((a.F + 127) / 128) * w.nc * a.H;
+    const int grid = ntiles < sw_sms() ? ntiles : sw_sms();
     swiglu_a_kernel<<<grid, SW_THREADS, SwLayout::DYN, st>>>(s.mode == 1 ? m.Ua : in.Xa, in.Ka, in.Va, m.W1a, m.W2a, a);
     return cudaGetLastError();
 }
