@@ -108,9 +108,16 @@ def kernel_source_sha(text, kind):
     return hashlib.sha256(text[i:j].encode()).hexdigest()[:16]
 
 
-def ncu_traffic(kind, chains):
+def shape_key(wl):
+    """The per-chain shape a DRAM-traffic record holds for (widths, segment, memory form, mode, loss)."""
+    return (f"{wl.d_in}x{wl.d_hid}x{wl.d_out}:T{wl.seg_T}:{wl.memory}:{'paper' if wl.mode == 1 else 'plain'}:"
+            f"{wl.loss}")
+
+
+def ncu_traffic(kind, chains, wl):
     """DRAM bytes per launch of `chains` chains from the committed ncu summary (scaled from the
-    captured launch's chain count), if the kernel source is unchanged."""
+    captured launch's chain count), if the kernel source is unchanged and the record was taken
+    on this per-chain shape."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
     src = os.path.join(ROOT, "paper_2608_17616_gb300", "csrc", "ttl_tc.cu")
     try:
@@ -119,7 +126,8 @@ def ncu_traffic(kind, chains):
             if line.lstrip().startswith("#"):
                 continue
             parts = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
-            if parts.get("kernel") == kind and parts.get("source_sha") == sha:
+            if (parts.get("kernel") == kind and parts.get("source_sha") == sha
+                    and parts.get("shape") == shape_key(wl)):
                 cap = float(parts.get("chains", chains))
                 note = parts.get("scaled_from", "")
                 if abs(cap - chains) > 1e-9:
@@ -500,7 +508,7 @@ def run_ours(args, wl):
                       "gbs": byts / (avg_ms / 1000) / 1e9}
     dom = max(kern, key=lambda k: kern[k]["share"])
     d = kern[dom]
-    traffic, traffic_note = ncu_traffic(dom, d["chains_per_launch"])
+    traffic, traffic_note = ncu_traffic(dom, d["chains_per_launch"], wl)
     if dom == "phase_b":
         roof = {"kernel": dom, "bound": "hbm", "achieved": d["gbs"], "peak": hbm, "unit": "GB/s",
                 "frac": d["gbs"] / hbm, "traffic": traffic, "peak_source": f"{peak_src} hbm_gbs"}
