@@ -95,6 +95,7 @@ mone_status validate_config(const mone_config* c) {
     if (c->loss != MONE_LOSS_DOT && c->loss != MONE_LOSS_MSE) return MONE_ERR_INVALID_ARG;
     if (c->loss == MONE_LOSS_MSE && c->dtype != MONE_BF16) return MONE_ERR_UNSUPPORTED;
     if (c->memory != MONE_MEM_MLP && c->memory != MONE_MEM_SWIGLU) return MONE_ERR_INVALID_ARG;
+    if (!std::isfinite(c->lr) || !(c->rms_eps >= 0.0f) || !std::isfinite(c->rms_eps)) return MONE_ERR_INVALID_ARG;
     if (c->memory == MONE_MEM_SWIGLU) {
         if (c->dtype != MONE_BF16 || c->loss != MONE_LOSS_DOT) return MONE_ERR_UNSUPPORTED;
         if (c->mem_heads < 1 || c->d_in % c->mem_heads) return MONE_ERR_INVALID_ARG;
@@ -106,7 +107,6 @@ mone_status validate_config(const mone_config* c) {
             return MONE_ERR_UNSUPPORTED_SHAPE;
         return MONE_OK;
     }
-    if (!std::isfinite(c->lr) || !(c->rms_eps >= 0.0f) || !std::isfinite(c->rms_eps)) return MONE_ERR_INVALID_ARG;
     if (c->head_dim != 64 && c->head_dim != 128) return MONE_ERR_UNSUPPORTED_SHAPE;
     if (c->d_out != 2 * c->n_kv_heads * c->head_dim) return MONE_ERR_UNSUPPORTED_SHAPE;
     if (c->seg_T > 4096) return MONE_ERR_UNSUPPORTED_SHAPE;

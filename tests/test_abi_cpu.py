@@ -78,6 +78,8 @@ def test_swiglu_memory_validation(L):
     assert init_rc(L, cfg(**{**sw, "d_hid": 300})) == 2                   # hidden units per head <= 256
     assert init_rc(L, cfg(**{**sw, "mem_heads": 2})) == 2                 # dh = 448 > 256
     assert init_rc(L, cfg(**{**sw, "d_out": 768, "n_kv_heads": 6})) == 2  # output width must equal d_in
+    assert init_rc(L, cfg(**{**sw, "lr": float("inf")})) == 1             # rates checked for every memory form
+    assert init_rc(L, cfg(**{**sw, "rms_eps": float("nan")})) == 1
 
 
 def test_squared_error_loss_is_bf16_only(L):
