@@ -241,6 +241,14 @@ mone_status mone_attention(mone_mem* m, const void* Q, int n_q_heads, int Lq, co
 mone_status mone_mem_set_timing(mone_mem* m, int enable);
 mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches);
 
+/*
+ * Busy time of one kernel kind since timing was last enabled: the length (ms) of the union
+ * of its launches' [start, end] event intervals, so launches that overlapped on different
+ * streams (the two chain groups of a call) count once.  Same kinds and waiting as
+ * mone_mem_kernel_time.  Errors: INVALID_ARG, CUDA.
+ */
+mone_status mone_mem_kernel_busy(mone_mem* m, int kind, double* busy_ms);
+
 const char* mone_status_string(mone_status s);
 
 /* Text of the last CUDA error this thread saw inside the library ("" if none);

@@ -28,7 +28,7 @@ STATUS = {0: "MONE_OK", 1: "MONE_ERR_INVALID_ARG", 2: "MONE_ERR_UNSUPPORTED_SHAP
 EXPORTS = ("mone_mem_init", "mone_ttl_segment", "mone_ttl_context", "mone_mem_generate_kv", "mone_mem_free",
            "mone_mem_read_state", "mone_mem_write_state", "mone_mem_sync", "mone_mem_launch_count",
            "mone_status_string", "mone_abi_version", "mone_mem_set_timing", "mone_mem_kernel_time",
-           "mone_last_error", "mone_mem_generate_kv_noalloc", "mone_attention")
+           "mone_last_error", "mone_mem_generate_kv_noalloc", "mone_attention", "mone_mem_kernel_busy")
 
 KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read", "mse", "attention")
 
@@ -82,6 +82,7 @@ def lib(path: Optional[str] = None) -> ctypes.CDLL:
         "mone_last_error": ([], ctypes.c_char_p),
         "mone_mem_set_timing": ([vp, i], i),
         "mone_mem_kernel_time": ([vp, i, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ll)], i),
+        "mone_mem_kernel_busy": ([vp, i, ctypes.POINTER(ctypes.c_double)], i),
     }
     for name, (args, res) in sig.items():
         fn = getattr(L, name)
@@ -211,6 +212,14 @@ def mone_mem_kernel_time(h: int, kind: int):
     n = ctypes.c_longlong()
     _check("mone_mem_kernel_time", lib().mone_mem_kernel_time(h, kind, ctypes.byref(ms), ctypes.byref(n)))
     return ms.value, n.value
+
+
+def mone_mem_kernel_busy(h: int, kind: int) -> float:
+    """Busy time (ms) of one kernel kind since timing was enabled: the union of its launches'
+    event intervals, overlapping launches counted once."""
+    ms = ctypes.c_double()
+    _check("mone_mem_kernel_busy", lib().mone_mem_kernel_busy(h, kind, ctypes.byref(ms)))
+    return ms.value
 
 
 def kv_strides(n_layers: int, n_kv: int, Q: int, head_dim: int):

@@ -27,6 +27,20 @@ struct KernelTiming {
     std::vector<Pending> pending;
     double ms[7] = {0, 0, 0, 0, 0, 0, 0};
     long long n[7] = {0, 0, 0, 0, 0, 0, 0};
+    // start and end of every launch, in ms after `ref` (recorded before the first timed launch
+    // since timing was enabled), for the busy time of a kernel kind (mone_mem_kernel_busy)
+    cudaEvent_t ref = nullptr;
+    bool ref_set = false;
+    std::vector<std::pair<double, double>> iv[7];
+
+    void reset() {
+        for (int k = 0; k < 7; ++k) {
+            ms[k] = 0;
+            n[k] = 0;
+            iv[k].clear();
+        }
+        ref_set = false;
+    }
 
     cudaEvent_t get() {
         if (!pool.empty()) {
@@ -42,11 +56,13 @@ struct KernelTiming {
         cudaError_t rc = cudaSuccess;
         for (auto& p : pending) {
             cudaError_t e = cudaEventSynchronize(p.b);
-            float t = 0.f;
+            float t = 0.f, t0 = 0.f;
             if (e == cudaSuccess) e = cudaEventElapsedTime(&t, p.a, p.b);
+            if (e == cudaSuccess && ref_set) e = cudaEventElapsedTime(&t0, ref, p.a);
             if (e == cudaSuccess) {
                 ms[p.kind] += t;
                 n[p.kind] += 1;
+                if (ref_set) iv[p.kind].push_back({t0, t0 + t});
             } else {
                 rc = e;
             }
@@ -59,6 +75,7 @@ struct KernelTiming {
     ~KernelTiming() {
         drain();
         for (cudaEvent_t e : pool) cudaEventDestroy(e);
+        if (ref) cudaEventDestroy(ref);
     }
 };
 
@@ -265,6 +282,11 @@ mone_status timed(mone_mem* m, int kind, cudaStream_t st, int kernels, F&& fn) {
     KernelTiming* T = m->timing;
     cudaEvent_t a = nullptr, b = nullptr;
     if (T && T->on) {
+        if (!T->ref_set) {  // time origin of the launch intervals: before every later timed launch
+            if (!T->ref && cudaEventCreate(&T->ref) != cudaSuccess) return MONE_ERR_CUDA;
+            if (cudaEventRecord(T->ref, st) != cudaSuccess) return MONE_ERR_CUDA;
+            T->ref_set = true;
+        }
         a = T->get();
         b = T->get();
         if (!a || !b) return MONE_ERR_CUDA;
@@ -763,11 +785,7 @@ mone_status mone_mem_set_timing(mone_mem* m, int enable) {
     KernelTiming* T = m->timing;
     const cudaError_t e = T->drain();
     T->on = enable != 0;
-    if (enable)
-        for (int k = 0; k < 5; ++k) {
-            T->ms[k] = 0;
-            T->n[k] = 0;
-        }
+    if (enable) T->reset();
     return cuda_status(e);
 }
 
@@ -779,6 +797,27 @@ mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* l
     MONE_CUDA(m->timing->drain());
     *ms = m->timing->ms[kind];
     *launches = m->timing->n[kind];
+    return MONE_OK;
+}
+
+mone_status mone_mem_kernel_busy(mone_mem* m, int kind, double* busy_ms) {
+    if (!is_live(m) || kind < 0 || kind > 6 || !busy_ms) return MONE_ERR_INVALID_ARG;
+    *busy_ms = 0;
+    if (!m->timing) return MONE_OK;
+    MONE_CUDA(m->timing->drain());
+    std::vector<std::pair<double, double>> v = m->timing->iv[kind];
+    std::sort(v.begin(), v.end());
+    double cur0 = 0, cur1 = -1;  // the union of the intervals, merged in start order
+    for (const auto& x : v) {
+        if (x.first > cur1) {
+            if (cur1 > cur0) *busy_ms += cur1 - cur0;
+            cur0 = x.first;
+            cur1 = x.second;
+        } else if (x.second > cur1) {
+            cur1 = x.second;
+        }
+    }
+    if (cur1 > cur0) *busy_ms += cur1 - cur0;
     return MONE_OK;
 }
 
