@@ -2,7 +2,8 @@
 //
 // The fp32 path (the tiny fp32 workload: 256 -> 512 -> 256, T = 128) is
 // latency-bound, so it uses plain CUDA-core FFMA tiles (64 x 64 per CTA, 4 x 4 per
-// thread) in fp32 throughout.  It computes the same two phases as the bf16
+// thread, 64-deep K slabs so that each thread has 32 loads in flight per slab) in fp32
+// throughout.  It computes the same two phases as the bf16
 // tensor-core path:
 //   phase A  H = U W1^T, R = Y W2^T (Y = [K || V]); A = SiLU(H);
 //            dH = c_t R * SiLU'(H), At = c_t A with c_t = -eta_t / T'   (Eq. 10)
@@ -19,7 +20,7 @@ namespace mone {
 
 namespace {
 
-constexpr int TM = 64, TN = 64, TK = 16;
+constexpr int TM = 64, TN = 64, TK = 64;
 
 // acc[i][j] += sum_k A(m0 + ty*4 + i, k) * B(n0 + tx*4 + j, k) for one 64 x 64 tile.
 // A(m, k) = A[m*sam + k*sak]; rows m >= m_valid and k >= k_valid read as 0.
@@ -28,15 +29,27 @@ __device__ __forceinline__ void simt_tile(float (&acc)[4][4], const float* A, lo
                                           int k_valid, float (*As)[TM + 4], float (*Bs)[TN + 4]) {
     const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
     for (int k0 = 0; k0 < K; k0 += TK) {
+        // 64 x TK elements of each operand, TK consecutive along the contiguous dimension
+        float av[TM * TK / 256], bv[TN * TK / 256];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
+        for (int r = 0; r < TM * TK / 256; ++r) {
             const int e = tid + 256 * r;
             int m, k;
-            if (sak == 1) { m = e >> 4; k = e & 15; } else { m = e & 63; k = e >> 6; }
-            As[k][m] = (m < m_valid && k0 + k < k_valid) ? A[m * sam + (k0 + k) * sak] : 0.0f;
+            if (sak == 1) { m = e / TK; k = e % TK; } else { m = e % TM; k = e / TM; }
+            av[r] = (m < m_valid && k0 + k < k_valid) ? A[m * sam + (k0 + k) * sak] : 0.0f;
             int n, kb;
-            if (sbk == 1) { n = e >> 4; kb = e & 15; } else { n = e & 63; kb = e >> 6; }
-            Bs[kb][n] = (k0 + kb < k_valid) ? B[n * sbn + (k0 + kb) * sbk] : 0.0f;
+            if (sbk == 1) { n = e / TK; kb = e % TK; } else { n = e % TN; kb = e / TN; }
+            bv[r] = (k0 + kb < k_valid) ? B[n * sbn + (k0 + kb) * sbk] : 0.0f;
+        }
+#pragma unroll
+        for (int r = 0; r < TM * TK / 256; ++r) {
+            const int e = tid + 256 * r;
+            int m, k;
+            if (sak == 1) { m = e / TK; k = e % TK; } else { m = e % TM; k = e / TM; }
+            As[k][m] = av[r];
+            int n, kb;
+            if (sbk == 1) { n = e / TK; kb = e % TK; } else { n = e % TN; kb = e / TN; }
+            Bs[kb][n] = bv[r];
         }
         __syncthreads();
 #pragma unroll
