@@ -268,9 +268,12 @@ F32SegArgs make_f32_args(const DevState& s, const SegWork& w) {
 // ------------------------------------------------------------------ state upkeep
 
 // Apply the pending renormalisation of the last segment (when asked) and refresh
-// the bf16 operand copies.  One CTA per (row, chain, matrix).
+// the bf16 operand copies.  One warp per (row, chain, matrix), 8 rows a CTA; each lane
+// moves 16-byte vectors, four of them in flight at a time (widths are multiples of 64).
 __global__ void __launch_bounds__(256) finalize_kernel(DevState s, int c0, int parity, int apply_scale) {
-    const int h = blockIdx.x, cs = c0 + blockIdx.y, which = blockIdx.z;
+    const int h = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    const int cs = c0 + blockIdx.y, which = blockIdx.z;
+    if (h >= s.d_hid) return;
     const int width = which ? s.d_out : s.d_in;
     float* w = (which ? s.W2 : s.W1) + ((size_t)cs * s.d_hid + h) * width;
     bf16* wb = s.dtype == 1 ? (which ? s.W2b : s.W1b) + ((size_t)cs * s.d_hid + h) * width : nullptr;
@@ -280,10 +283,24 @@ __global__ void __launch_bounds__(256) finalize_kernel(DevState s, int c0, int p
         const float* n0 = (which ? s.n2 : s.n1) + (size_t)cs * s.d_hid;
         sc = renorm_scale(n0[h], ss[h]);
     }
-    for (int i = threadIdx.x; i < width; i += 256) {
-        const float v = w[i] * sc;
-        if (apply_scale) w[i] = v;
-        if (wb) wb[i] = __float2bfloat16_rn(v);
+    for (int base = lane * 4; base < width; base += 4 * 128) {
+        float4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (base + u * 128 < width) v[u] = *reinterpret_cast<const float4*>(w + base + u * 128);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int i = base + u * 128;
+            if (i >= width) break;
+            const float4 x = make_float4(v[u].x * sc, v[u].y * sc, v[u].z * sc, v[u].w * sc);
+            if (apply_scale) *reinterpret_cast<float4*>(w + i) = x;
+            if (wb) {
+                uint2 p;
+                p.x = pack_bf16(x.x, x.y);
+                p.y = pack_bf16(x.z, x.w);
+                *reinterpret_cast<uint2*>(wb + i) = p;
+            }
+        }
     }
 }
 
@@ -381,7 +398,7 @@ cudaError_t launch_phase_b_f32(const DevState& s, const SegWork& w, cudaStream_t
 }
 
 cudaError_t launch_finalize(const DevState& s, int c0, int nc, int parity, int apply_scale, cudaStream_t st) {
-    finalize_kernel<<<dim3(s.d_hid, nc, 2), 256, 0, st>>>(s, c0, parity, apply_scale);
+    finalize_kernel<<<dim3((s.d_hid + 7) / 8, nc, 2), 256, 0, st>>>(s, c0, parity, apply_scale);
     return cudaGetLastError();
 }
 
