@@ -616,30 +616,66 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
 // TMA-loads chunks ahead of time; the two epilogue groups take alternate chunks,
 // update a chunk in place and TMA-store it back (the bf16 copy goes out with
 // coalesced 64-byte warp stores), and hand the slot back once the store has read it.
+//
+// PAIR: clusters of 2 CTAs run tcgen05.mma.cta_group::2 over 256 weight columns x 256
+// hidden rows.  CTA r stages its own 128 columns of U (or Y) and rows r*128 .. +127 of the
+// tile's 256 rows of dH (or At) per 64-token k-block, so each SM takes in 32 KB of operands
+// a k-block instead of 48 KB for the same 128 x 256 accumulator.  Both CTAs' loads complete
+// on rank 0's full barrier, rank 0 issues the MMAs, each commit arrives on both CTAs'
+// barriers, and the 16 epilogue warps of the pair release an accumulator buffer on rank 0's
+// tempty barrier.  Each CTA updates the state of its own 128 columns exactly as the one-CTA
+// kernel does.  A pair's 256 columns lie in one matrix (d_in and d_out multiples of 256).
 
 constexpr int S_ROWS = 32;                                 // hidden rows per state chunk
 constexpr int S_SLOTS = 4;
 constexpr int S_F32 = S_ROWS * B_BM * 4;                   // 16 KB
 constexpr int S_SLOT = 2 * S_F32;                          // W and mu: 32 KB
-constexpr int B_STAGES_V3 = 2;
 constexpr int B_THREADS = 12 * 32;
 constexpr int B_EPI_THREADS = 4 * 32;     // per epilogue group
 constexpr int B_STATE_WARP = 10;          // TMA loads of state chunks
 constexpr int B_STORE_WARP = 11;          // TMA stores of updated chunks, slot release
 
-struct LayoutB {
-    static constexpr int RING = B_STAGES_V3 * B_STAGE;
+template <bool PAIR>
+struct LayoutBT {
+    // operand stages: one CTA 48 KB (128 columns + 256 hidden rows); a pair member 32 KB
+    // (128 columns + its 128 hidden rows), three of them in the same space as two
+    static constexpr int STAGE = PAIR ? (B_BM + B_BN / 2) * BK * 2 : B_STAGE;
+    static constexpr int STAGES = PAIR ? 3 : 2;
+    static constexpr int RING = STAGES * STAGE;
     static constexpr int STATE = RING;
     static constexpr int BARS = STATE + S_SLOTS * S_SLOT;  // full[S] empty[S] tfull[2] tempty[2] sfull/sdone/sempty[N]
-    static constexpr int NBARS = 2 * B_STAGES_V3 + 4 + 3 * S_SLOTS;
+    static constexpr int NBARS = 2 * STAGES + 4 + 3 * S_SLOTS;
     static constexpr int SLOT = BARS + NBARS * 8;
     static constexpr int FLAG = SLOT + 16;
     static constexpr int TAB = FLAG + 16;                  // per group: [B_BN/2] renorm scales + [4] decay partials
     static constexpr int END = TAB + 2 * (B_BN / 2 + 4) * 4;
     static constexpr int DYN = END + 1024;
 };
-static_assert(LayoutB::DYN <= 227 * 1024, "phase B shared memory budget");
+using LayoutB = LayoutBT<false>;
+using LayoutB2 = LayoutBT<true>;
+static_assert(LayoutB::DYN <= 227 * 1024 && LayoutB2::DYN <= 227 * 1024, "phase B shared memory budget");
 
+// The tiles one CTA of phase B walks: t = first, first + step, ... < count, each giving
+// (chain of the launch, first hidden row, first weight column of this CTA).
+template <bool PAIR>
+struct BTiles {
+    int first, step, count, n_ht, n_ct, rank;
+    __device__ BTiles(const TcArgs& a) {
+        n_ht = a.d_hid / B_BN;
+        n_ct = (a.d_in + a.d_out) / (PAIR ? 2 * B_BM : B_BM);
+        count = a.nc * n_ht * n_ct;
+        rank = PAIR ? (int)cluster_ctarank() : 0;
+        first = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+        step = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+    }
+    __device__ void decode(int t, int& cz, int& h0, int& col0) const {
+        cz = t / (n_ht * n_ct);
+        h0 = ((t / n_ct) % n_ht) * B_BN;
+        col0 = (t % n_ct) * (PAIR ? 2 * B_BM : B_BM) + rank * B_BM;
+    }
+};
+
+template <bool PAIR>
 __global__ void __launch_bounds__(B_THREADS, 1)
 tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant__ CUtensorMap tmKb,
                   const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmDH,
@@ -648,25 +684,27 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                   const __grid_constant__ CUtensorMap tmM2s, const __grid_constant__ CUtensorMap tmW1o,
                   const __grid_constant__ CUtensorMap tmW2o, const TcArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    using L = LayoutB;
+    using L = LayoutBT<PAIR>;
+    constexpr int NS = L::STAGES;
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const uint32_t bars = smem_u32(base + L::BARS);
     auto full = [&](int s) { return bars + 8 * s; };
-    auto empty = [&](int s) { return bars + 8 * (B_STAGES_V3 + s); };
-    auto tfull = [&](int b) { return bars + 8 * (2 * B_STAGES_V3 + b); };
-    auto tempty = [&](int b) { return bars + 8 * (2 * B_STAGES_V3 + 2 + b); };
-    auto sfull = [&](int k) { return bars + 8 * (2 * B_STAGES_V3 + 4 + k); };
-    auto sempty = [&](int k) { return bars + 8 * (2 * B_STAGES_V3 + 4 + S_SLOTS + k); };
-    auto sdone = [&](int k) { return bars + 8 * (2 * B_STAGES_V3 + 4 + 2 * S_SLOTS + k); };
+    auto empty = [&](int s) { return bars + 8 * (NS + s); };
+    auto tfull = [&](int b) { return bars + 8 * (2 * NS + b); };
+    auto tempty = [&](int b) { return bars + 8 * (2 * NS + 2 + b); };
+    auto sfull = [&](int k) { return bars + 8 * (2 * NS + 4 + k); };
+    auto sempty = [&](int k) { return bars + 8 * (2 * NS + 4 + S_SLOTS + k); };
+    auto sdone = [&](int k) { return bars + 8 * (2 * NS + 4 + 2 * S_SLOTS + k); };
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const BTiles<PAIR> tl(a);
     if (threadIdx.x == 0) {
-        for (int i = 0; i < B_STAGES_V3; ++i) {
+        for (int i = 0; i < NS; ++i) {
             mbar_init(full(i), 1);
             mbar_init(empty(i), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull(b), 1);
-            mbar_init(tempty(b), 8);
+            mbar_init(tempty(b), PAIR ? 16 : 8);  // every epilogue warp (of both CTAs of a pair)
         }
         for (int k = 0; k < S_SLOTS; ++k) {
             mbar_init(sfull(k), 1);
@@ -676,16 +714,22 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
         fence_mbar_init();
     }
     if (warp == 0) {
-        tmem_alloc(smem_u32(base + L::SLOT), 512);
-        tmem_relinquish();
+        if constexpr (PAIR) {
+            tmem_alloc_pair(smem_u32(base + L::SLOT), 512);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(smem_u32(base + L::SLOT), 512);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
-    __syncthreads();
+    if constexpr (PAIR)
+        cluster_sync();  // barriers of both CTAs initialised, TMEM of the pair allocated
+    else
+        __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<uint32_t*>(base + L::SLOT);
 
-    const int n_ct = (a.d_in + a.d_out) / B_BM, n_ht = a.d_hid / B_BN;
-    const int ntiles = a.nc * n_ht * n_ct;
     const int KB = (a.Tp + BK - 1) / BK;  // tokens beyond T' carry zero dH / At
     const int dhalf = a.d_out / 2;
     const int chunk_bytes = a.momentum ? 2 * S_F32 : S_F32;
@@ -699,65 +743,102 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             tma_prefetch_map(&tmAT);
             uint32_t kc = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-                const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
-                const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
+            for (int t = tl.first; t < tl.count && ok; t += tl.step) {
+                int cz, h0, col0;
+                tl.decode(t, cz, h0, col0);
+                const int cs = a.c0 + cz;
                 const bool isW1 = col0 < a.d_in;
+                // this CTA's share of the tile's hidden rows: all 256, or 128 of a pair
+                const int hrow = h0 + (PAIR ? tl.rank * (B_BN / 2) : 0);
+                constexpr int HB = (PAIR ? B_BN / 2 : B_BN) / 64;  // 64-row boxes of hidden rows
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
-                    const int s = kc % B_STAGES_V3;
-                    if (kc >= B_STAGES_V3 && !mbar_wait(empty(s), ((kc / B_STAGES_V3) - 1) & 1, a.status)) {
+                    const int s = kc % NS;
+                    if (kc >= NS && !mbar_wait(empty(s), ((kc / NS) - 1) & 1, a.status)) {
                         ok = false;
                         break;
                     }
-                    const uint32_t sa = smem_u32(base + s * B_STAGE), sb = sa + B_BM * BK * 2, fb = full(s);
-                    mbar_expect_tx(fb, B_STAGE);
+                    const uint32_t sa = smem_u32(base + s * L::STAGE), sb = sa + B_BM * BK * 2;
+                    uint32_t fb = full(s);
+                    if constexpr (PAIR) {
+                        fb = map_to_cta(full(s), 0);  // both CTAs' loads complete on rank 0's barrier
+                        if (tl.rank == 0) mbar_expect_tx(full(s), 2 * L::STAGE);
+                    } else {
+                        mbar_expect_tx(fb, L::STAGE);
+                    }
 #pragma unroll
                     for (int bx = 0; bx < B_BM / 64; ++bx) {
                         const uint32_t dst = sa + bx * BOX;
+                        const CUtensorMap* map;
+                        int x, y, z;
                         if (isW1) {
-                            tma_load_3d(dst, &tmUb, fb, col0 + bx * 64, a.u_row0 + kb * BK, a.u_chain0 + cz);
+                            map = &tmUb;
+                            x = col0 + bx * 64;
+                            y = a.u_row0 + kb * BK;
+                            z = a.u_chain0 + cz;
                         } else {
                             const int o = col0 - a.d_in + bx * 64;
-                            if (o < dhalf)
-                                tma_load_3d(dst, &tmKb, fb, o, a.y_row0 + kb * BK, cz);
-                            else
-                                tma_load_3d(dst, &tmVb, fb, o - dhalf, a.y_row0 + kb * BK, cz);
+                            map = o < dhalf ? &tmKb : &tmVb;
+                            x = o < dhalf ? o : o - dhalf;
+                            y = a.y_row0 + kb * BK;
+                            z = cz;
                         }
+                        if constexpr (PAIR)
+                            tma_load_3d_pair(dst, map, fb, x, y, z);
+                        else
+                            tma_load_3d(dst, map, fb, x, y, z);
                     }
 #pragma unroll
-                    for (int bx = 0; bx < B_BN / 64; ++bx)
-                        tma_load_3d(sb + bx * BOX, isW1 ? &tmDH : &tmAT, fb, h0 + bx * 64, kb * BK, cs);
+                    for (int bx = 0; bx < HB; ++bx) {
+                        if constexpr (PAIR)
+                            tma_load_3d_pair(sb + bx * BOX, isW1 ? &tmDH : &tmAT, fb, hrow + bx * 64, kb * BK, cs);
+                        else
+                            tma_load_3d(sb + bx * BOX, isW1 ? &tmDH : &tmAT, fb, hrow + bx * 64, kb * BK, cs);
+                    }
                 }
             }
+            if (PAIR && !ok) pause_ns(200000);
         }
         __syncwarp();
     } else if (warp == 1) {
-        if (lane == 0) {
-            const uint32_t idesc = idesc_bf16_f32(B_BM, B_BN, true, true);
+        if (lane == 0 && (!PAIR || tl.rank == 0)) {
+            const uint32_t idesc = idesc_bf16_f32(PAIR ? 2 * B_BM : B_BM, B_BN, true, true);
             uint32_t kc = 0;
             int local = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++local) {
+            for (int t = tl.first; t < tl.count && ok; t += tl.step, ++local) {
                 const int b = local & 1;
                 if (local >= 2 && !mbar_wait(tempty(b), ((local >> 1) - 1) & 1, a.status)) break;
                 tc_fence_after();
                 const uint32_t d = tmem + b * 256;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
-                    const int s = kc % B_STAGES_V3;
-                    if (!mbar_wait(full(s), (kc / B_STAGES_V3) & 1, a.status)) {
+                    const int s = kc % NS;
+                    if (!mbar_wait(full(s), (kc / NS) & 1, a.status)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t sa = smem_u32(base + s * B_STAGE), sb = sa + B_BM * BK * 2;
+                    const uint32_t sa = smem_u32(base + s * L::STAGE), sb = sa + B_BM * BK * 2;
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k)
-                        umma_bf16(d, sdesc_sw128(sa + k * 16 * 128, BOX), sdesc_sw128(sb + k * 16 * 128, BOX), idesc,
-                                  (kb == 0 && k == 0) ? 0u : 1u);
-                    umma_commit(empty(s));
+                    for (int k = 0; k < BK / 16; ++k) {
+                        if constexpr (PAIR)
+                            umma_bf16_pair(d, sdesc_sw128(sa + k * 16 * 128, BOX), sdesc_sw128(sb + k * 16 * 128, BOX),
+                                           idesc, (kb == 0 && k == 0) ? 0u : 1u);
+                        else
+                            umma_bf16(d, sdesc_sw128(sa + k * 16 * 128, BOX), sdesc_sw128(sb + k * 16 * 128, BOX), idesc,
+                                      (kb == 0 && k == 0) ? 0u : 1u);
+                    }
+                    if constexpr (PAIR)
+                        umma_commit_pair(empty(s), 0x3);
+                    else
+                        umma_commit(empty(s));
                 }
-                umma_commit(tfull(b));
+                if (!ok) break;
+                if constexpr (PAIR)
+                    umma_commit_pair(tfull(b), 0x3);
+                else
+                    umma_commit(tfull(b));
             }
+            if (PAIR && !ok) pause_ns(200000);
         }
         __syncwarp();
     } else if (warp == B_STATE_WARP) {
@@ -771,9 +852,10 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             }
             uint32_t seq = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-                const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
-                const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
+            for (int t = tl.first; t < tl.count && ok; t += tl.step) {
+                int cz, h0, col0;
+                tl.decode(t, cz, h0, col0);
+                const int cs = a.c0 + cz;
                 const bool isW1 = col0 < a.d_in;
                 const int cl = isW1 ? col0 : col0 - a.d_in;
                 for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
@@ -795,9 +877,10 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
         if (lane == 0) {
             uint32_t seq = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-                const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
-                const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
+            for (int t = tl.first; t < tl.count && ok; t += tl.step) {
+                int cz, h0, col0;
+                tl.decode(t, cz, h0, col0);
+                const int cs = a.c0 + cz;
                 const bool isW1 = col0 < a.d_in;
                 const int cl = isW1 ? col0 : col0 - a.d_in;
                 for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
@@ -827,12 +910,14 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
         float* tab = reinterpret_cast<float*>(base + L::TAB) + grp * (B_BN / 2 + 4);  // [B_BN/2]
         float* bred = tab + B_BN / 2;                                                  // [4]
         int* flag = reinterpret_cast<int*>(base + L::FLAG) + grp * 2;
+        const uint32_t tempty_rank0 = PAIR ? map_to_cta(tempty(0), 0) : tempty(0);
         bool finite = true;
         uint32_t tile_seq0 = 0;  // chunk sequence number of the current tile's first chunk
         int local = 0;
-        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++local, tile_seq0 += B_BN / S_ROWS) {
-            const int cz = tile / (n_ht * n_ct), ht = (tile / n_ct) % n_ht, ct = tile % n_ct;
-            const int cs = a.c0 + cz, h0 = ht * B_BN, col0 = ct * B_BM;
+        for (int t = tl.first; t < tl.count; t += tl.step, ++local, tile_seq0 += B_BN / S_ROWS) {
+            int cz, h0, col0;
+            tl.decode(t, cz, h0, col0);
+            const int cs = a.c0 + cz;
             const bool isW1 = col0 < a.d_in;
             const int which = isW1 ? 0 : 1;
             const int cl = isW1 ? col0 : col0 - a.d_in;
@@ -847,7 +932,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             }
             if (a.momentum) {
                 float v = 0.f;
-                for (int t = et; t < a.Tp; t += B_EPI_THREADS) v += a.dbeta[(size_t)cs * a.win + a.tok0 + t];
+                for (int tk = et; tk < a.Tp; tk += B_EPI_THREADS) v += a.dbeta[(size_t)cs * a.win + a.tok0 + tk];
                 v = warp_sum(v);
                 if (lane == 0) bred[q] = v;
             }
@@ -875,7 +960,12 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 if (i == B_BN / S_ROWS / 2 - 1) {
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(tempty(b));
+                    if (lane == 0) {
+                        if constexpr (PAIR)
+                            mbar_arrive_remote(tempty_rank0 + 8 * b);
+                        else
+                            mbar_arrive(tempty(b));
+                    }
                 }
                 if (et == 0) flag[1] = mbar_wait(sfull(k), (seq / S_SLOTS) & 1, a.status) ? 1 : 0;
                 __syncwarp();
@@ -922,8 +1012,18 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
         }
         if (!finite) atomicOr(a.status, DEV_NONFINITE);
     }
-    __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, 512);
+    tc_fence_before();
+    if constexpr (PAIR)
+        cluster_sync();  // every MMA of the pair has completed and every TMEM read is done
+    else
+        __syncthreads();
+    tc_fence_after();
+    if (warp == 0) {
+        if constexpr (PAIR)
+            tmem_dealloc_pair(tmem, 512);
+        else
+            tmem_dealloc(tmem, 512);
+    }
 }
 
 TcArgs make_args(const DevState& s, const SegWork& w) {
@@ -1210,7 +1310,8 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 std::once_flag g_attr_once;
 cudaError_t g_attr_err = cudaSuccess;
 int g_sms = 0;
-int g_pair_clusters = 0;  // co-resident CTA pairs of the pair kernel (0: use the one-CTA kernel)
+int g_pair_clusters = 0;   // co-resident CTA pairs of the phase A pair kernel (0: use the one-CTA kernel)
+int g_pairb_clusters = 0;  // the same for the phase B pair kernel
 
 cudaError_t ensure_attrs() {
     std::call_once(g_attr_once, [] {
@@ -1221,8 +1322,11 @@ cudaError_t ensure_attrs() {
         if (g_attr_err == cudaSuccess)
             g_attr_err = cudaFuncSetAttribute(tc_phase_a_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LA::DYN);
         if (g_attr_err == cudaSuccess)
-            g_attr_err =
-                cudaFuncSetAttribute(tc_phase_b_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LayoutB::DYN);
+            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              LayoutB::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              LayoutB2::DYN);
         if (g_attr_err == cudaSuccess)
             g_attr_err =
                 cudaFuncSetAttribute(tc_phase_a_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LP::DYN);
@@ -1253,6 +1357,12 @@ cudaError_t ensure_attrs() {
             if (cudaOccupancyMaxActiveClusters(&g_pair_clusters, tc_phase_a_pair_kernel, &cfg) != cudaSuccess) {
                 cudaGetLastError();
                 g_pair_clusters = 0;
+            }
+            cfg.blockDim = dim3(B_THREADS);
+            cfg.dynamicSmemBytes = LayoutB2::DYN;
+            if (cudaOccupancyMaxActiveClusters(&g_pairb_clusters, tc_phase_b_kernel<true>, &cfg) != cudaSuccess) {
+                cudaGetLastError();
+                g_pairb_clusters = 0;
             }
         }
     });
@@ -1296,10 +1406,34 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
     cudaError_t e = ensure_attrs();
     if (e != cudaSuccess) return e;
     const TcArgs a = make_args(s, w);
+    const CUtensorMap& U = s.mode == 1 ? m.Ub : in.Xb;
+    // CTA pairs over 256-column x 256-hidden tiles (a pair's columns lie in one matrix) from
+    // T = 1024 on: there a tile's operand stream (768 KB a CTA) rivals its state stream, and the
+    // pair halves the dH / At share of it.  At T = 512 the pair's coupled loads and accumulator
+    // release cost more than they save (measured: 57.2 vs 54.8 ms a step on l16_d2048_128k).
+    constexpr int PAIR_MIN_T = 1024;
+    if (s.T >= PAIR_MIN_T && s.d_in % (2 * B_BM) == 0 && s.d_out % (2 * B_BM) == 0 && g_pairb_clusters > 0) {
+        const int npairs = w.nc * ((s.d_in + s.d_out) / (2 * B_BM)) * (s.d_hid / B_BN);
+        const int clusters = npairs < g_pairb_clusters ? npairs : g_pairb_clusters;
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 2;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(2 * clusters);
+        cfg.blockDim = dim3(B_THREADS);
+        cfg.dynamicSmemBytes = LayoutB2::DYN;
+        cfg.stream = st;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, tc_phase_b_kernel<true>, U, in.Kb, in.Vb, m.dH, m.At, m.W1s, m.W2s, m.M1s,
+                                  m.M2s, m.W1o, m.W2o, a);
+    }
     const int ntiles = w.nc * ((s.d_in + s.d_out) / B_BM) * (s.d_hid / B_BN);
     const int grid = ntiles < g_sms ? ntiles : g_sms;
-    tc_phase_b_kernel<<<grid, B_THREADS, LayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.dH, m.At,
-                                                              m.W1s, m.W2s, m.M1s, m.M2s, m.W1o, m.W2o, a);
+    tc_phase_b_kernel<false><<<grid, B_THREADS, LayoutB::DYN, st>>>(U, in.Kb, in.Vb, m.dH, m.At, m.W1s, m.W2s, m.M1s,
+                                                                     m.M2s, m.W1o, m.W2o, a);
     return cudaGetLastError();
 }
 
