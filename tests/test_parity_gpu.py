@@ -251,6 +251,48 @@ def test_generate_kv_into_strided_cache_and_reuse():
     run.close()
 
 
+# ----------------------------------------------------------------- CTA-pair phase B (segments of 1024 tokens and more)
+
+@pytest.mark.parametrize("mode,loss,lr", [(wk.PLAIN, "neg_inner", 0.3), (wk.PAPER, "neg_inner", 0.3),
+                                          (wk.PAPER, "mse", 0.3)])
+def test_bf16_pair_phase_b_context_parity(mode, loss, lr):
+    """From T = 1024 on, phase B runs on CTA pairs (256 columns x 256 hidden rows): 2 segments
+    and a ragged tail, 3 chains in two groups (2 + 1)."""
+    wl = small(mode, n_ctx=1, n_layers=3, T=1024, N=2 * 1024 + 300, lr=lr).replace(loss=loss)
+    run = GpuRun(wl)
+    run.ttl_context()
+    W1, W2, mu1, mu2 = run.state()
+    Xq = wk.query_inputs(wl, "cuda")
+    Kg, Vg = run.generate_kv(Xq)
+    for c in range(wl.chains):
+        st = check_chain(run, c, W1, W2, BF16_TOL)
+        if mode == wk.PAPER:
+            assert rel_fro(mu1[c], st.mu["W1"]) <= 5e-2 and rel_fro(mu2[c], st.mu["W2"]) <= 5e-2
+        Ko, Vo = oracle_read(run, st, c, Xq)
+        assert rel_fro(Kg[0, c].float(), Ko) <= BF16_TOL and rel_fro(Vg[0, c].float(), Vo) <= BF16_TOL
+    run.close()
+
+
+def test_bf16_pair_phase_b_one_chain_segment():
+    """A one-chain call (one group) through the pair kernel, with caller rates and the loss."""
+    wl = small(wk.PLAIN, n_ctx=1, n_layers=2, T=1024, N=1024)
+    run = GpuRun(wl)
+    eta = wk.token_lr(wl, 1, 900, "cuda")
+    loss = torch.zeros(1, device="cuda")
+    mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, :900], run.K[0, 1, :900], run.V[0, 1, :900], 900, eta, loss)
+    mone.mone_mem_sync(run.h)
+    W1, W2, _, _ = run.state()
+    X = O.f64(run.X[0, 1, :900])
+    Y = np.concatenate([O.f64(run.K[0, 1, :900]), O.f64(run.V[0, 1, :900])], axis=1)
+    st = O.init_state(W1=O.f64(run.W1_0[1]), W2=O.f64(run.W2_0[1]))
+    st, L = O.ttl_segment(st, X, Y, O.Hyper(mode=wk.PLAIN, lr=wl.lr), None, eta=O.f64(eta))
+    assert rel_fro(W1[1], st.W["W1"]) <= BF16_TOL and rel_fro(W2[1], st.W["W2"]) <= BF16_TOL
+    assert rel_fro(W1[1].double() - run.W1_0[1].cpu().double(), st.W["W1"] - O.f64(run.W1_0[1])) <= 5e-2
+    assert abs(loss.item() - L) <= BF16_TOL * max(1.0, abs(L))
+    assert torch.equal(W1[0], run.W1_0[0].cpu()) and torch.equal(W2[0], run.W2_0[0].cpu())
+    run.close()
+
+
 # ----------------------------------------------------------------- squared-error loss variant (bf16)
 
 @pytest.mark.parametrize("mode,lr", [(wk.PLAIN, 0.01), (wk.PAPER, 0.3)])  # plain: the delta rule diverges at 0.05 for inputs of RMS 2
