@@ -44,6 +44,9 @@ notes):
       gate g_h; eps = 1e-6.
   R7  Key/query transform u = z / sqrt(|z|^2 + 1e-12), z = SiLU(alpha*x + gamma).
   R8  Plain mode: u = x, eta_j = lr, beta = 0, no renormalisation.
+  R13 The squared-error variant (loss="mse") replaces Eq. 7's l_j by
+      1/2 |M(u_j) - y_j|^2 at the segment's starting weights; rates, momentum
+      and renormalisation are unchanged.
   R14 Consumer attention (Eq. 5): the memory tokens are a prefix every query
       token sees; the query tokens are causal among themselves; query head h
       reads key/value head h // (n_q / n_kv) (grouped heads).
