@@ -1059,17 +1059,19 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
 // lane quarter, lane = query) run the epilogue.  Each weight tile is read by ceil(Q/128)
 // CTAs; query rows >= Q arrive as TMA zero fill and are never stored.  W2 is [hidden][out],
 // so in the out kernel the weight operand is MN-major (64-column boxes, as in phase B).
-// Two CTAs share an SM (three 32 KB stages each), so one CTA's epilogue overlaps the other's
-// loads when a read has more tiles than SMs.
-constexpr int R_STAGES = 3;
-constexpr int R_CTAS_PER_SM = 2;
+// A launch with more tiles than SMs runs two CTAs per SM (three 32 KB stages each), so one
+// CTA's epilogue overlaps the other's loads; a launch that fits in one wave runs one CTA per
+// SM with six stages, twice the operand bytes in flight for its single K loop.
 constexpr int R_STAGE = 2 * 128 * BK * 2;  // 32 KB: 128 query rows + 128 weight rows / columns
 constexpr int R_THREADS = 6 * 32;
 constexpr uint32_t R_EPI_BAR = 1;
-struct LR {
-    static constexpr int RING = R_STAGES * R_STAGE;
+template <int NST>
+struct LRT {
+    static constexpr int STAGES = NST;
+    static constexpr int CTAS_PER_SM = NST <= 3 ? 2 : 1;
+    static constexpr int RING = NST * R_STAGE;
     static constexpr int BARS = RING;  // full[S] empty[S] tfull
-    static constexpr int NBARS = 2 * R_STAGES + 1;
+    static constexpr int NBARS = 2 * NST + 1;
     static constexpr int SLOT = BARS + (NBARS * 8 + 15) / 16 * 16;
     static constexpr int FLAG = SLOT + 16;
     static constexpr int TAB = FLAG + 16;  // MSE_HIDDEN: renorm scales s1, s2 of the tile's rows
@@ -1077,7 +1079,10 @@ struct LR {
     static constexpr int END = STG + 4 * 2048;
     static constexpr int DYN = END + 1024;
 };
-static_assert(R_CTAS_PER_SM * (LR::DYN + 1024) <= 228 * 1024, "read kernel CTAs per SM");
+using LR = LRT<3>;   // several waves
+using LR6 = LRT<6>;  // one wave
+static_assert(LR::CTAS_PER_SM * (LR::DYN + 1024) <= 228 * 1024, "read kernel CTAs per SM");
+static_assert(LR6::DYN <= 227 * 1024, "read kernel shared memory");
 static_assert(LR::STG % 16 == 0, "staging buffers hold 16-byte pieces");
 
 struct ReadArgs {
@@ -1106,19 +1111,19 @@ enum { READ_HIDDEN = 0, MSE_HIDDEN = 1, MSE_OUT = 2 };  // other MODEs: read out
 // of that width.  MODE MSE_HIDDEN: A' = SiLU(s1 (1/|z_t|) H) s2, the segment's activations
 // with the pending renorm scales (s2 folded in, so A' W2raw = A W2).  MODE MSE_OUT: the
 // residual target y_t - M(u_t) = y_t - A'_t W2raw (and the segment's squared-error loss).
-template <int MODE>
-__global__ void __launch_bounds__(R_THREADS, R_CTAS_PER_SM)
+template <int MODE, int NST>
+__global__ void __launch_bounds__(R_THREADS, LRT<NST>::CTAS_PER_SM)
 tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const ReadArgs a) {
     constexpr bool OUT = MODE != READ_HIDDEN && MODE != MSE_HIDDEN;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const uint32_t bars = smem_u32(base + LR::BARS);
+    const uint32_t bars = smem_u32(base + LRT<NST>::BARS);
     auto full = [&](int s) { return bars + 8 * s; };
-    auto empty = [&](int s) { return bars + 8 * (R_STAGES + s); };
-    const uint32_t tfull = bars + 8 * (2 * R_STAGES);
+    auto empty = [&](int s) { return bars + 8 * (NST + s); };
+    const uint32_t tfull = bars + 8 * (2 * NST);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
-        for (int s = 0; s < R_STAGES; ++s) {
+        for (int s = 0; s < NST; ++s) {
             mbar_init(full(s), 1);
             mbar_init(empty(s), 1);
         }
@@ -1126,24 +1131,24 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         fence_mbar_init();
     }
     if (warp == 0) {
-        tmem_alloc(smem_u32(base + LR::SLOT), 128);
+        tmem_alloc(smem_u32(base + LRT<NST>::SLOT), 128);
         tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tmem = *reinterpret_cast<uint32_t*>(base + LR::SLOT);
+    const uint32_t tmem = *reinterpret_cast<uint32_t*>(base + LRT<NST>::SLOT);
     const int q0 = blockIdx.x * 128, n0 = blockIdx.y * 128, c = blockIdx.z;
     const int KB = (OUT ? a.d_hid : a.d_in) / BK;
-    float* table = reinterpret_cast<float*>(base + LR::TAB);
+    float* table = reinterpret_cast<float*>(base + LRT<NST>::TAB);
 
     if (warp == 0) {
         if (lane == 0) {
             tma_prefetch_map(&tmA);
             tma_prefetch_map(&tmB);
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % R_STAGES;
-                if (kb >= R_STAGES && !mbar_wait(empty(s), ((kb / R_STAGES) - 1) & 1, a.status)) break;
+                const int s = kb % NST;
+                if (kb >= NST && !mbar_wait(empty(s), ((kb / NST) - 1) & 1, a.status)) break;
                 const uint32_t sa = smem_u32(base + s * R_STAGE), sb = sa + 128 * BK * 2, fb = full(s);
                 mbar_expect_tx(fb, R_STAGE);
                 tma_load_3d(sa, &tmA, fb, kb * BK, a.a_row0 + q0, a.a_chain0 + c);
@@ -1161,8 +1166,8 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             const uint32_t idesc = idesc_bf16_f32(128, 128, false, OUT);
             bool ok = true;
             for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % R_STAGES;
-                if (!mbar_wait(full(s), (kb / R_STAGES) & 1, a.status)) {
+                const int s = kb % NST;
+                if (!mbar_wait(full(s), (kb / NST) & 1, a.status)) {
                     ok = false;
                     break;
                 }
@@ -1180,7 +1185,7 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         __syncwarp();
     } else {
         const int q = warp & 3;  // TMEM lane quarter of this warp
-        int* flag = reinterpret_cast<int*>(base + LR::FLAG);
+        int* flag = reinterpret_cast<int*>(base + LRT<NST>::FLAG);
         if constexpr (MODE == MSE_HIDDEN) {
             // renorm scales of this tile's 128 hidden rows (one per epilogue thread)
             const int h = n0 + (int)threadIdx.x - 64, cs = a.b_chain0 + c;
@@ -1205,7 +1210,7 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if constexpr (MODE == MSE_HIDDEN) {
                 const int cs = a.b_chain0 + c, t = qw + lane;
                 const float zi = (t < a.Tp) ? (a.zinv ? a.zinv[(size_t)cs * a.win + a.tok0 + t] : 1.f) : 0.f;
-                uint8_t* stg = base + LR::STG + (warp - 2) * 2048;
+                uint8_t* stg = base + LRT<NST>::STG + (warp - 2) * 2048;
                 bf16* row0 = a.Aq + ((size_t)cs * a.T + qw) * a.d_hid + n0;
 #pragma unroll 1
                 for (int cc = 0; cc < 4; ++cc) {
@@ -1226,7 +1231,7 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                 const int col0 = kpart ? n0 : n0 - dh;
                 const bool live = t < a.Tp && a.row0 + t < a.n_rows;
                 const bf16* yrow = (kpart ? a.K : a.V) + (size_t)c * a.y_cstride + (size_t)(a.row0 + t) * dh + col0;
-                uint8_t* stg = base + LR::STG + (warp - 2) * 2048;
+                uint8_t* stg = base + LRT<NST>::STG + (warp - 2) * 2048;
                 bf16* row0 = (kpart ? a.Kres : a.Vres) + ((size_t)cs * a.T + qw) * dh + col0;
                 float lsum = 0.f;
 #pragma unroll 1
@@ -1255,7 +1260,7 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                     if (lane == 0) atomicAdd(&a.loss[c], 0.5f * lsum / (float)a.Tp);
                 }
             } else if constexpr (!OUT) {
-                uint8_t* stg = base + LR::STG + (warp - 2) * 2048;
+                uint8_t* stg = base + LRT<NST>::STG + (warp - 2) * 2048;
                 bf16* row0 = a.Aq + ((size_t)c * a.Q + qw) * a.d_hid + n0;
 #pragma unroll 1
                 for (int cc = 0; cc < 4; ++cc) {
@@ -1313,6 +1318,25 @@ int g_sms = 0;
 int g_pair_clusters = 0;   // co-resident CTA pairs of the phase A pair kernel (0: use the one-CTA kernel)
 int g_pairb_clusters = 0;  // the same for the phase B pair kernel
 
+template <int MODE>
+cudaError_t read_attrs() {
+    cudaError_t e = cudaFuncSetAttribute(tc_read_kernel<MODE, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(tc_read_kernel<MODE, 6>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR6::DYN);
+    return e;
+}
+
+// Launch a read-structured kernel with the stage count that suits its grid (see LRT).
+template <int MODE>
+cudaError_t launch_read_kernel(dim3 grid, const CUtensorMap& A, const CUtensorMap& B, const ReadArgs& a,
+                               cudaStream_t st) {
+    if ((long long)grid.x * grid.y * grid.z <= g_sms)
+        tc_read_kernel<MODE, 6><<<grid, R_THREADS, LR6::DYN, st>>>(A, B, a);
+    else
+        tc_read_kernel<MODE, 3><<<grid, R_THREADS, LR::DYN, st>>>(A, B, a);
+    return cudaGetLastError();
+}
+
 cudaError_t ensure_attrs() {
     std::call_once(g_attr_once, [] {
         int dev = 0;
@@ -1330,18 +1354,11 @@ cudaError_t ensure_attrs() {
         if (g_attr_err == cudaSuccess)
             g_attr_err =
                 cudaFuncSetAttribute(tc_phase_a_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LP::DYN);
-        if (g_attr_err == cudaSuccess)
-            g_attr_err = cudaFuncSetAttribute(tc_read_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
-        if (g_attr_err == cudaSuccess)
-            g_attr_err = cudaFuncSetAttribute(tc_read_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
-        if (g_attr_err == cudaSuccess)
-            g_attr_err = cudaFuncSetAttribute(tc_read_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
-        if (g_attr_err == cudaSuccess)
-            g_attr_err = cudaFuncSetAttribute(tc_read_kernel<MSE_HIDDEN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              LR::DYN);
-        if (g_attr_err == cudaSuccess)
-            g_attr_err =
-                cudaFuncSetAttribute(tc_read_kernel<MSE_OUT>, cudaFuncAttributeMaxDynamicSharedMemorySize, LR::DYN);
+        if (g_attr_err == cudaSuccess) g_attr_err = read_attrs<0>();
+        if (g_attr_err == cudaSuccess) g_attr_err = read_attrs<64>();
+        if (g_attr_err == cudaSuccess) g_attr_err = read_attrs<128>();
+        if (g_attr_err == cudaSuccess) g_attr_err = read_attrs<MSE_HIDDEN>();
+        if (g_attr_err == cudaSuccess) g_attr_err = read_attrs<MSE_OUT>();
         if (g_attr_err == cudaSuccess) {
             cudaLaunchConfig_t cfg = {};
             cudaLaunchAttribute at[1];
@@ -1460,14 +1477,12 @@ cudaError_t launch_mse_tc(const DevState& s, const TcMaps& m, const TcInputMaps&
     a.a_row0 = paper ? (int)w.u_off : (int)w.row0;
     a.a_chain0 = paper ? w.c0 : 0;
     a.b_chain0 = w.c0;
-    tc_read_kernel<MSE_HIDDEN><<<dim3(s.T / 128, s.d_hid / 128, w.nc), R_THREADS, LR::DYN, st>>>(
-        paper ? m.Ua : in.Xa, m.W1b, a);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    e = launch_read_kernel<MSE_HIDDEN>(dim3(s.T / 128, s.d_hid / 128, w.nc), paper ? m.Ua : in.Xa, m.W1b, a, st);
+    if (e != cudaSuccess) return e;
     // out: the activations of the same chains (absolute), W2 MN-major
     a.a_row0 = 0;
     a.a_chain0 = w.c0;
-    tc_read_kernel<MSE_OUT><<<dim3(s.T / 128, s.d_out / 128, w.nc), R_THREADS, LR::DYN, st>>>(m.Amse, m.W2m, a);
-    return cudaGetLastError();
+    return launch_read_kernel<MSE_OUT>(dim3(s.T / 128, s.d_out / 128, w.nc), m.Amse, m.W2m, a, st);
 }
 
 cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, void* Aq, int Q, int n_layers,
@@ -1488,13 +1503,9 @@ cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, v
     a.s0 = strides[0]; a.s1 = strides[1]; a.s2 = strides[2]; a.s3 = strides[3];
     a.status = s.status;
     const int nq = (Q + 127) / 128;
-    tc_read_kernel<0><<<dim3(nq, s.d_hid / 128, s.C), R_THREADS, LR::DYN, st>>>(mu, m.W1b, a);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    if (s.hd == 64)
-        tc_read_kernel<64><<<dim3(nq, s.d_out / 128, s.C), R_THREADS, LR::DYN, st>>>(ma, m.W2m, a);
-    else
-        tc_read_kernel<128><<<dim3(nq, s.d_out / 128, s.C), R_THREADS, LR::DYN, st>>>(ma, m.W2m, a);
-    return cudaGetLastError();
+    if ((e = launch_read_kernel<0>(dim3(nq, s.d_hid / 128, s.C), mu, m.W1b, a, st)) != cudaSuccess) return e;
+    if (s.hd == 64) return launch_read_kernel<64>(dim3(nq, s.d_out / 128, s.C), ma, m.W2m, a, st);
+    return launch_read_kernel<128>(dim3(nq, s.d_out / 128, s.C), ma, m.W2m, a, st);
 }
 
 // ------------------------------------------------------------------ tensor maps
