@@ -209,6 +209,13 @@ mone_status build_swiglu_maps(mone_mem* m) {
         ok = ok && encode_map_bf16_4d(&w.PG, s.dHt, d, st, b);
     }
     ok = ok && encode_map_bf16_3d(&w.Z, s.Att, F, T, CH, 64, 64);
+    // fp32 state chunks of phase B (rows past a head's F hidden units or columns past dh are
+    // never touched: the kernel skips such chunks and masks such columns)
+    ok = ok && encode_map_plain_3d(&w.W1s, s.W1, true, dh, 2 * F, CH, 128, 32) &&
+         encode_map_plain_3d(&w.W2s, s.W2, true, dh, F, CH, 128, 32);
+    if (ok && s.mu1)
+        ok = encode_map_plain_3d(&w.M1s, s.mu1, true, dh, 2 * F, CH, 128, 32) &&
+             encode_map_plain_3d(&w.M2s, s.mu2, true, dh, F, CH, 128, 32);
     if (ok && s.U) {  // input-transform window as (dh, H, rows, C)
         const uint64_t d[4] = {dh, H, (uint64_t)s.win_rows, (uint64_t)s.C};
         const uint64_t st[3] = {dh * 2, H * dh * 2, (uint64_t)s.win_rows * H * dh * 2};

@@ -103,6 +103,8 @@ struct SwMaps {
     CUtensorMap W1a;           // bf16 W1 as (dh, F, 2, chains*heads), K-major {64,128,1,1}
     CUtensorMap W2a, W2m;      // bf16 W2 (dh, F, chains*heads): K-major {64,128}, MN {64 outputs, 64 hidden}
     CUtensorMap PG, Z;         // phase A outputs, MN-major: (F, 2, T, chains*heads) {64,1,64,1}, (F, T, ..) {64,64}
+    CUtensorMap W1s, M1s;      // fp32 W1 / mu1 as (dh, 2F, chains*heads), state chunks {128 cols, 32 rows}
+    CUtensorMap W2s, M2s;      // fp32 W2 / mu2 as (dh, F, chains*heads), the same chunks
 };
 struct SwInputMaps {
     CUtensorMap Xa, Xb;        // caller's X of a group (dh, heads, rows, chains): K-major and MN boxes

@@ -53,12 +53,7 @@ struct SwLayoutT {
 };
 // phase A and the read kernels: 4 stages of up to 48 KB (A tile 16 KB + up to 32 KB of B)
 using SwLayout = SwLayoutT<4, 48 * 1024, true>;
-// phase B: 3 stages of 32 KB and no transpose buffers, so that two CTAs share an SM and
-// one CTA's state update overlaps the others' operand loads and MMAs
-constexpr int SWB_CTAS_PER_SM = 2;
-using SwLayoutB = SwLayoutT<3, 4 * SW_BOX, false>;
 static_assert(SwLayout::DYN <= 227 * 1024, "shared memory budget");
-static_assert(SWB_CTAS_PER_SM * (SwLayoutB::DYN + 1024) <= 228 * 1024, "phase B CTAs per SM");
 
 struct SwArgs {
     int H, Hk, dh, F, T, Tp, C, c0, paper, momentum, renorm_pending, parity, win;
@@ -324,46 +319,134 @@ swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__
 
 // ------------------------------------------------------------------ phase B (gradient + update)
 
-// One tile (matrix m, 128 weight columns, 128 hidden rows, head) per CTA; two CTAs per SM
-// (three 32 KB operand stages each, 128 TMEM columns).  The update walks the tile's rows in
-// chunks of 16: every chunk's W and mu loads are issued before its stores.
-constexpr int SWB_ROWS = 16;
+// Persistent, one CTA per SM, over tiles (matrix m of W_in / W_gate / W_out, 128 hidden rows,
+// 128 weight columns, head): the gradient with TMEM lane = weight column (both operands
+// MN-major) into one of two TMEM accumulators, so the MMAs of tile i+1 run while tile i is
+// updated.  Warps: 0 operand producer, 1 MMA issuer, 2..9 update in two groups of four (one warp
+// per TMEM lane quarter), 10 state producer, 11 store warp.  The fp32 state of a tile moves in
+// chunks of 32 rows x 128 columns (W and mu) through a 4-slot shared-memory ring: the state
+// producer TMA-loads chunks ahead, the two groups update alternate chunks in place, the store
+// warp TMA-stores them back and frees the slot.  Chunks whose rows lie past F are skipped
+// (F is a multiple of 32); columns past dh load as zeros, are clipped from the stores and
+// masked from the bf16 copy.
+constexpr int SWB_ROWS = 32;                               // hidden rows per state chunk
+constexpr int SWB_SLOTS = 4;
+constexpr int SWB_F32 = SWB_ROWS * 128 * 4;                // 16 KB
+constexpr int SWB_SLOT = 2 * SWB_F32;                      // W and mu: 32 KB
+constexpr int SWB_STAGES = 3;
+constexpr int SWB_STAGE = 4 * SW_BOX;                      // 32 KB: 128 columns + 128 hidden rows
+constexpr int SWB_THREADS = 12 * 32;
+constexpr int SWB_EPI_THREADS = 4 * 32;                    // per update group
+constexpr int SWB_STATE_WARP = 10, SWB_STORE_WARP = 11;
+struct SwLayoutB {
+    static constexpr int RING = SWB_STAGES * SWB_STAGE;
+    static constexpr int STATE = RING;
+    static constexpr int BARS = STATE + SWB_SLOTS * SWB_SLOT;  // full[S] empty[S] tfull[2] tempty[2] sfull/sempty/sdone[N]
+    static constexpr int NBARS = 2 * SWB_STAGES + 4 + 3 * SWB_SLOTS;
+    static constexpr int SLOT = BARS + NBARS * 8;
+    static constexpr int FLAG = SLOT + 16;
+    static constexpr int TAB = FLAG + 16;                      // per group: [64] renorm scales + [4] decay partials
+    static constexpr int END = TAB + 2 * (64 + 4) * 4;
+    static constexpr int DYN = END + 1024;
+};
+static_assert(SwLayoutB::DYN <= 227 * 1024, "phase B shared memory budget");
 
-__global__ void __launch_bounds__(SW_THREADS, SWB_CTAS_PER_SM)
+// The tiles of a launch: t -> (chain-head of the launch, matrix, first hidden row, first column).
+struct SwBTiles {
+    int NC, NR, count;
+    __device__ SwBTiles(const SwArgs& a) {
+        NC = (a.dh + 127) / 128;
+        NR = (a.F + 127) / 128;
+        count = a.nc_launch * a.H * 3 * NR * NC;
+    }
+    __device__ void decode(int t, int& zh, int& m, int& f0, int& col0) const {
+        col0 = (t % NC) * 128;
+        t /= NC;
+        f0 = (t % NR) * 128;
+        t /= NR;
+        m = t % 3;
+        zh = t / 3;
+    }
+};
+
+__global__ void __launch_bounds__(SWB_THREADS, 1)
 swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant__ CUtensorMap tmKb,
                 const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmPG,
-                const __grid_constant__ CUtensorMap tmZ, const SwArgs a) {
+                const __grid_constant__ CUtensorMap tmZ, const __grid_constant__ CUtensorMap tmW1s,
+                const __grid_constant__ CUtensorMap tmM1s, const __grid_constant__ CUtensorMap tmW2s,
+                const __grid_constant__ CUtensorMap tmM2s, const SwArgs a) {
     using L = SwLayoutB;
     extern __shared__ uint8_t smem_raw[];
-    const auto c = sw_setup<L>(smem_raw, 128);
-    const uint32_t tmem = *reinterpret_cast<uint32_t*>(c.base + L::SLOT);
+    uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const uint32_t bars = smem_u32(base + L::BARS);
+    auto full = [&](int s) { return bars + 8 * s; };
+    auto empty = [&](int s) { return bars + 8 * (SWB_STAGES + s); };
+    auto tfull = [&](int b) { return bars + 8 * (2 * SWB_STAGES + b); };
+    auto tempty = [&](int b) { return bars + 8 * (2 * SWB_STAGES + 2 + b); };
+    auto sfull = [&](int k) { return bars + 8 * (2 * SWB_STAGES + 4 + k); };
+    auto sempty = [&](int k) { return bars + 8 * (2 * SWB_STAGES + 4 + SWB_SLOTS + k); };
+    auto sdone = [&](int k) { return bars + 8 * (2 * SWB_STAGES + 4 + 2 * SWB_SLOTS + k); };
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int NC = (a.dh + 127) / 128;
-    const int m = blockIdx.x / NC, col0 = (blockIdx.x % NC) * 128, f0 = blockIdx.y * 128;
-    const int cz = blockIdx.z / a.H, h = blockIdx.z % a.H;
-    const int cs = a.c0 + cz, ch = cs * a.H + h;
+    const SwBTiles tl(a);
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < SWB_STAGES; ++i) {
+            mbar_init(full(i), 1);
+            mbar_init(empty(i), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(tfull(b), 1);
+            mbar_init(tempty(b), 8);  // every update warp, once per tile
+        }
+        for (int k = 0; k < SWB_SLOTS; ++k) {
+            mbar_init(sfull(k), 1);
+            mbar_init(sempty(k), 1);
+            mbar_init(sdone(k), 4);  // the four warps of the group that updated the chunk
+        }
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(base + L::SLOT), 256);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<uint32_t*>(base + L::SLOT);
     const int KB = (a.Tp + 63) / 64;  // tokens beyond T' carry zero gradients
+    const int chunk_bytes = a.momentum ? 2 * SWB_F32 : SWB_F32;
+    // state chunks of a tile: the rows of f0 .. f0 + 127 that lie below F
+    auto nchunks = [&](int f0) { return min(128, a.F - f0) / SWB_ROWS; };
 
     if (warp == 0) {
         if (lane == 0) {
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % L::NSTAGES;
-                if (kb >= L::NSTAGES && !mbar_wait(c.empty(s), ((kb / L::NSTAGES) - 1) & 1, a.status)) break;
-                const uint32_t sa = smem_u32(c.base + s * (4 * SW_BOX)), sb = sa + 2 * SW_BOX, fb = c.full(s);
-                mbar_expect_tx(fb, 4 * SW_BOX);
+            uint32_t kc = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < tl.count && ok; t += gridDim.x) {
+                int zh, m, f0, col0;
+                tl.decode(t, zh, m, f0, col0);
+                const int cz = zh / a.H, h = zh % a.H, ch = (a.c0 + cz) * a.H + h;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % SWB_STAGES;
+                    if (kc >= SWB_STAGES && !mbar_wait(empty(s), ((kc / SWB_STAGES) - 1) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sa = smem_u32(base + s * SWB_STAGE), sb = sa + 2 * SW_BOX, fb = full(s);
+                    mbar_expect_tx(fb, SWB_STAGE);
 #pragma unroll
-                for (int bx = 0; bx < 2; ++bx) {
-                    const uint32_t dst = sa + bx * SW_BOX;
-                    if (m < 2)
-                        tma_load_4d(dst, &tmUb, fb, col0 + bx * 64, h, a.u_row0 + kb * 64, a.u_chain0 + cz);
-                    else if (h < a.Hk)
-                        tma_load_4d(dst, &tmKb, fb, col0 + bx * 64, h, a.y_row0 + kb * 64, cz);
-                    else
-                        tma_load_4d(dst, &tmVb, fb, col0 + bx * 64, h - a.Hk, a.y_row0 + kb * 64, cz);
-                    if (m < 2)
-                        tma_load_4d(sb + bx * SW_BOX, &tmPG, fb, f0 + bx * 64, m, kb * 64, ch);
-                    else
-                        tma_load_3d(sb + bx * SW_BOX, &tmZ, fb, f0 + bx * 64, kb * 64, ch);
+                    for (int bx = 0; bx < 2; ++bx) {
+                        const uint32_t dst = sa + bx * SW_BOX;
+                        if (m < 2)
+                            tma_load_4d(dst, &tmUb, fb, col0 + bx * 64, h, a.u_row0 + kb * 64, a.u_chain0 + cz);
+                        else if (h < a.Hk)
+                            tma_load_4d(dst, &tmKb, fb, col0 + bx * 64, h, a.y_row0 + kb * 64, cz);
+                        else
+                            tma_load_4d(dst, &tmVb, fb, col0 + bx * 64, h - a.Hk, a.y_row0 + kb * 64, cz);
+                        if (m < 2)
+                            tma_load_4d(sb + bx * SW_BOX, &tmPG, fb, f0 + bx * 64, m, kb * 64, ch);
+                        else
+                            tma_load_3d(sb + bx * SW_BOX, &tmZ, fb, f0 + bx * 64, kb * 64, ch);
+                    }
                 }
             }
         }
@@ -371,118 +454,203 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
     } else if (warp == 1) {
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(128, 128, true, true);
+            uint32_t kc = 0;
+            int local = 0;
             bool ok = true;
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % L::NSTAGES;
-                if (!mbar_wait(c.full(s), (kb / L::NSTAGES) & 1, a.status)) {
-                    ok = false;
-                    break;
-                }
+            for (int t = blockIdx.x; t < tl.count && ok; t += gridDim.x, ++local) {
+                const int b = local & 1;
+                if (local >= 2 && !mbar_wait(tempty(b), ((local >> 1) - 1) & 1, a.status)) break;
                 tc_fence_after();
-                const uint32_t sa = smem_u32(c.base + s * (4 * SW_BOX)), sb = sa + 2 * SW_BOX;
+                const uint32_t d = tmem + b * 128;
+                for (int kb = 0; kb < KB; ++kb, ++kc) {
+                    const int s = kc % SWB_STAGES;
+                    if (!mbar_wait(full(s), (kc / SWB_STAGES) & 1, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(base + s * SWB_STAGE), sb = sa + 2 * SW_BOX;
 #pragma unroll
-                for (int k = 0; k < 4; ++k)
-                    umma_bf16(tmem, sdesc_sw128(sa + k * 16 * 128, SW_BOX), sdesc_sw128(sb + k * 16 * 128, SW_BOX),
-                              idesc, (kb == 0 && k == 0) ? 0u : 1u);
-                umma_commit(c.empty(s));
+                    for (int k = 0; k < 4; ++k)
+                        umma_bf16(d, sdesc_sw128(sa + k * 16 * 128, SW_BOX), sdesc_sw128(sb + k * 16 * 128, SW_BOX),
+                                  idesc, (kb == 0 && k == 0) ? 0u : 1u);
+                    umma_commit(empty(s));
+                }
+                if (ok) umma_commit(tfull(b));
             }
-            if (ok) umma_commit(c.tfull());
+        }
+        __syncwarp();
+    } else if (warp == SWB_STATE_WARP || warp == SWB_STORE_WARP) {
+        // ---- state producer (W and mu chunks of every tile, in update order) and store warp
+        //      (write each updated chunk back, then free its slot)
+        if (lane == 0) {
+            const bool producer = warp == SWB_STATE_WARP;
+            if (producer) {
+                tma_prefetch_map(&tmW1s);
+                tma_prefetch_map(&tmW2s);
+                if (a.momentum) {
+                    tma_prefetch_map(&tmM1s);
+                    tma_prefetch_map(&tmM2s);
+                }
+            }
+            uint32_t seq = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < tl.count && ok; t += gridDim.x) {
+                int zh, m, f0, col0;
+                tl.decode(t, zh, m, f0, col0);
+                const int ch = (a.c0 + zh / a.H) * a.H + zh % a.H;
+                const CUtensorMap* wm = m < 2 ? &tmW1s : &tmW2s;
+                const CUtensorMap* mm = m < 2 ? &tmM1s : &tmM2s;
+                const int row0 = (m == 1 ? a.F : 0) + f0;  // first state row of the tile within the head
+                const int nch = nchunks(f0);
+                for (int g = 0; g < nch; ++g, ++seq) {
+                    const int k = seq % SWB_SLOTS;
+                    const uint32_t slot = smem_u32(base + L::STATE + k * SWB_SLOT);
+                    if (producer) {
+                        if (seq >= SWB_SLOTS && !mbar_wait(sempty(k), ((seq / SWB_SLOTS) - 1) & 1, a.status)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_expect_tx(sfull(k), chunk_bytes);
+                        tma_load_3d(slot, wm, sfull(k), col0, row0 + g * SWB_ROWS, ch);
+                        if (a.momentum) tma_load_3d(slot + SWB_F32, mm, sfull(k), col0, row0 + g * SWB_ROWS, ch);
+                    } else {
+                        if (!mbar_wait(sdone(k), (seq / SWB_SLOTS) & 1, a.status)) {
+                            ok = false;
+                            break;
+                        }
+                        tma_store_3d(wm, slot, col0, row0 + g * SWB_ROWS, ch);
+                        if (a.momentum) tma_store_3d(mm, slot + SWB_F32, col0, row0 + g * SWB_ROWS, ch);
+                        bulk_commit();
+                        bulk_wait_read_all();  // the store has read the slot: hand it back
+                        mbar_arrive(sempty(k));
+                    }
+                }
+            }
+            if (!producer) bulk_wait_all();
         }
         __syncwarp();
     } else {
-        const int q = warp & 3, et = threadIdx.x - 64;
-        float* tab = reinterpret_cast<float*>(c.base + L::TAB);  // row scales [128], beta partials [4]
-        const int which = m < 2 ? 0 : 1;
-        const int rowbase = (m < 2 ? m * a.F : 0) + f0;  // first state row of the tile (within the head)
-        {
-            const int f = f0 + et;
-            float sc = 1.f;
-            if (a.renorm_pending && f < a.F) {
-                const float n = which ? a.n2[(size_t)ch * a.F + f] : a.n1[(size_t)ch * 2 * a.F + rowbase + et];
-                sc = renorm_scale(n, sw_ss(a, a.parity ^ 1, which, ch)[rowbase + et]);
+        // ---- update warps 2..9: group grp takes the tile's chunks grp, grp + 2; TMEM lane
+        //      quarter q = 32 weight columns, thread = one column
+        const int grp = (warp - 2) >> 2, q = warp & 3, et = threadIdx.x - 64 - grp * SWB_EPI_THREADS;
+        const uint32_t bar_id = 1 + grp;
+        float* tab = reinterpret_cast<float*>(base + L::TAB) + grp * (64 + 4);  // [64] scales
+        float* bred = tab + 64;                                                   // [4]
+        int* flag = reinterpret_cast<int*>(base + L::FLAG) + grp * 2;
+        bool finite = true;
+        uint32_t tile_seq0 = 0;  // state chunk sequence number of the current tile's first chunk
+        int local = 0;
+        for (int t = blockIdx.x; t < tl.count; t += gridDim.x, ++local) {
+            int zh, m, f0, col0;
+            tl.decode(t, zh, m, f0, col0);
+            const int cz = zh / a.H, cs = a.c0 + cz, ch = cs * a.H + zh % a.H;
+            const int which = m < 2 ? 0 : 1;
+            const int row0 = (m == 1 ? a.F : 0) + f0;   // first state row of the tile within the head
+            const int nch = nchunks(f0);
+            const int mine = (nch - grp + 1) / 2;         // this group's chunks: grp, grp + 2
+            const int b = local & 1;
+            {   // renorm scales of this group's chunks (32 rows each)
+                const int i = et >> 5, j = et & 31;
+                float sc = 1.f;
+                if (i < mine && a.renorm_pending) {
+                    const int r = row0 + (2 * i + grp) * SWB_ROWS + j;  // row within the head's matrix
+                    const float n = which ? a.n2[(size_t)ch * a.F + r] : a.n1[(size_t)ch * 2 * a.F + r];
+                    sc = renorm_scale(n, sw_ss(a, a.parity ^ 1, which, ch)[r]);
+                }
+                if (i < 2) tab[et] = sc;
             }
-            tab[et] = sc;
-            float v = 0.f;
-            if (a.momentum)
-                for (int t = et; t < a.Tp; t += 128) v += a.dbeta[(size_t)cs * a.win + a.tok0 + t];
-            v = warp_sum(v);
-            if (lane == 0) tab[128 + (warp - 2)] = v;
-        }
-        if (sw_wait_acc(c, a.status)) {
+            if (a.momentum) {
+                float v = 0.f;
+                for (int tk = et; tk < a.Tp; tk += SWB_EPI_THREADS) v += a.dbeta[(size_t)cs * a.win + a.tok0 + tk];
+                v = warp_sum(v);
+                if (lane == 0) bred[q] = v;
+            }
+            if (et == 0) flag[0] = mbar_wait(tfull(b), (local >> 1) & 1, a.status) ? 1 : 0;
+            __syncwarp();
+            named_bar_sync(bar_id, SWB_EPI_THREADS);
+            if (!flag[0]) break;
+            tc_fence_after();
             float beta = 0.f;
-            if (a.momentum) beta = sigmoidf_((tab[128] + tab[129] + tab[130] + tab[131]) / (float)a.Tp + a.b_beta[cs]);
-            const int col = col0 + q * 32 + lane;
-            const bool live = col < a.dh;
-            float* W = which ? a.W2 : a.W1;
-            float* M = which ? a.mu2 : a.mu1;
-            bf16* Wb = which ? a.W2b : a.W1b;
-            const size_t rows_head = which ? a.F : 2 * a.F;
-            const size_t base = ((size_t)ch * rows_head + rowbase) * a.dh + col;
-            const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
-            const uint64_t wpol = l2_evict_last_policy();  // phase A of the next segment reads the copy
+            if (a.momentum) beta = sigmoidf_((bred[0] + bred[1] + bred[2] + bred[3]) / (float)a.Tp + a.b_beta[cs]);
             float* cur = sw_ss(a, a.parity, which, ch);
-            bool finite = true;
-            // F is a multiple of 32, so a chunk of 16 rows is either wholly live or past F.  The loads
-            // of chunk cc + 1 are issued before chunk cc is updated and stored, so two chunks' loads
-            // are in flight per thread (the stores could alias them as far as the compiler knows,
-            // so it would not hoist them itself)
-            int nchunks = 0;
-            while (nchunks < 128 / SWB_ROWS && f0 + nchunks * SWB_ROWS < a.F) ++nchunks;
-            float v[SWB_ROWS], mo[SWB_ROWS];
-#pragma unroll
-            for (int j = 0; j < SWB_ROWS; ++j) {
-                const size_t idx = base + (size_t)j * a.dh;
-                v[j] = (live && nchunks > 0) ? W[idx] : 0.f;
-                mo[j] = (live && a.momentum && nchunks > 0) ? M[idx] : 0.f;
+            const int col = q * 32 + lane;  // column within the tile (= TMEM lane)
+            const bool live = col0 + col < a.dh;
+            const size_t rows_head = which ? a.F : 2 * a.F;
+            bf16* Wb = (which ? a.W2b : a.W1b) + (size_t)ch * rows_head * a.dh + col0 + col;
+            const uint64_t wpol = l2_evict_last_policy();  // phase A of the next segment reads the copy
+            const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 128;
+            if (mine == 0) {  // a group without chunks still hands the accumulator back
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(tempty(b));
             }
+            bool ok = true;
 #pragma unroll 1
-            for (int cc = 0; cc < nchunks; ++cc) {
-                float nv[SWB_ROWS], nmo[SWB_ROWS], gv[SWB_ROWS];
-                const bool more = cc + 1 < nchunks;
-#pragma unroll
-                for (int j = 0; j < SWB_ROWS; ++j) {
-                    const size_t idx = base + (size_t)((cc + 1) * SWB_ROWS + j) * a.dh;
-                    nv[j] = (live && more) ? W[idx] : 0.f;
-                    nmo[j] = (live && more && a.momentum) ? M[idx] : 0.f;
+            for (int i = 0; i < mine; ++i) {
+                const int c = 2 * i + grp;
+                const uint32_t seq = tile_seq0 + c;
+                const int k = seq % SWB_SLOTS;
+                const int r0 = row0 + c * SWB_ROWS;
+                float gv[32];
+                tmem_ld32(lane_base + c * SWB_ROWS, gv);
+                if (i == mine - 1) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(tempty(b));
                 }
-                tmem_ld16(lane_base + cc * SWB_ROWS, gv);
-#pragma unroll
-                for (int j = 0; j < SWB_ROWS; ++j) {
-                    const size_t idx = base + (size_t)(cc * SWB_ROWS + j) * a.dh;
-                    const float mn = fmaf(beta, mo[j], gv[j]);
-                    const float wn = fmaf(tab[cc * SWB_ROWS + j], v[j], -mn);
-                    if (live) {
-                        W[idx] = wn;
-                        if (a.momentum) M[idx] = mn;
-                        st_bf16_hint(Wb + idx, __float2bfloat16_rn(wn), wpol);
-                    }
-                    gv[j] = live ? wn * wn : 0.f;
+                if (et == 0) flag[1] = mbar_wait(sfull(k), (seq / SWB_SLOTS) & 1, a.status) ? 1 : 0;
+                __syncwarp();
+                named_bar_sync(bar_id, SWB_EPI_THREADS);
+                if (!flag[1]) {
+                    ok = false;
+                    break;
                 }
-                // transpose-reduce over the 16 rows: afterwards lane l holds the partial of row
-                // l & 15 over the 16 lanes that share bit 4 of l; the xor-16 exchange adds the rest
+                uint8_t* slot = base + L::STATE + k * SWB_SLOT;
+                float* Ws = reinterpret_cast<float*>(slot);
+                float* Ms = reinterpret_cast<float*>(slot + SWB_F32);
+                bf16* bp = Wb + (size_t)r0 * a.dh;
+                float v[32];
 #pragma unroll
-                for (int sft = SWB_ROWS / 2; sft >= 1; sft >>= 1) {
+                for (int j = 0; j < 32; ++j) {
+                    const float sc = tab[i * SWB_ROWS + j];
+                    const float mo = a.momentum ? Ms[j * 128 + col] : 0.f;
+                    const float mn = fmaf(beta, mo, gv[j]);
+                    const float wn = fmaf(sc, Ws[j * 128 + col], -mn);
+                    Ws[j * 128 + col] = wn;
+                    if (a.momentum) Ms[j * 128 + col] = mn;
+                    if (live) st_bf16_hint(bp + (size_t)j * a.dh, __float2bfloat16_rn(wn), wpol);
+                    v[j] = wn * wn;  // columns past dh hold zeros; a NaN or Inf makes its row's sum non-finite
+                }
+                // transpose-reduce: afterwards lane j holds this warp's 32-column partial of row j
+#pragma unroll
+                for (int sft = 16; sft >= 1; sft >>= 1) {
                     const bool upper = (lane & sft) != 0;
 #pragma unroll
                     for (int u = 0; u < sft; ++u) {
-                        const float send = upper ? gv[u] : gv[u + sft];
-                        const float keep = upper ? gv[u + sft] : gv[u];
-                        gv[u] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+                        const float send = upper ? v[u] : v[u + sft];
+                        const float keep = upper ? v[u + sft] : v[u];
+                        v[u] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
                     }
                 }
-                gv[0] += __shfl_xor_sync(0xffffffffu, gv[0], 16);
-                finite = finite && isfinite(gv[0]);
-                if (lane < SWB_ROWS) atomicAdd(&cur[rowbase + cc * SWB_ROWS + lane], gv[0]);
-#pragma unroll
-                for (int j = 0; j < SWB_ROWS; ++j) {
-                    v[j] = nv[j];
-                    mo[j] = nmo[j];
-                }
+                finite = finite && isfinite(v[0]);
+                atomicAdd(&cur[r0 + lane], v[0]);
+                // make this warp's shared-memory writes visible to the TMA store, then tell the store warp
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(sdone(k));
             }
-            if (!finite) atomicOr(a.status, DEV_NONFINITE);
+            if (!ok) break;
+            tile_seq0 += nch;
+            // the scale table is rewritten for the next tile only after every warp of the group is done
+            named_bar_sync(bar_id, SWB_EPI_THREADS);
         }
+        if (!finite) atomicOr(a.status, DEV_NONFINITE);
     }
-    sw_teardown(tmem, 128);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, 256);
 }
 
 // ------------------------------------------------------------------ memory read
@@ -715,9 +883,12 @@ cudaError_t launch_swiglu_phase_b(const DevState& s, const SwMaps& m, const SwIn
                                   cudaStream_t st) {
     cudaError_t e = sw_attrs();
     if (e != cudaSuccess) return e;
-    const SwArgs a = sw_args(s, w);
-    dim3 grid(3 * ((a.dh + 127) / 128), (a.F + 127) / 128, w.nc * a.H);
-    swiglu_b_kernel<<<grid, SW_THREADS, SwLayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.PG, m.Z, a);
+    SwArgs a = sw_args(s, w);
+    a.nc_launch = w.nc;
+    const int ntiles = w.nc * a.H * 3 * ((a.F + 127) / 128) * ((a.dh + 127) / 128);
+    const int grid = ntiles < sw_sms() ? ntiles : sw_sms();
+    swiglu_b_kernel<<<grid, SWB_THREADS, SwLayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.PG, m.Z,
+                                                               m.W1s, m.M1s, m.W2s, m.M2s, a);
     return cudaGetLastError();
 }
 
