@@ -319,7 +319,7 @@ swiglu_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__
 
 // ------------------------------------------------------------------ phase B (gradient + update)
 
-// Persistent, one CTA per SM, over tiles (matrix m of W_in / W_gate / W_out, 128 hidden rows,
+// Persistent, one CTA per SM, over tiles (matrix m of W_in / W_gate / W_out, 256 hidden rows,
 // 128 weight columns, head): the gradient with TMEM lane = weight column (both operands
 // MN-major) into one of two TMEM accumulators, so the MMAs of tile i+1 run while tile i is
 // updated.  Warps: 0 operand producer, 1 MMA issuer, 2..9 update in two groups of four (one warp
@@ -333,8 +333,9 @@ constexpr int SWB_ROWS = 32;                               // hidden rows per st
 constexpr int SWB_SLOTS = 4;
 constexpr int SWB_F32 = SWB_ROWS * 128 * 4;                // 16 KB
 constexpr int SWB_SLOT = 2 * SWB_F32;                      // W and mu: 32 KB
-constexpr int SWB_STAGES = 3;
-constexpr int SWB_STAGE = 4 * SW_BOX;                      // 32 KB: 128 columns + 128 hidden rows
+constexpr int SWB_N = 256;                                 // hidden rows per tile (all of F <= 256)
+constexpr int SWB_STAGES = 2;
+constexpr int SWB_STAGE = (2 + SWB_N / 64) * SW_BOX;       // 48 KB: 128 columns + 256 hidden rows
 constexpr int SWB_THREADS = 12 * 32;
 constexpr int SWB_EPI_THREADS = 4 * 32;                    // per update group
 constexpr int SWB_STATE_WARP = 10, SWB_STORE_WARP = 11;
@@ -345,8 +346,8 @@ struct SwLayoutB {
     static constexpr int NBARS = 2 * SWB_STAGES + 4 + 3 * SWB_SLOTS;
     static constexpr int SLOT = BARS + NBARS * 8;
     static constexpr int FLAG = SLOT + 16;
-    static constexpr int TAB = FLAG + 16;                      // per group: [64] renorm scales + [4] decay partials
-    static constexpr int END = TAB + 2 * (64 + 4) * 4;
+    static constexpr int TAB = FLAG + 16;                      // per group: [SWB_N/2] renorm scales + [4] decay partials
+    static constexpr int END = TAB + 2 * (SWB_N / 2 + 4) * 4;
     static constexpr int DYN = END + 1024;
 };
 static_assert(SwLayoutB::DYN <= 227 * 1024, "phase B shared memory budget");
@@ -356,13 +357,13 @@ struct SwBTiles {
     int NC, NR, count;
     __device__ SwBTiles(const SwArgs& a) {
         NC = (a.dh + 127) / 128;
-        NR = (a.F + 127) / 128;
+        NR = (a.F + SWB_N - 1) / SWB_N;
         count = a.nc_launch * a.H * 3 * NR * NC;
     }
     __device__ void decode(int t, int& zh, int& m, int& f0, int& col0) const {
         col0 = (t % NC) * 128;
         t /= NC;
-        f0 = (t % NR) * 128;
+        f0 = (t % NR) * SWB_N;
         t /= NR;
         m = t % 3;
         zh = t / 3;
@@ -405,7 +406,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
         fence_mbar_init();
     }
     if (warp == 0) {
-        tmem_alloc(smem_u32(base + L::SLOT), 256);
+        tmem_alloc(smem_u32(base + L::SLOT), 2 * SWB_N);
         tmem_relinquish();
     }
     tc_fence_before();
@@ -414,8 +415,8 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
     const uint32_t tmem = *reinterpret_cast<uint32_t*>(base + L::SLOT);
     const int KB = (a.Tp + 63) / 64;  // tokens beyond T' carry zero gradients
     const int chunk_bytes = a.momentum ? 2 * SWB_F32 : SWB_F32;
-    // state chunks of a tile: the rows of f0 .. f0 + 127 that lie below F
-    auto nchunks = [&](int f0) { return min(128, a.F - f0) / SWB_ROWS; };
+    // state chunks of a tile: the rows of f0 .. f0 + SWB_N - 1 that lie below F
+    auto nchunks = [&](int f0) { return min(SWB_N, a.F - f0) / SWB_ROWS; };
 
     if (warp == 0) {
         if (lane == 0) {
@@ -442,6 +443,9 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
                             tma_load_4d(dst, &tmKb, fb, col0 + bx * 64, h, a.y_row0 + kb * 64, cz);
                         else
                             tma_load_4d(dst, &tmVb, fb, col0 + bx * 64, h - a.Hk, a.y_row0 + kb * 64, cz);
+                    }
+#pragma unroll
+                    for (int bx = 0; bx < SWB_N / 64; ++bx) {  // hidden rows past F load as zeros
                         if (m < 2)
                             tma_load_4d(sb + bx * SW_BOX, &tmPG, fb, f0 + bx * 64, m, kb * 64, ch);
                         else
@@ -453,7 +457,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
         __syncwarp();
     } else if (warp == 1) {
         if (lane == 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, 128, true, true);
+            const uint32_t idesc = idesc_bf16_f32(128, SWB_N, true, true);
             uint32_t kc = 0;
             int local = 0;
             bool ok = true;
@@ -461,7 +465,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
                 const int b = local & 1;
                 if (local >= 2 && !mbar_wait(tempty(b), ((local >> 1) - 1) & 1, a.status)) break;
                 tc_fence_after();
-                const uint32_t d = tmem + b * 128;
+                const uint32_t d = tmem + b * SWB_N;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
                     const int s = kc % SWB_STAGES;
                     if (!mbar_wait(full(s), (kc / SWB_STAGES) & 1, a.status)) {
@@ -535,8 +539,8 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
         //      quarter q = 32 weight columns, thread = one column
         const int grp = (warp - 2) >> 2, q = warp & 3, et = threadIdx.x - 64 - grp * SWB_EPI_THREADS;
         const uint32_t bar_id = 1 + grp;
-        float* tab = reinterpret_cast<float*>(base + L::TAB) + grp * (64 + 4);  // [64] scales
-        float* bred = tab + 64;                                                   // [4]
+        float* tab = reinterpret_cast<float*>(base + L::TAB) + grp * (SWB_N / 2 + 4);  // [SWB_N/2] scales
+        float* bred = tab + SWB_N / 2;                                                  // [4]
         int* flag = reinterpret_cast<int*>(base + L::FLAG) + grp * 2;
         bool finite = true;
         uint32_t tile_seq0 = 0;  // state chunk sequence number of the current tile's first chunk
@@ -558,7 +562,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
                     const float n = which ? a.n2[(size_t)ch * a.F + r] : a.n1[(size_t)ch * 2 * a.F + r];
                     sc = renorm_scale(n, sw_ss(a, a.parity ^ 1, which, ch)[r]);
                 }
-                if (i < 2) tab[et] = sc;
+                tab[et] = sc;  // i < SWB_N / 64: four chunks of this group at most
             }
             if (a.momentum) {
                 float v = 0.f;
@@ -579,7 +583,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
             const size_t rows_head = which ? a.F : 2 * a.F;
             bf16* Wb = (which ? a.W2b : a.W1b) + (size_t)ch * rows_head * a.dh + col0 + col;
             const uint64_t wpol = l2_evict_last_policy();  // phase A of the next segment reads the copy
-            const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * 128;
+            const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + b * SWB_N;
             if (mine == 0) {  // a group without chunks still hands the accumulator back
                 tc_fence_before();
                 __syncwarp();
@@ -650,7 +654,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 0) tmem_dealloc(tmem, 256);
+    if (warp == 0) tmem_dealloc(tmem, 2 * SWB_N);
 }
 
 // ------------------------------------------------------------------ memory read
@@ -885,7 +889,7 @@ cudaError_t launch_swiglu_phase_b(const DevState& s, const SwMaps& m, const SwIn
     if (e != cudaSuccess) return e;
     SwArgs a = sw_args(s, w);
     a.nc_launch = w.nc;
-    const int ntiles = w.nc * a.H * 3 * ((a.F + 127) / 128) * ((a.dh + 127) / 128);
+    const int ntiles = w.nc * a.H * 3 * ((a.F + SWB_N - 1) / SWB_N) * ((a.dh + 127) / 128);
     const int grid = ntiles < sw_sms() ? ntiles : sw_sms();
     swiglu_b_kernel<<<grid, SWB_THREADS, SwLayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.PG, m.Z,
                                                                m.W1s, m.M1s, m.W2s, m.M2s, a);
