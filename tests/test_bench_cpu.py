@@ -1,0 +1,53 @@
+"""The bench's bookkeeping, without a GPU: algorithmic work per launch and the use of the
+recorded DRAM traffic."""
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+import workloads as wk  # noqa: E402
+
+
+def test_phase_b_algorithmic_bytes_per_launch():
+    # one segment of 8 chains of the 16-layer shape: 18 B per parameter of state (W and
+    # momentum read and written in fp32, the bf16 operand copy written), U and Y in bf16,
+    # dH and At in bf16
+    wl = wk.WORKLOADS["l16_d2048_128k"]
+    params = wl.d_hid * (wl.d_in + wl.d_out)
+    per_chain = params * 18 + wl.seg_T * (wl.d_in + wl.d_out) * 2 + wl.seg_T * wl.d_hid * 2 * 2
+    flops, byts = bench.kernel_work(wl, "phase_b", 8)
+    assert byts == pytest.approx(8 * per_chain)
+    assert byts == pytest.approx(494.5e6, rel=1e-3)
+    assert flops == pytest.approx(8 * 2 * wl.seg_T * wl.d_hid * (wl.d_in + wl.d_out))
+
+
+def test_recorded_traffic_applies_only_to_its_shape(tmp_path, monkeypatch):
+    # a record for this source of the kernel, taken on one segment of 8 chains of the 16-layer
+    # shape at T = 512, in a scratch copy of the layout bench.py reads
+    src = open(os.path.join(ROOT, "paper_2608_17616_gb300", "csrc", "ttl_tc.cu")).read()
+    (tmp_path / "paper_2608_17616_gb300" / "csrc").mkdir(parents=True)
+    (tmp_path / "paper_2608_17616_gb300" / "csrc" / "ttl_tc.cu").write_text(src)
+    (tmp_path / "profiles").mkdir()
+    sha = bench.kernel_source_sha(src, "phase_b")
+    shape = bench.shape_key(wk.WORKLOADS["l16_d2048_128k"])
+    (tmp_path / "profiles" / "ncu_traffic.txt").write_text(
+        f"# test record\nkernel=phase_b source_sha={sha} shape={shape} bytes_per_launch=400000000 chains=8\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    got = {n: bench.ncu_traffic("phase_b", 8.0, wk.WORKLOADS[n])[0]
+           for n in ("l16_d2048_128k", "l16_d2048_32k", "ctx8_l16_T512", "ctx8_l16_T1024", "l28_d3072_128k",
+                     "swiglu_l24_d896_32k")}
+    assert got["l16_d2048_128k"] == pytest.approx(4e8)
+    assert got["l16_d2048_32k"] == got["l16_d2048_128k"] and got["ctx8_l16_T512"] == got["l16_d2048_128k"]
+    for other in ("ctx8_l16_T1024", "l28_d3072_128k", "swiglu_l24_d896_32k"):
+        assert got[other] is None, other
+    # scaled in proportion to the chains of a launch
+    assert bench.ncu_traffic("phase_b", 16.0, wk.WORKLOADS["l16_d2048_128k"])[0] == pytest.approx(8e8)
+    # a record of another version of the kernel is not used
+    banner = "// ------------------------------------------------------------------ phase B"
+    (tmp_path / "paper_2608_17616_gb300" / "csrc" / "ttl_tc.cu").write_text(
+        src.replace(banner, banner + "\n// edited", 1))
+    assert bench.ncu_traffic("phase_b", 8.0, wk.WORKLOADS["l16_d2048_128k"])[0] is None
