@@ -22,31 +22,41 @@ namespace {
 
 constexpr int TM = 64, TN = 64, TK = 64;
 
-// acc[i][j] += sum_k A(m0 + ty*4 + i, k) * B(n0 + tx*4 + j, k) for one 64 x 64 tile.
+// acc[i][j] += sum_k A(m0 + ty*MR + i, k) * B(n0 + tx*4 + j, k) for one (16 MR) x 64 tile.
 // A(m, k) = A[m*sam + k*sak]; rows m >= m_valid and k >= k_valid read as 0.
-__device__ __forceinline__ void simt_tile(float (&acc)[4][4], const float* A, long long sam, long long sak,
+template <int MR>
+__device__ __forceinline__ void simt_tile(float (&acc)[MR][4], const float* A, long long sam, long long sak,
                                           const float* B, long long sbn, long long sbk, int K, int m_valid,
-                                          int k_valid, float (*As)[TM + 4], float (*Bs)[TN + 4]) {
+                                          int k_valid, float (*As)[16 * MR + 4], float (*Bs)[TN + 4]) {
+    constexpr int TMR = 16 * MR;  // rows of the tile
     const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
     for (int k0 = 0; k0 < K; k0 += TK) {
-        // 64 x TK elements of each operand, TK consecutive along the contiguous dimension
-        float av[TM * TK / 256], bv[TN * TK / 256];
+        // TMR x TK elements of A and 64 x TK of B, TK consecutive along the contiguous dimension
+        float av[TMR * TK / 256], bv[TN * TK / 256];
 #pragma unroll
-        for (int r = 0; r < TM * TK / 256; ++r) {
+        for (int r = 0; r < TMR * TK / 256; ++r) {
             const int e = tid + 256 * r;
             int m, k;
-            if (sak == 1) { m = e / TK; k = e % TK; } else { m = e % TM; k = e / TM; }
+            if (sak == 1) { m = e / TK; k = e % TK; } else { m = e % TMR; k = e / TMR; }
             av[r] = (m < m_valid && k0 + k < k_valid) ? A[m * sam + (k0 + k) * sak] : 0.0f;
+        }
+#pragma unroll
+        for (int r = 0; r < TN * TK / 256; ++r) {
+            const int e = tid + 256 * r;
             int n, kb;
             if (sbk == 1) { n = e / TK; kb = e % TK; } else { n = e % TN; kb = e / TN; }
             bv[r] = (k0 + kb < k_valid) ? B[n * sbn + (k0 + kb) * sbk] : 0.0f;
         }
 #pragma unroll
-        for (int r = 0; r < TM * TK / 256; ++r) {
+        for (int r = 0; r < TMR * TK / 256; ++r) {
             const int e = tid + 256 * r;
             int m, k;
-            if (sak == 1) { m = e / TK; k = e % TK; } else { m = e % TM; k = e / TM; }
+            if (sak == 1) { m = e / TK; k = e % TK; } else { m = e % TMR; k = e / TMR; }
             As[k][m] = av[r];
+        }
+#pragma unroll
+        for (int r = 0; r < TN * TK / 256; ++r) {
+            const int e = tid + 256 * r;
             int n, kb;
             if (sbk == 1) { n = e / TK; kb = e % TK; } else { n = e % TN; kb = e / TN; }
             Bs[kb][n] = bv[r];
@@ -54,13 +64,13 @@ __device__ __forceinline__ void simt_tile(float (&acc)[4][4], const float* A, lo
         __syncthreads();
 #pragma unroll
         for (int k = 0; k < TK; ++k) {
-            float a[4], b[4];
+            float a[MR], b[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) a[i] = As[k][ty * 4 + i];
+            for (int i = 0; i < MR; ++i) a[i] = As[k][ty * MR + i];
 #pragma unroll
             for (int j = 0; j < 4; ++j) b[j] = Bs[k][tx * 4 + j];
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
+            for (int i = 0; i < MR; ++i)
 #pragma unroll
                 for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
         }
@@ -95,13 +105,17 @@ __device__ __forceinline__ const float* ss_ptr(const F32SegArgs& a, int parity, 
     return a.sumsq + ((size_t)(parity * 2 + which) * a.C) * a.d_hid;
 }
 
+// Phase A takes tiles of 32 tokens x 64 hidden units (2 x 4 per thread): the fp32 workload has
+// only T = 128 tokens a segment, so 64-row tiles would leave all but 16 SMs idle.
+constexpr int A_MR = 2, A_TM = 16 * A_MR;
+
 __global__ void __launch_bounds__(256) phase_a_f32_kernel(const F32SegArgs a) {
-    __shared__ float As[TK][TM + 4], Bs[TK][TN + 4];
+    __shared__ float As[TK][A_TM + 4], Bs[TK][TN + 4];
     __shared__ float red[8];
     const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
-    const int t0 = blockIdx.x * TM, h0 = blockIdx.y * TN, cz = blockIdx.z, cs = a.c0 + cz;
+    const int t0 = blockIdx.x * A_TM, h0 = blockIdx.y * TN, cz = blockIdx.z, cs = a.c0 + cz;
     long long avail = a.row_avail - t0;
-    int m_valid = (int)min((long long)min(TM, a.Tp - t0), avail);
+    int m_valid = (int)min((long long)min(A_TM, a.Tp - t0), avail);
     if (m_valid < 0) m_valid = 0;
     // zero this segment's row sums of squares (read by phase B of this segment)
     if (blockIdx.x == 0 && tid < TN) {
@@ -109,7 +123,7 @@ __global__ void __launch_bounds__(256) phase_a_f32_kernel(const F32SegArgs a) {
         cur[0] = 0.f;
         cur[(size_t)a.C * a.d_hid] = 0.f;
     }
-    float accH[4][4] = {}, accR[4][4] = {};
+    float accH[A_MR][4] = {}, accR[A_MR][4] = {};
     const float* U = a.U + cz * a.u_cstride + (long long)t0 * a.d_in;
     simt_tile(accH, U, a.d_in, 1, a.W1 + ((size_t)cs * a.d_hid + h0) * a.d_in, a.d_in, 1, a.d_in, m_valid,
               a.d_in, As, Bs);
@@ -130,8 +144,8 @@ __global__ void __launch_bounds__(256) phase_a_f32_kernel(const F32SegArgs a) {
     }
     float lsum = 0.f;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int t = t0 + ty * 4 + i;
+    for (int i = 0; i < A_MR; ++i) {
+        const int t = t0 + ty * A_MR + i;
         float ct = 0.f;
         if (t < a.Tp && t - t0 < m_valid) {
             float e;
@@ -385,7 +399,7 @@ __global__ void __launch_bounds__(256) read_norm_kernel(DevState s, int Q, Tout*
 
 cudaError_t launch_phase_a_f32(const DevState& s, const SegWork& w, cudaStream_t st) {
     F32SegArgs a = make_f32_args(s, w);
-    dim3 grid((s.T + TM - 1) / TM, s.d_hid / TN, w.nc);
+    dim3 grid((s.T + A_TM - 1) / A_TM, s.d_hid / TN, w.nc);
     phase_a_f32_kernel<<<grid, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
