@@ -181,23 +181,26 @@ __global__ void __launch_bounds__(256) phase_a_f32_kernel(const F32SegArgs a) {
     }
 }
 
+// Phase B takes tiles of 32 hidden rows x 64 weight columns (2 x 4 per thread), for the same reason.
+constexpr int B_MR = 2, B_TM = 16 * B_MR;
+
 __global__ void __launch_bounds__(256) phase_b_f32_kernel(const F32SegArgs a) {
-    __shared__ float As[TK][TM + 4], Bs[TK][TN + 4];
+    __shared__ float As[TK][B_TM + 4], Bs[TK][TN + 4];
     __shared__ float red[8];
     __shared__ float s_beta;
     const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
-    const int col0 = blockIdx.x * TN, h0 = blockIdx.y * TM, cz = blockIdx.z, cs = a.c0 + cz;
+    const int col0 = blockIdx.x * TN, h0 = blockIdx.y * B_TM, cz = blockIdx.z, cs = a.c0 + cz;
     const bool isW1 = col0 < a.d_in;
     const int kv = (int)min((long long)a.Tp, a.row_avail);
-    float acc[4][4] = {};
+    float acc[B_MR][4] = {};
     if (isW1) {
         const float* U = a.U + cz * a.u_cstride + col0;
-        simt_tile(acc, a.dH + (size_t)cs * a.T * a.d_hid + h0, 1, a.d_hid, U, 1, a.d_in, a.Tp, TM, kv, As, Bs);
+        simt_tile(acc, a.dH + (size_t)cs * a.T * a.d_hid + h0, 1, a.d_hid, U, 1, a.d_in, a.Tp, B_TM, kv, As, Bs);
     } else {
         const int dh = a.d_out / 2;
         const int o0 = col0 - a.d_in;
         const float* Y = (o0 < dh ? a.K + o0 : a.V + (o0 - dh)) + cz * a.y_cstride;
-        simt_tile(acc, a.At + (size_t)cs * a.T * a.d_hid + h0, 1, a.d_hid, Y, 1, dh, a.Tp, TM, kv, As, Bs);
+        simt_tile(acc, a.At + (size_t)cs * a.T * a.d_hid + h0, 1, a.d_hid, Y, 1, dh, a.Tp, B_TM, kv, As, Bs);
     }
     // momentum decay beta_s = sigmoid(mean_t w_beta . x_t + b_beta)
     if (a.momentum) {
@@ -224,8 +227,8 @@ __global__ void __launch_bounds__(256) phase_b_f32_kernel(const F32SegArgs a) {
     float* cur = a.sumsq + ((size_t)(a.parity * 2 + which) * a.C + cs) * a.d_hid;
     bool finite = true;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int h = h0 + ty * 4 + i;
+    for (int i = 0; i < B_MR; ++i) {
+        const int h = h0 + ty * B_MR + i;
         const float s = a.renorm_pending ? renorm_scale(n0[h], prev[h]) : 1.f;
         float* wrow = W + (size_t)h * width + c_local + tx * 4;
         float* mrow = M ? M + (size_t)h * width + c_local + tx * 4 : nullptr;
@@ -406,7 +409,7 @@ cudaError_t launch_phase_a_f32(const DevState& s, const SegWork& w, cudaStream_t
 
 cudaError_t launch_phase_b_f32(const DevState& s, const SegWork& w, cudaStream_t st) {
     F32SegArgs a = make_f32_args(s, w);
-    dim3 grid((s.d_in + s.d_out) / TN, s.d_hid / TM, w.nc);
+    dim3 grid((s.d_in + s.d_out) / TN, s.d_hid / B_TM, w.nc);
     phase_b_f32_kernel<<<grid, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
