@@ -257,9 +257,7 @@ mone_status build_state_maps(mone_mem* m) {
              encode_map_bf16_3d(&m->maps.Ub, s.U, s.d_in, s.win_rows, s.C, 64, 64);
     if (ok)
         ok = encode_map_plain_3d(&m->maps.W1s, s.W1, true, s.d_in, s.d_hid, s.C, 128, 32) &&
-             encode_map_plain_3d(&m->maps.W2s, s.W2, true, s.d_out, s.d_hid, s.C, 128, 32) &&
-             encode_map_plain_3d(&m->maps.W1o, s.W1b, false, s.d_in, s.d_hid, s.C, 128, 32) &&
-             encode_map_plain_3d(&m->maps.W2o, s.W2b, false, s.d_out, s.d_hid, s.C, 128, 32);
+             encode_map_plain_3d(&m->maps.W2s, s.W2, true, s.d_out, s.d_hid, s.C, 128, 32);
     if (ok && s.mu1)
         ok = encode_map_plain_3d(&m->maps.M1s, s.mu1, true, s.d_in, s.d_hid, s.C, 128, 32) &&
              encode_map_plain_3d(&m->maps.M2s, s.mu2, true, s.d_out, s.d_hid, s.C, 128, 32);

@@ -133,7 +133,6 @@ struct TcMaps {
     CUtensorMap dH, At;          // MN-major boxes {64, 64} over [C][T][d_hid]
     CUtensorMap Ua, Ub;          // scratch U: K-major {64,128} and MN {64,64}
     CUtensorMap W1s, W2s, M1s, M2s;  // fp32 state chunks {128 cols, 32 rows}, no swizzle
-    CUtensorMap W1o, W2o;            // bf16 operand-copy chunks {128 cols, 32 rows}, no swizzle
     CUtensorMap W2m;                 // bf16 W2 copy, MN-major boxes {64 outputs, 64 hidden} (memory read)
     CUtensorMap Amse;                // squared-error activations, K-major {64, 128}
 };

@@ -681,8 +681,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                   const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmDH,
                   const __grid_constant__ CUtensorMap tmAT, const __grid_constant__ CUtensorMap tmW1s,
                   const __grid_constant__ CUtensorMap tmW2s, const __grid_constant__ CUtensorMap tmM1s,
-                  const __grid_constant__ CUtensorMap tmM2s, const __grid_constant__ CUtensorMap tmW1o,
-                  const __grid_constant__ CUtensorMap tmW2o, const TcArgs a) {
+                  const __grid_constant__ CUtensorMap tmM2s, const TcArgs a) {
     extern __shared__ uint8_t smem_raw[];
     using L = LayoutBT<PAIR>;
     constexpr int NS = L::STAGES;
@@ -1445,12 +1444,12 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
         cfg.attrs = at;
         cfg.numAttrs = 1;
         return cudaLaunchKernelEx(&cfg, tc_phase_b_kernel<true>, U, in.Kb, in.Vb, m.dH, m.At, m.W1s, m.W2s, m.M1s,
-                                  m.M2s, m.W1o, m.W2o, a);
+                                  m.M2s, a);
     }
     const int ntiles = w.nc * ((s.d_in + s.d_out) / B_BM) * (s.d_hid / B_BN);
     const int grid = ntiles < g_sms ? ntiles : g_sms;
     tc_phase_b_kernel<false><<<grid, B_THREADS, LayoutB::DYN, st>>>(U, in.Kb, in.Vb, m.dH, m.At, m.W1s, m.W2s, m.M1s,
-                                                                     m.M2s, m.W1o, m.W2o, a);
+                                                                     m.M2s, a);
     return cudaGetLastError();
 }
 
