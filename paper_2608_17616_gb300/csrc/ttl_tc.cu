@@ -83,6 +83,8 @@ struct TcArgs {
     bf16 *dH, *At;              // [C][T][d_hid]
     float* loss;                // [nc] or null
     int* status;
+    int r_only;                 // phase A pairs: At and c SiLU'(x) / |z| come from the squared-error
+                                // pre-pass (the latter in dH); accumulate R only and form dH in place
 };
 
 __device__ __forceinline__ float* ss_row(const TcArgs& a, int parity, int which, int cs) {
@@ -332,6 +334,64 @@ __device__ __forceinline__ bool phase_a_epilogue_split(const TcArgs& a, uint32_t
     return true;
 }
 
+// Epilogue of a phase A pair tile in the R-only form (squared-error loss): At and
+// s' = c_t SiLU'(x) / |z_t| were written by the pre-pass (s' in dH), so dH = R s2 s' in place.
+template <int BN, class Release>
+__device__ __forceinline__ bool phase_a_epilogue_r_only(const TcArgs& a, uint32_t tmem, uint32_t tfull_bar,
+                                                        int parity_bit, float* tab, int* flag, int cs, int h0,
+                                                        int trow, bool zero_ss, uint8_t* stg, Release&& release) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int e = warp - 2, q = warp & 3, ch = e >> 2, et = threadIdx.x - 64;
+    if (et < BN) {
+        const int h = h0 + et;
+        float s2 = 1.f;
+        if (a.renorm_pending)
+            s2 = renorm_scale(a.n2[(size_t)cs * a.d_hid + h], ss_row(a, a.parity ^ 1, 1, cs)[h]);
+        tab[BN + et] = s2;
+        if (zero_ss) {
+            ss_row(a, a.parity, 0, cs)[h] = 0.f;
+            ss_row(a, a.parity, 1, cs)[h] = 0.f;
+        }
+    }
+    if (et == 0) *flag = mbar_wait(tfull_bar, parity_bit, a.status) ? 1 : 0;
+    __syncwarp();
+    named_bar_sync(EPI_BAR, EPI_THREADS);
+    if (!*flag) return false;
+    tc_fence_after();
+    const int row = q * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+    const size_t r0 = ((size_t)cs * a.T + trow + q * 32) * a.d_hid + h0;  // this warp's first row
+    const bf16* sp_row = a.dH + ((size_t)cs * a.T + trow + row) * a.d_hid + h0;
+    constexpr int CHUNKS = BN / 64;
+#pragma unroll 1
+    for (int cc = 0; cc < CHUNKS; ++cc) {
+        const int c0 = ch * (BN / 2) + cc * 32;
+        float rv[32];
+        tmem_ld32(lane_base + BN + c0, rv);
+        if (cc == CHUNKS - 1) {
+            tc_fence_before();
+            __syncwarp();
+            release();
+        }
+        uint4 sv[4];
+#pragma unroll
+        for (int v = 0; v < 4; ++v) sv[v] = *reinterpret_cast<const uint4*>(sp_row + c0 + v * 8);
+        uint32_t pd[16];
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const __nv_bfloat162* sb = reinterpret_cast<const __nv_bfloat162*>(&sv[v]);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float2 sf = __bfloat1622float2(sb[u]);
+                const int j = v * 8 + 2 * u;
+                pd[j / 2] = pack_bf16(rv[j] * tab[BN + c0 + j] * sf.x, rv[j + 1] * tab[BN + c0 + j + 1] * sf.y);
+            }
+        }
+        store_rows_coalesced(stg, pd, a.dH + r0 + c0, a.d_hid, lane);  // in place: every lane has read its row
+    }
+    return true;
+}
+
 __global__ void __launch_bounds__(THREADS, 1)
 tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmW1,
@@ -499,7 +559,8 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
     const int n_tp = a.T / (2 * A_BM), n_ht = a.d_hid / P_BN;
     const int npairs = a.nc * n_ht * n_tp;
     const int cluster = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
-    const int KB1 = a.d_in / BK, KB = KB1 + a.d_out / BK, half = (a.d_out / 2) / BK;
+    // the R-only form (squared-error loss) takes no H k-blocks
+    const int KB1 = a.r_only ? 0 : a.d_in / BK, KB = KB1 + a.d_out / BK, half = (a.d_out / 2) / BK;
 
     if (warp == 0) {
         if (lane == 0) {
@@ -593,11 +654,14 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
             float* tab = table + (local & 1) * 2 * P_BN;
             int* fl = flag + (local & 1) * 4;
             uint8_t* stg = c.base + LP::STG + (warp - 2) * 2048;
-            const bool ok = a.loss ? phase_a_epilogue<P_BN>(a, tmem, c.tfull(0, P_STAGES), local & 1, tab, fl, cz,
-                                                             a.c0 + cz, ht * P_BN, tt * A_BM, tt == 0, stg, release)
-                                   : phase_a_epilogue_split<P_BN>(a, tmem, c.tfull(1, P_STAGES), c.tfull(0, P_STAGES),
-                                                                  local & 1, tab, fl, cz, a.c0 + cz, ht * P_BN,
-                                                                  tt * A_BM, tt == 0, stg, release);
+            const bool ok =
+                a.r_only ? phase_a_epilogue_r_only<P_BN>(a, tmem, c.tfull(0, P_STAGES), local & 1, tab, fl, a.c0 + cz,
+                                                         ht * P_BN, tt * A_BM, tt == 0, stg, release)
+                : a.loss ? phase_a_epilogue<P_BN>(a, tmem, c.tfull(0, P_STAGES), local & 1, tab, fl, cz, a.c0 + cz,
+                                                  ht * P_BN, tt * A_BM, tt == 0, stg, release)
+                         : phase_a_epilogue_split<P_BN>(a, tmem, c.tfull(1, P_STAGES), c.tfull(0, P_STAGES), local & 1,
+                                                        tab, fl, cz, a.c0 + cz, ht * P_BN, tt * A_BM, tt == 0, stg,
+                                                        release);
             if (!ok) break;
         }
     }
@@ -1102,6 +1166,13 @@ struct ReadArgs {
     const bf16 *K, *V;     // caller's targets of the group (chain z at z * y_cstride)
     bf16 *Kres, *Vres;     // [C][T][d_out/2] residual targets y - M(u)
     float* loss;           // [nc] or null
+    // MSE_HIDDEN, when phase A runs in its R-only form: also write At = c_t SiLU(x) and
+    // c_t SiLU'(x) / |z_t| (into dH), with c_t = -eta_t / T'
+    bf16 *At, *Sp;         // [C][T][d_hid] or null
+    int paper;
+    float lr;
+    const float *eta, *eta_in;
+    long long eta_cstride;
 };
 
 enum { READ_HIDDEN = 0, MSE_HIDDEN = 1, MSE_OUT = 2 };  // other MODEs: read out with heads of width MODE
@@ -1209,8 +1280,15 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if constexpr (MODE == MSE_HIDDEN) {
                 const int cs = a.b_chain0 + c, t = qw + lane;
                 const float zi = (t < a.Tp) ? (a.zinv ? a.zinv[(size_t)cs * a.win + a.tok0 + t] : 1.f) : 0.f;
+                float ct = 0.f;  // c_t = -eta_t / T' (R-only outputs)
+                if (a.At && t < a.Tp) {
+                    const float ev = a.paper ? a.eta[(size_t)cs * a.win + a.tok0 + t]
+                                             : (a.eta_in ? a.eta_in[c * a.eta_cstride + t] : a.lr);
+                    ct = -ev / (float)a.Tp;
+                }
+                const float czi = ct * zi;
                 uint8_t* stg = base + LRT<NST>::STG + (warp - 2) * 2048;
-                bf16* row0 = a.Aq + ((size_t)cs * a.T + qw) * a.d_hid + n0;
+                const size_t roff = ((size_t)cs * a.T + qw) * a.d_hid + n0;
 #pragma unroll 1
                 for (int cc = 0; cc < 4; ++cc) {
                     float hv[32];
@@ -1222,7 +1300,20 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                         const float x0 = hv[2 * j] * table[k0] * zi, x1 = hv[2 * j + 1] * table[k0 + 1] * zi;
                         pk[j] = pack_bf16(x0 * sigmoidf_(x0) * table[128 + k0], x1 * sigmoidf_(x1) * table[128 + k0 + 1]);
                     }
-                    store_rows_coalesced(stg, pk, row0 + cc * 32, a.d_hid, lane);
+                    store_rows_coalesced(stg, pk, a.Aq + roff + cc * 32, a.d_hid, lane);
+                    if (a.At) {  // the R-only form of phase A takes At and c SiLU'(x) / |z| from here
+                        uint32_t pa[16], ps[16];
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const int k0 = cc * 32 + 2 * j;
+                            const float x0 = hv[2 * j] * table[k0] * zi, x1 = hv[2 * j + 1] * table[k0 + 1] * zi;
+                            const float g0 = sigmoid_tanh(x0), g1 = sigmoid_tanh(x1);
+                            pa[j] = pack_bf16(ct * x0 * g0, ct * x1 * g1);
+                            ps[j] = pack_bf16(czi * (g0 * fmaf(x0, 1.f - g0, 1.f)), czi * (g1 * fmaf(x1, 1.f - g1, 1.f)));
+                        }
+                        store_rows_coalesced(stg, pa, a.At + roff + cc * 32, a.d_hid, lane);
+                        store_rows_coalesced(stg, ps, a.Sp + roff + cc * 32, a.d_hid, lane);
+                    }
                 }
             } else if constexpr (MODE == MSE_OUT) {
                 const int cs = a.b_chain0 + c, t = qw + lane, dh = a.d_out / 2;
@@ -1385,15 +1476,22 @@ cudaError_t ensure_attrs() {
     return g_attr_err;
 }
 
+// Whether phase A runs on CTA pairs (256-token x 256-hidden tiles) for this handle's shape.
+bool phase_a_pairs(const DevState& s) {
+    return (s.T / A_BM) % 2 == 0 && s.d_hid % P_BN == 0 && g_pair_clusters > 0;
+}
+
 }  // namespace
 
 cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,
                               cudaStream_t st) {
     cudaError_t e = ensure_attrs();
     if (e != cudaSuccess) return e;
-    const TcArgs a = make_args(s, w);
+    TcArgs a = make_args(s, w);
     const CUtensorMap& U = s.mode == 1 ? m.Ua : in.Xa;
-    if ((s.T / A_BM) % 2 == 0 && s.d_hid % P_BN == 0 && g_pair_clusters > 0) {
+    if (phase_a_pairs(s)) {
+        // squared-error segments: the pre-pass wrote At and c SiLU'(x) / |z|, only R is left
+        a.r_only = (s.loss == 1) ? 1 : 0;  // 1: MONE_LOSS_MSE
         // CTA pairs over 256-token x 256-hidden tiles
         const int npairs = w.nc * (s.T / (2 * A_BM)) * (s.d_hid / P_BN);
         const int clusters = npairs < g_pair_clusters ? npairs : g_pair_clusters;
@@ -1471,6 +1569,15 @@ cudaError_t launch_mse_tc(const DevState& s, const TcMaps& m, const TcInputMaps&
     a.Kres = s.Kres; a.Vres = s.Vres;
     a.loss = w.loss;
     a.Aq = s.Amse;
+    if (phase_a_pairs(s)) {  // phase A runs in its R-only form: write At and c SiLU'(x) / |z| here
+        a.At = reinterpret_cast<bf16*>(s.Att);
+        a.Sp = reinterpret_cast<bf16*>(s.dHt);
+        a.paper = paper ? 1 : 0;
+        a.lr = s.lr;
+        a.eta = s.eta;
+        a.eta_in = w.eta_in ? w.eta_in + w.row0 : nullptr;
+        a.eta_cstride = w.eta_cstride;
+    }
     // hidden: U rows of the segment (paper: the transformed window, absolute chain; plain: the
     // caller's X of the group), W1 of chain c0 + z
     a.a_row0 = paper ? (int)w.u_off : (int)w.row0;
