@@ -104,6 +104,11 @@ def kernel_work(wl, kind, chains=None):
     flops = T * flops_per_token(wl) * C // 2
     act = T * (di + do) * 2            # U and Y tiles, bf16, read once
     grads = T * dh * 2 * (2 if wl.memory == "mlp" else 3 * wl.heads)  # phase A outputs, bf16
+    if kind == "resident":
+        # fp32 chains resident on chip: `chains` counts chain-segments; U and Y (fp32) stream
+        # once, and W (and mu in paper mode) cross HBM once per launch (a window of segments)
+        state = wl.chains * params * (8 + (8 if wl.mode == 1 else 0))
+        return T * flops_per_token(wl) * C, C * T * (di + do) * 4 + state
     if kind == "phase_a":
         byts = C * (act + grads + params * 2)          # + bf16 weight operand read
     else:
@@ -511,7 +516,7 @@ def run_ours(args, wl):
     # ---- roofline of the dominant kernel
     hbm, tf_burst, tf_sus, peak_src = peaks()
     kern = {}
-    for name in ("phase_a", "phase_b"):
+    for name in ("phase_a", "phase_b", "resident"):
         tot, n = ktimes[name]
         if n == 0:
             continue
@@ -570,9 +575,13 @@ def run_ours(args, wl):
                             "frac": ach / pk, "unit": "TFLOP/s"}
     # the whole step against HBM: algorithmic bytes of every kernel of the step / step time
     S = (wl.N + wl.seg_T - 1) // wl.seg_T
-    step_bytes = S * (kernel_work(wl, "phase_a")[1] + kernel_work(wl, "phase_b")[1])
+    if "resident" in kern:  # one launch per input window, each streaming its segments
+        n_win = max(1, round(ktimes["resident"][1] / args.steps))
+        step_bytes = n_win * kernel_work(wl, "resident", wl.chains * S / n_win)[1]
+    else:
+        step_bytes = S * (kernel_work(wl, "phase_a")[1] + kernel_work(wl, "phase_b")[1])
     if wl.mode == 1:
-        step_bytes += wl.chains * wl.N * wl.d_in * 2 * 2      # input transform: read X, write z (bf16)
+        step_bytes += wl.chains * wl.N * wl.d_in * 2 * (2 if wl.dtype == "bf16" else 4)  # input transform: read X, write U
     step_roof = {"bytes_per_step": step_bytes, "achieved": step_bytes / (ms / 1000) / 1e9, "peak": hbm,
                  "unit": "GB/s", "frac": step_bytes / (ms / 1000) / 1e9 / hbm,
                  "frac_of_nominal_8000": step_bytes / (ms / 1000) / 1e9 / NOMINAL_HBM_GBS}

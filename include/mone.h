@@ -236,7 +236,9 @@ mone_status mone_attention(mone_mem* m, const void* Q, int n_q_heads, int Lq, co
  * last enabled.  Kinds: 0 input prepass, 1 phase A (forward + fused backward
  * epilogue), 2 phase B (gradient + fused update), 3 finalize (renorm apply /
  * operand refresh), 4 memory read, 5 squared-error pre-pass (M(u) and the residual
- * target, MONE_LOSS_MSE only), 6 consumer attention.  Errors: INVALID_ARG, CUDA.
+ * target, MONE_LOSS_MSE only), 6 consumer attention, 7 resident chains (the fp32 MLP
+ * path when d_in + d_out <= 512: every segment of an input window in one launch,
+ * forward, backward and update together).  Errors: INVALID_ARG, CUDA.
  */
 mone_status mone_mem_set_timing(mone_mem* m, int enable);
 mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches);

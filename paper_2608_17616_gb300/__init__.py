@@ -30,7 +30,7 @@ EXPORTS = ("mone_mem_init", "mone_ttl_segment", "mone_ttl_context", "mone_mem_ge
            "mone_status_string", "mone_abi_version", "mone_mem_set_timing", "mone_mem_kernel_time",
            "mone_last_error", "mone_mem_generate_kv_noalloc", "mone_attention", "mone_mem_kernel_busy")
 
-KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read", "mse", "attention")
+KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read", "mse", "attention", "resident")
 
 
 class MoneError(RuntimeError):

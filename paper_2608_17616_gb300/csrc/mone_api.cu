@@ -25,16 +25,16 @@ struct KernelTiming {
     };
     std::vector<cudaEvent_t> pool;
     std::vector<Pending> pending;
-    double ms[7] = {0, 0, 0, 0, 0, 0, 0};
-    long long n[7] = {0, 0, 0, 0, 0, 0, 0};
+    double ms[8] = {};
+    long long n[8] = {};
     // start and end of every launch, in ms after `ref` (recorded before the first timed launch
     // since timing was enabled), for the busy time of a kernel kind (mone_mem_kernel_busy)
     cudaEvent_t ref = nullptr;
     bool ref_set = false;
-    std::vector<std::pair<double, double>> iv[7];
+    std::vector<std::pair<double, double>> iv[8];
 
     void reset() {
-        for (int k = 0; k < 7; ++k) {
+        for (int k = 0; k < 8; ++k) {
             ms[k] = 0;
             n[k] = 0;
             iv[k].clear();
@@ -278,7 +278,8 @@ mone_status build_input_maps(const DevState& s, TcInputMaps* in, const void* X, 
     return ok ? MONE_OK : MONE_ERR_CUDA;
 }
 
-enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4, K_MSE = 5, K_ATTN = 6 };
+enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4, K_MSE = 5, K_ATTN = 6,
+       K_RESIDENT = 7, K_KINDS = 8 };
 
 // Launch through `fn` (which returns a cudaError_t), bracketed by timing events
 // when timing is on; `kernels` is the number of device kernels `fn` launches.
@@ -329,6 +330,22 @@ mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInput
         }
         return MONE_OK;
     };
+    if (resident_f32_fits(s)) {
+        // fp32 chains that fit on chip: one launch per input window covers all of its segments
+        const long long win = s.mode == MONE_PAPER ? s.win_rows : N;
+        for (long long row0 = 0; row0 < N; row0 += win) {
+            SegWork x = w;
+            x.row0 = row0;
+            x.u_off = 0;
+            const long long n = std::min(win, N - row0);
+            if (s.mode == MONE_PAPER) {
+                x.Tp = (int)n;
+                MONE_TRY(timed(m, K_PREPASS, st, 1, [&] { return launch_prepass(s, x, st); }));
+            }
+            MONE_TRY(timed(m, K_RESIDENT, st, 1, [&] { return launch_resident_f32(s, x, n, st); }));
+        }
+        return MONE_OK;
+    }
     const long long S = (N + s.T - 1) / s.T;
     long long win0 = -1;  // first token of the current paper-mode input window
     for (long long i = 0; i < S; ++i) {
@@ -795,7 +812,7 @@ mone_status mone_mem_set_timing(mone_mem* m, int enable) {
 }
 
 mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches) {
-    if (!is_live(m) || kind < 0 || kind > 6 || !ms || !launches) return MONE_ERR_INVALID_ARG;
+    if (!is_live(m) || kind < 0 || kind >= K_KINDS || !ms || !launches) return MONE_ERR_INVALID_ARG;
     *ms = 0;
     *launches = 0;
     if (!m->timing) return MONE_OK;
@@ -806,7 +823,7 @@ mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* l
 }
 
 mone_status mone_mem_kernel_busy(mone_mem* m, int kind, double* busy_ms) {
-    if (!is_live(m) || kind < 0 || kind > 6 || !busy_ms) return MONE_ERR_INVALID_ARG;
+    if (!is_live(m) || kind < 0 || kind >= K_KINDS || !busy_ms) return MONE_ERR_INVALID_ARG;
     *busy_ms = 0;
     if (!m->timing) return MONE_OK;
     MONE_CUDA(m->timing->drain());

@@ -83,6 +83,11 @@ cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, voi
 // ---- kernels in ttl_simt.cu (fp32 path, state upkeep, read path)
 cudaError_t launch_phase_a_f32(const DevState& s, const SegWork& w, cudaStream_t st);
 cudaError_t launch_phase_b_f32(const DevState& s, const SegWork& w, cudaStream_t st);
+// The whole call in one launch per input window, each CTA keeping RB hidden units of one chain
+// on chip across the segments (fp32 MLP with the Eq. 7 loss, d_in + d_out <= 512).  Leaves the
+// weights renormalised, so no finalize follows.  w: the call's chains, row0 / u_off of the window.
+bool resident_f32_fits(const DevState& s);
+cudaError_t launch_resident_f32(const DevState& s, const SegWork& w, long long n_tok, cudaStream_t st);
 cudaError_t launch_finalize(const DevState& s, int c0, int nc, int parity, int apply_scale, cudaStream_t st);
 cudaError_t launch_row_norms(const DevState& s, cudaStream_t st);
 cudaError_t launch_read(const DevState& s, int Q, int n_layers, void* K_out, void* V_out,

@@ -1,7 +1,8 @@
 // fp32 path of the TTL step, state upkeep kernels and the memory read.
 //
-// The fp32 path (the tiny fp32 workload: 256 -> 512 -> 256, T = 128) is
-// latency-bound, so it uses plain CUDA-core FFMA tiles (64 x 64 per CTA, 4 x 4 per
+// When d_in + d_out <= 512 the fp32 path runs every segment of a call in one launch
+// with the rows resident on chip (ttl_resident_f32_kernel, below).  Otherwise it
+// runs two kernels a segment.  Those are latency-bound, so they use plain CUDA-core FFMA tiles (64 x 64 per CTA, 4 x 4 per
 // thread, 64-deep K slabs so that each thread has 32 loads in flight per slab) in fp32
 // throughout.  It computes the same two phases as the bf16
 // tensor-core path:
@@ -282,6 +283,316 @@ F32SegArgs make_f32_args(const DevState& s, const SegWork& w) {
     return a;
 }
 
+// ------------------------------------------------------------------ resident chains (fp32)
+//
+// When a chain's rows fit on chip, a whole call runs in one launch with the fast
+// weights resident.  A CTA owns RB hidden units of one chain: their rows of W1 and
+// W2, kept side by side as [W1 | W2] (width D = d_in + d_out) in shared memory, and
+// their momentum and gradient in registers.  Hidden units do not interact within a
+// step: H[:, r] = U W1[r]^T and R[:, r] = Y W2[r]^T use only row r, dL/dO does not
+// depend on W (Eq. 10), the gradient rows dW1[r] = dH[:, r]^T U and dW2[r] =
+// At[:, r]^T Y use only column r of dH and At, and Eq. 8's renormalisation is per
+// row.  So a CTA takes its rows through every segment of the call without waiting
+// for any other CTA, and the weights cross HBM once per call instead of once per
+// segment.  Each segment streams its rows [U | K | V] once, RC tokens at a time,
+// through a double-buffered cp.async stage: forward (H, R), the backward epilogue
+// (dH, At), then the gradient accumulation from the same staged rows.  At the end
+// of the segment the update (momentum, W -= mu) and the row renormalisation are
+// applied in place.
+//
+// Forward: an output group is 2 tokens x 2 hidden units, its contraction split over
+// KS = 32 / RB lanes (float4 steps over interleaved columns), then summed by
+// shuffles.  Backward: thread i owns columns 2i, 2i + 1 of all RB rows.
+constexpr int RES_RC = 32;                                             // tokens per streamed chunk
+__host__ __device__ constexpr int res_ld(int D) { return (D + 31) / 32 * 32 + 16; }  // row pitch, floats
+
+struct ResArgs {
+    int d_in, d_out, d_hid, T, c0, win, paper, momentum, renorm, n_seg;
+    long long n_tok;             // tokens of this launch, from its first row
+    const float* U;              // first row of the launch, chain cz at U + cz * u_cstride
+    long long u_cstride;
+    const float *K, *V;          // first row of the launch
+    long long y_cstride;
+    const float* eta;            // paper mode: rates [C][win] at the launch's first row (state chain index)
+    const float* dbeta;          // paper mode: w_beta . x_t, same layout
+    const float* eta_in;         // plain mode: caller rates at the launch's first row, or null
+    long long eta_cstride;
+    float lr;
+    const float* b_beta;
+    float *W1, *W2, *mu1, *mu2;
+    const float *n1, *n2;
+    float* loss;                 // [nc] per-segment loss accumulator or null
+    int* status;
+};
+
+__device__ __forceinline__ void cp_async16(float* dst, const float* src, int src_bytes) {
+    const unsigned d = (unsigned)__cvta_generic_to_shared(dst);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N> __device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ float dot4(const float4 a, const float4 b, float acc) {
+    acc = fmaf(a.x, b.x, acc);
+    acc = fmaf(a.y, b.y, acc);
+    acc = fmaf(a.z, b.z, acc);
+    return fmaf(a.w, b.w, acc);
+}
+
+// Sum of v over the CTA (256 threads); every thread gets the total.  red: 8 floats.
+__device__ __forceinline__ float block_sum256(float v, float* red) {
+    v = warp_sum(v);
+    __syncthreads();
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += red[w];
+    return t;
+}
+
+template <int RB>
+__global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) {
+    constexpr int RC = RES_RC, KS = 32 / RB, RH = RB / 2;
+    static_assert(RB == 4 || RB == 8, "rows per CTA");
+    extern __shared__ float4 res_smem[];
+    const int D = a.d_in + a.d_out, LD = res_ld(D), dh = a.d_out / 2;
+    float* Ws = reinterpret_cast<float*>(res_smem);  // [RB][LD]
+    float* Xs = Ws + RB * LD;                        // [2][RC][LD]: rows [U | K | V] of a chunk
+    float* Gs = Xs + 2 * RC * LD;                    // [RC][2][RB]: c dH, c A of the chunk
+    float* red = Gs + RC * 2 * RB;                   // [8][2 RB]
+    float* scl = red + 8 * 2 * RB;                   // [2 RB] row scales
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int h0 = blockIdx.x * RB, cz = blockIdx.y, cs = a.c0 + cz;
+    const float* Uc = a.U + cz * a.u_cstride;
+    const float* Kc = a.K + cz * a.y_cstride;
+    const float* Vc = a.V + cz * a.y_cstride;
+
+    // stage RC token rows of segment seg, chunk ch into buffer b; rows past the segment read as 0
+    auto issue = [&](int seg, int ch, int b) {
+        const long long t_seg = (long long)seg * a.T;
+        const int Tp = (int)min((long long)a.T, a.n_tok - t_seg);
+        const int nvalid = min(RC, Tp - ch * RC);
+        const long long r0 = t_seg + ch * RC;
+        const int Q4 = D / 4;
+        float* dst0 = Xs + b * RC * LD;
+        for (int i = tid; i < RC * Q4; i += 256) {
+            const int t = i / Q4, c = 4 * (i - t * Q4);
+            const bool v = t < nvalid;
+            const long long r = r0 + (v ? t : 0);
+            const float* src = c < a.d_in        ? Uc + r * a.d_in + c
+                               : c < a.d_in + dh ? Kc + r * dh + (c - a.d_in)
+                                                 : Vc + r * dh + (c - a.d_in - dh);
+            cp_async16(dst0 + t * LD + c, src, v ? 16 : 0);
+        }
+    };
+
+    // resident rows, momentum (registers) and the thread's columns for the backward
+    for (int i = tid; i < RB * (D / 4); i += 256) {
+        const int r = i / (D / 4), c = 4 * (i - r * (D / 4));
+        const size_t row = (size_t)cs * a.d_hid + h0 + r;
+        const float* src = c < a.d_in ? a.W1 + row * a.d_in + c : a.W2 + row * a.d_out + (c - a.d_in);
+        *reinterpret_cast<float4*>(Ws + r * LD + c) = *reinterpret_cast<const float4*>(src);
+    }
+    const int cb = 2 * tid;                      // first owned column
+    const bool own = cb < D;
+    const int kind = cb < a.d_in ? 0 : 1;        // d_in is even: both columns are in one matrix
+    float mu[RB][2], acc[RB][2];
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+        mu[r][0] = mu[r][1] = 0.f;
+        acc[r][0] = acc[r][1] = 0.f;
+        if (own && a.momentum) {
+            const size_t row = (size_t)cs * a.d_hid + h0 + r;
+            const float2 m2 = kind == 0 ? *reinterpret_cast<const float2*>(a.mu1 + row * a.d_in + cb)
+                                        : *reinterpret_cast<const float2*>(a.mu2 + row * a.d_out + (cb - a.d_in));
+            mu[r][0] = m2.x;
+            mu[r][1] = m2.y;
+        }
+    }
+
+    // forward mapping: output group og = (token pair tp, row pair rp), contraction lane ks
+    const int ks = tid % KS, og = tid / KS, rp = og % RH, tp = og / RH;
+    const int er = ks & 1, et = (ks >> 1) & 1;   // the output this lane finishes (ks < 4)
+    bool finite = true;
+    int buf = 0;
+    issue(0, 0, 0);
+    cp_async_commit();
+    for (int seg = 0; seg < a.n_seg; ++seg) {
+        const long long t_seg = (long long)seg * a.T;
+        const int Tp = (int)min((long long)a.T, a.n_tok - t_seg);
+        const int nch = (Tp + RC - 1) / RC;
+        float lsum = 0.f;
+        for (int ch = 0; ch < nch; ++ch) {
+            if (ch + 1 < nch)
+                issue(seg, ch + 1, buf ^ 1);
+            else if (seg + 1 < a.n_seg)
+                issue(seg + 1, 0, buf ^ 1);
+            cp_async_commit();
+            cp_async_wait<1>();
+            __syncthreads();
+            const float* Xb = Xs + buf * RC * LD;
+            // H and R of tokens (tp, tp + 16) x rows (rp, rp + RH)
+            float h[2][2] = {}, q[2][2] = {};
+            {
+                const float* x0 = Xb + tp * LD;
+                const float* x1 = Xb + (tp + 16) * LD;
+                const float* w0 = Ws + rp * LD;
+                const float* w1 = Ws + (rp + RH) * LD;
+                for (int c = 4 * ks; c < a.d_in; c += 4 * KS) {
+                    const float4 u0 = *reinterpret_cast<const float4*>(x0 + c);
+                    const float4 u1 = *reinterpret_cast<const float4*>(x1 + c);
+                    const float4 b0 = *reinterpret_cast<const float4*>(w0 + c);
+                    const float4 b1 = *reinterpret_cast<const float4*>(w1 + c);
+                    h[0][0] = dot4(u0, b0, h[0][0]);
+                    h[0][1] = dot4(u0, b1, h[0][1]);
+                    h[1][0] = dot4(u1, b0, h[1][0]);
+                    h[1][1] = dot4(u1, b1, h[1][1]);
+                }
+                for (int c = a.d_in + 4 * ks; c < D; c += 4 * KS) {
+                    const float4 y0 = *reinterpret_cast<const float4*>(x0 + c);
+                    const float4 y1 = *reinterpret_cast<const float4*>(x1 + c);
+                    const float4 b0 = *reinterpret_cast<const float4*>(w0 + c);
+                    const float4 b1 = *reinterpret_cast<const float4*>(w1 + c);
+                    q[0][0] = dot4(y0, b0, q[0][0]);
+                    q[0][1] = dot4(y0, b1, q[0][1]);
+                    q[1][0] = dot4(y1, b0, q[1][0]);
+                    q[1][1] = dot4(y1, b1, q[1][1]);
+                }
+            }
+#pragma unroll
+            for (int o = 1; o < KS; o <<= 1)
+#pragma unroll
+                for (int i = 0; i < 2; ++i)
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) {
+                        h[i][j] += __shfl_xor_sync(0xffffffffu, h[i][j], o);
+                        q[i][j] += __shfl_xor_sync(0xffffffffu, q[i][j], o);
+                    }
+            if (ks < 4) {
+                // epilogue of one output: c_t = -eta_t / T' (Eq. 10), A = SiLU(H)
+                const int t = tp + 16 * et, r = rp + RH * er;
+                const float hv = et ? (er ? h[1][1] : h[1][0]) : (er ? h[0][1] : h[0][0]);
+                const float rv = et ? (er ? q[1][1] : q[1][0]) : (er ? q[0][1] : q[0][0]);
+                const int ts = ch * RC + t;  // token within the segment
+                float ct = 0.f;
+                if (ts < Tp) {
+                    const long long tl = t_seg + ts;
+                    const float e = a.paper    ? a.eta[(size_t)cs * a.win + tl]
+                                    : a.eta_in ? a.eta_in[cz * a.eta_cstride + tl]
+                                               : a.lr;
+                    ct = -e / (float)Tp;
+                }
+                const float sg = sigmoidf_(hv);
+                const float av = hv * sg;
+                const float ds = sg * (1.f + hv * (1.f - sg));
+                if (ts < Tp) lsum = fmaf(av, rv, lsum);
+                Gs[(t * 2 + 0) * RB + r] = ct * rv * ds;
+                Gs[(t * 2 + 1) * RB + r] = ct * av;
+            }
+            __syncthreads();
+            // gradient rows: acc[r][j] += sum_t G[t][kind][r] * X[t][cb + j]
+            if (own) {
+                const int nv = min(RC, Tp - ch * RC);
+                const float* gk = Gs + kind * RB;
+                for (int t = 0; t < nv; ++t) {
+                    const float2 x = *reinterpret_cast<const float2*>(Xb + t * LD + cb);
+                    float g[RB];
+#pragma unroll
+                    for (int r4 = 0; r4 < RB; r4 += 4) {
+                        const float4 g4 = *reinterpret_cast<const float4*>(gk + t * 2 * RB + r4);
+                        g[r4] = g4.x; g[r4 + 1] = g4.y; g[r4 + 2] = g4.z; g[r4 + 3] = g4.w;
+                    }
+#pragma unroll
+                    for (int r = 0; r < RB; ++r) {
+                        acc[r][0] = fmaf(g[r], x.x, acc[r][0]);
+                        acc[r][1] = fmaf(g[r], x.y, acc[r][1]);
+                    }
+                }
+            }
+            __syncthreads();
+            buf ^= 1;
+        }
+        // end of segment: Eq. 8 update, then the row renormalisation to the norms of W_0
+        float beta = 0.f;
+        if (a.momentum) {
+            float v = 0.f;
+            for (int t = tid; t < Tp; t += 256) v += a.dbeta[(size_t)cs * a.win + t_seg + t];
+            beta = sigmoidf_(block_sum256(v, red) / (float)Tp + a.b_beta[cs]);
+        }
+        if (a.loss) {
+            const float tot = block_sum256(lsum, red);
+            if (tid == 0) atomicAdd(&a.loss[cz], -tot / (float)Tp);
+        }
+        float wn[RB][2], ss[RB];
+#pragma unroll
+        for (int r = 0; r < RB; ++r) {
+            ss[r] = 0.f;
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+                const float mn = a.momentum ? fmaf(beta, mu[r][j], acc[r][j]) : acc[r][j];
+                mu[r][j] = mn;
+                acc[r][j] = 0.f;
+                wn[r][j] = own ? Ws[r * LD + cb + j] - mn : 0.f;
+                ss[r] = fmaf(wn[r][j], wn[r][j], ss[r]);
+            }
+        }
+        if (a.renorm) {
+            // row sums of squares per (matrix, row); a warp may hold columns of both matrices
+            __syncthreads();  // red may still be read by block_sum256 above
+#pragma unroll
+            for (int k = 0; k < 2; ++k)
+#pragma unroll
+                for (int r = 0; r < RB; ++r) {
+                    const float v = warp_sum(kind == k ? ss[r] : 0.f);
+                    if (lane == 0) red[warp * 2 * RB + k * RB + r] = v;
+                }
+            __syncthreads();
+            if (tid < 2 * RB) {
+                float tot = 0.f;
+                for (int w = 0; w < 8; ++w) tot += red[w * 2 * RB + tid];
+                const int k = tid / RB, r = tid % RB;
+                const float n0 = (k ? a.n2 : a.n1)[(size_t)cs * a.d_hid + h0 + r];
+                scl[tid] = renorm_scale(n0, tot);
+            }
+            __syncthreads();
+        }
+        if (own) {
+#pragma unroll
+            for (int r = 0; r < RB; ++r) {
+                const float sc = a.renorm ? scl[kind * RB + r] : 1.f;
+                const float w0 = wn[r][0] * sc, w1 = wn[r][1] * sc;
+                finite = finite && isfinite(w0) && isfinite(w1);
+                *reinterpret_cast<float2*>(Ws + r * LD + cb) = make_float2(w0, w1);
+            }
+        }
+        __syncthreads();
+    }
+    cp_async_wait<0>();
+    // write the rows and the momentum back
+    for (int i = tid; i < RB * (D / 4); i += 256) {
+        const int r = i / (D / 4), c = 4 * (i - r * (D / 4));
+        const size_t row = (size_t)cs * a.d_hid + h0 + r;
+        float* dst = c < a.d_in ? a.W1 + row * a.d_in + c : a.W2 + row * a.d_out + (c - a.d_in);
+        *reinterpret_cast<float4*>(dst) = *reinterpret_cast<const float4*>(Ws + r * LD + c);
+    }
+    if (own && a.momentum) {
+#pragma unroll
+        for (int r = 0; r < RB; ++r) {
+            const size_t row = (size_t)cs * a.d_hid + h0 + r;
+            float* dst = kind == 0 ? a.mu1 + row * a.d_in + cb : a.mu2 + row * a.d_out + (cb - a.d_in);
+            *reinterpret_cast<float2*>(dst) = make_float2(mu[r][0], mu[r][1]);
+        }
+    }
+    if (!finite) atomicOr(a.status, DEV_NONFINITE);
+}
+
+template <int RB> constexpr size_t res_smem_bytes(int D) {
+    return sizeof(float) * ((size_t)(RB + 2 * RES_RC) * res_ld(D) + RES_RC * 2 * RB + 8 * 2 * RB + 2 * RB);
+}
+
 // ------------------------------------------------------------------ state upkeep
 
 // Apply the pending renormalisation of the last segment (when asked) and refresh
@@ -411,6 +722,57 @@ cudaError_t launch_phase_b_f32(const DevState& s, const SegWork& w, cudaStream_t
     F32SegArgs a = make_f32_args(s, w);
     dim3 grid((s.d_in + s.d_out) / TN, s.d_hid / B_TM, w.nc);
     phase_b_f32_kernel<<<grid, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+bool resident_f32_fits(const DevState& s) {
+    return s.dtype == 0 && s.memory == 0 && s.loss == 0 && s.d_in + s.d_out <= 512 && s.d_in % 4 == 0 &&
+           s.d_out % 8 == 0 && s.d_hid % 8 == 0;
+}
+
+cudaError_t launch_resident_f32(const DevState& s, const SegWork& w, long long n_tok, cudaStream_t st) {
+    ResArgs a{};
+    a.d_in = s.d_in; a.d_out = s.d_out; a.d_hid = s.d_hid; a.T = s.T; a.c0 = w.c0; a.win = s.win_rows;
+    a.paper = s.mode == 1; a.momentum = s.momentum; a.renorm = s.renorm;
+    a.n_tok = n_tok;
+    a.n_seg = (int)((n_tok + s.T - 1) / s.T);
+    const int dh = s.d_out / 2;
+    if (a.paper) {
+        a.U = reinterpret_cast<const float*>(s.U) + ((size_t)w.c0 * s.win_rows + w.u_off) * s.d_in;
+        a.u_cstride = (long long)s.win_rows * s.d_in;
+        a.eta = s.eta + w.u_off;
+        a.dbeta = s.dbeta + w.u_off;
+    } else {
+        a.U = reinterpret_cast<const float*>(w.X) + w.row0 * s.d_in;
+        a.u_cstride = w.x_cstride;
+    }
+    a.K = reinterpret_cast<const float*>(w.K) + w.row0 * dh;
+    a.V = reinterpret_cast<const float*>(w.V) + w.row0 * dh;
+    a.y_cstride = w.y_cstride;
+    a.eta_in = w.eta_in ? w.eta_in + w.row0 : nullptr;
+    a.eta_cstride = w.eta_cstride;
+    a.lr = s.lr;
+    a.b_beta = s.b_beta;
+    a.W1 = s.W1; a.W2 = s.W2; a.mu1 = s.mu1; a.mu2 = s.mu2; a.n1 = s.n1; a.n2 = s.n2;
+    a.loss = w.loss;
+    a.status = s.status;
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    // four rows a CTA while that still fits the chains in one wave, else eight (less re-streaming)
+    const int D = s.d_in + s.d_out;
+    if ((long long)w.nc * (s.d_hid / 4) <= sms) {
+        const size_t bytes = res_smem_bytes<4>(D);
+        e = cudaFuncSetAttribute(ttl_resident_f32_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+        if (e != cudaSuccess) return e;
+        ttl_resident_f32_kernel<4><<<dim3(s.d_hid / 4, w.nc), 256, bytes, st>>>(a);
+    } else {
+        const size_t bytes = res_smem_bytes<8>(D);
+        e = cudaFuncSetAttribute(ttl_resident_f32_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+        if (e != cudaSuccess) return e;
+        ttl_resident_f32_kernel<8><<<dim3(s.d_hid / 8, w.nc), 256, bytes, st>>>(a);
+    }
     return cudaGetLastError();
 }
 

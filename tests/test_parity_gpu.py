@@ -104,6 +104,62 @@ def test_f32_paper_mode_ragged():
     run.close()
 
 
+def launches(run, kind):
+    return mone.mone_mem_kernel_time(run.h, mone.KERNEL_KINDS.index(kind))[1]
+
+
+def test_f32_tiled_path_paper_ragged():
+    # d_in + d_out > 512: the rows stay in HBM and the per-segment fp32 phase kernels run
+    wl = small(wk.PAPER, "f32", n_ctx=1, T=64, N=3 * 64 + 20, d_in=512, d_hid=128, d_out=256, lr=0.5)
+    run = GpuRun(wl)
+    mone.mone_mem_set_timing(run.h, 1)
+    run.ttl_context()
+    assert launches(run, "resident") == 0 and launches(run, "phase_a") == wl.S
+    W1, W2, mu1, mu2 = run.state()
+    for c in range(wl.chains):
+        st = check_chain(run, c, W1, W2, F32_TOL)
+        assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+    run.close()
+
+
+def test_f32_resident_segment_caller_rates_and_loss():
+    # a partial segment of one chain with caller rates and the loss output, on the resident kernel
+    wl = small(wk.PLAIN, "f32", n_ctx=1, n_layers=3, T=128, N=128)
+    run = GpuRun(wl)
+    mone.mone_mem_set_timing(run.h, 1)
+    eta = wk.token_lr(wl, 1, 100, "cuda")
+    loss = torch.zeros(1, device="cuda")
+    mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, :100], run.K[0, 1, :100], run.V[0, 1, :100], 100, eta, loss)
+    mone.mone_mem_sync(run.h)
+    assert launches(run, "resident") == 1 and launches(run, "phase_a") == 0
+    W1, W2, _, _ = run.state()
+    X = O.f64(run.X[0, 1, :100])
+    Y = np.concatenate([O.f64(run.K[0, 1, :100]), O.f64(run.V[0, 1, :100])], axis=1)
+    st = O.init_state(W1=O.f64(run.W1_0[1]), W2=O.f64(run.W2_0[1]))
+    st, L = O.ttl_segment(st, X, Y, O.Hyper(mode=wk.PLAIN, lr=wl.lr), None, eta=O.f64(eta))
+    assert rel_fro(W1[1], st.W["W1"]) <= F32_TOL and rel_fro(W2[1], st.W["W2"]) <= F32_TOL
+    assert abs(loss.item() - L) <= F32_TOL * max(1.0, abs(L))
+    for c in (0, 2):
+        assert torch.equal(W1[c], run.W1_0[c].cpu()) and torch.equal(W2[c], run.W2_0[c].cpu())
+    run.close()
+
+
+def test_f32_resident_two_input_windows():
+    # a paper-mode context longer than one input-transform window (64 segments): one resident
+    # launch per window, the state handed from the first to the second through HBM
+    wl = small(wk.PAPER, "f32", n_ctx=1, n_layers=2, T=64, N=64 * 64 + 64 + 40, d_in=64, d_hid=64, d_out=128,
+               lr=0.5)
+    run = GpuRun(wl)
+    mone.mone_mem_set_timing(run.h, 1)
+    run.ttl_context()
+    assert launches(run, "resident") == 2 and launches(run, "prepass") == 2
+    W1, W2, mu1, mu2 = run.state()
+    for c in range(wl.chains):
+        st = check_chain(run, c, W1, W2, F32_TOL)
+        assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+    run.close()
+
+
 # ----------------------------------------------------------------- bf16 tensor-core path (small shapes)
 
 @pytest.mark.parametrize("mode", [wk.PLAIN, wk.PAPER])
