@@ -329,6 +329,10 @@ __device__ __forceinline__ void cp_async16(float* dst, const float* src, int src
     const unsigned d = (unsigned)__cvta_generic_to_shared(dst);
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(src_bytes) : "memory");
 }
+__device__ __forceinline__ void cp_async4(float* dst, const float* src, int src_bytes) {
+    const unsigned d = (unsigned)__cvta_generic_to_shared(dst);
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(d), "l"(src), "r"(src_bytes) : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N> __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
@@ -363,29 +367,50 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
     float* Xs = Ws + RB * LD;                        // [2][RC][LD]: rows [U | K | V] of a chunk
     float* Gs = Xs + 2 * RC * LD;                    // [RC][2][RB]: c dH, c A of the chunk
     float* red = Gs + RC * 2 * RB;                   // [8][2 RB]
-    float* scl = red + 8 * 2 * RB;                   // [2 RB] row scales
+    float* scl = red + 8 * 2 * RB;                   // [2 RB] row scales, then beta
+    float* etaS = scl + 2 * RB + 4;                  // [2][RC] rates of the chunk's tokens
+    float* dbS = etaS + 2 * RC;                      // [2][RC] w_beta . x of the chunk's tokens
+    float* nS = dbS + 2 * RC;                        // [2 RB] renormalisation targets
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int h0 = blockIdx.x * RB, cz = blockIdx.y, cs = a.c0 + cz;
     const float* Uc = a.U + cz * a.u_cstride;
     const float* Kc = a.K + cz * a.y_cstride;
     const float* Vc = a.V + cz * a.y_cstride;
 
-    // stage RC token rows of segment seg, chunk ch into buffer b; rows past the segment read as 0
+    // stage RC token rows of segment seg, chunk ch into buffer b (a warp per row, lanes over
+    // columns), with the tokens' rates and w_beta . x terms; rows past the segment read as 0
     auto issue = [&](int seg, int ch, int b) {
         const long long t_seg = (long long)seg * a.T;
         const int Tp = (int)min((long long)a.T, a.n_tok - t_seg);
         const int nvalid = min(RC, Tp - ch * RC);
         const long long r0 = t_seg + ch * RC;
-        const int Q4 = D / 4;
-        float* dst0 = Xs + b * RC * LD;
-        for (int i = tid; i < RC * Q4; i += 256) {
-            const int t = i / Q4, c = 4 * (i - t * Q4);
+        for (int t = warp; t < RC; t += 8) {
             const bool v = t < nvalid;
             const long long r = r0 + (v ? t : 0);
-            const float* src = c < a.d_in        ? Uc + r * a.d_in + c
-                               : c < a.d_in + dh ? Kc + r * dh + (c - a.d_in)
-                                                 : Vc + r * dh + (c - a.d_in - dh);
-            cp_async16(dst0 + t * LD + c, src, v ? 16 : 0);
+            const float* ur = Uc + r * a.d_in;
+            const float* kr = Kc + r * dh;
+            const float* vr = Vc + r * dh;
+            float* dr = Xs + (b * RC + t) * LD;
+            for (int c = 4 * lane; c < D; c += 128) {
+                const float* src = c < a.d_in ? ur + c : c < a.d_in + dh ? kr + (c - a.d_in) : vr + (c - a.d_in - dh);
+                cp_async16(dr + c, src, v ? 16 : 0);
+            }
+        }
+        if (tid < 2 * RC) {
+            const int t = tid & (RC - 1);
+            const bool v = t < nvalid;
+            const long long r = r0 + (v ? t : 0);
+            if (tid < RC) {
+                float* d = etaS + b * RC + t;
+                if (a.paper)
+                    cp_async4(d, a.eta + (size_t)cs * a.win + r, v ? 4 : 0);
+                else if (a.eta_in)
+                    cp_async4(d, a.eta_in + cz * a.eta_cstride + r, v ? 4 : 0);
+                else
+                    *d = v ? a.lr : 0.f;
+            } else if (a.momentum) {
+                cp_async4(dbS + b * RC + t, a.dbeta + (size_t)cs * a.win + r, v ? 4 : 0);
+            }
         }
     };
 
@@ -396,6 +421,8 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
         const float* src = c < a.d_in ? a.W1 + row * a.d_in + c : a.W2 + row * a.d_out + (c - a.d_in);
         *reinterpret_cast<float4*>(Ws + r * LD + c) = *reinterpret_cast<const float4*>(src);
     }
+    if (tid < 2 * RB) nS[tid] = (tid < RB ? a.n1 : a.n2)[(size_t)cs * a.d_hid + h0 + tid % RB];
+    const float b_beta = a.momentum ? a.b_beta[cs] : 0.f;
     const int cb = 2 * tid;                      // first owned column
     const bool own = cb < D;
     const int kind = cb < a.d_in ? 0 : 1;        // d_in is even: both columns are in one matrix
@@ -424,7 +451,7 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
         const long long t_seg = (long long)seg * a.T;
         const int Tp = (int)min((long long)a.T, a.n_tok - t_seg);
         const int nch = (Tp + RC - 1) / RC;
-        float lsum = 0.f;
+        float lsum = 0.f, dbsum = 0.f;
         for (int ch = 0; ch < nch; ++ch) {
             if (ch + 1 < nch)
                 issue(seg, ch + 1, buf ^ 1);
@@ -441,6 +468,7 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
                 const float* x1 = Xb + (tp + 16) * LD;
                 const float* w0 = Ws + rp * LD;
                 const float* w1 = Ws + (rp + RH) * LD;
+#pragma unroll 2
                 for (int c = 4 * ks; c < a.d_in; c += 4 * KS) {
                     const float4 u0 = *reinterpret_cast<const float4*>(x0 + c);
                     const float4 u1 = *reinterpret_cast<const float4*>(x1 + c);
@@ -451,6 +479,7 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
                     h[1][0] = dot4(u1, b0, h[1][0]);
                     h[1][1] = dot4(u1, b1, h[1][1]);
                 }
+#pragma unroll 2
                 for (int c = a.d_in + 4 * ks; c < D; c += 4 * KS) {
                     const float4 y0 = *reinterpret_cast<const float4*>(x0 + c);
                     const float4 y1 = *reinterpret_cast<const float4*>(x1 + c);
@@ -471,20 +500,14 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
                         h[i][j] += __shfl_xor_sync(0xffffffffu, h[i][j], o);
                         q[i][j] += __shfl_xor_sync(0xffffffffu, q[i][j], o);
                     }
+            if (a.momentum && warp == 0) dbsum += warp_sum(lane < Tp - ch * RC ? dbS[buf * RC + lane] : 0.f);
             if (ks < 4) {
                 // epilogue of one output: c_t = -eta_t / T' (Eq. 10), A = SiLU(H)
                 const int t = tp + 16 * et, r = rp + RH * er;
                 const float hv = et ? (er ? h[1][1] : h[1][0]) : (er ? h[0][1] : h[0][0]);
                 const float rv = et ? (er ? q[1][1] : q[1][0]) : (er ? q[0][1] : q[0][0]);
                 const int ts = ch * RC + t;  // token within the segment
-                float ct = 0.f;
-                if (ts < Tp) {
-                    const long long tl = t_seg + ts;
-                    const float e = a.paper    ? a.eta[(size_t)cs * a.win + tl]
-                                    : a.eta_in ? a.eta_in[cz * a.eta_cstride + tl]
-                                               : a.lr;
-                    ct = -e / (float)Tp;
-                }
+                const float ct = ts < Tp ? -etaS[buf * RC + t] / (float)Tp : 0.f;
                 const float sg = sigmoidf_(hv);
                 const float av = hv * sg;
                 const float ds = sg * (1.f + hv * (1.f - sg));
@@ -497,6 +520,7 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
             if (own) {
                 const int nv = min(RC, Tp - ch * RC);
                 const float* gk = Gs + kind * RB;
+#pragma unroll 4
                 for (int t = 0; t < nv; ++t) {
                     const float2 x = *reinterpret_cast<const float2*>(Xb + t * LD + cb);
                     float g[RB];
@@ -517,10 +541,10 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
         }
         // end of segment: Eq. 8 update, then the row renormalisation to the norms of W_0
         float beta = 0.f;
-        if (a.momentum) {
-            float v = 0.f;
-            for (int t = tid; t < Tp; t += 256) v += a.dbeta[(size_t)cs * a.win + t_seg + t];
-            beta = sigmoidf_(block_sum256(v, red) / (float)Tp + a.b_beta[cs]);
+        if (a.momentum) {  // beta_s = sigmoid(mean_t w_beta . x_t + b_beta); warp 0 holds the sum
+            if (tid == 0) scl[2 * RB] = sigmoidf_(dbsum / (float)Tp + b_beta);
+            __syncthreads();
+            beta = scl[2 * RB];
         }
         if (a.loss) {
             const float tot = block_sum256(lsum, red);
@@ -553,9 +577,7 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
             if (tid < 2 * RB) {
                 float tot = 0.f;
                 for (int w = 0; w < 8; ++w) tot += red[w * 2 * RB + tid];
-                const int k = tid / RB, r = tid % RB;
-                const float n0 = (k ? a.n2 : a.n1)[(size_t)cs * a.d_hid + h0 + r];
-                scl[tid] = renorm_scale(n0, tot);
+                scl[tid] = renorm_scale(nS[tid], tot);
             }
             __syncthreads();
         }
@@ -590,7 +612,8 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
 }
 
 template <int RB> constexpr size_t res_smem_bytes(int D) {
-    return sizeof(float) * ((size_t)(RB + 2 * RES_RC) * res_ld(D) + RES_RC * 2 * RB + 8 * 2 * RB + 2 * RB);
+    return sizeof(float) *
+           ((size_t)(RB + 2 * RES_RC) * res_ld(D) + RES_RC * 2 * RB + 8 * 2 * RB + 2 * RB + 4 + 4 * RES_RC + 2 * RB);
 }
 
 // ------------------------------------------------------------------ state upkeep
