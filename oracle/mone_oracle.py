@@ -50,13 +50,19 @@ notes):
   R14 Consumer attention (Eq. 5): the memory tokens are a prefix every query
       token sees; the query tokens are causal among themselves; query head h
       reads key/value head h // (n_q / n_kv) (grouped heads).
+  R15 The other reading of "channel-wise" (App. A), renorm_axis="out": a channel is
+      an output channel of each matrix, so W1 (hidden units out) keeps its rows and
+      W2 (output features out) rescales each column to its norm in W_0.  MLP only.
+  R16 The other reading of "SiLU-gated" (App. A), gate_act="silu": the learned
+      per-head scalar gate enters the read through SiLU, o_h <- SiLU(g_h) o_h / rms.
 
 Pinned by tests (tests/test_oracle_pins.py): the gradient (finite
 differences), the loss (closed-form one-hot case), the update (closed form of
 one step of a linear memory, Hebbian for Eq. 7 and the delta rule for a
 squared-error loss), the momentum recurrence (geometric-sum closed form), the
-renormalisation invariant, lr = 0 leaving W bit-identical, the read's
-RMS = |gate| invariant, the read of a linear memory against brute force, and
+renormalisation invariant (rows, and for R15 W1 rows and W2 columns), lr = 0
+leaving W bit-identical, the read's RMS = |gate| invariant (R16: |SiLU(g)|, and
+a zero output at g = 0), the read of a linear memory against brute force, and
 the chain identities (context = loop of segments = split contexts), and the
 consumer attention against its special cases (one visible key returns its
 value, equal keys average the visible values, causality, grouped heads).
@@ -130,6 +136,8 @@ class Hyper:
     renorm: Optional[bool] = None       # default: on in PAPER mode
     n_heads: int = 1                    # swiglu heads
     rms_eps: float = RMS_EPS
+    renorm_axis: str = "rows"           # "rows" (R4) | "out": W1 rows, W2 columns (R15)
+    gate_act: str = "linear"            # read gate g_h (R6) | "silu": SiLU(g_h) (R16)
 
     @property
     def use_momentum(self) -> bool:
@@ -164,21 +172,28 @@ class State:
     W: dict            # name -> float64 array (rows = hidden units for mlp/swiglu)
     mu: dict
     n0: dict           # name -> row norms of W_0
+    c0: dict = dataclasses.field(default_factory=dict)  # name -> column norms of W_0 (R15)
 
     def copy(self) -> "State":
         return State({k: v.copy() for k, v in self.W.items()},
                      {k: v.copy() for k, v in self.mu.items()},
-                     {k: v.copy() for k, v in self.n0.items()})
+                     {k: v.copy() for k, v in self.n0.items()},
+                     {k: v.copy() for k, v in self.c0.items()})
 
 
 def row_norms(W):
     return np.sqrt(np.sum(W * W, axis=-1))
 
 
+def col_norms(W):
+    return np.sqrt(np.sum(W * W, axis=-2))
+
+
 def init_state(**W0) -> State:
     """W_0 given by the caller (learned in the paper, Sec. 3.3); mu_0 = 0."""
     W = {k: f64(v) for k, v in W0.items()}
-    return State(W, {k: np.zeros_like(v) for k, v in W.items()}, {k: row_norms(v) for k, v in W.items()})
+    return State(W, {k: np.zeros_like(v) for k, v in W.items()}, {k: row_norms(v) for k, v in W.items()},
+                 {k: col_norms(v) for k, v in W.items()})
 
 
 # --------------------------------------------------------------------------- input transform (prepass)
@@ -302,9 +317,13 @@ def ttl_segment(state: State, X, Y, hp: Hyper, meta: Optional[Meta] = None, eta=
     for k in new.W:
         new.mu[k] = beta * new.mu[k] + G[k]          # App. A momentum
         new.W[k] = new.W[k] - new.mu[k]              # Eq. 8
-        if hp.use_renorm:                            # App. A, R4
+        if hp.use_renorm:                            # App. A, R4 (R15)
             Wk = new.W[k]
-            if Wk.ndim == 2:
+            if hp.renorm_axis == "out" and k == "W2":
+                if hp.memory != "mlp":
+                    raise ValueError("renorm_axis='out' is defined for the MLP memory")
+                new.W[k] = Wk * (new.c0[k] / col_norms(Wk))[None, :]
+            elif Wk.ndim == 2:
                 new.W[k] = Wk * (new.n0[k] / row_norms(Wk))[:, None]
             else:
                 for h in range(Wk.shape[0]):
@@ -346,6 +365,8 @@ def generate_kv(state: State, Xq, hp: Hyper, meta: Optional[Meta], n_kv_heads: i
     n_heads = 2 * n_kv_heads
     out = np.empty((n_heads, Q, head_dim))
     gate = np.ones(n_heads) if meta is None else meta.gate
+    if hp.gate_act == "silu":                        # R16
+        gate = silu(gate)
     for h in range(n_heads):
         o = O[:, h * head_dim:(h + 1) * head_dim]
         rms = np.sqrt(np.mean(o * o, axis=1, keepdims=True) + eps)

@@ -279,6 +279,55 @@ def test_renorm_keeps_initial_row_norms():
     assert moved > 1e-3
 
 
+def _column_norms_by_loop(W):
+    return np.array([math.sqrt(sum(W[h, c] ** 2 for h in range(W.shape[0]))) for c in range(W.shape[1])])
+
+
+def test_output_channel_renorm_keeps_w1_rows_and_w2_columns():
+    # R15: W1 keeps its row norms, W2 its column norms; W2's rows are free to move
+    r = rng(21)
+    st = rand_mlp_state(r, 8, 16, 8)
+    n1, n2 = O.row_norms(st.W["W1"]), O.row_norms(st.W["W2"])
+    c2 = _column_norms_by_loop(st.W["W2"])
+    meta = rand_meta(r, 8, 4, lr=0.5)
+    X = r.standard_normal((20, 8))
+    Y = r.standard_normal((20, 8))
+    _, _, trail = O.ttl_context(st, X, Y, 4, O.Hyper(mode=O.PAPER, renorm_axis="out"), meta, return_all=True)
+    for s in trail:
+        np.testing.assert_allclose(O.row_norms(s.W["W1"]), n1, rtol=1e-13)
+        np.testing.assert_allclose(_column_norms_by_loop(s.W["W2"]), c2, rtol=1e-13)
+    assert np.abs(O.row_norms(trail[-1].W["W2"]) - n2).max() > 1e-3
+
+
+def test_output_channel_renorm_is_a_column_rescale_of_the_same_step():
+    # one segment from the same state: W1, mu agree exactly with the row reading; each reading
+    # rescales the same W2 - mu, by rows (ratios constant along a row) or by columns
+    r = rng(22)
+    st = rand_mlp_state(r, 8, 16, 8)
+    meta = rand_meta(r, 8, 4, lr=0.5)
+    X = r.standard_normal((4, 8))
+    Y = r.standard_normal((4, 8))
+    a, La = O.ttl_segment(st.copy(), X, Y, O.Hyper(mode=O.PAPER), meta)
+    b, Lb = O.ttl_segment(st.copy(), X, Y, O.Hyper(mode=O.PAPER, renorm_axis="out"), meta)
+    assert np.array_equal(a.W["W1"], b.W["W1"]) and np.array_equal(a.mu["W2"], b.mu["W2"]) and La == Lb
+    raw = st.W["W2"] - a.mu["W2"]
+    ra, rb = a.W["W2"] / raw, b.W["W2"] / raw
+    np.testing.assert_allclose(ra, np.repeat(ra[:, :1], 8, axis=1), rtol=1e-12)
+    np.testing.assert_allclose(rb, np.repeat(rb[:1, :], 16, axis=0), rtol=1e-12)
+    assert np.abs(ra - rb).max() > 1e-3
+
+
+def test_output_channel_renorm_zero_learning_rate_is_bit_identical():
+    r = rng(23)
+    st0 = rand_mlp_state(r, 8, 16, 8)
+    X = r.standard_normal((12, 8))
+    Y = r.standard_normal((12, 8))
+    st, _ = O.ttl_context(st0.copy(), X, Y, 4, O.Hyper(mode=O.PAPER, renorm_axis="out"), rand_meta(r, 8, 4),
+                          eta=np.zeros(12))
+    for k in st.W:
+        assert np.array_equal(st.W[k], st0.W[k])
+
+
 # ----------------------------------------------------------------- prepass transforms (App. A)
 
 def test_key_transform_unit_norm_and_plain_identity():
@@ -355,6 +404,24 @@ def test_read_head_rms_equals_gate():
     for h in range(4):
         rms = np.sqrt(np.mean(heads[h] ** 2, axis=1))
         np.testing.assert_allclose(rms, abs(meta.gate[h]), rtol=1e-13)
+
+
+def test_read_silu_gate_rms_sign_and_zero_gate():
+    # R16: each head's RMS is |SiLU(g_h)| (by hand: g / (1 + e^-g)), a zero gate silences the
+    # head, and the output is the linear-gate output times SiLU(g) / g
+    r = rng(24)
+    st = rand_mlp_state(r, 8, 16, 8)
+    meta = rand_meta(r, 8, 4)
+    meta.gate = np.array([0.0, 1.0, -2.0, 3.0])
+    Xq = r.standard_normal((5, 8))
+    K, V = O.generate_kv(st, Xq, O.Hyper(mode=O.PAPER, gate_act="silu"), meta, n_kv_heads=2, head_dim=2, eps=0.0)
+    Kl, Vl = O.generate_kv(st, Xq, O.Hyper(mode=O.PAPER), meta, n_kv_heads=2, head_dim=2, eps=0.0)
+    heads, lin = np.concatenate([K, V]), np.concatenate([Kl, Vl])
+    sg = [0.0, 1 / (1 + math.exp(-1.0)), -2 / (1 + math.exp(2.0)), 3 / (1 + math.exp(-3.0))]
+    assert not np.any(heads[0])
+    for h in range(1, 4):
+        np.testing.assert_allclose(np.sqrt(np.mean(heads[h] ** 2, axis=1)), abs(sg[h]), rtol=1e-13)
+        np.testing.assert_allclose(heads[h], lin[h] * (sg[h] / meta.gate[h]), rtol=1e-13)
 
 
 def test_read_of_linear_memory_brute_force():
