@@ -54,6 +54,9 @@ def parse():
     p.add_argument("--n-tokens", type=int, default=0, help="override the context length (small profiling cases)")
     p.add_argument("--loss", default="neg_inner", choices=["neg_inner", "mse"],
                    help="per-token loss: Eq. 7 (the measured workload) or the squared-error variant")
+    p.add_argument("--renorm-axis", default="rows", choices=["rows", "out"],
+                   help="paper-mode renormalisation channels: rows of W1 and W2, or W1 rows and W2 columns")
+    p.add_argument("--gate", default="linear", choices=["linear", "silu"], help="read gate: g_h or SiLU(g_h)")
     return p.parse_args()
 
 
@@ -230,7 +233,8 @@ def oracle_sample(wl, seconds, chain=0):
     W1all, W2all = wk.initial_weights(wl, "cpu")
     W1, W2 = W1all[chain], W2all[chain]
     meta = O.Meta.from_torch(wk.meta_params(wl, "cpu"), chain) if wl.mode == wk.PAPER else None
-    hp = O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss, memory=wl.memory, n_heads=wl.heads)
+    hp = O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss, memory=wl.memory, n_heads=wl.heads,
+                 renorm_axis=wl.renorm_axis, gate_act=wl.gate_act)
 
     def init():
         if wl.memory == "swiglu":
@@ -338,6 +342,7 @@ def config_of(wl):
     return {"workload": wl.name, "n_ctx": wl.n_ctx, "n_layers": wl.n_layers, "chains": wl.chains,
             "N": wl.N, "seg_T": wl.seg_T, "d_in": wl.d_in, "d_hid": wl.d_hid, "d_out": wl.d_out, "Q": wl.Q,
             "mode": "paper" if wl.mode == 1 else "plain", "loss": wl.loss, "memory": wl.memory, "heads": wl.heads,
+            "renorm_axis": wl.renorm_axis, "gate": wl.gate_act,
             "masters": "fp32", "operands": wl.dtype,
             "l2": "inputs larger than L2 (no flush needed)"}
 
@@ -369,7 +374,9 @@ def run_ours(args, wl):
                            mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr,
                            loss=mone.MONE_LOSS_MSE if wl.loss == "mse" else mone.MONE_LOSS_DOT,
                            memory=mone.MONE_MEM_SWIGLU if wl.memory == "swiglu" else mone.MONE_MEM_MLP,
-                           mem_heads=wl.heads)
+                           mem_heads=wl.heads,
+                           renorm_axis=mone.MONE_RENORM_OUT if wl.renorm_axis == "out" else mone.MONE_RENORM_ROWS,
+                           gate_act=mone.MONE_GATE_SILU if wl.gate_act == "silu" else mone.MONE_GATE_LINEAR)
     h = mone.mone_mem_init(cfg, W1_0, W2_0, meta)
     stream = torch.cuda.current_stream()
 
@@ -619,6 +626,8 @@ def main():
         wl = wl.replace(N=args.n_tokens)
     if args.loss != "neg_inner":
         wl = wl.replace(loss=args.loss)
+    if args.renorm_axis != "rows" or args.gate != "linear":
+        wl = wl.replace(renorm_axis=args.renorm_axis, gate_act=args.gate)
     if args.impl == "reference":
         run_reference(args, wl)
     else:

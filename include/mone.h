@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define MONE_ABI_VERSION 4
+#define MONE_ABI_VERSION 5
 
 typedef struct mone_mem mone_mem; /* opaque; created by mone_mem_init */
 
@@ -57,6 +57,8 @@ enum { MONE_FP32 = 0, MONE_BF16 = 1 };  /* dtype of X, K, V, Xq and generated K/
 enum { MONE_PLAIN = 0, MONE_PAPER = 1 };
 enum { MONE_LOSS_DOT = 0, MONE_LOSS_MSE = 1 };  /* per-token loss of a segment step */
 enum { MONE_MEM_MLP = 0, MONE_MEM_SWIGLU = 1 };  /* form of the memory network M */
+enum { MONE_RENORM_ROWS = 0, MONE_RENORM_OUT = 1 };  /* channels of the App. A renormalisation */
+enum { MONE_GATE_LINEAR = 0, MONE_GATE_SILU = 1 };   /* how the read's per-head gate scales a head */
 
 /*
  * Configuration, fixed for the life of a handle.
@@ -83,6 +85,14 @@ enum { MONE_MEM_MLP = 0, MONE_MEM_SWIGLU = 1 };  /* form of the memory network M
  *     ([mem_heads][2 d_hid][dh]) and W2 = Wout ([mem_heads][d_hid][dh]).  BF16 only, loss DOT only;
  *     dh and d_hid multiples of 32 and <= 256, (d_out / 2) a multiple of dh, seg_T a multiple of 128.
  *
+ * renorm_axis (paper mode; App. A's "channel-wise" renormalisation): MONE_RENORM_ROWS rescales
+ *     every row (hidden unit) of W1 and of W2 to its norm in W_0; MONE_RENORM_OUT takes the
+ *     channels to be each matrix's output channels: rows of W1 and columns of W2 (every column
+ *     of W2 rescaled to its norm in W_0, by a column pass after each segment's update).  MLP
+ *     memory only (SwiGLU: MONE_ERR_UNSUPPORTED).  Ignored in MONE_PLAIN mode.
+ * gate_act (the read, App. A's "SiLU-gated" output): MONE_GATE_LINEAR scales head h by its
+ *     learned scalar gate g_h; MONE_GATE_SILU by SiLU(g_h).
+ *
  * Supported shapes: FP32: d_in, d_hid, d_out multiples of 64, seg_T multiple of 64.
  *   BF16 (MLP): d_in, d_out/2, seg_T multiples of 128; d_hid a multiple of 256.  Both: head_dim in {64,128},
  *   d_out == 2*n_kv_heads*head_dim, seg_T <= 4096.
@@ -99,6 +109,8 @@ typedef struct {
     int loss;      /* MONE_LOSS_DOT (Eq. 7) | MONE_LOSS_MSE */
     int memory;    /* MONE_MEM_MLP | MONE_MEM_SWIGLU */
     int mem_heads; /* SwiGLU heads (ignored for the MLP; 0 reads as 1) */
+    int renorm_axis; /* MONE_RENORM_ROWS | MONE_RENORM_OUT */
+    int gate_act;    /* MONE_GATE_LINEAR | MONE_GATE_SILU */
 } mone_config;
 
 /*

@@ -20,6 +20,8 @@ MONE_FP32, MONE_BF16 = 0, 1
 MONE_PLAIN, MONE_PAPER = 0, 1
 MONE_LOSS_DOT, MONE_LOSS_MSE = 0, 1
 MONE_MEM_MLP, MONE_MEM_SWIGLU = 0, 1
+MONE_RENORM_ROWS, MONE_RENORM_OUT = 0, 1
+MONE_GATE_LINEAR, MONE_GATE_SILU = 0, 1
 
 STATUS = {0: "MONE_OK", 1: "MONE_ERR_INVALID_ARG", 2: "MONE_ERR_UNSUPPORTED_SHAPE", 3: "MONE_ERR_OOM",
           4: "MONE_ERR_CUDA", 5: "MONE_ERR_TIMEOUT", 6: "MONE_ERR_NONFINITE", 7: "MONE_ERR_UNSUPPORTED"}
@@ -44,7 +46,8 @@ class mone_config(ctypes.Structure):
                 ("d_hid", ctypes.c_int), ("d_out", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("seg_T", ctypes.c_int), ("dtype", ctypes.c_int),
                 ("mode", ctypes.c_int), ("lr", ctypes.c_float), ("rms_eps", ctypes.c_float), ("loss", ctypes.c_int),
-                ("memory", ctypes.c_int), ("mem_heads", ctypes.c_int)]
+                ("memory", ctypes.c_int), ("mem_heads", ctypes.c_int), ("renorm_axis", ctypes.c_int),
+                ("gate_act", ctypes.c_int)]
 
 
 class mone_meta(ctypes.Structure):
@@ -117,9 +120,9 @@ def _check(fn: str, rc: int):
 
 
 def make_config(n_ctx, n_layers, d_in, d_hid, d_out, n_kv_heads, head_dim, seg_T, dtype, mode, lr,
-                rms_eps=1e-6, loss=0, memory=0, mem_heads=1) -> mone_config:
+                rms_eps=1e-6, loss=0, memory=0, mem_heads=1, renorm_axis=0, gate_act=0) -> mone_config:
     return mone_config(n_ctx, n_layers, d_in, d_hid, d_out, n_kv_heads, head_dim, seg_T, dtype, mode, lr, rms_eps,
-                       loss, memory, mem_heads)
+                       loss, memory, mem_heads, renorm_axis, gate_act)
 
 
 def make_meta(meta: Optional[dict]) -> Optional[mone_meta]:

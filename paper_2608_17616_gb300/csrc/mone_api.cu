@@ -112,6 +112,9 @@ mone_status validate_config(const mone_config* c) {
     if (c->loss != MONE_LOSS_DOT && c->loss != MONE_LOSS_MSE) return MONE_ERR_INVALID_ARG;
     if (c->loss == MONE_LOSS_MSE && c->dtype != MONE_BF16) return MONE_ERR_UNSUPPORTED;
     if (c->memory != MONE_MEM_MLP && c->memory != MONE_MEM_SWIGLU) return MONE_ERR_INVALID_ARG;
+    if (c->renorm_axis != MONE_RENORM_ROWS && c->renorm_axis != MONE_RENORM_OUT) return MONE_ERR_INVALID_ARG;
+    if (c->gate_act != MONE_GATE_LINEAR && c->gate_act != MONE_GATE_SILU) return MONE_ERR_INVALID_ARG;
+    if (c->renorm_axis == MONE_RENORM_OUT && c->memory != MONE_MEM_MLP) return MONE_ERR_UNSUPPORTED;
     if (!std::isfinite(c->lr) || !(c->rms_eps >= 0.0f) || !std::isfinite(c->rms_eps)) return MONE_ERR_INVALID_ARG;
     if (c->memory == MONE_MEM_SWIGLU) {
         if (c->dtype != MONE_BF16 || c->loss != MONE_LOSS_DOT) return MONE_ERR_UNSUPPORTED;
@@ -164,7 +167,7 @@ mone_status dalloc(T** p, size_t n) {
 void free_state(DevState& s) {
     void* ptrs[] = {s.W1, s.W2, s.mu1, s.mu2, s.W1b, s.W2b, s.n1, s.n2, s.sumsq, s.status, s.alpha, s.gamma,
                     s.w_eta, s.b_eta, s.w_beta, s.b_beta, s.gate, s.U, s.eta, s.dbeta, s.zinv, s.dHt, s.Att, s.Uq, s.Aq,
-                    s.Oq, s.Amse, s.Kres, s.Vres};
+                    s.Oq, s.Amse, s.Kres, s.Vres, s.nc2, s.colpart};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     std::memset(&s, 0, sizeof(s));
@@ -396,6 +399,8 @@ mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInput
                 MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_phase_a_f32(s, x, sg); }));
                 MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_phase_b_f32(s, x, sg); }));
             }
+            if (s.col_renorm)  // output channels: the columns of W2 back to their norms in W_0
+                MONE_TRY(timed(m, K_FINALIZE, sg, 2, [&] { return launch_col_renorm(s, x.c0, x.nc, sg); }));
         }
     }
     MONE_TRY(join());
@@ -505,6 +510,7 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
     s.loss = cfg->loss;
     s.memory = cfg->memory;
     s.heads = cfg->memory == MONE_MEM_SWIGLU ? cfg->mem_heads : 1;
+    s.col_renorm = (s.renorm && cfg->renorm_axis == MONE_RENORM_OUT) ? 1 : 0;
     if (s.mode == MONE_PAPER) {
         // the input transform covers a window of whole segments whose scratch stays within ~2 GiB
         const size_t row_bytes = (size_t)s.C * s.d_in * elsize(s.dtype);
@@ -547,7 +553,12 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
         step(dalloc(&s.dbeta, C * s.win_rows));
         step(dalloc(&s.zinv, C * s.win_rows));
     }
-    if (meta && meta->gate) step(dalloc(&s.gate, C * 2 * s.n_kv));
+    const bool silu_gate = cfg->gate_act == MONE_GATE_SILU;
+    if ((meta && meta->gate) || silu_gate) step(dalloc(&s.gate, C * 2 * s.n_kv));
+    if (s.col_renorm) {
+        step(dalloc(&s.nc2, C * s.d_out));
+        step(dalloc(&s.colpart, (size_t)kColRowSlices * C * s.d_out));
+    }
     const size_t elt = s.dtype == MONE_BF16 ? 2 : 4;
     // phase A outputs: c dH and c A ([C][T][d_hid]); SwiGLU: c [dP | dG] ([C*H][T][2 d_hid]) and c Z
     step(dalloc(reinterpret_cast<uint8_t**>(&s.dHt), r1 * s.T * elt));
@@ -565,7 +576,10 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
         cp(s.b_eta, meta->b_eta, C * 4);
         cp(s.b_beta, meta->b_beta, C * 4);
     }
-    if (s.gate) cp(s.gate, meta->gate, C * 2 * s.n_kv * 4);
+    const bool caller_gate = meta && meta->gate;
+    if (caller_gate) cp(s.gate, meta->gate, C * 2 * s.n_kv * 4);
+    if (silu_gate && rc == MONE_OK)  // the read scales head h by SiLU(g_h) (g_h = 1 when not given)
+        step(cuda_status(launch_gate_silu(s.gate, C * 2 * s.n_kv, caller_gate ? 0 : 1, st)));
     if (rc == MONE_OK && s.momentum) {
         step(cuda_status(cudaMemsetAsync(s.mu1, 0, n1 * 4, st)));
         step(cuda_status(cudaMemsetAsync(s.mu2, 0, n2 * 4, st)));
@@ -576,6 +590,7 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
         if (rc == MONE_OK) step(cuda_status(launch_swiglu_rows(s, 0, 0, 0, s.C, st)));  // targets + bf16 copies
     } else {
         if (rc == MONE_OK) step(cuda_status(launch_row_norms(s, st)));
+        if (rc == MONE_OK && s.col_renorm) step(cuda_status(launch_col_targets(s, st)));
         if (rc == MONE_OK && s.dtype == MONE_BF16) step(cuda_status(launch_finalize(s, 0, s.C, 0, 0, st)));
     }
     if (rc == MONE_OK) step(build_state_maps(m));

@@ -47,7 +47,7 @@ template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __flo
 
 // Renormalisation scale of one row: target norm / current norm (1 when the row is 0).
 __device__ __forceinline__ float renorm_scale(float n0, float ss) {
-    return ss > 0.0f ? n0 / sqrtf(ss) : 1.0f;
+    return (n0 >= 0.0f && ss > 0.0f) ? n0 / sqrtf(ss) : 1.0f;  // n0 < 0: row not renormalised
 }
 
 __device__ __forceinline__ uint64_t globaltimer_ns() {

@@ -21,7 +21,10 @@ struct DevState {
     float lr, rms_eps;
     float *W1, *W2, *mu1, *mu2;   // fp32 masters [C][d_hid][d_in|d_out]; mu only with momentum
     bf16 *W1b, *W2b;              // bf16 operand copies (bf16 path)
-    float *n1, *n2;               // renormalisation targets [C][d_hid]
+    float *n1, *n2;               // renormalisation targets [C][d_hid]; -1: row not renormalised
+    int col_renorm;               // W2 columns renormalised instead of its rows (output channels)
+    float* nc2;                   // [C][d_out] column norms of W2_0 (col_renorm)
+    float* colpart;               // [kColRowSlices][C][d_out] partial column sums of squares
     float* sumsq;                 // [2 parity][2 matrix][C][d_hid] row sums of squares
     int* status;                  // device status word
     // meta-parameters (owned copies)
@@ -42,6 +45,9 @@ struct DevState {
     int q_cap;
     float *Uq, *Aq, *Oq;          // [C][q_cap][d_in|d_hid|d_out]
 };
+
+// Row slices of the column sums of squares of W2 (output-channel renormalisation).
+constexpr int kColRowSlices = 8;
 
 // Elements of the state matrices and rows per chain.  MLP: W1 [d_hid][d_in], W2 [d_hid][d_out].
 // SwiGLU: W1 [heads][2 d_hid][dh] (Win; Wg), W2 [heads][d_hid][dh] (Wout), dh = d_in / heads.
@@ -90,6 +96,13 @@ bool resident_f32_fits(const DevState& s);
 cudaError_t launch_resident_f32(const DevState& s, const SegWork& w, long long n_tok, cudaStream_t st);
 cudaError_t launch_finalize(const DevState& s, int c0, int nc, int parity, int apply_scale, cudaStream_t st);
 cudaError_t launch_row_norms(const DevState& s, cudaStream_t st);
+// Output-channel renormalisation: every column of W2 of chains [c0, c0 + nc) rescaled to its norm
+// in W_0 (fp32 masters and, on the bf16 path, the operand copy).  Two kernels.
+cudaError_t launch_col_renorm(const DevState& s, int c0, int nc, cudaStream_t st);
+// At init: the column norms of W2_0 into s.nc2, and n2 = -1 (no row renormalisation of W2).
+cudaError_t launch_col_targets(const DevState& s, cudaStream_t st);
+// At init: gate[i] = SiLU(gate[i]) (from_one: SiLU(1)), n entries.
+cudaError_t launch_gate_silu(float* gate, size_t n, int from_one, cudaStream_t st);
 cudaError_t launch_read(const DevState& s, int Q, int n_layers, void* K_out, void* V_out,
                         const long long* strides, cudaStream_t st);
 cudaError_t launch_zero_f32(float* p, size_t n, cudaStream_t st);

@@ -672,6 +672,91 @@ __global__ void __launch_bounds__(256) row_norms_kernel(DevState s) {
     }
 }
 
+// ------------------------------------------------------------------ output-channel renormalisation
+//
+// The other reading of App. A's channel-wise renormalisation: a channel is an output
+// channel of each matrix, so W1 keeps its rows (hidden units, renormalised inside the
+// phase kernels) and every column of W2 (an output feature) is rescaled to its norm in
+// W_0 after each update.  A column spans all hidden units, which the phase kernels tile
+// apart, so this is a pass of its own over W2: partial column sums of squares over
+// kColRowSlices row slices, then the rescale.  Warps cover 32 consecutive columns.
+
+// 64 columns a CTA as 16 float4 column quads x 16 row groups: a warp reads 256 contiguous bytes
+// of each of two rows.
+__global__ void __launch_bounds__(256) col_partial_kernel(DevState s, int c0) {
+    __shared__ float4 red[16][16];
+    const int cq = threadIdx.x & 15, rg = threadIdx.x >> 4;
+    const int col = blockIdx.x * 64 + 4 * cq, rs = blockIdx.y, cs = c0 + blockIdx.z;
+    const int per = (s.d_hid + kColRowSlices - 1) / kColRowSlices;
+    const int r1 = min(s.d_hid, (rs + 1) * per);
+    const float* w = s.W2 + (size_t)cs * s.d_hid * s.d_out + col;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int r = rs * per + rg; r < r1; r += 16) {
+        const float4 x = *reinterpret_cast<const float4*>(w + (size_t)r * s.d_out);
+        v.x = fmaf(x.x, x.x, v.x);
+        v.y = fmaf(x.y, x.y, v.y);
+        v.z = fmaf(x.z, x.z, v.z);
+        v.w = fmaf(x.w, x.w, v.w);
+    }
+    red[rg][cq] = v;
+    __syncthreads();
+    if (rg == 0) {
+        float4 t = red[0][cq];
+        for (int g = 1; g < 16; ++g) {
+            t.x += red[g][cq].x; t.y += red[g][cq].y; t.z += red[g][cq].z; t.w += red[g][cq].w;
+        }
+        *reinterpret_cast<float4*>(s.colpart + ((size_t)rs * s.C + cs) * s.d_out + col) = t;
+    }
+}
+
+__device__ __forceinline__ float col_sumsq(const DevState& s, int cs, int col) {
+    float ss = 0.f;
+    for (int rs = 0; rs < kColRowSlices; ++rs) ss += s.colpart[((size_t)rs * s.C + cs) * s.d_out + col];
+    return ss;
+}
+
+// 64 rows x 64 columns a CTA (float4 column quads): W2[:, col] *= nc2[col] / |W2[:, col]|, and
+// the bf16 copy.
+__global__ void __launch_bounds__(256) col_scale_kernel(DevState s, int c0) {
+    __shared__ float sc[64];
+    const int cq = threadIdx.x & 15, rg = threadIdx.x >> 4;
+    const int cs = c0 + blockIdx.z;
+    if (threadIdx.x < 64) {
+        const int col = blockIdx.x * 64 + threadIdx.x;
+        sc[threadIdx.x] = renorm_scale(s.nc2[(size_t)cs * s.d_out + col], col_sumsq(s, cs, col));
+    }
+    __syncthreads();
+    const float4 f = make_float4(sc[4 * cq], sc[4 * cq + 1], sc[4 * cq + 2], sc[4 * cq + 3]);
+    const size_t base = (size_t)cs * s.d_hid * s.d_out + blockIdx.x * 64 + 4 * cq;
+    const int r1 = min(s.d_hid, (int)blockIdx.y * 64 + 64);
+    for (int r = blockIdx.y * 64 + rg; r < r1; r += 16) {
+        const size_t i = base + (size_t)r * s.d_out;
+        float4 x = *reinterpret_cast<const float4*>(s.W2 + i);
+        x.x *= f.x; x.y *= f.y; x.z *= f.z; x.w *= f.w;
+        *reinterpret_cast<float4*>(s.W2 + i) = x;
+        if (s.dtype == 1) {
+            uint2 p;
+            p.x = pack_bf16(x.x, x.y);
+            p.y = pack_bf16(x.z, x.w);
+            *reinterpret_cast<uint2*>(s.W2b + i) = p;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(256) col_targets_kernel(DevState s) {
+    const int col = blockIdx.x * 256 + threadIdx.x, cs = blockIdx.y;
+    if (col < s.d_out) s.nc2[(size_t)cs * s.d_out + col] = sqrtf(col_sumsq(s, cs, col));
+    for (int h = col; h < s.d_hid; h += gridDim.x * 256) s.n2[(size_t)cs * s.d_hid + h] = -1.f;
+}
+
+__global__ void __launch_bounds__(256) gate_silu_kernel(float* g, size_t n, int from_one) {
+    const size_t i = (size_t)blockIdx.x * 256 + threadIdx.x;
+    if (i < n) {
+        const float v = from_one ? 1.f : g[i];
+        g[i] = v * sigmoidf_(v);
+    }
+}
+
 // ------------------------------------------------------------------ memory read (Eq. 4)
 
 __global__ void __launch_bounds__(256) read_hidden_kernel(DevState s, int Q) {
@@ -749,7 +834,7 @@ cudaError_t launch_phase_b_f32(const DevState& s, const SegWork& w, cudaStream_t
 }
 
 bool resident_f32_fits(const DevState& s) {
-    return s.dtype == 0 && s.memory == 0 && s.loss == 0 && s.d_in + s.d_out <= 512 && s.d_in % 4 == 0 &&
+    return s.dtype == 0 && s.memory == 0 && s.loss == 0 && !s.col_renorm && s.d_in + s.d_out <= 512 && s.d_in % 4 == 0 &&
            s.d_out % 8 == 0 && s.d_hid % 8 == 0;
 }
 
@@ -801,6 +886,27 @@ cudaError_t launch_resident_f32(const DevState& s, const SegWork& w, long long n
 
 cudaError_t launch_finalize(const DevState& s, int c0, int nc, int parity, int apply_scale, cudaStream_t st) {
     finalize_kernel<<<dim3((s.d_hid + 7) / 8, nc, 2), 256, 0, st>>>(s, c0, parity, apply_scale);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_col_renorm(const DevState& s, int c0, int nc, cudaStream_t st) {
+    col_partial_kernel<<<dim3(s.d_out / 64, kColRowSlices, nc), 256, 0, st>>>(s, c0);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    col_scale_kernel<<<dim3(s.d_out / 64, (s.d_hid + 63) / 64, nc), 256, 0, st>>>(s, c0);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_col_targets(const DevState& s, cudaStream_t st) {
+    col_partial_kernel<<<dim3(s.d_out / 64, kColRowSlices, s.C), 256, 0, st>>>(s, 0);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    col_targets_kernel<<<dim3((s.d_out + 255) / 256, s.C), 256, 0, st>>>(s);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gate_silu(float* gate, size_t n, int from_one, cudaStream_t st) {
+    gate_silu_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(gate, n, from_one);
     return cudaGetLastError();
 }
 

@@ -25,7 +25,9 @@ def config_of(wl: wk.Workload) -> "mone.mone_config":
                             wl.seg_T, mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr,
                             loss=mone.MONE_LOSS_MSE if wl.loss == "mse" else mone.MONE_LOSS_DOT,
                             memory=mone.MONE_MEM_SWIGLU if wl.memory == "swiglu" else mone.MONE_MEM_MLP,
-                            mem_heads=wl.heads)
+                            mem_heads=wl.heads,
+                            renorm_axis=mone.MONE_RENORM_OUT if wl.renorm_axis == "out" else mone.MONE_RENORM_ROWS,
+                            gate_act=mone.MONE_GATE_SILU if wl.gate_act == "silu" else mone.MONE_GATE_LINEAR)
 
 
 class GpuRun:
@@ -79,7 +81,8 @@ class GpuRun:
 
 
 def oracle_hyper(wl: wk.Workload) -> O.Hyper:
-    return O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss, memory=wl.memory, n_heads=wl.heads)
+    return O.Hyper(mode=wl.mode, lr=wl.lr, loss=wl.loss, memory=wl.memory, n_heads=wl.heads,
+                   renorm_axis=wl.renorm_axis, gate_act=wl.gate_act)
 
 
 def oracle_init(wl: wk.Workload, W1_0, W2_0) -> O.State:

@@ -35,7 +35,7 @@ def test_library_exports_every_declared_symbol(L):
     raw = ctypes.CDLL(mone.LIB_PATH)
     for name in header_functions():
         assert hasattr(raw, name), name
-    assert L.mone_abi_version() == 4
+    assert L.mone_abi_version() == 5
 
 
 def test_status_strings(L):
@@ -80,6 +80,14 @@ def test_swiglu_memory_validation(L):
     assert init_rc(L, cfg(**{**sw, "d_out": 768, "n_kv_heads": 6})) == 2  # output width must equal d_in
     assert init_rc(L, cfg(**{**sw, "lr": float("inf")})) == 1             # rates checked for every memory form
     assert init_rc(L, cfg(**{**sw, "rms_eps": float("nan")})) == 1
+
+
+def test_renorm_axis_and_gate_validation(L):
+    assert init_rc(L, cfg(renorm_axis=2)) == 1                  # no such renormalisation axis
+    assert init_rc(L, cfg(gate_act=2)) == 1                     # no such gate activation
+    sw = dict(d_in=896, d_hid=224, d_out=896, n_kv_heads=7, head_dim=64, seg_T=128, memory=mone.MONE_MEM_SWIGLU,
+              mem_heads=4)
+    assert init_rc(L, cfg(**{**sw, "renorm_axis": mone.MONE_RENORM_OUT})) == 7  # output channels: MLP only
 
 
 def test_squared_error_loss_is_bf16_only(L):

@@ -160,6 +160,54 @@ def test_f32_resident_two_input_windows():
     run.close()
 
 
+# ----------------------------------------------------------------- output-channel renorm, SiLU gate
+
+@pytest.mark.parametrize("dtype,loss", [("bf16", "neg_inner"), ("bf16", "mse"), ("f32", "neg_inner")])
+def test_output_channel_renorm_parity(dtype, loss):
+    # W1 rows and W2 columns renormalised to their norms in W_0 (the other reading of App. A)
+    if dtype == "bf16":
+        wl = small(wk.PAPER, N=3 * 256 + 37).replace(renorm_axis="out", loss=loss)
+    else:
+        wl = small(wk.PAPER, "f32", T=128, N=3 * 128 + 50, d_in=128, d_hid=192, d_out=256,
+                   lr=0.5).replace(renorm_axis="out")
+    tol = F32_TOL if dtype == "f32" else BF16_TOL
+    run = GpuRun(wl)
+    mone.mone_mem_set_timing(run.h, 1)
+    run.ttl_context()
+    assert launches(run, "resident") == 0
+    W1, W2, _, _ = run.state()
+    Xq = wk.query_inputs(wl, "cuda")
+    Kg, Vg = run.generate_kv(Xq)
+    for c in range(wl.chains):
+        st = check_chain(run, c, W1, W2, tol)
+        col0 = run.W2_0[c].cpu().double().pow(2).sum(0).sqrt()
+        row0 = run.W1_0[c].cpu().double().pow(2).sum(1).sqrt()
+        assert torch.allclose(W2[c].double().pow(2).sum(0).sqrt(), col0, rtol=1e-5)
+        assert torch.allclose(W1[c].double().pow(2).sum(1).sqrt(), row0, rtol=1e-5)
+        Ko, Vo = oracle_read(run, st, c, Xq)
+        assert rel_fro(Kg[c // 2, c % 2].float(), Ko) <= tol and rel_fro(Vg[c // 2, c % 2].float(), Vo) <= tol
+    run.close()
+
+
+@pytest.mark.parametrize("dtype,mode", [("bf16", wk.PAPER), ("bf16", wk.PLAIN), ("f32", wk.PAPER)])
+def test_silu_gate_read_parity(dtype, mode):
+    # the read scales head h by SiLU(g_h); in plain mode without caller gates, by SiLU(1)
+    if dtype == "bf16":
+        wl = small(mode, N=2 * 256 + 10).replace(gate_act="silu")
+    else:
+        wl = small(mode, "f32", T=128, N=2 * 128 + 10, d_in=128, d_hid=192, d_out=256).replace(gate_act="silu")
+    tol = F32_TOL if dtype == "f32" else BF16_TOL
+    run = GpuRun(wl)
+    run.ttl_context()
+    Xq = wk.query_inputs(wl, "cuda")
+    Kg, Vg = run.generate_kv(Xq)
+    for c in range(wl.chains):
+        st, _ = oracle_chain(run, c)
+        Ko, Vo = oracle_read(run, st, c, Xq)
+        assert rel_fro(Kg[c // 2, c % 2].float(), Ko) <= tol and rel_fro(Vg[c // 2, c % 2].float(), Vo) <= tol
+    run.close()
+
+
 # ----------------------------------------------------------------- bf16 tensor-core path (small shapes)
 
 @pytest.mark.parametrize("mode", [wk.PLAIN, wk.PAPER])

@@ -52,6 +52,8 @@ class Workload:
     loss: str = "neg_inner"  # "neg_inner" (Eq. 7) or "mse" (squared-error variant)
     memory: str = "mlp"      # "mlp" (two-matrix SiLU MLP) or "swiglu" (per-head SwiGLU of Eq. 3)
     heads: int = 1           # swiglu heads: each sees d_in / heads input dimensions, d_hid hidden units
+    renorm_axis: str = "rows"  # paper-mode renormalisation: "rows" of W1 and W2, or "out" (W1 rows, W2 columns)
+    gate_act: str = "linear"   # read gate: g_h ("linear") or SiLU(g_h) ("silu")
 
     @property
     def chains(self) -> int:
