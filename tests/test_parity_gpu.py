@@ -12,7 +12,7 @@ import torch
 import oracle as O
 import paper_2608_17616_gb300 as mone
 import workloads as wk
-from harness import GpuRun, gpu_layout, oracle_chain, oracle_read, rel_fro
+from harness import GpuRun, gpu_layout, oracle_chain, oracle_hyper, oracle_meta, oracle_read, rel_fro
 
 pytestmark = pytest.mark.gpu
 
@@ -205,6 +205,63 @@ def test_silu_gate_read_parity(dtype, mode):
         st, _ = oracle_chain(run, c)
         Ko, Vo = oracle_read(run, st, c, Xq)
         assert rel_fro(Kg[c // 2, c % 2].float(), Ko) <= tol and rel_fro(Vg[c // 2, c % 2].float(), Vo) <= tol
+    run.close()
+
+
+# ----------------------------------------------------------------- edge sizes
+
+def _edge_small(dtype, **kw):
+    if dtype == "bf16":
+        return small(wk.PAPER, **kw)
+    return small(wk.PAPER, "f32", **{**dict(d_in=128, d_hid=192, d_out=256, lr=0.5), **kw})
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_context_shorter_than_a_segment_then_a_one_token_segment(dtype):
+    wl = _edge_small(dtype, n_ctx=1, T=256 if dtype == "bf16" else 128, N=37)
+    tol = F32_TOL if dtype == "f32" else BF16_TOL
+    run = GpuRun(wl)
+    run.ttl_context()                                        # one partial segment: T' = 37
+    W1, W2, _, _ = run.state()
+    for c in range(wl.chains):
+        check_chain(run, c, W1, W2, tol)
+    # then a segment of a single token (T' = 1) on chain 1
+    mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, 36:37], run.K[0, 1, 36:37], run.V[0, 1, 36:37], 1)
+    mone.mone_mem_sync(run.h)
+    W1, W2, _, _ = run.state()
+    st, _ = oracle_chain(run, 1)
+    Y1 = np.concatenate([O.f64(run.K[0, 1, 36:37]), O.f64(run.V[0, 1, 36:37])], axis=1)
+    st, _ = O.ttl_segment(st, O.f64(run.X[0, 1, 36:37]), Y1, oracle_hyper(wl), oracle_meta(run, 1))
+    assert rel_fro(W1[1], st.W["W1"]) <= tol and rel_fro(W2[1], st.W["W2"]) <= tol
+    run.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_largest_segment_T4096_ragged(dtype):
+    # seg_T = 4096 (the largest the library takes) and a ragged second segment; on bf16 with
+    # d_in = d_out = 256 phase B runs on CTA pairs, on fp32 the resident kernel streams 128 chunks
+    wl = _edge_small(dtype, n_ctx=1, T=4096, N=4096 + 300)
+    tol = F32_TOL if dtype == "f32" else BF16_TOL
+    run = GpuRun(wl)
+    run.ttl_context()
+    W1, W2, _, _ = run.state()
+    for c in range(wl.chains):
+        check_chain(run, c, W1, W2, tol)
+    run.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_generate_kv_largest_query_4096(dtype):
+    wl = _edge_small(dtype, n_ctx=1, n_layers=1, T=256 if dtype == "bf16" else 128, N=300, Q=4096)
+    tol = F32_TOL if dtype == "f32" else BF16_TOL
+    run = GpuRun(wl)
+    run.ttl_context()
+    Xq = wk.query_inputs(wl, "cuda")
+    assert Xq.shape[2] == 4096
+    Kg, Vg = run.generate_kv(Xq)
+    st, _ = oracle_chain(run, 0)
+    Ko, Vo = oracle_read(run, st, 0, Xq)
+    assert rel_fro(Kg[0, 0].float(), Ko) <= tol and rel_fro(Vg[0, 0].float(), Vo) <= tol
     run.close()
 
 
