@@ -16,6 +16,10 @@
 
 using namespace mone;
 
+// Kernel kinds of the per-kernel timing (mone_mem_kernel_time).
+enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4, K_MSE = 5, K_ATTN = 6,
+       K_RESIDENT = 7, K_KINDS = 8 };
+
 // Optional per-kernel device timing (mone_mem_set_timing).
 struct KernelTiming {
     bool on = false;
@@ -25,16 +29,16 @@ struct KernelTiming {
     };
     std::vector<cudaEvent_t> pool;
     std::vector<Pending> pending;
-    double ms[8] = {};
-    long long n[8] = {};
+    double ms[K_KINDS] = {};
+    long long n[K_KINDS] = {};
     // start and end of every launch, in ms after `ref` (recorded before the first timed launch
     // since timing was enabled), for the busy time of a kernel kind (mone_mem_kernel_busy)
     cudaEvent_t ref = nullptr;
     bool ref_set = false;
-    std::vector<std::pair<double, double>> iv[8];
+    std::vector<std::pair<double, double>> iv[K_KINDS];
 
     void reset() {
-        for (int k = 0; k < 8; ++k) {
+        for (int k = 0; k < K_KINDS; ++k) {
             ms[k] = 0;
             n[k] = 0;
             iv[k].clear();
@@ -281,8 +285,6 @@ mone_status build_input_maps(const DevState& s, TcInputMaps* in, const void* X, 
     return ok ? MONE_OK : MONE_ERR_CUDA;
 }
 
-enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4, K_MSE = 5, K_ATTN = 6,
-       K_RESIDENT = 7, K_KINDS = 8 };
 
 // Launch through `fn` (which returns a cudaError_t), bracketed by timing events
 // when timing is on; `kernels` is the number of device kernels `fn` launches.
