@@ -75,8 +75,8 @@ enum { MONE_GATE_LINEAR = 0, MONE_GATE_SILU = 1 };   /* how the read's per-head 
  * with l_j = -y_j . M(u_j) (loss MONE_LOSS_DOT: Eq. 7, Eq. 10).  loss MONE_LOSS_MSE
  * replaces l_j by 1/2 |M(u_j) - y_j|^2 (the squared-error, delta-rule form of the
  * same step; its gradient needs M(u_j) at the segment's starting weights, computed
- * by two more kernels per segment).  MONE_LOSS_MSE is supported on the BF16 path;
- * on FP32 mone_mem_init returns MONE_ERR_UNSUPPORTED.
+ * by two more kernels per segment, tcgen05 on BF16, CUDA cores on FP32).  MONE_LOSS_MSE
+ * is supported for the MLP memory on both paths.
  *
  * memory MONE_MEM_MLP: M(u) = SiLU(u W1^T) W2, W1 [d_hid][d_in], W2 [d_hid][d_out] per chain.
  * memory MONE_MEM_SWIGLU (Eq. 3 itself): u splits into mem_heads heads of width dh = d_in / mem_heads;

@@ -114,7 +114,6 @@ mone_status validate_config(const mone_config* c) {
     if (c->dtype != MONE_FP32 && c->dtype != MONE_BF16) return MONE_ERR_INVALID_ARG;
     if (c->mode != MONE_PLAIN && c->mode != MONE_PAPER) return MONE_ERR_INVALID_ARG;
     if (c->loss != MONE_LOSS_DOT && c->loss != MONE_LOSS_MSE) return MONE_ERR_INVALID_ARG;
-    if (c->loss == MONE_LOSS_MSE && c->dtype != MONE_BF16) return MONE_ERR_UNSUPPORTED;
     if (c->memory != MONE_MEM_MLP && c->memory != MONE_MEM_SWIGLU) return MONE_ERR_INVALID_ARG;
     if (c->renorm_axis != MONE_RENORM_ROWS && c->renorm_axis != MONE_RENORM_OUT) return MONE_ERR_INVALID_ARG;
     if (c->gate_act != MONE_GATE_LINEAR && c->gate_act != MONE_GATE_SILU) return MONE_ERR_INVALID_ARG;
@@ -171,7 +170,7 @@ mone_status dalloc(T** p, size_t n) {
 void free_state(DevState& s) {
     void* ptrs[] = {s.W1, s.W2, s.mu1, s.mu2, s.W1b, s.W2b, s.n1, s.n2, s.sumsq, s.status, s.alpha, s.gamma,
                     s.w_eta, s.b_eta, s.w_beta, s.b_beta, s.gate, s.U, s.eta, s.dbeta, s.zinv, s.dHt, s.Att, s.Uq, s.Aq,
-                    s.Oq, s.Amse, s.Kres, s.Vres, s.nc2, s.colpart};
+                    s.Oq, s.Amse, s.Kres, s.Vres, s.Kres32, s.Vres32, s.nc2, s.colpart};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     std::memset(&s, 0, sizeof(s));
@@ -397,6 +396,13 @@ mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInput
             } else if (s.dtype == MONE_BF16) {
                 MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_phase_a_tc(s, m->maps, gin[g], x, sg); }));
                 MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_phase_b_tc(s, m->maps, gin[g], x, sg); }));
+            } else if (s.loss == MONE_LOSS_MSE) {  // fp32: the same scheme on the CUDA cores
+                MONE_TRY(timed(m, K_MSE, sg, 2, [&] { return launch_mse_f32(s, x, sg); }));
+                SegWork xr = x;
+                xr.y_scratch = 1;
+                xr.loss = nullptr;
+                MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_phase_a_f32(s, xr, sg); }));
+                MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_phase_b_f32(s, xr, sg); }));
             } else {
                 MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_phase_a_f32(s, x, sg); }));
                 MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_phase_b_f32(s, x, sg); }));
@@ -538,6 +544,10 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
             step(dalloc(&s.Kres, C * s.T * (s.d_out / 2)));
             step(dalloc(&s.Vres, C * s.T * (s.d_out / 2)));
         }
+    }
+    if (s.dtype == MONE_FP32 && s.loss == MONE_LOSS_MSE) {
+        step(dalloc(&s.Kres32, C * s.T * (s.d_out / 2)));
+        step(dalloc(&s.Vres32, C * s.T * (s.d_out / 2)));
     }
     step(dalloc(&s.n1, r1));
     step(dalloc(&s.n2, w2_rows(s)));

@@ -41,6 +41,7 @@ struct DevState {
     // in, and the residual targets y - M(u) that phase A and phase B read in place of K, V
     bf16* Amse;                   // [C][T][d_hid]
     bf16 *Kres, *Vres;            // [C][T][d_out/2]
+    float *Kres32, *Vres32;       // the same on the fp32 path
     // read scratch (grown on demand)
     int q_cap;
     float *Uq, *Aq, *Oq;          // [C][q_cap][d_in|d_hid|d_out]
@@ -89,6 +90,9 @@ cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, voi
 // ---- kernels in ttl_simt.cu (fp32 path, state upkeep, read path)
 cudaError_t launch_phase_a_f32(const DevState& s, const SegWork& w, cudaStream_t st);
 cudaError_t launch_phase_b_f32(const DevState& s, const SegWork& w, cudaStream_t st);
+// Squared-error pre-pass of one segment on the fp32 path (two kernels): M(u) at the segment's
+// starting weights, the residual targets y - M(u) into s.Kres32 / s.Vres32, the loss into w.loss.
+cudaError_t launch_mse_f32(const DevState& s, const SegWork& w, cudaStream_t st);
 // The whole call in one launch per input window, each CTA keeping RB hidden units of one chain
 // on chip across the segments (fp32 MLP with the Eq. 7 loss, d_in + d_out <= 512).  Leaves the
 // weights renormalised, so no finalize follows.  w: the call's chains, row0 / u_off of the window.

@@ -267,9 +267,15 @@ F32SegArgs make_f32_args(const DevState& s, const SegWork& w) {
         a.U = reinterpret_cast<const float*>(w.X) + w.row0 * s.d_in;
         a.u_cstride = w.x_cstride;
     }
-    a.K = reinterpret_cast<const float*>(w.K) + w.row0 * dh;
-    a.V = reinterpret_cast<const float*>(w.V) + w.row0 * dh;
-    a.y_cstride = w.y_cstride;
+    if (w.y_scratch) {  // squared error: the residual targets of this segment, rows from 0
+        a.K = s.Kres32 + (size_t)w.c0 * s.T * dh;
+        a.V = s.Vres32 + (size_t)w.c0 * s.T * dh;
+        a.y_cstride = (long long)s.T * dh;
+    } else {
+        a.K = reinterpret_cast<const float*>(w.K) + w.row0 * dh;
+        a.V = reinterpret_cast<const float*>(w.V) + w.row0 * dh;
+        a.y_cstride = w.y_cstride;
+    }
     a.row_avail = w.n_rows - w.row0;
     a.eta_in = w.eta_in ? w.eta_in + w.row0 : nullptr;
     a.eta_cstride = w.eta_cstride;
@@ -281,6 +287,77 @@ F32SegArgs make_f32_args(const DevState& s, const SegWork& w) {
     a.loss = w.loss;
     a.status = s.status;
     return a;
+}
+
+// ------------------------------------------------------------------ squared-error pre-pass (fp32)
+//
+// Under the squared-error loss dL/dO = eta (M(u) - y) / T' = -eta (y - M(u)) / T', so the
+// residual target y - M(u), with M(u) at the segment's starting weights, takes the place of
+// y in both phases.  Two kernels: A' = SiLU(s1 H) s2 with the pending row scales folded in
+// (so A' W2raw = A W2), written to the At scratch, which phase A overwrites only after
+// the second kernel has read it; then the residual y - A' W2raw into the residual scratch
+// and 1/2 |y - M(u)|^2 / T' into the loss.
+
+__global__ void __launch_bounds__(256) mse_hidden_f32_kernel(const F32SegArgs a) {
+    __shared__ float As[TK][A_TM + 4], Bs[TK][TN + 4];
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    const int t0 = blockIdx.x * A_TM, h0 = blockIdx.y * TN, cz = blockIdx.z, cs = a.c0 + cz;
+    int m_valid = (int)min((long long)min(A_TM, a.Tp - t0), a.row_avail - t0);
+    if (m_valid < 0) m_valid = 0;
+    float acc[A_MR][4] = {};
+    simt_tile(acc, a.U + cz * a.u_cstride + (long long)t0 * a.d_in, a.d_in, 1,
+              a.W1 + ((size_t)cs * a.d_hid + h0) * a.d_in, a.d_in, 1, a.d_in, m_valid, a.d_in, As, Bs);
+    const float* prev1 = ss_ptr(a, a.parity ^ 1, 0) + (size_t)cs * a.d_hid;
+    const float* prev2 = ss_ptr(a, a.parity ^ 1, 1) + (size_t)cs * a.d_hid;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const int h = h0 + tx * 4 + j;
+        const float s1 = a.renorm_pending ? renorm_scale(a.n1[(size_t)cs * a.d_hid + h], prev1[h]) : 1.f;
+        const float s2 = a.renorm_pending ? renorm_scale(a.n2[(size_t)cs * a.d_hid + h], prev2[h]) : 1.f;
+#pragma unroll
+        for (int i = 0; i < A_MR; ++i) {
+            const int t = t0 + ty * A_MR + i;
+            const float x = acc[i][j] * s1;
+            a.At[((size_t)cs * a.T + t) * a.d_hid + h] = x * sigmoidf_(x) * s2;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(256) mse_out_f32_kernel(const F32SegArgs a, float* Kres, float* Vres) {
+    __shared__ float As[TK][A_TM + 4], Bs[TK][TN + 4];
+    __shared__ float red[8];
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    const int t0 = blockIdx.x * A_TM, o0 = blockIdx.y * TN, cz = blockIdx.z, cs = a.c0 + cz;
+    const int dh = a.d_out / 2;
+    float acc[A_MR][4] = {};
+    simt_tile(acc, a.At + ((size_t)cs * a.T + t0) * a.d_hid, a.d_hid, 1, a.W2 + (size_t)cs * a.d_hid * a.d_out + o0,
+              1, a.d_out, a.d_hid, min(A_TM, a.T - t0), a.d_hid, As, Bs);
+    const bool kpart = o0 < dh;  // dh is a multiple of 64: a tile is all K or all V
+    const int col0 = (kpart ? o0 : o0 - dh) + tx * 4;
+    const float* Y = (kpart ? a.K : a.V) + cz * a.y_cstride + col0;
+    float* R = (kpart ? Kres : Vres) + (size_t)cs * a.T * dh + col0;
+    float lsum = 0.f;
+#pragma unroll
+    for (int i = 0; i < A_MR; ++i) {
+        const int t = t0 + ty * A_MR + i;
+        const bool live = t < a.Tp && t < a.row_avail;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float r = live ? Y[(long long)t * dh + j] - acc[i][j] : 0.f;
+            R[(size_t)t * dh + j] = r;
+            lsum = fmaf(r, r, lsum);
+        }
+    }
+    if (a.loss) {
+        lsum = warp_sum(lsum);
+        if ((tid & 31) == 0) red[tid >> 5] = lsum;
+        __syncthreads();
+        if (tid == 0) {
+            float tot = 0.f;
+            for (int w = 0; w < 8; ++w) tot += red[w];
+            atomicAdd(&a.loss[cz], 0.5f * tot / (float)a.Tp);
+        }
+    }
 }
 
 // ------------------------------------------------------------------ resident chains (fp32)
@@ -881,6 +958,15 @@ cudaError_t launch_resident_f32(const DevState& s, const SegWork& w, long long n
         if (e != cudaSuccess) return e;
         ttl_resident_f32_kernel<8><<<dim3(s.d_hid / 8, w.nc), 256, bytes, st>>>(a);
     }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_mse_f32(const DevState& s, const SegWork& w, cudaStream_t st) {
+    F32SegArgs a = make_f32_args(s, w);
+    mse_hidden_f32_kernel<<<dim3((s.T + A_TM - 1) / A_TM, s.d_hid / TN, w.nc), 256, 0, st>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    mse_out_f32_kernel<<<dim3((s.T + A_TM - 1) / A_TM, s.d_out / TN, w.nc), 256, 0, st>>>(a, s.Kres32, s.Vres32);
     return cudaGetLastError();
 }
 

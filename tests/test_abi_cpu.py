@@ -90,9 +90,15 @@ def test_renorm_axis_and_gate_validation(L):
     assert init_rc(L, cfg(**{**sw, "renorm_axis": mone.MONE_RENORM_OUT})) == 7  # output channels: MLP only
 
 
-def test_squared_error_loss_is_bf16_only(L):
-    # the squared-error variant runs on the tensor-core path only: the fp32 path reports it unsupported
-    assert init_rc(L, cfg(dtype=mone.MONE_FP32, loss=mone.MONE_LOSS_MSE)) == 7
+def test_squared_error_loss_passes_validation_on_both_paths(L):
+    # the squared-error variant runs on both paths (MLP memory).  The configuration is checked
+    # before the weight pointers, so a misaligned W1_0 (argument error, no device work) shows
+    # that the configuration itself was accepted
+    for dtype in (mone.MONE_FP32, mone.MONE_BF16):
+        assert init_rc(L, cfg(dtype=dtype, loss=mone.MONE_LOSS_MSE), w1=8) == 1
+    # (an unsupported configuration still answers 7 with the same misaligned pointer)
+    assert init_rc(L, cfg(memory=mone.MONE_MEM_SWIGLU, d_in=896, d_hid=224, d_out=896, n_kv_heads=7, mem_heads=4,
+                          loss=mone.MONE_LOSS_MSE), w1=8) == 7
 
 
 def test_init_rejects_unsupported_shapes(L):

@@ -108,6 +108,39 @@ def launches(run, kind):
     return mone.mone_mem_kernel_time(run.h, mone.KERNEL_KINDS.index(kind))[1]
 
 
+def test_f32_mse_per_step_parity_and_loss():
+    # the squared-error (delta-rule) variant on the fp32 path: per-step weights and loss at 1e-4
+    wl = wk.WORKLOADS["tiny_f32"].replace(loss="mse", N=8 * 128)
+    run = GpuRun(wl)
+    _, losses, trail = oracle_chain(run, 0, return_all=True)
+    loss_dev = torch.zeros(1, device="cuda")
+    T = wl.seg_T
+    for s in range(wl.S):
+        sl = slice(s * T, (s + 1) * T)
+        mone.mone_ttl_segment(run.h, 0, 0, run.X[0, 0, sl], run.K[0, 0, sl], run.V[0, 0, sl], T, None, loss_dev)
+        mone.mone_mem_sync(run.h)
+        W1, W2, _, _ = run.state()
+        assert rel_fro(W1[0], trail[s].W["W1"]) <= F32_TOL, s
+        assert rel_fro(W2[0], trail[s].W["W2"]) <= F32_TOL, s
+        assert abs(loss_dev.item() - losses[s]) <= F32_TOL * max(1.0, abs(losses[s])), s
+    run.close()
+
+
+def test_f32_mse_paper_ragged():
+    wl = small(wk.PAPER, "f32", T=128, N=3 * 128 + 50, d_in=128, d_hid=192, d_out=256).replace(loss="mse")
+    run = GpuRun(wl)
+    run.ttl_context()
+    W1, W2, mu1, mu2 = run.state()
+    Xq = wk.query_inputs(wl, "cuda")
+    Kg, Vg = run.generate_kv(Xq)
+    for c in range(wl.chains):
+        st = check_chain(run, c, W1, W2, F32_TOL)
+        assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+        Ko, Vo = oracle_read(run, st, c, Xq)
+        assert rel_fro(Kg[c // 2, c % 2], Ko) <= F32_TOL and rel_fro(Vg[c // 2, c % 2], Vo) <= F32_TOL
+    run.close()
+
+
 def test_f32_tiled_path_paper_ragged():
     # d_in + d_out > 512: the rows stay in HBM and the per-segment fp32 phase kernels run
     wl = small(wk.PAPER, "f32", n_ctx=1, T=64, N=3 * 64 + 20, d_in=512, d_hid=128, d_out=256, lr=0.5)
