@@ -168,7 +168,10 @@ mone_status mone_ttl_context(mone_mem* m, const void* X, const void* K, const vo
  * Xq: [n_ctx][n_layers][Q][d_in] contiguous.  strides[4] are ELEMENT strides of the
  * output for (ctx, layer, kv_head, q); head_dim is contiguous, so memory tokens can
  * be written straight into an attention cache (e.g. after the query's own K/V,
- * as in Eq. 5's concatenation).  1 <= Q <= 4096.
+ * as in Eq. 5's concatenation).  1 <= Q <= 4096.  gate_h is SiLU(g_h) under
+ * MONE_GATE_SILU.  The second and later consecutive calls with the same Xq, K_out,
+ * V_out, Q and strides replay the launches of that read as one captured CUDA graph
+ * (same kernels, same results; the weights and inputs are read when it runs).
  * Errors: INVALID_ARG, OOM (first call with a larger Q allocates scratch), CUDA.
  */
 mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out, void* V_out,
