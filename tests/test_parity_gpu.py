@@ -241,6 +241,30 @@ def test_silu_gate_read_parity(dtype, mode):
     run.close()
 
 
+# ----------------------------------------------------------------- contexts over several input windows
+
+@pytest.mark.parametrize("dtype,loss", [("bf16", "neg_inner"), ("bf16", "mse"), ("f32", "neg_inner")])
+def test_context_over_several_input_windows(dtype, loss):
+    # paper mode transforms the input 64 segments at a time (one window), and both chain groups
+    # join before each window's transform: 3 full windows and a ragged fourth (bf16, both losses),
+    # and 2 + ragged on the fp32 tiled path
+    if dtype == "bf16":
+        wl = small(wk.PAPER, T=128, N=3 * 64 * 128 + 100).replace(loss=loss)
+    else:
+        wl = small(wk.PAPER, "f32", n_ctx=1, T=64, N=2 * 64 * 64 + 100, d_in=512, d_hid=128, d_out=256, lr=0.5)
+    tol = F32_TOL if dtype == "f32" else BF16_TOL
+    run = GpuRun(wl)
+    mone.mone_mem_set_timing(run.h, 1)
+    run.ttl_context()
+    assert launches(run, "prepass") == -(-wl.S // 64)
+    W1, W2, mu1, mu2 = run.state()
+    for c in range(wl.chains):
+        st = check_chain(run, c, W1, W2, tol)
+        if dtype == "f32":
+            assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+    run.close()
+
+
 # ----------------------------------------------------------------- edge sizes
 
 def _edge_small(dtype, **kw):

@@ -57,6 +57,18 @@ def test_swiglu_small_paper_mode_ragged_hidden_tiles():
     run.close()
 
 
+def test_swiglu_context_over_several_input_windows():
+    # 64 segments a window: 3 full windows and a ragged fourth, each transformed after both
+    # chain groups are done with the previous one
+    wl = swiglu(n_ctx=1, N=3 * 64 * 128 + 70)
+    run = GpuRun(wl)
+    mone.mone_mem_set_timing(run.h, 1)
+    run.ttl_context()
+    assert mone.mone_mem_kernel_time(run.h, mone.KERNEL_KINDS.index("prepass"))[1] == 4
+    check(run, range(wl.chains), wk.query_inputs(wl, "cuda"))
+    run.close()
+
+
 def test_swiglu_paper_head_shape():
     # the paper's head shape: d = 896 as 4 heads of 224, 224 hidden units (k-blocks and hidden tiles
     # both run past 224), K || V = 2 x 7 heads of 64
