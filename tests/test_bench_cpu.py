@@ -51,3 +51,15 @@ def test_recorded_traffic_applies_only_to_its_shape(tmp_path, monkeypatch):
     (tmp_path / "paper_2608_17616_gb300" / "csrc" / "ttl_tc.cu").write_text(
         src.replace(banner, banner + "\n// edited", 1))
     assert bench.ncu_traffic("phase_b", 8.0, wk.WORKLOADS["l16_d2048_128k"])[0] is None
+
+
+def test_resident_kernel_work_counts_inputs_per_segment_and_state_per_launch():
+    # the resident fp32 kernel covers a window of segments in one launch: U and Y (fp32) stream once
+    # per segment, W (and mu in paper mode) cross HBM once per launch
+    wl = wk.WORKLOADS["tiny_f32"]
+    S = wl.S
+    flops, byts = bench.kernel_work(wl, "resident", wl.chains * S)
+    assert flops == wl.N * 4 * (256 * 512 + 512 * 256)
+    assert byts == wl.N * (256 + 256) * 4 + 512 * (256 + 256) * 8      # plain mode: W read and write
+    paper = wl.replace(mode=wk.PAPER)
+    assert bench.kernel_work(paper, "resident", wl.chains * S)[1] == byts + 512 * (256 + 256) * 8  # + momentum
