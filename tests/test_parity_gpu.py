@@ -195,14 +195,14 @@ def test_f32_resident_two_input_windows():
 
 # ----------------------------------------------------------------- output-channel renorm, SiLU gate
 
-@pytest.mark.parametrize("dtype,loss", [("bf16", "neg_inner"), ("bf16", "mse"), ("f32", "neg_inner")])
+@pytest.mark.parametrize("dtype,loss", [("bf16", "neg_inner"), ("bf16", "mse"), ("f32", "neg_inner"), ("f32", "mse")])
 def test_output_channel_renorm_parity(dtype, loss):
     # W1 rows and W2 columns renormalised to their norms in W_0 (the other reading of App. A)
     if dtype == "bf16":
         wl = small(wk.PAPER, N=3 * 256 + 37).replace(renorm_axis="out", loss=loss)
     else:
         wl = small(wk.PAPER, "f32", T=128, N=3 * 128 + 50, d_in=128, d_hid=192, d_out=256,
-                   lr=0.5).replace(renorm_axis="out")
+                   lr=0.5).replace(renorm_axis="out", loss=loss)
     tol = F32_TOL if dtype == "f32" else BF16_TOL
     run = GpuRun(wl)
     mone.mone_mem_set_timing(run.h, 1)

@@ -69,6 +69,15 @@ def test_swiglu_context_over_several_input_windows():
     run.close()
 
 
+def test_swiglu_read_with_silu_gate():
+    # the read scales head h by SiLU(g_h) (the other reading of the gate), on the SwiGLU memory too
+    wl = swiglu(n_ctx=1).replace(gate_act="silu")
+    run = GpuRun(wl)
+    run.ttl_context()
+    check(run, range(wl.chains), wk.query_inputs(wl, "cuda"))
+    run.close()
+
+
 def test_swiglu_paper_head_shape():
     # the paper's head shape: d = 896 as 4 heads of 224, 224 hidden units (k-blocks and hidden tiles
     # both run past 224), K || V = 2 x 7 heads of 64
