@@ -265,6 +265,37 @@ def test_context_over_several_input_windows(dtype, loss):
     run.close()
 
 
+# ----------------------------------------------------------------- a zero learning rate
+
+@pytest.mark.parametrize("dtype,shape", [("bf16", {}), ("f32", dict(d_in=128, d_hid=192, d_out=256, T=128)),
+                                         ("f32", dict(d_in=512, d_hid=128, d_out=256, T=64))])
+def test_zero_learning_rate_leaves_the_weights_bit_identical(dtype, shape):
+    # plain mode with lr = 0: every gradient is exactly zero, so W comes back bit for bit (bf16
+    # path, fp32 resident kernel, fp32 tiled kernels)
+    wl = small(wk.PLAIN, dtype, lr=0.0, **shape)
+    run = GpuRun(wl)
+    run.ttl_context()
+    W1, W2, _, _ = run.state()
+    assert torch.equal(W1, run.W1_0.cpu()) and torch.equal(W2, run.W2_0.cpu())
+    run.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_zero_caller_rates_in_paper_mode_keep_the_state(dtype):
+    # paper mode, caller rates all zero: the momentum stays exactly zero and W moves only by the
+    # rounding of the renormalisation scale (n0 / |row|, both fp32 sums of the same row)
+    n = 200 if dtype == "bf16" else 100  # one partial segment (T = 256 / 128)
+    wl = _edge_small(dtype, n_ctx=1, T=256 if dtype == "bf16" else 128, N=n)
+    run = GpuRun(wl)
+    eta = torch.zeros(n, device="cuda")
+    mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, :n], run.K[0, 1, :n], run.V[0, 1, :n], n, eta)
+    mone.mone_mem_sync(run.h)
+    W1, W2, mu1, mu2 = run.state()
+    assert not torch.any(mu1) and not torch.any(mu2)
+    assert rel_fro(W1[1], O.f64(run.W1_0[1])) <= 1e-6 and rel_fro(W2[1], O.f64(run.W2_0[1])) <= 1e-6
+    run.close()
+
+
 # ----------------------------------------------------------------- edge sizes
 
 def _edge_small(dtype, **kw):
