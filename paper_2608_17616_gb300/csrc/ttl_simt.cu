@@ -377,9 +377,12 @@ __global__ void __launch_bounds__(256) mse_out_f32_kernel(const F32SegArgs a, fl
 // of the segment the update (momentum, W -= mu) and the row renormalisation are
 // applied in place.
 //
-// Forward: an output group is 2 tokens x 2 hidden units, its contraction split over
-// KS = 32 / RB lanes (float4 steps over interleaved columns), then summed by
-// shuffles.  Backward: thread i owns columns 2i, 2i + 1 of all RB rows.
+// 512 threads (16 warps), so that shared-memory and FMA latencies are hidden.  Forward: half
+// of the CTA contracts U with the W1 rows (H), the other half Y with the W2 rows (R); an
+// output group is 2 tokens x 2 hidden units, its contraction split over KS = 32 / RB lanes
+// (float4 steps over interleaved columns) and summed by shuffles; one thread per (token,
+// hidden unit) then finishes the epilogue.  Backward: thread i owns column i of [W1 | W2]
+// for all RB rows.
 constexpr int RES_RC = 32;                                             // tokens per streamed chunk
 __host__ __device__ constexpr int res_ld(int D) { return (D + 31) / 32 * 32 + 16; }  // row pitch, floats
 
@@ -422,29 +425,32 @@ __device__ __forceinline__ float dot4(const float4 a, const float4 b, float acc)
     return fmaf(a.w, b.w, acc);
 }
 
-// Sum of v over the CTA (256 threads); every thread gets the total.  red: 8 floats.
-__device__ __forceinline__ float block_sum256(float v, float* red) {
+constexpr int RES_NT = 512, RES_NW = RES_NT / 32;  // threads and warps of a resident CTA
+
+// Sum of v over the CTA; every thread gets the total.  red: RES_NW floats.
+__device__ __forceinline__ float block_sum_res(float v, float* red) {
     v = warp_sum(v);
     __syncthreads();
     if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
     __syncthreads();
     float t = 0.f;
 #pragma unroll
-    for (int w = 0; w < 8; ++w) t += red[w];
+    for (int w = 0; w < RES_NW; ++w) t += red[w];
     return t;
 }
 
 template <int RB>
-__global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) {
-    constexpr int RC = RES_RC, KS = 32 / RB, RH = RB / 2;
+__global__ void __launch_bounds__(RES_NT, 1) ttl_resident_f32_kernel(const ResArgs a) {
+    constexpr int RC = RES_RC, KS = 32 / RB, RH = RB / 2, NW = RES_NW;
     static_assert(RB == 4 || RB == 8, "rows per CTA");
     extern __shared__ float4 res_smem[];
     const int D = a.d_in + a.d_out, LD = res_ld(D), dh = a.d_out / 2;
     float* Ws = reinterpret_cast<float*>(res_smem);  // [RB][LD]
     float* Xs = Ws + RB * LD;                        // [2][RC][LD]: rows [U | K | V] of a chunk
     float* Gs = Xs + 2 * RC * LD;                    // [RC][2][RB]: c dH, c A of the chunk
-    float* red = Gs + RC * 2 * RB;                   // [8][2 RB]
-    float* scl = red + 8 * 2 * RB;                   // [2 RB] row scales, then beta
+    float* HQ = Gs + RC * 2 * RB;                    // [2][RC][RB]: H and R of the chunk
+    float* red = HQ + 2 * RC * RB;                   // [NW][2 RB]
+    float* scl = red + NW * 2 * RB;                  // [2 RB] row scales, then beta
     float* etaS = scl + 2 * RB + 4;                  // [2][RC] rates of the chunk's tokens
     float* dbS = etaS + 2 * RC;                      // [2][RC] w_beta . x of the chunk's tokens
     float* nS = dbS + 2 * RC;                        // [2 RB] renormalisation targets
@@ -461,7 +467,7 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
         const int Tp = (int)min((long long)a.T, a.n_tok - t_seg);
         const int nvalid = min(RC, Tp - ch * RC);
         const long long r0 = t_seg + ch * RC;
-        for (int t = warp; t < RC; t += 8) {
+        for (int t = warp; t < RC; t += NW) {
             const bool v = t < nvalid;
             const long long r = r0 + (v ? t : 0);
             const float* ur = Uc + r * a.d_in;
@@ -491,8 +497,8 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
         }
     };
 
-    // resident rows, momentum (registers) and the thread's columns for the backward
-    for (int i = tid; i < RB * (D / 4); i += 256) {
+    // resident rows, and the momentum of the thread's column (registers)
+    for (int i = tid; i < RB * (D / 4); i += RES_NT) {
         const int r = i / (D / 4), c = 4 * (i - r * (D / 4));
         const size_t row = (size_t)cs * a.d_hid + h0 + r;
         const float* src = c < a.d_in ? a.W1 + row * a.d_in + c : a.W2 + row * a.d_out + (c - a.d_in);
@@ -500,26 +506,25 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
     }
     if (tid < 2 * RB) nS[tid] = (tid < RB ? a.n1 : a.n2)[(size_t)cs * a.d_hid + h0 + tid % RB];
     const float b_beta = a.momentum ? a.b_beta[cs] : 0.f;
-    const int cb = 2 * tid;                      // first owned column
+    const int cb = tid;                          // owned column of [W1 | W2]
     const bool own = cb < D;
-    const int kind = cb < a.d_in ? 0 : 1;        // d_in is even: both columns are in one matrix
-    float mu[RB][2], acc[RB][2];
+    const int kind = cb < a.d_in ? 0 : 1;
+    float mu[RB], acc[RB];
 #pragma unroll
     for (int r = 0; r < RB; ++r) {
-        mu[r][0] = mu[r][1] = 0.f;
-        acc[r][0] = acc[r][1] = 0.f;
+        mu[r] = 0.f;
+        acc[r] = 0.f;
         if (own && a.momentum) {
             const size_t row = (size_t)cs * a.d_hid + h0 + r;
-            const float2 m2 = kind == 0 ? *reinterpret_cast<const float2*>(a.mu1 + row * a.d_in + cb)
-                                        : *reinterpret_cast<const float2*>(a.mu2 + row * a.d_out + (cb - a.d_in));
-            mu[r][0] = m2.x;
-            mu[r][1] = m2.y;
+            mu[r] = kind == 0 ? a.mu1[row * a.d_in + cb] : a.mu2[row * a.d_out + (cb - a.d_in)];
         }
     }
 
-    // forward mapping: output group og = (token pair tp, row pair rp), contraction lane ks
-    const int ks = tid % KS, og = tid / KS, rp = og % RH, tp = og / RH;
-    const int er = ks & 1, et = (ks >> 1) & 1;   // the output this lane finishes (ks < 4)
+    // forward mapping: half 0 contracts U with W1 (H), half 1 Y with W2 (R); within a half an
+    // output group og = (token pair tp, row pair rp) and a contraction lane ks
+    const int half = tid >> 8, ht = tid & 255;
+    const int ks = ht % KS, og = ht / KS, rp = og % RH, tp = og / RH;
+    const int c_lo = half ? a.d_in : 0, c_hi = half ? D : a.d_in;
     bool finite = true;
     int buf = 0;
     issue(0, 0, 0);
@@ -538,34 +543,23 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
             cp_async_wait<1>();
             __syncthreads();
             const float* Xb = Xs + buf * RC * LD;
-            // H and R of tokens (tp, tp + 16) x rows (rp, rp + RH)
-            float h[2][2] = {}, q[2][2] = {};
+            // tokens (tp, tp + 16) x rows (rp, rp + RH) of H (half 0) or R (half 1)
+            float p[2][2] = {};
             {
                 const float* x0 = Xb + tp * LD;
                 const float* x1 = Xb + (tp + 16) * LD;
                 const float* w0 = Ws + rp * LD;
                 const float* w1 = Ws + (rp + RH) * LD;
 #pragma unroll 2
-                for (int c = 4 * ks; c < a.d_in; c += 4 * KS) {
+                for (int c = c_lo + 4 * ks; c < c_hi; c += 4 * KS) {
                     const float4 u0 = *reinterpret_cast<const float4*>(x0 + c);
                     const float4 u1 = *reinterpret_cast<const float4*>(x1 + c);
                     const float4 b0 = *reinterpret_cast<const float4*>(w0 + c);
                     const float4 b1 = *reinterpret_cast<const float4*>(w1 + c);
-                    h[0][0] = dot4(u0, b0, h[0][0]);
-                    h[0][1] = dot4(u0, b1, h[0][1]);
-                    h[1][0] = dot4(u1, b0, h[1][0]);
-                    h[1][1] = dot4(u1, b1, h[1][1]);
-                }
-#pragma unroll 2
-                for (int c = a.d_in + 4 * ks; c < D; c += 4 * KS) {
-                    const float4 y0 = *reinterpret_cast<const float4*>(x0 + c);
-                    const float4 y1 = *reinterpret_cast<const float4*>(x1 + c);
-                    const float4 b0 = *reinterpret_cast<const float4*>(w0 + c);
-                    const float4 b1 = *reinterpret_cast<const float4*>(w1 + c);
-                    q[0][0] = dot4(y0, b0, q[0][0]);
-                    q[0][1] = dot4(y0, b1, q[0][1]);
-                    q[1][0] = dot4(y1, b0, q[1][0]);
-                    q[1][1] = dot4(y1, b1, q[1][1]);
+                    p[0][0] = dot4(u0, b0, p[0][0]);
+                    p[0][1] = dot4(u0, b1, p[0][1]);
+                    p[1][0] = dot4(u1, b0, p[1][0]);
+                    p[1][1] = dot4(u1, b1, p[1][1]);
                 }
             }
 #pragma unroll
@@ -573,16 +567,19 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
 #pragma unroll
                 for (int i = 0; i < 2; ++i)
 #pragma unroll
-                    for (int j = 0; j < 2; ++j) {
-                        h[i][j] += __shfl_xor_sync(0xffffffffu, h[i][j], o);
-                        q[i][j] += __shfl_xor_sync(0xffffffffu, q[i][j], o);
-                    }
+                    for (int j = 0; j < 2; ++j) p[i][j] += __shfl_xor_sync(0xffffffffu, p[i][j], o);
+            if (ks == 0) {
+#pragma unroll
+                for (int i = 0; i < 2; ++i)
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) HQ[(half * RC + tp + 16 * i) * RB + rp + RH * j] = p[i][j];
+            }
             if (a.momentum && warp == 0) dbsum += warp_sum(lane < Tp - ch * RC ? dbS[buf * RC + lane] : 0.f);
-            if (ks < 4) {
-                // epilogue of one output: c_t = -eta_t / T' (Eq. 10), A = SiLU(H)
-                const int t = tp + 16 * et, r = rp + RH * er;
-                const float hv = et ? (er ? h[1][1] : h[1][0]) : (er ? h[0][1] : h[0][0]);
-                const float rv = et ? (er ? q[1][1] : q[1][0]) : (er ? q[0][1] : q[0][0]);
+            __syncthreads();
+            if (tid < RC * RB) {
+                // epilogue of output (t, r): c_t = -eta_t / T' (Eq. 10), A = SiLU(H)
+                const int t = tid / RB, r = tid % RB;
+                const float hv = HQ[t * RB + r], rv = HQ[(RC + t) * RB + r];
                 const int ts = ch * RC + t;  // token within the segment
                 const float ct = ts < Tp ? -etaS[buf * RC + t] / (float)Tp : 0.f;
                 const float sg = sigmoidf_(hv);
@@ -593,23 +590,20 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
                 Gs[(t * 2 + 1) * RB + r] = ct * av;
             }
             __syncthreads();
-            // gradient rows: acc[r][j] += sum_t G[t][kind][r] * X[t][cb + j]
+            // gradient rows: acc[r] += sum_t G[t][kind][r] * X[t][cb]
             if (own) {
                 const int nv = min(RC, Tp - ch * RC);
                 const float* gk = Gs + kind * RB;
 #pragma unroll 4
                 for (int t = 0; t < nv; ++t) {
-                    const float2 x = *reinterpret_cast<const float2*>(Xb + t * LD + cb);
-                    float g[RB];
+                    const float x = Xb[t * LD + cb];
 #pragma unroll
                     for (int r4 = 0; r4 < RB; r4 += 4) {
                         const float4 g4 = *reinterpret_cast<const float4*>(gk + t * 2 * RB + r4);
-                        g[r4] = g4.x; g[r4 + 1] = g4.y; g[r4 + 2] = g4.z; g[r4 + 3] = g4.w;
-                    }
-#pragma unroll
-                    for (int r = 0; r < RB; ++r) {
-                        acc[r][0] = fmaf(g[r], x.x, acc[r][0]);
-                        acc[r][1] = fmaf(g[r], x.y, acc[r][1]);
+                        acc[r4] = fmaf(g4.x, x, acc[r4]);
+                        acc[r4 + 1] = fmaf(g4.y, x, acc[r4 + 1]);
+                        acc[r4 + 2] = fmaf(g4.z, x, acc[r4 + 2]);
+                        acc[r4 + 3] = fmaf(g4.w, x, acc[r4 + 3]);
                     }
                 }
             }
@@ -624,36 +618,31 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
             beta = scl[2 * RB];
         }
         if (a.loss) {
-            const float tot = block_sum256(lsum, red);
+            const float tot = block_sum_res(lsum, red);
             if (tid == 0) atomicAdd(&a.loss[cz], -tot / (float)Tp);
         }
-        float wn[RB][2], ss[RB];
+        float wn[RB];
 #pragma unroll
         for (int r = 0; r < RB; ++r) {
-            ss[r] = 0.f;
-#pragma unroll
-            for (int j = 0; j < 2; ++j) {
-                const float mn = a.momentum ? fmaf(beta, mu[r][j], acc[r][j]) : acc[r][j];
-                mu[r][j] = mn;
-                acc[r][j] = 0.f;
-                wn[r][j] = own ? Ws[r * LD + cb + j] - mn : 0.f;
-                ss[r] = fmaf(wn[r][j], wn[r][j], ss[r]);
-            }
+            const float mn = a.momentum ? fmaf(beta, mu[r], acc[r]) : acc[r];
+            mu[r] = mn;
+            acc[r] = 0.f;
+            wn[r] = own ? Ws[r * LD + cb] - mn : 0.f;
         }
         if (a.renorm) {
             // row sums of squares per (matrix, row); a warp may hold columns of both matrices
-            __syncthreads();  // red may still be read by block_sum256 above
+            __syncthreads();  // red may still be read by block_sum_res above
 #pragma unroll
             for (int k = 0; k < 2; ++k)
 #pragma unroll
                 for (int r = 0; r < RB; ++r) {
-                    const float v = warp_sum(kind == k ? ss[r] : 0.f);
+                    const float v = warp_sum(kind == k ? wn[r] * wn[r] : 0.f);
                     if (lane == 0) red[warp * 2 * RB + k * RB + r] = v;
                 }
             __syncthreads();
             if (tid < 2 * RB) {
                 float tot = 0.f;
-                for (int w = 0; w < 8; ++w) tot += red[w * 2 * RB + tid];
+                for (int w = 0; w < NW; ++w) tot += red[w * 2 * RB + tid];
                 scl[tid] = renorm_scale(nS[tid], tot);
             }
             __syncthreads();
@@ -661,17 +650,16 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
         if (own) {
 #pragma unroll
             for (int r = 0; r < RB; ++r) {
-                const float sc = a.renorm ? scl[kind * RB + r] : 1.f;
-                const float w0 = wn[r][0] * sc, w1 = wn[r][1] * sc;
-                finite = finite && isfinite(w0) && isfinite(w1);
-                *reinterpret_cast<float2*>(Ws + r * LD + cb) = make_float2(w0, w1);
+                const float wv = wn[r] * (a.renorm ? scl[kind * RB + r] : 1.f);
+                finite = finite && isfinite(wv);
+                Ws[r * LD + cb] = wv;
             }
         }
         __syncthreads();
     }
     cp_async_wait<0>();
     // write the rows and the momentum back
-    for (int i = tid; i < RB * (D / 4); i += 256) {
+    for (int i = tid; i < RB * (D / 4); i += RES_NT) {
         const int r = i / (D / 4), c = 4 * (i - r * (D / 4));
         const size_t row = (size_t)cs * a.d_hid + h0 + r;
         float* dst = c < a.d_in ? a.W1 + row * a.d_in + c : a.W2 + row * a.d_out + (c - a.d_in);
@@ -681,16 +669,15 @@ __global__ void __launch_bounds__(256) ttl_resident_f32_kernel(const ResArgs a) 
 #pragma unroll
         for (int r = 0; r < RB; ++r) {
             const size_t row = (size_t)cs * a.d_hid + h0 + r;
-            float* dst = kind == 0 ? a.mu1 + row * a.d_in + cb : a.mu2 + row * a.d_out + (cb - a.d_in);
-            *reinterpret_cast<float2*>(dst) = make_float2(mu[r][0], mu[r][1]);
+            (kind == 0 ? a.mu1[row * a.d_in + cb] : a.mu2[row * a.d_out + (cb - a.d_in)]) = mu[r];
         }
     }
     if (!finite) atomicOr(a.status, DEV_NONFINITE);
 }
 
 template <int RB> constexpr size_t res_smem_bytes(int D) {
-    return sizeof(float) *
-           ((size_t)(RB + 2 * RES_RC) * res_ld(D) + RES_RC * 2 * RB + 8 * 2 * RB + 2 * RB + 4 + 4 * RES_RC + 2 * RB);
+    return sizeof(float) * ((size_t)(RB + 2 * RES_RC) * res_ld(D) + RES_RC * 2 * RB + 2 * RES_RC * RB +
+                            RES_NW * 2 * RB + 2 * RB + 4 + 4 * RES_RC + 2 * RB);
 }
 
 // ------------------------------------------------------------------ state upkeep
@@ -951,12 +938,12 @@ cudaError_t launch_resident_f32(const DevState& s, const SegWork& w, long long n
         const size_t bytes = res_smem_bytes<4>(D);
         e = cudaFuncSetAttribute(ttl_resident_f32_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
         if (e != cudaSuccess) return e;
-        ttl_resident_f32_kernel<4><<<dim3(s.d_hid / 4, w.nc), 256, bytes, st>>>(a);
+        ttl_resident_f32_kernel<4><<<dim3(s.d_hid / 4, w.nc), RES_NT, bytes, st>>>(a);
     } else {
         const size_t bytes = res_smem_bytes<8>(D);
         e = cudaFuncSetAttribute(ttl_resident_f32_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
         if (e != cudaSuccess) return e;
-        ttl_resident_f32_kernel<8><<<dim3(s.d_hid / 8, w.nc), 256, bytes, st>>>(a);
+        ttl_resident_f32_kernel<8><<<dim3(s.d_hid / 8, w.nc), RES_NT, bytes, st>>>(a);
     }
     return cudaGetLastError();
 }
