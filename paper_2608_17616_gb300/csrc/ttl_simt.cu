@@ -1,11 +1,11 @@
 // fp32 path of the TTL step, state upkeep kernels and the memory read.
 //
-// When d_in + d_out <= 512 the fp32 path runs every segment of a call in one launch
-// with the rows resident on chip (ttl_resident_f32_kernel, below).  Otherwise it
-// runs two kernels a segment.  Those are latency-bound, so they use plain CUDA-core FFMA tiles (64 x 64 per CTA, 4 x 4 per
-// thread, 64-deep K slabs so that each thread has 32 loads in flight per slab) in fp32
-// throughout.  It computes the same two phases as the bf16
-// tensor-core path:
+// When d_in + d_out <= 512 the fp32 path runs every segment of a call in one launch with
+// the rows resident on chip (ttl_resident_f32_kernel, below).  Otherwise it runs two
+// kernels a segment (three with the squared-error pre-pass).  Those are latency-bound,
+// so they use plain CUDA-core FFMA tiles (64 x 64 per CTA, 4 x 4 per thread, 64-deep K
+// slabs so that each thread has 32 loads in flight per slab) in fp32 throughout, and
+// compute the same two phases as the bf16 tensor-core path:
 //   phase A  H = U W1^T, R = Y W2^T (Y = [K || V]); A = SiLU(H);
 //            dH = c_t R * SiLU'(H), At = c_t A with c_t = -eta_t / T'   (Eq. 10)
 //   phase B  G1 = dH^T U, G2 = At^T Y; mu = beta mu + G; W = s W_raw - mu  (Eq. 8)
