@@ -30,7 +30,7 @@ def config_of(wl: wk.Workload) -> "mone.mone_config":
                             gate_act=mone.MONE_GATE_SILU if wl.gate_act == "silu" else mone.MONE_GATE_LINEAR)
 
 
-class GpuRun:
+class DeviceRun:
     """A live libmone handle for one workload plus its generated device inputs."""
 
     def __init__(self, wl: wk.Workload, n_tokens=None, device="cuda"):
@@ -100,11 +100,11 @@ def gpu_layout(wl: wk.Workload, W: dict):
     return W["W1"], W["W2"]
 
 
-def oracle_meta(run: GpuRun, chain: int):
+def oracle_meta(run: DeviceRun, chain: int):
     return O.Meta.from_torch(run.meta, chain) if run.meta is not None else None
 
 
-def oracle_chain(run: GpuRun, chain: int, n_tokens=None, return_all=False):
+def oracle_chain(run: DeviceRun, chain: int, n_tokens=None, return_all=False):
     """Replay one chain in the oracle from the run's own generated inputs."""
     wl = run.wl
     n = run.N if n_tokens is None else n_tokens
@@ -115,7 +115,7 @@ def oracle_chain(run: GpuRun, chain: int, n_tokens=None, return_all=False):
     return O.ttl_context(st, X, Y, wl.seg_T, oracle_hyper(wl), oracle_meta(run, chain), return_all=return_all)
 
 
-def oracle_read(run: GpuRun, state: O.State, chain: int, Xq):
+def oracle_read(run: DeviceRun, state: O.State, chain: int, Xq):
     wl = run.wl
     ctx, layer = divmod(chain, wl.n_layers)
     return O.generate_kv(state, O.f64(Xq[ctx, layer]), oracle_hyper(wl), oracle_meta(run, chain),

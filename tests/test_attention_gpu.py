@@ -11,7 +11,7 @@ import torch
 import oracle as O
 import paper_2608_17616_gb300 as mone
 import workloads as wk
-from harness import GpuRun, rel_fro
+from harness import DeviceRun, rel_fro
 
 pytestmark = pytest.mark.gpu
 
@@ -30,7 +30,7 @@ def small(mode=wk.PAPER, dtype="bf16", n_ctx=1, n_layers=2, d_out=256, hd=64, N=
 
 
 def run_case(wl, n_q, Lq, n_mem, seed, memory_from_read=True):
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     dt = wl.torch_dtype()
     g = torch.Generator(device="cuda").manual_seed(seed)
@@ -84,7 +84,7 @@ def test_attention_fp32():
 
 def test_attention_argument_errors_launch_nothing():
     wl = small()
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     Kc = torch.zeros(1, 2, wl.n_kv_heads, 16, wl.head_dim, dtype=torch.bfloat16, device="cuda")
     Qt = torch.zeros(1, 2, 2 * wl.n_kv_heads, 4, wl.head_dim, dtype=torch.bfloat16, device="cuda")
     st = Kc.stride()[:4]

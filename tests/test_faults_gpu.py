@@ -10,7 +10,7 @@ import torch
 
 import paper_2608_17616_gb300 as mone
 import workloads as wk
-from harness import GpuRun, config_of
+from harness import DeviceRun, config_of
 
 pytestmark = pytest.mark.gpu
 
@@ -46,7 +46,7 @@ def test_injected_allocation_failure_reports_oom_and_leaks_nothing():
 
 def test_freed_handle_is_rejected():
     wl = small()
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     h = run.h
     mone.mone_mem_free(h)
     run.h = None
@@ -57,7 +57,7 @@ def test_freed_handle_is_rejected():
 
 def test_argument_errors_launch_nothing():
     wl = small()
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     before = mone.mone_mem_launch_count(run.h)
     x = run.X[0, 0]
     assert code_of(mone.mone_ttl_segment, run.h, 0, 0, x, run.K[0, 0], run.V[0, 0], wl.seg_T + 1) == 1
@@ -76,7 +76,7 @@ def test_argument_errors_launch_nothing():
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 def test_nonfinite_weight_is_latched_and_the_handle_recovers(dtype):
     wl = small(dtype=dtype)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     X = run.X.clone()
     X[0, 1, 3, 5] = float("nan")
     mone.mone_ttl_context(run.h, X, run.K, run.V, wl.N)

@@ -12,7 +12,7 @@ import torch
 import oracle as O
 import paper_2608_17616_gb300 as mone
 import workloads as wk
-from harness import GpuRun, gpu_layout, oracle_chain, oracle_hyper, oracle_meta, oracle_read, rel_fro
+from harness import DeviceRun, gpu_layout, oracle_chain, oracle_hyper, oracle_meta, oracle_read, rel_fro
 
 pytestmark = pytest.mark.gpu
 
@@ -50,7 +50,7 @@ def check_chain(run, chain, W1, W2, tol, n_tokens=None):
 
 def test_tiny_f32_per_step_parity_and_loss():
     wl = wk.WORKLOADS["tiny_f32"]
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     _, losses, trail = oracle_chain(run, 0, return_all=True)
     loss_dev = torch.zeros(1, device="cuda")
     T = wl.seg_T
@@ -67,10 +67,10 @@ def test_tiny_f32_per_step_parity_and_loss():
 
 def test_tiny_f32_context_equals_segment_loop_and_read():
     wl = wk.WORKLOADS["tiny_f32"]
-    a = GpuRun(wl)
+    a = DeviceRun(wl)
     a.ttl_context()
     W1a, W2a, _, _ = a.state()
-    b = GpuRun(wl)
+    b = DeviceRun(wl)
     T = wl.seg_T
     for s in range(wl.S):
         sl = slice(s * T, (s + 1) * T)
@@ -89,7 +89,7 @@ def test_tiny_f32_context_equals_segment_loop_and_read():
 
 def test_f32_paper_mode_ragged():
     wl = small(wk.PAPER, "f32", T=128, N=3 * 128 + 50, d_in=128, d_hid=192, d_out=256, lr=0.5)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, mu1, mu2 = run.state()
     for c in range(wl.chains):
@@ -111,7 +111,7 @@ def launches(run, kind):
 def test_f32_mse_per_step_parity_and_loss():
     # the squared-error (delta-rule) variant on the fp32 path: per-step weights and loss at 1e-4
     wl = wk.WORKLOADS["tiny_f32"].replace(loss="mse", N=8 * 128)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     _, losses, trail = oracle_chain(run, 0, return_all=True)
     loss_dev = torch.zeros(1, device="cuda")
     T = wl.seg_T
@@ -128,7 +128,7 @@ def test_f32_mse_per_step_parity_and_loss():
 
 def test_f32_mse_paper_ragged():
     wl = small(wk.PAPER, "f32", T=128, N=3 * 128 + 50, d_in=128, d_hid=192, d_out=256).replace(loss="mse")
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, mu1, mu2 = run.state()
     Xq = wk.query_inputs(wl, "cuda")
@@ -144,7 +144,7 @@ def test_f32_mse_paper_ragged():
 def test_f32_tiled_path_paper_ragged():
     # d_in + d_out > 512: the rows stay in HBM and the per-segment fp32 phase kernels run
     wl = small(wk.PAPER, "f32", n_ctx=1, T=64, N=3 * 64 + 20, d_in=512, d_hid=128, d_out=256, lr=0.5)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     mone.mone_mem_set_timing(run.h, 1)
     run.ttl_context()
     assert launches(run, "resident") == 0 and launches(run, "phase_a") == wl.S
@@ -158,7 +158,7 @@ def test_f32_tiled_path_paper_ragged():
 def test_f32_resident_segment_caller_rates_and_loss():
     # a partial segment of one chain with caller rates and the loss output, on the resident kernel
     wl = small(wk.PLAIN, "f32", n_ctx=1, n_layers=3, T=128, N=128)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     mone.mone_mem_set_timing(run.h, 1)
     eta = wk.token_lr(wl, 1, 100, "cuda")
     loss = torch.zeros(1, device="cuda")
@@ -182,7 +182,7 @@ def test_f32_resident_two_input_windows():
     # launch per window, the state handed from the first to the second through HBM
     wl = small(wk.PAPER, "f32", n_ctx=1, n_layers=2, T=64, N=64 * 64 + 64 + 40, d_in=64, d_hid=64, d_out=128,
                lr=0.5)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     mone.mone_mem_set_timing(run.h, 1)
     run.ttl_context()
     assert launches(run, "resident") == 2 and launches(run, "prepass") == 2
@@ -204,7 +204,7 @@ def test_output_channel_renorm_parity(dtype, loss):
         wl = small(wk.PAPER, "f32", T=128, N=3 * 128 + 50, d_in=128, d_hid=192, d_out=256,
                    lr=0.5).replace(renorm_axis="out", loss=loss)
     tol = F32_TOL if dtype == "f32" else BF16_TOL
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     mone.mone_mem_set_timing(run.h, 1)
     run.ttl_context()
     assert launches(run, "resident") == 0
@@ -230,7 +230,7 @@ def test_silu_gate_read_parity(dtype, mode):
     else:
         wl = small(mode, "f32", T=128, N=2 * 128 + 10, d_in=128, d_hid=192, d_out=256).replace(gate_act="silu")
     tol = F32_TOL if dtype == "f32" else BF16_TOL
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     Xq = wk.query_inputs(wl, "cuda")
     Kg, Vg = run.generate_kv(Xq)
@@ -253,7 +253,7 @@ def test_context_over_several_input_windows(dtype, loss):
     else:
         wl = small(wk.PAPER, "f32", n_ctx=1, T=64, N=2 * 64 * 64 + 100, d_in=512, d_hid=128, d_out=256, lr=0.5)
     tol = F32_TOL if dtype == "f32" else BF16_TOL
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     mone.mone_mem_set_timing(run.h, 1)
     run.ttl_context()
     assert launches(run, "prepass") == -(-wl.S // 64)
@@ -273,7 +273,7 @@ def test_zero_learning_rate_leaves_the_weights_bit_identical(dtype, shape):
     # plain mode with lr = 0: every gradient is exactly zero, so W comes back bit for bit (bf16
     # path, fp32 resident kernel, fp32 tiled kernels)
     wl = small(wk.PLAIN, dtype, lr=0.0, **shape)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, _, _ = run.state()
     assert torch.equal(W1, run.W1_0.cpu()) and torch.equal(W2, run.W2_0.cpu())
@@ -286,7 +286,7 @@ def test_zero_caller_rates_in_paper_mode_keep_the_state(dtype):
     # rounding of the renormalisation scale (n0 / |row|, both fp32 sums of the same row)
     n = 200 if dtype == "bf16" else 100  # one partial segment (T = 256 / 128)
     wl = _edge_small(dtype, n_ctx=1, T=256 if dtype == "bf16" else 128, N=n)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     eta = torch.zeros(n, device="cuda")
     mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, :n], run.K[0, 1, :n], run.V[0, 1, :n], n, eta)
     mone.mone_mem_sync(run.h)
@@ -308,7 +308,7 @@ def _edge_small(dtype, **kw):
 def test_context_shorter_than_a_segment_then_a_one_token_segment(dtype):
     wl = _edge_small(dtype, n_ctx=1, T=256 if dtype == "bf16" else 128, N=37)
     tol = F32_TOL if dtype == "f32" else BF16_TOL
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()                                        # one partial segment: T' = 37
     W1, W2, _, _ = run.state()
     for c in range(wl.chains):
@@ -330,7 +330,7 @@ def test_largest_segment_T4096_ragged(dtype):
     # d_in = d_out = 256 phase B runs on CTA pairs, on fp32 the resident kernel streams 128 chunks
     wl = _edge_small(dtype, n_ctx=1, T=4096, N=4096 + 300)
     tol = F32_TOL if dtype == "f32" else BF16_TOL
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, _, _ = run.state()
     for c in range(wl.chains):
@@ -342,7 +342,7 @@ def test_largest_segment_T4096_ragged(dtype):
 def test_generate_kv_largest_query_4096(dtype):
     wl = _edge_small(dtype, n_ctx=1, n_layers=1, T=256 if dtype == "bf16" else 128, N=300, Q=4096)
     tol = F32_TOL if dtype == "f32" else BF16_TOL
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     Xq = wk.query_inputs(wl, "cuda")
     assert Xq.shape[2] == 4096
@@ -358,7 +358,7 @@ def test_generate_kv_largest_query_4096(dtype):
 @pytest.mark.parametrize("mode", [wk.PLAIN, wk.PAPER])
 def test_bf16_small_context_parity(mode):
     wl = small(mode)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, mu1, mu2 = run.state()
     Xq = wk.query_inputs(wl, "cuda")
@@ -373,7 +373,7 @@ def test_bf16_small_context_parity(mode):
 
 def test_bf16_segment_with_caller_rates_and_loss():
     wl = small(wk.PLAIN, n_ctx=1, n_layers=3, N=256)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     eta = wk.token_lr(wl, 1, 200, "cuda")
     loss = torch.zeros(1, device="cuda")
     mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, :200], run.K[0, 1, :200], run.V[0, 1, :200], 200, eta, loss)
@@ -394,9 +394,9 @@ def test_bf16_segment_with_caller_rates_and_loss():
 
 def test_bf16_context_split_equals_whole():
     wl = small(wk.PAPER, N=6 * 256)
-    a = GpuRun(wl)
+    a = DeviceRun(wl)
     a.ttl_context()
-    b = GpuRun(wl)
+    b = DeviceRun(wl)
     n1 = 2 * 256
     X1, K1, V1 = (t[:, :, :n1].contiguous() for t in (b.X, b.K, b.V))
     X2, K2, V2 = (t[:, :, n1:].contiguous() for t in (b.X, b.K, b.V))
@@ -412,11 +412,11 @@ def test_bf16_context_split_equals_whole():
 
 def test_bf16_layer_permutation_permutes_results():
     wl = small(wk.PAPER, n_ctx=1, n_layers=4, N=512)
-    a = GpuRun(wl)
+    a = DeviceRun(wl)
     a.ttl_context()
     W1a, W2a, _, _ = a.state()
     perm = [2, 0, 3, 1]
-    b = GpuRun(wl)
+    b = DeviceRun(wl)
     mone.mone_mem_free(b.h)
     meta = {k: v[perm].contiguous() for k, v in a.meta.items()}
     from harness import config_of
@@ -437,7 +437,7 @@ def test_bf16_chain_groups_match_one_chain_handles(mode):
     # input-transform windows exist only in paper mode
     N = 2 * 64 * 128 + 300 if mode == wk.PAPER else 5 * 128 + 50
     wl = small(mode, n_ctx=1, n_layers=3, T=128, N=N)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, mu1, mu2 = run.state()
     from harness import config_of
@@ -467,7 +467,7 @@ def test_bf16_generate_kv_several_query_tiles(Q, hd):
     """The tensor-core read takes queries 128 at a time: Q > 128 spans several tiles and a
     ragged last one (rows beyond Q are never written); hd = 128 puts one head per tile."""
     wl = small(wk.PAPER, n_ctx=1, n_layers=2, d_out=512, N=300, hd=hd, Q=Q)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, _, _ = run.state()
     Xq = wk.query_inputs(wl, "cuda")
@@ -482,7 +482,7 @@ def test_bf16_generate_kv_several_query_tiles(Q, hd):
 
 def test_generate_kv_into_strided_cache_and_reuse():
     wl = small(wk.PAPER, N=512)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     Q, off, S_tot = wl.Q, 7, wl.Q + 19
     Xq = wk.query_inputs(wl, "cuda")
@@ -506,7 +506,7 @@ def test_replayed_read_matches_the_launched_one_and_follows_the_state(dtype):
     # equals the first (launched) read bit for bit, and after more learning it reads the new state
     wl = _edge_small(dtype, n_ctx=1, T=256 if dtype == "bf16" else 128, N=4 * (256 if dtype == "bf16" else 128) + 9)
     tol = F32_TOL if dtype == "f32" else BF16_TOL
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     n1 = 2 * wl.seg_T
     X1, K1, V1 = (t[:, :, :n1].contiguous() for t in (run.X, run.K, run.V))
     X2, K2, V2 = (t[:, :, n1:].contiguous() for t in (run.X, run.K, run.V))
@@ -541,7 +541,7 @@ def test_bf16_pair_phase_b_context_parity(mode, loss, lr):
     """From T = 1024 on, phase B runs on CTA pairs (256 columns x 256 hidden rows): 2 segments
     and a ragged tail, 3 chains in two groups (2 + 1)."""
     wl = small(mode, n_ctx=1, n_layers=3, T=1024, N=2 * 1024 + 300, lr=lr).replace(loss=loss)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, mu1, mu2 = run.state()
     Xq = wk.query_inputs(wl, "cuda")
@@ -558,7 +558,7 @@ def test_bf16_pair_phase_b_context_parity(mode, loss, lr):
 def test_bf16_pair_phase_b_one_chain_segment():
     """A one-chain call (one group) through the pair kernel, with caller rates and the loss."""
     wl = small(wk.PLAIN, n_ctx=1, n_layers=2, T=1024, N=1024)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     eta = wk.token_lr(wl, 1, 900, "cuda")
     loss = torch.zeros(1, device="cuda")
     mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, :900], run.K[0, 1, :900], run.V[0, 1, :900], 900, eta, loss)
@@ -582,7 +582,7 @@ def test_bf16_mse_context_parity(mode, lr):
     """Loss 1/2 |M(u) - y|^2: the pre-pass forms y - M(u) at the segment's starting weights,
     then the same two phases run on it; 4 segments + a ragged tail, 4 chains in two groups."""
     wl = small(mode, lr=lr).replace(loss="mse")
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, mu1, mu2 = run.state()
     Xq = wk.query_inputs(wl, "cuda")
@@ -599,7 +599,7 @@ def test_bf16_mse_context_parity(mode, lr):
 
 def test_bf16_mse_segment_with_caller_rates_and_loss():
     wl = small(wk.PLAIN, n_ctx=1, n_layers=3, N=256, lr=0.01).replace(loss="mse")
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     eta = wk.token_lr(wl, 1, 200, "cuda")
     loss = torch.zeros(1, device="cuda")
     mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, :200], run.K[0, 1, :200], run.V[0, 1, :200], 200, eta, loss)
@@ -619,7 +619,7 @@ def test_bf16_mse_segment_with_caller_rates_and_loss():
 
 def test_bf16_mse_chain_groups_match_one_chain_handles():
     wl = small(wk.PAPER, n_ctx=1, n_layers=3, T=128, N=2 * 64 * 128 + 300).replace(loss="mse")
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     W1, W2, _, _ = run.state()
     from harness import config_of
@@ -656,7 +656,7 @@ def test_bf16_mse_chain_groups_match_one_chain_handles():
 ])
 def test_full_size_sampled_chains(name, chains, n_tokens, loss):
     wl = wk.WORKLOADS[name].replace(loss=loss)
-    run = GpuRun(wl, n_tokens=n_tokens)
+    run = DeviceRun(wl, n_tokens=n_tokens)
     run.ttl_context()
     W1, W2, _, _ = run.state()
     Xq = wk.query_inputs(wl, "cuda")

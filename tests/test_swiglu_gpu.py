@@ -9,7 +9,7 @@ import torch
 import oracle as O
 import paper_2608_17616_gb300 as mone
 import workloads as wk
-from harness import GpuRun, gpu_layout, oracle_chain, oracle_init, oracle_read, rel_fro
+from harness import DeviceRun, gpu_layout, oracle_chain, oracle_init, oracle_read, rel_fro
 
 pytestmark = pytest.mark.gpu
 
@@ -51,7 +51,7 @@ def check(run, chains, Xq=None):
 def test_swiglu_small_paper_mode_ragged_hidden_tiles():
     # 2 heads of 128, 96 hidden units (one hidden tile, 32 rows past F), 3 segments + a ragged tail
     wl = swiglu(n_ctx=2)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     check(run, range(wl.chains), wk.query_inputs(wl, "cuda"))
     run.close()
@@ -61,7 +61,7 @@ def test_swiglu_context_over_several_input_windows():
     # 64 segments a window: 3 full windows and a ragged fourth, each transformed after both
     # chain groups are done with the previous one
     wl = swiglu(n_ctx=1, N=3 * 64 * 128 + 70)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     mone.mone_mem_set_timing(run.h, 1)
     run.ttl_context()
     assert mone.mone_mem_kernel_time(run.h, mone.KERNEL_KINDS.index("prepass"))[1] == 4
@@ -72,7 +72,7 @@ def test_swiglu_context_over_several_input_windows():
 def test_swiglu_read_with_silu_gate():
     # the read scales head h by SiLU(g_h) (the other reading of the gate), on the SwiGLU memory too
     wl = swiglu(n_ctx=1).replace(gate_act="silu")
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     check(run, range(wl.chains), wk.query_inputs(wl, "cuda"))
     run.close()
@@ -82,7 +82,7 @@ def test_swiglu_paper_head_shape():
     # the paper's head shape: d = 896 as 4 heads of 224, 224 hidden units (k-blocks and hidden tiles
     # both run past 224), K || V = 2 x 7 heads of 64
     wl = swiglu(d=896, heads=4, F=224, n_kv=7, T=512, N=2 * 512 + 37, n_layers=3)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     check(run, range(wl.chains), wk.query_inputs(wl, "cuda"))
     run.close()
@@ -90,7 +90,7 @@ def test_swiglu_paper_head_shape():
 
 def test_swiglu_plain_mode():
     wl = swiglu(mode=wk.PLAIN, lr=0.05, N=2 * 128 + 17)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     check(run, range(wl.chains), wk.query_inputs(wl, "cuda"))
     run.close()
@@ -98,7 +98,7 @@ def test_swiglu_plain_mode():
 
 def test_swiglu_segment_with_caller_rates_and_loss():
     wl = swiglu(mode=wk.PLAIN, n_layers=3, lr=0.05, N=128)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     eta = wk.token_lr(wl, 1, 100, "cuda")
     loss = torch.zeros(1, device="cuda")
     mone.mone_ttl_segment(run.h, 0, 1, run.X[0, 1, :100], run.K[0, 1, :100], run.V[0, 1, :100], 100, eta, loss)
@@ -119,7 +119,7 @@ def test_swiglu_segment_with_caller_rates_and_loss():
 
 def test_swiglu_full_size_sampled_chains():
     wl = wk.WORKLOADS["swiglu_l24_d896_32k"]
-    run = GpuRun(wl, n_tokens=8192)
+    run = DeviceRun(wl, n_tokens=8192)
     run.ttl_context()
     check(run, (0, 23), wk.query_inputs(wl, "cuda"))
     run.close()

@@ -15,7 +15,7 @@ import torch
 
 import paper_2608_17616_gb300 as mone
 import workloads as wk
-from harness import GpuRun, rel_fro
+from harness import DeviceRun, rel_fro
 
 pytestmark = pytest.mark.gpu
 
@@ -37,7 +37,7 @@ def outputs(wl, Q, dtype):
 @pytest.mark.parametrize("dtype,mode", [("bf16", wk.PAPER), ("f32", wk.PLAIN)])
 def test_noalloc_read_matches_the_allocating_read_twice(dtype, mode):
     wl = wk.Workload(f"noalloc_{dtype}", 30 + mode, 2, 2, 256, 256, 256, 2, 64, 256, 512 + 77, 40, dtype, mode, 0.3)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     run.ttl_context()
     Xq = wk.query_inputs(wl, "cuda")
     strides = mone.kv_strides(wl.n_layers, wl.n_kv_heads, wl.Q, wl.head_dim)
@@ -55,7 +55,7 @@ def test_noalloc_read_matches_the_allocating_read_twice(dtype, mode):
 
 def test_noalloc_read_rejects_work_beyond_its_scratch():
     wl = wk.Workload("noalloc_big", 32, 1, 4, 256, 256, 256, 2, 64, 256, 256, 4096, "bf16", wk.PLAIN, 0.3)
-    run = GpuRun(wl)
+    run = DeviceRun(wl)
     Xq = torch.zeros(wl.n_ctx, wl.n_layers, wl.Q, wl.d_in, dtype=torch.bfloat16, device="cuda")
     K, V = outputs(wl, wl.Q, Xq.dtype)
     arr = (ctypes.c_longlong * 4)(*mone.kv_strides(wl.n_layers, wl.n_kv_heads, wl.Q, wl.head_dim))
