@@ -66,6 +66,11 @@ a zero output at g = 0), the read of a linear memory against brute force, and
 the chain identities (context = loop of segments = split contexts), and the
 consumer attention against its special cases (one visible key returns its
 value, equal keys average the visible values, causality, grouped heads).
+The data-dependent terms of R3 are pinned too: the rates and the decay against
+explicit loops over tokens and features (nonzero w_eta, w_beta), and two
+paper-mode segments of a linear memory against the same loops, so a rate taken
+from u instead of x, or a decay pooled by a sum, the last token or the wrong
+axis, fails.
 Parity unpinned: the exact numbers of the paper-mode readings R3, R6, R7
 (their forms are the build's reading; only the invariants above constrain
 them).

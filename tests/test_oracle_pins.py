@@ -354,6 +354,147 @@ def test_token_rate_and_decay_special_cases():
     assert O.momentum_decay(X, O.Hyper(mode=O.PLAIN), meta) == 0.0
 
 
+def _rates_by_loop(X, meta):
+    """eta_j = ln(1 + exp(sum_i w_i x_ji + b)) for every token j, by explicit loops."""
+    out = []
+    for j in range(X.shape[0]):
+        z = meta.b_eta
+        for i in range(X.shape[1]):
+            z += meta.w_eta[i] * X[j, i]
+        out.append(math.log1p(math.exp(z)))
+    return np.array(out)
+
+
+def _decay_by_loop(X, meta):
+    """beta = 1 / (1 + exp(-(sum_i w_i (1/T') sum_j x_ji + b))), by explicit loops."""
+    n, d = X.shape
+    z = meta.b_beta
+    for i in range(d):
+        col = 0.0
+        for j in range(n):
+            col += X[j, i]
+        z += meta.w_beta[i] * (col / n)
+    return 1.0 / (1.0 + math.exp(-z))
+
+
+def _transform_by_loop(X, meta):
+    """u_j = z_j / sqrt(|z_j|^2 + 1e-12), z_ji = SiLU(alpha_i x_ji + gamma_i), by explicit loops."""
+    U = np.empty_like(X)
+    for j in range(X.shape[0]):
+        z = []
+        for i in range(X.shape[1]):
+            a = meta.alpha[i] * X[j, i] + meta.gamma[i]
+            z.append(a / (1.0 + math.exp(-a)))
+        nrm = math.sqrt(sum(v * v for v in z) + 1e-12)
+        for i in range(X.shape[1]):
+            U[j, i] = z[i] / nrm
+    return U
+
+
+def _rate_inputs(seed):
+    """Tokens with a clearly nonzero mean, so that a mean, a sum and a last token all differ,
+    and meta-parameters whose data terms (w_eta . x, w_beta . mean x) are far from zero."""
+    r = rng(seed)
+    T, d = 6, 5
+    X = 0.8 + r.standard_normal((T, d))
+    meta = rand_meta(r, d, lr=0.05)
+    meta.w_eta = 0.9 * r.standard_normal(d)
+    meta.b_eta = 0.3
+    meta.w_beta = 0.8 * r.standard_normal(d)
+    meta.b_beta = -0.4
+    return X, meta
+
+
+def _pin_rates_and_decay():
+    X, meta = _rate_inputs(40)
+    hp = O.Hyper(mode=O.PAPER)
+    rates = O.mone_oracle.token_rates(X, hp, meta)
+    ref = _rates_by_loop(X, meta)
+    assert rates.shape == ref.shape
+    np.testing.assert_allclose(rates, ref, rtol=1e-13, atol=0)
+    assert abs(O.mone_oracle.momentum_decay(X, hp, meta) - _decay_by_loop(X, meta)) < 1e-14
+
+
+def _pin_two_segment_linear_memory():
+    """Two paper-mode segments of a linear memory under Eq. 7, whose gradient does not
+    depend on W: G_s = -(1/T) sum_j eta_sj y_sj u_sj^T, mu_1 = G_1, mu_2 = beta_2 mu_1 + G_2,
+    W_s = W_{s-1} - mu_s (Eq. 8, App. A momentum).  Rates and decay come from the raw
+    tokens x, the memory input from u = phi(x), each computed by loops."""
+    X1, meta = _rate_inputs(41)
+    r = rng(42)
+    T, d = X1.shape
+    X2 = -0.5 + 1.3 * r.standard_normal((T, d))
+    Y1, Y2 = r.standard_normal((T, 3)), r.standard_normal((T, 3))
+    W0 = r.standard_normal((3, d))
+    hp = O.Hyper(mode=O.PAPER, memory="linear", renorm=False)
+    st, _ = O.mone_oracle.ttl_context(O.init_state(W=W0), np.concatenate([X1, X2]), np.concatenate([Y1, Y2]), T,
+                                      hp, meta)
+    W, mu = W0.copy(), np.zeros_like(W0)
+    for X, Y in ((X1, Y1), (X2, Y2)):
+        U, eta, beta = _transform_by_loop(X, meta), _rates_by_loop(X, meta), _decay_by_loop(X, meta)
+        G = np.zeros_like(W0)
+        for j in range(T):
+            for o in range(3):
+                for i in range(d):
+                    G[o, i] -= eta[j] * Y[j, o] * U[j, i] / T
+        mu = beta * mu + G
+        W = W - mu
+    np.testing.assert_allclose(st.mu["W"], mu, rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(st.W["W"], W, rtol=1e-12, atol=1e-15)
+
+
+def test_token_rates_and_decay_by_loops():
+    """Data-dependent terms of App. A's rate and decay (R3) element by element."""
+    _pin_rates_and_decay()
+
+
+def test_paper_mode_two_segments_of_a_linear_memory_by_loops():
+    _pin_two_segment_linear_memory()
+
+
+def _rates_from_u(X, hp, meta, eta=None):
+    if eta is not None:
+        return O.f64(eta)
+    return O.softplus(O.transform_inputs(X, hp, meta) @ meta.w_eta + meta.b_eta)
+
+
+def _rates_without_softplus(X, hp, meta, eta=None):
+    if eta is not None:
+        return O.f64(eta)
+    return O.f64(X) @ meta.w_eta + meta.b_eta
+
+
+def _decay_from_sum(X, hp, meta):
+    return float(O.sigmoid(np.sum(O.f64(X), axis=0) @ meta.w_beta + meta.b_beta))
+
+
+def _decay_from_last_token(X, hp, meta):
+    return float(O.sigmoid(O.f64(X)[-1] @ meta.w_beta + meta.b_beta))
+
+
+def _decay_from_u(X, hp, meta):
+    return float(O.sigmoid(np.mean(O.transform_inputs(X, hp, meta), axis=0) @ meta.w_beta + meta.b_beta))
+
+
+def _decay_wrong_axis(X, hp, meta):
+    return float(O.sigmoid(np.mean(O.f64(X), axis=1) @ meta.w_beta[:X.shape[0]] + meta.b_beta))
+
+
+@pytest.mark.parametrize("name,slip", [
+    ("token_rates", _rates_from_u), ("token_rates", _rates_without_softplus),
+    ("momentum_decay", _decay_from_sum), ("momentum_decay", _decay_from_last_token),
+    ("momentum_decay", _decay_from_u), ("momentum_decay", _decay_wrong_axis)])
+def test_planted_rate_and_decay_slips_fail_both_pins(monkeypatch, name, slip):
+    """A plausible slip in the rate or the decay (the transformed u in place of x, a sum or
+    the last token in place of the mean, the wrong pooling axis, a missing softplus),
+    planted in the oracle, fails the direct pin and the two-segment pin."""
+    monkeypatch.setattr(O.mone_oracle, name, slip)
+    with pytest.raises((AssertionError, ValueError)):
+        _pin_rates_and_decay()
+    with pytest.raises((AssertionError, ValueError)):
+        _pin_two_segment_linear_memory()
+
+
 # ----------------------------------------------------------------- chain (Eq. 9)
 
 def test_context_split_and_segment_loop_agree():
