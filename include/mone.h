@@ -186,9 +186,12 @@ mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out
  * mone_mem_generate_kv may allocate read scratch on its first call or when Q
  * grows; this variant instead uses one fixed 16 MiB device array compiled into
  * the library (every GPU that loads the library holds it until the process
- * exits).  Same arguments, outputs and error behaviour as mone_mem_generate_kv,
- * plus MONE_ERR_UNSUPPORTED_SHAPE when chains * Q * (d_in + d_hid + d_out) exceeds
- * 4,194,304 floats (the size is checked before any work; mone_last_error says why).
+ * exits).  Same arguments and outputs as mone_mem_generate_kv (bit for bit: the
+ * same kernels on the same inputs), and its errors plus two of its own, both
+ * returned before any GPU work with mone_last_error saying why:
+ * MONE_ERR_UNSUPPORTED_SHAPE when chains * Q * (d_in + d_hid + d_out) exceeds
+ * 4,194,304 floats, and MONE_ERR_UNSUPPORTED for a SwiGLU-memory handle
+ * (MONE_MEM_SWIGLU), whose read has no fixed-scratch variant.
  * It calls no cudaMalloc, cudaFree or allocating library routine.
  * The first call on a device resolves the array's device address
  * (cudaGetSymbolAddress) with that device current; make that first call before

@@ -20,6 +20,26 @@ def rel_fro(a, b) -> float:
     return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
 
 
+# Observed errors of every parity check of this session: (check, key, value, bound), printed
+# at the end of the run (tests/conftest.py) so that the margins under each bound are visible.
+MARGINS: list = []
+
+
+def record(check: str, key: str, value: float, bound: float) -> float:
+    MARGINS.append((check, key, float(value), float(bound)))
+    return value
+
+
+def row_rel_errors(a, b, floor=1e-6):
+    """Per-row relative error |a_r - b_r| / |b_r| over the last axis (leading axes flattened);
+    rows whose reference norm is below `floor` x the largest are skipped (nothing moved there)."""
+    a = np.asarray(a, dtype=np.float64).reshape(-1, np.shape(a)[-1])
+    b = np.asarray(b, dtype=np.float64).reshape(-1, np.shape(b)[-1])
+    nb = np.linalg.norm(b, axis=1)
+    keep = nb > floor * max(nb.max(), 1e-300)
+    return np.linalg.norm(a - b, axis=1)[keep] / nb[keep]
+
+
 def config_of(wl: wk.Workload) -> "mone.mone_config":
     return mone.make_config(wl.n_ctx, wl.n_layers, wl.d_in, wl.d_hid, wl.d_out, wl.n_kv_heads, wl.head_dim,
                             wl.seg_T, mone.MONE_FP32 if wl.dtype == "f32" else mone.MONE_BF16, wl.mode, wl.lr,

@@ -12,7 +12,8 @@ import torch
 import oracle as O
 import paper_2608_17616_gb300 as mone
 import workloads as wk
-from harness import DeviceRun, gpu_layout, oracle_chain, oracle_hyper, oracle_meta, oracle_read, rel_fro
+from harness import (DeviceRun, gpu_layout, oracle_chain, oracle_hyper, oracle_meta, oracle_read, record, rel_fro,
+                     row_rel_errors)
 
 pytestmark = pytest.mark.gpu
 
@@ -34,16 +35,36 @@ def small(mode, dtype="bf16", n_ctx=2, n_layers=2, d_in=256, d_hid=256, d_out=25
                        T, N, Q, dtype, mode, lr)
 
 
+# Per hidden row, the relative error of the weight change W_S - W_0 (a few rows off, such as
+# one mis-scaled 128-row tile, move the whole-matrix figure very little).
+ROW_DW_TOL = {F32_TOL: 1e-2, BF16_TOL: 1e-1}
+# The momentum is the last step, far smaller than W; the same absolute rounding is a larger
+# fraction of it than of W.
+MU_TOL = 1e-3
+
+
 def check_chain(run, chain, W1, W2, tol, n_tokens=None):
     st, _ = oracle_chain(run, chain, n_tokens)
     o1, o2 = gpu_layout(run.wl, st.W)
-    e1 = rel_fro(W1[chain], o1)
-    e2 = rel_fro(W2[chain], o2)
-    d1 = rel_fro(W1[chain].double() - run.W1_0[chain].cpu().double(), o1 - O.f64(run.W1_0[chain]))
-    d2 = rel_fro(W2[chain].double() - run.W2_0[chain].cpu().double(), o2 - O.f64(run.W2_0[chain]))
+    name = "f32" if tol == F32_TOL else "bf16"
+    e1 = record(name, "W1", rel_fro(W1[chain], o1), tol)
+    e2 = record(name, "W2", rel_fro(W2[chain], o2), tol)
+    w01, w02 = O.f64(run.W1_0[chain]), O.f64(run.W2_0[chain])
+    g1, g2 = W1[chain].double().numpy() - w01, W2[chain].double().numpy() - w02
+    d1 = record(name, "dW1", rel_fro(g1, o1 - w01), max(tol, 5e-2))
+    d2 = record(name, "dW2", rel_fro(g2, o2 - w02), max(tol, 5e-2))
+    r1 = record(name, "dW1 row", row_rel_errors(g1, o1 - w01).max(), ROW_DW_TOL[tol])
+    r2 = record(name, "dW2 row", row_rel_errors(g2, o2 - w02).max(), ROW_DW_TOL[tol])
     assert e1 <= tol and e2 <= tol, (chain, e1, e2)
     assert d1 <= max(tol, 5e-2) and d2 <= max(tol, 5e-2), (chain, d1, d2)
+    assert r1 <= ROW_DW_TOL[tol] and r2 <= ROW_DW_TOL[tol], (chain, r1, r2)
     return st
+
+
+def check_mu(mu1, mu2, c, st, tol=MU_TOL):
+    m1 = record("f32" if tol == MU_TOL else "bf16", "mu1", rel_fro(mu1[c], st.mu["W1"]), tol)
+    m2 = record("f32" if tol == MU_TOL else "bf16", "mu2", rel_fro(mu2[c], st.mu["W2"]), tol)
+    assert m1 <= tol and m2 <= tol, (c, m1, m2)
 
 
 # ----------------------------------------------------------------- fp32 path (tiny workload)
@@ -94,7 +115,7 @@ def test_f32_paper_mode_ragged():
     W1, W2, mu1, mu2 = run.state()
     for c in range(wl.chains):
         st = check_chain(run, c, W1, W2, F32_TOL)
-        assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+        check_mu(mu1, mu2, c, st)
     Xq = wk.query_inputs(wl, "cuda")
     Kg, Vg = run.generate_kv(Xq)
     for c in range(wl.chains):
@@ -135,7 +156,7 @@ def test_f32_mse_paper_ragged():
     Kg, Vg = run.generate_kv(Xq)
     for c in range(wl.chains):
         st = check_chain(run, c, W1, W2, F32_TOL)
-        assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+        check_mu(mu1, mu2, c, st)
         Ko, Vo = oracle_read(run, st, c, Xq)
         assert rel_fro(Kg[c // 2, c % 2], Ko) <= F32_TOL and rel_fro(Vg[c // 2, c % 2], Vo) <= F32_TOL
     run.close()
@@ -151,7 +172,7 @@ def test_f32_tiled_path_paper_ragged():
     W1, W2, mu1, mu2 = run.state()
     for c in range(wl.chains):
         st = check_chain(run, c, W1, W2, F32_TOL)
-        assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+        check_mu(mu1, mu2, c, st)
     run.close()
 
 
@@ -189,7 +210,7 @@ def test_f32_resident_two_input_windows():
     W1, W2, mu1, mu2 = run.state()
     for c in range(wl.chains):
         st = check_chain(run, c, W1, W2, F32_TOL)
-        assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+        check_mu(mu1, mu2, c, st)
     run.close()
 
 
@@ -261,7 +282,7 @@ def test_context_over_several_input_windows(dtype, loss):
     for c in range(wl.chains):
         st = check_chain(run, c, W1, W2, tol)
         if dtype == "f32":
-            assert rel_fro(mu1[c], st.mu["W1"]) <= 1e-3 and rel_fro(mu2[c], st.mu["W2"]) <= 1e-3
+            check_mu(mu1, mu2, c, st)
     run.close()
 
 
