@@ -122,6 +122,84 @@ def kernel_work(wl, kind, chains=None):
     return flops, byts
 
 
+def e2e_breakdown(ev, h2d_bytes, chunk_tensors):
+    """Where the end-to-end step's time goes: per chunk, its host-to-device copy and its learning
+    (CUDA events on the copy stream and the learning stream), and the achieved copy rate, so a
+    slow host link can be told apart from a stall of the pipeline.  `ev[step][chunk]` holds the
+    events (copy start, copy end, learning start, learning end)."""
+    chunk_bytes = sum(t.numel() * t.element_size() for t in chunk_tensors)
+    copy_ms = [[c0.elapsed_time(c1) for c0, c1, _, _ in st] for st in ev]
+    learn_ms = [[l0.elapsed_time(l1) for _, _, l0, l1 in st] for st in ev]
+    # learning of chunk k waiting for its copy: start of learning k minus end of learning k-1
+    wait_ms = [[max(0.0, st[k - 1][3].elapsed_time(st[k][2])) for k in range(1, len(st))] for st in ev]
+    flat_c = [x for row in copy_ms for x in row]
+    flat_l = [x for row in learn_ms for x in row]
+    flat_w = [x for row in wait_ms for x in row]
+    rates = [chunk_bytes / (x / 1000) / 1e9 for x in flat_c if x > 0]
+    tot_copy = sum(flat_c)
+    return {"h2d_gbs": (h2d_bytes * len(ev)) / (tot_copy / 1000) / 1e9 if tot_copy > 0 else None,
+            "chunk_h2d_gbs": {"min": min(rates), "median": sorted(rates)[len(rates) // 2], "max": max(rates)}
+            if rates else None,
+            "chunk_copy_ms": {"min": min(flat_c), "median": sorted(flat_c)[len(flat_c) // 2], "max": max(flat_c)},
+            "chunk_learn_ms": {"min": min(flat_l), "median": sorted(flat_l)[len(flat_l) // 2], "max": max(flat_l)},
+            "learn_wait_ms_per_step": sum(flat_w) / len(ev),
+            "last_step_copy_ms": copy_ms[-1], "last_step_learn_ms": learn_ms[-1]}
+
+
+def dominant_roofline(wl, dom, d, busy_ms, timed_segments, timed_ms, pk, alu_peak=None, traffic=None):
+    """Roofline of the dominant kernel of the step.
+
+    The work is the algorithmic work of the path: 2 T d_hid (d_in + d_out) flops per
+    chain-segment for each phase kernel (half of the 4 (d_in d_hid + d_hid d_out) per token of
+    forward plus backward).  On the bf16 path it is set against the tensor peak: the sustained
+    one, since the kernel is timed inside a long step (`frac`), and the burst one beside it.
+    `achieved` is one launch's work over the kernel's average launch duration; `busy` is the
+    work of all timed launches over the union of their launch intervals on both streams (the
+    two chain groups' launches overlap, so the average launch duration counts shared time
+    twice).  Phase B also streams the fp32 state (W and mu read and written, the bf16 operand
+    copy written): its bytes with that state are under `hbm`, against the HBM peak.  The fp32
+    path's resident kernel runs on the CUDA cores: its flops are set against the FP32 FMA peak."""
+    hbm, tf_burst, tf_sus, src = pk
+    flops1, byts1 = kernel_work(wl, dom, d["chains_per_launch"])
+    avg_s = d["avg_us"] * 1e-6
+    flops_all, byts_all = kernel_work(wl, dom, wl.chains)
+    if alu_peak:
+        ach = flops1 / avg_s / 1e12
+        roof = {"kernel": dom, "bound": "alu", "achieved": ach, "peak": alu_peak, "unit": "TFLOP/s",
+                "frac": ach / alu_peak, "traffic": traffic,
+                "peak_source": "FP32 FMA: SMs x 128 lanes x 2 flop x max SM clock"}
+        if busy_ms > 0:
+            b = flops_all * timed_segments / (busy_ms / 1000) / 1e12
+            roof["busy"] = {"ms": busy_ms, "share_of_steps": busy_ms / timed_ms, "achieved": b,
+                            "frac": b / alu_peak, "unit": "TFLOP/s"}
+        return roof
+    ach = flops1 / avg_s / 1e12
+    roof = {"kernel": dom, "bound": "tensor", "achieved": ach, "peak": tf_sus, "unit": "TFLOP/s",
+            "frac": ach / tf_sus, "frac_of_burst": ach / tf_burst, "traffic": traffic,
+            "peak_source": f"{src} bf16_tflops_sustained (burst: bf16_tflops)",
+            "work": "2 T d_hid (d_in + d_out) flops per chain-segment, algorithmic"}
+    if busy_ms > 0:
+        b = flops_all * timed_segments / (busy_ms / 1000) / 1e12
+        roof["busy"] = {"ms": busy_ms, "share_of_steps": busy_ms / timed_ms, "achieved": b, "frac": b / tf_sus,
+                        "frac_of_burst": b / tf_burst, "unit": "TFLOP/s"}
+    if dom == "phase_b":
+        g = byts1 / avg_s / 1e9
+        roof["hbm"] = {"achieved": g, "peak": hbm, "unit": "GB/s", "frac": g / hbm,
+                       "bytes_per_launch": byts1,
+                       "bytes_note": "state-inclusive: W and mu read and written in fp32 and the bf16 operand "
+                                     "copy written every segment (18 B per parameter), plus U, Y, dH, At"}
+        if busy_ms > 0:
+            gb = byts_all * timed_segments / (busy_ms / 1000) / 1e9
+            roof["hbm"]["busy"] = {"achieved": gb, "frac": gb / hbm}
+    if d["chains_per_launch"] < wl.chains:
+        roof["note"] = ("launches of the two chain groups run concurrently on two streams; a launch's "
+                        "duration includes the SMs and HBM bandwidth the other group's kernels take, "
+                        "so two overlapping launches each count the shared time; 'busy' divides the "
+                        "kernel's algorithmic work over the timed steps by the union of its launch "
+                        "intervals instead")
+    return roof
+
+
 def kernel_source_sha(text, kind):
     """sha256[:16] of one kernel's section of ttl_tc.cu (phase B: from its section banner to
     make_args), so that the recorded counters stay valid while that kernel's source is unchanged."""
@@ -447,32 +525,41 @@ def run_ours(args, wl):
         copied = [torch.cuda.Event() for _ in range(n_chunks)]
         consumed = [torch.cuda.Event() for _ in range(n_chunks)]
 
-        def e2e_step():
+        n_e2e = max(1, min(args.steps, 5))
+        # per step and chunk: copy start/end on the copy stream, learning start/end on the stream
+        ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_chunks)]
+              for _ in range(n_e2e + 1)]
+
+        def e2e_step(tag):
             mone.mone_mem_write_state(h, W1_0, W2_0, mu0_1, mu0_2)
             for k in range(n_chunks):
                 b = k % 2
+                c0, c1, l0, l1 = ev[tag][k]
                 with torch.cuda.stream(copy_stream):
                     if k >= 2:
                         copy_stream.wait_event(consumed[k - 2])
+                    c0.record(copy_stream)
                     dX[b].copy_(hX[k], non_blocking=True)
                     dK[b].copy_(hK[k], non_blocking=True)
                     dV[b].copy_(hV[k], non_blocking=True)
                     if k == n_chunks - 1:
                         dXq.copy_(hXq, non_blocking=True)
+                    c1.record(copy_stream)
                     copied[k].record(copy_stream)
                 stream.wait_event(copied[k])
+                l0.record(stream)
                 mone.mone_ttl_context(h, dX[b], dK[b], dV[b], nc_tok)
+                l1.record(stream)
                 consumed[k].record(stream)
             mone.mone_mem_generate_kv(h, dXq, wl.Q, Kout, Vout, strides)
             hKo.copy_(Kout, non_blocking=True)
             hVo.copy_(Vout, non_blocking=True)
-        e2e_step()
+        e2e_step(n_e2e)
         torch.cuda.synchronize()
         barrier()
         e0.record(stream)
-        n_e2e = max(1, min(args.steps, 5))
-        for _ in range(n_e2e):
-            e2e_step()
+        for i in range(n_e2e):
+            e2e_step(i)
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
@@ -481,6 +568,7 @@ def run_ours(args, wl):
         d2h = sum(t.numel() * t.element_size() for t in (hKo, hVo))
         e2e = {"value": ws * tokens_per_step / (ms_e2e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e, "chunks": n_chunks}
+        e2e.update(e2e_breakdown(ev[:n_e2e], h2d, (hX[0], hK[0], hV[0])))
 
     # ---- consumer attention of the read (Eq. 5): the query's tokens over [memory tokens || their own
     # keys], timed on its own (it is not part of the test-time-learning step).  The memory tokens are
@@ -539,16 +627,8 @@ def run_ours(args, wl):
     d = kern[dom]
     traffic, traffic_note = ncu_traffic(dom, d["chains_per_launch"], wl)
     alu_peak = fp32_alu_peak_tflops(dev) if wl.dtype == "f32" else None
-    if dom == "phase_b":
-        roof = {"kernel": dom, "bound": "hbm", "achieved": d["gbs"], "peak": hbm, "unit": "GB/s",
-                "frac": d["gbs"] / hbm, "traffic": traffic, "peak_source": f"{peak_src} hbm_gbs"}
-    elif alu_peak:
-        roof = {"kernel": dom, "bound": "alu", "achieved": d["tflops"], "peak": alu_peak, "unit": "TFLOP/s",
-                "frac": d["tflops"] / alu_peak, "traffic": traffic,
-                "peak_source": "FP32 FMA: SMs x 128 lanes x 2 flop x max SM clock"}
-    else:
-        roof = {"kernel": dom, "bound": "tensor", "achieved": d["tflops"], "peak": tf_sus, "unit": "TFLOP/s",
-                "frac": d["tflops"] / tf_sus, "traffic": traffic, "peak_source": f"{peak_src} bf16_tflops_sustained"}
+    roof = dominant_roofline(wl, dom, d, kbusy.get(dom, 0.0), timed_segments, ms * args.steps,
+                             (hbm, tf_burst, tf_sus, peak_src), alu_peak, traffic)
     if traffic_note.strip("; "):
         roof["traffic_note"] = traffic_note.strip("; ")
     # the memory read: latency of one generate_kv call and its weight-streaming rate
@@ -561,25 +641,6 @@ def run_ours(args, wl):
         byts = wl.chains * (fast_params(wl) * el + wl.Q * (wl.d_in + wl.d_out) * el)
         gkv = {"us": us, "bytes": byts, "gbs": byts / (us * 1e-6) / 1e9, "frac_of_hbm": byts / (us * 1e-6) / 1e9 / hbm,
                "Q": wl.Q}
-    if d["chains_per_launch"] < wl.chains:
-        roof["note"] = ("launches of the two chain groups run concurrently on two streams; a launch's "
-                        "duration includes the SMs and HBM bandwidth the other group's kernels take, "
-                        "so two overlapping launches each count the shared time; 'busy' divides the "
-                        "kernel's algorithmic work over the timed steps by the union of its launch "
-                        "intervals instead")
-    busy_ms = kbusy.get(dom, 0.0)
-    if busy_ms > 0:
-        flops_all, byts_all = kernel_work(wl, dom, wl.chains)
-        units = timed_segments  # segments of all chains processed in the timed steps
-        if dom == "phase_b":
-            ach = byts_all * units / (busy_ms / 1000) / 1e9
-            roof["busy"] = {"ms": busy_ms, "share_of_steps": busy_ms / (ms * args.steps), "achieved": ach,
-                            "frac": ach / hbm, "unit": "GB/s"}
-        else:
-            ach = flops_all * units / (busy_ms / 1000) / 1e12
-            pk = alu_peak or tf_sus
-            roof["busy"] = {"ms": busy_ms, "share_of_steps": busy_ms / (ms * args.steps), "achieved": ach,
-                            "frac": ach / pk, "unit": "TFLOP/s"}
     # the whole step against HBM: algorithmic bytes of every kernel of the step / step time
     S = (wl.N + wl.seg_T - 1) // wl.seg_T
     if "resident" in kern:  # one launch per input window, each streaming its segments

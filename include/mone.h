@@ -27,7 +27,8 @@
  *     (a cudaStream_t cast to void*; NULL = legacy default stream).
  *   - Argument errors are returned synchronously and nothing is launched.
  *     Errors found on the device (a bounded wait that gave up, a non-finite
- *     weight) are latched in a device status word; mone_mem_sync returns them.
+ *     weight, a failed index check of a MONE_DEBUG build) are latched in a device
+ *     status word; mone_mem_sync returns them.
  *   - There is no CPU fallback: without a usable sm_103a GPU, init fails with
  *     MONE_ERR_CUDA.
  */
@@ -38,7 +39,7 @@
 extern "C" {
 #endif
 
-#define MONE_ABI_VERSION 5
+#define MONE_ABI_VERSION 6
 
 typedef struct mone_mem mone_mem; /* opaque; created by mone_mem_init */
 
@@ -50,7 +51,8 @@ typedef enum {
     MONE_ERR_CUDA = 4,              /* a CUDA call failed (no device, launch failure, ...) */
     MONE_ERR_TIMEOUT = 5,           /* a bounded device-side wait gave up (latched) */
     MONE_ERR_NONFINITE = 6,         /* an updated fast weight was NaN/Inf (latched) */
-    MONE_ERR_UNSUPPORTED = 7        /* valid request this build does not implement */
+    MONE_ERR_UNSUPPORTED = 7,       /* valid request this build does not implement */
+    MONE_ERR_CHECK = 8              /* a device-side index check failed (MONE_DEBUG builds; latched) */
 } mone_status;
 
 enum { MONE_FP32 = 0, MONE_BF16 = 1 };  /* dtype of X, K, V, Xq and generated K/V */
@@ -161,6 +163,25 @@ mone_status mone_ttl_context(mone_mem* m, const void* X, const void* K, const vo
                              long long N, void* stream);
 
 /*
+ * mone_ttl_context, with per-segment metrics of every chain written into caller
+ * buffers, so the learning of a whole context can be followed segment by segment
+ * (Sec. 3.4's chain W_0 -> ... -> W_S).  With S = ceil(N / seg_T) segments of this
+ * call (numbered from the call's first token) and C = n_ctx * n_layers chains,
+ * element [s * C + c] of
+ *   seg_loss  is L_s of chain c: the segment mean of Eq. 7's loss (or of the
+ *             squared-error variant) at the segment's starting weights;
+ *   seg_step  is |mu_s|_F^2 of chain c: the squared Frobenius norm over W1 and W2
+ *             of the step of Eq. 8 (W_s = W_{s-1} - mu_s, before the row
+ *             renormalisation; without momentum mu_s is the rate-weighted gradient).
+ * Both are fp32 device buffers of S * C elements owned by the caller, 4-byte
+ * aligned; either may be null.  The library zeroes them on the stream first, then
+ * accumulates into them.  Same inputs, state update and ordering as mone_ttl_context.
+ * Errors: INVALID_ARG, CUDA, and UNSUPPORTED for seg_step on a SwiGLU-memory handle.
+ */
+mone_status mone_ttl_context_metrics(mone_mem* m, const void* X, const void* K, const void* V, long long N,
+                                     float* seg_loss, float* seg_step, void* stream);
+
+/*
  * Memory read (Eq. 4 and the normalisation after it): for every chain and query
  * token, o = M(phi(x_q); W_S) with phi the key/query transform of the mode, then
  * every output head h (width head_dim) becomes gate_h * o_h / sqrt(mean(o_h^2) + eps).
@@ -219,7 +240,10 @@ mone_status mone_mem_read_state(const mone_mem* m, float* W1, float* W2, float* 
 mone_status mone_mem_write_state(mone_mem* m, const float* W1, const float* W2, const float* mu1,
                                  const float* mu2, void* stream);
 
-/* Synchronise the stream and return (and clear) any latched device error. */
+/* Synchronise the stream and return (and clear) any latched device error.  A library
+ * built with MONE_DEBUG also checks tile and row indices on the device: a failed check
+ * skips the access, is latched, and is returned here as MONE_ERR_CHECK with the site in
+ * mone_last_error. */
 mone_status mone_mem_sync(mone_mem* m, void* stream);
 
 /* Number of device kernels the library has launched on this handle so far. */

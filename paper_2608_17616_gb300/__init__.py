@@ -14,7 +14,9 @@ import os
 from typing import Optional, Sequence
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "libmone.so")
+# MONE_LIB selects another build of the library, e.g. the MONE_DEBUG build (libmone_debug.so)
+LIB_PATH = os.environ.get("MONE_LIB") or os.path.join(_PKG, "libmone.so")
+DEBUG_LIB_PATH = os.path.join(_PKG, "libmone_debug.so")
 
 MONE_FP32, MONE_BF16 = 0, 1
 MONE_PLAIN, MONE_PAPER = 0, 1
@@ -24,13 +26,15 @@ MONE_RENORM_ROWS, MONE_RENORM_OUT = 0, 1
 MONE_GATE_LINEAR, MONE_GATE_SILU = 0, 1
 
 STATUS = {0: "MONE_OK", 1: "MONE_ERR_INVALID_ARG", 2: "MONE_ERR_UNSUPPORTED_SHAPE", 3: "MONE_ERR_OOM",
-          4: "MONE_ERR_CUDA", 5: "MONE_ERR_TIMEOUT", 6: "MONE_ERR_NONFINITE", 7: "MONE_ERR_UNSUPPORTED"}
+          4: "MONE_ERR_CUDA", 5: "MONE_ERR_TIMEOUT", 6: "MONE_ERR_NONFINITE", 7: "MONE_ERR_UNSUPPORTED",
+          8: "MONE_ERR_CHECK"}
 
 # Every symbol include/mone.h declares.
 EXPORTS = ("mone_mem_init", "mone_ttl_segment", "mone_ttl_context", "mone_mem_generate_kv", "mone_mem_free",
            "mone_mem_read_state", "mone_mem_write_state", "mone_mem_sync", "mone_mem_launch_count",
            "mone_status_string", "mone_abi_version", "mone_mem_set_timing", "mone_mem_kernel_time",
-           "mone_last_error", "mone_mem_generate_kv_noalloc", "mone_attention", "mone_mem_kernel_busy")
+           "mone_last_error", "mone_mem_generate_kv_noalloc", "mone_attention", "mone_mem_kernel_busy",
+           "mone_ttl_context_metrics")
 
 KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read", "mse", "attention", "resident")
 
@@ -72,6 +76,7 @@ def lib(path: Optional[str] = None) -> ctypes.CDLL:
                            ctypes.POINTER(vp)], i),
         "mone_ttl_segment": ([vp, i, i, vp, vp, vp, i, vp, vp, vp], i),
         "mone_ttl_context": ([vp, vp, vp, vp, ll, vp], i),
+        "mone_ttl_context_metrics": ([vp, vp, vp, vp, ll, vp, vp, vp], i),
         "mone_mem_generate_kv": ([vp, vp, i, vp, vp, ctypes.POINTER(ll), vp], i),
         "mone_mem_generate_kv_noalloc": ([vp, vp, i, vp, vp, ctypes.POINTER(ll), vp], i),
         "mone_attention": ([vp, vp, i, i, vp, vp, ctypes.POINTER(ll), i, vp, vp], i),
@@ -115,7 +120,7 @@ def _stream(stream) -> Optional[int]:
 
 def _check(fn: str, rc: int):
     if rc != 0:
-        detail = lib().mone_last_error().decode() if rc in (3, 4) else ""
+        detail = lib().mone_last_error().decode() if rc in (3, 4, 8) else ""
         raise MoneError(fn, rc, detail)
 
 
@@ -148,6 +153,12 @@ def mone_ttl_segment(h: int, ctx: int, layer: int, X, K, V, n_tok: int, eta=None
 
 def mone_ttl_context(h: int, X, K, V, N: int, stream=None):
     _check("mone_ttl_context", lib().mone_ttl_context(h, _ptr(X), _ptr(K), _ptr(V), N, _stream(stream)))
+
+
+def mone_ttl_context_metrics(h: int, X, K, V, N: int, seg_loss=None, seg_step=None, stream=None):
+    """mone_ttl_context with per-segment loss and squared step norm ([S][C] fp32 device buffers)."""
+    _check("mone_ttl_context_metrics", lib().mone_ttl_context_metrics(h, _ptr(X), _ptr(K), _ptr(V), N, _ptr(seg_loss),
+                                                                      _ptr(seg_step), _stream(stream)))
 
 
 def mone_mem_generate_kv(h: int, Xq, Q: int, K_out, V_out, strides: Sequence[int], stream=None):

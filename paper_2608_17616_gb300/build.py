@@ -61,12 +61,17 @@ def _stamp(target: str, digest: str) -> None:
         f.write(digest)
 
 
-def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False) -> str:
+def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False, debug: bool = False) -> str:
+    """Compile every translation unit and link libmone.so.  debug=True builds the MONE_DEBUG
+    variant instead (device-side index checks on, -lineinfo as always) into libmone_debug.so,
+    with its objects apart; load it with MONE_LIB=<path>."""
+    BUILD = os.path.join(PKG, "_build_debug" if debug else "_build")
+    LIB = os.path.join(PKG, "libmone_debug.so" if debug else "libmone.so")
     os.makedirs(BUILD, exist_ok=True)
     headers = [os.path.join(CSRC, h) for h in os.listdir(CSRC) if h.endswith((".h", ".cuh"))]
     headers.append(os.path.join(ROOT, "include", "mone.h"))
     cc = nvcc()
-    extra = ["-Xptxas", "-v"] if ptxas_info else []
+    extra = (["-Xptxas", "-v"] if ptxas_info else []) + (["-DMONE_DEBUG"] if debug else [])
 
     machine = os.uname().machine
 
@@ -102,4 +107,5 @@ def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False) 
 
 
 if __name__ == "__main__":
-    print(build(verbose=True, force="--force" in sys.argv, ptxas_info="--ptxas" in sys.argv))
+    print(build(verbose=True, force="--force" in sys.argv, ptxas_info="--ptxas" in sys.argv,
+                debug="--debug" in sys.argv))

@@ -360,6 +360,8 @@ mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInput
             SegWork x = w;
             x.row0 = row0;
             x.u_off = 0;
+            if (x.loss0) x.loss0 += (row0 / s.T) * x.mstride;  // per-segment metrics from the window's first
+            if (x.step0) x.step0 += (row0 / s.T) * x.mstride;
             const long long n = std::min(win, N - row0);
             if (s.mode == MONE_PAPER) {
                 x.Tp = (int)n;
@@ -400,6 +402,8 @@ mone_status run_segment_loop(mone_mem* m, SegWork* gw, TcInputMaps* gin, TcInput
             x.parity = (int)(i & 1);
             x.renorm_pending = (s.renorm && i > 0) ? 1 : 0;
             x.u_off = u_off;
+            if (x.loss0) x.loss = x.loss0 + i * x.mstride;
+            if (x.step0) x.step_sq = x.step0 + i * x.mstride;
             if (s.memory == MONE_MEM_SWIGLU) {
                 MONE_TRY(timed(m, K_PHASE_A, sg, 1, [&] { return launch_swiglu_phase_a(s, m->swmaps, sin[g], x, sg); }));
                 MONE_TRY(timed(m, K_PHASE_B, sg, 1, [&] { return launch_swiglu_phase_b(s, m->swmaps, sin[g], x, sg); }));
@@ -458,6 +462,8 @@ mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
         gw[g].V = static_cast<const uint8_t*>(w.V) + (size_t)off * w.y_cstride * el;
         if (w.eta_in) gw[g].eta_in = w.eta_in + (size_t)off * w.eta_cstride;
         if (w.loss) gw[g].loss = w.loss + off;
+        if (w.loss0) gw[g].loss0 = w.loss0 + off;
+        if (w.step0) gw[g].step0 = w.step0 + off;
         std::memset(&gin[g], 0, sizeof(TcInputMaps));
         std::memset(&rin[g], 0, sizeof(TcInputMaps));
         std::memset(&sin[g], 0, sizeof(SwInputMaps));
@@ -504,6 +510,7 @@ const char* mone_status_string(mone_status st) {
         case MONE_ERR_TIMEOUT: return "device wait timed out";
         case MONE_ERR_NONFINITE: return "non-finite fast weight";
         case MONE_ERR_UNSUPPORTED: return "unsupported request";
+        case MONE_ERR_CHECK: return "device index check failed";
     }
     return "unknown status";
 }
@@ -571,7 +578,9 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
     step(dalloc(&s.n1, r1));
     step(dalloc(&s.n2, w2_rows(s)));
     step(dalloc(&s.sumsq, 4 * r1));
-    step(dalloc(&s.status, 1));
+    step(dalloc(&s.status, 2));  // flags, and the first failing check site (MONE_DEBUG builds)
+    if (const char* f = std::getenv("MONE_FAULT_STALL"))  // test knob: see DevState::fault_stall
+        s.fault_stall = std::atoi(f) > 0 ? std::atoi(f) : 0;
     if (s.mode == MONE_PAPER) {
         step(dalloc(&s.alpha, C * s.d_in));
         step(dalloc(&s.gamma, C * s.d_in));
@@ -616,7 +625,7 @@ mone_status mone_mem_init(const mone_config* cfg, const float* W1_0, const float
         step(cuda_status(cudaMemsetAsync(s.mu2, 0, n2 * 4, st)));
     }
     if (rc == MONE_OK) step(cuda_status(cudaMemsetAsync(s.sumsq, 0, 4 * r1 * 4, st)));
-    if (rc == MONE_OK) step(cuda_status(cudaMemsetAsync(s.status, 0, 4, st)));
+    if (rc == MONE_OK) step(cuda_status(cudaMemsetAsync(s.status, 0, 2 * sizeof(int), st)));
     if (s.memory == MONE_MEM_SWIGLU) {
         if (rc == MONE_OK) step(cuda_status(launch_swiglu_rows(s, 0, 0, 0, s.C, st)));  // targets + bf16 copies
     } else {
@@ -676,6 +685,37 @@ mone_status mone_ttl_segment(mone_mem* m, int ctx, int layer, const void* X, con
     w.loss = loss_out;
     if (loss_out) MONE_CUDA(cudaMemsetAsync(loss_out, 0, sizeof(float), st));
     return run_segments(m, w, n_tok, st);
+}
+
+mone_status mone_ttl_context_metrics(mone_mem* m, const void* X, const void* K, const void* V, long long N,
+                                     float* seg_loss, float* seg_step, void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    const DevState& s = m->s;
+    if (N < 1 || N > (1ll << 31) - 1) return MONE_ERR_INVALID_ARG;
+    if (!X || !K || !V || !aligned16(X) || !aligned16(K) || !aligned16(V)) return MONE_ERR_INVALID_ARG;
+    if ((seg_loss && (reinterpret_cast<uintptr_t>(seg_loss) & 3u)) ||
+        (seg_step && (reinterpret_cast<uintptr_t>(seg_step) & 3u)))
+        return MONE_ERR_INVALID_ARG;
+    if (seg_step && s.memory == MONE_MEM_SWIGLU) {
+        std::snprintf(g_last_error, sizeof(g_last_error),
+                      "mone_ttl_context_metrics: the step norm is not available for the SwiGLU memory");
+        return MONE_ERR_UNSUPPORTED;
+    }
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const long long S = (N + s.T - 1) / s.T;
+    if (seg_loss) MONE_CUDA(cudaMemsetAsync(seg_loss, 0, (size_t)S * s.C * sizeof(float), st));
+    if (seg_step) MONE_CUDA(cudaMemsetAsync(seg_step, 0, (size_t)S * s.C * sizeof(float), st));
+    SegWork w{};
+    w.c0 = 0;
+    w.nc = s.C;
+    w.X = X; w.K = K; w.V = V;
+    w.x_cstride = N * s.d_in;
+    w.y_cstride = N * (s.d_out / 2);
+    w.n_rows = N;
+    w.loss0 = seg_loss;
+    w.step0 = seg_step;
+    w.mstride = s.C;
+    return run_segments(m, w, N, st);
 }
 
 mone_status mone_ttl_context(mone_mem* m, const void* X, const void* K, const void* V, long long N, void* stream) {
@@ -864,8 +904,17 @@ mone_status mone_mem_sync(mone_mem* m, void* stream) {
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     MONE_CUDA(cudaStreamSynchronize(st));
     int flag = 0;
-    MONE_CUDA(cudaMemcpy(&flag, m->s.status, sizeof(int), cudaMemcpyDeviceToHost));
-    if (flag) MONE_CUDA(cudaMemset(m->s.status, 0, sizeof(int)));
+    int word[2] = {0, 0};
+    MONE_CUDA(cudaMemcpy(word, m->s.status, sizeof(word), cudaMemcpyDeviceToHost));
+    flag = word[0];
+    if (flag) MONE_CUDA(cudaMemset(m->s.status, 0, sizeof(word)));
+    if (flag & DEV_CHECK) {
+        static const char* const sites[] = {"?", "phase A tile", "phase B tile", "read tile", "resident rows",
+                                            "TMA x coordinate"};
+        const int site = word[1] >= 1 && word[1] <= 5 ? word[1] : 0;
+        std::snprintf(g_last_error, sizeof(g_last_error), "device index check failed: %s", sites[site]);
+        return MONE_ERR_CHECK;
+    }
     if (flag & DEV_TIMEOUT) return MONE_ERR_TIMEOUT;
     if (flag & DEV_NONFINITE) return MONE_ERR_NONFINITE;
     return MONE_OK;

@@ -56,6 +56,22 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
     return t;
 }
 
+// Device-side index checks (MONE_DEBUG builds): a failed check latches DEV_CHECK, keeps the
+// first failing site in status[1] and returns false, so the caller skips the access instead
+// of faulting.  In release builds MONE_DCHECK is the constant true and costs nothing.
+#ifdef MONE_DEBUG
+__device__ __forceinline__ bool dcheck(bool ok, int* status, int site) {
+    if (!ok) {
+        atomicOr(status, DEV_CHECK);
+        atomicCAS(status + 1, 0, site);
+    }
+    return ok;
+}
+#define MONE_DCHECK(cond, status, site) ::mone::dcheck((cond), (status), (site))
+#else
+#define MONE_DCHECK(cond, status, site) true
+#endif
+
 // Bounded waits give up after this long, latch DEV_TIMEOUT and let the kernel exit.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
@@ -91,15 +107,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Wait for phase `parity` of an mbarrier; false (and DEV_TIMEOUT latched) after kWaitLimitNs.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* status) {
+// Wait for phase `parity` of an mbarrier; false (and DEV_TIMEOUT latched) after `limit_ns`
+// (kernels whose arguments carry a limit pass it; the others wait kWaitLimitNs).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* status,
+                                          uint64_t limit_ns = kWaitLimitNs) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
 #pragma unroll 1
         for (int i = 0; i < 32; ++i)
             if (mbar_try_wait(bar, parity)) return true;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        if (globaltimer_ns() - t0 > limit_ns) {
             atomicOr(status, DEV_TIMEOUT);
             return false;
         }

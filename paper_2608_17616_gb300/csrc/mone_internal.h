@@ -12,7 +12,11 @@ namespace mone {
 using bf16 = __nv_bfloat16;
 
 // Bits of the device status word (latched until mone_mem_sync reads it).
-enum : int { DEV_TIMEOUT = 1, DEV_NONFINITE = 2 };
+enum : int { DEV_TIMEOUT = 1, DEV_NONFINITE = 2, DEV_CHECK = 4 };
+// Sites of the device-side index checks of a MONE_DEBUG build; the first failing site is kept
+// in status[1] (the word after the status flags) and named by mone_mem_sync's error text.
+enum : int { DS_PHASE_A_TILE = 1, DS_PHASE_B_TILE = 2, DS_READ_TILE = 3, DS_RESIDENT_ROWS = 4,
+             DS_TMA_X = 5 };
 
 // Device-resident state of all chains (see mone_mem_init).
 struct DevState {
@@ -27,6 +31,9 @@ struct DevState {
     float* colpart;               // [kColRowSlices][C][d_out] partial column sums of squares
     float* sumsq;                 // [2 parity][2 matrix][C][d_hid] row sums of squares
     int* status;                  // device status word
+    // test knob (MONE_FAULT_STALL=n at init): the next n tensor-core phase-A launches issue no
+    // loads and wait 1 ms, so their bounded waits run out and latch DEV_TIMEOUT
+    mutable int fault_stall;
     // meta-parameters (owned copies)
     float *alpha, *gamma, *w_eta, *b_eta, *w_beta, *b_beta, *gate;
     // paper-mode input scratch for a window of win_rows tokens (a multiple of T)
@@ -78,7 +85,11 @@ struct SegWork {
     long long eta_cstride;
     int parity;                  // segment index parity within the call
     int renorm_pending;          // previous segment's renorm scale still to apply
-    float* loss;                 // [C] loss accumulator or null
+    float* loss;                 // [C] loss accumulator of this segment or null
+    float* step_sq;              // [C] squared norm of this segment's Eq. 8 step, or null
+    // per-segment metrics of a whole call: segment i of chain c at [i * mstride + c], or null
+    float *loss0, *step0;
+    long long mstride;
     int y_scratch;               // targets are the residual scratch (rows from 0), not the caller's K, V
 };
 

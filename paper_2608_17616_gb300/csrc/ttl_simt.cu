@@ -99,6 +99,7 @@ struct F32SegArgs {
     float* sumsq;             // [2][2][C][d_hid]
     float *dH, *At;           // [C][T][d_hid]
     float* loss;
+    float* step_sq;           // [nc] squared norm of this segment's Eq. 8 step, or null
     int* status;
 };
 
@@ -227,6 +228,7 @@ __global__ void __launch_bounds__(256) phase_b_f32_kernel(const F32SegArgs a) {
     const float* prev = ss_ptr(a, a.parity ^ 1, which) + (size_t)cs * a.d_hid;
     float* cur = a.sumsq + ((size_t)(a.parity * 2 + which) * a.C + cs) * a.d_hid;
     bool finite = true;
+    float step = 0.f;  // sum of mu_s^2 over this thread's elements
 #pragma unroll
     for (int i = 0; i < B_MR; ++i) {
         const int h = h0 + ty * B_MR + i;
@@ -242,6 +244,7 @@ __global__ void __launch_bounds__(256) phase_b_f32_kernel(const F32SegArgs a) {
             wrow[j] = wn;
             if (M) mrow[j] = mn;
             ss = fmaf(wn, wn, ss);
+            step = fmaf(mn, mn, step);
             finite = finite && isfinite(wn);
         }
         ss += __shfl_xor_sync(0xffffffffu, ss, 8);
@@ -249,6 +252,10 @@ __global__ void __launch_bounds__(256) phase_b_f32_kernel(const F32SegArgs a) {
         ss += __shfl_xor_sync(0xffffffffu, ss, 2);
         ss += __shfl_xor_sync(0xffffffffu, ss, 1);
         if (tx == 0) atomicAdd(&cur[h], ss);
+    }
+    if (a.step_sq) {
+        step = warp_sum(step);
+        if ((tid & 31) == 0) atomicAdd(&a.step_sq[cz], step);
     }
     if (!finite) atomicOr(a.status, DEV_NONFINITE);
 }
@@ -285,6 +292,7 @@ F32SegArgs make_f32_args(const DevState& s, const SegWork& w) {
     a.dH = reinterpret_cast<float*>(s.dHt);
     a.At = reinterpret_cast<float*>(s.Att);
     a.loss = w.loss;
+    a.step_sq = w.step_sq;
     a.status = s.status;
     return a;
 }
@@ -401,7 +409,9 @@ struct ResArgs {
     const float* b_beta;
     float *W1, *W2, *mu1, *mu2;
     const float *n1, *n2;
-    float* loss;                 // [nc] per-segment loss accumulator or null
+    float* loss;                 // loss of segment seg of chain cz at loss[seg * m_sstride + cz], or null
+    float* step_sq;              // squared norm of the Eq. 8 step, same layout, or null
+    long long m_sstride;         // stride between segments of loss and step_sq (0: one accumulator)
     int* status;
 };
 
@@ -619,15 +629,21 @@ __global__ void __launch_bounds__(RES_NT, 1) ttl_resident_f32_kernel(const ResAr
         }
         if (a.loss) {
             const float tot = block_sum_res(lsum, red);
-            if (tid == 0) atomicAdd(&a.loss[cz], -tot / (float)Tp);
+            if (tid == 0) atomicAdd(&a.loss[seg * a.m_sstride + cz], -tot / (float)Tp);
         }
-        float wn[RB];
+        float wn[RB], step = 0.f;
 #pragma unroll
         for (int r = 0; r < RB; ++r) {
             const float mn = a.momentum ? fmaf(beta, mu[r], acc[r]) : acc[r];
             mu[r] = mn;
             acc[r] = 0.f;
             wn[r] = own ? Ws[r * LD + cb] - mn : 0.f;
+            step = own ? fmaf(mn, mn, step) : step;
+        }
+        if (a.step_sq) {
+            __syncthreads();  // red may still be read by block_sum_res above
+            const float tot = block_sum_res(step, red);
+            if (tid == 0) atomicAdd(&a.step_sq[seg * a.m_sstride + cz], tot);
         }
         if (a.renorm) {
             // row sums of squares per (matrix, row); a warp may hold columns of both matrices
@@ -658,7 +674,9 @@ __global__ void __launch_bounds__(RES_NT, 1) ttl_resident_f32_kernel(const ResAr
         __syncthreads();
     }
     cp_async_wait<0>();
-    // write the rows and the momentum back
+    // write the rows and the momentum back (the CTA's rows lie inside the chain: index check of
+    // MONE_DEBUG builds)
+    if (!MONE_DCHECK(h0 + RB <= a.d_hid, a.status, DS_RESIDENT_ROWS)) return;
     for (int i = tid; i < RB * (D / 4); i += RES_NT) {
         const int r = i / (D / 4), c = 4 * (i - r * (D / 4));
         const size_t row = (size_t)cs * a.d_hid + h0 + r;
@@ -926,7 +944,9 @@ cudaError_t launch_resident_f32(const DevState& s, const SegWork& w, long long n
     a.lr = s.lr;
     a.b_beta = s.b_beta;
     a.W1 = s.W1; a.W2 = s.W2; a.mu1 = s.mu1; a.mu2 = s.mu2; a.n1 = s.n1; a.n2 = s.n2;
-    a.loss = w.loss;
+    a.loss = w.loss0 ? w.loss0 : w.loss;
+    a.step_sq = w.step0;
+    a.m_sstride = w.loss0 || w.step0 ? w.mstride : 0;
     a.status = s.status;
     int dev = 0, sms = 0;
     cudaError_t e = cudaGetDevice(&dev);

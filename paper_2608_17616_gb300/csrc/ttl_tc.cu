@@ -82,9 +82,13 @@ struct TcArgs {
     float* sumsq;               // [2 parity][2 matrix][C][d_hid]
     bf16 *dH, *At;              // [C][T][d_hid]
     float* loss;                // [nc] or null
+    float* step_sq;             // [nc] squared norm of this segment's Eq. 8 step (phase B), or null
     int* status;
     int r_only;                 // phase A pairs: At and c SiLU'(x) / |z| come from the squared-error
                                 // pre-pass (the latter in dH); accumulate R only and form dH in place
+    unsigned long long wait_ns; // limit of every mbarrier wait of the launch (kWaitLimitNs)
+    int stall;                  // test knob (phase A): the producer issues no loads, so the first
+                                // wait for a full stage runs out; nothing is in flight when it does
 };
 
 __device__ __forceinline__ float* ss_row(const TcArgs& a, int parity, int which, int cs) {
@@ -143,6 +147,8 @@ __device__ __forceinline__ bool phase_a_epilogue(const TcArgs& a, uint32_t tmem,
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int e = warp - 2, q = warp & 3, ch = e >> 2, et = threadIdx.x - 64;
     static_assert(BN <= EPI_THREADS && BN % 64 == 0, "one scale per epilogue thread, 32-column chunks");
+    // the tile's rows of dH / At lie inside the [C][T][d_hid] scratch (index check of MONE_DEBUG builds)
+    const bool wr = MONE_DCHECK(cs < a.C && trow + 128 <= a.T && h0 + BN <= a.d_hid, a.status, DS_PHASE_A_TILE);
     if (et < BN) {
         const int h = h0 + et;
         float s1 = 1.f, s2 = 1.f;
@@ -157,7 +163,7 @@ __device__ __forceinline__ bool phase_a_epilogue(const TcArgs& a, uint32_t tmem,
             ss_row(a, a.parity, 1, cs)[h] = 0.f;
         }
     }
-    if (et == 0) *flag = mbar_wait(tfull_bar, parity_bit, a.status) ? 1 : 0;
+    if (et == 0) *flag = mbar_wait(tfull_bar, parity_bit, a.status, a.wait_ns) ? 1 : 0;
     __syncwarp();
     named_bar_sync(EPI_BAR, EPI_THREADS);
     if (!*flag) return false;
@@ -211,7 +217,8 @@ __device__ __forceinline__ bool phase_a_epilogue(const TcArgs& a, uint32_t tmem,
             pa[j / 2] = pack_bf16(av4[0], av4[1]);
             pa[j / 2 + 1] = pack_bf16(av4[2], av4[3]);
         }
-        if (stg) {
+        if (!wr) {
+        } else if (stg) {
             // rows trow + q*32 .. +31 of this warp, columns h0 + c0 .. +31
             const size_t r0 = ((size_t)cs * a.T + trow + q * 32) * a.d_hid + h0 + c0;
             store_rows_coalesced(stg, pd, a.dH + r0, a.d_hid, lane);
@@ -247,6 +254,8 @@ __device__ __forceinline__ bool phase_a_epilogue_split(const TcArgs& a, uint32_t
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int e = warp - 2, q = warp & 3, ch = e >> 2, et = threadIdx.x - 64;
     static_assert(BN <= EPI_THREADS && BN % 64 == 0, "one scale per epilogue thread, 32-column chunks");
+    // the tile's rows of dH / At lie inside the [C][T][d_hid] scratch (index check of MONE_DEBUG builds)
+    const bool wr = MONE_DCHECK(cs < a.C && trow + 128 <= a.T && h0 + BN <= a.d_hid, a.status, DS_PHASE_A_TILE);
     if (et < BN) {
         const int h = h0 + et;
         float s1 = 1.f, s2 = 1.f;
@@ -261,7 +270,7 @@ __device__ __forceinline__ bool phase_a_epilogue_split(const TcArgs& a, uint32_t
             ss_row(a, a.parity, 1, cs)[h] = 0.f;
         }
     }
-    if (et == 0) *flag = mbar_wait(hfull_bar, parity_bit, a.status) ? 1 : 0;
+    if (et == 0) *flag = mbar_wait(hfull_bar, parity_bit, a.status, a.wait_ns) ? 1 : 0;
     __syncwarp();
     named_bar_sync(EPI_BAR, EPI_THREADS);
     if (!*flag) return false;
@@ -302,11 +311,11 @@ __device__ __forceinline__ bool phase_a_epilogue_split(const TcArgs& a, uint32_t
             pa[j / 2 + 1] = pack_bf16(av4[2], av4[3]);
         }
         tmem_st32(lane_base + c0, hv);
-        store_rows_coalesced(stg, pa, a.At + r0 + c0, a.d_hid, lane);
+        if (wr) store_rows_coalesced(stg, pa, a.At + r0 + c0, a.d_hid, lane);
     }
     tmem_wait_st();
     // ---- part 2, after the main loop: dH = R s2 s'
-    if (et == 0) flag[2] = mbar_wait(tfull_bar, parity_bit, a.status) ? 1 : 0;
+    if (et == 0) flag[2] = mbar_wait(tfull_bar, parity_bit, a.status, a.wait_ns) ? 1 : 0;
     __syncwarp();
     named_bar_sync(EPI_BAR, EPI_THREADS);
     if (!flag[2]) return false;
@@ -329,7 +338,7 @@ __device__ __forceinline__ bool phase_a_epilogue_split(const TcArgs& a, uint32_t
             pd[j / 2] = pack_bf16(rv[j] * s2v.x * sp[j], rv[j + 1] * s2v.y * sp[j + 1]);
             pd[j / 2 + 1] = pack_bf16(rv[j + 2] * s2v.z * sp[j + 2], rv[j + 3] * s2v.w * sp[j + 3]);
         }
-        store_rows_coalesced(stg, pd, a.dH + r0 + c0, a.d_hid, lane);
+        if (wr) store_rows_coalesced(stg, pd, a.dH + r0 + c0, a.d_hid, lane);
     }
     return true;
 }
@@ -342,6 +351,8 @@ __device__ __forceinline__ bool phase_a_epilogue_r_only(const TcArgs& a, uint32_
                                                         int trow, bool zero_ss, uint8_t* stg, Release&& release) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int e = warp - 2, q = warp & 3, ch = e >> 2, et = threadIdx.x - 64;
+    // the tile's rows of dH lie inside the [C][T][d_hid] scratch (index check of MONE_DEBUG builds)
+    const bool wr = MONE_DCHECK(cs < a.C && trow + 128 <= a.T && h0 + BN <= a.d_hid, a.status, DS_PHASE_A_TILE);
     if (et < BN) {
         const int h = h0 + et;
         float s2 = 1.f;
@@ -353,7 +364,7 @@ __device__ __forceinline__ bool phase_a_epilogue_r_only(const TcArgs& a, uint32_
             ss_row(a, a.parity, 1, cs)[h] = 0.f;
         }
     }
-    if (et == 0) *flag = mbar_wait(tfull_bar, parity_bit, a.status) ? 1 : 0;
+    if (et == 0) *flag = mbar_wait(tfull_bar, parity_bit, a.status, a.wait_ns) ? 1 : 0;
     __syncwarp();
     named_bar_sync(EPI_BAR, EPI_THREADS);
     if (!*flag) return false;
@@ -387,7 +398,7 @@ __device__ __forceinline__ bool phase_a_epilogue_r_only(const TcArgs& a, uint32_
                 pd[j / 2] = pack_bf16(rv[j] * tab[BN + c0 + j] * sf.x, rv[j + 1] * tab[BN + c0 + j + 1] * sf.y);
             }
         }
-        store_rows_coalesced(stg, pd, a.dH + r0 + c0, a.d_hid, lane);  // in place: every lane has read its row
+        if (wr) store_rows_coalesced(stg, pd, a.dH + r0 + c0, a.d_hid, lane);  // in place: every lane has read its row
     }
     return true;
 }
@@ -414,12 +425,12 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             const uint64_t wpol = l2_evict_last_policy();  // the bf16 W copy phase B wrote
             uint32_t kc = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+            for (int tile = blockIdx.x; tile < ntiles && ok && !a.stall; tile += gridDim.x) {
                 const int cz = tile / (n_ht * n_tt), ht = (tile / n_tt) % n_ht, tt = tile % n_tt;
                 const int cs = a.c0 + cz, h0 = ht * A_BN, trow = tt * A_BM;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
                     const int s = kc % A_STAGES;
-                    if (kc >= A_STAGES && !mbar_wait(c.empty(s, A_STAGES), ((kc / A_STAGES) - 1) & 1, a.status)) {
+                    if (kc >= A_STAGES && !mbar_wait(c.empty(s, A_STAGES), ((kc / A_STAGES) - 1) & 1, a.status, a.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -448,12 +459,12 @@ tc_phase_a_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             bool ok = true;
             for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++local) {
                 const int b = local & 1;
-                if (local >= 2 && !mbar_wait(c.tempty(b, A_STAGES), ((local >> 1) - 1) & 1, a.status)) break;
+                if (local >= 2 && !mbar_wait(c.tempty(b, A_STAGES), ((local >> 1) - 1) & 1, a.status, a.wait_ns)) break;
                 tc_fence_after();
                 const uint32_t dH = tmem + b * 256, dR = dH + A_BN;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
                     const int s = kc % A_STAGES;
-                    if (!mbar_wait(c.full(s), (kc / A_STAGES) & 1, a.status)) {
+                    if (!mbar_wait(c.full(s), (kc / A_STAGES) & 1, a.status, a.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -572,13 +583,13 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
             const uint64_t wpol = l2_evict_last_policy();  // the bf16 W copy phase B wrote
             uint32_t kc = 0;
             bool ok = true;
-            for (int pt = cluster; pt < npairs && ok; pt += nclusters) {
+            for (int pt = cluster; pt < npairs && ok && !a.stall; pt += nclusters) {
                 const int cz = pt / (n_ht * n_tp), ht = (pt / n_tp) % n_ht, tp = pt % n_tp;
                 const int cs = a.c0 + cz, hrow = ht * P_BN + (int)rank * (P_BN / 2);
                 const int trow = tp * 2 * A_BM + (int)rank * A_BM;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
                     const int s = kc % P_STAGES;
-                    if (kc >= P_STAGES && !mbar_wait(c.empty(s, P_STAGES), ((kc / P_STAGES) - 1) & 1, a.status)) {
+                    if (kc >= P_STAGES && !mbar_wait(c.empty(s, P_STAGES), ((kc / P_STAGES) - 1) & 1, a.status, a.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -610,7 +621,7 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
             bool ok = true;
             for (int pt = cluster; pt < npairs && ok; pt += nclusters, ++local) {
                 // one accumulator buffer: wait until both CTAs' epilogues have read the last tile
-                if (local >= 1 && !mbar_wait(c.tempty(0, P_STAGES), (local - 1) & 1, a.status)) {
+                if (local >= 1 && !mbar_wait(c.tempty(0, P_STAGES), (local - 1) & 1, a.status, a.wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -618,7 +629,7 @@ tc_phase_a_pair_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_con
                 const uint32_t dH = tmem, dR = tmem + P_BN;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
                     const int s = kc % P_STAGES;
-                    if (!mbar_wait(c.full(s), (kc / P_STAGES) & 1, a.status)) {
+                    if (!mbar_wait(c.full(s), (kc / P_STAGES) & 1, a.status, a.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -816,7 +827,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 constexpr int HB = (PAIR ? B_BN / 2 : B_BN) / 64;  // 64-row boxes of hidden rows
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
                     const int s = kc % NS;
-                    if (kc >= NS && !mbar_wait(empty(s), ((kc / NS) - 1) & 1, a.status)) {
+                    if (kc >= NS && !mbar_wait(empty(s), ((kc / NS) - 1) & 1, a.status, a.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -845,6 +856,8 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                             y = a.y_row0 + kb * BK;
                             z = cz;
                         }
+                        // a tiled copy's innermost coordinate must be 16-byte aligned (8 bf16)
+                        if (!MONE_DCHECK((x & 7) == 0, a.status, DS_TMA_X)) continue;
                         if constexpr (PAIR)
                             tma_load_3d_pair(dst, map, fb, x, y, z);
                         else
@@ -870,12 +883,12 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             bool ok = true;
             for (int t = tl.first; t < tl.count && ok; t += tl.step, ++local) {
                 const int b = local & 1;
-                if (local >= 2 && !mbar_wait(tempty(b), ((local >> 1) - 1) & 1, a.status)) break;
+                if (local >= 2 && !mbar_wait(tempty(b), ((local >> 1) - 1) & 1, a.status, a.wait_ns)) break;
                 tc_fence_after();
                 const uint32_t d = tmem + b * 256;
                 for (int kb = 0; kb < KB; ++kb, ++kc) {
                     const int s = kc % NS;
-                    if (!mbar_wait(full(s), (kc / NS) & 1, a.status)) {
+                    if (!mbar_wait(full(s), (kc / NS) & 1, a.status, a.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -923,7 +936,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 const int cl = isW1 ? col0 : col0 - a.d_in;
                 for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
                     const int k = seq % S_SLOTS;
-                    if (seq >= S_SLOTS && !mbar_wait(sempty(k), ((seq / S_SLOTS) - 1) & 1, a.status)) {
+                    if (seq >= S_SLOTS && !mbar_wait(sempty(k), ((seq / S_SLOTS) - 1) & 1, a.status, a.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -948,7 +961,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 const int cl = isW1 ? col0 : col0 - a.d_in;
                 for (int g = 0; g < B_BN / S_ROWS; ++g, ++seq) {
                     const int k = seq % S_SLOTS;
-                    if (!mbar_wait(sdone(k), (seq / S_SLOTS) & 1, a.status)) {
+                    if (!mbar_wait(sdone(k), (seq / S_SLOTS) & 1, a.status, a.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -975,6 +988,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
         int* flag = reinterpret_cast<int*>(base + L::FLAG) + grp * 2;
         const uint32_t tempty_rank0 = PAIR ? map_to_cta(tempty(0), 0) : tempty(0);
         bool finite = true;
+        float step = 0.f;        // sum of mu_s^2 over this thread's elements of the current tile
         uint32_t tile_seq0 = 0;  // chunk sequence number of the current tile's first chunk
         int local = 0;
         for (int t = tl.first; t < tl.count; t += tl.step, ++local, tile_seq0 += B_BN / S_ROWS) {
@@ -986,6 +1000,9 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
             const int cl = isW1 ? col0 : col0 - a.d_in;
             const int width = isW1 ? a.d_in : a.d_out;
             const int b = local & 1;
+            // the tile's rows and columns lie inside the chain's W (index check of MONE_DEBUG builds)
+            const bool wr = MONE_DCHECK(cs < a.C && h0 + B_BN <= a.d_hid && cl + B_BM <= width, a.status,
+                                        DS_PHASE_B_TILE);
             const float* n0 = (isW1 ? a.n1 : a.n2) + (size_t)cs * a.d_hid;
             const float* prevss = ss_row(a, a.parity ^ 1, which, cs);
             {   // scales of this group's 4 chunks x 32 rows
@@ -999,7 +1016,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 v = warp_sum(v);
                 if (lane == 0) bred[q] = v;
             }
-            if (et == 0) flag[0] = mbar_wait(tfull(b), (local >> 1) & 1, a.status) ? 1 : 0;
+            if (et == 0) flag[0] = mbar_wait(tfull(b), (local >> 1) & 1, a.status, a.wait_ns) ? 1 : 0;
             __syncwarp();
             named_bar_sync(bar_id, B_EPI_THREADS);
             if (!flag[0]) break;
@@ -1030,7 +1047,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                             mbar_arrive(tempty(b));
                     }
                 }
-                if (et == 0) flag[1] = mbar_wait(sfull(k), (seq / S_SLOTS) & 1, a.status) ? 1 : 0;
+                if (et == 0) flag[1] = mbar_wait(sfull(k), (seq / S_SLOTS) & 1, a.status, a.wait_ns) ? 1 : 0;
                 __syncwarp();
                 named_bar_sync(bar_id, B_EPI_THREADS);
                 if (!flag[1]) {
@@ -1050,8 +1067,9 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                     const float wn = fmaf(sc, Ws[j * B_BM + col], -mn);
                     Ws[j * B_BM + col] = wn;
                     if (a.momentum) Ms[j * B_BM + col] = mn;
-                    st_bf16_hint(bp + j * width, __float2bfloat16_rn(wn), wpol);
+                    if (wr) st_bf16_hint(bp + j * width, __float2bfloat16_rn(wn), wpol);
                     v[j] = wn * wn;  // a NaN or Inf weight makes its row's sum non-finite
+                    step = fmaf(mn, mn, step);
                 }
                 // transpose-reduce: afterwards lane j holds this warp's 32-column partial of row j
 #pragma unroll
@@ -1065,13 +1083,18 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                     }
                 }
                 finite = finite && isfinite(v[0]);
-                atomicAdd(&cur[r0 + lane], v[0]);
+                if (wr) atomicAdd(&cur[r0 + lane], v[0]);
                 // make this warp's shared-memory writes visible to the TMA store, then tell the store warp
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(sdone(k));
             }
             if (!ok) break;
+            if (a.step_sq) {  // per-segment metric: the tile's share of |mu_s|^2
+                const float t = warp_sum(step);
+                if (lane == 0) atomicAdd(&a.step_sq[cz], t);
+            }
+            step = 0.f;
         }
         if (!finite) atomicOr(a.status, DEV_NONFINITE);
     }
@@ -1107,7 +1130,8 @@ TcArgs make_args(const DevState& s, const SegWork& w) {
     a.W1 = s.W1; a.W2 = s.W2; a.mu1 = s.mu1; a.mu2 = s.mu2; a.W1b = s.W1b; a.W2b = s.W2b;
     a.n1 = s.n1; a.n2 = s.n2; a.sumsq = s.sumsq;
     a.dH = reinterpret_cast<bf16*>(s.dHt); a.At = reinterpret_cast<bf16*>(s.Att);
-    a.loss = w.loss; a.status = s.status;
+    a.loss = w.loss; a.step_sq = w.step_sq; a.status = s.status;
+    a.wait_ns = kWaitLimitNs;
     return a;
 }
 
@@ -1352,6 +1376,8 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             } else if constexpr (!OUT) {
                 uint8_t* stg = base + LRT<NST>::STG + (warp - 2) * 2048;
                 bf16* row0 = a.Aq + ((size_t)c * a.Q + qw) * a.d_hid + n0;
+                // the tile's columns of A_q lie inside [Q][d_hid] (index check of MONE_DEBUG builds)
+                const bool wr = MONE_DCHECK(n0 + 128 <= a.d_hid, a.status, DS_READ_TILE);
 #pragma unroll 1
                 for (int cc = 0; cc < 4; ++cc) {
                     float hv[32];
@@ -1360,7 +1386,7 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
                         pk[j] = pack_bf16(hv[2 * j] * sigmoidf_(hv[2 * j]), hv[2 * j + 1] * sigmoidf_(hv[2 * j + 1]));
-                    store_rows_coalesced(stg, pk, row0 + cc * 32, a.d_hid, lane, a.Q - qw);
+                    if (wr) store_rows_coalesced(stg, pk, row0 + cc * 32, a.d_hid, lane, a.Q - qw);
                 }
             } else {
                 constexpr int HD = MODE;
@@ -1376,9 +1402,10 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
                     for (int i = 0; i < HD; ++i) ss = fmaf(v[i], v[i], ss);
                     const int head = n0 / HD + hh;
-                    const float g = a.gate ? a.gate[(size_t)c * nh + head] : 1.f;
+                    const bool wr = MONE_DCHECK(head < nh, a.status, DS_READ_TILE);
+                    const float g = a.gate && wr ? a.gate[(size_t)c * nh + head] : 1.f;
                     const float sc = g / sqrtf(ss / (float)HD + a.eps);
-                    if (qi < a.Q) {
+                    if (qi < a.Q && wr) {
                         const int kvh = head < a.n_kv ? head : head - a.n_kv;
                         bf16* out = (head < a.n_kv ? a.Kout : a.Vout) + (long long)(c / a.L) * a.s0 +
                                     (long long)(c % a.L) * a.s1 + (long long)kvh * a.s2 + (long long)qi * a.s3;
@@ -1488,6 +1515,11 @@ cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputM
     cudaError_t e = ensure_attrs();
     if (e != cudaSuccess) return e;
     TcArgs a = make_args(s, w);
+    if (s.fault_stall > 0) {  // test knob: this launch's waits run out after 1 ms with nothing in flight
+        --s.fault_stall;
+        a.stall = 1;
+        a.wait_ns = 1000000ull;
+    }
     const CUtensorMap& U = s.mode == 1 ? m.Ua : in.Xa;
     if (phase_a_pairs(s)) {
         // squared-error segments: the pre-pass wrote At and c SiLU'(x) / |z|, only R is left

@@ -35,11 +35,11 @@ def test_library_exports_every_declared_symbol(L):
     raw = ctypes.CDLL(mone.LIB_PATH)
     for name in header_functions():
         assert hasattr(raw, name), name
-    assert L.mone_abi_version() == 5
+    assert L.mone_abi_version() == 6
 
 
 def test_status_strings(L):
-    for code in range(8):
+    for code in range(9):
         assert mone.mone_status_string(code)
     assert mone.mone_status_string(0) == "ok"
 
@@ -127,3 +127,16 @@ def test_calls_on_invalid_handles(L):
 def test_init_without_gpu_fails_loudly(L):
     # valid arguments, no device: the library reports a CUDA error, it never falls back to the CPU
     assert init_rc(L, cfg()) == 4
+
+
+def test_debug_build_compiles_and_exports_every_symbol():
+    # the MONE_DEBUG variant (device-side index checks) cross-compiles for sm_103a and exports
+    # the same boundary; its checks run on a GPU in tests/test_debug_build_gpu.py
+    from paper_2608_17616_gb300 import build
+    path = build.build(debug=True)
+    assert path.endswith("libmone_debug.so")
+    raw = ctypes.CDLL(path)
+    for name in header_functions():
+        assert hasattr(raw, name), name
+    raw.mone_abi_version.restype = ctypes.c_int
+    assert raw.mone_abi_version() == 6

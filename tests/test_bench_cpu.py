@@ -63,3 +63,24 @@ def test_resident_kernel_work_counts_inputs_per_segment_and_state_per_launch():
     assert byts == wl.N * (256 + 256) * 4 + 512 * (256 + 256) * 8      # plain mode: W read and write
     paper = wl.replace(mode=wk.PAPER)
     assert bench.kernel_work(paper, "resident", wl.chains * S)[1] == byts + 512 * (256 + 256) * 8  # + momentum
+
+
+def test_dominant_roofline_is_the_tensor_work_of_the_path():
+    # phase B of the 16-layer shape: 2 T d_hid (d_in + d_out) flops per chain-segment, 8 chains a
+    # launch; the per-launch and busy-time figures of a 20-step run (116.79 us a launch, 850.4 ms
+    # busy over 20 x 256 segments of all 16 chains) against the measured bf16 peaks
+    wl = wk.WORKLOADS["l16_d2048_128k"]
+    per_chain = 2 * wl.seg_T * wl.d_hid * (wl.d_in + wl.d_out)
+    assert per_chain == 2 * 512 * 1024 * 3072
+    d = {"chains_per_launch": 8.0, "avg_us": 116.79}
+    pk = (6681.8, 1909.7, 1723.2, "measured")
+    roof = bench.dominant_roofline(wl, "phase_b", d, 850.4, 20 * 256, 20 * 54.17, pk)
+    assert roof["bound"] == "tensor" and roof["unit"] == "TFLOP/s" and roof["peak"] == 1723.2
+    assert roof["achieved"] == pytest.approx(8 * per_chain / 116.79e-6 / 1e12)
+    assert roof["achieved"] == pytest.approx(220.6, rel=1e-3)
+    assert roof["frac_of_burst"] == pytest.approx(0.1155, abs=5e-4)
+    assert roof["busy"]["achieved"] == pytest.approx(16 * per_chain * 20 * 256 / 0.8504 / 1e12)
+    assert roof["busy"]["frac_of_burst"] == pytest.approx(0.1625, abs=5e-4)
+    # the state-inclusive HBM view of the same launch stays beside it
+    assert roof["hbm"]["bytes_per_launch"] == pytest.approx(494.5e6, rel=1e-3)
+    assert roof["hbm"]["frac"] == pytest.approx(494.5e6 / 116.79e-6 / 1e9 / 6681.8, rel=1e-3)

@@ -1,9 +1,10 @@
 """GPU parity: the CUDA path (through the C ABI) against the fp64 oracle.
 
 Tolerances: fp32 path, per-step relative Frobenius error of W1 and W2 <= 1e-4;
-bf16 path, <= 2e-2 after the full context (and the same bound on the weight
-*change* W_S - W_0, which is the part the kernels compute); generated K/V
-<= 2e-2 (fp32 path: 1e-4).
+bf16 path, <= 2e-2 after the full context; the same bounds on the weight
+*change* W_S - W_0, which is the part the kernels compute (and per hidden row:
+1e-4 on the fp32 path, 8e-2 on the bf16 path); generated K/V <= 2e-2 (fp32
+path: 1e-4).
 """
 import numpy as np
 import pytest
@@ -35,12 +36,16 @@ def small(mode, dtype="bf16", n_ctx=2, n_layers=2, d_in=256, d_hid=256, d_out=25
                        T, N, Q, dtype, mode, lr)
 
 
-# Per hidden row, the relative error of the weight change W_S - W_0 (a few rows off, such as
-# one mis-scaled 128-row tile, move the whole-matrix figure very little).
-ROW_DW_TOL = {F32_TOL: 1e-2, BF16_TOL: 1e-1}
-# The momentum is the last step, far smaller than W; the same absolute rounding is a larger
-# fraction of it than of W.
-MU_TOL = 1e-3
+# The weight change W_S - W_0 is the part the kernels compute: it is held to the same bound as
+# the weights (fp32: the per-step 1e-4; bf16: 2e-2 after the context), as a whole and, on the
+# fp32 path, per hidden row.  On the bf16 path a row's change carries the bf16 rounding of its
+# own operands only, so its error spreads wider than the whole matrix's (worst observed 3.9e-2
+# against 4e-3); its bound, 8e-2, still fails a 128-row tile whose change is 10% off, which
+# moves the whole-matrix figure by only about 3.5%.
+DW_TOL = {F32_TOL: F32_TOL, BF16_TOL: BF16_TOL}
+ROW_DW_TOL = {F32_TOL: F32_TOL, BF16_TOL: 8e-2}
+# The momentum on the fp32 path: the same per-step bound as the weights.
+MU_TOL = F32_TOL
 
 
 def check_chain(run, chain, W1, W2, tol, n_tokens=None):
@@ -51,12 +56,12 @@ def check_chain(run, chain, W1, W2, tol, n_tokens=None):
     e2 = record(name, "W2", rel_fro(W2[chain], o2), tol)
     w01, w02 = O.f64(run.W1_0[chain]), O.f64(run.W2_0[chain])
     g1, g2 = W1[chain].double().numpy() - w01, W2[chain].double().numpy() - w02
-    d1 = record(name, "dW1", rel_fro(g1, o1 - w01), max(tol, 5e-2))
-    d2 = record(name, "dW2", rel_fro(g2, o2 - w02), max(tol, 5e-2))
+    d1 = record(name, "dW1", rel_fro(g1, o1 - w01), DW_TOL[tol])
+    d2 = record(name, "dW2", rel_fro(g2, o2 - w02), DW_TOL[tol])
     r1 = record(name, "dW1 row", row_rel_errors(g1, o1 - w01).max(), ROW_DW_TOL[tol])
     r2 = record(name, "dW2 row", row_rel_errors(g2, o2 - w02).max(), ROW_DW_TOL[tol])
     assert e1 <= tol and e2 <= tol, (chain, e1, e2)
-    assert d1 <= max(tol, 5e-2) and d2 <= max(tol, 5e-2), (chain, d1, d2)
+    assert d1 <= DW_TOL[tol] and d2 <= DW_TOL[tol], (chain, d1, d2)
     assert r1 <= ROW_DW_TOL[tol] and r2 <= ROW_DW_TOL[tol], (chain, r1, r2)
     return st
 
@@ -405,7 +410,8 @@ def test_bf16_segment_with_caller_rates_and_loss():
     st = O.init_state(W1=O.f64(run.W1_0[1]), W2=O.f64(run.W2_0[1]))
     st, L = O.ttl_segment(st, X, Y, O.Hyper(mode=wk.PLAIN, lr=wl.lr), None, eta=O.f64(eta))
     assert rel_fro(W1[1], st.W["W1"]) <= BF16_TOL and rel_fro(W2[1], st.W["W2"]) <= BF16_TOL
-    assert rel_fro(W1[1].double() - run.W1_0[1].cpu().double(), st.W["W1"] - O.f64(run.W1_0[1])) <= 5e-2
+    assert record("bf16", "dW1 1 seg", rel_fro(W1[1].double() - run.W1_0[1].cpu().double(),
+                                               st.W["W1"] - O.f64(run.W1_0[1])), 5e-2) <= 5e-2
     assert abs(loss.item() - L) <= BF16_TOL * max(1.0, abs(L))
     # untouched chains keep W_0 exactly
     for c in (0, 2):
@@ -570,7 +576,8 @@ def test_bf16_pair_phase_b_context_parity(mode, loss, lr):
     for c in range(wl.chains):
         st = check_chain(run, c, W1, W2, BF16_TOL)
         if mode == wk.PAPER:
-            assert rel_fro(mu1[c], st.mu["W1"]) <= 5e-2 and rel_fro(mu2[c], st.mu["W2"]) <= 5e-2
+            assert record("bf16", "mu1", rel_fro(mu1[c], st.mu["W1"]), 5e-2) <= 5e-2
+            assert record("bf16", "mu2", rel_fro(mu2[c], st.mu["W2"]), 5e-2) <= 5e-2
         Ko, Vo = oracle_read(run, st, c, Xq)
         assert rel_fro(Kg[0, c].float(), Ko) <= BF16_TOL and rel_fro(Vg[0, c].float(), Vo) <= BF16_TOL
     run.close()
@@ -590,7 +597,8 @@ def test_bf16_pair_phase_b_one_chain_segment():
     st = O.init_state(W1=O.f64(run.W1_0[1]), W2=O.f64(run.W2_0[1]))
     st, L = O.ttl_segment(st, X, Y, O.Hyper(mode=wk.PLAIN, lr=wl.lr), None, eta=O.f64(eta))
     assert rel_fro(W1[1], st.W["W1"]) <= BF16_TOL and rel_fro(W2[1], st.W["W2"]) <= BF16_TOL
-    assert rel_fro(W1[1].double() - run.W1_0[1].cpu().double(), st.W["W1"] - O.f64(run.W1_0[1])) <= 5e-2
+    assert record("bf16", "dW1 1 seg", rel_fro(W1[1].double() - run.W1_0[1].cpu().double(),
+                                               st.W["W1"] - O.f64(run.W1_0[1])), 5e-2) <= 5e-2
     assert abs(loss.item() - L) <= BF16_TOL * max(1.0, abs(L))
     assert torch.equal(W1[0], run.W1_0[0].cpu()) and torch.equal(W2[0], run.W2_0[0].cpu())
     run.close()
@@ -611,7 +619,8 @@ def test_bf16_mse_context_parity(mode, lr):
     for c in range(wl.chains):
         st = check_chain(run, c, W1, W2, BF16_TOL)
         if mode == wk.PAPER:
-            assert rel_fro(mu1[c], st.mu["W1"]) <= 5e-2 and rel_fro(mu2[c], st.mu["W2"]) <= 5e-2
+            assert record("bf16", "mu1", rel_fro(mu1[c], st.mu["W1"]), 5e-2) <= 5e-2
+            assert record("bf16", "mu2", rel_fro(mu2[c], st.mu["W2"]), 5e-2) <= 5e-2
         Ko, Vo = oracle_read(run, st, c, Xq)
         assert rel_fro(Kg[c // 2, c % 2].float(), Ko) <= BF16_TOL
         assert rel_fro(Vg[c // 2, c % 2].float(), Vo) <= BF16_TOL
@@ -631,7 +640,8 @@ def test_bf16_mse_segment_with_caller_rates_and_loss():
     st = O.init_state(W1=O.f64(run.W1_0[1]), W2=O.f64(run.W2_0[1]))
     st, L = O.ttl_segment(st, X, Y, O.Hyper(mode=wk.PLAIN, lr=wl.lr, loss="mse"), None, eta=O.f64(eta))
     assert rel_fro(W1[1], st.W["W1"]) <= BF16_TOL and rel_fro(W2[1], st.W["W2"]) <= BF16_TOL
-    assert rel_fro(W1[1].double() - run.W1_0[1].cpu().double(), st.W["W1"] - O.f64(run.W1_0[1])) <= 5e-2
+    assert record("bf16", "dW1 1 seg", rel_fro(W1[1].double() - run.W1_0[1].cpu().double(),
+                                               st.W["W1"] - O.f64(run.W1_0[1])), 5e-2) <= 5e-2
     assert abs(loss.item() - L) <= BF16_TOL * max(1.0, abs(L))
     for c in (0, 2):
         assert torch.equal(W1[c], run.W1_0[c].cpu()) and torch.equal(W2[c], run.W2_0[c].cpu())
@@ -690,3 +700,52 @@ def test_full_size_sampled_chains(name, chains, n_tokens, loss):
         assert rel_fro(Vg[ctx, layer].float(), Vo) <= BF16_TOL
     run.close()
     torch.cuda.empty_cache()
+
+
+# ----------------------------------------------------------------- per-segment metrics of a whole context
+
+@pytest.mark.parametrize("case", ["bf16_paper", "bf16_mse", "f32_resident", "f32_tiled", "swiglu"])
+def test_context_metrics_per_segment(case):
+    # mone_ttl_context_metrics: per segment and chain, the loss L_s (Eq. 7, or the squared-error
+    # variant) at the segment's starting weights and |mu_s|^2 (the Eq. 8 step), against the
+    # oracle's per-segment losses and momenta; the state it leaves matches the oracle's
+    if case == "bf16_paper":
+        wl, tol = small(wk.PAPER), BF16_TOL
+    elif case == "bf16_mse":
+        wl, tol = small(wk.PAPER).replace(loss="mse"), BF16_TOL
+    elif case == "f32_resident":
+        wl, tol = wk.WORKLOADS["tiny_f32"].replace(N=8 * 128 + 50), F32_TOL
+    elif case == "f32_tiled":
+        wl, tol = small(wk.PAPER, "f32", n_ctx=1, T=64, N=3 * 64 + 20, d_in=512, d_hid=128, d_out=256, lr=0.5), F32_TOL
+    else:
+        wl, tol = wk.Workload("metrics_sw", 61, 1, 2, 256, 96, 256, 2, 64, 128, 3 * 128 + 50, 16, "bf16", wk.PAPER,
+                              0.3, memory="swiglu", heads=2), BF16_TOL
+    run = DeviceRun(wl)
+    S = -(-wl.N // wl.seg_T)
+    loss = torch.full((S, wl.chains), 7.0, device="cuda")
+    step = torch.full((S, wl.chains), 7.0, device="cuda")
+    if case == "swiglu":
+        with pytest.raises(mone.MoneError) as ei:
+            mone.mone_ttl_context_metrics(run.h, run.X, run.K, run.V, wl.N, loss, step)
+        assert ei.value.code == 7  # MONE_ERR_UNSUPPORTED: no step norm for the SwiGLU memory
+        mone.mone_ttl_context_metrics(run.h, run.X, run.K, run.V, wl.N, loss, None)
+    else:
+        mone.mone_ttl_context_metrics(run.h, run.X, run.K, run.V, wl.N, loss, step)
+    mone.mone_mem_sync(run.h)
+    W1, W2, _, _ = run.state()
+    if case != "swiglu":
+        for c in range(wl.chains):
+            check_chain(run, c, W1, W2, tol)
+    loss, step = loss.cpu().double().numpy(), step.cpu().double().numpy()
+    name = "f32" if tol == F32_TOL else "bf16"
+    for c in range(wl.chains):
+        _, losses, trail = oracle_chain(run, c, return_all=True)
+        for s in range(S):
+            L = losses[s]
+            e = record(name, "seg loss", abs(loss[s, c] - L) / max(1.0, abs(L)), tol)
+            assert e <= tol, (c, s, loss[s, c], L)
+            if case != "swiglu":
+                m2 = sum(float(np.sum(v * v)) for v in trail[s].mu.values())
+                e = record(name, "seg |mu|^2", abs(step[s, c] - m2) / m2, tol)
+                assert e <= tol, (c, s, step[s, c], m2)
+    run.close()

@@ -1,7 +1,7 @@
 """GPU parity of the per-head SwiGLU memory (Eq. 3; memory = MONE_MEM_SWIGLU) against the
 oracle's swiglu form.  Tolerances as for the two-matrix memory: weights and generated K/V
 within 2e-2 relative Frobenius error after the whole context (bf16 operands, fp32 state),
-and the weight change W_S - W_0 within 5e-2."""
+and the weight change W_S - W_0 within the same 2e-2 (per hidden row: 8e-2)."""
 import numpy as np
 import pytest
 import torch
@@ -30,7 +30,8 @@ def swiglu(mode=wk.PAPER, n_ctx=1, n_layers=2, d=256, heads=2, F=96, n_kv=2, hd=
                        memory="swiglu", heads=heads)
 
 
-ROW_DW_TOL = 1e-1   # per hidden row, relative error of the weight change W_S - W_0
+DW_TOL = 2e-2      # the weight change W_S - W_0, as the weights
+ROW_DW_TOL = 8e-2  # per hidden row, relative error of the weight change (see test_parity_gpu)
 
 
 def check(run, chains, Xq=None):
@@ -46,9 +47,9 @@ def check(run, chains, Xq=None):
         assert e1 <= TOL and e2 <= TOL, (c, e1, e2)
         s1, s2 = gpu_layout(run.wl, oracle_init(run.wl, run.W1_0[c], run.W2_0[c]).W)
         g1, g2 = W1[c].double().numpy() - s1, W2[c].double().numpy() - s2
-        d1 = record("swiglu", "dW1", rel_fro(g1, o1 - s1), 5e-2)
-        d2 = record("swiglu", "dW2", rel_fro(g2, o2 - s2), 5e-2)
-        assert d1 <= 5e-2 and d2 <= 5e-2, (c, d1, d2)
+        d1 = record("swiglu", "dW1", rel_fro(g1, o1 - s1), DW_TOL)
+        d2 = record("swiglu", "dW2", rel_fro(g2, o2 - s2), DW_TOL)
+        assert d1 <= DW_TOL and d2 <= DW_TOL, (c, d1, d2)
         # rows of the library layout: W1 holds [W_in | W_gate] per hidden unit, W2 = W_out
         r1 = record("swiglu", "dW1 row", row_rel_errors(g1, o1 - s1).max(), ROW_DW_TOL)
         r2 = record("swiglu", "dW2 row", row_rel_errors(g2, o2 - s2).max(), ROW_DW_TOL)
