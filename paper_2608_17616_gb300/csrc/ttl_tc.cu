@@ -1429,6 +1429,207 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     if (warp == 0) tmem_dealloc(tmem, 128);
 }
 
+// ------------------------------------------------------------------ memory read, weights as the MMA rows
+//
+// For a query of Q <= 256 tokens the read runs with the operands the other way round: the
+// weight tile is the tcgen05 A operand (M = 128 weight rows) and the queries are the B
+// operand (N = NT = Q rounded up to 32), so neither an MMA row nor a staged query row is
+// padding and each CTA takes in half the query bytes of the 128-query form.
+//   hidden (HD = 0):  D[h][q] = W1[h] . u_q;  A_q[q][h] = SiLU(D[h][q]), bf16 [C][Q][d_hid],
+//                     stored through a per-warp 32 x 32 transpose so each row leaves as
+//                     64 contiguous bytes
+//   out (HD = 64/128): D[o][q] = sum_h W2[h][o] A_q[q][h] (W2 MN-major); per head of HD
+//                     features the RMS of each query's HD values is a reduction across the
+//                     head's TMEM lanes (warp transpose-sums, then shared memory), then the
+//                     gate, then the store into the caller's K / V (lanes = contiguous features)
+// Warp 0 streams the weight tile and the query rows with TMA (up to 8 stages), warp 1 issues
+// the MMAs into one NT-column TMEM accumulator, warps 2..5 (one TMEM lane quarter each) run
+// the epilogue.  Query rows >= Q arrive as TMA zero fill and are never stored.
+constexpr int RT_THREADS = 6 * 32;
+constexpr int RT_MAX_NT = 256;
+constexpr int RT_A = 128 * BK * 2;  // 16 KB: the weight tile of one k-block
+__host__ __device__ constexpr int rt_stage(int nt) { return RT_A + nt * BK * 2; }
+__host__ __device__ constexpr int rt_stages(int nt) { return (192 * 1024) / rt_stage(nt) < 8 ? (192 * 1024) / rt_stage(nt) : 8; }
+// shared memory after the ring: barriers, TMEM slot and flag, then the epilogue's buffers:
+// 4 warps x 2 KB transposes (hidden) or 4 x NT column partial sums + 2 x NT scales (out)
+__host__ __device__ constexpr int rt_bars(int nt) { return rt_stages(nt) * rt_stage(nt); }
+__host__ __device__ constexpr int rt_epi(int nt) { return rt_bars(nt) + 256; }
+__host__ __device__ constexpr int rt_dyn(int nt) {
+    return rt_epi(nt) + (4 * 2048 > 6 * nt * 4 ? 4 * 2048 : 6 * nt * 4) + 1024;
+}
+static_assert(rt_dyn(RT_MAX_NT) <= 227 * 1024 && rt_dyn(32) <= 227 * 1024, "read shared memory budget");
+
+template <int HD>
+__global__ void __launch_bounds__(RT_THREADS, 1)
+tc_read_t_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmQ, const ReadArgs a,
+                 int NT) {
+    constexpr bool OUT = HD != 0;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int NST = rt_stages(NT), STAGE = rt_stage(NT);
+    const uint32_t bars = smem_u32(base + rt_bars(NT));
+    auto full = [&](int s) { return bars + 8 * s; };
+    auto empty = [&](int s) { return bars + 8 * (8 + s); };
+    const uint32_t tfull = bars + 8 * 16;
+    uint32_t* slot = reinterpret_cast<uint32_t*>(base + rt_bars(NT) + 8 * 17);
+    int* flag = reinterpret_cast<int*>(base + rt_bars(NT) + 8 * 17 + 8);
+    uint8_t* epi = base + rt_epi(NT);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < NST; ++s) {
+            mbar_init(full(s), 1);
+            mbar_init(empty(s), 1);
+        }
+        mbar_init(tfull, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(slot), RT_MAX_NT);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *slot;
+    const int q0 = blockIdx.x * NT, n0 = blockIdx.y * 128, c = blockIdx.z;
+    const int KB = (OUT ? a.d_hid : a.d_in) / BK;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            tma_prefetch_map(&tmW);
+            tma_prefetch_map(&tmQ);
+            for (int kb = 0; kb < KB; ++kb) {
+                const int s = kb % NST;
+                if (kb >= NST && !mbar_wait(empty(s), ((kb / NST) - 1) & 1, a.status)) break;
+                const uint32_t sa = smem_u32(base + s * STAGE), sb = sa + RT_A, fb = full(s);
+                mbar_expect_tx(fb, STAGE);
+                if (OUT) {  // W2 rows kb*64.. as [64 hidden][64 outputs] boxes: the MN-major A operand
+                    tma_load_3d(sa, &tmW, fb, n0, kb * BK, a.b_chain0 + c);
+                    tma_load_3d(sa + BOX, &tmW, fb, n0 + 64, kb * BK, a.b_chain0 + c);
+                } else {
+                    tma_load_3d(sa, &tmW, fb, kb * BK, n0, a.b_chain0 + c);
+                }
+                tma_load_3d(sb, &tmQ, fb, kb * BK, a.a_row0 + q0, a.a_chain0 + c);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, NT, OUT, false);
+            bool ok = true;
+            for (int kb = 0; kb < KB; ++kb) {
+                const int s = kb % NST;
+                if (!mbar_wait(full(s), (kb / NST) & 1, a.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sa = smem_u32(base + s * STAGE), sb = sa + RT_A;
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k)
+                    umma_bf16(tmem, OUT ? sdesc_sw128(sa + k * 16 * 128, BOX) : sdesc_sw128(sa + k * 32, 16),
+                              sdesc_sw128(sb + k * 32, 16), idesc, (kb == 0 && k == 0) ? 0u : 1u);
+                umma_commit(empty(s));
+            }
+            if (ok) umma_commit(tfull);
+        }
+        __syncwarp();
+    } else {
+        const int q = warp & 3;  // TMEM lane quarter: weight rows n0 + 32 q .. + 31
+        const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+        if (threadIdx.x == 64) *flag = mbar_wait(tfull, 0, a.status) ? 1 : 0;
+        __syncwarp();
+        named_bar_sync(R_EPI_BAR, 128);
+        if (*flag) {
+            tc_fence_after();
+            const int nch = NT / 32;
+            if constexpr (!OUT) {
+                // the tile's columns of A_q lie inside [Q][d_hid] (index check of MONE_DEBUG builds)
+                const bool wr = MONE_DCHECK(n0 + 128 <= a.d_hid, a.status, DS_READ_TILE);
+                uint16_t* stg = reinterpret_cast<uint16_t*>(epi + (warp - 2) * 2048);  // [32 queries][32 rows]
+                const int h = n0 + q * 32;
+#pragma unroll 1
+                for (int cc = 0; cc < nch; ++cc) {
+                    float v[32];
+                    tmem_ld32(lane_base + cc * 32, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const bf16 b = __float2bfloat16_rn(v[j] * sigmoidf_(v[j]));
+                        stg[j * 32 + lane] = *reinterpret_cast<const uint16_t*>(&b);
+                    }
+                    __syncwarp();
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const int r = 8 * k + (lane >> 2), i = lane & 3;
+                        const int qi = q0 + cc * 32 + r;
+                        const uint4 val = *reinterpret_cast<const uint4*>(stg + r * 32 + i * 8);
+                        if (qi < a.Q && wr)
+                            *reinterpret_cast<uint4*>(a.Aq + ((size_t)c * a.Q + qi) * a.d_hid + h + i * 8) = val;
+                    }
+                    __syncwarp();
+                }
+            } else {
+                // per-column sums of squares of this warp's 32 features, then the head's total
+                float* part = reinterpret_cast<float*>(epi);  // [4 warps][NT]
+                float* scl = part + 4 * NT;                   // [2 heads of the tile][NT]
+                constexpr int HPT = 128 / HD;                 // heads per 128-feature tile
+                constexpr int WPH = HD / 32;                  // warps per head
+#pragma unroll 1
+                for (int cc = 0; cc < nch; ++cc) {
+                    float v[32];
+                    tmem_ld32(lane_base + cc * 32, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] *= v[j];
+                    // transpose-reduce: afterwards lane j holds the sum over the warp's lanes of column j
+#pragma unroll
+                    for (int sft = 16; sft >= 1; sft >>= 1) {
+                        const bool upper = (lane & sft) != 0;
+#pragma unroll
+                        for (int u = 0; u < sft; ++u) {
+                            const float send = upper ? v[u] : v[u + sft];
+                            const float keep = upper ? v[u + sft] : v[u];
+                            v[u] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+                        }
+                    }
+                    part[q * NT + cc * 32 + lane] = v[0];
+                }
+                named_bar_sync(R_EPI_BAR, 128);
+                const int nh = 2 * a.n_kv;
+                for (int i = threadIdx.x - 64; i < HPT * NT; i += 128) {
+                    const int hl = i / NT, j = i - hl * NT;
+                    float ss = 0.f;
+#pragma unroll
+                    for (int w = 0; w < WPH; ++w) ss += part[(hl * WPH + w) * NT + j];
+                    const int head = n0 / HD + hl;
+                    const float g = a.gate && head < nh ? a.gate[(size_t)c * nh + head] : 1.f;
+                    scl[hl * NT + j] = g / sqrtf(ss / (float)HD + a.eps);
+                }
+                named_bar_sync(R_EPI_BAR, 128);
+                const int o = n0 + q * 32 + lane;  // this thread's output feature
+                const int hl = (q * 32) / HD, head = n0 / HD + hl, d = o - head * HD;
+                const bool wr = MONE_DCHECK(head < nh, a.status, DS_READ_TILE);
+                const int kvh = head < a.n_kv ? head : head - a.n_kv;
+                bf16* outp = (head < a.n_kv ? a.Kout : a.Vout) + (long long)(c / a.L) * a.s0 +
+                             (long long)(c % a.L) * a.s1 + (long long)kvh * a.s2 + d;
+#pragma unroll 1
+                for (int cc = 0; cc < nch; ++cc) {
+                    float v[32];
+                    tmem_ld32(lane_base + cc * 32, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int qi = q0 + cc * 32 + j;
+                        if (qi < a.Q && wr)
+                            outp[(long long)qi * a.s3] = __float2bfloat16_rn(v[j] * scl[hl * NT + cc * 32 + j]);
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, RT_MAX_NT);
+}
+
 std::once_flag g_attr_once;
 cudaError_t g_attr_err = cudaSuccess;
 int g_sms = 0;
@@ -1476,6 +1677,9 @@ cudaError_t ensure_attrs() {
         if (g_attr_err == cudaSuccess) g_attr_err = read_attrs<128>();
         if (g_attr_err == cudaSuccess) g_attr_err = read_attrs<MSE_HIDDEN>();
         if (g_attr_err == cudaSuccess) g_attr_err = read_attrs<MSE_OUT>();
+        for (auto fn : {tc_read_t_kernel<0>, tc_read_t_kernel<64>, tc_read_t_kernel<128>})
+            if (g_attr_err == cudaSuccess)
+                g_attr_err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, rt_dyn(RT_MAX_NT));
         if (g_attr_err == cudaSuccess) {
             cudaLaunchConfig_t cfg = {};
             cudaLaunchAttribute at[1];
@@ -1640,6 +1844,20 @@ cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, v
     a.Vout = static_cast<bf16*>(V_out);
     a.s0 = strides[0]; a.s1 = strides[1]; a.s2 = strides[2]; a.s3 = strides[3];
     a.status = s.status;
+    if (Q <= RT_MAX_NT) {  // weights as the 128-row operand, the queries as N
+        const int NT = (Q + 31) / 32 * 32;
+        CUtensorMap tu, ta;
+        if (!encode_map_bf16_3d(&tu, Uq, s.d_in, Q, s.C, 64, NT) || !encode_map_bf16_3d(&ta, Aq, s.d_hid, Q, s.C, 64, NT))
+            return cudaErrorInvalidValue;
+        const size_t dyn = rt_dyn(NT);
+        tc_read_t_kernel<0><<<dim3(1, s.d_hid / 128, s.C), RT_THREADS, dyn, st>>>(m.W1b, tu, a, NT);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if (s.hd == 64)
+            tc_read_t_kernel<64><<<dim3(1, s.d_out / 128, s.C), RT_THREADS, dyn, st>>>(m.W2m, ta, a, NT);
+        else
+            tc_read_t_kernel<128><<<dim3(1, s.d_out / 128, s.C), RT_THREADS, dyn, st>>>(m.W2m, ta, a, NT);
+        return cudaGetLastError();
+    }
     const int nq = (Q + 127) / 128;
     if ((e = launch_read_kernel<0>(dim3(nq, s.d_hid / 128, s.C), mu, m.W1b, a, st)) != cudaSuccess) return e;
     if (s.hd == 64) return launch_read_kernel<64>(dim3(nq, s.d_out / 128, s.C), ma, m.W2m, a, st);
