@@ -74,7 +74,9 @@ __device__ __forceinline__ void stage_rows(float* dst, const T* src, long long s
 
 template <typename T, int HD>
 struct AttnSmem {
-    static constexpr int KP = HD + 1;                        // key rows padded: lane-per-row reads hit distinct banks
+    // key rows padded by 4 floats: a lane reads its key row 16 bytes at a time, and the 8 lanes of a
+    // quarter warp (one shared-memory wavefront of 128-bit loads) start 68 / 132 floats apart: 8 bank groups
+    static constexpr int KP = HD + 4;
     static constexpr int K_OFF = 0;                          // [KC][KP] keys (fp32)
     static constexpr int V_OFF = K_OFF + KC * KP;            // [KC][HD] values
     static constexpr int Q_OFF = V_OFF + KC * HD;            // [warp][MAXI][HD] scaled queries
@@ -83,7 +85,7 @@ struct AttnSmem {
 };
 
 template <typename T, int HD>
-__global__ void __launch_bounds__(ATT_WARPS * 32, 1) attention_kernel(const AttnArgs a) {
+__global__ void __launch_bounds__(ATT_WARPS * 32, 2) attention_kernel(const AttnArgs a) {
     using SM = AttnSmem<T, HD>;
     constexpr int D = HD / 32;  // value / accumulator dimensions per lane
     extern __shared__ float sh[];
@@ -130,21 +132,25 @@ __global__ void __launch_bounds__(ATT_WARPS * 32, 1) attention_kernel(const Attn
         __syncthreads();
         stage_rows<T, HD>(Ks, Kc, a.s3, j0, nk, a.vec, SM::KP);
         stage_rows<T, HD>(Vs, Vc, a.s3, j0, nk, a.vec, HD);
+        // value rows up to the next multiple of 4 are read with probability 0: make them finite
+        for (int e = threadIdx.x; e < (((nk + 3) & ~3) - nk) * HD; e += ATT_WARPS * 32) Vs[nk * HD + e] = 0.f;
         __syncthreads();
-        // scores: lane owns keys j0 + lane and j0 + lane + 32 of the chunk
+        // scores: lane owns keys j0 + lane and j0 + lane + 32 of the chunk; keys and the (broadcast)
+        // queries are read 4 dimensions at a time
         float z0[MAXI], z1[MAXI];
 #pragma unroll
         for (int k = 0; k < MAXI; ++k) z0[k] = z1[k] = 0.f;
-        const float* k0 = Ks + lane * SM::KP;
-        const float* k1 = Ks + (lane + 32) * SM::KP;
-#pragma unroll 4
-        for (int d = 0; d < HD; ++d) {
-            const float a0 = k0[d], a1 = k1[d];
+        const float4* k0 = reinterpret_cast<const float4*>(Ks + lane * SM::KP);
+        const float4* k1 = reinterpret_cast<const float4*>(Ks + (lane + 32) * SM::KP);
+        const float4* q4 = reinterpret_cast<const float4*>(Qs);
+#pragma unroll 2
+        for (int d4 = 0; d4 < HD / 4; ++d4) {
+            const float4 a0 = k0[d4], a1 = k1[d4];
 #pragma unroll
             for (int k = 0; k < MAXI; ++k) {
-                const float qd = Qs[k * HD + d];
-                z0[k] = fmaf(qd, a0, z0[k]);
-                z1[k] = fmaf(qd, a1, z1[k]);
+                const float4 qd = q4[k * (HD / 4) + d4];
+                z0[k] = fmaf(qd.x, a0.x, fmaf(qd.y, a0.y, fmaf(qd.z, a0.z, fmaf(qd.w, a0.w, z0[k]))));
+                z1[k] = fmaf(qd.x, a1.x, fmaf(qd.y, a1.y, fmaf(qd.z, a1.z, fmaf(qd.w, a1.w, z1[k]))));
             }
         }
 #pragma unroll
@@ -167,16 +173,21 @@ __global__ void __launch_bounds__(ATT_WARPS * 32, 1) attention_kernel(const Attn
             Ps[k * KC + lane + 32] = p1;
         }
         __syncwarp();
-        // values: lane owns dimensions lane + 32 d
-        for (int j = 0; j < nk; ++j) {
-            float vd[D];
+        // values: lane owns dimensions lane + 32 d; the probabilities are read 4 keys at a time
+        // (positions of the chunk past nk hold p = 0 and finite staged values)
+        const float4* p4 = reinterpret_cast<const float4*>(Ps);
+        for (int j = 0; j < nk; j += 4) {
+            float vd[4][D];
 #pragma unroll
-            for (int d = 0; d < D; ++d) vd[d] = Vs[j * HD + lane + 32 * d];
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int d = 0; d < D; ++d) vd[u][d] = Vs[(j + u) * HD + lane + 32 * d];
 #pragma unroll
             for (int k = 0; k < MAXI; ++k) {
-                const float p = Ps[k * KC + j];
+                const float4 p = p4[(k * KC + j) / 4];
 #pragma unroll
-                for (int d = 0; d < D; ++d) acc[k][d] = fmaf(p, vd[d], acc[k][d]);
+                for (int d = 0; d < D; ++d)
+                    acc[k][d] = fmaf(p.x, vd[0][d], fmaf(p.y, vd[1][d], fmaf(p.z, vd[2][d], fmaf(p.w, vd[3][d], acc[k][d]))));
             }
         }
         __syncwarp();

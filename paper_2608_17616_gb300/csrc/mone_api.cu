@@ -766,8 +766,7 @@ mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out
             return e != cudaSuccess ? e : launch_read_norm(s, Q, L, K_out, V_out, strides, sx);
         }
         if (s.dtype == MONE_BF16) {  // tensor-core read: bf16 queries and hidden activations in the scratch
-            e = launch_query_transform(s, Xq, Q, s.Uq, true, sx);
-            return e != cudaSuccess ? e : launch_read_tc(s, m->maps, s.Uq, s.Aq, Q, L, K_out, V_out, strides, sx);
+            return launch_read_tc(s, m->maps, Xq, s.Uq, s.Aq, s.Oq, Q, L, K_out, V_out, strides, sx);
         }
         e = launch_query_transform(s, Xq, Q, s.Uq, false, sx);
         return e != cudaSuccess ? e : launch_read(s, Q, L, K_out, V_out, strides, sx);

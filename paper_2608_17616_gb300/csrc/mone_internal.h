@@ -97,6 +97,9 @@ struct SegWork {
 cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st);
 // Query transform of the read into U ([C][Q][d_in]: fp32, or bf16 when bf16_out).
 cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, void* U, bool bf16_out, cudaStream_t st);
+// The read's query side on the bf16 path in one pass: Z = SiLU(alpha x + gamma) unnormalised
+// (bf16 [C][Q][d_in]) and zinv = 1/|z| per query ([C][Q]) in paper mode; Z = x in plain mode.
+cudaError_t launch_query_z(const DevState& s, const void* Xq, int Q, void* Z, float* zinv, cudaStream_t st);
 
 // ---- kernels in ttl_simt.cu (fp32 path, state upkeep, read path)
 cudaError_t launch_phase_a_f32(const DevState& s, const SegWork& w, cudaStream_t st);
@@ -177,10 +180,11 @@ cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputM
 cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,
                               cudaStream_t st);
 int tc_kernels_per_segment();
-// Memory read on the tensor cores (bf16 path): Uq = transformed queries (bf16 [C][Q][d_in]),
-// Aq = bf16 scratch [C][Q][d_hid]; writes K/V (bf16) with the caller's strides.
-cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, void* Aq, int Q, int n_layers,
-                           void* K_out, void* V_out, const long long* strides, cudaStream_t st);
+// The whole memory read on the tensor cores (bf16 path), query side included: Xq bf16
+// [C][Q][d_in]; Uq, Aq bf16 scratch [C][Q][d_in], [C][Q][d_hid]; zq fp32 scratch [C][Q]; writes
+// K/V (bf16) with the caller's strides.
+cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Xq, void* Uq, void* Aq, float* zq, int Q,
+                           int n_layers, void* K_out, void* V_out, const long long* strides, cudaStream_t st);
 // Squared-error pre-pass of one segment (two kernels): M(u) at the segment's starting
 // weights and the residual targets y - M(u) into s.Kres / s.Vres (plus the loss into w.loss).
 cudaError_t launch_mse_tc(const DevState& s, const TcMaps& m, const TcInputMaps& in, const SegWork& w,

@@ -299,6 +299,77 @@ cudaError_t launch_prepass(const DevState& s, const SegWork& w, cudaStream_t st)
     return s.dtype == 0 ? launch_one<float, float>(a, w.nc, st) : launch_one<bf16, bf16>(a, w.nc, st);
 }
 
+// Query side of the read on the bf16 path, in one pass: one warp per (chain, query token).
+// Paper mode: z = SiLU(alpha x + gamma), stored in bf16 unnormalised, and 1/|z| per token into
+// zinv (the read scales each query's pre-activation by it: the row scale commutes with the
+// contraction over d_in, Sec. 3.3's L2 normalisation); plain mode: z = x.  A lane's x, alpha
+// and gamma loads of a 4-vector group are all issued before any arithmetic.
+__global__ void __launch_bounds__(256) query_z_kernel(const bf16* X, int Q, int d, int paper, const float* alpha,
+                                                      const float* gamma, bf16* Z, float* zinv, int total) {
+    // the read's hidden kernel, launched after this one with programmatic stream serialisation,
+    // may start now; it waits for this grid's completion before it reads Z or zinv
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    if (row >= total) return;
+    const int c = row / Q;
+    const bf16* x = X + (size_t)row * d;
+    bf16* z = Z + (size_t)row * d;
+    const float* al = paper ? alpha + (size_t)c * d : nullptr;
+    const float* ga = paper ? gamma + (size_t)c * d : nullptr;
+    float ss = 0.f;
+    constexpr int G = 4;  // 16-byte vectors of a group
+    for (int base = lane * 8; base < d; base += G * 256) {
+        uint4 xr[G];
+        float4 av[G][2], gv[G][2];
+#pragma unroll
+        for (int q = 0; q < G; ++q) {
+            const int i0 = base + q * 256;
+            if (i0 < d) {
+                xr[q] = __ldg(reinterpret_cast<const uint4*>(x + i0));
+                if (paper) {
+                    av[q][0] = __ldg(reinterpret_cast<const float4*>(al + i0));
+                    av[q][1] = __ldg(reinterpret_cast<const float4*>(al + i0 + 4));
+                    gv[q][0] = __ldg(reinterpret_cast<const float4*>(ga + i0));
+                    gv[q][1] = __ldg(reinterpret_cast<const float4*>(ga + i0 + 4));
+                }
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < G; ++q) {
+            const int i0 = base + q * 256;
+            if (i0 >= d) break;
+            if (!paper) {
+                *reinterpret_cast<uint4*>(z + i0) = xr[q];
+                continue;
+            }
+            float xv[8];
+            Vec<bf16>::unpack(xr[q], xv);
+            const float a8[8] = {av[q][0].x, av[q][0].y, av[q][0].z, av[q][0].w,
+                                 av[q][1].x, av[q][1].y, av[q][1].z, av[q][1].w};
+            const float g8[8] = {gv[q][0].x, gv[q][0].y, gv[q][0].z, gv[q][0].w,
+                                 gv[q][1].x, gv[q][1].y, gv[q][1].z, gv[q][1].w};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const float zp = fmaf(a8[e], xv[e], g8[e]);
+                xv[e] = zp * sig<bf16>(zp);
+                ss = fmaf(xv[e], xv[e], ss);
+            }
+            store_vec<bf16, 8>(z + i0, xv);
+        }
+    }
+    if (paper) {
+        ss = warp_sum(ss);
+        if (lane == 0) zinv[row] = 1.0f / sqrtf(ss + 1e-12f);
+    }
+}
+
+cudaError_t launch_query_z(const DevState& s, const void* Xq, int Q, void* Z, float* zinv, cudaStream_t st) {
+    const int total = s.C * Q;
+    query_z_kernel<<<(total + 7) / 8, 256, 0, st>>>(static_cast<const bf16*>(Xq), Q, s.d_in, s.mode == 1, s.alpha,
+                                                    s.gamma, static_cast<bf16*>(Z), zinv, total);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, void* U, bool bf16_out, cudaStream_t st) {
     PrepassArgs a{};
     a.X = Xq;

@@ -1082,10 +1082,7 @@ cudaError_t launch_read_noalloc(const DevState& s, const TcMaps* tc, const void*
     t.Uq = base;
     t.Aq = t.Uq + (size_t)s.C * Q * s.d_in;
     t.Oq = t.Aq + (size_t)s.C * Q * s.d_hid;
-    if (tc) {
-        e = launch_query_transform(t, Xq, Q, t.Uq, true, st);
-        return e != cudaSuccess ? e : launch_read_tc(t, *tc, t.Uq, t.Aq, Q, n_layers, K_out, V_out, strides, st);
-    }
+    if (tc) return launch_read_tc(t, *tc, Xq, t.Uq, t.Aq, t.Oq, Q, n_layers, K_out, V_out, strides, st);
     e = launch_query_transform(t, Xq, Q, t.Uq, false, st);
     return e != cudaSuccess ? e : launch_read(t, Q, n_layers, K_out, V_out, strides, st);
 }

@@ -1197,6 +1197,7 @@ struct ReadArgs {
     float lr;
     const float *eta, *eta_in;
     long long eta_cstride;
+    const float* qzinv;    // read with the weights as M: 1/|z| per query [C][Q] (paper mode), or null
 };
 
 enum { READ_HIDDEN = 0, MSE_HIDDEN = 1, MSE_OUT = 2 };  // other MODEs: read out with heads of width MODE
@@ -1435,27 +1436,33 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 // weight tile is the tcgen05 A operand (M = 128 weight rows) and the queries are the B
 // operand (N = NT = Q rounded up to 32), so neither an MMA row nor a staged query row is
 // padding and each CTA takes in half the query bytes of the 128-query form.
-//   hidden (HD = 0):  D[h][q] = W1[h] . u_q;  A_q[q][h] = SiLU(D[h][q]), bf16 [C][Q][d_hid],
-//                     stored through a per-warp 32 x 32 transpose so each row leaves as
-//                     64 contiguous bytes
+//   hidden (HD = 0):  D[h][q] = W1[h] . z_q;  A_q[q][h] = SiLU(D[h][q] / |z_q|) (paper mode; the
+//                     unnormalised z_q = SiLU(alpha x_q + gamma) comes from query_z_kernel, and
+//                     the row scale commutes with the contraction), bf16 [C][Q][d_hid], stored
+//                     through a per-warp 32 x 32 transpose so each row leaves as 64 contiguous bytes
 //   out (HD = 64/128): D[o][q] = sum_h W2[h][o] A_q[q][h] (W2 MN-major); per head of HD
 //                     features the RMS of each query's HD values is a reduction across the
 //                     head's TMEM lanes (warp transpose-sums, then shared memory), then the
 //                     gate, then the store into the caller's K / V (lanes = contiguous features)
-// Warp 0 streams the weight tile and the query rows with TMA (up to 8 stages), warp 1 issues
+// Warp 0 streams the weight tile and the query rows with TMA (4 to 8 stages), warp 1 issues
 // the MMAs into one NT-column TMEM accumulator, warps 2..5 (one TMEM lane quarter each) run
 // the epilogue.  Query rows >= Q arrive as TMA zero fill and are never stored.
+// Both kernels are launched with programmatic stream serialisation: a CTA may start while the
+// kernel before it (the query transform, or the hidden kernel) is still running, loads the
+// weight tiles of its first stages, which that kernel does not write, and only then waits for
+// that kernel's completion (griddepcontrol.wait) before it loads the query rows it produced.
 constexpr int RT_THREADS = 6 * 32;
 constexpr int RT_MAX_NT = 256;
 constexpr int RT_A = 128 * BK * 2;  // 16 KB: the weight tile of one k-block
 __host__ __device__ constexpr int rt_stage(int nt) { return RT_A + nt * BK * 2; }
 __host__ __device__ constexpr int rt_stages(int nt) { return (192 * 1024) / rt_stage(nt) < 8 ? (192 * 1024) / rt_stage(nt) : 8; }
 // shared memory after the ring: barriers, TMEM slot and flag, then the epilogue's buffers:
-// 4 warps x 2 KB transposes (hidden) or 4 x NT column partial sums + 2 x NT scales (out)
+// 4 warps x 2 KB transposes and the queries' 1/|z| (hidden), or 4 x NT column partial sums +
+// 2 x NT scales (out)
 __host__ __device__ constexpr int rt_bars(int nt) { return rt_stages(nt) * rt_stage(nt); }
 __host__ __device__ constexpr int rt_epi(int nt) { return rt_bars(nt) + 256; }
 __host__ __device__ constexpr int rt_dyn(int nt) {
-    return rt_epi(nt) + (4 * 2048 > 6 * nt * 4 ? 4 * 2048 : 6 * nt * 4) + 1024;
+    return rt_epi(nt) + (4 * 2048 + RT_MAX_NT * 4 > 6 * nt * 4 ? 4 * 2048 + RT_MAX_NT * 4 : 6 * nt * 4) + 1024;
 }
 static_assert(rt_dyn(RT_MAX_NT) <= 227 * 1024 && rt_dyn(32) <= 227 * 1024, "read shared memory budget");
 
@@ -1493,21 +1500,35 @@ tc_read_t_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
     const uint32_t tmem = *slot;
     const int q0 = blockIdx.x * NT, n0 = blockIdx.y * 128, c = blockIdx.z;
     const int KB = (OUT ? a.d_hid : a.d_in) / BK;
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");  // the out kernel may start
 
     if (warp == 0) {
         if (lane == 0) {
             tma_prefetch_map(&tmW);
             tma_prefetch_map(&tmQ);
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % NST;
-                if (kb >= NST && !mbar_wait(empty(s), ((kb / NST) - 1) & 1, a.status)) break;
-                const uint32_t sa = smem_u32(base + s * STAGE), sb = sa + RT_A, fb = full(s);
-                mbar_expect_tx(fb, STAGE);
+            auto load_w = [&](int kb, uint32_t sa, uint32_t fb) {
                 if (OUT) {  // W2 rows kb*64.. as [64 hidden][64 outputs] boxes: the MN-major A operand
                     tma_load_3d(sa, &tmW, fb, n0, kb * BK, a.b_chain0 + c);
                     tma_load_3d(sa + BOX, &tmW, fb, n0 + 64, kb * BK, a.b_chain0 + c);
                 } else {
                     tma_load_3d(sa, &tmW, fb, kb * BK, n0, a.b_chain0 + c);
+                }
+            };
+            // the first stages' weight tiles, then the wait for the kernel that writes the queries
+            const int pre = KB < NST ? KB : NST;
+            for (int kb = 0; kb < pre; ++kb) {
+                const uint32_t sa = smem_u32(base + kb * STAGE), fb = full(kb);
+                mbar_expect_tx(fb, STAGE);
+                load_w(kb, sa, fb);
+            }
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            for (int kb = 0; kb < KB; ++kb) {
+                const int s = kb % NST;
+                const uint32_t sa = smem_u32(base + s * STAGE), sb = sa + RT_A, fb = full(s);
+                if (kb >= pre) {
+                    if (!mbar_wait(empty(s), ((kb / NST) - 1) & 1, a.status)) break;
+                    mbar_expect_tx(fb, STAGE);
+                    load_w(kb, sa, fb);
                 }
                 tma_load_3d(sb, &tmQ, fb, kb * BK, a.a_row0 + q0, a.a_chain0 + c);
             }
@@ -1537,6 +1558,12 @@ tc_read_t_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
     } else {
         const int q = warp & 3;  // TMEM lane quarter: weight rows n0 + 32 q .. + 31
         const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+        float* zs = reinterpret_cast<float*>(epi + 4 * 2048);  // hidden: 1/|z| of the tile's queries
+        if constexpr (!OUT) {
+            asm volatile("griddepcontrol.wait;" ::: "memory");  // zinv comes from the kernel before
+            for (int j = threadIdx.x - 64; j < NT; j += 128)
+                zs[j] = (a.qzinv && q0 + j < a.Q) ? a.qzinv[(size_t)c * a.Q + q0 + j] : 1.f;
+        }
         if (threadIdx.x == 64) *flag = mbar_wait(tfull, 0, a.status) ? 1 : 0;
         __syncwarp();
         named_bar_sync(R_EPI_BAR, 128);
@@ -1554,7 +1581,8 @@ tc_read_t_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
                     tmem_ld32(lane_base + cc * 32, v);
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
-                        const bf16 b = __float2bfloat16_rn(v[j] * sigmoidf_(v[j]));
+                        const float x = v[j] * zs[cc * 32 + j];
+                        const bf16 b = __float2bfloat16_rn(x * sigmoidf_(x));
                         stg[j * 32 + lane] = *reinterpret_cast<const uint16_t*>(&b);
                     }
                     __syncwarp();
@@ -1827,11 +1855,18 @@ cudaError_t launch_mse_tc(const DevState& s, const TcMaps& m, const TcInputMaps&
     return launch_read_kernel<MSE_OUT>(dim3(s.T / 128, s.d_out / 128, w.nc), m.Amse, m.W2m, a, st);
 }
 
-cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, void* Aq, int Q, int n_layers,
-                           void* K_out, void* V_out, const long long* strides, cudaStream_t st) {
+cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Xq, void* Uq, void* Aq, float* zq, int Q,
+                           int n_layers, void* K_out, void* V_out, const long long* strides, cudaStream_t st) {
     cudaError_t e = ensure_attrs();
     if (e != cudaSuccess) return e;
     if (s.hd != 64 && s.hd != 128) return cudaErrorInvalidValue;
+    // the query side: unnormalised z and 1/|z| for the read with the weights as M (Q <= 256),
+    // the normalised u for the 128-query form
+    if (Q <= RT_MAX_NT)
+        e = launch_query_z(s, Xq, Q, Uq, zq, st);
+    else
+        e = launch_query_transform(s, Xq, Q, Uq, true, st);
+    if (e != cudaSuccess) return e;
     CUtensorMap mu, ma;
     if (!encode_map_bf16_3d(&mu, Uq, s.d_in, Q, s.C, 64, 128) || !encode_map_bf16_3d(&ma, Aq, s.d_hid, Q, s.C, 64, 128))
         return cudaErrorInvalidValue;
@@ -1845,18 +1880,26 @@ cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Uq, v
     a.s0 = strides[0]; a.s1 = strides[1]; a.s2 = strides[2]; a.s3 = strides[3];
     a.status = s.status;
     if (Q <= RT_MAX_NT) {  // weights as the 128-row operand, the queries as N
+        a.qzinv = s.mode == 1 ? zq : nullptr;
         const int NT = (Q + 31) / 32 * 32;
         CUtensorMap tu, ta;
         if (!encode_map_bf16_3d(&tu, Uq, s.d_in, Q, s.C, 64, NT) || !encode_map_bf16_3d(&ta, Aq, s.d_hid, Q, s.C, 64, NT))
             return cudaErrorInvalidValue;
-        const size_t dyn = rt_dyn(NT);
-        tc_read_t_kernel<0><<<dim3(1, s.d_hid / 128, s.C), RT_THREADS, dyn, st>>>(m.W1b, tu, a, NT);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-        if (s.hd == 64)
-            tc_read_t_kernel<64><<<dim3(1, s.d_out / 128, s.C), RT_THREADS, dyn, st>>>(m.W2m, ta, a, NT);
-        else
-            tc_read_t_kernel<128><<<dim3(1, s.d_out / 128, s.C), RT_THREADS, dyn, st>>>(m.W2m, ta, a, NT);
-        return cudaGetLastError();
+        // programmatic stream serialisation: each kernel may start before the one it follows ends
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        at[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.blockDim = dim3(RT_THREADS);
+        cfg.dynamicSmemBytes = rt_dyn(NT);
+        cfg.stream = st;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        cfg.gridDim = dim3(1, s.d_hid / 128, s.C);
+        if ((e = cudaLaunchKernelEx(&cfg, tc_read_t_kernel<0>, m.W1b, tu, a, NT)) != cudaSuccess) return e;
+        cfg.gridDim = dim3(1, s.d_out / 128, s.C);
+        if (s.hd == 64) return cudaLaunchKernelEx(&cfg, tc_read_t_kernel<64>, m.W2m, ta, a, NT);
+        return cudaLaunchKernelEx(&cfg, tc_read_t_kernel<128>, m.W2m, ta, a, NT);
     }
     const int nq = (Q + 127) / 128;
     if ((e = launch_read_kernel<0>(dim3(nq, s.d_hid / 128, s.C), mu, m.W1b, a, st)) != cudaSuccess) return e;
