@@ -370,7 +370,82 @@ cudaError_t launch_query_z(const DevState& s, const void* Xq, int Q, void* Z, fl
     return cudaGetLastError();
 }
 
+// Query side of the read, normalised (the SwiGLU read, the fp32 read and the 128-query form):
+// one warp per (chain, query token), d_in <= 2048.  A lane keeps its z values in registers, so
+// the row is read once: z = SiLU(alpha x + gamma), then u = z / sqrt(|z|^2 + 1e-12) (paper mode),
+// u = x in plain mode.  The loads of a 4-vector group are issued before any arithmetic.
+constexpr int QU_MAX_D = 2048;
+template <typename Tin, typename Tout>
+__global__ void __launch_bounds__(256) query_u_kernel(const Tin* X, int Q, int d, int paper, const float* alpha,
+                                                      const float* gamma, Tout* U, int total) {
+    constexpr int V = Vec<Tin>::N;                 // elements per 16-byte load
+    constexpr int MAXV = QU_MAX_D / (32 * V);      // vectors per lane
+    constexpr int G = 4;
+    const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    if (row >= total) return;
+    const int c = row / Q;
+    const Tin* x = X + (size_t)row * d;
+    Tout* u = U + (size_t)row * d;
+    const float* al = paper ? alpha + (size_t)c * d : nullptr;
+    const float* ga = paper ? gamma + (size_t)c * d : nullptr;
+    float zv[MAXV][V];
+    float ss = 0.f;
+#pragma unroll
+    for (int k0 = 0; k0 < MAXV; k0 += G) {
+        uint4 xr[G];
+        float av[G][V], gv[G][V];
+#pragma unroll
+        for (int k = 0; k < G; ++k) {
+            const int i0 = (lane + 32 * (k0 + k)) * V;
+            if (i0 < d) {
+                xr[k] = __ldg(reinterpret_cast<const uint4*>(x + i0));
+                if (paper) {
+                    load_f32<V>(al + i0, av[k]);
+                    load_f32<V>(ga + i0, gv[k]);
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < G; ++k) {
+            const int i0 = (lane + 32 * (k0 + k)) * V;
+            if (i0 < d) {
+                Vec<Tin>::unpack(xr[k], zv[k0 + k]);
+                if (paper) {
+#pragma unroll
+                    for (int e = 0; e < V; ++e) {
+                        const float zp = fmaf(av[k][e], zv[k0 + k][e], gv[k][e]);
+                        zv[k0 + k][e] = zp * sig<Tin>(zp);
+                        ss = fmaf(zv[k0 + k][e], zv[k0 + k][e], ss);
+                    }
+                }
+            }
+        }
+    }
+    const float inv = paper ? 1.0f / sqrtf(warp_sum(ss) + 1e-12f) : 1.0f;
+#pragma unroll
+    for (int k = 0; k < MAXV; ++k) {
+        const int i0 = (lane + 32 * k) * V;
+        if (i0 < d) {
+#pragma unroll
+            for (int e = 0; e < V; ++e) zv[k][e] *= inv;
+            store_vec<Tout, V>(u + i0, zv[k]);
+        }
+    }
+}
+
+template <typename Tin, typename Tout>
+cudaError_t launch_query_u(const DevState& s, const void* Xq, int Q, void* U, cudaStream_t st) {
+    const int total = s.C * Q;
+    query_u_kernel<Tin, Tout><<<(total + 7) / 8, 256, 0, st>>>(static_cast<const Tin*>(Xq), Q, s.d_in, s.mode == 1,
+                                                               s.alpha, s.gamma, static_cast<Tout*>(U), total);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_query_transform(const DevState& s, const void* Xq, int Q, void* U, bool bf16_out, cudaStream_t st) {
+    if (s.d_in <= QU_MAX_D) {  // one warp per query row, its values kept in registers
+        if (s.dtype == 0) return launch_query_u<float, float>(s, Xq, Q, U, st);
+        return bf16_out ? launch_query_u<bf16, bf16>(s, Xq, Q, U, st) : launch_query_u<bf16, float>(s, Xq, Q, U, st);
+    }
     PrepassArgs a{};
     a.X = Xq;
     a.x_cstride = (long long)Q * s.d_in;

@@ -1444,7 +1444,7 @@ tc_read_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 //                     features the RMS of each query's HD values is a reduction across the
 //                     head's TMEM lanes (warp transpose-sums, then shared memory), then the
 //                     gate, then the store into the caller's K / V (lanes = contiguous features)
-// Warp 0 streams the weight tile and the query rows with TMA (4 to 8 stages), warp 1 issues
+// Warp 0 streams the weight tile and the query rows with TMA (2 to 8 stages), warp 1 issues
 // the MMAs into one NT-column TMEM accumulator, warps 2..5 (one TMEM lane quarter each) run
 // the epilogue.  Query rows >= Q arrive as TMA zero fill and are never stored.
 // Both kernels are launched with programmatic stream serialisation: a CTA may start while the
@@ -1455,32 +1455,40 @@ constexpr int RT_THREADS = 6 * 32;
 constexpr int RT_MAX_NT = 256;
 constexpr int RT_A = 128 * BK * 2;  // 16 KB: the weight tile of one k-block
 __host__ __device__ constexpr int rt_stage(int nt) { return RT_A + nt * BK * 2; }
-__host__ __device__ constexpr int rt_stages(int nt) { return (192 * 1024) / rt_stage(nt) < 8 ? (192 * 1024) / rt_stage(nt) : 8; }
+// Ring budget: 192 KB (one CTA per SM) when the grid fits in one wave; 96 KB (two CTAs per SM,
+// one's epilogue overlapping the other's loads) when it takes several.
+constexpr int RT_RING_1 = 192 * 1024, RT_RING_2 = 96 * 1024;
+__host__ __device__ constexpr int rt_stages(int nt, int ring = RT_RING_1) {
+    return ring / rt_stage(nt) < 8 ? ring / rt_stage(nt) : 8;
+}
 // shared memory after the ring: barriers, TMEM slot and flag, then the epilogue's buffers:
 // 4 warps x 2 KB transposes and the queries' 1/|z| (hidden), or 4 x NT column partial sums +
 // 2 x NT scales (out)
-__host__ __device__ constexpr int rt_bars(int nt) { return rt_stages(nt) * rt_stage(nt); }
-__host__ __device__ constexpr int rt_epi(int nt) { return rt_bars(nt) + 256; }
-__host__ __device__ constexpr int rt_dyn(int nt) {
-    return rt_epi(nt) + (4 * 2048 + RT_MAX_NT * 4 > 6 * nt * 4 ? 4 * 2048 + RT_MAX_NT * 4 : 6 * nt * 4) + 1024;
+__host__ __device__ constexpr int rt_bars(int nt, int ring = RT_RING_1) { return rt_stages(nt, ring) * rt_stage(nt); }
+__host__ __device__ constexpr int rt_epi(int nt, int ring = RT_RING_1) { return rt_bars(nt, ring) + 256; }
+__host__ __device__ constexpr int rt_dyn(int nt, int ring = RT_RING_1) {
+    return rt_epi(nt, ring) + (4 * 2048 + RT_MAX_NT * 4 > 6 * nt * 4 ? 4 * 2048 + RT_MAX_NT * 4 : 6 * nt * 4) + 1024;
 }
 static_assert(rt_dyn(RT_MAX_NT) <= 227 * 1024 && rt_dyn(32) <= 227 * 1024, "read shared memory budget");
+static_assert(rt_dyn(RT_MAX_NT, RT_RING_2) <= 113 * 1024 && rt_dyn(32, RT_RING_2) <= 113 * 1024,
+              "two read CTAs per SM");
+static_assert(rt_stages(RT_MAX_NT, RT_RING_2) >= 2, "read pipeline depth");
 
 template <int HD>
-__global__ void __launch_bounds__(RT_THREADS, 1)
+__global__ void __launch_bounds__(RT_THREADS, 2)
 tc_read_t_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmQ, const ReadArgs a,
-                 int NT) {
+                 int NT, int ring) {
     constexpr bool OUT = HD != 0;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const int NST = rt_stages(NT), STAGE = rt_stage(NT);
-    const uint32_t bars = smem_u32(base + rt_bars(NT));
+    const int NST = rt_stages(NT, ring), STAGE = rt_stage(NT);
+    const uint32_t bars = smem_u32(base + rt_bars(NT, ring));
     auto full = [&](int s) { return bars + 8 * s; };
     auto empty = [&](int s) { return bars + 8 * (8 + s); };
     const uint32_t tfull = bars + 8 * 16;
-    uint32_t* slot = reinterpret_cast<uint32_t*>(base + rt_bars(NT) + 8 * 17);
-    int* flag = reinterpret_cast<int*>(base + rt_bars(NT) + 8 * 17 + 8);
-    uint8_t* epi = base + rt_epi(NT);
+    uint32_t* slot = reinterpret_cast<uint32_t*>(base + rt_bars(NT, ring) + 8 * 17);
+    int* flag = reinterpret_cast<int*>(base + rt_bars(NT, ring) + 8 * 17 + 8);
+    uint8_t* epi = base + rt_epi(NT, ring);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
         for (int s = 0; s < NST; ++s) {
@@ -1891,15 +1899,19 @@ cudaError_t launch_read_tc(const DevState& s, const TcMaps& m, const void* Xq, v
         at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
         at[0].val.programmaticStreamSerializationAllowed = 1;
         cfg.blockDim = dim3(RT_THREADS);
-        cfg.dynamicSmemBytes = rt_dyn(NT);
         cfg.stream = st;
         cfg.attrs = at;
         cfg.numAttrs = 1;
+        // one CTA per SM with the deep ring when a kernel's tiles fit in one wave, else two
+        const int ring1 = (long long)(s.d_hid / 128) * s.C <= g_sms ? RT_RING_1 : RT_RING_2;
+        const int ring2 = (long long)(s.d_out / 128) * s.C <= g_sms ? RT_RING_1 : RT_RING_2;
         cfg.gridDim = dim3(1, s.d_hid / 128, s.C);
-        if ((e = cudaLaunchKernelEx(&cfg, tc_read_t_kernel<0>, m.W1b, tu, a, NT)) != cudaSuccess) return e;
+        cfg.dynamicSmemBytes = rt_dyn(NT, ring1);
+        if ((e = cudaLaunchKernelEx(&cfg, tc_read_t_kernel<0>, m.W1b, tu, a, NT, ring1)) != cudaSuccess) return e;
         cfg.gridDim = dim3(1, s.d_out / 128, s.C);
-        if (s.hd == 64) return cudaLaunchKernelEx(&cfg, tc_read_t_kernel<64>, m.W2m, ta, a, NT);
-        return cudaLaunchKernelEx(&cfg, tc_read_t_kernel<128>, m.W2m, ta, a, NT);
+        cfg.dynamicSmemBytes = rt_dyn(NT, ring2);
+        if (s.hd == 64) return cudaLaunchKernelEx(&cfg, tc_read_t_kernel<64>, m.W2m, ta, a, NT, ring2);
+        return cudaLaunchKernelEx(&cfg, tc_read_t_kernel<128>, m.W2m, ta, a, NT, ring2);
     }
     const int nq = (Q + 127) / 128;
     if ((e = launch_read_kernel<0>(dim3(nq, s.d_hid / 128, s.C), mu, m.W1b, a, st)) != cudaSuccess) return e;
