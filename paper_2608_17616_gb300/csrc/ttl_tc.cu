@@ -750,7 +750,9 @@ struct BTiles {
     }
 };
 
-template <bool PAIR>
+// STEP: also sum |mu_s|^2 per chain (the per-segment metrics); a separate instance, so the update
+// loop of the ordinary one keeps its registers
+template <bool PAIR, bool STEP>
 __global__ void __launch_bounds__(B_THREADS, 1)
 tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant__ CUtensorMap tmKb,
                   const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmDH,
@@ -1069,7 +1071,7 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                     if (a.momentum) Ms[j * B_BM + col] = mn;
                     if (wr) st_bf16_hint(bp + j * width, __float2bfloat16_rn(wn), wpol);
                     v[j] = wn * wn;  // a NaN or Inf weight makes its row's sum non-finite
-                    step = fmaf(mn, mn, step);
+                    if constexpr (STEP) step = fmaf(mn, mn, step);
                 }
                 // transpose-reduce: afterwards lane j holds this warp's 32-column partial of row j
 #pragma unroll
@@ -1090,11 +1092,11 @@ tc_phase_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constan
                 if (lane == 0) mbar_arrive(sdone(k));
             }
             if (!ok) break;
-            if (a.step_sq) {  // per-segment metric: the tile's share of |mu_s|^2
+            if constexpr (STEP) {  // per-segment metric: the tile's share of |mu_s|^2
                 const float t = warp_sum(step);
                 if (lane == 0) atomicAdd(&a.step_sq[cz], t);
+                step = 0.f;
             }
-            step = 0.f;
         }
         if (!finite) atomicOr(a.status, DEV_NONFINITE);
     }
@@ -1700,10 +1702,16 @@ cudaError_t ensure_attrs() {
         if (g_attr_err == cudaSuccess)
             g_attr_err = cudaFuncSetAttribute(tc_phase_a_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, LA::DYN);
         if (g_attr_err == cudaSuccess)
-            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               LayoutB::DYN);
         if (g_attr_err == cudaSuccess)
-            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              LayoutB::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              LayoutB2::DYN);
+        if (g_attr_err == cudaSuccess)
+            g_attr_err = cudaFuncSetAttribute(tc_phase_b_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               LayoutB2::DYN);
         if (g_attr_err == cudaSuccess)
             g_attr_err =
@@ -1734,7 +1742,7 @@ cudaError_t ensure_attrs() {
             }
             cfg.blockDim = dim3(B_THREADS);
             cfg.dynamicSmemBytes = LayoutB2::DYN;
-            if (cudaOccupancyMaxActiveClusters(&g_pairb_clusters, tc_phase_b_kernel<true>, &cfg) != cudaSuccess) {
+            if (cudaOccupancyMaxActiveClusters(&g_pairb_clusters, tc_phase_b_kernel<true, false>, &cfg) != cudaSuccess) {
                 cudaGetLastError();
                 g_pairb_clusters = 0;
             }
@@ -1813,13 +1821,20 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
         cfg.stream = st;
         cfg.attrs = at;
         cfg.numAttrs = 1;
-        return cudaLaunchKernelEx(&cfg, tc_phase_b_kernel<true>, U, in.Kb, in.Vb, m.dH, m.At, m.W1s, m.W2s, m.M1s,
-                                  m.M2s, a);
+        if (a.step_sq)
+            return cudaLaunchKernelEx(&cfg, tc_phase_b_kernel<true, true>, U, in.Kb, in.Vb, m.dH, m.At, m.W1s, m.W2s,
+                                      m.M1s, m.M2s, a);
+        return cudaLaunchKernelEx(&cfg, tc_phase_b_kernel<true, false>, U, in.Kb, in.Vb, m.dH, m.At, m.W1s, m.W2s,
+                                  m.M1s, m.M2s, a);
     }
     const int ntiles = w.nc * ((s.d_in + s.d_out) / B_BM) * (s.d_hid / B_BN);
     const int grid = ntiles < g_sms ? ntiles : g_sms;
-    tc_phase_b_kernel<false><<<grid, B_THREADS, LayoutB::DYN, st>>>(U, in.Kb, in.Vb, m.dH, m.At, m.W1s, m.W2s, m.M1s,
-                                                                     m.M2s, a);
+    if (a.step_sq)
+        tc_phase_b_kernel<false, true><<<grid, B_THREADS, LayoutB::DYN, st>>>(U, in.Kb, in.Vb, m.dH, m.At, m.W1s,
+                                                                              m.W2s, m.M1s, m.M2s, a);
+    else
+        tc_phase_b_kernel<false, false><<<grid, B_THREADS, LayoutB::DYN, st>>>(U, in.Kb, in.Vb, m.dH, m.At, m.W1s,
+                                                                               m.W2s, m.M1s, m.M2s, a);
     return cudaGetLastError();
 }
 

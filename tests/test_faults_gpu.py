@@ -72,6 +72,10 @@ def test_argument_errors_launch_nothing():
     Ko = torch.empty(1, 2, 2, 16, 64, dtype=torch.bfloat16, device="cuda")
     assert code_of(mone.mone_mem_generate_kv, run.h, Xq, 0, Ko, Ko, (0, 0, 0, 0)) == 1
     assert code_of(mone.mone_mem_generate_kv, run.h, Xq, 16, Ko, Ko, (-1, 0, 0, 0)) == 1
+    seg = torch.zeros(8, wl.chains, device="cuda")
+    assert code_of(mone.mone_ttl_context_metrics, run.h, run.X, run.K, run.V, wl.N, seg.data_ptr() + 2, None) == 1
+    assert code_of(mone.mone_ttl_context_metrics, run.h, run.X, run.K, run.V, wl.N, None, seg.data_ptr() + 1) == 1
+    assert code_of(mone.mone_ttl_context_metrics, run.h, run.X, run.K, run.V, 0, seg, seg) == 1
     assert mone.mone_mem_launch_count(run.h) == before
     run.close()
 
