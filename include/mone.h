@@ -170,13 +170,14 @@ mone_status mone_ttl_context(mone_mem* m, const void* X, const void* K, const vo
  * element [s * C + c] of
  *   seg_loss  is L_s of chain c: the segment mean of Eq. 7's loss (or of the
  *             squared-error variant) at the segment's starting weights;
- *   seg_step  is |mu_s|_F^2 of chain c: the squared Frobenius norm over W1 and W2
- *             of the step of Eq. 8 (W_s = W_{s-1} - mu_s, before the row
+ *   seg_step  is |mu_s|_F^2 of chain c: the squared Frobenius norm over all fast
+ *             weights (W1 and W2; for the SwiGLU memory W_in, W_gate and W_out of
+ *             every head) of the step of Eq. 8 (W_s = W_{s-1} - mu_s, before the row
  *             renormalisation; without momentum mu_s is the rate-weighted gradient).
  * Both are fp32 device buffers of S * C elements owned by the caller, 4-byte
  * aligned; either may be null.  The library zeroes them on the stream first, then
  * accumulates into them.  Same inputs, state update and ordering as mone_ttl_context.
- * Errors: INVALID_ARG, CUDA, and UNSUPPORTED for seg_step on a SwiGLU-memory handle.
+ * Errors: INVALID_ARG, CUDA.
  */
 mone_status mone_ttl_context_metrics(mone_mem* m, const void* X, const void* K, const void* V, long long N,
                                      float* seg_loss, float* seg_step, void* stream);

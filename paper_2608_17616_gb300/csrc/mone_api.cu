@@ -696,11 +696,6 @@ mone_status mone_ttl_context_metrics(mone_mem* m, const void* X, const void* K, 
     if ((seg_loss && (reinterpret_cast<uintptr_t>(seg_loss) & 3u)) ||
         (seg_step && (reinterpret_cast<uintptr_t>(seg_step) & 3u)))
         return MONE_ERR_INVALID_ARG;
-    if (seg_step && s.memory == MONE_MEM_SWIGLU) {
-        std::snprintf(g_last_error, sizeof(g_last_error),
-                      "mone_ttl_context_metrics: the step norm is not available for the SwiGLU memory");
-        return MONE_ERR_UNSUPPORTED;
-    }
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const long long S = (N + s.T - 1) / s.T;
     if (seg_loss) MONE_CUDA(cudaMemsetAsync(seg_loss, 0, (size_t)S * s.C * sizeof(float), st));

@@ -68,6 +68,7 @@ struct SwArgs {
     float* sumsq;            // [2 parity][2 matrix][C*H][2F]
     bf16 *dPG, *Zt;          // [C*H][T][2F], [C*H][T][F]
     float* loss;             // [nc] or null
+    float* step_sq;          // [nc] squared norm of this segment's Eq. 8 step (phase B), or null
     int* status;
     // memory read
     int Q, d_out;
@@ -370,6 +371,8 @@ struct SwBTiles {
     }
 };
 
+// STEP: also sum |mu_s|^2 per chain (the per-segment metrics), in a separate instance
+template <bool STEP>
 __global__ void __launch_bounds__(SWB_THREADS, 1)
 swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant__ CUtensorMap tmKb,
                 const __grid_constant__ CUtensorMap tmVb, const __grid_constant__ CUtensorMap tmPG,
@@ -543,6 +546,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
         float* bred = tab + SWB_N / 2;                                                  // [4]
         int* flag = reinterpret_cast<int*>(base + L::FLAG) + grp * 2;
         bool finite = true;
+        float step = 0.f;        // sum of mu_s^2 over this thread's live elements of the current tile
         uint32_t tile_seq0 = 0;  // state chunk sequence number of the current tile's first chunk
         int local = 0;
         for (int t = blockIdx.x; t < tl.count; t += gridDim.x, ++local) {
@@ -624,6 +628,7 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
                     Ws[j * 128 + col] = wn;
                     if (a.momentum) Ms[j * 128 + col] = mn;
                     if (live) st_bf16_hint(bp + (size_t)j * a.dh, __float2bfloat16_rn(wn), wpol);
+                    if constexpr (STEP) step = live ? fmaf(mn, mn, step) : step;
                     v[j] = wn * wn;  // columns past dh hold zeros; a NaN or Inf makes its row's sum non-finite
                 }
                 // transpose-reduce: afterwards lane j holds this warp's 32-column partial of row j
@@ -645,6 +650,11 @@ swiglu_b_kernel(const __grid_constant__ CUtensorMap tmUb, const __grid_constant_
                 if (lane == 0) mbar_arrive(sdone(k));
             }
             if (!ok) break;
+            if constexpr (STEP) {  // per-segment metric: the tile's share of |mu_s|^2
+                const float t = warp_sum(step);
+                if (lane == 0) atomicAdd(&a.step_sq[cz], t);
+                step = 0.f;
+            }
             tile_seq0 += nch;
             // the scale table is rewritten for the next tile only after every warp of the group is done
             named_bar_sync(bar_id, SWB_EPI_THREADS);
@@ -837,13 +847,16 @@ cudaError_t g_sw_err = cudaSuccess;
 
 cudaError_t sw_attrs() {
     std::call_once(g_sw_once, [] {
-        const void* ks[] = {reinterpret_cast<const void*>(swiglu_a_kernel), reinterpret_cast<const void*>(swiglu_b_kernel),
-                            reinterpret_cast<const void*>(swiglu_rh_kernel), reinterpret_cast<const void*>(swiglu_ro_kernel)};
+        const void* kb[] = {reinterpret_cast<const void*>(swiglu_b_kernel<false>),
+                            reinterpret_cast<const void*>(swiglu_b_kernel<true>)};
+        const void* ks[] = {reinterpret_cast<const void*>(swiglu_a_kernel), reinterpret_cast<const void*>(swiglu_rh_kernel),
+                            reinterpret_cast<const void*>(swiglu_ro_kernel)};
+        for (const void* k : kb)
+            if (g_sw_err == cudaSuccess)
+                g_sw_err = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, SwLayoutB::DYN);
         for (const void* k : ks)
             if (g_sw_err == cudaSuccess)
-                g_sw_err = cudaFuncSetAttribute(
-                    k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                    k == reinterpret_cast<const void*>(swiglu_b_kernel) ? SwLayoutB::DYN : SwLayout::DYN);
+                g_sw_err = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, SwLayout::DYN);
     });
     return g_sw_err;
 }
@@ -864,7 +877,7 @@ SwArgs sw_args(const DevState& s, const SegWork& w) {
     a.W1 = s.W1; a.W2 = s.W2; a.mu1 = s.mu1; a.mu2 = s.mu2; a.W1b = s.W1b; a.W2b = s.W2b;
     a.n1 = s.n1; a.n2 = s.n2; a.sumsq = s.sumsq;
     a.dPG = static_cast<bf16*>(s.dHt); a.Zt = static_cast<bf16*>(s.Att);
-    a.loss = w.loss; a.status = s.status;
+    a.loss = w.loss; a.step_sq = w.step_sq; a.status = s.status;
     a.d_out = s.d_out;
     return a;
 }
@@ -891,8 +904,12 @@ cudaError_t launch_swiglu_phase_b(const DevState& s, const SwMaps& m, const SwIn
     a.nc_launch = w.nc;
     const int ntiles = w.nc * a.H * 3 * ((a.F + SWB_N - 1) / SWB_N) * ((a.dh + 127) / 128);
     const int grid = ntiles < sw_sms() ? ntiles : sw_sms();
-    swiglu_b_kernel<<<grid, SWB_THREADS, SwLayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.PG, m.Z,
-                                                               m.W1s, m.M1s, m.W2s, m.M2s, a);
+    if (a.step_sq)
+        swiglu_b_kernel<true><<<grid, SWB_THREADS, SwLayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.PG,
+                                                                         m.Z, m.W1s, m.M1s, m.W2s, m.M2s, a);
+    else
+        swiglu_b_kernel<false><<<grid, SWB_THREADS, SwLayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.PG,
+                                                                          m.Z, m.W1s, m.M1s, m.W2s, m.M2s, a);
     return cudaGetLastError();
 }
 

@@ -724,18 +724,11 @@ def test_context_metrics_per_segment(case):
     S = -(-wl.N // wl.seg_T)
     loss = torch.full((S, wl.chains), 7.0, device="cuda")
     step = torch.full((S, wl.chains), 7.0, device="cuda")
-    if case == "swiglu":
-        with pytest.raises(mone.MoneError) as ei:
-            mone.mone_ttl_context_metrics(run.h, run.X, run.K, run.V, wl.N, loss, step)
-        assert ei.value.code == 7  # MONE_ERR_UNSUPPORTED: no step norm for the SwiGLU memory
-        mone.mone_ttl_context_metrics(run.h, run.X, run.K, run.V, wl.N, loss, None)
-    else:
-        mone.mone_ttl_context_metrics(run.h, run.X, run.K, run.V, wl.N, loss, step)
+    mone.mone_ttl_context_metrics(run.h, run.X, run.K, run.V, wl.N, loss, step)
     mone.mone_mem_sync(run.h)
     W1, W2, _, _ = run.state()
-    if case != "swiglu":
-        for c in range(wl.chains):
-            check_chain(run, c, W1, W2, tol)
+    for c in range(wl.chains):
+        check_chain(run, c, W1, W2, tol)
     loss, step = loss.cpu().double().numpy(), step.cpu().double().numpy()
     name = "f32" if tol == F32_TOL else "bf16"
     for c in range(wl.chains):
@@ -744,8 +737,7 @@ def test_context_metrics_per_segment(case):
             L = losses[s]
             e = record(name, "seg loss", abs(loss[s, c] - L) / max(1.0, abs(L)), tol)
             assert e <= tol, (c, s, loss[s, c], L)
-            if case != "swiglu":
-                m2 = sum(float(np.sum(v * v)) for v in trail[s].mu.values())
-                e = record(name, "seg |mu|^2", abs(step[s, c] - m2) / m2, tol)
-                assert e <= tol, (c, s, step[s, c], m2)
+            m2 = sum(float(np.sum(v * v)) for v in trail[s].mu.values())
+            e = record(name, "seg |mu|^2", abs(step[s, c] - m2) / m2, tol)
+            assert e <= tol, (c, s, step[s, c], m2)
     run.close()
