@@ -3,14 +3,16 @@
 // tokens visible to every query token and the query tokens causal among themselves;
 // query head h reads key/value head h / (n_q / n_kv) (grouped heads).
 //
-// A small, bandwidth-bound contraction, run on the CUDA cores in flash-decode form: a CTA
-// takes one (chain, key/value head, tile of query tokens) and stages the cache rows its
-// tokens can see through shared memory in chunks of KC = 64 positions (converted to fp32
-// once, shared by every query head of the group).  Each warp owns up to MAXI (query
-// head, token) items: per chunk, lane l scores keys l and l + 32 against every item
-// (queries in shared memory), the chunk's max and sum are reduced once per item, and
-// the probabilities pass through shared memory into the value accumulation, where a
-// lane owns hd / 32 dimensions.
+// Two forms.  bf16 with 16-byte-aligned rows runs on the tensor cores
+// (attention_tc_kernel: S = Q K^T and O = P V as tcgen05 MMAs with TMEM accumulators, the
+// softmax one row per thread in between).  fp32, and bf16 caches with other strides, run
+// on the CUDA cores in flash-decode form: a CTA takes one (chain, key/value head, tile of
+// query tokens) and stages the cache rows its tokens can see through shared memory in
+// chunks of KC = 64 positions (converted to fp32 once, shared by every query head of the
+// group).  Each warp owns up to MAXI (query head, token) items: per chunk, lane l scores
+// keys l and l + 32 against every item (queries in shared memory), the chunk's max and sum
+// are reduced once per item, and the probabilities pass through shared memory into the
+// value accumulation, where a lane owns hd / 32 dimensions.
 #include <algorithm>
 #include <mutex>
 
@@ -33,6 +35,7 @@ struct AttnArgs {
     int L, n_q, n_kv, group, Lq, n_mem, rows;  // rows: query tokens per CTA (group * rows <= ATT_ITEMS)
     float scale;            // 1 / sqrt(hd)
     int vec;                // caches 16-byte aligned (base and every stride): stage with 16-byte loads
+    int* status;            // device status word (bounded waits of the tensor-core form)
 };
 
 // Stage cache positions [j0, j0 + nk) of one head into shared memory as fp32 rows of HD
@@ -204,28 +207,303 @@ __global__ void __launch_bounds__(ATT_WARPS * 32, 2) attention_kernel(const Attn
     }
 }
 
+// ---------------------------------------------------------------- tensor-core form (bf16)
+// One CTA of 512 threads per (chain, key/value head, tile of query tokens).  Its 128 rows are
+// (query head of the group, token) pairs, `rows` = 128 / group tokens of each of the group's
+// heads, so the group's heads share every staged key and value row.  Keys are taken in chunks
+// of up to AT_NC positions: S = Q K^T accumulates in TMEM columns [0, AT_NC).  Four threads
+// share a row (TMEM lane): each reads its 32-key blocks of the row, the row max is exchanged
+// through shared memory, and each writes its bf16 probabilities to shared memory and
+// keeps its own part of the row sum.  O_c = P V accumulates in TMEM columns [AT_NC, AT_NC + HD),
+// of which each of the four threads takes hd / 4; the running max rescales the output columns
+// and the partial sums from one chunk to the next, and the partial sums meet once at the end.
+// Q, K and V reach shared memory through 16-byte asynchronous copies (cp.async, zero-filled
+// past the last key), all in flight at once, written in the 128-byte-swizzled layout the MMA
+// descriptors read: Q, K and P as K-major operands, V as the MN-major B operand of P V (a value
+// row holds 64 dimensions per 128-byte line, the same bytes as a key row).  S = Q K^T is issued
+// once the queries and keys have landed, with the values still in flight.
+constexpr int AT_THREADS = 512;
+constexpr int AT_GROUPS = AT_THREADS / 128;  // threads per row, each with its own columns
+constexpr int AT_NC = 256;     // key positions per chunk: S's MMA N and TMEM columns
+constexpr int AT_TMEM = 512;   // S (AT_NC columns) + O (HD <= 128 columns), a power of two
+
+template <int HD>
+struct AtSmem {
+    static constexpr int SLAB_Q = 128 * 128;    // one 64-dimension slab of the 128 query rows
+    static constexpr int SLAB_K = AT_NC * 128;  // one 64-dimension slab of AT_NC key (or value) rows
+    static constexpr int SLAB_P = 128 * 128;    // one 64-key slab of the 128 probability rows
+    static constexpr int Q_OFF = 0;
+    static constexpr int K_OFF = Q_OFF + (HD / 64) * SLAB_Q;
+    static constexpr int V_OFF = K_OFF + (HD / 64) * SLAB_K;
+    // hd 128: the probabilities take the key buffer (the same size; keys are dead once S is in TMEM)
+    static constexpr int P_OFF = HD == 128 ? K_OFF : V_OFF + (HD / 64) * SLAB_K;
+    static constexpr int RED_OFF = HD == 128 ? V_OFF + (HD / 64) * SLAB_K : P_OFF + (AT_NC / 64) * SLAB_P;
+    static constexpr int BAR_OFF = RED_OFF + AT_GROUPS * 128 * 4;
+    static constexpr int DYN = BAR_OFF + 64 + 1024;  // + barriers, TMEM slot, flag; + alignment slack
+};
+static_assert(AtSmem<128>::DYN <= 227 * 1024 && AtSmem<64>::DYN <= 227 * 1024, "attention tile exceeds shared memory");
+
+// Byte offset of 16-byte piece `p` (0..7) of row `r` in a 128-byte-swizzled slab (8-row atoms).
+__device__ __forceinline__ uint32_t sw128_off(int r, int p) { return r * 128 + ((p ^ (r & 7)) << 4); }
+
+// 16-byte asynchronous copy global -> shared; src_bytes 0 fills the 16 bytes with zeros.
+__device__ __forceinline__ void at_cp16(uint32_t dst, const void* src, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void at_cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+// Wait until at most N of this thread's committed copy groups are still pending.
+template <int N>
+__device__ __forceinline__ void at_cp_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Issue the copies of n_pad rows of HD bf16 into 64-dimension slabs `slab` bytes apart; row r
+// comes from row_ptr(r) (16-byte aligned) when r < n and row_ptr(r) is non-null, else it is
+// zero-filled (from `any`, a valid global address of which no byte is read).  Nothing waits
+// here: every copy of the tile is in flight at once.
+template <int HD, typename RowPtr>
+__device__ __forceinline__ void at_stage(uint8_t* dst, int slab, int n, int n_pad, const bf16* any, RowPtr row_ptr) {
+    constexpr int VPR = HD / 8;  // 16-byte pieces per row
+    const uint32_t d0 = smem_u32(dst);
+    for (int e = threadIdx.x; e < n_pad * VPR; e += AT_THREADS) {
+        const int r = e / VPR, v = e - r * VPR;
+        const bf16* p = r < n ? row_ptr(r) : nullptr;
+        at_cp16(d0 + (v >> 3) * slab + sw128_off(r, v & 7), p ? p + v * 8 : any, p ? 16 : 0);
+    }
+}
+
+// 2^x on the special-function unit (PTX ex2.approx: relative error ~2^-22, far below the
+// bf16 rounding of the probabilities it feeds).
+__device__ __forceinline__ float at_exp2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+template <int HD>
+__global__ void __launch_bounds__(AT_THREADS, 1) attention_tc_kernel(const AttnArgs a) {
+    using SM = AtSmem<HD>;
+    constexpr int OC = HD / AT_GROUPS;  // output columns per thread
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* Qs = base + SM::Q_OFF;
+    uint8_t* Ks = base + SM::K_OFF;
+    uint8_t* Vs = base + SM::V_OFF;
+    uint8_t* Ps = base + SM::P_OFF;
+    float* red = reinterpret_cast<float*>(base + SM::RED_OFF);  // [AT_GROUPS][128] per-row partials
+    const uint32_t bar_s = smem_u32(base + SM::BAR_OFF), bar_o = bar_s + 8;
+    uint32_t* slot = reinterpret_cast<uint32_t*>(base + SM::BAR_OFF + 16);
+    int* abort_flag = reinterpret_cast<int*>(base + SM::BAR_OFF + 24);
+    const int tid = threadIdx.x, warp = tid >> 5;
+    // thread -> (row, column group): a warp reaches TMEM lanes 32 (warp % 4) .. + 31, so the four
+    // warps of a lane quarter share its 32 rows and split the columns
+    const int row = (warp & 3) * 32 + (tid & 31), grp = warp >> 2;
+    if (tid == 0) {
+        mbar_init(bar_s, 1);
+        mbar_init(bar_o, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(slot), AT_TMEM);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *slot;
+    const uint32_t t_row = tmem + ((uint32_t)((warp & 3) * 32) << 16);  // this thread's TMEM lane = its row
+
+    const int c = blockIdx.z, g = blockIdx.y, rt = a.rows, r0 = blockIdx.x * rt;
+    const bf16* Qb = static_cast<const bf16*>(a.Q);
+    const long long kv_off = (long long)(c / a.L) * a.s0 + (long long)(c % a.L) * a.s1 + (long long)g * a.s2;
+    const bf16* Kc = static_cast<const bf16*>(a.K) + kv_off;
+    const bf16* Vc = static_cast<const bf16*>(a.V) + kv_off;
+    // row r of the tile: query head g * group + r / rt of the group, token r0 + r % rt
+    auto q_row = [&](int r) -> const bf16* {
+        const int hr = r / rt, ir = r0 + r % rt;
+        if (hr >= a.group || ir >= a.Lq) return nullptr;
+        return Qb + (((size_t)c * a.n_q + g * a.group + hr) * a.Lq + ir) * HD;
+    };
+    const int hg = row / rt, i = r0 + row % rt;
+    const bool live = hg < a.group && i < a.Lq;
+    const int vis = live ? a.n_mem + i + 1 : 0;     // keys this row sees (causal among the query tokens)
+    const int keys = a.n_mem + min(a.Lq, r0 + rt);  // keys the tile's last token sees
+    const float k2 = a.scale * 1.4426950408889634f;  // softmax scale in base 2: exp(s x) = 2^(s log2(e) x)
+
+    at_stage<HD>(Qs, SM::SLAB_Q, 128, 128, Qb, q_row);
+    float o[OC];
+#pragma unroll
+    for (int d = 0; d < OC; ++d) o[d] = 0.f;
+    float m_run = -INFINITY, l_part = 0.f;  // row max so far; this thread's share of the row sum
+    bool ok = true;
+    int chunk = 0;
+    for (int j0 = 0; j0 < keys; j0 += AT_NC, ++chunk) {
+        const int nk = min(AT_NC, keys - j0), nc = (nk + 15) & ~15;
+        // copy groups: (the queries and) the keys, then the values, which S = Q K^T does not wait for
+        at_stage<HD>(Ks, SM::SLAB_K, nk, nc, Kc, [&](int r) { return Kc + (long long)(j0 + r) * a.s3; });
+        at_cp_commit();
+        at_stage<HD>(Vs, SM::SLAB_K, nk, nc, Vc, [&](int r) { return Vc + (long long)(j0 + r) * a.s3; });
+        at_cp_commit();
+        at_cp_wait<1>();
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {  // S = Q K^T over HD (K-major both)
+            tc_fence_after();
+            const uint32_t idesc = idesc_bf16_f32(128, nc, false, false);
+#pragma unroll
+            for (int kb = 0; kb < HD / 64; ++kb)
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    umma_bf16(tmem, sdesc_sw128(smem_u32(Qs + kb * SM::SLAB_Q) + k * 32, 16),
+                              sdesc_sw128(smem_u32(Ks + kb * SM::SLAB_K) + k * 32, 16), idesc, (kb | k) ? 1u : 0u);
+            umma_commit(bar_s);
+        }
+        if (!mbar_wait(bar_s, chunk & 1, a.status)) atomicOr(abort_flag, 1);
+        __syncthreads();
+        if (*abort_flag) {
+            ok = false;
+            break;
+        }
+        tc_fence_after();
+        // this thread's 32-key blocks of the chunk: cb = 32 (grp + AT_GROUPS k); its row sees keys [0, nv)
+        const int nv = min(max(vis - j0, 0), nc);
+        float cm = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < AT_NC / (32 * AT_GROUPS); ++k) {
+            const int cb = 32 * (grp + AT_GROUPS * k);
+            if (cb < nc) {  // uniform over the warp
+                float v[32];
+                tmem_ld32(t_row + cb, v);
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (cb + j < nv) cm = fmaxf(cm, v[j]);
+            }
+        }
+        red[grp * 128 + row] = cm;
+        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < AT_GROUPS; ++q) cm = fmaxf(cm, red[q * 128 + row]);
+        const float mn = fmaxf(m_run, cm);
+        // rescale of what earlier chunks accumulated (none yet: m_run = -inf gives 0)
+        const float corr = mn == -INFINITY ? 1.f : at_exp2((m_run - mn) * k2);
+        const float moff = mn == -INFINITY ? 0.f : -mn * k2;
+        float ps = 0.f;
+#pragma unroll
+        for (int k = 0; k < AT_NC / (32 * AT_GROUPS); ++k) {
+            const int cb = 32 * (grp + AT_GROUPS * k);
+            if (cb < nc) {
+                float v[32];  // the scores again (a TMEM reload is cheaper than holding them over the exchange)
+                tmem_ld32(t_row + cb, v);
+                uint32_t pk[16];
+#pragma unroll
+                for (int j = 0; j < 32; j += 2) {
+                    const float p0 = cb + j < nv ? at_exp2(fmaf(v[j], k2, moff)) : 0.f;
+                    const float p1 = cb + j + 1 < nv ? at_exp2(fmaf(v[j + 1], k2, moff)) : 0.f;
+                    const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
+                    const float2 pr = __bfloat1622float2(pb);  // the sum takes the probabilities the MMA sees
+                    ps += pr.x + pr.y;
+                    pk[j / 2] = *reinterpret_cast<const uint32_t*>(&pb);
+                }
+                uint8_t* prow = Ps + (cb >> 6) * SM::SLAB_P;
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    *reinterpret_cast<uint4*>(prow + sw128_off(row, ((cb & 63) >> 3) + u)) =
+                        make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+            }
+        }
+        l_part = fmaf(l_part, corr, ps);
+        at_cp_wait<0>();  // this thread's value copies
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {  // O_c = P V over the chunk's keys (P K-major, V MN-major)
+            tc_fence_after();
+            const uint32_t idesc = idesc_bf16_f32(128, HD, false, true);
+            for (int kk = 0; kk < nc / 16; ++kk)
+                umma_bf16(tmem + AT_NC, sdesc_sw128(smem_u32(Ps + (kk >> 2) * SM::SLAB_P) + (kk & 3) * 32, 16),
+                          sdesc_sw128(smem_u32(Vs) + kk * 16 * 128, SM::SLAB_K), idesc, kk ? 1u : 0u);
+            umma_commit(bar_o);
+        }
+        if (!mbar_wait(bar_o, chunk & 1, a.status)) atomicOr(abort_flag, 1);
+        __syncthreads();
+        if (*abort_flag) {
+            ok = false;
+            break;
+        }
+        tc_fence_after();
+        {  // this thread's OC output columns
+            float w[OC];
+            if constexpr (OC == 32)
+                tmem_ld32(t_row + AT_NC + grp * OC, w);
+            else
+                tmem_ld16(t_row + AT_NC + grp * OC, w);
+#pragma unroll
+            for (int d = 0; d < OC; ++d) o[d] = fmaf(o[d], corr, w[d]);
+        }
+        m_run = mn;
+        // the next chunk restages K, V (and P) and rewrites red: the MMAs that read the buffers
+        // have completed and every thread passed the barrier after its last read of red
+    }
+    red[grp * 128 + row] = l_part;
+    __syncthreads();
+    if (ok && live) {
+        float l = 0.f;
+#pragma unroll
+        for (int q = 0; q < AT_GROUPS; ++q) l += red[q * 128 + row];
+        const float inv = 1.f / l;
+        bf16* orow = static_cast<bf16*>(a.out) + (((size_t)c * a.n_q + g * a.group + hg) * a.Lq + i) * HD + grp * OC;
+#pragma unroll
+        for (int v8 = 0; v8 < OC / 8; ++v8)
+            *reinterpret_cast<uint4*>(orow + v8 * 8) =
+                make_uint4(pack_bf16(o[8 * v8] * inv, o[8 * v8 + 1] * inv), pack_bf16(o[8 * v8 + 2] * inv, o[8 * v8 + 3] * inv),
+                           pack_bf16(o[8 * v8 + 4] * inv, o[8 * v8 + 5] * inv),
+                           pack_bf16(o[8 * v8 + 6] * inv, o[8 * v8 + 7] * inv));
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, AT_TMEM);
+}
+
 std::mutex g_attr_mu;
+
+// The shared-memory opt-in belongs to a device: set it once per device and kernel (a driver
+// call on every launch would cost more than the kernel).
+template <typename K>
+cudaError_t smem_opt_in(K kernel, size_t smem, bool (&done)[64]) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_attr_mu);
+    if (!done[dev]) {
+        e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        done[dev] = true;
+    }
+    return cudaSuccess;
+}
 
 template <typename T, int HD>
 cudaError_t launch_t(const AttnArgs& a, int C, cudaStream_t st) {
     const size_t smem = AttnSmem<T, HD>::FLOATS * sizeof(float);
-    {
-        // the shared-memory opt-in belongs to a device: set it once per device (a driver call
-        // on every launch would cost more than the kernel)
-        static bool done[64] = {};
-        int dev = 0;
-        cudaError_t e = cudaGetDevice(&dev);
-        if (e != cudaSuccess) return e;
-        if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-        std::lock_guard<std::mutex> lk(g_attr_mu);
-        if (!done[dev]) {
-            e = cudaFuncSetAttribute(attention_kernel<T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-            if (e != cudaSuccess) return e;
-            done[dev] = true;
-        }
-    }
+    static bool done[64] = {};
+    cudaError_t e = smem_opt_in(attention_kernel<T, HD>, smem, done);
+    if (e != cudaSuccess) return e;
     dim3 grid((a.Lq + a.rows - 1) / a.rows, a.n_kv, C);
     attention_kernel<T, HD><<<grid, ATT_WARPS * 32, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+template <int HD>
+cudaError_t launch_tc(AttnArgs a, int C, cudaStream_t st) {
+    static bool done[64] = {};
+    cudaError_t e = smem_opt_in(attention_tc_kernel<HD>, AtSmem<HD>::DYN, done);
+    if (e != cudaSuccess) return e;
+    a.rows = 128 / a.group;  // tokens per tile: the group's heads x rows fill the 128 MMA rows
+    dim3 grid((a.Lq + a.rows - 1) / a.rows, a.n_kv, C);
+    attention_tc_kernel<HD><<<grid, AT_THREADS, AtSmem<HD>::DYN, st>>>(a);
     return cudaGetLastError();
 }
 
@@ -242,8 +520,13 @@ cudaError_t launch_attention(const DevState& s, int n_layers, const void* Q, int
     const long long el = s.dtype == 0 ? 4 : 2;
     a.vec = ((reinterpret_cast<uintptr_t>(K) | reinterpret_cast<uintptr_t>(V)) & 15u) == 0 && (a.s0 * el) % 16 == 0 &&
             (a.s1 * el) % 16 == 0 && (a.s2 * el) % 16 == 0 && (a.s3 * el) % 16 == 0;
+    a.status = s.status;
     if (s.dtype == 0)
         return s.hd == 64 ? launch_t<float, 64>(a, s.C, st) : launch_t<float, 128>(a, s.C, st);
+    // bf16 on the tensor cores when every row it stages is 16-byte aligned (the queries and the
+    // output are dense rows of hd elements); other cache layouts take the CUDA-core kernel
+    if (a.vec && ((reinterpret_cast<uintptr_t>(Q) | reinterpret_cast<uintptr_t>(out)) & 15u) == 0)
+        return s.hd == 64 ? launch_tc<64>(a, s.C, st) : launch_tc<128>(a, s.C, st);
     return s.hd == 64 ? launch_t<bf16, 64>(a, s.C, st) : launch_t<bf16, 128>(a, s.C, st);
 }
 

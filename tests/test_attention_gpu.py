@@ -4,6 +4,8 @@ The caches hold memory tokens at positions [0, n_mem) and the query tokens' own 
 values after them.  Where the case says so, the memory tokens are the library's own read
 (mone_mem_generate_kv after a test-time-learning pass); otherwise they are random.
 Tolerances: bf16 path 1e-2 (outputs rounded to bf16, fp32 accumulation), fp32 path 1e-5.
+bf16 caches whose rows are 16-byte aligned take the tensor-core kernel (keys in chunks of 256
+positions); other bf16 layouts and fp32 take the CUDA-core kernel.  Both are covered here.
 """
 import pytest
 import torch
@@ -29,15 +31,16 @@ def small(mode=wk.PAPER, dtype="bf16", n_ctx=1, n_layers=2, d_out=256, hd=64, N=
                        "bf16" else 128, N, Q, dtype, mode, 0.3 if dtype == "bf16" else 1e-2)
 
 
-def run_case(wl, n_q, Lq, n_mem, seed, memory_from_read=True):
+def run_case(wl, n_q, Lq, n_mem, seed, memory_from_read=True, pos_pad=0):
+    """pos_pad: extra elements after each cache position (a position stride of head_dim + pos_pad)."""
     run = DeviceRun(wl)
     run.ttl_context()
     dt = wl.torch_dtype()
     g = torch.Generator(device="cuda").manual_seed(seed)
     S = n_mem + Lq + 3  # spare positions at the end: the kernel must not read them
-    shape = (wl.n_ctx, wl.n_layers, wl.n_kv_heads, S, wl.head_dim)
-    Kc = torch.randn(*shape, generator=g, device="cuda").to(dt)
-    Vc = torch.randn(*shape, generator=g, device="cuda").to(dt)
+    shape = (wl.n_ctx, wl.n_layers, wl.n_kv_heads, S, wl.head_dim + pos_pad)
+    Kc = torch.randn(*shape, generator=g, device="cuda").to(dt)[..., :wl.head_dim]
+    Vc = torch.randn(*shape, generator=g, device="cuda").to(dt)[..., :wl.head_dim]
     strides = Kc.stride()[:4]
     if memory_from_read and n_mem:
         Xq = wk.query_inputs(wl, "cuda", Q=n_mem)
@@ -61,12 +64,22 @@ def check(wl, Qt, Kc, Vc, out, n_mem, Lq, tol):
     (2, 40, 40),      # query heads in pairs, memory = the read of 40 query tokens
     (1, 70, 0),       # no memory: causal self-attention; 70 tokens = two tiles, the last ragged
     (7, 20, 150),     # 7 heads per KV head (tiles of 9 tokens), memory over three 64-position chunks
-    (2, 1, 300),      # one decode token over a long memory
+    (2, 1, 300),      # one decode token over a long memory: two key chunks on the tensor cores
+    (1, 130, 400),    # 128-token tiles, the second ragged; up to 530 keys = three chunks
+    (64, 5, 10),      # the largest group: 2 tokens x 64 heads per 128-row tile
 ])
 def test_attention_bf16(group, Lq, n_mem):
     wl = small(n_ctx=2)
     n_q = group * wl.n_kv_heads
     Qt, Kc, Vc, out = run_case(wl, n_q, Lq, n_mem, seed=group * 100 + Lq)
+    check(wl, Qt, Kc, Vc, out, n_mem, Lq, 1e-2)
+
+
+@pytest.mark.parametrize("group,Lq,n_mem", [(2, 40, 40), (3, 9, 70)])
+def test_attention_bf16_unaligned_cache_rows(group, Lq, n_mem):
+    """Position stride head_dim + 4 (8 bytes past a 16-byte multiple): the CUDA-core kernel."""
+    wl = small()
+    Qt, Kc, Vc, out = run_case(wl, group * wl.n_kv_heads, Lq, n_mem, seed=31 + group, pos_pad=4)
     check(wl, Qt, Kc, Vc, out, n_mem, Lq, 1e-2)
 
 
