@@ -123,28 +123,18 @@ def kernel_work(wl, kind, chains=None):
     return flops, byts
 
 
-def e2e_breakdown(ev, h2d_bytes, chunk_tensors):
-    """Where the end-to-end step's time goes: per chunk, its host-to-device copy and its learning
-    (CUDA events on the copy stream and the learning stream), and the achieved copy rate, so a
-    slow host link can be told apart from a stall of the pipeline.  `ev[step][chunk]` holds the
-    events (copy start, copy end, learning start, learning end)."""
-    chunk_bytes = sum(t.numel() * t.element_size() for t in chunk_tensors)
-    copy_ms = [[c0.elapsed_time(c1) for c0, c1, _, _ in st] for st in ev]
-    learn_ms = [[l0.elapsed_time(l1) for _, _, l0, l1 in st] for st in ev]
-    # learning of chunk k waiting for its copy: start of learning k minus end of learning k-1
-    wait_ms = [[max(0.0, st[k - 1][3].elapsed_time(st[k][2])) for k in range(1, len(st))] for st in ev]
-    flat_c = [x for row in copy_ms for x in row]
-    flat_l = [x for row in learn_ms for x in row]
-    flat_w = [x for row in wait_ms for x in row]
-    rates = [chunk_bytes / (x / 1000) / 1e9 for x in flat_c if x > 0]
-    tot_copy = sum(flat_c)
-    return {"h2d_gbs": (h2d_bytes * len(ev)) / (tot_copy / 1000) / 1e9 if tot_copy > 0 else None,
-            "chunk_h2d_gbs": {"min": min(rates), "median": sorted(rates)[len(rates) // 2], "max": max(rates)}
-            if rates else None,
-            "chunk_copy_ms": {"min": min(flat_c), "median": sorted(flat_c)[len(flat_c) // 2], "max": max(flat_c)},
-            "chunk_learn_ms": {"min": min(flat_l), "median": sorted(flat_l)[len(flat_l) // 2], "max": max(flat_l)},
-            "learn_wait_ms_per_step": sum(flat_w) / len(ev),
-            "last_step_copy_ms": copy_ms[-1], "last_step_learn_ms": learn_ms[-1]}
+def e2e_breakdown(context_bytes, gather_ms, gathers, gather_busy_ms, step_ms):
+    """Where the end-to-end step's time goes, from one instrumented step: the library's host-input
+    gathers (kernel kind "stage": `gathers` launches, `gather_ms` summed, `gather_busy_ms` the
+    union of their intervals) moved `context_bytes` over the host link.  The achieved link rate,
+    and the share of the step during which a gather was running, tell a slow link apart from a
+    stalled pipeline (a step near the gathers' busy time is bound by the link)."""
+    busy = gather_busy_ms if gather_busy_ms > 0 else gather_ms
+    return {"h2d_gbs": context_bytes / (busy / 1000) / 1e9 if busy > 0 else None,
+            "gathers_per_step": gathers,
+            "gather_ms_mean": gather_ms / gathers if gathers else None,
+            "gather_busy_ms_per_step": busy,
+            "gather_share_of_step": busy / step_ms if step_ms > 0 else None}
 
 
 def dominant_roofline(wl, dom, d, busy_ms, timed_segments, timed_ms, pk, alu_peak=None, traffic=None):
@@ -496,80 +486,55 @@ def run_ours(args, wl):
     tokens_per_step = wl.n_ctx * wl.N
     ms, value = job_rate(ms, tokens_per_step, ws, dev)
 
-    # ---- end to end through the public calls with host buffers: the context arrives from
-    # pinned host memory in chunks of whole segments; chunk k+1 is copied (copy stream) while
-    # chunk k is learned (mone_ttl_context continues the state), then the query is read and
-    # the memory K/V are copied back.
+    # ---- end to end through the public calls with host buffers: the context is handed to the
+    # library in pinned host memory (mone_ttl_context_host), which gathers chunks of whole segments
+    # into its device windows while it learns the previous chunk; then the query is copied in, read,
+    # and the memory K/V are copied back.
     e2e = None
     if not args.no_e2e:
-        n_chunks = 8 if wl.N % (8 * wl.seg_T) == 0 else 1
-        nc_tok = wl.N // n_chunks
-        hX = [torch.empty(wl.n_ctx, wl.n_layers, nc_tok, wl.d_in, dtype=X.dtype, pin_memory=True)
-              for _ in range(n_chunks)]
-        hK = [torch.empty(wl.n_ctx, wl.n_layers, nc_tok, wl.d_out // 2, dtype=K.dtype, pin_memory=True)
-              for _ in range(n_chunks)]
-        hV = [torch.empty_like(t) for t in hK]
-        for k in range(n_chunks):
-            sl = slice(k * nc_tok, (k + 1) * nc_tok)
-            hX[k].copy_(X[:, :, sl])
-            hK[k].copy_(K[:, :, sl])
-            hV[k].copy_(V[:, :, sl])
+        hX = torch.empty(X.shape, dtype=X.dtype, pin_memory=True)
+        hK = torch.empty(K.shape, dtype=K.dtype, pin_memory=True)
+        hV = torch.empty(V.shape, dtype=V.dtype, pin_memory=True)
+        hX.copy_(X)
+        hK.copy_(K)
+        hV.copy_(V)
         hXq = torch.empty(Xq.shape, dtype=Xq.dtype, pin_memory=True)
         hXq.copy_(Xq)
         hKo = torch.empty(Kout.shape, dtype=Kout.dtype, pin_memory=True)
         hVo = torch.empty(Vout.shape, dtype=Vout.dtype, pin_memory=True)
-        dX = [torch.empty_like(hX[0], device=dev) for _ in range(2)]
-        dK = [torch.empty_like(hK[0], device=dev) for _ in range(2)]
-        dV = [torch.empty_like(hV[0], device=dev) for _ in range(2)]
         dXq = torch.empty_like(Xq)
-        copy_stream = torch.cuda.Stream()
-        copied = [torch.cuda.Event() for _ in range(n_chunks)]
-        consumed = [torch.cuda.Event() for _ in range(n_chunks)]
 
-        n_e2e = max(1, min(args.steps, 5))
-        # per step and chunk: copy start/end on the copy stream, learning start/end on the stream
-        ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_chunks)]
-              for _ in range(n_e2e + 1)]
-
-        def e2e_step(tag):
+        def e2e_step():
             mone.mone_mem_write_state(h, W1_0, W2_0, mu0_1, mu0_2)
-            for k in range(n_chunks):
-                b = k % 2
-                c0, c1, l0, l1 = ev[tag][k]
-                with torch.cuda.stream(copy_stream):
-                    if k >= 2:
-                        copy_stream.wait_event(consumed[k - 2])
-                    c0.record(copy_stream)
-                    dX[b].copy_(hX[k], non_blocking=True)
-                    dK[b].copy_(hK[k], non_blocking=True)
-                    dV[b].copy_(hV[k], non_blocking=True)
-                    if k == n_chunks - 1:
-                        dXq.copy_(hXq, non_blocking=True)
-                    c1.record(copy_stream)
-                    copied[k].record(copy_stream)
-                stream.wait_event(copied[k])
-                l0.record(stream)
-                mone.mone_ttl_context(h, dX[b], dK[b], dV[b], nc_tok)
-                l1.record(stream)
-                consumed[k].record(stream)
+            mone.mone_ttl_context_host(h, hX, hK, hV, wl.N)
+            dXq.copy_(hXq, non_blocking=True)
             mone.mone_mem_generate_kv(h, dXq, wl.Q, Kout, Vout, strides)
             hKo.copy_(Kout, non_blocking=True)
             hVo.copy_(Vout, non_blocking=True)
-        e2e_step(n_e2e)
+
+        n_e2e = max(1, min(args.steps, 5))
+        e2e_step()  # first call: the library sizes its staging windows
         torch.cuda.synchronize()
         barrier()
         e0.record(stream)
-        for i in range(n_e2e):
-            e2e_step(i)
+        for _ in range(n_e2e):
+            e2e_step()
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
         ms_e2e, _ = job_rate(e0.elapsed_time(e1) / n_e2e, tokens_per_step, ws, dev)
-        h2d = sum(t.numel() * t.element_size() for t in (*hX, *hK, *hV, hXq))
+        h2d = sum(t.numel() * t.element_size() for t in (hX, hK, hV, hXq))
         d2h = sum(t.numel() * t.element_size() for t in (hKo, hVo))
+        # one more step with the library's per-kernel timing on, for the breakdown (not timed above)
+        mone.mone_mem_set_timing(h, True)
+        e2e_step()
+        st_ms, st_n = mone.mone_mem_kernel_time(h, mone.KERNEL_KINDS.index("stage"))
+        st_busy = mone.mone_mem_kernel_busy(h, mone.KERNEL_KINDS.index("stage"))
+        mone.mone_mem_set_timing(h, False)
+        mone.mone_mem_sync(h)
         e2e = {"value": ws * tokens_per_step / (ms_e2e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e, "chunks": n_chunks}
-        e2e.update(e2e_breakdown(ev[:n_e2e], h2d, (hX[0], hK[0], hV[0])))
+               "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e, "api": "mone_ttl_context_host"}
+        e2e.update(e2e_breakdown(h2d - hXq.numel() * hXq.element_size(), st_ms, st_n, st_busy, ms_e2e))
 
     # ---- consumer attention of the read (Eq. 5): the query's tokens over [memory tokens || their own
     # keys], timed on its own (it is not part of the test-time-learning step).  The memory tokens are

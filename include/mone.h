@@ -39,7 +39,7 @@
 extern "C" {
 #endif
 
-#define MONE_ABI_VERSION 6
+#define MONE_ABI_VERSION 7
 
 typedef struct mone_mem mone_mem; /* opaque; created by mone_mem_init */
 
@@ -163,6 +163,27 @@ mone_status mone_ttl_context(mone_mem* m, const void* X, const void* K, const vo
                              long long N, void* stream);
 
 /*
+ * mone_ttl_context for a context held in HOST memory (the end-to-end form of Eq. 9's
+ * chain: the inputs arrive from the host while the memory learns).  X, K, V have the
+ * layouts of mone_ttl_context and live in host memory the device can read: page-locked
+ * (cudaHostAlloc / cudaHostRegister) or, where the device reads host memory through the
+ * host's page tables (Grace), any host memory.  The caller guarantees that each tensor's
+ * whole range is allocated: the library checks its first and last bytes only.
+ * The context is learned in chunks of chunk_tokens tokens (a multiple of seg_T; 0 lets
+ * the library choose about 512 MB of X, K and V per chunk): the library gathers chunk
+ * k+1 into one of two device windows (owned by the handle, grown on demand; growing
+ * synchronises the stream) on its own staging stream while chunk k is learned on
+ * `stream`, so the result equals mone_ttl_context on the same tokens.  Asynchronous:
+ * the host buffers must stay valid and unchanged until `stream` has passed the call
+ * (mone_mem_sync or a stream synchronisation).  Kernel kind 8 times the gathers.
+ * Errors: INVALID_ARG (null or unaligned pointer, device or managed memory, a range
+ * the device cannot read, N, chunk_tokens), UNSUPPORTED_SHAPE (a row of X, K or V not
+ * a multiple of 16 bytes), OOM (windows), CUDA.
+ */
+mone_status mone_ttl_context_host(mone_mem* m, const void* X, const void* K, const void* V, long long N,
+                                  long long chunk_tokens, void* stream);
+
+/*
  * mone_ttl_context, with per-segment metrics of every chain written into caller
  * buffers, so the learning of a whole context can be followed segment by segment
  * (Sec. 3.4's chain W_0 -> ... -> W_S).  With S = ceil(N / seg_T) segments of this
@@ -281,7 +302,8 @@ mone_status mone_attention(mone_mem* m, const void* Q, int n_q_heads, int Lq, co
  * operand refresh), 4 memory read, 5 squared-error pre-pass (M(u) and the residual
  * target, MONE_LOSS_MSE only), 6 consumer attention, 7 resident chains (the fp32 MLP
  * path when d_in + d_out <= 512: every segment of an input window in one launch,
- * forward, backward and update together).  Errors: INVALID_ARG, CUDA.
+ * forward, backward and update together), 8 host-input gathers (mone_ttl_context_host;
+ * timed on the library's staging stream).  Errors: INVALID_ARG, CUDA.
  */
 mone_status mone_mem_set_timing(mone_mem* m, int enable);
 mone_status mone_mem_kernel_time(mone_mem* m, int kind, double* ms, long long* launches);

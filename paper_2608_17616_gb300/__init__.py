@@ -34,9 +34,9 @@ EXPORTS = ("mone_mem_init", "mone_ttl_segment", "mone_ttl_context", "mone_mem_ge
            "mone_mem_read_state", "mone_mem_write_state", "mone_mem_sync", "mone_mem_launch_count",
            "mone_status_string", "mone_abi_version", "mone_mem_set_timing", "mone_mem_kernel_time",
            "mone_last_error", "mone_mem_generate_kv_noalloc", "mone_attention", "mone_mem_kernel_busy",
-           "mone_ttl_context_metrics")
+           "mone_ttl_context_metrics", "mone_ttl_context_host")
 
-KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read", "mse", "attention", "resident")
+KERNEL_KINDS = ("prepass", "phase_a", "phase_b", "finalize", "read", "mse", "attention", "resident", "stage")
 
 
 class MoneError(RuntimeError):
@@ -77,6 +77,7 @@ def lib(path: Optional[str] = None) -> ctypes.CDLL:
         "mone_ttl_segment": ([vp, i, i, vp, vp, vp, i, vp, vp, vp], i),
         "mone_ttl_context": ([vp, vp, vp, vp, ll, vp], i),
         "mone_ttl_context_metrics": ([vp, vp, vp, vp, ll, vp, vp, vp], i),
+        "mone_ttl_context_host": ([vp, vp, vp, vp, ll, ll, vp], i),
         "mone_mem_generate_kv": ([vp, vp, i, vp, vp, ctypes.POINTER(ll), vp], i),
         "mone_mem_generate_kv_noalloc": ([vp, vp, i, vp, vp, ctypes.POINTER(ll), vp], i),
         "mone_attention": ([vp, vp, i, i, vp, vp, ctypes.POINTER(ll), i, vp, vp], i),
@@ -159,6 +160,13 @@ def mone_ttl_context_metrics(h: int, X, K, V, N: int, seg_loss=None, seg_step=No
     """mone_ttl_context with per-segment loss and squared step norm ([S][C] fp32 device buffers)."""
     _check("mone_ttl_context_metrics", lib().mone_ttl_context_metrics(h, _ptr(X), _ptr(K), _ptr(V), N, _ptr(seg_loss),
                                                                       _ptr(seg_step), _stream(stream)))
+
+
+def mone_ttl_context_host(h: int, X, K, V, N: int, chunk_tokens: int = 0, stream=None):
+    """mone_ttl_context over host tensors (pinned CPU tensors, or host memory the device reads through
+    the host's page tables): the library stages chunks of whole segments into its device windows."""
+    _check("mone_ttl_context_host", lib().mone_ttl_context_host(h, _ptr(X), _ptr(K), _ptr(V), N, chunk_tokens,
+                                                                _stream(stream)))
 
 
 def mone_mem_generate_kv(h: int, Xq, Q: int, K_out, V_out, strides: Sequence[int], stream=None):

@@ -18,7 +18,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmone.so")
-SOURCES = ["mone_api.cu", "ttl_prepass.cu", "ttl_simt.cu", "ttl_tc.cu", "attention.cu", "swiglu_tc.cu"]
+SOURCES = ["mone_api.cu", "ttl_prepass.cu", "ttl_simt.cu", "ttl_tc.cu", "attention.cu", "swiglu_tc.cu", "host_stage.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

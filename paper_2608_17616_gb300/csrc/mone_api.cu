@@ -18,7 +18,7 @@ using namespace mone;
 
 // Kernel kinds of the per-kernel timing (mone_mem_kernel_time).
 enum { K_PREPASS = 0, K_PHASE_A = 1, K_PHASE_B = 2, K_FINALIZE = 3, K_READ = 4, K_MSE = 5, K_ATTN = 6,
-       K_RESIDENT = 7, K_KINDS = 8 };
+       K_RESIDENT = 7, K_STAGE = 8, K_KINDS = 9 };
 
 // Optional per-kernel device timing (mone_mem_set_timing).
 struct KernelTiming {
@@ -104,6 +104,13 @@ struct mone_mem {
     cudaEvent_t ev_fork, ev_join;    // caller stream -> side stream, side stream -> caller stream
     cudaStream_t cap;                // capture stream of the read graph (created on first capture)
     ReadGraph* rg;                   // the captured read, or null
+    // host-input pipeline (mone_ttl_context_host, created on first use): two device windows of
+    // a chunk, the staging stream, and events: hstart (the caller's stream at the call), and per
+    // window hstaged (its gather has finished) and hfree (the learning that last read it has)
+    void* hwin[2];
+    size_t hwin_bytes;
+    cudaStream_t hstream;
+    cudaEvent_t hstart, hstaged[2], hfree[2];
 };
 
 namespace {
@@ -190,7 +197,23 @@ void free_state(DevState& s) {
 
 size_t elsize(int dtype) { return dtype == MONE_FP32 ? 4 : 2; }
 
+void destroy_host_pipeline(mone_mem* m) {
+    for (int b = 0; b < 2; ++b) {
+        if (m->hwin[b]) cudaFree(m->hwin[b]);
+        if (m->hstaged[b]) cudaEventDestroy(m->hstaged[b]);
+        if (m->hfree[b]) cudaEventDestroy(m->hfree[b]);
+        m->hwin[b] = nullptr;
+        m->hstaged[b] = m->hfree[b] = nullptr;
+    }
+    if (m->hstart) cudaEventDestroy(m->hstart);
+    if (m->hstream) cudaStreamDestroy(m->hstream);
+    m->hstart = nullptr;
+    m->hstream = nullptr;
+    m->hwin_bytes = 0;
+}
+
 void destroy_streams(mone_mem* m) {
+    destroy_host_pipeline(m);
     if (m->rg) {
         if (m->rg->exec) cudaGraphExecDestroy(m->rg->exec);
         delete m->rg;
@@ -492,6 +515,42 @@ mone_status run_segments(mone_mem* m, SegWork w, long long N, cudaStream_t st) {
     return rc;
 }
 
+// The device address of `bytes` of host memory the device can read: page-locked memory
+// (cudaHostAlloc, cudaHostRegister), or any host memory where the device reads through the
+// host's page tables (Grace).  Only the first and last bytes are checked (the caller
+// guarantees the range between them).  Device and managed memory are refused:
+// mone_ttl_context takes those.
+mone_status host_device_view(const void* p, size_t bytes, const void** out) {
+    cudaPointerAttributes a{}, b{};
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess ||
+        cudaPointerGetAttributes(&b, static_cast<const uint8_t*>(p) + bytes - 1) != cudaSuccess) {
+        cudaGetLastError();
+        return MONE_ERR_INVALID_ARG;
+    }
+    if (a.type == cudaMemoryTypeHost && b.type == cudaMemoryTypeHost && a.devicePointer &&
+        static_cast<const uint8_t*>(b.devicePointer) == static_cast<const uint8_t*>(a.devicePointer) + bytes - 1) {
+        *out = a.devicePointer;
+        return MONE_OK;
+    }
+    if (a.type == cudaMemoryTypeUnregistered && b.type == cudaMemoryTypeUnregistered) {
+        int dev = 0, via_host_tables = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&via_host_tables, cudaDevAttrPageableMemoryAccessUsesHostPageTables, dev) !=
+                cudaSuccess)
+            return MONE_ERR_CUDA;
+        if (via_host_tables) {
+            *out = p;
+            return MONE_OK;
+        }
+    }
+    return MONE_ERR_INVALID_ARG;
+}
+
+// Bytes of X, K and V per staged chunk when the caller leaves the chunk length to the library:
+// large enough that a chunk's learning amortises the per-call setup, small enough that the
+// first chunk's gather (not overlapped) stays short.
+constexpr long long kHostChunkBytes = 512ll << 20;
+
 }  // namespace
 
 extern "C" {
@@ -729,6 +788,78 @@ mone_status mone_ttl_context(mone_mem* m, const void* X, const void* K, const vo
     w.eta_in = nullptr;
     w.loss = nullptr;
     return run_segments(m, w, N, st);
+}
+
+// Test-time learning of a context held in host memory: chunks of whole segments are gathered
+// into two device windows on the staging stream while the previous chunk is learned on the
+// caller's stream (the learning of each chunk is the call mone_ttl_context makes, continuing
+// the state, so the chunks together equal one call on all N tokens).
+mone_status mone_ttl_context_host(mone_mem* m, const void* X, const void* K, const void* V, long long N,
+                                  long long chunk_tokens, void* stream) {
+    if (!is_live(m)) return MONE_ERR_INVALID_ARG;
+    const DevState& s = m->s;
+    if (N < 1 || N > (1ll << 31) - 1) return MONE_ERR_INVALID_ARG;
+    if (!X || !K || !V || !aligned16(X) || !aligned16(K) || !aligned16(V)) return MONE_ERR_INVALID_ARG;
+    if (chunk_tokens < 0 || (chunk_tokens > 0 && chunk_tokens % s.T)) return MONE_ERR_INVALID_ARG;
+    const long long el = (long long)elsize(s.dtype), C = s.C;
+    const long long row_b[3] = {s.d_in * el, (s.d_out / 2) * el, (s.d_out / 2) * el};
+    if (row_b[0] % 16 || row_b[1] % 16) return MONE_ERR_UNSUPPORTED_SHAPE;  // 16-byte units per row
+    const void* hv[3];
+    const void* hp[3] = {X, K, V};
+    for (int t = 0; t < 3; ++t) MONE_TRY(host_device_view(hp[t], (size_t)(C * N * row_b[t]), &hv[t]));
+    const long long tok_b = C * (row_b[0] + row_b[1] + row_b[2]);  // bytes of one token over all chains
+    long long ct = chunk_tokens;
+    if (ct == 0) ct = std::max<long long>(s.T, kHostChunkBytes / tok_b / s.T * s.T);
+    ct = std::min(ct, (N + s.T - 1) / s.T * s.T);
+    const size_t win_bytes = (size_t)(ct * tok_b);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (!m->hstream) {
+        MONE_CUDA(cudaStreamCreateWithFlags(&m->hstream, cudaStreamNonBlocking));
+        MONE_CUDA(cudaEventCreateWithFlags(&m->hstart, cudaEventDisableTiming));
+        for (int b = 0; b < 2; ++b) {
+            MONE_CUDA(cudaEventCreateWithFlags(&m->hstaged[b], cudaEventDisableTiming));
+            MONE_CUDA(cudaEventCreateWithFlags(&m->hfree[b], cudaEventDisableTiming));
+        }
+    }
+    if (win_bytes > m->hwin_bytes) {  // grow the windows (not while earlier work may read them)
+        MONE_CUDA(cudaStreamSynchronize(st));
+        MONE_CUDA(cudaStreamSynchronize(m->hstream));
+        for (int b = 0; b < 2; ++b) {
+            if (m->hwin[b]) cudaFree(m->hwin[b]);
+            m->hwin[b] = nullptr;
+        }
+        m->hwin_bytes = 0;
+        for (int b = 0; b < 2; ++b)
+            if (cudaMalloc(&m->hwin[b], win_bytes) != cudaSuccess) {
+                cudaGetLastError();
+                return MONE_ERR_OOM;
+            }
+        m->hwin_bytes = win_bytes;
+    }
+    // the gathers start after what the caller queued before this call
+    MONE_CUDA(cudaEventRecord(m->hstart, st));
+    MONE_CUDA(cudaStreamWaitEvent(m->hstream, m->hstart, 0));
+    for (long long r0 = 0, k = 0; r0 < N; r0 += ct, ++k) {
+        const long long nr = std::min(ct, N - r0);
+        const int b = (int)(k & 1);
+        uint8_t* win = static_cast<uint8_t*>(m->hwin[b]);
+        void* dst[3] = {win, win + C * nr * row_b[0], win + C * nr * (row_b[0] + row_b[1])};
+        MONE_CUDA(cudaStreamWaitEvent(m->hstream, m->hfree[b], 0));  // never recorded: no wait
+        MONE_TRY(timed(m, K_STAGE, m->hstream, 1,
+                       [&] { return launch_stage_rows(hv, dst, row_b, N, r0, nr, s.C, m->hstream); }));
+        MONE_CUDA(cudaEventRecord(m->hstaged[b], m->hstream));
+        MONE_CUDA(cudaStreamWaitEvent(st, m->hstaged[b], 0));
+        SegWork w{};
+        w.c0 = 0;
+        w.nc = s.C;
+        w.X = dst[0]; w.K = dst[1]; w.V = dst[2];
+        w.x_cstride = nr * s.d_in;
+        w.y_cstride = nr * (s.d_out / 2);
+        w.n_rows = nr;
+        MONE_TRY(run_segments(m, w, nr, st));
+        MONE_CUDA(cudaEventRecord(m->hfree[b], st));
+    }
+    return MONE_OK;
 }
 
 mone_status mone_mem_generate_kv(mone_mem* m, const void* Xq, int Q, void* K_out, void* V_out,

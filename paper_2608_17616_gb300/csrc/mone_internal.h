@@ -159,6 +159,12 @@ cudaError_t launch_swiglu_read(const DevState& s, const SwMaps& m, const void* U
 cudaError_t launch_read_norm(const DevState& s, int Q, int n_layers, void* K_out, void* V_out,
                              const long long* strides, cudaStream_t st);
 
+// ---- kernels in host_stage.cu
+// Gather rows [r0, r0 + nr) of every chain of three host tensors ([C][N][row_bytes[t]], device
+// addresses of host memory) into device windows ([C][nr][row_bytes[t]]); row_bytes multiples of 16.
+cudaError_t launch_stage_rows(const void* const src[3], void* const dst[3], const long long row_bytes[3], long long N,
+                              long long r0, long long nr, int C, cudaStream_t st);
+
 // ---- kernels in attention.cu
 cudaError_t launch_attention(const DevState& s, int n_layers, const void* Q, int n_q, int Lq, const void* K,
                              const void* V, const long long* strides, int n_mem, void* out, cudaStream_t st);

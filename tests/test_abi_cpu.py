@@ -35,7 +35,7 @@ def test_library_exports_every_declared_symbol(L):
     raw = ctypes.CDLL(mone.LIB_PATH)
     for name in header_functions():
         assert hasattr(raw, name), name
-    assert L.mone_abi_version() == 6
+    assert L.mone_abi_version() == 7
 
 
 def test_status_strings(L):
@@ -139,4 +139,4 @@ def test_debug_build_compiles_and_exports_every_symbol():
     for name in header_functions():
         assert hasattr(raw, name), name
     raw.mone_abi_version.restype = ctypes.c_int
-    assert raw.mone_abi_version() == 6
+    assert raw.mone_abi_version() == 7

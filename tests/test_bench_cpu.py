@@ -86,36 +86,13 @@ def test_dominant_roofline_is_the_tensor_work_of_the_path():
     assert roof["hbm"]["frac"] == pytest.approx(494.5e6 / 116.79e-6 / 1e9 / 6681.8, rel=1e-3)
 
 
-class _Ev:
-    """A stand-in for a CUDA event: a time stamp in ms."""
-
-    def __init__(self, t):
-        self.t = t
-
-    def elapsed_time(self, other):
-        return other.t - self.t
-
-
 def test_e2e_breakdown_separates_the_link_from_the_pipeline():
-    # two steps of 3 chunks: copies of 10, 40, 20 ms; learning of 5 ms each, starting when its copy
-    # has landed or the previous chunk's learning has ended
-    steps = []
-    for _ in range(2):
-        ev, t_copy, t_learn = [], 0.0, 0.0
-        for c in (10.0, 40.0, 20.0):
-            c0, c1 = t_copy, t_copy + c
-            l0 = max(c1, t_learn)
-            l1 = l0 + 5.0
-            ev.append((_Ev(c0), _Ev(c1), _Ev(l0), _Ev(l1)))
-            t_copy, t_learn = c1, l1
-        steps.append(ev)
-    chunk = (type("T", (), {"numel": lambda self: 1000, "element_size": lambda self: 1000})(),)
-    out = bench.e2e_breakdown(steps, 3e6, chunk)
-    assert out["chunk_copy_ms"] == {"min": 10.0, "median": 20.0, "max": 40.0}
-    assert out["chunk_learn_ms"]["median"] == 5.0
-    # 1 MB chunks at 10, 40, 20 ms
-    assert out["chunk_h2d_gbs"]["max"] == pytest.approx(1e6 / 10e-3 / 1e9)
-    assert out["h2d_gbs"] == pytest.approx(2 * 3e6 / (2 * 70e-3) / 1e9)
-    # the learning of chunk 1 waited from 15 (chunk 0 learned) to 50 (its copy landed): 35 ms; of
-    # chunk 2 from 55 to 70: 15 ms
-    assert out["learn_wait_ms_per_step"] == pytest.approx(35.0 + 15.0)
+    # 26 gathers of 4 ms each, busy 104 ms of a 110 ms step, 20.8 GB over the link: the step is
+    # bound by the link (96% of it has a gather running), which ran at 200 GB/s
+    out = bench.e2e_breakdown(20.8e9, 104.0, 26, 104.0, 110.0)
+    assert out["h2d_gbs"] == pytest.approx(200.0)
+    assert out["gathers_per_step"] == 26 and out["gather_ms_mean"] == pytest.approx(4.0)
+    assert out["gather_share_of_step"] == pytest.approx(104.0 / 110.0)
+    # overlapping gathers (busy below the summed time): the rate uses the busy time
+    out = bench.e2e_breakdown(10e9, 80.0, 10, 50.0, 100.0)
+    assert out["h2d_gbs"] == pytest.approx(200.0) and out["gather_share_of_step"] == pytest.approx(0.5)
