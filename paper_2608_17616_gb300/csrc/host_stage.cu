@@ -6,8 +6,10 @@
 // Why SM loads and not the copy engines: on this part both top out at the link's read rate
 // (211 GB/s measured), but copy-engine transfers fell to 24-50 GB/s for stretches of a
 // multi-GB pinned footprint, while SM loads held 211 GB/s on every chunk.  A small grid
-// suffices (32 CTAs already reach 208 GB/s): the kernel runs beside the learning kernels,
-// whose CTAs leave room for a 256-thread CTA of ~40 registers on every SM.
+// suffices (32 CTAs reach 208 GB/s alone): the kernel runs beside the learning kernels, whose
+// CTAs leave room for a 256-thread CTA of 48 registers on an SM.  Larger grids slowed the
+// learning they share the SMs with (a 128K-token step through mone_ttl_context_host: 24-32
+// CTAs 71-72 ms, 48 CTAs 75 ms, 96-152 CTAs 82-93 ms), smaller ones lost link rate.
 #include "mone_common.cuh"
 
 namespace mone {
@@ -16,7 +18,7 @@ namespace {
 
 constexpr int ST_THREADS = 256;
 constexpr int ST_UNROLL = 8;  // 16-byte loads in flight per thread (32 KB per CTA)
-constexpr int ST_GRID = 48;
+constexpr int ST_GRID = 32;
 
 struct StageArgs {
     const uint4* src[3];   // host tensors (device addresses) [C][N][row16[t]] in 16-byte units
