@@ -243,20 +243,6 @@ struct AtSmem {
 };
 static_assert(AtSmem<128>::DYN <= 227 * 1024 && AtSmem<64>::DYN <= 227 * 1024, "attention tile exceeds shared memory");
 
-// Byte offset of 16-byte piece `p` (0..7) of row `r` in a 128-byte-swizzled slab (8-row atoms).
-__device__ __forceinline__ uint32_t sw128_off(int r, int p) { return r * 128 + ((p ^ (r & 7)) << 4); }
-
-// 16-byte asynchronous copy global -> shared; src_bytes 0 fills the 16 bytes with zeros.
-__device__ __forceinline__ void at_cp16(uint32_t dst, const void* src, int src_bytes) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
-}
-__device__ __forceinline__ void at_cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-// Wait until at most N of this thread's committed copy groups are still pending.
-template <int N>
-__device__ __forceinline__ void at_cp_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
 // Issue the copies of n_pad rows of HD bf16 into 64-dimension slabs `slab` bytes apart; row r
 // comes from row_ptr(r) (16-byte aligned) when r < n and row_ptr(r) is non-null, else it is
 // zero-filled (from `any`, a valid global address of which no byte is read).  Nothing waits
@@ -268,7 +254,7 @@ __device__ __forceinline__ void at_stage(uint8_t* dst, int slab, int n, int n_pa
     for (int e = threadIdx.x; e < n_pad * VPR; e += AT_THREADS) {
         const int r = e / VPR, v = e - r * VPR;
         const bf16* p = r < n ? row_ptr(r) : nullptr;
-        at_cp16(d0 + (v >> 3) * slab + sw128_off(r, v & 7), p ? p + v * 8 : any, p ? 16 : 0);
+        cpa16(d0 + (v >> 3) * slab + sw128_off(r, v & 7), p ? p + v * 8 : any, p ? 16 : 0);
     }
 }
 
@@ -342,10 +328,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attention_tc_kernel(const AttnA
         const int nk = min(AT_NC, keys - j0), nc = (nk + 15) & ~15;
         // copy groups: (the queries and) the keys, then the values, which S = Q K^T does not wait for
         at_stage<HD>(Ks, SM::SLAB_K, nk, nc, Kc, [&](int r) { return Kc + (long long)(j0 + r) * a.s3; });
-        at_cp_commit();
+        cpa_commit();
         at_stage<HD>(Vs, SM::SLAB_K, nk, nc, Vc, [&](int r) { return Vc + (long long)(j0 + r) * a.s3; });
-        at_cp_commit();
-        at_cp_wait<1>();
+        cpa_commit();
+        cpa_wait(1);
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
@@ -414,7 +400,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attention_tc_kernel(const AttnA
             }
         }
         l_part = fmaf(l_part, corr, ps);
-        at_cp_wait<0>();  // this thread's value copies
+        cpa_wait(0);  // this thread's value copies
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();

@@ -124,6 +124,27 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* st
     }
 }
 
+// ------------------------------------------------------------------ cp.async (16-byte copies on the LSU path)
+// Copy 16 bytes global -> shared (`dst` in the shared window); src_bytes 0 writes 16 zero
+// bytes and reads nothing (src must still be a valid global address).
+__device__ __forceinline__ void cpa16(uint32_t dst, const void* src, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cpa_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+// Wait until at most n (0..4; larger n waits as for 4) of this thread's committed groups are pending.
+__device__ __forceinline__ void cpa_wait(int n) {
+    switch (n) {
+        case 0: asm volatile("cp.async.wait_group 0;" ::: "memory"); break;
+        case 1: asm volatile("cp.async.wait_group 1;" ::: "memory"); break;
+        case 2: asm volatile("cp.async.wait_group 2;" ::: "memory"); break;
+        case 3: asm volatile("cp.async.wait_group 3;" ::: "memory"); break;
+        default: asm volatile("cp.async.wait_group 4;" ::: "memory"); break;
+    }
+}
+// Byte offset of 16-byte piece p (0..7) of 128-byte line r in a 128-byte-swizzled tile (8-line
+// atoms, 1024-byte aligned): the layout a SWIZZLE_128B tensor copy writes and the MMA reads.
+__device__ __forceinline__ uint32_t sw128_off(int r, int p) { return r * 128 + ((p ^ (r & 7)) << 4); }
+
 // ------------------------------------------------------------------ TMA
 __device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* m) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
