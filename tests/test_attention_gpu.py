@@ -83,10 +83,14 @@ def test_attention_bf16_unaligned_cache_rows(group, Lq, n_mem):
     check(wl, Qt, Kc, Vc, out, n_mem, Lq, 1e-2)
 
 
-def test_attention_bf16_head_dim_128_random_memory():
+@pytest.mark.parametrize("Lq,n_mem", [
+    (33, 77),    # one key chunk
+    (5, 400),    # two key chunks: at hd 128 the probabilities take the key buffer, restaged per chunk
+])
+def test_attention_bf16_head_dim_128_random_memory(Lq, n_mem):
     wl = small(d_out=512, hd=128)
-    Qt, Kc, Vc, out = run_case(wl, 3 * wl.n_kv_heads, 33, 77, seed=5, memory_from_read=False)
-    check(wl, Qt, Kc, Vc, out, 77, 33, 1e-2)
+    Qt, Kc, Vc, out = run_case(wl, 3 * wl.n_kv_heads, Lq, n_mem, seed=5 + n_mem, memory_from_read=False)
+    check(wl, Qt, Kc, Vc, out, n_mem, Lq, 1e-2)
 
 
 def test_attention_fp32():

@@ -6,7 +6,7 @@ mone_ttl_context called on the same chunks from device memory, and the state mus
 oracle's chain (Eq. 9) within the path's tolerance (bf16 2e-2, fp32 1e-4; see test_parity_gpu).
 
 "Equal" is bit for bit where the learning is deterministic: plain mode and the fp32 resident
-kernel.  With row renormalisation (paper mode) on the bf16 and fp32 tiled paths, phase B adds a
+kernel.  With row renormalisation (paper mode) on the bf16 (MLP and SwiGLU) and fp32 tiled paths, phase B adds a
 row's sum of squares from its column tiles with float atomics, so two runs of the same call
 differ in the last bits of the renormalisation scale; there the bound is relative (bf16 1e-3,
 the bound of the split-context test, which also covers bf16 rounding flips that such a bit
@@ -19,6 +19,7 @@ import paper_2608_17616_gb300 as mone
 import workloads as wk
 from harness import DeviceRun, rel_fro
 from test_parity_gpu import BF16_TOL, F32_TOL, check_chain, small
+from test_swiglu_gpu import check as check_swiglu, swiglu
 
 pytestmark = pytest.mark.gpu
 
@@ -63,6 +64,7 @@ CASES = [
     ("bf16_plain", 256, 0.0),
     ("f32_tiled", 3 * 64, 1e-5),
     ("f32_resident", 3 * 128, 0.0),
+    ("swiglu", 2 * 256, 1e-3),
 ]
 
 
@@ -73,6 +75,8 @@ def workload(name):
         return small(wk.PLAIN)
     if name == "f32_tiled":
         return small(wk.PAPER, "f32", n_ctx=1, T=64, N=7 * 64 + 20, d_in=512, d_hid=128, d_out=256, lr=0.5)
+    if name == "swiglu":  # the per-head SwiGLU of Eq. 3: 2 heads of 128, ragged hidden tiles (96 units)
+        return swiglu(T=256, N=4 * 256 + 37)
     return wk.WORKLOADS["tiny_f32"]
 
 
@@ -89,10 +93,13 @@ def test_host_context_equals_device_chunks_and_the_oracle(name, chunk, same):
     b = DeviceRun(wl)
     device_chunks(b, ct)
     assert_same_state(a, b, same)
-    W1, W2, _, _ = a.state()
-    tol = F32_TOL if wl.dtype == "f32" else BF16_TOL
-    for c in range(wl.chains):
-        check_chain(a, c, W1, W2, tol)
+    if wl.memory == "swiglu":
+        check_swiglu(a, range(wl.chains))
+    else:
+        W1, W2, _, _ = a.state()
+        tol = F32_TOL if wl.dtype == "f32" else BF16_TOL
+        for c in range(wl.chains):
+            check_chain(a, c, W1, W2, tol)
     a.close()
     b.close()
 
