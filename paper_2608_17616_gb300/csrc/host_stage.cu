@@ -5,20 +5,26 @@
 //
 // Why SM loads and not the copy engines: on this part both top out at the link's read rate
 // (211 GB/s measured), but copy-engine transfers fell to 24-50 GB/s for stretches of a
-// multi-GB pinned footprint, while SM loads held 211 GB/s on every chunk.  A small grid
-// suffices (32 CTAs reach 208 GB/s alone): the kernel runs beside the learning kernels, whose
-// CTAs leave room for a 256-thread CTA of 48 registers on an SM.  Larger grids slowed the
-// learning they share the SMs with (a 128K-token step through mone_ttl_context_host: 24-32
-// CTAs 71-72 ms, 48 CTAs 75 ms, 96-152 CTAs 82-93 ms), smaller ones lost link rate.
+// multi-GB pinned footprint, while SM loads held 211 GB/s on every chunk.
+//
+// Where the gather runs: on SMs of its own.  A gather CTA sharing an SM with a learning CTA
+// slowed the learning far more than the gather's own work (a 128K-token step: 72 ms with 32
+// shared SMs, 81-96 ms with 64-152), so the gather's CTAs ask for more shared memory than an
+// SM has beside any learning CTA (at least 195 KB), and while mone_ttl_context_host runs the
+// persistent learning kernels leave ST_GRID SMs free (DevState::reserve_sms).  8 CTAs of 512
+// threads, 8 loads in flight each, reach 210 GB/s alone.
+#include <mutex>
+
 #include "mone_common.cuh"
 
 namespace mone {
 
 namespace {
 
-constexpr int ST_THREADS = 256;
-constexpr int ST_UNROLL = 8;  // 16-byte loads in flight per thread (32 KB per CTA)
-constexpr int ST_GRID = 32;
+constexpr int ST_THREADS = 512;
+constexpr int ST_UNROLL = 8;  // 16-byte loads in flight per thread (64 KB per CTA)
+constexpr int ST_GRID = 8;
+constexpr int ST_SMEM = 120 * 1024;  // unused: one gather CTA an SM, none beside a learning CTA
 
 struct StageArgs {
     const uint4* src[3];   // host tensors (device addresses) [C][N][row16[t]] in 16-byte units
@@ -54,9 +60,7 @@ __device__ __forceinline__ void stage_tensor(const uint4* src0, uint4* dst0, lon
     }
 }
 
-// At most 48 registers a thread (launch bounds of five CTAs an SM): a CTA then fits beside
-// the largest learning-kernel CTA (384 threads x 128 registers).
-__global__ void __launch_bounds__(ST_THREADS, 5) stage_rows_kernel(const StageArgs a) {
+__global__ void __launch_bounds__(ST_THREADS, 1) stage_rows_kernel(const StageArgs a) {
     stage_tensor(a.src[0], a.dst[0], a.row16[0], a.N, a.r0, a.nr, a.C);
     stage_tensor(a.src[1], a.dst[1], a.row16[1], a.N, a.r0, a.nr, a.C);
     stage_tensor(a.src[2], a.dst[2], a.row16[2], a.N, a.r0, a.nr, a.C);
@@ -76,8 +80,22 @@ cudaError_t launch_stage_rows(const void* const src[3], void* const dst[3], cons
     a.r0 = r0;
     a.nr = nr;
     a.C = C;
-    stage_rows_kernel<<<ST_GRID, ST_THREADS, 0, st>>>(a);
+    static std::mutex mu;
+    static bool opted_in[64] = {};  // the shared-memory opt-in belongs to a device
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(mu);
+    if (!opted_in[dev]) {
+        e = cudaFuncSetAttribute(stage_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, ST_SMEM);
+        if (e != cudaSuccess) return e;
+        opted_in[dev] = true;
+    }
+    stage_rows_kernel<<<ST_GRID, ST_THREADS, ST_SMEM, st>>>(a);
     return cudaGetLastError();
 }
+
+int stage_sms() { return ST_GRID; }
 
 }  // namespace mone

@@ -839,6 +839,12 @@ mone_status mone_ttl_context_host(mone_mem* m, const void* X, const void* K, con
     // the gathers start after what the caller queued before this call
     MONE_CUDA(cudaEventRecord(m->hstart, st));
     MONE_CUDA(cudaStreamWaitEvent(m->hstream, m->hstart, 0));
+    // the persistent learning kernels leave the gather's SMs free for the rest of this call
+    struct Reserve {
+        const DevState& s;
+        explicit Reserve(const DevState& d) : s(d) { s.reserve_sms = stage_sms(); }
+        ~Reserve() { s.reserve_sms = 0; }
+    } reserve(s);
     for (long long r0 = 0, k = 0; r0 < N; r0 += ct, ++k) {
         const long long nr = std::min(ct, N - r0);
         const int b = (int)(k & 1);

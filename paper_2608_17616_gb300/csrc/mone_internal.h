@@ -34,6 +34,9 @@ struct DevState {
     // test knob (MONE_FAULT_STALL=n at init): the next n tensor-core phase-A launches issue no
     // loads and wait 1 ms, so their bounded waits run out and latch DEV_TIMEOUT
     mutable int fault_stall;
+    // SMs the persistent learning kernels leave free while mone_ttl_context_host runs: its
+    // host-input gathers take them (one gather CTA an SM, never beside a learning CTA)
+    mutable int reserve_sms;
     // meta-parameters (owned copies)
     float *alpha, *gamma, *w_eta, *b_eta, *w_beta, *b_beta, *gate;
     // paper-mode input scratch for a window of win_rows tokens (a multiple of T)
@@ -164,6 +167,8 @@ cudaError_t launch_read_norm(const DevState& s, int Q, int n_layers, void* K_out
 // addresses of host memory) into device windows ([C][nr][row_bytes[t]]); row_bytes multiples of 16.
 cudaError_t launch_stage_rows(const void* const src[3], void* const dst[3], const long long row_bytes[3], long long N,
                               long long r0, long long nr, int C, cudaStream_t st);
+// SMs the gather occupies (one CTA on each); the learning kernels leave that many free.
+int stage_sms();
 
 // ---- kernels in attention.cu
 cudaError_t launch_attention(const DevState& s, int n_layers, const void* Q, int n_q, int Lq, const void* K,

@@ -891,7 +891,8 @@ cudaError_t launch_swiglu_phase_a(const DevState& s, const SwMaps& m, const SwIn
     SwArgs a = sw_args(s, w);
     a.nc_launch = w.nc;
     const int ntiles = (s.T / 128) * ((a.F + 127) / 128) * w.nc * a.H;
-    const int grid = ntiles < sw_sms() ? ntiles : sw_sms();
+    const int sms = sw_sms() - s.reserve_sms;  // leave the host-input gather's SMs free
+    const int grid = ntiles < sms ? ntiles : sms;
     swiglu_a_kernel<<<grid, SW_THREADS, SwLayout::DYN, st>>>(s.mode == 1 ? m.Ua : in.Xa, in.Ka, in.Va, m.W1a, m.W2a, a);
     return cudaGetLastError();
 }
@@ -903,7 +904,8 @@ cudaError_t launch_swiglu_phase_b(const DevState& s, const SwMaps& m, const SwIn
     SwArgs a = sw_args(s, w);
     a.nc_launch = w.nc;
     const int ntiles = w.nc * a.H * 3 * ((a.F + SWB_N - 1) / SWB_N) * ((a.dh + 127) / 128);
-    const int grid = ntiles < sw_sms() ? ntiles : sw_sms();
+    const int sms = sw_sms() - s.reserve_sms;  // leave the host-input gather's SMs free
+    const int grid = ntiles < sms ? ntiles : sms;
     if (a.step_sq)
         swiglu_b_kernel<true><<<grid, SWB_THREADS, SwLayoutB::DYN, st>>>(s.mode == 1 ? m.Ub : in.Xb, in.Kb, in.Vb, m.PG,
                                                                          m.Z, m.W1s, m.M1s, m.W2s, m.M2s, a);

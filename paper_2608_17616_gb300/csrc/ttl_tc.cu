@@ -1774,7 +1774,8 @@ cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputM
         a.r_only = (s.loss == 1) ? 1 : 0;  // 1: MONE_LOSS_MSE
         // CTA pairs over 256-token x 256-hidden tiles
         const int npairs = w.nc * (s.T / (2 * A_BM)) * (s.d_hid / P_BN);
-        const int clusters = npairs < g_pair_clusters ? npairs : g_pair_clusters;
+        const int maxc = g_pair_clusters - (s.reserve_sms + 1) / 2;  // leave reserved SMs free
+        const int clusters = npairs < maxc ? npairs : maxc;
         cudaLaunchConfig_t cfg = {};
         cudaLaunchAttribute at[1];
         at[0].id = cudaLaunchAttributeClusterDimension;
@@ -1790,7 +1791,8 @@ cudaError_t launch_phase_a_tc(const DevState& s, const TcMaps& m, const TcInputM
         return cudaLaunchKernelEx(&cfg, tc_phase_a_pair_kernel, U, in.Ka, in.Va, m.W1b, m.W2b, a);
     }
     const int ntiles = w.nc * (s.T / A_BM) * (s.d_hid / A_BN);
-    const int grid = ntiles < g_sms ? ntiles : g_sms;
+    const int sms = g_sms - s.reserve_sms;
+    const int grid = ntiles < sms ? ntiles : sms;
     tc_phase_a_kernel<<<grid, THREADS, LA::DYN, st>>>(U, in.Ka, in.Va, m.W1b, m.W2b, a);
     return cudaGetLastError();
 }
@@ -1808,7 +1810,8 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
     constexpr int PAIR_MIN_T = 1024;
     if (s.T >= PAIR_MIN_T && s.d_in % (2 * B_BM) == 0 && s.d_out % (2 * B_BM) == 0 && g_pairb_clusters > 0) {
         const int npairs = w.nc * ((s.d_in + s.d_out) / (2 * B_BM)) * (s.d_hid / B_BN);
-        const int clusters = npairs < g_pairb_clusters ? npairs : g_pairb_clusters;
+        const int maxc = g_pairb_clusters - (s.reserve_sms + 1) / 2;
+        const int clusters = npairs < maxc ? npairs : maxc;
         cudaLaunchConfig_t cfg = {};
         cudaLaunchAttribute at[1];
         at[0].id = cudaLaunchAttributeClusterDimension;
@@ -1828,7 +1831,8 @@ cudaError_t launch_phase_b_tc(const DevState& s, const TcMaps& m, const TcInputM
                                   m.M1s, m.M2s, a);
     }
     const int ntiles = w.nc * ((s.d_in + s.d_out) / B_BM) * (s.d_hid / B_BN);
-    const int grid = ntiles < g_sms ? ntiles : g_sms;
+    const int sms = g_sms - s.reserve_sms;
+    const int grid = ntiles < sms ? ntiles : sms;
     if (a.step_sq)
         tc_phase_b_kernel<false, true><<<grid, B_THREADS, LayoutB::DYN, st>>>(U, in.Kb, in.Vb, m.dH, m.At, m.W1s,
                                                                               m.W2s, m.M1s, m.M2s, a);

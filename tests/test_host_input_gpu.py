@@ -38,11 +38,11 @@ def pinned(t):
     return h
 
 
-def device_chunks(run, ct):
-    """mone_ttl_context on device copies of the chunks [r0, r0 + ct) in order."""
-    N = run.N
-    for r0 in range(0, N, ct):
-        nr = min(ct, N - r0)
+def device_chunks(run, bounds):
+    """mone_ttl_context on device copies of the chunks (r0, n) in order (an int: chunks of that length)."""
+    if isinstance(bounds, int):
+        bounds = [(r0, min(bounds, run.N - r0)) for r0 in range(0, run.N, bounds)]
+    for r0, nr in bounds:
         X, K, V = (t[:, :, r0:r0 + nr].contiguous() for t in (run.X, run.K, run.V))
         mone.mone_ttl_context(run.h, X, K, V, nr)
     mone.mone_mem_sync(run.h)
@@ -61,6 +61,7 @@ CASES = [
     # chunk length (one chunk here), plain mode, the fp32 tiled path and the fp32 resident path
     ("bf16_paper", 2 * 256, 1e-3),
     ("bf16_paper", 0, 1e-3),
+    ("bf16_plain", 0, 0.0),
     ("bf16_plain", 256, 0.0),
     ("f32_tiled", 3 * 64, 1e-5),
     ("f32_resident", 3 * 128, 0.0),
