@@ -5,12 +5,12 @@ One step = one pass of the whole hot path over one synthetic context: reset the
 fast weights to W_0, test-time learning of every layer's memory over all N/T
 segments (prepass, phase A, phase B per segment, final renormalisation), then
 the memory read (generate_kv) for a Q-token query.  Inputs are resident in HBM
-when the timed region starts; the e2e figure repeats the step through the same
-C-ABI calls with the inputs copied from pinned host memory and the generated
-K/V copied back inside the timed region.
+when the timed region starts; the e2e figure repeats the step with the context
+in pinned host memory (mone_ttl_context_host streams it over the host link inside
+the timed region), the query copied in and the generated K/V copied back.
 
---impl reference times the fp64 CPU oracle (the baseline of this build) on the
-host cores over a bounded sample of the same workload.
+--impl reference times the fp64 CPU oracle (the comparison point: the paper ships
+no implementation) on the host cores over a bounded sample of the same workload.
 
 Multi-GPU (torchrun): every rank runs an independent replica of the workload
 (independent contexts; no collective on the data path); value = all ranks'
