@@ -121,6 +121,9 @@ def test_calls_on_invalid_handles(L):
     assert L.mone_mem_generate_kv(bogus, 16, 1, 16, 16, arr, None) == 1
     assert L.mone_mem_sync(bogus, None) == 1
     assert L.mone_mem_launch_count(bogus) == -1
+    assert L.mone_ttl_context_host(bogus, 16, 16, 16, 128, 0, None) == 1
+    assert L.mone_ttl_context_metrics(bogus, 16, 16, 16, 128, None, None, None) == 1
+    assert L.mone_attention(bogus, 16, 2, 4, 16, 16, arr, 0, 16, None) == 1
 
 
 @pytest.mark.skipif(os.path.exists("/dev/nvidia0"), reason="checks the behaviour on a machine without a GPU")
