@@ -258,8 +258,8 @@ __device__ __forceinline__ void at_stage(uint8_t* dst, int slab, int n, int n_pa
     }
 }
 
-// 2^x on the special-function unit (PTX ex2.approx: relative error ~2^-22, far below the
-// bf16 rounding of the probabilities it feeds).
+// 2^x on the special-function unit (PTX ex2.approx), whose error is far below the bf16
+// rounding of the probabilities it feeds (the parity tests bound the result at 1e-2).
 __device__ __forceinline__ float at_exp2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
