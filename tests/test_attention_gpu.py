@@ -93,6 +93,14 @@ def test_attention_bf16_head_dim_128_random_memory(Lq, n_mem):
     check(wl, Qt, Kc, Vc, out, n_mem, Lq, 1e-2)
 
 
+def test_attention_at_the_bench_shape():
+    """The shape bench.py times: 16 chains (one context, 16 layers), 8 KV heads x 2 query heads,
+    hd 64, 64 memory tokens from the read plus 64 query tokens; every chain checked."""
+    wl = small(n_ctx=1, n_layers=16, d_out=1024, hd=64, N=256, Q=64)
+    Qt, Kc, Vc, out = run_case(wl, 2 * wl.n_kv_heads, 64, 64, seed=77)
+    check(wl, Qt, Kc, Vc, out, 64, 64, 1e-2)
+
+
 def test_attention_fp32():
     wl = small(mode=wk.PLAIN, dtype="f32", N=300, Q=32)
     Qt, Kc, Vc, out = run_case(wl, 2 * wl.n_kv_heads, 33, 32, seed=9)
