@@ -17,7 +17,7 @@ import torch
 
 import paper_2608_17616_gb300 as mone
 import workloads as wk
-from harness import DeviceRun, rel_fro
+from harness import DeviceRun, oracle_read, rel_fro
 from test_parity_gpu import BF16_TOL, F32_TOL, check_chain, small
 from test_swiglu_gpu import check as check_swiglu, swiglu
 
@@ -165,3 +165,30 @@ def test_host_context_argument_errors_launch_nothing():
         assert e.value.code == 1, (N, ct)
     assert mone.mone_mem_launch_count(run.h) == n0
     run.close()
+
+
+def test_host_context_at_the_bench_size_sampled_chains():
+    """The configuration bench.py's e2e runs: l16_d2048_128k, the 128K-token context in pinned
+    host memory (8.6 GB of X: offsets past 2^31 bytes), the library's chunks (5,120 tokens, 26
+    gathers) on SMs of their own.  The first and the last chain are checked against the oracle
+    (state and read)."""
+    wl = wk.WORKLOADS["l16_d2048_128k"]
+    run = DeviceRun(wl)
+    hX, hK, hV = pinned(run.X), pinned(run.K), pinned(run.V)
+    mone.mone_mem_set_timing(run.h, 1)
+    mone.mone_ttl_context_host(run.h, hX, hK, hV, run.N)
+    mone.mone_mem_sync(run.h)
+    assert mone.mone_mem_kernel_time(run.h, mone.KERNEL_KINDS.index("stage"))[1] == -(-run.N // 5120)
+    mone.mone_mem_set_timing(run.h, 0)
+    del hX, hK, hV
+    W1, W2, _, _ = run.state()
+    Xq = wk.query_inputs(wl, "cuda")
+    Kg, Vg = run.generate_kv(Xq)
+    for c in (0, wl.chains - 1):
+        st = check_chain(run, c, W1, W2, BF16_TOL)
+        Ko, Vo = oracle_read(run, st, c, Xq)
+        ctx, layer = divmod(c, wl.n_layers)
+        assert rel_fro(Kg[ctx, layer].float(), Ko) <= BF16_TOL
+        assert rel_fro(Vg[ctx, layer].float(), Vo) <= BF16_TOL
+    run.close()
+    torch.cuda.empty_cache()
